@@ -1,0 +1,172 @@
+"""CPU oracle for LAM's quantized-memory hot path (test infrastructure only).
+
+The oracle is plain C (``lam_oracle.c``), compiled with ``-O2 -ffp-contract=off
+-fno-fast-math`` so that no multiply-add is fused on either x86-64 or aarch64.
+Only the test suite, the smoke check and the benchmark's CPU-baseline leg may
+load it; the product library never does, and the two share no code.
+
+What it follows (paper: "LAM: Lossy Agent Memory"):
+  * quantize   -- Sec. 3.2, layer L1: Q_eps(x) = round(x / 2 eps);
+  * dequantize -- xhat = 2 eps * Q_eps(x), the reading under which one cell has
+                  half-width eps (Sec. 3.1, App. "Rank invariance, in full");
+  * scores     -- exact search is a matrix-vector product over the stored
+                  vectors (Sec. "Brute-force scan crossover"); metrics inner
+                  product, cosine and squared L2 (Eq. 1 ties L2 to cosine);
+  * top-k      -- full sort, best first, equal scores by lower id (the
+                  lowest-index rule of Algorithm 1).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "lam_oracle.c")
+_LIB = os.path.join(_HERE, "liblam_oracle.so")
+
+IP, COSINE, L2 = 0, 1, 2
+CFLAGS = ["-O2", "-ffp-contract=off", "-fno-fast-math", "-fPIC", "-shared",
+          "-std=c11", "-pthread"]
+
+
+def build(force: bool = False) -> str:
+    """Compile lam_oracle.c into liblam_oracle.so beside it (gcc)."""
+    if (not force and os.path.exists(_LIB)
+            and os.path.getmtime(_LIB) >= os.path.getmtime(_SRC)):
+        return _LIB
+    tmp = _LIB + ".tmp%d" % os.getpid()
+    subprocess.run(["gcc", *CFLAGS, "-o", tmp, _SRC, "-lm"], check=True)
+    os.replace(tmp, _LIB)
+    return _LIB
+
+
+_lib = None
+
+
+def _load():
+    global _lib
+    if _lib is None:
+        build()
+        lib = ctypes.CDLL(_LIB)
+        f32p = ctypes.POINTER(ctypes.c_float)
+        i32p = ctypes.POINTER(ctypes.c_int32)
+        i64p = ctypes.POINTER(ctypes.c_int64)
+        f64p = ctypes.POINTER(ctypes.c_double)
+        lib.lam_oracle_step.argtypes = [ctypes.c_float]
+        lib.lam_oracle_step.restype = ctypes.c_float
+        lib.lam_oracle_quantize.argtypes = [f32p, ctypes.c_int64, ctypes.c_float,
+                                            i32p, f64p, f64p, i64p]
+        lib.lam_oracle_quantize.restype = None
+        lib.lam_oracle_width.argtypes = [ctypes.c_double, ctypes.c_double]
+        lib.lam_oracle_width.restype = ctypes.c_int32
+        lib.lam_oracle_dequantize.argtypes = [i32p, ctypes.c_int64, ctypes.c_float,
+                                              f32p]
+        lib.lam_oracle_dequantize.restype = None
+        lib.lam_oracle_scores.argtypes = [f32p, ctypes.c_int64, i32p, ctypes.c_int64,
+                                          ctypes.c_int32, ctypes.c_float,
+                                          ctypes.c_int32, f32p]
+        lib.lam_oracle_scores.restype = None
+        lib.lam_oracle_topk.argtypes = [f32p, ctypes.c_int64, ctypes.c_int64,
+                                        ctypes.c_int32, ctypes.c_int32, f32p, i64p]
+        lib.lam_oracle_topk.restype = ctypes.c_int
+        lib.lam_oracle_search.argtypes = [f32p, ctypes.c_int64, i32p,
+                                          ctypes.c_int64, ctypes.c_int32,
+                                          ctypes.c_float, ctypes.c_int32,
+                                          ctypes.c_int32, f32p, i64p,
+                                          ctypes.c_int32]
+        lib.lam_oracle_search.restype = ctypes.c_int
+        _lib = lib
+    return _lib
+
+
+def _ptr(a: np.ndarray, ctype):
+    return a.ctypes.data_as(ctypes.POINTER(ctype))
+
+
+def step(eps: float) -> np.float32:
+    """s = fl32(2 eps), the quantizer step."""
+    return np.float32(_load().lam_oracle_step(ctypes.c_float(np.float32(eps))))
+
+
+def quantize(x: np.ndarray, eps: float):
+    """Q_eps over a flat fp32 array.
+
+    Returns ``(codes int32, rmin, rmax, n_nonfinite)``; rmin/rmax are the
+    smallest/largest rounded quotient over the finite inputs (exact, as float).
+    Codes of values outside int32 or non-finite inputs are 0.
+    """
+    x = np.ascontiguousarray(x, dtype=np.float32).reshape(-1)
+    codes = np.empty(x.size, dtype=np.int32)
+    rmin = ctypes.c_double()
+    rmax = ctypes.c_double()
+    nnf = ctypes.c_int64()
+    _load().lam_oracle_quantize(_ptr(x, ctypes.c_float), x.size,
+                                ctypes.c_float(np.float32(eps)),
+                                _ptr(codes, ctypes.c_int32), ctypes.byref(rmin),
+                                ctypes.byref(rmax), ctypes.byref(nnf))
+    return codes, rmin.value, rmax.value, nnf.value
+
+
+def width(rmin: float, rmax: float) -> int:
+    """Narrowest width in bytes (1, 2, 4) holding [rmin, rmax]; 0 if none."""
+    return int(_load().lam_oracle_width(rmin, rmax))
+
+
+def dequantize(codes: np.ndarray, scale: float) -> np.ndarray:
+    """xhat = fl32(scale * code)."""
+    c = np.ascontiguousarray(codes, dtype=np.int32).reshape(-1)
+    out = np.empty(c.size, dtype=np.float32)
+    _load().lam_oracle_dequantize(_ptr(c, ctypes.c_int32), c.size,
+                                  ctypes.c_float(np.float32(scale)),
+                                  _ptr(out, ctypes.c_float))
+    return out.reshape(np.shape(codes))
+
+
+def scores(queries: np.ndarray, codes: np.ndarray, eps: float, metric: int):
+    """All scores [B, N] of queries [B, D] against code rows [N, D]."""
+    q = np.ascontiguousarray(queries, dtype=np.float32)
+    c = np.ascontiguousarray(codes, dtype=np.int32)
+    B, D = q.shape
+    N = c.shape[0]
+    assert c.shape[1] == D
+    out = np.empty((B, N), dtype=np.float32)
+    _load().lam_oracle_scores(_ptr(q, ctypes.c_float), B, _ptr(c, ctypes.c_int32),
+                              N, D, ctypes.c_float(np.float32(eps)), metric,
+                              _ptr(out, ctypes.c_float))
+    return out
+
+
+def topk(score_matrix: np.ndarray, k: int, metric: int):
+    """Top-k per row of a score matrix: (scores [B, k] f32, ids [B, k] i64)."""
+    s = np.ascontiguousarray(score_matrix, dtype=np.float32)
+    B, N = s.shape
+    os_ = np.empty((B, k), dtype=np.float32)
+    oi = np.empty((B, k), dtype=np.int64)
+    rc = _load().lam_oracle_topk(_ptr(s, ctypes.c_float), B, N, k, metric,
+                                 _ptr(os_, ctypes.c_float), _ptr(oi, ctypes.c_int64))
+    if rc:
+        raise ValueError("oracle topk failed (%d)" % rc)
+    return os_, oi
+
+
+def search(queries: np.ndarray, codes: np.ndarray, eps: float, metric: int,
+           k: int, nthreads: int = 1):
+    """Exact search: scores of every row, then top-k per query."""
+    q = np.ascontiguousarray(queries, dtype=np.float32)
+    c = np.ascontiguousarray(codes, dtype=np.int32)
+    B, D = q.shape
+    N = c.shape[0]
+    assert c.shape[1] == D
+    os_ = np.empty((B, k), dtype=np.float32)
+    oi = np.empty((B, k), dtype=np.int64)
+    rc = _load().lam_oracle_search(_ptr(q, ctypes.c_float), B,
+                                   _ptr(c, ctypes.c_int32), N, D,
+                                   ctypes.c_float(np.float32(eps)), metric, k,
+                                   _ptr(os_, ctypes.c_float),
+                                   _ptr(oi, ctypes.c_int64), nthreads)
+    if rc:
+        raise ValueError("oracle search failed (%d)" % rc)
+    return os_, oi

@@ -1,0 +1,334 @@
+/*
+ * lam_oracle.c -- plain, slow CPU oracle for LAM's quantized-memory hot path.
+ *
+ * TEST INFRASTRUCTURE ONLY.  Nothing in the product library links, loads or
+ * calls this file.  Only the test suite, the smoke check and the benchmark's
+ * CPU-baseline leg may use it.  It shares no code, header or constant
+ * generator with the CUDA path.
+ *
+ * What it computes (paper: "LAM: Lossy Agent Memory"):
+ *   - Q_eps(x) = round(x / 2 eps), coordinatewise, one global eps
+ *     (Sec. 3.2 "Three layers", layer L1; Algorithm 1 applies it to each
+ *     arriving embedding).
+ *   - Dequantisation xhat = 2 eps * Q_eps(x).  The paper never writes it out;
+ *     it is the reading under which a quantization cell has half-width eps
+ *     (Sec. 3.1, the coordinatewise tolerance ||a-b||_inf <= 2 eps between
+ *     two members of one cell; App. "Rank invariance, in full").
+ *   - Exact search: every query scored against every retained (here:
+ *     dequantised) embedding, i.e. a matrix-vector product per query
+ *     (Sec. "Brute-force scan crossover"), followed by a top-k.  Metrics:
+ *     inner product, cosine, squared L2 (Eq. 1 relates L2 and cosine).
+ *
+ * Readings where the paper is silent (each also listed in the design doc):
+ *   - "round" is IEEE round-half-to-even, evaluated as nearbyintf() under
+ *     FE_TONEAREST on the fp32 quotient.
+ *   - x / 2 eps is one fp32 IEEE division by s = fl32(2 * eps), eps given in
+ *     fp32 (doubling is exact).
+ *   - Dequantisation is one fp32 multiply s * (float)c.
+ *   - Cosine uses the norm of the dequantised vector; a zero norm gives 0.
+ *   - L2 score is the squared distance, ranked ascending; inner product and
+ *     cosine rank descending.  Equal scores rank the lower id first (the
+ *     paper's lowest-index rule, Algorithm 1).
+ *   - Scores are accumulated in double and rounded once to fp32.
+ *
+ * Build flags matter: -O2 -ffp-contract=off -fno-fast-math, so that no
+ * multiply-add is contracted into an FMA on either x86-64 or aarch64.
+ */
+#include <fenv.h>
+#include <math.h>
+#include <pthread.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+#define ORACLE_IP 0
+#define ORACLE_COSINE 1
+#define ORACLE_L2 2
+
+/* Step of the quantizer: s = 2 eps in fp32 (Sec. 3.2, L1). */
+float lam_oracle_step(float eps) { return 2.0f * eps; }
+
+/*
+ * Q_eps over n fp32 values (Sec. 3.2, L1: Q_eps(x) = round(x / 2 eps)).
+ *   r_i = nearbyintf(fl32(x_i / s)); codes_i = (int32) r_i when r_i fits int32.
+ * Outputs: codes (may be NULL), the smallest and largest rounded quotient over
+ * the finite inputs (as doubles, exact), and the count of non-finite inputs.
+ * With n == 0, rmin = rmax = 0.
+ */
+void lam_oracle_quantize(const float *x, int64_t n, float eps, int32_t *codes,
+                         double *rmin_out, double *rmax_out,
+                         int64_t *n_nonfinite_out) {
+  int old_mode = fegetround();
+  fesetround(FE_TONEAREST);
+  float s = lam_oracle_step(eps);
+  double rmin = 0.0, rmax = 0.0;
+  int seen = 0;
+  int64_t nonfinite = 0;
+  for (int64_t i = 0; i < n; ++i) {
+    float xi = x[i];
+    if (!isfinite(xi)) {
+      nonfinite++;
+      if (codes) codes[i] = 0;
+      continue;
+    }
+    float q = xi / s;
+    float r = nearbyintf(q);
+    if (!seen) {
+      rmin = rmax = (double)r;
+      seen = 1;
+    } else {
+      if ((double)r < rmin) rmin = (double)r;
+      if ((double)r > rmax) rmax = (double)r;
+    }
+    if (codes) {
+      if ((double)r >= -2147483648.0 && (double)r <= 2147483647.0)
+        codes[i] = (int32_t)r;
+      else
+        codes[i] = 0;
+    }
+  }
+  fesetround(old_mode);
+  *rmin_out = rmin;
+  *rmax_out = rmax;
+  *n_nonfinite_out = nonfinite;
+}
+
+/*
+ * Narrowest two's-complement width (bytes: 1, 2 or 4) whose range holds
+ * [rmin, rmax]; 0 when even int32 cannot hold it.
+ */
+int32_t lam_oracle_width(double rmin, double rmax) {
+  if (rmin >= -128.0 && rmax <= 127.0) return 1;
+  if (rmin >= -32768.0 && rmax <= 32767.0) return 2;
+  if (rmin >= -2147483648.0 && rmax <= 2147483647.0) return 4;
+  return 0;
+}
+
+/* Dequantisation xhat_i = fl32(s * (float) c_i) with s = fl32(2 eps). */
+void lam_oracle_dequantize(const int32_t *codes, int64_t n, float scale,
+                           float *out) {
+  for (int64_t i = 0; i < n; ++i) out[i] = scale * (float)codes[i];
+}
+
+/* Score of one query against one dequantised row, in double, rounded to fp32. */
+static float score_one(const float *q, const int32_t *c, int32_t D, float s,
+                       int metric) {
+  if (metric == ORACLE_IP) {
+    double acc = 0.0;
+    for (int32_t d = 0; d < D; ++d) {
+      float xh = s * (float)c[d];
+      acc += (double)q[d] * (double)xh;
+    }
+    return (float)acc;
+  }
+  if (metric == ORACLE_COSINE) {
+    double dot = 0.0, qq = 0.0, xx = 0.0;
+    for (int32_t d = 0; d < D; ++d) {
+      float xh = s * (float)c[d];
+      dot += (double)q[d] * (double)xh;
+      qq += (double)q[d] * (double)q[d];
+      xx += (double)xh * (double)xh;
+    }
+    if (qq == 0.0 || xx == 0.0) return 0.0f;
+    return (float)(dot / (sqrt(qq) * sqrt(xx)));
+  }
+  /* squared L2, direct form */
+  double acc = 0.0;
+  for (int32_t d = 0; d < D; ++d) {
+    float xh = s * (float)c[d];
+    double diff = (double)q[d] - (double)xh;
+    acc += diff * diff;
+  }
+  return (float)acc;
+}
+
+/* Scores of B queries [B, D] against N code rows [N, D]: out [B, N]. */
+void lam_oracle_scores(const float *queries, int64_t B, const int32_t *codes,
+                       int64_t N, int32_t D, float eps, int32_t metric,
+                       float *out) {
+  float s = lam_oracle_step(eps);
+  for (int64_t b = 0; b < B; ++b)
+    for (int64_t i = 0; i < N; ++i)
+      out[b * N + i] =
+          score_one(queries + b * (int64_t)D, codes + i * (int64_t)D, D, s,
+                    metric);
+}
+
+/* ---- top-k: full sort of (score, id), best first, ties by lower id ---- */
+
+typedef struct {
+  float score;
+  int64_t id;
+} scored_t;
+
+static int cmp_desc(const void *a, const void *b) {
+  const scored_t *x = (const scored_t *)a, *y = (const scored_t *)b;
+  if (x->score > y->score) return -1;
+  if (x->score < y->score) return 1;
+  return (x->id < y->id) ? -1 : (x->id > y->id);
+}
+
+static int cmp_asc(const void *a, const void *b) {
+  const scored_t *x = (const scored_t *)a, *y = (const scored_t *)b;
+  if (x->score < y->score) return -1;
+  if (x->score > y->score) return 1;
+  return (x->id < y->id) ? -1 : (x->id > y->id);
+}
+
+/* Top-k of one row of N scores. */
+static void topk_row(const float *scores, int64_t N, int32_t k, int32_t metric,
+                     scored_t *tmp, float *out_scores, int64_t *out_ids) {
+  for (int64_t i = 0; i < N; ++i) {
+    tmp[i].score = scores[i];
+    tmp[i].id = i;
+  }
+  qsort(tmp, (size_t)N, sizeof(scored_t),
+        metric == ORACLE_L2 ? cmp_asc : cmp_desc);
+  for (int32_t j = 0; j < k; ++j) {
+    out_scores[j] = tmp[j].score;
+    out_ids[j] = tmp[j].id;
+  }
+}
+
+/* Top-k of B rows of N given scores: out [B, k]. Returns 0 on success. */
+int lam_oracle_topk(const float *scores, int64_t B, int64_t N, int32_t k,
+                    int32_t metric, float *out_scores, int64_t *out_ids) {
+  if (k < 1 || k > N) return 1;
+  scored_t *tmp = (scored_t *)malloc(sizeof(scored_t) * (size_t)N);
+  if (!tmp) return 2;
+  for (int64_t b = 0; b < B; ++b)
+    topk_row(scores + b * N, N, k, metric, tmp, out_scores + b * (int64_t)k,
+             out_ids + b * (int64_t)k);
+  free(tmp);
+  return 0;
+}
+
+/* ---- exhaustive search driver: score + top-k, threads split the work ---- */
+
+typedef struct {
+  const float *queries;
+  const int32_t *codes;
+  int64_t N;
+  int32_t D;
+  float s;
+  int32_t metric;
+  int32_t k;
+  int64_t B;
+  float *out_scores;
+  int64_t *out_ids;
+  /* scratch for the query being processed collectively */
+  float *row_scores;
+  int nthreads;
+  int tid;
+  int64_t b_single; /* query index for the row-split phase */
+  int phase;        /* 0: whole queries per thread; 1: rows of b_single */
+  int status;
+} search_job_t;
+
+static void *search_worker(void *arg) {
+  search_job_t *j = (search_job_t *)arg;
+  if (j->phase == 1) {
+    /* rows [lo, hi) of one query */
+    int64_t lo = j->N * j->tid / j->nthreads;
+    int64_t hi = j->N * (j->tid + 1) / j->nthreads;
+    const float *q = j->queries + j->b_single * (int64_t)j->D;
+    for (int64_t i = lo; i < hi; ++i)
+      j->row_scores[i] = score_one(q, j->codes + i * (int64_t)j->D, j->D, j->s,
+                                   j->metric);
+    return NULL;
+  }
+  float *scores = (float *)malloc(sizeof(float) * (size_t)j->N);
+  scored_t *tmp = (scored_t *)malloc(sizeof(scored_t) * (size_t)j->N);
+  if (!scores || !tmp) {
+    j->status = 2;
+    free(scores);
+    free(tmp);
+    return NULL;
+  }
+  for (int64_t b = j->tid; b < j->B; b += j->nthreads) {
+    const float *q = j->queries + b * (int64_t)j->D;
+    for (int64_t i = 0; i < j->N; ++i)
+      scores[i] = score_one(q, j->codes + i * (int64_t)j->D, j->D, j->s,
+                            j->metric);
+    topk_row(scores, j->N, j->k, j->metric, tmp,
+             j->out_scores + b * (int64_t)j->k, j->out_ids + b * (int64_t)j->k);
+  }
+  free(scores);
+  free(tmp);
+  return NULL;
+}
+
+/*
+ * Exact search: for each of B queries, score all N dequantised rows and keep
+ * the k best (Sec. "Brute-force scan crossover": a matrix-vector product per
+ * query).  nthreads worker threads: whole queries per thread when B >= the
+ * thread count, otherwise the rows of each query are split across threads.
+ * Returns 0 on success.
+ */
+int lam_oracle_search(const float *queries, int64_t B, const int32_t *codes,
+                      int64_t N, int32_t D, float eps, int32_t metric,
+                      int32_t k, float *out_scores, int64_t *out_ids,
+                      int32_t nthreads) {
+  if (k < 1 || k > N || D < 1 || B < 0) return 1;
+  if (nthreads < 1) nthreads = 1;
+  float s = lam_oracle_step(eps);
+  pthread_t *th = (pthread_t *)malloc(sizeof(pthread_t) * (size_t)nthreads);
+  search_job_t *jobs =
+      (search_job_t *)calloc((size_t)nthreads, sizeof(search_job_t));
+  if (!th || !jobs) {
+    free(th);
+    free(jobs);
+    return 2;
+  }
+  int status = 0;
+  for (int t = 0; t < nthreads; ++t) {
+    jobs[t].queries = queries;
+    jobs[t].codes = codes;
+    jobs[t].N = N;
+    jobs[t].D = D;
+    jobs[t].s = s;
+    jobs[t].metric = metric;
+    jobs[t].k = k;
+    jobs[t].B = B;
+    jobs[t].out_scores = out_scores;
+    jobs[t].out_ids = out_ids;
+    jobs[t].nthreads = nthreads;
+    jobs[t].tid = t;
+  }
+  if (B >= nthreads) {
+    for (int t = 0; t < nthreads; ++t) {
+      jobs[t].phase = 0;
+      pthread_create(&th[t], NULL, search_worker, &jobs[t]);
+    }
+    for (int t = 0; t < nthreads; ++t) {
+      pthread_join(th[t], NULL);
+      if (jobs[t].status) status = jobs[t].status;
+    }
+  } else {
+    float *row_scores = (float *)malloc(sizeof(float) * (size_t)N);
+    scored_t *tmp = (scored_t *)malloc(sizeof(scored_t) * (size_t)N);
+    if (!row_scores || !tmp) {
+      free(row_scores);
+      free(tmp);
+      free(th);
+      free(jobs);
+      return 2;
+    }
+    for (int64_t b = 0; b < B; ++b) {
+      for (int t = 0; t < nthreads; ++t) {
+        jobs[t].phase = 1;
+        jobs[t].b_single = b;
+        jobs[t].row_scores = row_scores;
+        pthread_create(&th[t], NULL, search_worker, &jobs[t]);
+      }
+      for (int t = 0; t < nthreads; ++t) pthread_join(th[t], NULL);
+      topk_row(row_scores, N, k, metric, tmp, out_scores + b * (int64_t)k,
+               out_ids + b * (int64_t)k);
+    }
+    free(row_scores);
+    free(tmp);
+  }
+  free(th);
+  free(jobs);
+  return status;
+}

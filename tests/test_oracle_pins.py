@@ -1,0 +1,250 @@
+"""Pins of the CPU oracle to what the paper and the mathematics fix.
+
+None of these compares the oracle with itself: each checks a value the paper
+prints, a hand computation, a closed form, an invariant of Q_eps, or a brute
+force over tiny inputs.  A dropped factor of 2 in the step, a different tie
+rule, a transposed code index, a wrong norm in the cosine, a sign slip in the
+L2 cross term or a reversed ranking direction each fails at least one test.
+"""
+import math
+
+import numpy as np
+import pytest
+
+import oracle
+from tests.conftest import golden
+from paper_2609_32256_gb300 import inputs
+
+EPS_SWEEP = (1e-2, 1e-3, 1e-4)
+
+
+# --- Q_eps (Sec. 3.2, layer L1) -------------------------------------------------
+
+def test_worked_ties_half_to_even():
+    eps = np.float32(2.0 ** -10)
+    s = np.float32(2.0 ** -9)
+    rows = golden("q_eps_ties.txt")
+    v = np.array([float(r[0]) for r in rows], dtype=np.float32)
+    want = np.array([int(r[1]) for r in rows], dtype=np.int64)
+    x = v * s  # power-of-two scaling: exact
+    codes, rmin, rmax, nnf = oracle.quantize(x, eps)
+    assert nnf == 0
+    np.testing.assert_array_equal(codes.astype(np.int64), want)
+    assert rmin == want.min() and rmax == want.max()
+
+
+def test_step_is_two_eps():
+    # x = 0.9 * 2eps must land in cell 1 (a step of eps would give 2).
+    for eps in EPS_SWEEP:
+        s = np.float32(2.0) * np.float32(eps)
+        x = np.array([0.9, -0.9, 1.9, 0.45], dtype=np.float32) * s
+        codes, *_ = oracle.quantize(x, eps)
+        assert list(codes) == [1, -1, 2, 0]
+    assert oracle.step(np.float32(1e-3)) == np.float32(2.0) * np.float32(1e-3)
+
+
+def _bound_slack(x, eps):
+    # |x - s*c| <= eps + one rounding of the quotient and one of the product.
+    return eps * (1 + 2.0 ** -23) + np.abs(x.astype(np.float64)) * 2.0 ** -23
+
+
+@pytest.mark.parametrize("eps", EPS_SWEEP)
+def test_dequant_error_bound_and_tight(eps):
+    x = inputs.flat_values(1 << 20, seed=7)
+    codes, *_ = oracle.quantize(x, eps)
+    xh = oracle.dequantize(codes, oracle.step(eps))
+    err = np.abs(x.astype(np.float64) - xh.astype(np.float64))
+    assert np.all(err <= _bound_slack(x, np.float64(np.float32(eps))))
+    # Tightness: the cell half-width is eps, so dense inputs reach it.
+    dense = np.linspace(-50 * eps, 50 * eps, 200001, dtype=np.float32)
+    c2, *_ = oracle.quantize(dense, eps)
+    e2 = np.abs(dense.astype(np.float64) - oracle.dequantize(c2, oracle.step(eps)))
+    assert e2.max() > 0.99 * eps
+
+
+@pytest.mark.parametrize("eps", EPS_SWEEP)
+def test_idempotent_on_every_int16_code(eps):
+    c = np.arange(-32768, 32768, dtype=np.int32)
+    xh = oracle.dequantize(c, oracle.step(eps))
+    c2, rmin, rmax, nnf = oracle.quantize(xh, eps)
+    np.testing.assert_array_equal(c2, c)
+    assert (rmin, rmax, nnf) == (-32768, 32767, 0)
+
+
+def test_monotone_and_odd():
+    x = np.sort(inputs.flat_values(200000, seed=3))
+    for eps in EPS_SWEEP:
+        c, *_ = oracle.quantize(x, eps)
+        assert np.all(np.diff(c) >= 0)
+        cn, *_ = oracle.quantize(-x, eps)
+        np.testing.assert_array_equal(cn, -c)
+
+
+@pytest.mark.parametrize("lo,hi,w", [
+    (0, 0, 1), (-128, 127, 1), (-129, 0, 2), (0, 128, 2), (-32768, 32767, 2),
+    (-32769, 0, 4), (0, 32768, 4), (-2147483648, 2147483647, 4),
+    (-2147483649, 0, 0), (0, 2147483648, 0)])
+def test_width_boundaries(lo, hi, w):
+    assert oracle.width(float(lo), float(hi)) == w
+
+
+def test_width_from_quantized_range():
+    eps = np.float32(2.0 ** -10)
+    s = np.float32(2.0 ** -9)
+    for vals, w in [([127.4, -128.4], 1), ([127.5], 2), ([-128.6], 2),
+                    ([32767.4], 2), ([32767.5], 4)]:
+        x = np.array(vals, dtype=np.float32) * s
+        _, rmin, rmax, _ = oracle.quantize(x, eps)
+        assert oracle.width(rmin, rmax) == w
+
+
+def test_nonfinite_counted():
+    x = np.array([0.1, np.nan, np.inf, -np.inf, 0.2], dtype=np.float32)
+    codes, rmin, rmax, nnf = oracle.quantize(x, 1e-2)
+    assert nnf == 3
+    assert list(codes) == [5, 0, 0, 0, 10]
+    assert (rmin, rmax) == (5, 10)
+
+
+def test_empty_input():
+    codes, rmin, rmax, nnf = oracle.quantize(np.zeros(0, np.float32), 1e-3)
+    assert codes.size == 0 and (rmin, rmax, nnf) == (0, 0, 0)
+
+
+# --- scores (exact search, Sec. "Brute-force scan crossover"; Eq. 1) -----------
+
+def test_scores_d2_hand_computed():
+    q = np.array([[0.6, 0.8]], dtype=np.float32)
+    c = np.array([[3, -1]], dtype=np.int32)
+    for metric, want in golden("scores_d2_hand.txt"):
+        got = oracle.scores(q, c, 0.25, int(metric))[0, 0]
+        assert got == np.float32(float(want))
+
+
+def test_scores_d1_closed_form():
+    eps = 0.125  # s = 0.25
+    q = np.array([[-2.0], [0.0], [3.0]], dtype=np.float32)
+    c = np.array([[4], [-3], [0]], dtype=np.int32)
+    ip = oracle.scores(q, c, eps, oracle.IP)
+    np.testing.assert_array_equal(ip, np.outer(q[:, 0], 0.25 * c[:, 0]).astype(np.float32))
+    cos = oracle.scores(q, c, eps, oracle.COSINE)
+    np.testing.assert_array_equal(
+        cos, np.array([[-1, 1, 0], [0, 0, 0], [1, -1, 0]], dtype=np.float32))
+    l2 = oracle.scores(q, c, eps, oracle.L2)
+    want = (q[:, 0][:, None] - 0.25 * c[:, 0][None, :]) ** 2
+    np.testing.assert_array_equal(l2, want.astype(np.float32))
+
+
+def test_basis_queries_read_codes():
+    # IP with the unit vector e_d equals s * c[i, d]: pins the code indexing.
+    rng = np.random.default_rng(5)
+    N, D, eps = 7, 5, 1e-2
+    c = rng.integers(-100, 100, size=(N, D), dtype=np.int32)
+    q = np.eye(D, dtype=np.float32)
+    ip = oracle.scores(q, c, eps, oracle.IP)
+    s = oracle.step(eps)
+    np.testing.assert_array_equal(ip, (s * c.T.astype(np.float32)).astype(np.float32))
+
+
+def test_self_query_cosine_one_l2_zero():
+    x = inputs.unit_rows(64, 768, seed=11)
+    eps = 1e-3
+    codes, *_ = oracle.quantize(x, eps)
+    codes = codes.reshape(x.shape)
+    xh = oracle.dequantize(codes, oracle.step(eps))
+    cos = oracle.scores(xh, codes, eps, oracle.COSINE)
+    assert np.all(np.abs(np.diag(cos) - 1.0) <= 2 ** -23)
+    l2 = oracle.scores(xh, codes, eps, oracle.L2)
+    assert np.all(np.diag(l2) == 0.0)
+    assert np.all(l2[~np.eye(64, dtype=bool)] > 0.5)
+
+
+def test_margin_constants_match_paper():
+    for eps, printed in golden("margin_bound_constants.txt"):
+        assert round(2 * float(eps) * math.sqrt(768), 4) == float(printed)
+
+
+@pytest.mark.parametrize("eps", (1e-3, 1e-2))
+def test_score_deviation_within_paper_bound(eps):
+    # One vector quantized to within eps per coordinate moves an inner product
+    # by at most ||q||_1 eps (Hoelder) <= sqrt(D) eps ||q||_2, i.e. half the
+    # pairwise 2 eps sqrt(D) constant the paper prints.
+    x = inputs.unit_rows(300, 768, seed=21)
+    q = inputs.queries(40, 768, seed=22)
+    codes, *_ = oracle.quantize(x, eps)
+    codes = codes.reshape(x.shape)
+    ip_q = oracle.scores(q, codes, eps, oracle.IP).astype(np.float64)
+    ip_x = q.astype(np.float64) @ x.astype(np.float64).T
+    l1 = np.abs(q.astype(np.float64)).sum(1)[:, None]
+    slack = 1e-6
+    assert np.all(np.abs(ip_q - ip_x) <= l1 * eps * (1 + 1e-6) + slack)
+    printed = {1e-3: 0.0554, 1e-2: 0.5543}[eps]
+    assert np.abs(ip_q - ip_x).max() <= printed / 2 + 1e-4
+    # cosine: |cos(q,x) - cos(q,xh)| <= 2 ||x - xh|| / ||x|| <= 2 eps sqrt(D)
+    cos_q = oracle.scores(q, codes, eps, oracle.COSINE).astype(np.float64)
+    cos_x = ip_x  # unit rows, unit queries
+    assert np.abs(cos_q - cos_x).max() <= printed + 1e-4
+    # L2: | ||q-x|| - ||q-xh|| | <= ||x - xh|| <= eps sqrt(D)
+    l2_q = oracle.scores(q, codes, eps, oracle.L2).astype(np.float64)
+    l2_x = ((q.astype(np.float64)[:, None, :] - x.astype(np.float64)[None]) ** 2).sum(-1)
+    assert np.abs(np.sqrt(l2_q) - np.sqrt(l2_x)).max() <= printed / 2 + 1e-4
+
+
+# --- top-k ---------------------------------------------------------------------
+
+def _brute_rank(scores_row, k, ascending):
+    n = scores_row.size
+    better = np.zeros(n, dtype=np.int64)
+    for i in range(n):
+        for j in range(n):
+            if ascending:
+                b = scores_row[j] < scores_row[i] or (scores_row[j] == scores_row[i] and j < i)
+            else:
+                b = scores_row[j] > scores_row[i] or (scores_row[j] == scores_row[i] and j < i)
+            better[i] += b
+    order = np.argsort(better)
+    return order[:k]
+
+
+@pytest.mark.parametrize("metric", [oracle.IP, oracle.COSINE, oracle.L2])
+def test_topk_brute_force_with_ties(metric):
+    rng = np.random.default_rng(metric + 1)
+    for n in (1, 2, 7, 33, 64):
+        s = rng.integers(-4, 5, size=(3, n)).astype(np.float32) / 4  # many exact ties
+        for k in sorted({1, min(3, n), n}):
+            got_s, got_i = oracle.topk(s, k, metric)
+            for b in range(3):
+                want = _brute_rank(s[b], k, ascending=(metric == oracle.L2))
+                np.testing.assert_array_equal(got_i[b], want)
+                np.testing.assert_array_equal(got_s[b], s[b][want])
+
+
+def test_topk_direction_and_lowest_index():
+    s = np.array([[0.5, 0.9, 0.9, -0.1]], dtype=np.float32)
+    _, ids = oracle.topk(s, 3, oracle.IP)
+    assert list(ids[0]) == [1, 2, 0]
+    _, ids = oracle.topk(s, 3, oracle.L2)
+    assert list(ids[0]) == [3, 0, 1]
+
+
+def test_search_driver_threads_agree():
+    x = inputs.unit_rows(500, 64, seed=2)
+    q = inputs.queries(5, 64, seed=3)
+    codes, *_ = oracle.quantize(x, 1e-2)
+    codes = codes.reshape(x.shape)
+    for metric in (oracle.IP, oracle.COSINE, oracle.L2):
+        full = oracle.scores(q, codes, 1e-2, metric)
+        ws, wi = oracle.topk(full, 17, metric)
+        for nt in (1, 3, 8):
+            gs, gi = oracle.search(q, codes, 1e-2, metric, 17, nthreads=nt)
+            np.testing.assert_array_equal(gi, wi)
+            np.testing.assert_array_equal(gs, ws)
+
+
+def test_numpy_rint_cross_check():
+    # Not a pin (it restates the formula), but a guard on the C build flags.
+    x = inputs.flat_values(1 << 21, seed=9)
+    for eps in EPS_SWEEP:
+        codes, *_ = oracle.quantize(x, eps)
+        s = np.float32(2.0) * np.float32(eps)
+        np.testing.assert_array_equal(codes, np.rint(x / s).astype(np.int32))
