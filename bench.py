@@ -1,0 +1,418 @@
+"""Benchmark of LAM's quantized-memory hot path on GB300.
+
+One step is one pass of the whole path over one batch: for each eps of the
+sweep, Q_eps with the narrowest width (range pass + quantize), dequantisation
+of the codes (round trip), and exact top-k search of the query batch on the
+codes (fused dequant + score + top-k, then the merge of partial lists).  All
+of it runs through the C ABI on device-resident inputs; the value is memory
+vectors per second through the whole path.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+    python bench.py --impl reference ...   # the CPU oracle, timed on host cores
+
+With --gpus N > 1 (launched by torchrun) every rank runs an independent
+replica of the workload on its own GPU; there is no exchange between ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "Q_ε GB/s and fused score+top-k memory vectors/s at D=768; % of HBM roofline"
+UNIT = "memory vectors/s"
+L2_FLUSH_BYTES = 512 << 20
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=300)
+    p.add_argument("--warmup", type=int, default=10)
+    p.add_argument("--impl", default="lam", choices=["lam", "reference"])
+    p.add_argument("--workload", default="chunks_n27986_ip")
+    p.add_argument("--batch", type=int, default=0, help="query batch (default: workload's first)")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    return p.parse_args()
+
+
+def load_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            pk = json.load(f)
+        return pk["hbm_gbs"], pk["bf16_tflops"], "measured"
+    except Exception:
+        return 6800.0, 1900.0, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle-reason samples during the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.path = os.path.join(ROOT, "gpurun_out", "clocks_bench_rank%d.csv" % index)
+
+    def __enter__(self):
+        try:
+            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.FIELDS,
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=self.fh, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+            self.fh.close()
+
+    def summary(self):
+        if self.proc is None:
+            return None
+        rows = []
+        try:
+            for line in open(self.path):
+                f = [x.strip() for x in line.split(",")]
+                if len(f) >= 9:
+                    rows.append(f)
+        except Exception:
+            return None
+        if not rows:
+            return None
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[j] for r in rows for j in range(4) if r[5 + j] == "Active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons,
+                "samples": len(rows)}
+
+
+def dist_setup(args):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        backend = "nccl" if args.impl == "lam" else "gloo"
+        dist.init_process_group(backend=backend)
+    return world, rank, local
+
+
+def max_over_ranks(value, world, device=None):
+    if world == 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+# ----------------------------------------------------------------- lam arm --
+
+class Pipeline:
+    """Buffers and calls of one step, all through the C ABI."""
+
+    def __init__(self, lam, torch, x, q, eps_list, k, metric, dev):
+        self.lam, self.torch = lam, torch
+        self.x, self.q = x, q
+        self.eps_list, self.k, self.metric = eps_list, k, metric
+        self.N, self.D = x.shape
+        self.B = q.shape[0]
+        self.dev = dev
+        n = x.numel()
+        self.codes = torch.empty(n * 4, dtype=torch.uint8, device=dev)  # fits any width
+        self.deq = torch.empty_like(x)
+        self.qws = torch.zeros(64, dtype=torch.uint8, device=dev)
+        self.scores = [torch.empty((self.B, k), dtype=torch.float32, device=dev) for _ in eps_list]
+        self.ids = [torch.empty((self.B, k), dtype=torch.int64, device=dev) for _ in eps_list]
+        # widths and code bounds from a first (untimed) quantization
+        self.plan = []
+        wsz = 0
+        for e in eps_list:
+            st, w, s, cmin, cmax = lam.lam_quantize(x, e, 0, None, self.qws)
+            bound = max(-cmin, cmax)
+            wsz = max(wsz, lam.lam_score_topk_workspace_size(self.B, self.N, self.D, k, w, bound))
+            self.plan.append((w, bound, lam.lam_score_topk_path(self.B, self.N, self.D, k, w, bound)))
+        self.sws = torch.empty(wsz, dtype=torch.uint8, device=dev)
+
+    def launches_per_step(self):
+        n = 0
+        for (_, _, path) in self.plan:
+            n += 2 + 1  # range + quantize, dequantize
+            n += 3 if path == self.lam.PATH_TENSOR else 2  # (qprep) + score + merge
+        return n
+
+    def step(self, ev=None):
+        lam = self.lam
+        for j, e in enumerate(self.eps_list):
+            if ev is not None:
+                ev[j][0].record()
+            st, w, s, cmin, cmax = lam.lam_quantize(self.x, e, 0, self.codes, self.qws)
+            if ev is not None:
+                ev[j][1].record()
+            lam.lam_dequantize(self.codes, w, self.x.numel(), s, self.deq)
+            if ev is not None:
+                ev[j][2].record()
+            lam.lam_score_topk(self.q, self.codes, w, self.N, self.D, e, max(-cmin, cmax), self.k,
+                               self.metric, self.scores[j], self.ids[j], self.sws)
+            if ev is not None:
+                ev[j][3].record()
+
+
+def cpu_baseline_lam_units(x_np, q_np, eps_list, k, metric, cores, budget_q=64):
+    """Times the oracle on host cores on a bounded sample; returns a dict."""
+    import numpy as np
+    import oracle
+    N, D = x_np.shape
+    B = q_np.shape[0]
+    b = min(B, budget_q)
+    t_total = 0.0
+    for e in eps_list:
+        t0 = time.perf_counter()
+        oc, *_ = oracle.quantize(x_np, e)
+        t1 = time.perf_counter()
+        oracle.dequantize(oc, oracle.step(e))
+        t2 = time.perf_counter()
+        oracle.search(q_np[:b], oc.reshape(N, D), e, metric, k, nthreads=cores)
+        t3 = time.perf_counter()
+        t_total += (t1 - t0) + (t2 - t1) + (t3 - t2) * (B / b)
+    units = N * len(eps_list)
+    return {"value": units / t_total, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": "quantize + dequantize of all %dx%d values per eps and exact search of "
+                      "%d of the %d queries (search time scaled to %d), eps %s" %
+                      (N, D, b, B, B, list(eps_list))}
+
+
+def run_lam(args):
+    import numpy as np
+    import torch
+    import paper_2609_32256_gb300 as lam
+    from paper_2609_32256_gb300 import build as lam_build, inputs
+
+    world, rank, local = dist_setup(args)
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if rank == 0 or world == 1:
+        lam_build.build()
+    barrier(world)
+    lam.load()
+
+    wl = inputs.WORKLOADS[args.workload]
+    B = args.batch or wl.batches[0]
+    if wl.planted:
+        x_np = inputs.planted_rows(wl.n, wl.d, seed=0)
+    else:
+        x_np = inputs.unit_rows(wl.n, wl.d, seed=0)
+    q_np = inputs.queries(B, wl.d, seed=1)
+    x = torch.from_numpy(x_np).to(dev)
+    q = torch.from_numpy(q_np).to(dev)
+    pipe = Pipeline(lam, torch, x, q, wl.eps, wl.k, wl.metric, dev)
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    for i in range(args.warmup):
+        flush.fill_(float(i))
+        pipe.step()
+    torch.cuda.synchronize(dev)
+
+    ne = len(wl.eps)
+    evs = [[[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(ne)]
+           for _ in range(args.steps)]
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    sampler = ClockSampler(local)
+    with sampler:
+        for i in range(args.steps):
+            flush.fill_(float(i))  # L2 flush between timed steps (outside the events)
+            pipe.step(evs[i])
+        torch.cuda.synchronize(dev)
+    barrier(world)
+
+    t_q = t_d = t_s = 0.0
+    for i in range(args.steps):
+        for j in range(ne):
+            e = evs[i][j]
+            t_q += e[0].elapsed_time(e[1])
+            t_d += e[1].elapsed_time(e[2])
+            t_s += e[2].elapsed_time(e[3])
+    ms_step = (t_q + t_d + t_s) / args.steps
+    ms_step = max_over_ranks(ms_step, world, dev)
+    units_per_step = wl.n * ne
+    value = units_per_step * world / (ms_step / 1e3)
+
+    # per-stage figures (rank-local)
+    nd = wl.n * wl.d
+    widths = [w for (w, _, _) in pipe.plan]
+    q_bytes = sum((4 + w) * nd for w in widths)       # one quantize pass at the resolved width
+    d_bytes = sum((w + 4) * nd for w in widths)
+    flops = 2.0 * wl.n * wl.d * B * ne
+    ms_q, ms_d, ms_s = t_q / args.steps, t_d / args.steps, t_s / args.steps
+    hbm_peak, tc_peak, peak_kind = load_peaks()
+    path_names = {0: "bandwidth", 1: "tensor", 2: "generic"}
+    paths = [path_names[p] for (_, _, p) in pipe.plan]
+    if all(p == "tensor" for p in paths):
+        achieved = flops / (ms_s / 1e3) / 1e12
+        roofline = {"bound": "tensor", "achieved": round(achieved, 2), "peak": tc_peak,
+                    "unit": "TFLOP/s", "frac": round(achieved / tc_peak, 4), "traffic": None,
+                    "kernel": "score_tc_kernel (timed span: lam_score_topk = query prep + "
+                              "tcgen05 score + merge)", "peak_source": peak_kind + " bf16 dense burst "
+                              "(fp16 has the same nominal rate)"}
+    else:
+        sb = sum(w * nd for w in widths)
+        achieved = sb / (ms_s / 1e3) / 1e9
+        roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": hbm_peak,
+                    "unit": "GB/s", "frac": round(achieved / hbm_peak, 4), "traffic": None,
+                    "kernel": "score (lam_score_topk span)", "peak_source": peak_kind + " copy"}
+
+    # end to end: host (pinned) inputs, copies inside the timed region
+    x_h = x.cpu().pin_memory()
+    q_h = q.cpu().pin_memory()
+    res_h = [(torch.empty((B, wl.k), dtype=torch.float32).pin_memory(),
+              torch.empty((B, wl.k), dtype=torch.int64).pin_memory()) for _ in wl.eps]
+    e2e_steps = max(3, min(args.steps, 50))
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    tot = 0.0
+    for i in range(e2e_steps + 2):
+        flush.fill_(float(i))
+        e0.record()
+        x.copy_(x_h, non_blocking=True)
+        q.copy_(q_h, non_blocking=True)
+        pipe.step()
+        for j in range(ne):
+            res_h[j][0].copy_(pipe.scores[j], non_blocking=True)
+            res_h[j][1].copy_(pipe.ids[j], non_blocking=True)
+        e1.record()
+        torch.cuda.synchronize(dev)
+        if i >= 2:
+            tot += e0.elapsed_time(e1)
+    ms_e2e = max_over_ranks(tot / e2e_steps, world, dev)
+    e2e = {"value": units_per_step * world / (ms_e2e / 1e3), "unit": UNIT,
+           "h2d_bytes_per_step": x_h.numel() * 4 + q_h.numel() * 4,
+           "d2h_bytes_per_step": ne * B * wl.k * (4 + 8)}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cores = os.cpu_count() or 1
+        cpu = cpu_baseline_lam_units(x_np, q_np, wl.eps, wl.k, wl.metric, cores)
+
+    if rank == 0:
+        out = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "f32 in, int%d codes, fp16x2-split tensor / fp32 accumulate" % (8 * max(widths)),
+            "data": "synthetic (seeded unit-Gaussian rows shaped like bge-base D=768 embeddings)",
+            "config": {"workload": wl.name, "N": wl.n, "D": wl.d, "batch": B, "k": wl.k,
+                       "metric": ["ip", "cosine", "l2"][wl.metric], "eps": list(wl.eps),
+                       "widths": widths, "paths": paths, "parallelism": "replicas only",
+                       "l2": "flushed between timed steps (512 MB write, outside the events)"},
+            "breakdown": {
+                "quantize_ms": ms_q, "quantize_gbs_algorithmic": q_bytes / (ms_q / 1e3) / 1e9,
+                "quantize_note": "lam_quantize span: range pass + quantize + status read-back",
+                "dequantize_ms": ms_d, "dequantize_gbs": d_bytes / (ms_d / 1e3) / 1e9,
+                "score_ms": ms_s, "score_vectors_per_s": wl.n * ne / (ms_s / 1e3),
+                "score_tflops": flops / (ms_s / 1e3) / 1e12},
+            "roofline": roofline,
+            "cpu_baseline": cpu,
+            "e2e": e2e,
+            "gpu_launches": pipe.launches_per_step() * args.steps,
+            "clocks": sampler.summary(),
+        }
+        print(json.dumps(out))
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+# ----------------------------------------------------------- reference arm --
+
+def run_reference(args):
+    """The CPU oracle on the host cores, same metric, bounded sample per step."""
+    world, rank, _ = dist_setup(args)
+    if rank != 0:
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+        return
+    import numpy as np
+    import oracle
+    from paper_2609_32256_gb300 import inputs
+    oracle.build()
+    wl = inputs.WORKLOADS[args.workload]
+    B = args.batch or wl.batches[0]
+    x_np = inputs.planted_rows(wl.n, wl.d, seed=0) if wl.planted else inputs.unit_rows(wl.n, wl.d, seed=0)
+    q_np = inputs.queries(B, wl.d, seed=1)
+    cores = os.cpu_count() or 1
+    S, b = 2048, 4  # rows and queries per step
+    ne = len(wl.eps)
+
+    def one(i):
+        e = wl.eps[i % ne]
+        r0 = (i * S) % max(1, wl.n - S)
+        xs = x_np[r0:r0 + S]
+        t0 = time.perf_counter()
+        oc, *_ = oracle.quantize(xs, e)
+        oracle.dequantize(oc, oracle.step(e))
+        t1 = time.perf_counter()
+        oracle.search(q_np[:b], oc.reshape(xs.shape), e, wl.metric, wl.k, nthreads=cores)
+        t2 = time.perf_counter()
+        return (t1 - t0) + (t2 - t1) * (B / b)
+
+    for i in range(args.warmup):
+        one(i)
+    tot = sum(one(i) for i in range(args.steps))
+    ms = tot / args.steps * 1e3
+    value = S / (ms / 1e3)
+    out = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+           "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+           "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+           "data": "synthetic", "config": {"workload": wl.name, "N": wl.n, "D": wl.d, "batch": B,
+                                           "k": wl.k, "eps": list(wl.eps)},
+           "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                            "sample": "per step %d rows quantized, dequantized and searched by "
+                                      "%d queries (search time scaled to %d queries), eps rotating"
+                                      % (S, b, B)},
+           "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(out))
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_lam(args)
+
+
+if __name__ == "__main__":
+    main()

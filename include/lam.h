@@ -1,0 +1,180 @@
+/*
+ * lam.h -- C ABI of the GB300 (sm_103a) library for LAM's quantized memory.
+ *
+ * The method (paper: "LAM: Lossy Agent Memory"):
+ *   - Q_eps(x) = round(x / 2 eps), coordinatewise with one global eps
+ *     (Sec. 3.2 "Three layers", layer L1; Algorithm 1 applies it to every
+ *     arriving embedding).
+ *   - Dequantisation xhat = 2 eps * Q_eps(x): a cell of the quantizer has
+ *     half-width eps (Sec. 3.1; App. "Rank invariance, in full").
+ *   - Exact search over the stored vectors is one matrix-vector product per
+ *     query followed by a top-k (Sec. "Brute-force scan crossover"); here it
+ *     runs directly on the integer codes, with dequantisation folded into the
+ *     score.
+ *
+ * Conventions shared by every call:
+ *   - Every array argument is a DEVICE pointer on the current CUDA device,
+ *     allocated and owned by the caller.  The library allocates no memory.
+ *     Only the scalar outputs of lam_quantize and lam_score_topk_status are
+ *     host pointers.
+ *   - Arrays are dense and row-major.  Codes are two's-complement integers of
+ *     1, 2 or 4 bytes ("width").
+ *   - `stream` is a cudaStream_t (NULL = the legacy default stream).  Work is
+ *     queued on it; lam_quantize and lam_score_topk_status also wait for it.
+ *   - Arguments are checked on the host before anything is queued; a bad
+ *     argument returns LAM_ERR_INVALID and queues nothing.
+ *   - Rounding: the quotient x / 2eps is one IEEE fp32 division by
+ *     s = fl32(2 * eps) and is rounded half-to-even; dequantisation is one
+ *     fp32 multiply s * code.  No fast-math arithmetic is used.
+ */
+#ifndef LAM_H
+#define LAM_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* A cudaStream_t. */
+typedef struct CUstream_st *lam_stream_t;
+
+typedef enum lam_status {
+  LAM_OK = 0,
+  LAM_ERR_INVALID = 1,     /* bad argument; nothing was queued             */
+  LAM_ERR_RANGE = 2,       /* codes do not fit the requested/needed width  */
+  LAM_ERR_NONFINITE = 3,   /* NaN or Inf in the input of lam_quantize      */
+  LAM_ERR_WORKSPACE = 4,   /* an output or workspace buffer is too small   */
+  LAM_ERR_CUDA = 5,        /* a CUDA runtime call or launch failed         */
+  LAM_ERR_TIMEOUT = 6,     /* a bounded device-side wait gave up           */
+  LAM_ERR_UNSUPPORTED = 7  /* a forced kernel path cannot take this shape  */
+} lam_status;
+
+/* Code widths, in bytes.  LAM_WIDTH_AUTO asks lam_quantize for the narrowest. */
+enum { LAM_WIDTH_AUTO = 0, LAM_I8 = 1, LAM_I16 = 2, LAM_I32 = 4 };
+
+/* Scores: inner product and cosine rank descending, squared L2 ascending. */
+enum { LAM_METRIC_IP = 0, LAM_METRIC_COSINE = 1, LAM_METRIC_L2 = 2 };
+
+/* Library version, major*10000 + minor*100 + patch. */
+int32_t lam_version(void);
+
+/* Static text for a status code. */
+const char *lam_status_string(int32_t status);
+
+/* Bytes of device workspace lam_quantize needs (a small status block). */
+size_t lam_quantize_workspace_size(void);
+
+/*
+ * lam_quantize -- Q_eps over n fp32 values (Sec. 3.2, layer L1).
+ *
+ *   code_i = round_half_even(fl32(x_i / s)),  s = fl32(2 * eps)
+ *
+ * x          [n] fp32, device, 4-byte aligned (16-byte alignment of x and
+ *            codes selects the 128-bit vector path).
+ * n          number of values, 0 <= n < 2^62.
+ * eps        finite, > 0, and 2*eps a normal fp32 number.
+ * width_req  LAM_I8, LAM_I16, LAM_I32, or LAM_WIDTH_AUTO for the narrowest
+ *            width whose range holds [min code, max code] (int8 when n == 0).
+ * codes      [n] codes of the resolved width, device, aligned to the width
+ *            (AUTO: 4-byte aligned); may be NULL to ask only for the range and
+ *            width.  Contents are undefined unless LAM_OK.
+ * codes_bytes  size of `codes`; must be >= n * width (AUTO: of the width that
+ *            is resolved -- n * 4 always suffices).
+ * workspace  >= lam_quantize_workspace_size() bytes of device memory,
+ *            16-byte aligned; it may be reused between calls on one stream.
+ * width_out, scale_out, code_min_out, code_max_out   host outputs (any may be
+ *            NULL): the width used, s = 2*eps, and the smallest and largest
+ *            code.  They are written for LAM_OK and LAM_ERR_RANGE.
+ *
+ * Synchronous on `stream`: the status block is read back, because the width
+ * and the range are outputs.  Errors: LAM_ERR_NONFINITE (NaN/Inf in x),
+ * LAM_ERR_RANGE (a forced width, or int32, cannot hold the codes),
+ * LAM_ERR_WORKSPACE (codes_bytes or the workspace is too small), LAM_ERR_CUDA.
+ */
+lam_status lam_quantize(const float *x, int64_t n, float eps, int32_t width_req,
+                        void *codes, size_t codes_bytes, void *workspace,
+                        size_t workspace_bytes, int32_t *width_out,
+                        float *scale_out, int32_t *code_min_out,
+                        int32_t *code_max_out, lam_stream_t stream);
+
+/*
+ * lam_dequantize -- xhat_i = fl32(scale * code_i), the inverse map of Q_eps
+ * up to the cell half-width eps (|x - xhat| <= eps, Sec. 3.1).
+ *
+ * codes  [n] of `width` bytes (1, 2 or 4), device, aligned to the width.
+ * out    [n] fp32, device, 4-byte aligned.
+ * scale  the step s returned by lam_quantize (s = 2 eps).
+ * Asynchronous on `stream`.  Errors: LAM_ERR_INVALID, LAM_ERR_CUDA.
+ */
+lam_status lam_dequantize(const void *codes, int32_t width, int64_t n,
+                          float scale, float *out, lam_stream_t stream);
+
+/*
+ * Bytes of device workspace lam_score_topk needs for this shape on the
+ * current device (arguments as for lam_score_topk).  0 for invalid shapes.
+ */
+size_t lam_score_topk_workspace_size(int64_t B, int64_t N, int32_t D,
+                                     int32_t k, int32_t width,
+                                     int32_t code_bound);
+
+/*
+ * lam_score_topk -- exact search on the codes (Sec. "Brute-force scan
+ * crossover"): every query against every stored row, dequantisation folded
+ * into the score, then the k best per query.
+ *
+ *   inner product  s * sum_d q_d c_d                     (descending)
+ *   cosine         sum_d q_d c_d / (||q|| ||c||)          (descending; 0 if a
+ *                  norm is 0 -- the norm of the dequantised row, s cancels)
+ *   squared L2     ||q||^2 - 2 s q.c + s^2 ||c||^2        (ascending)
+ *
+ * with s = fl32(2 * eps).  Ties between equal fp32 scores go to the lower row
+ * id (the paper's lowest-index rule, Algorithm 1).
+ *
+ * queries    [B, D] fp32, device, 4-byte aligned.  B >= 1.
+ * codes      [N, D] codes of `width` bytes, device, aligned to the width (a
+ *            16-byte aligned base enables the bulk-copy and TMA paths).
+ *            1 <= k <= N < 2^31.
+ * code_bound the largest |code| if known (e.g. max(-code_min, code_max) from
+ *            lam_quantize), else 0; with int16 codes a bound <= 2048 enables
+ *            the tensor-core path.  A bound smaller than the real codes gives
+ *            LAM_ERR_RANGE from lam_score_topk_status.
+ * k          1 <= k <= min(N, 1024).
+ * scores     [B, k] fp32, device, best first.  ids [B, k] int64, device
+ *            (naturally aligned).
+ * workspace  >= lam_score_topk_workspace_size(...) bytes, device, 256-byte
+ *            aligned.  Calls that share a workspace must not overlap.
+ *
+ * Asynchronous on `stream`.  Device-side faults of the data (a code beyond
+ * code_bound) and bounded-wait timeouts are recorded in the workspace; read
+ * them with lam_score_topk_status.  The environment variable LAM_SCORE_PATH
+ * (auto|bandwidth|tensor|generic) forces one kernel path for testing; a
+ * forced path that cannot take the shape returns LAM_ERR_UNSUPPORTED.
+ */
+lam_status lam_score_topk(const float *queries, int64_t B, const void *codes,
+                          int32_t width, int64_t N, int32_t D, float eps,
+                          int32_t code_bound, int32_t k, int32_t metric,
+                          float *scores, int64_t *ids, void *workspace,
+                          size_t workspace_bytes, lam_stream_t stream);
+
+/*
+ * Waits for `stream`, then reads the device status the last lam_score_topk
+ * on this workspace recorded: LAM_OK, LAM_ERR_RANGE or LAM_ERR_TIMEOUT
+ * (written to *status_out).  Returns LAM_ERR_CUDA if the read fails.
+ */
+lam_status lam_score_topk_status(const void *workspace, lam_stream_t stream,
+                                 int32_t *status_out);
+
+/*
+ * The kernel path lam_score_topk takes for a shape: 0 bandwidth (CUDA cores,
+ * small batches), 1 tensor (tcgen05), 2 generic; -1 if the shape is invalid.
+ */
+int32_t lam_score_topk_path(int64_t B, int64_t N, int32_t D, int32_t k,
+                            int32_t width, int32_t code_bound);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* LAM_H */

@@ -1,0 +1,74 @@
+"""GB300 (sm_103a) library for LAM's quantized agent memory.
+
+The C ABI (include/lam.h, built as liblam.so) computes the error-bounded
+quantizer Q_eps(x) = round(x / 2 eps) over fp32 embeddings, its inverse, and
+exact top-k retrieval scored directly on the integer codes.  This package is
+the Python side: the ctypes binding (`_lib`, same names as the C calls) and a
+few conveniences that allocate outputs with PyTorch.  PyTorch only provides
+device memory and streams; every step runs in the library's kernels.
+"""
+from __future__ import annotations
+
+from ._lib import (LAM_ERR_CUDA, LAM_ERR_INVALID, LAM_ERR_NONFINITE, LAM_ERR_RANGE,
+                   LAM_ERR_TIMEOUT, LAM_ERR_UNSUPPORTED, LAM_ERR_WORKSPACE, LAM_I8, LAM_I16,
+                   LAM_I32, LAM_METRIC_COSINE, LAM_METRIC_IP, LAM_METRIC_L2, LAM_OK,
+                   LAM_WIDTH_AUTO, PATH_BANDWIDTH, PATH_GENERIC, PATH_TENSOR, LamError,
+                   lam_dequantize, lam_quantize, lam_quantize_workspace_size,
+                   lam_score_topk, lam_score_topk_path, lam_score_topk_status,
+                   lam_score_topk_workspace_size, lam_status_string, lam_version, load)
+
+CODE_DTYPES = {1: "int8", 2: "int16", 4: "int32"}
+
+
+def _torch():
+    import torch
+    return torch
+
+
+def quantize(x, eps, width=LAM_WIDTH_AUTO, stream=None):
+    """Q_eps of a CUDA fp32 tensor.
+
+    Returns (codes, width, scale, code_min, code_max); codes has x's shape and
+    the narrowest integer dtype (or the forced one).
+    """
+    torch = _torch()
+    x = x.contiguous()
+    n = x.numel()
+    ws = torch.empty(max(16, lam_quantize_workspace_size()), dtype=torch.uint8, device=x.device)
+    if width == LAM_WIDTH_AUTO:
+        _, w, _, _, _ = lam_quantize(x, eps, LAM_WIDTH_AUTO, None, ws, stream)
+    else:
+        w = width
+    codes = torch.empty(x.shape, dtype=getattr(torch, CODE_DTYPES[w]), device=x.device)
+    _, w2, scale, cmin, cmax = lam_quantize(x, eps, w, codes if n else None, ws, stream)
+    return codes, w2, scale, cmin, cmax
+
+
+def dequantize(codes, scale, stream=None):
+    """scale * codes as a CUDA fp32 tensor of the same shape."""
+    torch = _torch()
+    w = codes.element_size()
+    out = torch.empty(codes.shape, dtype=torch.float32, device=codes.device)
+    lam_dequantize(codes.contiguous(), w, codes.numel(), scale, out, stream)
+    return out
+
+
+def search(queries, codes, eps, k, metric=LAM_METRIC_IP, code_bound=0, stream=None):
+    """Top-k of every query against every code row: (scores [B,k] f32, ids [B,k] i64)."""
+    torch = _torch()
+    queries = queries.contiguous()
+    codes = codes.contiguous()
+    B, D = queries.shape
+    N = codes.shape[0]
+    w = codes.element_size()
+    nbytes = lam_score_topk_workspace_size(B, N, D, k, w, code_bound)
+    if nbytes == 0:
+        raise LamError(LAM_ERR_INVALID, "lam_score_topk_workspace_size")
+    ws = torch.empty(nbytes, dtype=torch.uint8, device=queries.device)
+    scores = torch.empty((B, k), dtype=torch.float32, device=queries.device)
+    ids = torch.empty((B, k), dtype=torch.int64, device=queries.device)
+    lam_score_topk(queries, codes, w, N, D, eps, code_bound, k, metric, scores, ids, ws, stream)
+    st = lam_score_topk_status(ws, stream)
+    if st != LAM_OK:
+        raise LamError(st, "lam_score_topk")
+    return scores, ids

@@ -1,0 +1,151 @@
+"""Thin ctypes binding of the C ABI in include/lam.h (argument marshalling only).
+
+Every function keeps the name of the C entry point it wraps.  Tensors are
+passed by device pointer; the CUDA stream defaults to torch's current stream
+on the tensor's device.  Every computation runs in liblam.so: if the library
+is missing, the first call raises instead of falling back to anything else.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "liblam.so")
+
+LAM_OK, LAM_ERR_INVALID, LAM_ERR_RANGE, LAM_ERR_NONFINITE = 0, 1, 2, 3
+LAM_ERR_WORKSPACE, LAM_ERR_CUDA, LAM_ERR_TIMEOUT, LAM_ERR_UNSUPPORTED = 4, 5, 6, 7
+LAM_WIDTH_AUTO, LAM_I8, LAM_I16, LAM_I32 = 0, 1, 2, 4
+LAM_METRIC_IP, LAM_METRIC_COSINE, LAM_METRIC_L2 = 0, 1, 2
+PATH_BANDWIDTH, PATH_TENSOR, PATH_GENERIC = 0, 1, 2
+
+
+class LamError(RuntimeError):
+    """A non-OK lam_status."""
+
+    def __init__(self, status: int, where: str):
+        self.status = int(status)
+        super().__init__("%s: %s (status %d)" % (where, lam_status_string(status), status))
+
+
+_lib = None
+
+
+def load():
+    """Load liblam.so (raises if it has not been built)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise RuntimeError("liblam.so is not built: call paper_2609_32256_gb300.build.build()")
+    lib = ctypes.CDLL(LIB_PATH)
+    vp, i32, i64, f32, sz = (ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64,
+                             ctypes.c_float, ctypes.c_size_t)
+    P = ctypes.POINTER
+    sig = {
+        "lam_version": (i32, []),
+        "lam_status_string": (ctypes.c_char_p, [i32]),
+        "lam_quantize_workspace_size": (sz, []),
+        "lam_quantize": (i32, [vp, i64, f32, i32, vp, sz, vp, sz, P(i32), P(f32), P(i32),
+                               P(i32), vp]),
+        "lam_dequantize": (i32, [vp, i32, i64, f32, vp, vp]),
+        "lam_score_topk_workspace_size": (sz, [i64, i64, i32, i32, i32, i32]),
+        "lam_score_topk": (i32, [vp, i64, vp, i32, i64, i32, f32, i32, i32, i32, vp, vp, vp,
+                                 sz, vp]),
+        "lam_score_topk_status": (i32, [vp, vp, P(i32)]),
+        "lam_score_topk_path": (i32, [i64, i64, i32, i32, i32, i32]),
+    }
+    for name, (res, args) in sig.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    _lib = lib
+    return lib
+
+
+def _stream(stream, device=None):
+    if stream is not None:
+        return ctypes.c_void_p(int(stream))
+    import torch
+    return ctypes.c_void_p(torch.cuda.current_stream(device).cuda_stream)
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _nbytes(t):
+    return 0 if t is None else t.numel() * t.element_size()
+
+
+def _check(status, where):
+    if status != LAM_OK:
+        raise LamError(status, where)
+
+
+def lam_version() -> int:
+    return int(load().lam_version())
+
+
+def lam_status_string(status: int) -> str:
+    return load().lam_status_string(int(status)).decode()
+
+
+def lam_quantize_workspace_size() -> int:
+    return int(load().lam_quantize_workspace_size())
+
+
+def lam_quantize(x, eps, width_req=LAM_WIDTH_AUTO, codes=None, workspace=None, stream=None,
+                 raise_on_error=True):
+    """Q_eps of the fp32 CUDA tensor x into `codes` (a CUDA tensor or None).
+
+    Returns (status, width, scale, code_min, code_max).  `workspace` is a CUDA
+    tensor of >= lam_quantize_workspace_size() bytes (16-byte aligned).
+    """
+    w = ctypes.c_int32(0)
+    s = ctypes.c_float(0)
+    cmin = ctypes.c_int32(0)
+    cmax = ctypes.c_int32(0)
+    st = load().lam_quantize(_ptr(x), x.numel(), ctypes.c_float(eps), int(width_req),
+                             _ptr(codes), _nbytes(codes), _ptr(workspace), _nbytes(workspace),
+                             ctypes.byref(w), ctypes.byref(s), ctypes.byref(cmin),
+                             ctypes.byref(cmax), _stream(stream, x.device))
+    if raise_on_error and st not in (LAM_OK,):
+        raise LamError(st, "lam_quantize")
+    return int(st), w.value, s.value, cmin.value, cmax.value
+
+
+def lam_dequantize(codes, width, n, scale, out, stream=None):
+    """out[0:n] = scale * codes[0:n] (fp32), asynchronous on the stream."""
+    st = load().lam_dequantize(_ptr(codes), int(width), int(n), ctypes.c_float(scale),
+                               _ptr(out), _stream(stream, out.device))
+    _check(st, "lam_dequantize")
+
+
+def lam_score_topk_workspace_size(B, N, D, k, width, code_bound) -> int:
+    return int(load().lam_score_topk_workspace_size(int(B), int(N), int(D), int(k), int(width),
+                                                    int(code_bound)))
+
+
+def lam_score_topk_path(B, N, D, k, width, code_bound) -> int:
+    return int(load().lam_score_topk_path(int(B), int(N), int(D), int(k), int(width),
+                                          int(code_bound)))
+
+
+def lam_score_topk(queries, codes, width, N, D, eps, code_bound, k, metric, scores, ids,
+                   workspace, stream=None):
+    """Exact search on the codes; writes scores [B, k] and ids [B, k] (asynchronous)."""
+    B = queries.shape[0]
+    st = load().lam_score_topk(_ptr(queries), int(B), _ptr(codes), int(width), int(N), int(D),
+                               ctypes.c_float(eps), int(code_bound), int(k), int(metric),
+                               _ptr(scores), _ptr(ids), _ptr(workspace), _nbytes(workspace),
+                               _stream(stream, queries.device))
+    _check(st, "lam_score_topk")
+
+
+def lam_score_topk_status(workspace, stream=None) -> int:
+    out = ctypes.c_int32(0)
+    st = load().lam_score_topk_status(_ptr(workspace), _stream(stream, workspace.device),
+                                      ctypes.byref(out))
+    _check(st, "lam_score_topk_status")
+    return out.value

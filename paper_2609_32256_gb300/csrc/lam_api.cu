@@ -1,0 +1,325 @@
+// lam_api.cu -- the C ABI (include/lam.h): argument checks, planning of the
+// scoring path and its workspace, and the launches.  The library allocates no
+// device memory; its only state is a per-device cache of the SM count.
+#include <math.h>
+#include <stdlib.h>
+#include <string.h>
+
+#include "lam_internal.cuh"
+
+namespace {
+
+using namespace lam;
+
+int device_sms() {
+  static int cache[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+  if (dev >= 0 && dev < 64 && cache[dev] > 0) return cache[dev];
+  int v = 0;
+  if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+  if (dev >= 0 && dev < 64) cache[dev] = v;
+  return v;
+}
+
+bool valid_width(int32_t w) { return w == 1 || w == 2 || w == 4; }
+
+// eps finite, > 0, and s = 2 eps a normal fp32 number.
+bool valid_eps(float eps) {
+  if (!(eps > 0.0f) || !isfinite(eps)) return false;
+  const float s = 2.0f * eps;
+  return isfinite(s) && isnormal(s);
+}
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// Host replica of the device width resolution (same fp32 ops, half-to-even).
+float host_qround(float x, float s) {
+  const float q = x / s;
+  return nearbyintf(q);
+}
+
+float unord_host(uint32_t o) {
+  uint32_t b = (o & 0x80000000u) ? (o & 0x7FFFFFFFu) : ~o;
+  float f;
+  memcpy(&f, &b, 4);
+  return f;
+}
+
+int width_of(float rmin, float rmax) {
+  if (rmin >= -128.0f && rmax <= 127.0f) return 1;
+  if (rmin >= -32768.0f && rmax <= 32767.0f) return 2;
+  if (rmin >= -2147483648.0f && rmax < 2147483648.0f) return 4;
+  return 0;
+}
+
+struct Plan {
+  int path = -1;
+  int n_lists = 0;
+  int64_t Bpad = 0;
+  size_t partial_off = 0, qprep_off = 0, total = 0;
+};
+
+int forced_path() {
+  const char *e = getenv("LAM_SCORE_PATH");
+  if (e == nullptr || *e == 0 || strcmp(e, "auto") == 0) return -1;
+  if (strcmp(e, "bandwidth") == 0) return kPathBandwidth;
+  if (strcmp(e, "tensor") == 0) return kPathTensor;
+  if (strcmp(e, "generic") == 0) return kPathGeneric;
+  return -2;
+}
+
+bool shape_ok(int64_t B, int64_t N, int32_t D, int32_t k, int32_t width, int32_t code_bound) {
+  return B >= 1 && B <= (1LL << 31) && N >= 1 && N < 2147483647LL && D >= 1 &&
+         D <= (1 << 20) && k >= 1 && k <= kMaxK && k <= N && valid_width(width) &&
+         code_bound >= 0 && (int64_t)N * D < (1LL << 46);
+}
+
+bool bandwidth_ok(int64_t B, int32_t D, int32_t k, int32_t width) {
+  return B <= 2 && (width == 1 || width == 2) && D % 8 == 0 && (D * width) % 16 == 0 &&
+         D <= 1024 && k <= 128;
+}
+
+bool tensor_ok(int64_t B, int64_t N, int32_t D, int32_t k, int32_t width, int32_t code_bound) {
+  (void)N;
+  const bool codes_exact = width == 1 || (width == 2 && code_bound > 0 && code_bound <= 2048);
+  return codes_exact && D % 16 == 0 && tensor_fits(width, k) && B <= (1LL << 23);
+}
+
+// Chooses the path (or honours LAM_SCORE_PATH) and lays out the workspace:
+// [status 256 B][partial lists n_lists x B x k keys][tensor: query prep].
+bool make_plan(int64_t B, int64_t N, int32_t D, int32_t k, int32_t width, int32_t code_bound,
+               int sms, Plan *p) {
+  if (!shape_ok(B, N, D, k, width, code_bound) || sms <= 0) return false;
+  const bool bw = bandwidth_ok(B, D, k, width);
+  const bool tc = tensor_ok(B, N, D, k, width, code_bound);
+  const int f = forced_path();
+  if (f == -2) return false;
+  int path;
+  if (f >= 0) {
+    if ((f == kPathBandwidth && !bw) || (f == kPathTensor && !tc)) {
+      p->path = -2;
+      return false;
+    }
+    path = f;
+  } else if (bw) {
+    path = kPathBandwidth;
+  } else if (tc) {
+    path = kPathTensor;
+  } else {
+    path = kPathGeneric;
+  }
+  p->path = path;
+  if (path == kPathBandwidth) p->n_lists = bandwidth_ctas(N, D, width, sms);
+  else if (path == kPathTensor) p->n_lists = tensor_splits(B, N, sms);
+  else p->n_lists = generic_ctas(B, N, sms);
+  p->Bpad = (B + 127) / 128 * 128;
+  p->partial_off = kHeaderBytes;
+  const size_t partial = (size_t)p->n_lists * (size_t)B * (size_t)k * 8;
+  p->qprep_off = align_up(p->partial_off + partial, 256);
+  p->total = p->qprep_off;
+  if (path == kPathTensor) p->total += align_up(tensor_qprep_bytes(p->Bpad, D), 256);
+  return true;
+}
+
+}  // namespace
+
+extern "C" {
+
+int32_t lam_version(void) { return 100; }
+
+const char *lam_status_string(int32_t status) {
+  switch (status) {
+    case LAM_OK: return "ok";
+    case LAM_ERR_INVALID: return "invalid argument";
+    case LAM_ERR_RANGE: return "codes out of range for the width";
+    case LAM_ERR_NONFINITE: return "non-finite input";
+    case LAM_ERR_WORKSPACE: return "buffer or workspace too small";
+    case LAM_ERR_CUDA: return "CUDA error";
+    case LAM_ERR_TIMEOUT: return "device wait timed out";
+    case LAM_ERR_UNSUPPORTED: return "forced kernel path cannot take this shape";
+    default: return "unknown status";
+  }
+}
+
+size_t lam_quantize_workspace_size(void) { return sizeof(QuantStatus); }
+
+lam_status lam_quantize(const float *x, int64_t n, float eps, int32_t width_req, void *codes,
+                        size_t codes_bytes, void *workspace, size_t workspace_bytes,
+                        int32_t *width_out, float *scale_out, int32_t *code_min_out,
+                        int32_t *code_max_out, lam_stream_t stream) {
+  if (n < 0 || n >= (1LL << 62) || !valid_eps(eps)) return LAM_ERR_INVALID;
+  if (width_req != LAM_WIDTH_AUTO && !valid_width(width_req)) return LAM_ERR_INVALID;
+  if (n > 0 && x == nullptr) return LAM_ERR_INVALID;
+  // natural alignment: fp32 input; codes aligned to their width (AUTO: 4 bytes)
+  if ((reinterpret_cast<uintptr_t>(x) & 3u) != 0) return LAM_ERR_INVALID;
+  const uintptr_t calign = width_req == LAM_WIDTH_AUTO ? 4u : (uintptr_t)width_req;
+  if (codes != nullptr && (reinterpret_cast<uintptr_t>(codes) & (calign - 1)) != 0)
+    return LAM_ERR_INVALID;
+  const float s = 2.0f * eps;
+  if (n == 0) {
+    if (width_out) *width_out = width_req == LAM_WIDTH_AUTO ? 1 : width_req;
+    if (scale_out) *scale_out = s;
+    if (code_min_out) *code_min_out = 0;
+    if (code_max_out) *code_max_out = 0;
+    return LAM_OK;
+  }
+  if (workspace == nullptr || (reinterpret_cast<uintptr_t>(workspace) & 15u) != 0)
+    return LAM_ERR_INVALID;
+  if (workspace_bytes < sizeof(QuantStatus)) return LAM_ERR_WORKSPACE;
+  if (codes != nullptr && width_req != LAM_WIDTH_AUTO &&
+      (unsigned long long)n * (unsigned long long)width_req > codes_bytes)
+    return LAM_ERR_WORKSPACE;
+  const int sms = device_sms();
+  if (sms <= 0) return LAM_ERR_CUDA;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  QuantStatus *dst = static_cast<QuantStatus *>(workspace);
+  if (cudaMemsetAsync(dst, 0, sizeof(QuantStatus), st) != cudaSuccess) return LAM_ERR_CUDA;
+  cudaError_t e = cudaSuccess;
+  if (width_req == LAM_WIDTH_AUTO) {
+    e = launch_quant_range(x, n, dst, sms, st);
+    if (e == cudaSuccess) e = launch_quantize(x, n, s, LAM_WIDTH_AUTO, codes, codes_bytes, dst, sms, st);
+  } else if (codes != nullptr) {
+    e = launch_quantize(x, n, s, width_req, codes, codes_bytes, dst, sms, st);
+  } else {
+    e = launch_quant_range(x, n, dst, sms, st);
+  }
+  if (e != cudaSuccess) return LAM_ERR_CUDA;
+  QuantStatus h;
+  if (cudaMemcpyAsync(&h, dst, sizeof(h), cudaMemcpyDeviceToHost, st) != cudaSuccess)
+    return LAM_ERR_CUDA;
+  if (cudaStreamSynchronize(st) != cudaSuccess) return LAM_ERR_CUDA;
+  if (h.flags & kFlagNonfinite) return LAM_ERR_NONFINITE;
+  float rmin = 0.0f, rmax = 0.0f;
+  if (h.neg_min != 0) {
+    rmin = host_qround(unord_host(~h.neg_min), s);
+    rmax = host_qround(unord_host(h.max), s);
+  }
+  const int need = width_of(rmin, rmax);
+  const int w = width_req == LAM_WIDTH_AUTO ? need : width_req;
+  if (scale_out) *scale_out = s;
+  if (width_out) *width_out = w;
+  if (need != 0) {
+    if (code_min_out) *code_min_out = (int32_t)rmin;
+    if (code_max_out) *code_max_out = (int32_t)rmax;
+  } else {
+    if (code_min_out) *code_min_out = rmin < -2147483648.0f ? INT32_MIN : (int32_t)rmin;
+    if (code_max_out) *code_max_out = rmax >= 2147483648.0f ? INT32_MAX : (int32_t)rmax;
+  }
+  if (need == 0 || (h.flags & kFlagRange)) return LAM_ERR_RANGE;
+  if (width_req != LAM_WIDTH_AUTO && need > width_req) return LAM_ERR_RANGE;
+  if (width_req == LAM_WIDTH_AUTO && (int)h.width != need) return LAM_ERR_CUDA;  // must agree
+  if (h.flags & kFlagWorkspace) return LAM_ERR_WORKSPACE;
+  return LAM_OK;
+}
+
+lam_status lam_dequantize(const void *codes, int32_t width, int64_t n, float scale, float *out,
+                          lam_stream_t stream) {
+  if (n < 0 || !valid_width(width) || !isfinite(scale)) return LAM_ERR_INVALID;
+  if (n == 0) return LAM_OK;
+  if (codes == nullptr || out == nullptr) return LAM_ERR_INVALID;
+  if ((reinterpret_cast<uintptr_t>(codes) & (uintptr_t)(width - 1)) != 0 ||
+      (reinterpret_cast<uintptr_t>(out) & 3u) != 0)
+    return LAM_ERR_INVALID;
+  const int sms = device_sms();
+  if (sms <= 0) return LAM_ERR_CUDA;
+  if (launch_dequantize(codes, width, n, scale, out, sms, reinterpret_cast<cudaStream_t>(stream)) !=
+      cudaSuccess)
+    return LAM_ERR_CUDA;
+  return LAM_OK;
+}
+
+size_t lam_score_topk_workspace_size(int64_t B, int64_t N, int32_t D, int32_t k, int32_t width,
+                                     int32_t code_bound) {
+  Plan p;
+  const int sms = device_sms();
+  if (!make_plan(B, N, D, k, width, code_bound, sms, &p)) return 0;
+  // misaligned codes fall back to the generic path at call time
+  const size_t generic = align_up(kHeaderBytes + (size_t)generic_ctas(B, N, sms) * B * k * 8, 256);
+  return p.total > generic ? p.total : generic;
+}
+
+int32_t lam_score_topk_path(int64_t B, int64_t N, int32_t D, int32_t k, int32_t width,
+                            int32_t code_bound) {
+  Plan p;
+  if (!make_plan(B, N, D, k, width, code_bound, device_sms(), &p)) return -1;
+  return p.path;
+}
+
+lam_status lam_score_topk(const float *queries, int64_t B, const void *codes, int32_t width,
+                          int64_t N, int32_t D, float eps, int32_t code_bound, int32_t k,
+                          int32_t metric, float *scores, int64_t *ids, void *workspace,
+                          size_t workspace_bytes, lam_stream_t stream) {
+  if (queries == nullptr || codes == nullptr || scores == nullptr || ids == nullptr ||
+      workspace == nullptr)
+    return LAM_ERR_INVALID;
+  if (metric != LAM_METRIC_IP && metric != LAM_METRIC_COSINE && metric != LAM_METRIC_L2)
+    return LAM_ERR_INVALID;
+  if (!valid_eps(eps)) return LAM_ERR_INVALID;
+  if (!shape_ok(B, N, D, k, width, code_bound)) return LAM_ERR_INVALID;
+  if ((reinterpret_cast<uintptr_t>(workspace) & 255u) != 0) return LAM_ERR_INVALID;
+  if ((reinterpret_cast<uintptr_t>(codes) & (uintptr_t)(width - 1)) != 0 ||
+      (reinterpret_cast<uintptr_t>(queries) & 3u) != 0 ||
+      (reinterpret_cast<uintptr_t>(scores) & 3u) != 0 || (reinterpret_cast<uintptr_t>(ids) & 7u) != 0)
+    return LAM_ERR_INVALID;
+  const int sms = device_sms();
+  if (sms <= 0) return LAM_ERR_CUDA;
+  Plan p;
+  if (!make_plan(B, N, D, k, width, code_bound, sms, &p))
+    return p.path == -2 ? LAM_ERR_UNSUPPORTED : LAM_ERR_INVALID;
+  // TMA and bulk copies need a 16-byte aligned code base
+  const bool aligned = (reinterpret_cast<uintptr_t>(codes) & 15u) == 0;
+  if (!aligned && p.path != kPathGeneric) {
+    if (forced_path() >= 0) return LAM_ERR_UNSUPPORTED;
+    p.path = kPathGeneric;
+    p.n_lists = generic_ctas(B, N, sms);
+    p.qprep_off = align_up(p.partial_off + (size_t)p.n_lists * B * k * 8, 256);
+    p.total = p.qprep_off;
+  }
+  if (workspace_bytes < p.total) return LAM_ERR_WORKSPACE;
+
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  uint8_t *ws = static_cast<uint8_t *>(workspace);
+  if (cudaMemsetAsync(ws, 0, kHeaderBytes, st) != cudaSuccess) return LAM_ERR_CUDA;
+  ScoreArgs a;
+  a.queries = queries;
+  a.B = B;
+  a.codes = codes;
+  a.width = width;
+  a.N = N;
+  a.D = D;
+  a.s = 2.0f * eps;
+  a.code_bound = code_bound;
+  a.k = k;
+  a.metric = metric;
+  a.scores = scores;
+  a.ids = ids;
+  a.gflags = reinterpret_cast<uint32_t *>(ws);
+  a.partial = reinterpret_cast<uint64_t *>(ws + p.partial_off);
+  a.n_lists = p.n_lists;
+  a.qprep = ws + p.qprep_off;
+  a.Bpad = p.Bpad;
+  a.sms = sms;
+  cudaError_t e;
+  if (p.path == kPathBandwidth) e = launch_score_bandwidth(a, st);
+  else if (p.path == kPathTensor) e = launch_score_tensor(a, st);
+  else e = launch_score_generic(a, st);
+  if (e != cudaSuccess) return LAM_ERR_CUDA;
+  if (launch_topk_merge(a, st) != cudaSuccess) return LAM_ERR_CUDA;
+  return LAM_OK;
+}
+
+lam_status lam_score_topk_status(const void *workspace, lam_stream_t stream, int32_t *status_out) {
+  if (workspace == nullptr || status_out == nullptr) return LAM_ERR_INVALID;
+  uint32_t flags = 0;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  if (cudaMemcpyAsync(&flags, workspace, 4, cudaMemcpyDeviceToHost, st) != cudaSuccess)
+    return LAM_ERR_CUDA;
+  if (cudaStreamSynchronize(st) != cudaSuccess) return LAM_ERR_CUDA;
+  if (flags & kFlagTimeout) *status_out = LAM_ERR_TIMEOUT;
+  else if (flags & kFlagRange) *status_out = LAM_ERR_RANGE;
+  else *status_out = LAM_OK;
+  return LAM_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,172 @@
+// lam_internal.cuh -- shared device helpers and launcher declarations of the
+// sm_103a library.  Nothing here is visible through the C ABI.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/lam.h"
+
+namespace lam {
+
+// ---------------------------------------------------------------- constants --
+constexpr uint32_t kFlagNonfinite = 1u;   // quantize: NaN/Inf seen
+constexpr uint32_t kFlagRange = 2u;       // codes beyond a width / code bound
+constexpr uint32_t kFlagWorkspace = 4u;   // codes buffer too small (AUTO)
+constexpr uint32_t kFlagTimeout = 8u;     // a bounded wait gave up
+
+constexpr int kMaxK = 1024;
+constexpr int kHeaderBytes = 256;         // status block at the head of a workspace
+
+// Wait budget of every device-side spin: ~1 s of SM clock.
+constexpr long long kWaitCycles = 2000000000LL;
+
+// Status block of lam_quantize (16 bytes, zeroed before each call).
+struct QuantStatus {
+  uint32_t neg_min;   // max over inputs of ~ord(x)   (0: no finite input seen)
+  uint32_t max;       // max over inputs of ord(x)
+  uint32_t flags;
+  uint32_t width;     // width the AUTO kernel resolved
+};
+
+// ----------------------------------------------------- ordered float keys --
+// ord() maps fp32 to uint32 so that unsigned order equals numeric order
+// (-0 is first folded into +0).
+__device__ __forceinline__ uint32_t ord_f32(float f) {
+  f = f + 0.0f;
+  uint32_t b = __float_as_uint(f);
+  return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+}
+__device__ __forceinline__ float unord_f32(uint32_t o) {
+  uint32_t b = (o & 0x80000000u) ? (o & 0x7FFFFFFFu) : ~o;
+  return __uint_as_float(b);
+}
+// 64-bit selection key: smaller is better.  High word: the score in rank
+// order (complemented for descending metrics); low word: the row id, so
+// equal scores rank the lower id first.
+__device__ __forceinline__ uint64_t make_key(float score, uint32_t row, bool desc) {
+  uint32_t o = ord_f32(score);
+  if (desc) o = ~o;
+  return ((uint64_t)o << 32) | (uint64_t)row;
+}
+constexpr uint64_t kSentinel = ~0ull;
+
+// ------------------------------------------------------------ PTX helpers --
+__device__ __forceinline__ uint32_t smem_u32(const void *p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t *bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count)
+               : "memory");
+}
+__device__ __forceinline__ void fence_barrier_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t *bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t *bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
+               "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Bounded wait for phase `parity` of `bar`.  Gives up after kWaitCycles or as
+// soon as *abort is set; on giving up sets *abort and the timeout flag.
+__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity,
+                                          volatile int *abort, uint32_t *gflags) {
+  if (mbar_try_wait(bar, parity)) return true;
+  long long t0 = clock64();
+  while (true) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (*abort) return false;
+    if (clock64() - t0 > kWaitCycles) {
+      *abort = 1;
+      if (gflags) atomicOr(gflags, kFlagTimeout);
+      return false;
+    }
+  }
+}
+
+// 1-D bulk copy global -> shared, completing on an mbarrier (16-byte
+// aligned addresses, size a multiple of 16).
+__device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t bytes,
+                                         uint64_t *bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::
+          "r"(smem_u32(dst)),
+      "l"(src), "r"(bytes), "r"(smem_u32(bar))
+      : "memory");
+}
+
+// 2-D tiled TMA load (coordinates: x = innermost element index, y = row).
+__device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, int32_t x,
+                                            int32_t y, uint64_t *bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3}], [%4];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar))
+      : "memory");
+}
+
+// ------------------------------------------------------------- launchers --
+// (defined in quantize.cu / score_bw.cu / score_tc.cu; all launch on `st`)
+cudaError_t launch_quant_range(const float *x, int64_t n, QuantStatus *status, int sms,
+                               cudaStream_t st);
+cudaError_t launch_quantize(const float *x, int64_t n, float s, int width_req, void *codes,
+                            size_t codes_bytes, QuantStatus *status, int sms,
+                            cudaStream_t st);
+cudaError_t launch_dequantize(const void *codes, int width, int64_t n, float s, float *out,
+                              int sms, cudaStream_t st);
+
+struct ScoreArgs {
+  const float *queries;
+  int64_t B;
+  const void *codes;
+  int width;
+  int64_t N;
+  int D;
+  float s;         // 2 eps
+  int code_bound;  // tensor path limit check
+  int k;
+  int metric;
+  float *scores;
+  int64_t *ids;
+  uint32_t *gflags;     // workspace status flags
+  uint64_t *partial;    // [n_lists][B][k] keys
+  int n_lists;
+  void *qprep;          // tensor path: fp16 [2*Bpad][D] then float4 [Bpad]
+  int64_t Bpad;
+  int sms;
+};
+
+cudaError_t launch_score_bandwidth(const ScoreArgs &a, cudaStream_t st);
+cudaError_t launch_score_generic(const ScoreArgs &a, cudaStream_t st);
+cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st);
+cudaError_t launch_topk_merge(const ScoreArgs &a, cudaStream_t st);
+
+// Planning shared by the workspace-size query and the launch.
+enum Path { kPathBandwidth = 0, kPathTensor = 1, kPathGeneric = 2 };
+int bandwidth_ctas(int64_t N, int D, int width, int sms);
+int tensor_splits(int64_t B, int64_t N, int sms);
+bool tensor_fits(int width, int k);  // shared memory holds >= 2 stages
+size_t tensor_qprep_bytes(int64_t Bpad, int D);
+int generic_ctas(int64_t B, int64_t N, int sms);
+
+}  // namespace lam

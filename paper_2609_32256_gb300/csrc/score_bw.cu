@@ -1,0 +1,444 @@
+// score_bw.cu -- exact search on the codes for small query batches (the
+// matrix-vector regime of Sec. "Brute-force scan crossover"), the generic
+// fallback for any shape, and the final top-k merge.
+//
+// Bandwidth kernel: one persistent CTA per SM streams a contiguous range of
+// code rows through a ring of shared-memory stages filled by 1-D bulk copies
+// (cp.async.bulk, completion on mbarriers).  Eight consumer warps each score
+// whole rows: a lane owns eight consecutive coordinates per 256-coordinate
+// chunk, converts the codes to fp32 exactly (byte-permute into the mantissa of
+// 2^23, then one subtraction), multiplies by the query held in registers, and
+// the warp sums with shuffles.  Each warp keeps its top-k in registers (one
+// key per lane per 32 entries); the CTA merges its eight lists by rank and
+// writes one partial list per query.  Work per element: a few integer/FP
+// instructions, so the kernel is bound by HBM at width bytes per element.
+#include "score_common.cuh"
+
+namespace lam {
+
+namespace {
+
+constexpr int kBwWarps = 8;
+constexpr int kBwThreads = (kBwWarps + 1) * 32;
+constexpr int kNchMax = 4;  // 8-coordinate vectors per lane per row: D <= 1024
+constexpr int kBwStageTarget = 32 * 1024;
+constexpr int kBwSmemBudget = 200 * 1024;
+
+// 8 codes -> 8 exact fp32 values.
+template <int W>
+__device__ __forceinline__ void decode8(const uint8_t *p, float *f) {
+  if (W == 1) {
+    const uint2 v = *reinterpret_cast<const uint2 *>(p);
+    const uint32_t a = v.x ^ 0x80808080u, b = v.y ^ 0x80808080u;
+    // bits 0x4B0000uu = 2^23 + u with u = code + 128
+    f[0] = __int_as_float(__byte_perm(a, 0x4B000000u, 0x7540)) - 8388736.0f;
+    f[1] = __int_as_float(__byte_perm(a, 0x4B000000u, 0x7541)) - 8388736.0f;
+    f[2] = __int_as_float(__byte_perm(a, 0x4B000000u, 0x7542)) - 8388736.0f;
+    f[3] = __int_as_float(__byte_perm(a, 0x4B000000u, 0x7543)) - 8388736.0f;
+    f[4] = __int_as_float(__byte_perm(b, 0x4B000000u, 0x7540)) - 8388736.0f;
+    f[5] = __int_as_float(__byte_perm(b, 0x4B000000u, 0x7541)) - 8388736.0f;
+    f[6] = __int_as_float(__byte_perm(b, 0x4B000000u, 0x7542)) - 8388736.0f;
+    f[7] = __int_as_float(__byte_perm(b, 0x4B000000u, 0x7543)) - 8388736.0f;
+  } else {
+    const uint4 v = *reinterpret_cast<const uint4 *>(p);
+    const uint32_t w[4] = {v.x ^ 0x80008000u, v.y ^ 0x80008000u, v.z ^ 0x80008000u,
+                           v.w ^ 0x80008000u};
+    // bits 0x4B00uuuu = 2^23 + u with u = code + 32768
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      f[2 * j] = __int_as_float(__byte_perm(w[j], 0x4B000000u, 0x7410)) - 8421376.0f;
+      f[2 * j + 1] = __int_as_float(__byte_perm(w[j], 0x4B000000u, 0x7432)) - 8421376.0f;
+    }
+  }
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+  return v;
+}
+
+// Waits (bounded, ignoring the abort flag) until a phase that is known to be
+// in flight completes; used only to drain copies before the CTA exits.
+__device__ __forceinline__ void drain_wait(uint64_t *bar, uint32_t parity) {
+  long long t0 = clock64();
+  while (!mbar_try_wait(bar, parity))
+    if (clock64() - t0 > kWaitCycles) break;
+}
+
+struct BwShape {
+  int tr;           // rows per stage (multiple of the consumer warp count)
+  int ns;           // stages
+  int stage_bytes;  // tr * D * width, a multiple of 16
+};
+
+inline BwShape bw_shape(int D, int width) {
+  const int row = D * width;
+  int tr = (kBwStageTarget / (row * kBwWarps)) * kBwWarps;
+  if (tr < kBwWarps) tr = kBwWarps;
+  BwShape sh;
+  sh.tr = tr;
+  sh.stage_bytes = tr * row;
+  sh.ns = kBwSmemBudget / sh.stage_bytes;
+  if (sh.ns > 8) sh.ns = 8;
+  if (sh.ns < 2) sh.ns = 2;
+  return sh;
+}
+
+template <int W, int QB, int KPL>
+__global__ void __launch_bounds__(kBwThreads, 1)
+    score_bw_kernel(ScoreArgs a, int tr, int ns, int stage_bytes) {
+  extern __shared__ __align__(1024) uint8_t smem[];
+  uint64_t *full = reinterpret_cast<uint64_t *>(smem + (size_t)ns * stage_bytes);
+  uint64_t *empty = full + ns;
+  volatile int *abort_flag = reinterpret_cast<volatile int *>(empty + ns);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t N = a.N;
+  const int D = a.D;
+  const int64_t r0 = (int64_t)blockIdx.x * N / gridDim.x;
+  const int64_t r1 = (int64_t)(blockIdx.x + 1) * N / gridDim.x;
+  const int64_t nrows = r1 - r0;
+  const int ntiles = (int)((nrows + tr - 1) / tr);
+  const size_t row_bytes = (size_t)D * W;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < ns; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], kBwWarps);
+    }
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  __syncthreads();
+
+  WarpList<KPL> lists[QB];
+#pragma unroll
+  for (int q = 0; q < QB; ++q) lists[q].init();
+
+  if (warp == kBwWarps) {
+    // ---------------- producer: one lane issues the bulk copies ----------
+    if (lane == 0) {
+      int issued = 0;
+      for (int t = 0; t < ntiles; ++t) {
+        const int s = t % ns, r = t / ns;
+        if (r > 0 && !mbar_wait(&empty[s], (r - 1) & 1, abort_flag, a.gflags)) break;
+        const int64_t nr = min((int64_t)tr, nrows - (int64_t)t * tr);
+        const uint32_t bytes = (uint32_t)(nr * row_bytes);
+        mbar_arrive_expect_tx(&full[s], bytes);
+        bulk_g2s(smem + (size_t)s * stage_bytes,
+                 static_cast<const uint8_t *>(a.codes) + (r0 + (int64_t)t * tr) * row_bytes,
+                 bytes, &full[s]);
+        issued = t + 1;
+      }
+      for (int t = max(0, issued - ns); t < issued; ++t) drain_wait(&full[t % ns], (t / ns) & 1);
+    }
+  } else {
+    // ---------------- consumers -----------------------------------------
+    const int nch = (D + 255) / 256;
+    float qreg[QB][kNchMax][8];
+    float qq[QB], qn[QB];
+#pragma unroll
+    for (int q = 0; q < QB; ++q) {
+      const bool qv = q < a.B;
+      float part = 0.0f;
+#pragma unroll
+      for (int j = 0; j < kNchMax; ++j) {
+        const int e0 = (j * 32 + lane) * 8;
+#pragma unroll
+        for (int t = 0; t < 8; ++t) {
+          const float v = (qv && j < nch && e0 + t < D) ? a.queries[(int64_t)q * D + e0 + t] : 0.0f;
+          qreg[q][j][t] = v;
+          part = fmaf(v, v, part);
+        }
+      }
+      qq[q] = warp_sum(part);
+      qn[q] = sqrtf(qq[q]);
+    }
+    const bool need_cc = a.metric != LAM_METRIC_IP;
+    const bool desc = a.metric != LAM_METRIC_L2;
+    const float s = a.s, s2 = a.s * a.s;
+
+    uint64_t thr[QB];
+#pragma unroll
+    for (int q = 0; q < QB; ++q) thr[q] = kSentinel;
+
+    for (int t = 0; t < ntiles; ++t) {
+      const int st = t % ns, r = t / ns;
+      if (!mbar_wait(&full[st], r & 1, abort_flag, a.gflags)) break;
+      const int nr = (int)min((int64_t)tr, nrows - (int64_t)t * tr);
+      const uint8_t *stage = smem + (size_t)st * stage_bytes;
+      for (int rr = warp; rr < nr; rr += kBwWarps) {
+        const uint8_t *rowp = stage + (size_t)rr * row_bytes;
+        float acc[QB];
+#pragma unroll
+        for (int q = 0; q < QB; ++q) acc[q] = 0.0f;
+        float cc = 0.0f;
+#pragma unroll
+        for (int j = 0; j < kNchMax; ++j) {
+          const int e0 = (j * 32 + lane) * 8;
+          if (j < nch && e0 < D) {
+            float f[8];
+            decode8<W>(rowp + (size_t)e0 * W, f);
+#pragma unroll
+            for (int q = 0; q < QB; ++q)
+#pragma unroll
+              for (int u = 0; u < 8; ++u) acc[q] = fmaf(qreg[q][j][u], f[u], acc[q]);
+            if (need_cc)
+#pragma unroll
+              for (int u = 0; u < 8; ++u) cc = fmaf(f[u], f[u], cc);
+          }
+        }
+#pragma unroll
+        for (int q = 0; q < QB; ++q) acc[q] = warp_sum(acc[q]);
+        if (need_cc) cc = warp_sum(cc);
+        const uint32_t row = (uint32_t)(r0 + (int64_t)t * tr + rr);
+#pragma unroll
+        for (int q = 0; q < QB; ++q) {
+          if (q >= a.B) continue;
+          const float sc = finish_score(a.metric, acc[q], cc, s, s2, qq[q], qn[q]);
+          const uint64_t key = make_key(sc, row, desc);
+          if (key < thr[q]) {
+            lists[q].insert(key, lane);
+            thr[q] = lists[q].kth(a.k);
+          }
+        }
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&empty[st]);
+    }
+  }
+  __syncthreads();  // every stage consumed and every copy drained: reuse them
+  uint64_t *cand = reinterpret_cast<uint64_t *>(smem);
+  if (warp < kBwWarps) {
+#pragma unroll
+    for (int q = 0; q < QB; ++q)
+      lists[q].store(cand + ((size_t)q * kBwWarps + warp) * a.k, a.k, lane);
+  }
+  __syncthreads();
+  // ---------------- CTA merge of the eight warp lists, per query ----------
+  for (int q = 0; q < QB && q < a.B; ++q)
+    rank_merge(cand + (size_t)q * kBwWarps * a.k, kBwWarps, a.k,
+               a.partial + ((size_t)blockIdx.x * a.B + q) * a.k, threadIdx.x, kBwThreads);
+}
+
+// ---------------------------------------------------------------------------
+// Generic path: any D, width 1/2/4, k <= 1024, any batch.  Grid (ctas, B):
+// a CTA scores one query against a range of rows, warp per row with plain
+// global loads, per-warp top-k lists in shared memory, then a rank merge.
+constexpr int kGenWarps = 8;
+
+__device__ __forceinline__ int32_t load_code(const void *codes, int width, int64_t i) {
+  if (width == 1) return reinterpret_cast<const int8_t *>(codes)[i];
+  if (width == 2) return reinterpret_cast<const int16_t *>(codes)[i];
+  return reinterpret_cast<const int32_t *>(codes)[i];
+}
+
+__global__ void __launch_bounds__(kGenWarps * 32) score_generic_kernel(ScoreArgs a) {
+  extern __shared__ __align__(16) uint8_t gsmem[];
+  uint64_t *lists = reinterpret_cast<uint64_t *>(gsmem);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int D = a.D, k = a.k;
+  uint64_t *L = lists + (size_t)warp * k;
+  for (int64_t b = blockIdx.y; b < a.B; b += gridDim.y) {
+  const float *q = a.queries + b * D;
+  for (int i = lane; i < k; i += 32) L[i] = kSentinel;
+  __syncwarp();
+  uint64_t thr = kSentinel;
+
+  float part = 0.0f;
+  for (int d = lane; d < D; d += 32) part = fmaf(q[d], q[d], part);
+  const float qq = warp_sum(part), qn = sqrtf(qq);
+  const bool desc = a.metric != LAM_METRIC_L2;
+  const float s = a.s, s2 = a.s * a.s;
+
+  const int64_t r0 = (int64_t)blockIdx.x * a.N / gridDim.x;
+  const int64_t r1 = (int64_t)(blockIdx.x + 1) * a.N / gridDim.x;
+  for (int64_t row = r0 + warp; row < r1; row += kGenWarps) {
+    float acc = 0.0f, cc = 0.0f;
+    const int64_t base = row * D;
+    for (int d = lane; d < D; d += 32) {
+      const float c = (float)load_code(a.codes, a.width, base + d);
+      acc = fmaf(q[d], c, acc);
+      cc = fmaf(c, c, cc);
+    }
+    acc = warp_sum(acc);
+    cc = warp_sum(cc);
+    const float sc = finish_score(a.metric, acc, cc, s, s2, qq, qn);
+    const uint64_t key = make_key(sc, (uint32_t)row, desc);
+    if (key < thr) smem_list_insert(L, k, key, lane, thr);
+  }
+  __syncthreads();
+  rank_merge(lists, kGenWarps, k, a.partial + ((size_t)blockIdx.x * a.B + b) * k, threadIdx.x,
+             kGenWarps * 32);
+  __syncthreads();
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Final merge: per query, n_lists partial lists of k keys -> the k best,
+// decoded to (score, id).  Bitonic sort in shared memory; when the candidates
+// exceed one buffer, chunks are sorted together with the running top-k.
+constexpr int kMergeThreads = 1024;
+constexpr int kMergeCap = 16384;
+
+__device__ __forceinline__ int next_pow2_dev(int x) {
+  int p = 1;
+  while (p < x) p <<= 1;
+  return p;
+}
+
+__device__ void bitonic_sort(uint64_t *buf, int P) {
+  for (int size = 2; size <= P; size <<= 1) {
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      for (int i = threadIdx.x; i < P / 2; i += blockDim.x) {
+        const int lo = 2 * i - (i & (stride - 1));
+        const int hi = lo + stride;
+        const bool up = (lo & size) == 0;
+        const uint64_t x = buf[lo], y = buf[hi];
+        if ((x > y) == up) {
+          buf[lo] = y;
+          buf[hi] = x;
+        }
+      }
+      __syncthreads();
+    }
+  }
+}
+
+__global__ void __launch_bounds__(kMergeThreads) topk_merge_kernel(ScoreArgs a, int P) {
+  extern __shared__ __align__(16) uint8_t msmem[];
+  uint64_t *buf = reinterpret_cast<uint64_t *>(msmem);
+  const int64_t b = blockIdx.x;
+  const int k = a.k;
+  const int64_t total = (int64_t)a.n_lists * k;
+  // candidate e of query b lives at partial[(l * B + b) * k + i], e = l*k + i
+  auto cand = [&](int64_t e) -> uint64_t {
+    const int64_t l = e / k, i = e - l * k;
+    return a.partial[((size_t)l * a.B + b) * k + i];
+  };
+  if (total <= P) {
+    for (int i = threadIdx.x; i < P; i += blockDim.x) buf[i] = i < total ? cand(i) : kSentinel;
+    __syncthreads();
+    bitonic_sort(buf, P);
+  } else {
+    for (int i = threadIdx.x; i < k; i += blockDim.x) buf[i] = kSentinel;
+    const int chunk = P - k;
+    for (int64_t c0 = 0; c0 < total; c0 += chunk) {
+      for (int i = threadIdx.x; i < chunk; i += blockDim.x)
+        buf[k + i] = (c0 + i < total) ? cand(c0 + i) : kSentinel;
+      __syncthreads();
+      bitonic_sort(buf, P);
+    }
+  }
+  const bool desc = a.metric != LAM_METRIC_L2;
+  if (!desc) {
+    // Squared L2 was ranked through ||q||^2 + s^2||c||^2 - 2 s q.c, which
+    // cancels for near neighbours; the k survivors are rescored in the direct
+    // form sum_d (q_d - s c_d)^2 and re-sorted.
+    uint64_t *rescored = buf + P;
+    __syncthreads();
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
+    const float *q = a.queries + b * a.D;
+    for (int i = warp; i < k; i += nw) {
+      const uint64_t key = buf[i];
+      const uint32_t row = (uint32_t)(key & 0xffffffffu);
+      float acc = 0.0f;
+      if (row < a.N) {
+        for (int d = lane; d < a.D; d += 32) {
+          const float xh = __fmul_rn(a.s, (float)load_code(a.codes, a.width, (int64_t)row * a.D + d));
+          const float df = __fsub_rn(q[d], xh);
+          acc = fmaf(df, df, acc);
+        }
+      }
+      acc = warp_sum(acc);
+      if (lane == 0) rescored[i] = row < a.N ? make_key(acc, row, false) : kSentinel;
+    }
+    __syncthreads();
+    const int P2 = next_pow2_dev(k);
+    for (int i = threadIdx.x; i < P2; i += blockDim.x) buf[i] = i < k ? rescored[i] : kSentinel;
+    __syncthreads();
+    bitonic_sort(buf, P2);
+  }
+  for (int i = threadIdx.x; i < k; i += blockDim.x) {
+    const uint64_t key = buf[i];
+    uint32_t o = (uint32_t)(key >> 32);
+    if (desc) o = ~o;
+    a.scores[b * k + i] = unord_f32(o);
+    a.ids[b * k + i] = (int64_t)(uint32_t)(key & 0xffffffffu);
+  }
+}
+
+inline int next_pow2(int64_t x) {
+  int p = 1;
+  while (p < x) p <<= 1;
+  return p;
+}
+
+}  // namespace
+
+int bandwidth_ctas(int64_t N, int D, int width, int sms) {
+  const BwShape sh = bw_shape(D, width);
+  int64_t c = (N + sh.tr - 1) / sh.tr;
+  if (c > sms) c = sms;
+  if (c < 1) c = 1;
+  return (int)c;
+}
+
+int generic_ctas(int64_t B, int64_t N, int sms) {
+  int64_t per_q = (2LL * sms + B - 1) / B;
+  int64_t by_rows = (N + 63) / 64;
+  int64_t c = per_q < by_rows ? per_q : by_rows;
+  if (c > 2LL * sms) c = 2LL * sms;
+  if (c < 1) c = 1;
+  return (int)c;
+}
+
+template <int W, int QB, int KPL>
+static cudaError_t launch_bw_t(const ScoreArgs &a, const BwShape &sh, cudaStream_t st) {
+  const size_t smem = (size_t)sh.ns * sh.stage_bytes + 2 * sh.ns * sizeof(uint64_t) + 16;
+  auto kern = score_bw_kernel<W, QB, KPL>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  kern<<<a.n_lists, kBwThreads, smem, st>>>(a, sh.tr, sh.ns, sh.stage_bytes);
+  return cudaGetLastError();
+}
+
+template <int W, int QB>
+static cudaError_t launch_bw_k(const ScoreArgs &a, const BwShape &sh, cudaStream_t st) {
+  if (a.k <= 32) return launch_bw_t<W, QB, 1>(a, sh, st);
+  if (a.k <= 64) return launch_bw_t<W, QB, 2>(a, sh, st);
+  return launch_bw_t<W, QB, 4>(a, sh, st);
+}
+
+cudaError_t launch_score_bandwidth(const ScoreArgs &a, cudaStream_t st) {
+  const BwShape sh = bw_shape(a.D, a.width);
+  // merge scratch (QB * 8 warps * k keys) must fit in the stage buffers
+  if ((size_t)2 * kBwWarps * a.k * 8 > (size_t)sh.ns * sh.stage_bytes) return cudaErrorInvalidValue;
+  if (a.width == 1) return a.B == 1 ? launch_bw_k<1, 1>(a, sh, st) : launch_bw_k<1, 2>(a, sh, st);
+  return a.B == 1 ? launch_bw_k<2, 1>(a, sh, st) : launch_bw_k<2, 2>(a, sh, st);
+}
+
+cudaError_t launch_score_generic(const ScoreArgs &a, cudaStream_t st) {
+  const size_t smem = (size_t)kGenWarps * a.k * sizeof(uint64_t);
+  cudaError_t e = cudaFuncSetAttribute(score_generic_kernel,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  dim3 grid(a.n_lists, (unsigned)(a.B < 65535 ? a.B : 65535));
+  score_generic_kernel<<<grid, kGenWarps * 32, smem, st>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_topk_merge(const ScoreArgs &a, cudaStream_t st) {
+  const int64_t total = (int64_t)a.n_lists * a.k;
+  int P = total <= kMergeCap ? next_pow2(total) : kMergeCap;
+  if (P < 64) P = 64;
+  const size_t smem = ((size_t)P + kMaxK) * sizeof(uint64_t);  // + rescoring scratch
+  cudaError_t e = cudaFuncSetAttribute(topk_merge_kernel,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  topk_merge_kernel<<<(unsigned)a.B, kMergeThreads, smem, st>>>(a, P);
+  return cudaGetLastError();
+}
+
+}  // namespace lam

@@ -1,0 +1,116 @@
+// score_common.cuh -- pieces shared by the scoring kernels: the score
+// formulas on integer codes, warp-level top-k lists, and the rank merge.
+#pragma once
+
+#include "lam_internal.cuh"
+
+namespace lam {
+
+// Score of one query against one code row, from
+//   acc = sum_d q_d c_d  and  cc = sum_d c_d^2  (both fp32),
+// with s = 2 eps, s2 = fl32(s*s), qq = ||q||^2, qn = ||q||.
+//   inner product: s * acc                     (= q . xhat)
+//   cosine:        acc / (||q|| sqrt(cc))       (s cancels; 0 for a zero norm)
+//   squared L2:    ||q||^2 + s^2 cc - 2 s acc   (two fused multiply-adds)
+__device__ __forceinline__ float finish_score(int metric, float acc, float cc, float s,
+                                              float s2, float qq, float qn) {
+  if (metric == LAM_METRIC_IP) return s * acc;
+  if (metric == LAM_METRIC_COSINE)
+    return (qn == 0.0f || cc == 0.0f) ? 0.0f : acc / (qn * sqrtf(cc));
+  return fmaf(-2.0f * s, acc, fmaf(s2, cc, qq));
+}
+
+// ---- register top-k list of one warp: slot i = r*32 + lane, ascending keys --
+template <int KPL>
+struct WarpList {
+  uint64_t v[KPL];
+  __device__ __forceinline__ void init() {
+#pragma unroll
+    for (int r = 0; r < KPL; ++r) v[r] = kSentinel;
+  }
+  // Current k-th smallest key (slot k-1), the admission threshold.
+  __device__ __forceinline__ uint64_t kth(int k) const {
+    const int r = (k - 1) >> 5, l = (k - 1) & 31;
+    uint64_t x = v[0];
+#pragma unroll
+    for (int j = 1; j < KPL; ++j)
+      if (j == r) x = v[j];
+    return __shfl_sync(0xffffffffu, x, l);
+  }
+  // Warp-uniform insertion of `key` (the caller checked key < kth).
+  __device__ __forceinline__ void insert(uint64_t key, int lane) {
+    int p = 0;
+#pragma unroll
+    for (int r = 0; r < KPL; ++r) p += __popc(__ballot_sync(0xffffffffu, v[r] < key));
+#pragma unroll
+    for (int r = KPL - 1; r >= 0; --r) {
+      uint64_t up = __shfl_up_sync(0xffffffffu, v[r], 1);
+      uint64_t carry = (r > 0) ? __shfl_sync(0xffffffffu, v[r > 0 ? r - 1 : 0], 31) : key;
+      if (lane == 0) up = carry;
+      const int i = r * 32 + lane;
+      v[r] = (i < p) ? v[r] : (i == p ? key : up);
+    }
+  }
+  // Writes slots [0, k) to dst.
+  __device__ __forceinline__ void store(uint64_t *dst, int k, int lane) const {
+#pragma unroll
+    for (int r = 0; r < KPL; ++r) {
+      const int i = r * 32 + lane;
+      if (i < k) dst[i] = v[r];
+    }
+  }
+};
+
+// ---- shared-memory top-k list of one warp (any k <= kMaxK) ----
+// L[0, k) ascending; *thr mirrors L[k-1].
+__device__ __forceinline__ void smem_list_insert(uint64_t *L, int k, uint64_t key, int lane,
+                                                 uint64_t &thr) {
+  int p = 0;
+  for (int c = 0; c < k; c += 32) {
+    const int i = c + lane;
+    p += __popc(__ballot_sync(0xffffffffu, i < k && L[i] < key));
+  }
+  for (int c = ((k - 1) >> 5) << 5; c >= 0; c -= 32) {
+    const int i = c + lane;
+    uint64_t prev = (i >= 1 && i - 1 < k) ? L[i - 1] : 0;
+    __syncwarp();
+    if (i < k && i > p) L[i] = prev;
+    __syncwarp();
+  }
+  if (lane == 0) L[p] = key;
+  __syncwarp();
+  thr = L[k - 1];
+}
+
+// ---- merge of nl ascending lists of length k (in shared memory) ----
+// Every element finds its rank in the union by binary search in the other
+// lists (ties between equal keys broken by list index); ranks < k are written
+// to out[rank].  Keys are unique except the sentinel, so out gets exactly k.
+__device__ __forceinline__ void rank_merge(const uint64_t *cand, int nl, int k, uint64_t *out,
+                                           int tid, int nthreads) {
+  for (int e = tid; e < nl * k; e += nthreads) {
+    const int l = e / k, i = e - l * k;
+    const uint64_t key = cand[e];
+    int rank = i;
+    for (int l2 = 0; l2 < nl && rank < k; ++l2) {
+      if (l2 == l) continue;
+      const uint64_t *L2 = cand + (size_t)l2 * k;
+      int lo = 0, hi = k;
+      if (l2 < l) {
+        while (lo < hi) {
+          const int mid = (lo + hi) >> 1;
+          if (L2[mid] <= key) lo = mid + 1; else hi = mid;
+        }
+      } else {
+        while (lo < hi) {
+          const int mid = (lo + hi) >> 1;
+          if (L2[mid] < key) lo = mid + 1; else hi = mid;
+        }
+      }
+      rank += lo;
+    }
+    if (rank < k) out[rank] = key;
+  }
+}
+
+}  // namespace lam

@@ -22,3 +22,24 @@ def golden(name):
                 continue
             rows.append(line.split())
     return rows
+
+
+@pytest.fixture(scope="session")
+def dev():
+    """cuda:0 with the library built and loaded (GPU tests only)."""
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2609_32256_gb300 import build as lam_build
+    lam_build.build()
+    import paper_2609_32256_gb300 as lam
+    lam.load()
+    return torch.device("cuda:0")
+
+
+@pytest.fixture
+def score_path(monkeypatch):
+    """Force one kernel path of lam_score_topk for the duration of a test."""
+    def force(name):
+        monkeypatch.setenv("LAM_SCORE_PATH", name)
+    return force

@@ -1,0 +1,126 @@
+"""The C ABI library builds, loads, exports every declared symbol, and rejects
+bad arguments on the host before touching a GPU."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from tests.conftest import ROOT
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2609_32256_gb300 import build as lam_build
+    lam_build.build()
+    import paper_2609_32256_gb300 as lam
+    return lam.load()
+
+
+def declared_symbols():
+    text = open(os.path.join(ROOT, "include", "lam.h")).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(lam_[a-z0-9_]+)\s*\(", text)))
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = declared_symbols()
+    assert len(names) >= 9
+    for name in names:
+        assert hasattr(lib, name), name
+
+
+def test_no_extra_exported_entry_points(lib):
+    # everything named lam_* in the dynamic symbol table is declared in lam.h
+    import subprocess
+    out = subprocess.run(["nm", "-D", "--defined-only", lib._name], capture_output=True,
+                         text=True).stdout
+    exported = {l.split()[-1] for l in out.splitlines() if " T " in l and "lam_" in l}
+    assert exported and exported <= set(declared_symbols())
+
+
+def test_status_strings(lib):
+    import paper_2609_32256_gb300 as lam
+    assert lam.lam_status_string(0) == "ok"
+    assert "invalid" in lam.lam_status_string(1)
+    assert lam.lam_version() >= 100
+    assert lam.lam_quantize_workspace_size() == 16
+
+
+@pytest.mark.parametrize("n,eps,width", [
+    (-1, 1e-3, 0), (10, 0.0, 0), (10, -1e-3, 0), (10, float("nan"), 0), (10, float("inf"), 0),
+    (10, 1e-39, 0), (10, 1e-3, 3), (10, 1e-3, 8)])
+def test_quantize_rejects_bad_arguments(lib, n, eps, width):
+    c = ctypes
+    st = lib.lam_quantize(c.c_void_p(16), n, c.c_float(eps), width, None, 0, c.c_void_p(256), 16,
+                          None, None, None, None, None)
+    assert st == 1
+
+
+def test_quantize_null_input_rejected(lib):
+    c = ctypes
+    assert lib.lam_quantize(None, 5, c.c_float(1e-3), 0, None, 0, c.c_void_p(256), 16, None,
+                            None, None, None, None) == 1
+
+
+def test_quantize_empty_needs_no_device(lib):
+    c = ctypes
+    w, s, lo, hi = c.c_int32(), c.c_float(), c.c_int32(7), c.c_int32(7)
+    st = lib.lam_quantize(None, 0, c.c_float(1e-3), 0, None, 0, None, 0, c.byref(w), c.byref(s),
+                          c.byref(lo), c.byref(hi), None)
+    assert st == 0 and w.value == 1 and s.value == c.c_float(2e-3).value
+    assert (lo.value, hi.value) == (0, 0)
+
+
+def test_quantize_forced_width_small_buffer(lib):
+    c = ctypes
+    st = lib.lam_quantize(c.c_void_p(256), 100, c.c_float(1e-3), 2, c.c_void_p(512), 199,
+                          c.c_void_p(1024), 16, None, None, None, None, None)
+    assert st == 4
+
+
+@pytest.mark.parametrize("args", [
+    dict(B=0), dict(N=0), dict(D=0), dict(k=0), dict(k=1025), dict(k=11, N=10), dict(width=3),
+    dict(metric=3), dict(eps=0.0), dict(code_bound=-1)])
+def test_score_rejects_bad_arguments(lib, args):
+    c = ctypes
+    p = dict(B=2, N=10, D=8, k=3, width=1, metric=0, eps=1e-3, code_bound=0)
+    p.update(args)
+    st = lib.lam_score_topk(c.c_void_p(256), p["B"], c.c_void_p(512), p["width"], p["N"], p["D"],
+                            c.c_float(p["eps"]), p["code_bound"], p["k"], p["metric"],
+                            c.c_void_p(768), c.c_void_p(1024), c.c_void_p(4096), 1 << 20, None)
+    assert st == 1
+
+
+def test_score_rejects_null_and_misaligned_workspace(lib):
+    c = ctypes
+    base = (c.c_void_p(256), 2, c.c_void_p(512), 1, 10, 8, c.c_float(1e-3), 0, 3, 0,
+            c.c_void_p(768), c.c_void_p(1024))
+    assert lib.lam_score_topk(*base, None, 1 << 20, None) == 1
+    assert lib.lam_score_topk(*base, c.c_void_p(4096 + 8), 1 << 20, None) == 1
+
+
+def test_dequantize_rejects_bad_arguments(lib):
+    c = ctypes
+    assert lib.lam_dequantize(None, 1, 10, c.c_float(1.0), c.c_void_p(256), None) == 1
+    assert lib.lam_dequantize(c.c_void_p(256), 3, 10, c.c_float(1.0), c.c_void_p(256), None) == 1
+    assert lib.lam_dequantize(c.c_void_p(256), 1, -1, c.c_float(1.0), c.c_void_p(256), None) == 1
+    assert lib.lam_dequantize(None, 1, 0, c.c_float(1.0), None, None) == 0
+
+
+def test_misaligned_buffers_rejected(lib):
+    c = ctypes
+    ws = c.c_void_p(4096)
+    # fp32 input not 4-byte aligned
+    assert lib.lam_quantize(c.c_void_p(258), 10, c.c_float(1e-3), 2, c.c_void_p(512), 20, ws, 16,
+                            None, None, None, None, None) == 1
+    # int16 codes at an odd address; AUTO codes not 4-byte aligned
+    assert lib.lam_quantize(c.c_void_p(256), 10, c.c_float(1e-3), 2, c.c_void_p(513), 20, ws, 16,
+                            None, None, None, None, None) == 1
+    assert lib.lam_quantize(c.c_void_p(256), 10, c.c_float(1e-3), 0, c.c_void_p(514), 40, ws, 16,
+                            None, None, None, None, None) == 1
+    assert lib.lam_dequantize(c.c_void_p(513), 2, 10, c.c_float(1.0), c.c_void_p(256), None) == 1
+    assert lib.lam_dequantize(c.c_void_p(512), 2, 10, c.c_float(1.0), c.c_void_p(258), None) == 1
+    base = (c.c_void_p(256), 2, c.c_void_p(513), 2, 10, 8, c.c_float(1e-3), 0, 3, 0,
+            c.c_void_p(768), c.c_void_p(1024), c.c_void_p(4096), 1 << 20, None)
+    assert lib.lam_score_topk(*base) == 1

@@ -1,0 +1,157 @@
+"""Exact search on the codes (dequantisation fused into the score, then top-k)
+against the CPU oracle, per kernel path, metric, width and shape, including
+ragged tiles, ragged query blocks, planted exact ties and error statuses."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_2609_32256_gb300 as lam
+from paper_2609_32256_gb300 import inputs
+from tests.parity import check_topk, oracle_topk
+
+pytestmark = pytest.mark.gpu
+METRICS = (oracle.IP, oracle.COSINE, oracle.L2)
+NP_DT = {1: np.int8, 2: np.int16, 4: np.int32}
+
+
+def make_codes(n, d, eps, width, seed=0, dup_every=0):
+    """Unit rows quantized by the oracle; optionally exact duplicate rows."""
+    x = inputs.unit_rows(n, d, seed=seed)
+    if dup_every:
+        x[dup_every::dup_every] = x[0]
+    oc, rmin, rmax, _ = oracle.quantize(x, eps)
+    assert oracle.width(rmin, rmax) <= width
+    return oc.reshape(n, d), max(-int(rmin), int(rmax))
+
+
+def run(dev, q, codes_i32, width, eps, k, metric, code_bound):
+    qt = torch.from_numpy(q).to(dev)
+    ct = torch.from_numpy(codes_i32.astype(NP_DT[width])).to(dev)
+    s, i = lam.search(qt, ct, eps, k, metric, code_bound=code_bound)
+    return s.cpu().numpy(), i.cpu().numpy()
+
+
+def check(dev, q, codes, width, eps, k, metric, bound):
+    gs, gi = run(dev, q, codes, width, eps, k, metric, bound)
+    os_, oi = oracle_topk(q, codes, eps, metric, k)
+    check_topk(gs, gi, q, codes, eps, metric, os_, oi)
+    return gs, gi, os_, oi
+
+
+@pytest.mark.parametrize("metric", METRICS)
+@pytest.mark.parametrize("width,eps", [(1, 1e-2), (2, 1e-3)])
+@pytest.mark.parametrize("B", [1, 2])
+@pytest.mark.parametrize("k", [1, 10, 100, 128])
+def test_bandwidth_path(dev, score_path, metric, width, eps, B, k):
+    score_path("bandwidth")
+    codes, bound = make_codes(5003, 768, eps, width)
+    q = inputs.queries(B, 768, seed=9)
+    assert lam.lam_score_topk_path(B, 5003, 768, k, width, bound) == lam.PATH_BANDWIDTH
+    check(dev, q, codes, width, eps, k, metric, bound)
+
+
+@pytest.mark.parametrize("D", [64, 256, 1024])
+def test_bandwidth_path_other_dims(dev, score_path, D):
+    score_path("bandwidth")
+    codes, bound = make_codes(777, D, 1e-2, 1, seed=D)
+    q = inputs.queries(2, D, seed=3)
+    for metric in METRICS:
+        check(dev, q, codes, 1, 1e-2, 10, metric, bound)
+
+
+@pytest.mark.parametrize("metric", METRICS)
+@pytest.mark.parametrize("width,eps", [(1, 1e-2), (2, 1e-3), (2, 1e-4)])
+@pytest.mark.parametrize("B", [3, 16, 130])
+def test_tensor_path(dev, score_path, metric, width, eps, B):
+    score_path("tensor")
+    codes, bound = make_codes(3001, 768, eps, width, seed=B)
+    q = inputs.queries(B, 768, seed=B + 100)
+    assert lam.lam_score_topk_path(B, 3001, 768, 10, width, bound) == lam.PATH_TENSOR
+    check(dev, q, codes, width, eps, 10, metric, bound)
+
+
+@pytest.mark.parametrize("D", [16, 48, 80, 1024])
+@pytest.mark.parametrize("k", [1, 64, 128])
+def test_tensor_path_dims_and_k(dev, score_path, D, k):
+    score_path("tensor")
+    codes, bound = make_codes(700, D, 1e-2, 1, seed=D + k)
+    q = inputs.queries(20, D, seed=k)
+    for metric in METRICS:
+        check(dev, q, codes, 1, 1e-2, k, metric, bound)
+
+
+@pytest.mark.parametrize("width,eps", [(1, 1e-2), (2, 1e-4), (4, 1e-6)])
+@pytest.mark.parametrize("D", [33, 768])
+def test_generic_path(dev, score_path, width, eps, D):
+    score_path("generic")
+    codes, bound = make_codes(1500, D, eps, width, seed=D)
+    q = inputs.queries(5, D, seed=D)
+    for metric in METRICS:
+        for k in (1, 10, 1024):
+            check(dev, q, codes, width, eps, k, metric, bound)
+
+
+@pytest.mark.parametrize("path", ["bandwidth", "tensor", "generic"])
+def test_exact_ties_rank_lower_id_first(dev, score_path, path):
+    score_path(path)
+    codes, bound = make_codes(2000, 768, 1e-2, 1, dup_every=97)  # rows 0,97,194,... identical
+    q = inputs.unit_rows(2000, 768, seed=0)[:2] if path == "bandwidth" else \
+        inputs.unit_rows(2000, 768, seed=0)[:8]
+    for metric in METRICS:
+        gs, gi, os_, oi = check(dev, q, codes, 1, 1e-2, 25, metric, bound)
+        # query 0 equals row 0, so the 21 copies of it lead, in id order
+        dup = np.arange(0, 2000, 97)
+        np.testing.assert_array_equal(gi[0][: dup.size], dup)
+        np.testing.assert_array_equal(oi[0][: dup.size], dup)
+
+
+def test_auto_selects_paths(dev):
+    assert lam.lam_score_topk_path(1, 361802, 768, 10, 2, 120) == lam.PATH_BANDWIDTH
+    assert lam.lam_score_topk_path(64, 361802, 768, 10, 2, 120) == lam.PATH_TENSOR
+    assert lam.lam_score_topk_path(64, 361802, 768, 10, 2, 0) == lam.PATH_GENERIC
+    assert lam.lam_score_topk_path(64, 361802, 768, 10, 2, 4000) == lam.PATH_GENERIC
+    assert lam.lam_score_topk_path(256, 8388608, 768, 100, 1, 0) == lam.PATH_TENSOR
+    assert lam.lam_score_topk_path(4, 1000, 768, 500, 1, 0) == lam.PATH_GENERIC
+
+
+def test_forced_path_unsupported(dev, score_path):
+    score_path("bandwidth")
+    codes, bound = make_codes(100, 768, 1e-2, 1)
+    q = torch.from_numpy(inputs.queries(5, 768, seed=1)).to(dev)
+    ct = torch.from_numpy(codes.astype(np.int8)).to(dev)
+    assert lam.lam_score_topk_workspace_size(5, 100, 768, 10, 1, bound) == 0
+    ws = torch.empty(1 << 20, dtype=torch.uint8, device=dev)
+    s = torch.empty((5, 10), dtype=torch.float32, device=dev)
+    i = torch.empty((5, 10), dtype=torch.int64, device=dev)
+    with pytest.raises(lam.LamError) as e:
+        lam.lam_score_topk(q, ct, 1, 100, 768, 1e-2, bound, 10, oracle.IP, s, i, ws)
+    assert e.value.status == lam.LAM_ERR_UNSUPPORTED
+
+
+def test_code_bound_violation_reported(dev, score_path):
+    score_path("tensor")
+    codes, _ = make_codes(600, 64, 1e-4, 2)
+    codes[5, 3] = 3000  # beyond what the tensor path can hold exactly
+    q = inputs.queries(4, 64, seed=2)
+    with pytest.raises(lam.LamError) as e:
+        run(dev, q, codes, 2, 1e-4, 10, oracle.IP, 2048)
+    assert e.value.status == lam.LAM_ERR_RANGE
+
+
+def test_k_equals_n_and_single_row(dev):
+    for path_n in (1, 7, 300):
+        codes, bound = make_codes(path_n, 768, 1e-2, 1, seed=path_n)
+        q = inputs.queries(3, 768, seed=4)
+        for metric in METRICS:
+            check(dev, q, codes, 1, 1e-2, path_n, metric, bound) if path_n <= 128 else \
+                check(dev, q, codes, 1, 1e-2, 128, metric, bound)
+
+
+def test_zero_rows_and_zero_query_cosine(dev):
+    codes, bound = make_codes(500, 768, 1e-2, 1)
+    codes[10:20] = 0
+    q = inputs.queries(4, 768, seed=5)
+    q[1] = 0.0
+    for metric in METRICS:
+        check(dev, q, codes, 1, 1e-2, 30, metric, bound)
