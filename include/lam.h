@@ -173,6 +173,40 @@ lam_status lam_score_topk_status(const void *workspace, lam_stream_t stream,
 int32_t lam_score_topk_path(int64_t B, int64_t N, int32_t D, int32_t k,
                             int32_t width, int32_t code_bound);
 
+/*
+ * lam_score_topk_noalloc -- lam_score_topk for callers that cannot allocate
+ * device memory.  (The paper has no counterpart: this is a packaging of the
+ * same search.)
+ *
+ * Who needs it: a caller whose host framework owns all device memory through
+ * its own pool and forbids allocations it did not make, or a latency-critical
+ * caller that cannot afford cudaMalloc's implicit synchronisation, has no way
+ * to provide the workspace lam_score_topk asks for.  This call takes the same
+ * inputs and outputs (all caller-owned device buffers) but keeps its scratch
+ * in a fixed 16 MiB array inside the library, which every GPU that loads the
+ * library holds until the process exits.  It calls no cudaMalloc, cudaFree or
+ * other allocating routine.
+ *
+ * Limits and behaviour:
+ *   - Shapes whose lam_score_topk_workspace_size exceeds 16 MiB (16777216
+ *     bytes) return LAM_ERR_WORKSPACE without queuing anything.
+ *   - The first call on a device looks up the array's device address (once
+ *     per device, with that device current); make that first call before any
+ *     stream capture begins.
+ *   - All calls share the one array, which keeps the last call's contents;
+ *     the status word is cleared at the start of every call.  Calls that
+ *     overlap on the GPU (other streams, other host threads) race on it and
+ *     must be serialised by the caller.
+ *   - Synchronous on `stream`: it waits for the search and returns the device
+ *     status (LAM_ERR_RANGE or LAM_ERR_TIMEOUT as lam_score_topk_status would
+ *     report them) as its own return value.
+ */
+lam_status lam_score_topk_noalloc(const float *queries, int64_t B,
+                                  const void *codes, int32_t width, int64_t N,
+                                  int32_t D, float eps, int32_t code_bound,
+                                  int32_t k, int32_t metric, float *scores,
+                                  int64_t *ids, lam_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -54,6 +54,8 @@ def load():
                                  sz, vp]),
         "lam_score_topk_status": (i32, [vp, vp, P(i32)]),
         "lam_score_topk_path": (i32, [i64, i64, i32, i32, i32, i32]),
+        "lam_score_topk_noalloc": (i32, [vp, i64, vp, i32, i64, i32, f32, i32, i32, i32, vp,
+                                         vp, vp]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -149,3 +151,15 @@ def lam_score_topk_status(workspace, stream=None) -> int:
                                       ctypes.byref(out))
     _check(st, "lam_score_topk_status")
     return out.value
+
+
+def lam_score_topk_noalloc(queries, codes, width, N, D, eps, code_bound, k, metric, scores, ids,
+                           stream=None):
+    """lam_score_topk for callers that cannot allocate: scratch lives in a fixed
+    16 MiB device array inside the library (synchronous; see include/lam.h)."""
+    B = queries.shape[0]
+    st = load().lam_score_topk_noalloc(_ptr(queries), int(B), _ptr(codes), int(width), int(N),
+                                       int(D), ctypes.c_float(eps), int(code_bound), int(k),
+                                       int(metric), _ptr(scores), _ptr(ids),
+                                       _stream(stream, queries.device))
+    _check(st, "lam_score_topk_noalloc")
