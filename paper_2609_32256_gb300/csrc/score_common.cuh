@@ -61,6 +61,63 @@ struct WarpList {
   }
 };
 
+// ---- per-thread top-k in registers: KR slots of (32-bit rank key, row) ----
+// Keys ascend (smaller is better).  The first KR - k slots hold a dummy key 0
+// that nothing can displace, so slot KR-1 is always the k-th best.  Rows must
+// be offered in increasing order: a new key is placed after equal keys, so
+// equal scores keep the lower row first.  Insertion compares the new key with
+// every slot of the unmodified list (no serial dependence) and shifts.
+template <int KR>
+struct RegTopK {
+  uint32_t key[KR];
+  uint32_t id[KR];
+  __device__ __forceinline__ void init(int k) {
+#pragma unroll
+    for (int i = 0; i < KR; ++i) {
+      key[i] = (i < KR - k) ? 0u : 0xffffffffu;
+      id[i] = 0xffffffffu;
+    }
+  }
+  // kc == 0xffffffff inserts nothing.
+  __device__ __forceinline__ void insert(uint32_t kc, uint32_t ic) {
+    bool lt[KR];
+#pragma unroll
+    for (int i = 0; i < KR; ++i) lt[i] = kc < key[i];
+#pragma unroll
+    for (int i = KR - 1; i > 0; --i) {
+      key[i] = lt[i - 1] ? key[i - 1] : (lt[i] ? kc : key[i]);
+      id[i] = lt[i - 1] ? id[i - 1] : (lt[i] ? ic : id[i]);
+    }
+    key[0] = lt[0] ? kc : key[0];
+    id[0] = lt[0] ? ic : id[0];
+  }
+};
+
+// 32-bit rank key of a score (smaller is better) and its inverse.
+__device__ __forceinline__ uint32_t rank_key32(float score, bool desc) {
+  const uint32_t o = ord_f32(score);
+  return desc ? ~o : o;
+}
+__device__ __forceinline__ float rank_key32_score(uint32_t key, bool desc) {
+  return unord_f32(desc ? ~key : key);
+}
+
+// Merges `cnt` buffered candidates (entry i of this thread at buf[i * stride +
+// slot]) into the register list, every lane of the warp in step (lanes with
+// fewer candidates insert nothing), then refreshes the k-th score threshold.
+template <int KR>
+__device__ __forceinline__ void merge_candidates(RegTopK<KR> &reg, const uint2 *buf, int slot,
+                                                 int stride, int &cnt, float &thr_s, bool desc) {
+  const int mx = __reduce_max_sync(0xffffffffu, cnt);
+  for (int i = 0; i < mx; ++i) {
+    const uint2 e = i < cnt ? buf[(size_t)i * stride + slot] : make_uint2(0xffffffffu, 0xffffffffu);
+    reg.insert(e.x, e.y);
+  }
+  cnt = 0;
+  const uint32_t tk = reg.key[KR - 1];
+  thr_s = tk == 0xffffffffu ? (desc ? -INFINITY : INFINITY) : rank_key32_score(tk, desc);
+}
+
 // ---- shared-memory top-k list of one warp (any k <= kMaxK) ----
 // L[0, k) ascending; *thr mirrors L[k-1].
 __device__ __forceinline__ void smem_list_insert(uint64_t *L, int k, uint64_t key, int lane,

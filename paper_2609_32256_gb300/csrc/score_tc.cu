@@ -11,9 +11,15 @@
 // every product being exact in fp32.  The score is then formed from acc*2^-e
 // exactly as the CUDA-core paths form it.
 //
-// CTA: 128 queries (MMA M) x a contiguous range of 256-row tiles (MMA N),
-// K = 32 fp16 per pipeline stage.  Warp roles (320 threads):
-//   warp 0      TMA producer: query hi/lo tiles (64B swizzle) and raw codes;
+// CTA: 128 queries (MMA M) x a contiguous range of 256-row tiles (MMA N).
+// Two shared-memory rings:
+//   MMA stages (K = 32): the query block's hi/lo tiles, laid out by the query
+//     preparation kernel exactly as the 64-byte-swizzled UMMA operand, so one
+//     16 KB bulk copy fills them; and the fp16 code tile the converters write;
+//   raw stages: 256 code rows x 128 bytes (K = 128 int8 / 64 int16, four or
+//     two MMA stages' worth) by one 2-D TMA load with the 128-byte swizzle.
+// Warp roles (320 threads):
+//   warp 0      producer: raw-code TMA loads and query bulk copies;
 //   warp 1      TMEM allocation; one lane issues tcgen05.mma (2 K-steps x
 //               hi/lo per stage) and commits stage/accumulator barriers;
 //   warps 2-5   convert raw int8/int16 codes to fp16 in the UMMA K-major
@@ -35,7 +41,12 @@ constexpr int kBK = 32;         // fp16 per stage along D (64-byte rows)
 constexpr int kUmmaK = 16;      // K of one kind::f16 MMA
 constexpr int kTcThreads = 320;
 constexpr int kABytes = kBM * kBK * 2;    // one of hi / lo: 8 KB
+constexpr int kAStage = 2 * kABytes;      // hi + lo, one bulk copy: 16 KB
 constexpr int kB16Bytes = kBN * kBK * 2;  // converted codes: 16 KB
+constexpr int kStageBytes = kAStage + kB16Bytes;  // one MMA stage: 32 KB
+constexpr int kRawRow = 128;              // bytes of one code row per raw stage
+constexpr int kRawBytes = kBN * kRawRow;  // one raw stage: 32 KB
+constexpr int kCBuf = 16;                 // epilogue candidate buffer per query
 constexpr uint32_t kTmemCols = 512;       // two 256-column accumulators
 constexpr int kMaxDynSmem = 232448;       // 227 KB
 constexpr int kTcMaxK = 128;
@@ -134,45 +145,94 @@ __device__ __forceinline__ void drain_wait_tc(uint64_t *bar, uint32_t parity) {
     if (clock64() - t0 > kWaitCycles) break;
 }
 
+
+// Score from the raw accumulator (2^e q.c), a per-query factor fq and a
+// per-row factor rowf (written by the converters at the end of each tile):
+//   inner product  fq acc                 fq = s 2^-e
+//   cosine         fq acc rowf            fq = 2^-e / ||q||, rowf = 1/||c||
+//   squared L2     fq acc + ||q||^2 + rowf    fq = -2 s 2^-e, rowf = s^2 ||c||^2
+// (the k L2 survivors are rescored in the direct form by the merge).
+__device__ __forceinline__ float tile_score(int metric, float acc, float fq, float qq,
+                                            float rowf) {
+  if (metric == LAM_METRIC_IP) return fq * acc;
+  if (metric == LAM_METRIC_COSINE) return (fq * acc) * rowf;
+  return fmaf(fq, acc, qq + rowf);
+}
+
+// v[j] for a run-time j, by a tree of selects (no local-memory indexing).
+__device__ __forceinline__ uint32_t select32(const uint32_t (&v)[32], int j) {
+  uint32_t t16[16], t8[8], t4[4], t2[2];
+#pragma unroll
+  for (int i = 0; i < 16; ++i) t16[i] = (j & 1) ? v[2 * i + 1] : v[2 * i];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) t8[i] = (j & 2) ? t16[2 * i + 1] : t16[2 * i];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) t4[i] = (j & 4) ? t8[2 * i + 1] : t8[2 * i];
+#pragma unroll
+  for (int i = 0; i < 2; ++i) t2[i] = (j & 8) ? t4[2 * i + 1] : t4[2 * i];
+  return (j & 16) ? t2[1] : t2[0];
+}
+
 struct TcLayout {
-  int ns;
-  int stage_bytes;
-  int raw_bytes;
-  size_t lists_off, cc_off, bar_off, smem_bytes;
+  int ns, nr;  // MMA stages, raw stages
+  size_t raw_off, lists_off, cbuf_off, cc_off, bar_off, smem_bytes;
 };
 
+// Shared memory: [MMA stages][raw stages][k > 32: per-query lists | k <= 32:
+// candidate buffers][c^2 per row, 2 tiles][barriers, TMEM slot, abort flag].
 inline TcLayout tc_layout(int width, int k) {
+  (void)width;
   TcLayout L;
-  L.raw_bytes = kBN * kBK * width;
-  L.stage_bytes = 2 * kABytes + kB16Bytes + L.raw_bytes;
-  const size_t lists = (size_t)kBM * k * 8;
+  const size_t lists = k > 32 ? (size_t)kBM * k * 8 : 0;
+  const size_t cbuf = k > 32 ? 0 : (size_t)kCBuf * kBM * 8;
   const size_t cc = 2 * kBN * 4;
-  const size_t fixed = lists + cc + 8 * 64 + 1024;  // barriers, slots, alignment slack
-  int ns = (int)((kMaxDynSmem - fixed) / L.stage_bytes);
-  if (ns > 6) ns = 6;
+  const size_t tailb = 64 * 8 + 1024;  // barriers, slots, alignment slack
+  const size_t avail = kMaxDynSmem - lists - cbuf - cc - tailb;
+  int ns = 4, nr = 2;
+  while ((size_t)ns * kStageBytes + (size_t)nr * kRawBytes > avail) {
+    if (ns > 2) {
+      --ns;
+    } else if (nr > 1) {
+      --nr;
+    } else {
+      ns = 0;
+      break;
+    }
+  }
   L.ns = ns;
-  L.lists_off = (size_t)ns * L.stage_bytes;
-  L.cc_off = L.lists_off + lists;
+  L.nr = nr;
+  L.raw_off = (size_t)ns * kStageBytes;
+  L.lists_off = L.raw_off + (size_t)nr * kRawBytes;
+  L.cbuf_off = L.lists_off + lists;
+  L.cc_off = L.cbuf_off + cbuf;
   L.bar_off = L.cc_off + cc;
-  L.smem_bytes = L.bar_off + 8 * 64 + 1024;
+  L.smem_bytes = L.bar_off + tailb;
   return L;
 }
 
-template <int W>
+struct TcGeom {
+  int ns, nr;
+  int raw_off, lists_off, cbuf_off, cc_off, bar_off;
+};
+
+template <int W, int KR>
 __global__ void __launch_bounds__(kTcThreads, 1)
-    score_tc_kernel(const __grid_constant__ CUtensorMap qmap,
-                    const __grid_constant__ CUtensorMap cmap, ScoreArgs a, int ns,
-                    int stage_bytes, int lists_off, int cc_off, int bar_off) {
+    score_tc_kernel(const __grid_constant__ CUtensorMap cmap, ScoreArgs a, TcGeom g) {
   extern __shared__ uint8_t tc_smem_raw[];
   // 1024-byte alignment for the swizzled tiles (address bits drive the swizzle)
   const uint32_t base_u32 = smem_u32(tc_smem_raw);
   uint8_t *smem = tc_smem_raw + (((base_u32 + 1023u) & ~1023u) - base_u32);
-  uint64_t *lists = reinterpret_cast<uint64_t *>(smem + lists_off);
-  float *ccbuf = reinterpret_cast<float *>(smem + cc_off);
-  uint64_t *full = reinterpret_cast<uint64_t *>(smem + bar_off);
-  uint64_t *conv = full + ns;
+  const int ns = g.ns, nr = g.nr;
+  uint8_t *raw_ring = smem + g.raw_off;
+  uint64_t *lists = reinterpret_cast<uint64_t *>(smem + g.lists_off);
+  uint2 *cbuf = reinterpret_cast<uint2 *>(smem + g.cbuf_off);
+  float *ccbuf = reinterpret_cast<float *>(smem + g.cc_off);
+  uint64_t *afull = reinterpret_cast<uint64_t *>(smem + g.bar_off);
+  uint64_t *conv = afull + ns;
   uint64_t *empty = conv + ns;
-  uint64_t *accf = empty + ns;
+  uint64_t *rfull = empty + ns;
+  uint64_t *rempty = rfull + nr;
+  uint64_t *accf = rempty + nr;
   uint64_t *acce = accf + 2;
   uint64_t *ccf = acce + 2;
   uint64_t *cce = ccf + 2;
@@ -187,14 +247,19 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   const int64_t te = (int64_t)(blockIdx.x + 1) * n_tiles / gridDim.x;
   const int ntl = (int)(te - tb);
   const int nk = (a.D + kBK - 1) / kBK;
+  constexpr int R = kRawRow / (kBK * W);  // MMA stages per raw stage: 4 (int8), 2 (int16)
   const bool need_cc = a.metric != LAM_METRIC_IP;
-  const int raw_off = 2 * kABytes + kB16Bytes;
+  const uint8_t *qA = static_cast<const uint8_t *>(a.qprep);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < ns; ++s) {
-      mbar_init(&full[s], 1);
+      mbar_init(&afull[s], 1);
       mbar_init(&conv[s], 128);
       mbar_init(&empty[s], 1);
+    }
+    for (int r = 0; r < nr; ++r) {
+      mbar_init(&rfull[r], 1);
+      mbar_init(&rempty[r], 128);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&accf[b], 1);
@@ -214,27 +279,37 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   const uint32_t tmem_base = *tmem_slot;
 
   if (warp == 0) {
-    // ------------------------------------------------ TMA producer -------
+    // ------------------------------------------------ producer -----------
     if (lane == 0) {
-      int it = 0, issued = 0;
+      int it = 0, gr = 0, a_issued = 0, r_issued = 0;
       bool ok = true;
       for (int lt = 0; lt < ntl && ok; ++lt) {
         const int tile = (int)(tb + lt);
         for (int kc = 0; kc < nk; ++kc, ++it) {
+          if (kc % R == 0) {
+            const int rs = gr % nr, rr = gr / nr;
+            if (rr > 0 && !mbar_wait(&rempty[rs], (rr - 1) & 1, abort_flag, a.gflags)) {
+              ok = false;
+              break;
+            }
+            mbar_arrive_expect_tx(&rfull[rs], kRawBytes);
+            tma_load_2d(raw_ring + (size_t)rs * kRawBytes, &cmap, (kc / R) * (kRawRow / W),
+                        tile * kBN, &rfull[rs]);
+            r_issued = ++gr;
+          }
           const int s = it % ns, r = it / ns;
           if (r > 0 && !mbar_wait(&empty[s], (r - 1) & 1, abort_flag, a.gflags)) {
             ok = false;
             break;
           }
-          uint8_t *st = smem + (size_t)s * stage_bytes;
-          mbar_arrive_expect_tx(&full[s], 2 * kABytes + kBN * kBK * W);
-          tma_load_2d(st, &qmap, kc * kBK, qb * kBM, &full[s]);
-          tma_load_2d(st + kABytes, &qmap, kc * kBK, (int)a.Bpad + qb * kBM, &full[s]);
-          tma_load_2d(st + raw_off, &cmap, kc * kBK, tile * kBN, &full[s]);
-          issued = it + 1;
+          mbar_arrive_expect_tx(&afull[s], kAStage);
+          bulk_g2s(smem + (size_t)s * kStageBytes, qA + ((size_t)qb * nk + kc) * kAStage, kAStage,
+                   &afull[s]);
+          a_issued = it + 1;
         }
       }
-      for (int t = max(0, issued - ns); t < issued; ++t) drain_wait_tc(&full[t % ns], (t / ns) & 1);
+      for (int t = max(0, a_issued - ns); t < a_issued; ++t) drain_wait_tc(&afull[t % ns], (t / ns) & 1);
+      for (int t = max(0, r_issued - nr); t < r_issued; ++t) drain_wait_tc(&rfull[t % nr], (t / nr) & 1);
     }
   } else if (warp == 1) {
     // ------------------------------------------------ MMA issuer ---------
@@ -248,15 +323,15 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         const uint32_t d_tmem = tmem_base + (uint32_t)(buf * kBN);
         for (int kc = 0; kc < nk; ++kc, ++it) {
           const int s = it % ns, r = it / ns;
-          if (!mbar_wait(&conv[s], r & 1, abort_flag, a.gflags) ||
-              !mbar_wait(&full[s], r & 1, abort_flag, a.gflags)) {
+          if (!mbar_wait(&afull[s], r & 1, abort_flag, a.gflags) ||
+              !mbar_wait(&conv[s], r & 1, abort_flag, a.gflags)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t st = smem_u32(smem + (size_t)s * stage_bytes);
+          const uint32_t st = smem_u32(smem + (size_t)s * kStageBytes);
           const uint64_t ahi = desc_sw64(st), alo = desc_sw64(st + kABytes),
-                         bd = desc_sw64(st + 2 * kABytes);
+                         bd = desc_sw64(st + kAStage);
 #pragma unroll
           for (int j = 0; j < kBK / kUmmaK; ++j) {
             const uint64_t koff = (uint64_t)((j * kUmmaK * 2) >> 4);
@@ -275,7 +350,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     const int ct = threadIdx.x - 64;  // 0..127
     constexpr int kTasks = (W == 1) ? 4 : 8;
     const __half2 bias = __float2half2_rn(1152.0f);
-    int it = 0;
+    int it = 0, gr = 0;
     bool ok = true;
     float amax = 0.0f;
     for (int lt = 0; lt < ntl && ok; ++lt) {
@@ -284,20 +359,26 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 #pragma unroll
       for (int i = 0; i < kTasks; ++i) ccp[i] = 0.0f;
       for (int kc = 0; kc < nk; ++kc, ++it) {
-        const int s = it % ns, r = it / ns;
-        if (!mbar_wait(&full[s], r & 1, abort_flag, a.gflags)) {
+        const int rs = gr % nr;
+        if (kc % R == 0 && !mbar_wait(&rfull[rs], (gr / nr) & 1, abort_flag, a.gflags)) {
           ok = false;
           break;
         }
-        uint8_t *st = smem + (size_t)s * stage_bytes;
-        const uint8_t *raw = st + raw_off;
-        uint8_t *b16 = st + 2 * kABytes;
+        const int s = it % ns, r = it / ns;
+        if (r > 0 && !mbar_wait(&empty[s], (r - 1) & 1, abort_flag, a.gflags)) {
+          ok = false;
+          break;
+        }
+        const uint8_t *raw = raw_ring + (size_t)rs * kRawBytes;
+        uint8_t *b16 = smem + (size_t)s * kStageBytes + kAStage;
+        const int j0 = (kc % R) * (kBK * W / 16);  // first 16-byte chunk of this K slice
 #pragma unroll
         for (int i = 0; i < kTasks; ++i) {
           const int task = ct + 128 * i;
           if (W == 1) {
             const int row = task >> 1, h = task & 1;
-            const uint4 v = *reinterpret_cast<const uint4 *>(raw + row * 32 + h * 16);
+            const uint4 v = *reinterpret_cast<const uint4 *>(
+                raw + row * kRawRow + (((j0 + h) ^ (row & 7)) << 4));
             const uint32_t w[4] = {v.x, v.y, v.z, v.w};
             uint32_t o[8];
 #pragma unroll
@@ -319,7 +400,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             }
           } else {
             const int row = task >> 2, qt = task & 3;
-            const uint4 v = *reinterpret_cast<const uint4 *>(raw + row * 64 + qt * 16);
+            const uint4 v = *reinterpret_cast<const uint4 *>(
+                raw + row * kRawRow + (((j0 + qt) ^ (row & 7)) << 4));
             const uint32_t w[4] = {v.x ^ 0x80008000u, v.y ^ 0x80008000u, v.z ^ 0x80008000u,
                                    v.w ^ 0x80008000u};
             uint32_t o[4];
@@ -339,6 +421,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         }
         fence_proxy_async_smem();
         mbar_arrive(&conv[s]);
+        if (kc % R == R - 1 || kc == nk - 1) {
+          mbar_arrive(&rempty[rs]);
+          ++gr;
+        }
       }
       if (!ok) break;
       if (need_cc) {
@@ -349,7 +435,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           float t = ccp[i] + __shfl_xor_sync(0xffffffffu, ccp[i], 1);
           if (W == 2) t += __shfl_xor_sync(0xffffffffu, t, 2);
           const bool writer = (W == 1) ? ((task & 1) == 0) : ((task & 3) == 0);
-          if (writer) ccbuf[buf * kBN + (W == 1 ? task >> 1 : task >> 2)] = t;
+          // per-row factor of the score: 1/||c|| for cosine, s^2 ||c||^2 for L2
+          const float rowf = a.metric == LAM_METRIC_COSINE ? (t > 0.0f ? 1.0f / sqrtf(t) : 0.0f)
+                                                          : a.s * a.s * t;
+          if (writer) ccbuf[buf * kBN + (W == 1 ? task >> 1 : task >> 2)] = rowf;
         }
         mbar_arrive(&ccf[buf]);
       }
@@ -363,16 +452,27 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     const bool qvalid = qidx < a.B;
     const int k = a.k;
     const bool desc = a.metric != LAM_METRIC_L2;
-    const float s = a.s, s2 = a.s * a.s;
+    const float s = a.s;
     float pw = 0.0f, qn = 0.0f, qq = 0.0f;
     if (qvalid) {
       const float4 qi = reinterpret_cast<const float4 *>(
-          static_cast<const uint8_t *>(a.qprep) + (size_t)2 * a.Bpad * a.D * 2)[qidx];
+          qA + (size_t)(a.Bpad / kBM) * nk * kAStage)[qidx];
       pw = qi.x;
       qn = qi.y;
       qq = qi.z;
     }
-    for (int i = 0; i < k; ++i) lists[(size_t)i * kBM + m] = kSentinel;
+    // per-query factor of the score: s 2^-e (IP), 2^-e / ||q|| (cosine),
+    // -2 s 2^-e (L2); see tile_score
+    const float fq = a.metric == LAM_METRIC_IP ? s * pw
+                     : a.metric == LAM_METRIC_COSINE ? (qn > 0.0f ? pw / qn : 0.0f)
+                                                     : -2.0f * s * pw;
+    constexpr int RK = KR > 0 ? KR : 1;
+    RegTopK<RK> reg;
+    reg.init(k);
+    float thr_s = desc ? -INFINITY : INFINITY;  // score of the k-th best so far
+    int cnt = 0;                                // buffered candidates of this query
+    if (KR == 0)
+      for (int i = 0; i < k; ++i) lists[(size_t)i * kBM + m] = kSentinel;
     uint64_t thr = kSentinel;
     for (int lt = 0; lt < ntl; ++lt) {
       const int buf = lt & 1, u = lt >> 1;
@@ -385,14 +485,41 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       for (int c = 0; c < kBN / 32; ++c) {
         uint32_t v[32];
         tmem_ld32(taddr + c * 32, v);
-        if (qvalid) {
+        if (KR > 0) {
+          // Candidates must beat the k-th score strictly (rows arrive in
+          // increasing order, so an equal score ranks later).  A compact pass
+          // marks them in a 32-bit mask; the warp then appends them to the
+          // per-query buffers and merges all buffers when one is full.
+          const int64_t nvalid = a.N - (row0 + c * 32);
+          uint32_t mask = 0;
+#pragma unroll
+          for (int j = 0; j < 32; ++j) {
+            const float rf = need_cc ? ccbuf[buf * kBN + c * 32 + j] : 0.0f;
+            const float sc = tile_score(a.metric, __uint_as_float(v[j]), fq, qq, rf);
+            mask |= (uint32_t)(desc ? sc > thr_s : sc < thr_s) << j;
+          }
+          if (!qvalid || nvalid <= 0) mask = 0;
+          else if (nvalid < 32) mask &= (1u << nvalid) - 1u;
+          while (__any_sync(0xffffffffu, mask != 0)) {
+            if (mask != 0) {
+              const int j = __ffs(mask) - 1;
+              mask &= mask - 1;
+              const float rf = need_cc ? ccbuf[buf * kBN + c * 32 + j] : 0.0f;
+              const float sc = tile_score(a.metric, __uint_as_float(select32(v, j)), fq, qq, rf);
+              cbuf[(size_t)cnt * kBM + m] =
+                  make_uint2(rank_key32(sc, desc), (uint32_t)(row0 + c * 32 + j));
+              ++cnt;
+            }
+            if (__any_sync(0xffffffffu, cnt == kCBuf))
+              merge_candidates(reg, cbuf, m, kBM, cnt, thr_s, desc);
+          }
+        } else if (KR == 0 && qvalid) {
 #pragma unroll
           for (int j = 0; j < 32; ++j) {
             const int64_t row = row0 + c * 32 + j;
             if (row < a.N) {
-              const float acc = __uint_as_float(v[j]) * pw;
-              const float cc = need_cc ? ccbuf[buf * kBN + c * 32 + j] : 0.0f;
-              const float sc = finish_score(a.metric, acc, cc, s, s2, qq, qn);
+              const float rf = need_cc ? ccbuf[buf * kBN + c * 32 + j] : 0.0f;
+              const float sc = tile_score(a.metric, __uint_as_float(v[j]), fq, qq, rf);
               const uint64_t key = make_key(sc, (uint32_t)row, desc);
               if (key < thr) {
                 int p = k - 1;
@@ -412,10 +539,18 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       tc_fence_before();
       mbar_arrive(&acce[buf]);
       if (need_cc) mbar_arrive(&cce[buf]);
+      if (KR > 0 && __any_sync(0xffffffffu, cnt > 0)) merge_candidates(reg, cbuf, m, kBM, cnt, thr_s, desc);
     }
+    if (KR > 0 && __any_sync(0xffffffffu, cnt > 0)) merge_candidates(reg, cbuf, m, kBM, cnt, thr_s, desc);
     if (qvalid) {
       uint64_t *out = a.partial + ((size_t)blockIdx.x * a.B + qidx) * k;
-      for (int i = 0; i < k; ++i) out[i] = lists[(size_t)i * kBM + m];
+      if (KR > 0) {
+#pragma unroll
+        for (int i = 0; i < RK; ++i)
+          if (i >= RK - k) out[i - (RK - k)] = ((uint64_t)reg.key[i] << 32) | reg.id[i];
+      } else {
+        for (int i = 0; i < k; ++i) out[i] = lists[(size_t)i * kBM + m];
+      }
     }
   }
 
@@ -427,31 +562,30 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   }
 }
 
-// Query preparation: per query the power-of-two scale, the fp16 hi/lo split
-// (rows [0, Bpad) hold hi, rows [Bpad, 2 Bpad) hold lo; padding rows are zero)
-// and (2^-e, ||q||, ||q||^2).  One warp per query.
+// Query preparation, one warp per query: the power-of-two scale 2^e, the fp16
+// split hi + lo of q 2^e written straight into the operand image the MMA
+// stages load (per query block and 32-wide K slice: [hi 128 x 64 B | lo], rows
+// 64 bytes apart with the 16-byte chunks of row r XOR-ed by (r >> 1) & 3, the
+// 64-byte swizzle), zeros for padding rows and columns; then (2^-e, ||q||,
+// ||q||^2, 0) per query after the images.
 __global__ void __launch_bounds__(256) qprep_kernel(const float *__restrict__ q, int64_t B, int D,
-                                                    int64_t Bpad, __half *__restrict__ qh,
-                                                    float4 *__restrict__ qinfo) {
+                                                    int64_t Bpad, uint8_t *__restrict__ qA) {
   const int64_t b = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (b >= Bpad) return;
-  __half *hi = qh + b * D;
-  __half *lo = qh + (Bpad + b) * D;
-  if (b >= B) {
-    for (int d = lane; d < D; d += 32) {
-      hi[d] = __float2half_rn(0.0f);
-      lo[d] = __float2half_rn(0.0f);
-    }
-    if (lane == 0) qinfo[b] = make_float4(0.f, 0.f, 0.f, 0.f);
-    return;
-  }
+  const int nk = (D + kBK - 1) / kBK;
+  const int64_t qb = b / kBM;
+  const int r = (int)(b % kBM);
+  float4 *qinfo = reinterpret_cast<float4 *>(qA + (size_t)(Bpad / kBM) * nk * kAStage);
+  const bool valid = b < B;
   const float *qr = q + b * D;
   float mx = 0.0f, qq = 0.0f;
-  for (int d = lane; d < D; d += 32) {
-    const float v = qr[d];
-    mx = fmaxf(mx, fabsf(v));
-    qq = fmaf(v, v, qq);
+  if (valid) {
+    for (int d = lane; d < D; d += 32) {
+      const float v = qr[d];
+      mx = fmaxf(mx, fabsf(v));
+      qq = fmaf(v, v, qq);
+    }
   }
   for (int off = 16; off > 0; off >>= 1) {
     mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
@@ -465,13 +599,19 @@ __global__ void __launch_bounds__(256) qprep_kernel(const float *__restrict__ q,
     e = max(-126, min(126, e));
   }
   const float sc = ldexpf(1.0f, e);
-  for (int d = lane; d < D; d += 32) {
-    const float v = qr[d] * sc;
+  for (int d = lane; d < nk * kBK; d += 32) {
+    const float v = (valid && d < D) ? qr[d] * sc : 0.0f;
     const __half h = __float2half_rn(v);
-    hi[d] = h;
-    lo[d] = __float2half_rn(v - __half2float(h));
+    const __half l = __float2half_rn(v - __half2float(h));
+    const int kc = d / kBK, kk = d % kBK;
+    const size_t off = ((size_t)qb * nk + kc) * kAStage + (size_t)r * 64 +
+                       (size_t)((((kk >> 3) ^ ((r >> 1) & 3)) << 4) + (kk & 7) * 2);
+    *reinterpret_cast<__half *>(qA + off) = h;
+    *reinterpret_cast<__half *>(qA + off + kABytes) = l;
   }
-  if (lane == 0) qinfo[b] = make_float4(ldexpf(1.0f, -e), sqrtf(qq), qq, 0.0f);
+  if (lane == 0)
+    qinfo[b] = valid ? make_float4(ldexpf(1.0f, -e), sqrtf(qq), qq, 0.0f)
+                     : make_float4(0.f, 0.f, 0.f, 0.f);
 }
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
@@ -534,47 +674,50 @@ int tensor_splits(int64_t B, int64_t N, int sms) {
 }
 
 size_t tensor_qprep_bytes(int64_t Bpad, int D) {
-  return (size_t)2 * Bpad * D * 2 + (size_t)Bpad * 16;
+  const int64_t nk = (D + kBK - 1) / kBK;
+  return (size_t)(Bpad / kBM) * nk * kAStage + (size_t)Bpad * 16;
 }
 
 cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st) {
   if (a.k > kTcMaxK || (a.width != 1 && a.width != 2)) return cudaErrorInvalidValue;
   const TcLayout L = tc_layout(a.width, a.k);
   if (L.ns < 2) return cudaErrorInvalidValue;
-  __half *qh = static_cast<__half *>(a.qprep);
-  float4 *qinfo = reinterpret_cast<float4 *>(static_cast<uint8_t *>(a.qprep) +
-                                             (size_t)2 * a.Bpad * a.D * 2);
-  qprep_kernel<<<(unsigned)((a.Bpad + 7) / 8), 256, 0, st>>>(a.queries, a.B, a.D, a.Bpad, qh,
-                                                             qinfo);
+  uint8_t *qA = static_cast<uint8_t *>(a.qprep);
+  qprep_kernel<<<(unsigned)((a.Bpad + 7) / 8), 256, 0, st>>>(a.queries, a.B, a.D, a.Bpad, qA);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
 
-  CUtensorMap qmap, cmap;
-  if (!make_map_2d(&qmap, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, qh, (uint64_t)a.D,
-                   (uint64_t)(2 * a.Bpad), (uint64_t)a.D * 2, kBK, kBM,
-                   CU_TENSOR_MAP_SWIZZLE_64B))
-    return cudaErrorInvalidValue;
+  CUtensorMap cmap;
   if (!make_map_2d(&cmap,
                    a.width == 1 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_UINT16,
-                   a.codes, (uint64_t)a.D, (uint64_t)a.N, (uint64_t)a.D * a.width, kBK, kBN,
-                   CU_TENSOR_MAP_SWIZZLE_NONE))
+                   a.codes, (uint64_t)a.D, (uint64_t)a.N, (uint64_t)a.D * a.width,
+                   (uint32_t)(kRawRow / a.width), kBN, CU_TENSOR_MAP_SWIZZLE_128B))
     return cudaErrorInvalidValue;
 
+  TcGeom g;
+  g.ns = L.ns;
+  g.nr = L.nr;
+  g.raw_off = (int)L.raw_off;
+  g.lists_off = (int)L.lists_off;
+  g.cbuf_off = (int)L.cbuf_off;
+  g.cc_off = (int)L.cc_off;
+  g.bar_off = (int)L.bar_off;
   const dim3 grid((unsigned)a.n_lists, (unsigned)(a.Bpad / kBM));
+  auto run = [&](auto kern) -> cudaError_t {
+    cudaError_t r = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)L.smem_bytes);
+    if (r != cudaSuccess) return r;
+    kern<<<grid, kTcThreads, L.smem_bytes, st>>>(cmap, a, g);
+    return cudaGetLastError();
+  };
   if (a.width == 1) {
-    e = cudaFuncSetAttribute(score_tc_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)L.smem_bytes);
-    if (e != cudaSuccess) return e;
-    score_tc_kernel<1><<<grid, kTcThreads, L.smem_bytes, st>>>(
-        qmap, cmap, a, L.ns, L.stage_bytes, (int)L.lists_off, (int)L.cc_off, (int)L.bar_off);
-  } else {
-    e = cudaFuncSetAttribute(score_tc_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)L.smem_bytes);
-    if (e != cudaSuccess) return e;
-    score_tc_kernel<2><<<grid, kTcThreads, L.smem_bytes, st>>>(
-        qmap, cmap, a, L.ns, L.stage_bytes, (int)L.lists_off, (int)L.cc_off, (int)L.bar_off);
+    if (a.k <= 16) return run(score_tc_kernel<1, 16>);
+    if (a.k <= 32) return run(score_tc_kernel<1, 32>);
+    return run(score_tc_kernel<1, 0>);
   }
-  return cudaGetLastError();
+  if (a.k <= 16) return run(score_tc_kernel<2, 16>);
+  if (a.k <= 32) return run(score_tc_kernel<2, 32>);
+  return run(score_tc_kernel<2, 0>);
 }
 
 }  // namespace lam

@@ -72,7 +72,7 @@ def test_tensor_path(dev, score_path, metric, width, eps, B):
 
 
 @pytest.mark.parametrize("D", [16, 48, 80, 1024])
-@pytest.mark.parametrize("k", [1, 64, 128])
+@pytest.mark.parametrize("k", [1, 16, 17, 32, 64, 112])
 def test_tensor_path_dims_and_k(dev, score_path, D, k):
     score_path("tensor")
     codes, bound = make_codes(700, D, 1e-2, 1, seed=D + k)
