@@ -30,11 +30,17 @@ METRIC = "Q_ε GB/s and fused score+top-k memory vectors/s at D=768; % of HBM ro
 UNIT = "memory vectors/s"
 L2_FLUSH_BYTES = 512 << 20
 
+# DRAM bytes (read + write) of one launch of the dominant kernel, from one ncu
+# capture (profiles/score_tc_kernel_chunks_n27986_ip.md).  Reported only while
+# the kernel source is the one the counters were taken on.
+TC_TRAFFIC = {"source_sha256_16": "7c88b5c46b34d835", "bytes": 24713728,
+              "launch": "int8 codes, eps=1e-2, 27,986 x 768, 1,024 queries"}
+
 
 def parse():
     p = argparse.ArgumentParser()
     p.add_argument("--gpus", type=int, default=1)
-    p.add_argument("--steps", type=int, default=300)
+    p.add_argument("--steps", type=int, default=1000)
     p.add_argument("--warmup", type=int, default=10)
     p.add_argument("--impl", default="lam", choices=["lam", "reference"])
     p.add_argument("--workload", default="chunks_n27986_ip")
@@ -277,10 +283,19 @@ def run_lam(args):
     hbm_peak, tc_peak, peak_kind = load_peaks()
     path_names = {0: "bandwidth", 1: "tensor", 2: "generic"}
     paths = [path_names[p] for (_, _, p) in pipe.plan]
+    traffic = None
+    try:
+        import hashlib
+        with open(os.path.join(ROOT, "paper_2609_32256_gb300", "csrc", "score_tc.cu"), "rb") as f:
+            if hashlib.sha256(f.read()).hexdigest()[:16] == TC_TRAFFIC["source_sha256_16"]:
+                traffic = TC_TRAFFIC["bytes"]
+    except OSError:
+        pass
     if all(p == "tensor" for p in paths):
         achieved = flops / (ms_s / 1e3) / 1e12
         roofline = {"bound": "tensor", "achieved": round(achieved, 2), "peak": tc_peak,
-                    "unit": "TFLOP/s", "frac": round(achieved / tc_peak, 4), "traffic": None,
+                    "unit": "TFLOP/s", "frac": round(achieved / tc_peak, 4), "traffic": traffic,
+                    "traffic_launch": TC_TRAFFIC["launch"] if traffic else None,
                     "kernel": "score_tc_kernel (timed span: lam_score_topk = query prep + "
                               "tcgen05 score + merge)", "peak_source": peak_kind + " bf16 dense burst "
                               "(fp16 has the same nominal rate)"}

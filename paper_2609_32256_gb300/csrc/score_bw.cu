@@ -437,7 +437,8 @@ cudaError_t launch_topk_merge(const ScoreArgs &a, cudaStream_t st) {
   cudaError_t e = cudaFuncSetAttribute(topk_merge_kernel,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  topk_merge_kernel<<<(unsigned)a.B, kMergeThreads, smem, st>>>(a, P);
+  const int threads = P / 2 < 32 ? 32 : (P / 2 > kMergeThreads ? kMergeThreads : P / 2);
+  topk_merge_kernel<<<(unsigned)a.B, threads, smem, st>>>(a, P);
   return cudaGetLastError();
 }
 

@@ -39,7 +39,8 @@ constexpr int kBM = 128;        // queries per CTA (MMA M)
 constexpr int kBN = 256;        // code rows per tile (MMA N)
 constexpr int kBK = 32;         // fp16 per stage along D (64-byte rows)
 constexpr int kUmmaK = 16;      // K of one kind::f16 MMA
-constexpr int kTcThreads = 320;
+constexpr int kTcThreads = 320;  // 10 warps, roles below
+constexpr int kConvThreads = 128;
 constexpr int kABytes = kBM * kBK * 2;    // one of hi / lo: 8 KB
 constexpr int kAStage = 2 * kABytes;      // hi + lo, one bulk copy: 16 KB
 constexpr int kB16Bytes = kBN * kBK * 2;  // converted codes: 16 KB
@@ -254,17 +255,17 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   if (threadIdx.x == 0) {
     for (int s = 0; s < ns; ++s) {
       mbar_init(&afull[s], 1);
-      mbar_init(&conv[s], 128);
+      mbar_init(&conv[s], kConvThreads);
       mbar_init(&empty[s], 1);
     }
     for (int r = 0; r < nr; ++r) {
       mbar_init(&rfull[r], 1);
-      mbar_init(&rempty[r], 128);
+      mbar_init(&rempty[r], kConvThreads);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&accf[b], 1);
       mbar_init(&acce[b], 128);
-      mbar_init(&ccf[b], 128);
+      mbar_init(&ccf[b], kConvThreads);
       mbar_init(&cce[b], 128);
     }
     mbar_init(done, 1);
@@ -347,8 +348,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     }
   } else if (warp < 6) {
     // ------------------------------------------------ converters ---------
-    const int ct = threadIdx.x - 64;  // 0..127
-    constexpr int kTasks = (W == 1) ? 4 : 8;
+    const int ct = threadIdx.x - 64;  // 0 .. 127
+    constexpr int kTasks = (W == 1 ? 512 : 1024) / kConvThreads;  // 16-byte chunks per thread
     const __half2 bias = __float2half2_rn(1152.0f);
     int it = 0, gr = 0;
     bool ok = true;
@@ -369,17 +370,25 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           ok = false;
           break;
         }
-        const uint8_t *raw = raw_ring + (size_t)rs * kRawBytes;
-        uint8_t *b16 = smem + (size_t)s * kStageBytes + kAStage;
+        const uint8_t *__restrict__ raw = raw_ring + (size_t)rs * kRawBytes;
+        uint8_t *__restrict__ b16 = smem + (size_t)s * kStageBytes + kAStage;
         const int j0 = (kc % R) * (kBK * W / 16);  // first 16-byte chunk of this K slice
+        // All loads first: the stores below could alias them as far as the
+        // compiler knows, which would otherwise serialise the tasks.
+        uint4 rv[kTasks];
 #pragma unroll
         for (int i = 0; i < kTasks; ++i) {
-          const int task = ct + 128 * i;
+          const int task = ct + kConvThreads * i;
+          const int row = (W == 1) ? task >> 1 : task >> 2;
+          const int sub = (W == 1) ? task & 1 : task & 3;
+          rv[i] = *reinterpret_cast<const uint4 *>(raw + row * kRawRow + (((j0 + sub) ^ (row & 7)) << 4));
+        }
+#pragma unroll
+        for (int i = 0; i < kTasks; ++i) {
+          const int task = ct + kConvThreads * i;
           if (W == 1) {
             const int row = task >> 1, h = task & 1;
-            const uint4 v = *reinterpret_cast<const uint4 *>(
-                raw + row * kRawRow + (((j0 + h) ^ (row & 7)) << 4));
-            const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+            const uint32_t w[4] = {rv[i].x, rv[i].y, rv[i].z, rv[i].w};
             uint32_t o[8];
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
@@ -400,10 +409,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             }
           } else {
             const int row = task >> 2, qt = task & 3;
-            const uint4 v = *reinterpret_cast<const uint4 *>(
-                raw + row * kRawRow + (((j0 + qt) ^ (row & 7)) << 4));
-            const uint32_t w[4] = {v.x ^ 0x80008000u, v.y ^ 0x80008000u, v.z ^ 0x80008000u,
-                                   v.w ^ 0x80008000u};
+            const uint32_t w[4] = {rv[i].x ^ 0x80008000u, rv[i].y ^ 0x80008000u,
+                                   rv[i].z ^ 0x80008000u, rv[i].w ^ 0x80008000u};
             uint32_t o[4];
             float c2 = 0.0f;
 #pragma unroll
@@ -431,7 +438,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         if (u > 0 && !mbar_wait(&cce[buf], (u - 1) & 1, abort_flag, a.gflags)) break;
 #pragma unroll
         for (int i = 0; i < kTasks; ++i) {
-          const int task = ct + 128 * i;
+          const int task = ct + kConvThreads * i;
           float t = ccp[i] + __shfl_xor_sync(0xffffffffu, ccp[i], 1);
           if (W == 2) t += __shfl_xor_sync(0xffffffffu, t, 2);
           const bool writer = (W == 1) ? ((task & 1) == 0) : ((task & 3) == 0);
@@ -446,6 +453,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     if (W == 2 && amax > 2048.0f) atomicOr(a.gflags, kFlagRange);
   } else {
     // ------------------------------------------------ epilogue -----------
+    // (warp w may read TMEM lanes 32 (w % 4) .. 32 (w % 4) + 31)
     const int quad = warp & 3;
     const int m = quad * 32 + lane;  // TMEM lane = query within the block
     const int64_t qidx = (int64_t)qb * kBM + m;
@@ -599,15 +607,25 @@ __global__ void __launch_bounds__(256) qprep_kernel(const float *__restrict__ q,
     e = max(-126, min(126, e));
   }
   const float sc = ldexpf(1.0f, e);
-  for (int d = lane; d < nk * kBK; d += 32) {
-    const float v = (valid && d < D) ? qr[d] * sc : 0.0f;
-    const __half h = __float2half_rn(v);
-    const __half l = __float2half_rn(v - __half2float(h));
-    const int kc = d / kBK, kk = d % kBK;
+  // lane writes whole 16-byte chunks (8 fp16) of the hi and lo images
+  for (int ch = lane; ch < nk * (kBK / 8); ch += 32) {
+    const int d0 = ch * 8, kc = d0 / kBK, c16 = (d0 % kBK) / 8;
+    uint32_t hw[4], lw[4];
+#pragma unroll
+    for (int t = 0; t < 4; ++t) {
+      const int d = d0 + 2 * t;
+      const float v0 = (valid && d < D) ? qr[d] * sc : 0.0f;
+      const float v1 = (valid && d + 1 < D) ? qr[d + 1] * sc : 0.0f;
+      const __half2 h = __floats2half2_rn(v0, v1);
+      const float2 hf = __half22float2(h);
+      const __half2 l = __floats2half2_rn(v0 - hf.x, v1 - hf.y);
+      hw[t] = h2_as_u32(h);
+      lw[t] = h2_as_u32(l);
+    }
     const size_t off = ((size_t)qb * nk + kc) * kAStage + (size_t)r * 64 +
-                       (size_t)((((kk >> 3) ^ ((r >> 1) & 3)) << 4) + (kk & 7) * 2);
-    *reinterpret_cast<__half *>(qA + off) = h;
-    *reinterpret_cast<__half *>(qA + off + kABytes) = l;
+                       (size_t)((c16 ^ ((r >> 1) & 3)) << 4);
+    *reinterpret_cast<uint4 *>(qA + off) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+    *reinterpret_cast<uint4 *>(qA + off + kABytes) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
   }
   if (lane == 0)
     qinfo[b] = valid ? make_float4(ldexpf(1.0f, -e), sqrtf(qq), qq, 0.0f)
