@@ -46,6 +46,11 @@ def parse():
     p.add_argument("--workload", default="chunks_n27986_ip")
     p.add_argument("--batch", type=int, default=0, help="query batch (default: workload's first)")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--kernels", action="store_true",
+                   help="time each C-ABI call of --workload separately (not the headline step)")
+    p.add_argument("--reps", type=int, default=20)
+    p.add_argument("--eps", type=float, default=0.0, help="(--kernels) one eps instead of the sweep")
+    p.add_argument("--width", type=int, default=-1, help="(--kernels) forced code width")
     return p.parse_args()
 
 
@@ -421,9 +426,98 @@ def run_reference(args):
         dist.destroy_process_group()
 
 
+def run_kernels(args):
+    """Per-call timing of one workload: Q_eps (AUTO and at the resolved width),
+    dequantisation and lam_score_topk per query batch, each as the mean of
+    --reps CUDA-event spans with a 512 MB L2 flush before every rep."""
+    import torch
+    import paper_2609_32256_gb300 as lam
+    from paper_2609_32256_gb300 import build as lam_build, inputs
+    lam_build.build()
+    lam.load()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    wl = inputs.WORKLOADS[args.workload]
+    if wl.d == 1:
+        x = torch.from_numpy(inputs.flat_values(wl.n, seed=0)).to(dev)
+    elif wl.slab_rows:
+        x = inputs.unit_rows_device(wl.n, wl.d, seed=0, device=dev)
+    elif wl.planted:
+        x = torch.from_numpy(inputs.planted_rows(wl.n, wl.d, seed=0)).to(dev)
+    else:
+        x = torch.from_numpy(inputs.unit_rows(wl.n, wl.d, seed=0)).to(dev)
+    n = x.numel()
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    ws = torch.zeros(64, dtype=torch.uint8, device=dev)
+    codes = torch.empty(n * 4, dtype=torch.uint8, device=dev)
+    out = torch.empty(n, dtype=torch.float32, device=dev)
+
+    def timed(fn):
+        for i in range(3):
+            flush.fill_(float(i))
+            fn()
+        tot = 0.0
+        for i in range(args.reps):
+            flush.fill_(float(i))
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            fn()
+            e1.record()
+            torch.cuda.synchronize(dev)
+            tot += e0.elapsed_time(e1)
+        return tot / args.reps
+
+    res = {"workload": wl.name, "n_values": n, "quantize": [], "dequantize": [], "score": []}
+    hbm, tc_peak, kind = load_peaks()
+    widths = {}
+    eps_list = (args.eps,) if args.eps else wl.eps
+    for e in eps_list:
+        _, w, sc, cmin, cmax = lam.lam_quantize(x, e, 0, None, ws)
+        wq = args.width if args.width > 0 else (wl.width or w)
+        widths[e] = (wq, sc, max(-cmin, cmax))
+        ms_auto = timed(lambda: lam.lam_quantize(x, e, 0, codes, ws))
+        ms_forced = timed(lambda: lam.lam_quantize(x, e, wq, codes, ws))
+        gbs = (4 + wq) * n / (ms_forced / 1e3) / 1e9
+        res["quantize"].append({"eps": e, "width": wq, "ms_auto_span": ms_auto,
+                                "ms_forced_span": ms_forced, "gbs_forced_span": gbs,
+                                "frac_of_hbm": gbs / hbm})
+        lam.lam_quantize(x, e, wq, codes, ws)
+        ms_d = timed(lambda: lam.lam_dequantize(codes, wq, n, sc, out))
+        gbd = (wq + 4) * n / (ms_d / 1e3) / 1e9
+        res["dequantize"].append({"eps": e, "width": wq, "ms": ms_d, "gbs": gbd,
+                                  "frac_of_hbm": gbd / hbm})
+    if wl.batches and wl.d > 1:
+        e = eps_list[0]
+        wq, sc, bound = widths[e]
+        lam.lam_quantize(x, e, wq, codes, ws)
+        N = wl.n
+        batches = [args.batch] if args.batch else list(wl.batches)
+        for B in batches:
+            q = torch.from_numpy(inputs.queries(B, wl.d, seed=1)).to(dev)
+            nb = lam.lam_score_topk_workspace_size(B, N, wl.d, wl.k, wq, bound)
+            sws = torch.empty(nb, dtype=torch.uint8, device=dev)
+            s_ = torch.empty((B, wl.k), dtype=torch.float32, device=dev)
+            i_ = torch.empty((B, wl.k), dtype=torch.int64, device=dev)
+            path = lam.lam_score_topk_path(B, N, wl.d, wl.k, wq, bound)
+            ms = timed(lambda: lam.lam_score_topk(q, codes, wq, N, wl.d, e, bound, wl.k, wl.metric,
+                                                  s_, i_, sws))
+            code_bytes = N * wl.d * wq
+            fl = 2.0 * N * wl.d * B
+            res["score"].append({"B": B, "path": ["bandwidth", "tensor", "generic"][path],
+                                 "ms_span": ms, "vectors_per_s": N / (ms / 1e3),
+                                 "code_gbs": code_bytes / (ms / 1e3) / 1e9,
+                                 "frac_of_hbm": code_bytes / (ms / 1e3) / 1e9 / hbm,
+                                 "tflops": fl / (ms / 1e3) / 1e12,
+                                 "frac_of_tensor": fl / (ms / 1e3) / 1e12 / tc_peak})
+    res["peaks"] = {"hbm_gbs": hbm, "bf16_tflops": tc_peak, "kind": kind}
+    print(json.dumps(res))
+
+
 def main():
     args = parse()
-    if args.impl == "reference":
+    if args.kernels:
+        run_kernels(args)
+    elif args.impl == "reference":
         run_reference(args)
     else:
         run_lam(args)

@@ -18,37 +18,40 @@ namespace lam {
 
 namespace {
 
-constexpr int kBwWarps = 8;
+constexpr int kBwWarps = 16;  // consumer warps; each scores two rows at a time
 constexpr int kBwThreads = (kBwWarps + 1) * 32;
 constexpr int kNchMax = 4;  // 8-coordinate vectors per lane per row: D <= 1024
-constexpr int kBwStageTarget = 32 * 1024;
+constexpr int kBwStageTarget = 48 * 1024;
 constexpr int kBwSmemBudget = 200 * 1024;
 
-// 8 codes -> 8 exact fp32 values.
+// 8 codes -> 8 exact fp32 values as 4 packed pairs (element 2i in .x, 2i+1 in
+// .y): the byte-permute places a biased code in the mantissa of 2^23, one
+// packed subtraction removes 2^23 and the bias.
 template <int W>
-__device__ __forceinline__ void decode8(const uint8_t *p, float *f) {
+__device__ __forceinline__ void decode8x2(const uint8_t *p, float2 *f) {
   if (W == 1) {
     const uint2 v = *reinterpret_cast<const uint2 *>(p);
     const uint32_t a = v.x ^ 0x80808080u, b = v.y ^ 0x80808080u;
     // bits 0x4B0000uu = 2^23 + u with u = code + 128
-    f[0] = __int_as_float(__byte_perm(a, 0x4B000000u, 0x7540)) - 8388736.0f;
-    f[1] = __int_as_float(__byte_perm(a, 0x4B000000u, 0x7541)) - 8388736.0f;
-    f[2] = __int_as_float(__byte_perm(a, 0x4B000000u, 0x7542)) - 8388736.0f;
-    f[3] = __int_as_float(__byte_perm(a, 0x4B000000u, 0x7543)) - 8388736.0f;
-    f[4] = __int_as_float(__byte_perm(b, 0x4B000000u, 0x7540)) - 8388736.0f;
-    f[5] = __int_as_float(__byte_perm(b, 0x4B000000u, 0x7541)) - 8388736.0f;
-    f[6] = __int_as_float(__byte_perm(b, 0x4B000000u, 0x7542)) - 8388736.0f;
-    f[7] = __int_as_float(__byte_perm(b, 0x4B000000u, 0x7543)) - 8388736.0f;
+    const float2 bias = make_float2(-8388736.0f, -8388736.0f);
+    f[0] = __fadd2_rn(make_float2(__int_as_float(__byte_perm(a, 0x4B000000u, 0x7540)),
+                                  __int_as_float(__byte_perm(a, 0x4B000000u, 0x7541))), bias);
+    f[1] = __fadd2_rn(make_float2(__int_as_float(__byte_perm(a, 0x4B000000u, 0x7542)),
+                                  __int_as_float(__byte_perm(a, 0x4B000000u, 0x7543))), bias);
+    f[2] = __fadd2_rn(make_float2(__int_as_float(__byte_perm(b, 0x4B000000u, 0x7540)),
+                                  __int_as_float(__byte_perm(b, 0x4B000000u, 0x7541))), bias);
+    f[3] = __fadd2_rn(make_float2(__int_as_float(__byte_perm(b, 0x4B000000u, 0x7542)),
+                                  __int_as_float(__byte_perm(b, 0x4B000000u, 0x7543))), bias);
   } else {
     const uint4 v = *reinterpret_cast<const uint4 *>(p);
     const uint32_t w[4] = {v.x ^ 0x80008000u, v.y ^ 0x80008000u, v.z ^ 0x80008000u,
                            v.w ^ 0x80008000u};
     // bits 0x4B00uuuu = 2^23 + u with u = code + 32768
+    const float2 bias = make_float2(-8421376.0f, -8421376.0f);
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      f[2 * j] = __int_as_float(__byte_perm(w[j], 0x4B000000u, 0x7410)) - 8421376.0f;
-      f[2 * j + 1] = __int_as_float(__byte_perm(w[j], 0x4B000000u, 0x7432)) - 8421376.0f;
-    }
+    for (int j = 0; j < 4; ++j)
+      f[j] = __fadd2_rn(make_float2(__int_as_float(__byte_perm(w[j], 0x4B000000u, 0x7410)),
+                                    __int_as_float(__byte_perm(w[j], 0x4B000000u, 0x7432))), bias);
   }
 }
 
@@ -56,6 +59,17 @@ __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
   return v;
+}
+
+// Sums a over the lanes 0-15 and b over the lanes 16-31 with one shared
+// butterfly: lanes 0-15 end with sum(a), lanes 16-31 with sum(b).
+__device__ __forceinline__ float pair_sum(float a, float b, int lane) {
+  const bool lo = lane < 16;
+  float keep = lo ? a : b;
+  keep += __shfl_xor_sync(0xffffffffu, lo ? b : a, 16);
+#pragma unroll
+  for (int off = 8; off > 0; off >>= 1) keep += __shfl_xor_sync(0xffffffffu, keep, off);
+  return keep;
 }
 
 // Waits (bounded, ignoring the abort flag) until a phase that is known to be
@@ -74,8 +88,8 @@ struct BwShape {
 
 inline BwShape bw_shape(int D, int width) {
   const int row = D * width;
-  int tr = (kBwStageTarget / (row * kBwWarps)) * kBwWarps;
-  if (tr < kBwWarps) tr = kBwWarps;
+  int tr = (kBwStageTarget / (row * 2 * kBwWarps)) * 2 * kBwWarps;
+  if (tr < 2 * kBwWarps) tr = 2 * kBwWarps;
   BwShape sh;
   sh.tr = tr;
   sh.stage_bytes = tr * row;
@@ -85,7 +99,7 @@ inline BwShape bw_shape(int D, int width) {
   return sh;
 }
 
-template <int W, int QB, int KPL>
+template <int W, int QB, int KPL, bool CC>
 __global__ void __launch_bounds__(kBwThreads, 1)
     score_bw_kernel(ScoreArgs a, int tr, int ns, int stage_bytes) {
   extern __shared__ __align__(1024) uint8_t smem[];
@@ -134,9 +148,9 @@ __global__ void __launch_bounds__(kBwThreads, 1)
       for (int t = max(0, issued - ns); t < issued; ++t) drain_wait(&full[t % ns], (t / ns) & 1);
     }
   } else {
-    // ---------------- consumers -----------------------------------------
+    // ---------------- consumers: two rows per warp at a time -------------
     const int nch = (D + 255) / 256;
-    float qreg[QB][kNchMax][8];
+    float2 qreg[QB][kNchMax][4];
     float qq[QB], qn[QB];
 #pragma unroll
     for (int q = 0; q < QB; ++q) {
@@ -146,61 +160,81 @@ __global__ void __launch_bounds__(kBwThreads, 1)
       for (int j = 0; j < kNchMax; ++j) {
         const int e0 = (j * 32 + lane) * 8;
 #pragma unroll
-        for (int t = 0; t < 8; ++t) {
-          const float v = (qv && j < nch && e0 + t < D) ? a.queries[(int64_t)q * D + e0 + t] : 0.0f;
-          qreg[q][j][t] = v;
-          part = fmaf(v, v, part);
+        for (int t = 0; t < 4; ++t) {
+          const int d = e0 + 2 * t;
+          const float v0 = (qv && j < nch && d < D) ? a.queries[(int64_t)q * D + d] : 0.0f;
+          const float v1 = (qv && j < nch && d + 1 < D) ? a.queries[(int64_t)q * D + d + 1] : 0.0f;
+          qreg[q][j][t] = make_float2(v0, v1);
+          part = fmaf(v0, v0, fmaf(v1, v1, part));
         }
       }
       qq[q] = warp_sum(part);
       qn[q] = sqrtf(qq[q]);
     }
-    const bool need_cc = a.metric != LAM_METRIC_IP;
     const bool desc = a.metric != LAM_METRIC_L2;
     const float s = a.s, s2 = a.s * a.s;
-
-    uint64_t thr[QB];
+    float thr_s[QB];  // score of each list's k-th entry; rows come in increasing
+                      // order, so only a strictly better score can enter
 #pragma unroll
-    for (int q = 0; q < QB; ++q) thr[q] = kSentinel;
+    for (int q = 0; q < QB; ++q) thr_s[q] = desc ? -INFINITY : INFINITY;
 
     for (int t = 0; t < ntiles; ++t) {
       const int st = t % ns, r = t / ns;
       if (!mbar_wait(&full[st], r & 1, abort_flag, a.gflags)) break;
       const int nr = (int)min((int64_t)tr, nrows - (int64_t)t * tr);
       const uint8_t *stage = smem + (size_t)st * stage_bytes;
-      for (int rr = warp; rr < nr; rr += kBwWarps) {
-        const uint8_t *rowp = stage + (size_t)rr * row_bytes;
-        float acc[QB];
+      for (int rr = warp; rr < nr; rr += 2 * kBwWarps) {
+        const int rb = rr + kBwWarps;
+        const bool has_b = rb < nr;
+        const uint8_t *pa = stage + (size_t)rr * row_bytes;
+        const uint8_t *pb = stage + (size_t)(has_b ? rb : rr) * row_bytes;
+        // packed pairs: two partial sums per lane, FFMA2 / FADD2
+        float2 acc_a[QB], acc_b[QB];
 #pragma unroll
-        for (int q = 0; q < QB; ++q) acc[q] = 0.0f;
-        float cc = 0.0f;
+        for (int q = 0; q < QB; ++q) acc_a[q] = acc_b[q] = make_float2(0.0f, 0.0f);
+        float2 cc_a = make_float2(0.0f, 0.0f), cc_b = make_float2(0.0f, 0.0f);
 #pragma unroll
         for (int j = 0; j < kNchMax; ++j) {
           const int e0 = (j * 32 + lane) * 8;
           if (j < nch && e0 < D) {
-            float f[8];
-            decode8<W>(rowp + (size_t)e0 * W, f);
+            float2 fa[4], fb[4];
+            decode8x2<W>(pa + (size_t)e0 * W, fa);
+            decode8x2<W>(pb + (size_t)e0 * W, fb);
 #pragma unroll
             for (int q = 0; q < QB; ++q)
 #pragma unroll
-              for (int u = 0; u < 8; ++u) acc[q] = fmaf(qreg[q][j][u], f[u], acc[q]);
-            if (need_cc)
+              for (int u = 0; u < 4; ++u) {
+                acc_a[q] = __ffma2_rn(qreg[q][j][u], fa[u], acc_a[q]);
+                acc_b[q] = __ffma2_rn(qreg[q][j][u], fb[u], acc_b[q]);
+              }
+            if (CC)
 #pragma unroll
-              for (int u = 0; u < 8; ++u) cc = fmaf(f[u], f[u], cc);
+              for (int u = 0; u < 4; ++u) {
+                cc_a = __ffma2_rn(fa[u], fa[u], cc_a);
+                cc_b = __ffma2_rn(fb[u], fb[u], cc_b);
+              }
           }
         }
-#pragma unroll
-        for (int q = 0; q < QB; ++q) acc[q] = warp_sum(acc[q]);
-        if (need_cc) cc = warp_sum(cc);
-        const uint32_t row = (uint32_t)(r0 + (int64_t)t * tr + rr);
+        const float cc = CC ? pair_sum(cc_a.x + cc_a.y, cc_b.x + cc_b.y, lane) : 0.0f;
 #pragma unroll
         for (int q = 0; q < QB; ++q) {
+          const float acc = pair_sum(acc_a[q].x + acc_a[q].y, acc_b[q].x + acc_b[q].y, lane);
+          // lanes 0-15 hold row rr, lanes 16-31 row rb
+          const float sc = finish_score(a.metric, acc, cc, s, s2, qq[q], qn[q]);
+          const float sa = __shfl_sync(0xffffffffu, sc, 0);
+          const float sb = __shfl_sync(0xffffffffu, sc, 16);
           if (q >= a.B) continue;
-          const float sc = finish_score(a.metric, acc[q], cc, s, s2, qq[q], qn[q]);
-          const uint64_t key = make_key(sc, row, desc);
-          if (key < thr[q]) {
-            lists[q].insert(key, lane);
-            thr[q] = lists[q].kth(a.k);
+          if (desc ? sa > thr_s[q] : sa < thr_s[q]) {
+            lists[q].insert(make_key(sa, (uint32_t)(r0 + (int64_t)t * tr + rr), desc), lane);
+            const uint64_t kk = lists[q].kth(a.k);
+            thr_s[q] = kk == kSentinel ? (desc ? -INFINITY : INFINITY)
+                                       : rank_key32_score((uint32_t)(kk >> 32), desc);
+          }
+          if (has_b && (desc ? sb > thr_s[q] : sb < thr_s[q])) {
+            lists[q].insert(make_key(sb, (uint32_t)(r0 + (int64_t)t * tr + rb), desc), lane);
+            const uint64_t kk = lists[q].kth(a.k);
+            thr_s[q] = kk == kSentinel ? (desc ? -INFINITY : INFINITY)
+                                       : rank_key32_score((uint32_t)(kk >> 32), desc);
           }
         }
       }
@@ -216,7 +250,7 @@ __global__ void __launch_bounds__(kBwThreads, 1)
       lists[q].store(cand + ((size_t)q * kBwWarps + warp) * a.k, a.k, lane);
   }
   __syncthreads();
-  // ---------------- CTA merge of the eight warp lists, per query ----------
+  // ---------------- CTA merge of the warp lists, per query -----------------
   for (int q = 0; q < QB && q < a.B; ++q)
     rank_merge(cand + (size_t)q * kBwWarps * a.k, kBwWarps, a.k,
                a.partial + ((size_t)blockIdx.x * a.B + q) * a.k, threadIdx.x, kBwThreads);
@@ -369,6 +403,120 @@ __global__ void __launch_bounds__(kMergeThreads) topk_merge_kernel(ScoreArgs a, 
   }
 }
 
+// k-way merge of the sorted partial lists, one warp per query.  The CTA first
+// copies the candidate lists of its qpc queries to shared memory; lane l then
+// owns lists l, l + 32, ... and keeps their heads in registers; each of the k
+// steps takes the warp-wide smallest head and advances that list.  Squared L2
+// survivors are rescored in the direct form and re-sorted, as in the
+// block-sort merge above.
+constexpr int kKmWarps = 8;
+
+template <int HPL>
+__global__ void __launch_bounds__(kKmWarps * 32) topk_kmerge_kernel(ScoreArgs a, int qpc) {
+  extern __shared__ __align__(16) uint8_t ksmem[];
+  const int L = a.n_lists, k = a.k;
+  uint64_t *cand = reinterpret_cast<uint64_t *>(ksmem);            // [qpc][L][k]
+  uint64_t *outk = cand + (size_t)qpc * L * k;                       // [kKmWarps][P2]
+  const int P2 = next_pow2_dev(k);
+  const int64_t b0 = (int64_t)blockIdx.x * qpc;
+  const int64_t per_q = (int64_t)L * k;
+  for (int64_t e = threadIdx.x; e < (int64_t)qpc * per_q; e += blockDim.x) {
+    const int64_t qi = e / per_q, rem = e - qi * per_q;
+    const int64_t l = rem / k, i = rem - l * k;
+    const int64_t b = b0 + qi;
+    cand[e] = b < a.B ? a.partial[((size_t)l * a.B + b) * k + i] : kSentinel;
+  }
+  __syncthreads();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const bool desc = a.metric != LAM_METRIC_L2;
+  uint64_t *O = outk + (size_t)warp * P2;
+  for (int qi = warp; qi < qpc; qi += kKmWarps) {
+    const int64_t b = b0 + qi;
+    if (b >= a.B) break;
+    const uint64_t *C = cand + (size_t)qi * per_q;
+    int pos[HPL];
+    uint64_t head[HPL];
+#pragma unroll
+    for (int h = 0; h < HPL; ++h) {
+      const int l = lane + 32 * h;
+      pos[h] = 0;
+      head[h] = l < L ? C[(size_t)l * k] : kSentinel;
+    }
+    for (int i = 0; i < k; ++i) {
+      uint64_t m = head[0];
+      int mh = 0;
+#pragma unroll
+      for (int h = 1; h < HPL; ++h)
+        if (head[h] < m) {
+          m = head[h];
+          mh = h;
+        }
+      uint64_t gm = m;
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) {
+        const uint64_t o = __shfl_xor_sync(0xffffffffu, gm, off);
+        gm = o < gm ? o : gm;
+      }
+      const unsigned bal = __ballot_sync(0xffffffffu, m == gm);
+      if (lane == __ffs(bal) - 1) {
+#pragma unroll
+        for (int h = 0; h < HPL; ++h)
+          if (h == mh) {
+            ++pos[h];
+            head[h] = pos[h] < k ? C[(size_t)(lane + 32 * h) * k + pos[h]] : kSentinel;
+          }
+      }
+      if (lane == 0) O[i] = gm;
+    }
+    __syncwarp();
+    if (!desc) {
+      const float *q = a.queries + b * a.D;
+      for (int i = 0; i < k; ++i) {
+        const uint32_t row = (uint32_t)(O[i] & 0xffffffffu);
+        float acc = 0.0f;
+        if (row < a.N) {
+          for (int d = lane; d < a.D; d += 32) {
+            const float xh = __fmul_rn(a.s, (float)load_code(a.codes, a.width, (int64_t)row * a.D + d));
+            const float df = __fsub_rn(q[d], xh);
+            acc = fmaf(df, df, acc);
+          }
+        }
+        acc = warp_sum(acc);
+        __syncwarp();
+        if (lane == 0) O[i] = row < a.N ? make_key(acc, row, false) : kSentinel;
+        __syncwarp();
+      }
+      for (int i = k + lane; i < P2; i += 32) O[i] = kSentinel;
+      __syncwarp();
+      for (int size = 2; size <= P2; size <<= 1) {
+        for (int stride = size >> 1; stride > 0; stride >>= 1) {
+          for (int t = lane; t < P2 / 2; t += 32) {
+            const int lo = 2 * t - (t & (stride - 1));
+            const int hi = lo + stride;
+            const bool up = (lo & size) == 0;
+            const uint64_t x = O[lo], y = O[hi];
+            if ((x > y) == up) {
+              O[lo] = y;
+              O[hi] = x;
+            }
+          }
+          __syncwarp();
+        }
+      }
+    }
+    for (int i = lane; i < k; i += 32) {
+      const uint64_t key = O[i];
+      uint32_t o = (uint32_t)(key >> 32);
+      if (desc) o = ~o;
+      a.scores[b * k + i] = unord_f32(o);
+      a.ids[b * k + i] = (int64_t)(uint32_t)(key & 0xffffffffu);
+    }
+    __syncwarp();
+  }
+}
+
+constexpr size_t kKmCandBytes = 160 * 1024;
+
 inline int next_pow2(int64_t x) {
   int p = 1;
   while (p < x) p <<= 1;
@@ -397,7 +545,8 @@ int generic_ctas(int64_t B, int64_t N, int sms) {
 template <int W, int QB, int KPL>
 static cudaError_t launch_bw_t(const ScoreArgs &a, const BwShape &sh, cudaStream_t st) {
   const size_t smem = (size_t)sh.ns * sh.stage_bytes + 2 * sh.ns * sizeof(uint64_t) + 16;
-  auto kern = score_bw_kernel<W, QB, KPL>;
+  auto kern = a.metric == LAM_METRIC_IP ? score_bw_kernel<W, QB, KPL, false>
+                                        : score_bw_kernel<W, QB, KPL, true>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   kern<<<a.n_lists, kBwThreads, smem, st>>>(a, sh.tr, sh.ns, sh.stage_bytes);
@@ -407,7 +556,6 @@ static cudaError_t launch_bw_t(const ScoreArgs &a, const BwShape &sh, cudaStream
 template <int W, int QB>
 static cudaError_t launch_bw_k(const ScoreArgs &a, const BwShape &sh, cudaStream_t st) {
   if (a.k <= 32) return launch_bw_t<W, QB, 1>(a, sh, st);
-  if (a.k <= 64) return launch_bw_t<W, QB, 2>(a, sh, st);
   return launch_bw_t<W, QB, 4>(a, sh, st);
 }
 
@@ -429,7 +577,29 @@ cudaError_t launch_score_generic(const ScoreArgs &a, cudaStream_t st) {
   return cudaGetLastError();
 }
 
+template <int HPL>
+static cudaError_t launch_kmerge_t(const ScoreArgs &a, cudaStream_t st) {
+  const size_t per_q = (size_t)a.n_lists * a.k * 8;
+  int64_t qpc = (int64_t)(kKmCandBytes / per_q);
+  if (qpc > 64) qpc = 64;
+  if (qpc > a.B) qpc = a.B;
+  const size_t smem = (size_t)qpc * per_q + (size_t)kKmWarps * next_pow2(a.k) * 8;
+  auto kern = topk_kmerge_kernel<HPL>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  kern<<<(unsigned)((a.B + qpc - 1) / qpc), kKmWarps * 32, smem, st>>>(a, (int)qpc);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_topk_merge(const ScoreArgs &a, cudaStream_t st) {
+  // warp k-way merge when one query's candidates fit the shared-memory budget
+  if ((size_t)a.n_lists * a.k * 8 <= kKmCandBytes && a.n_lists <= 512) {
+    if (a.n_lists <= 32) return launch_kmerge_t<1>(a, st);
+    if (a.n_lists <= 64) return launch_kmerge_t<2>(a, st);
+    if (a.n_lists <= 128) return launch_kmerge_t<4>(a, st);
+    if (a.n_lists <= 256) return launch_kmerge_t<8>(a, st);
+    return launch_kmerge_t<16>(a, st);
+  }
   const int64_t total = (int64_t)a.n_lists * a.k;
   int P = total <= kMergeCap ? next_pow2(total) : kMergeCap;
   if (P < 64) P = 64;
