@@ -118,6 +118,44 @@ __device__ __forceinline__ void merge_candidates(RegTopK<KR> &reg, const uint2 *
   thr_s = tk == 0xffffffffu ? (desc ? -INFINITY : INFINITY) : rank_key32_score(tk, desc);
 }
 
+// ---- per-thread max-heap of k keys in shared memory -------------------------
+// Entry i of this thread's heap is H[i * stride + slot]; the root (i = 0) is
+// the largest key, i.e. the worst of the k kept.
+__device__ __forceinline__ void heap_sift_down(uint64_t *H, int n, int stride, int slot, int i,
+                                               uint64_t key) {
+  while (true) {
+    const int l = 2 * i + 1;
+    if (l >= n) break;
+    int c = l;
+    uint64_t cv = H[(size_t)l * stride + slot];
+    if (l + 1 < n) {
+      const uint64_t cr = H[(size_t)(l + 1) * stride + slot];
+      if (cr > cv) {
+        cv = cr;
+        c = l + 1;
+      }
+    }
+    if (cv <= key) break;
+    H[(size_t)i * stride + slot] = cv;
+    i = c;
+  }
+  H[(size_t)i * stride + slot] = key;
+}
+// Replaces the root (the worst key) by a better key.
+__device__ __forceinline__ void heap_replace_root(uint64_t *H, int n, int stride, int slot,
+                                                  uint64_t key) {
+  heap_sift_down(H, n, stride, slot, 0, key);
+}
+// In-place heap sort: afterwards H[0..n) ascends.
+__device__ __forceinline__ void heap_sort_ascending(uint64_t *H, int n, int stride, int slot) {
+  for (int end = n - 1; end > 0; --end) {
+    const uint64_t top = H[slot];
+    const uint64_t last = H[(size_t)end * stride + slot];
+    H[(size_t)end * stride + slot] = top;
+    heap_sift_down(H, end, stride, slot, 0, last);
+  }
+}
+
 // ---- shared-memory top-k list of one warp (any k <= kMaxK) ----
 // L[0, k) ascending; *thr mirrors L[k-1].
 __device__ __forceinline__ void smem_list_insert(uint64_t *L, int k, uint64_t key, int lane,

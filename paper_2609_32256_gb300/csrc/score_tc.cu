@@ -481,7 +481,6 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     int cnt = 0;                                // buffered candidates of this query
     if (KR == 0)
       for (int i = 0; i < k; ++i) lists[(size_t)i * kBM + m] = kSentinel;
-    uint64_t thr = kSentinel;
     for (int lt = 0; lt < ntl; ++lt) {
       const int buf = lt & 1, u = lt >> 1;
       if (!warp_wait(&accf[buf], u & 1, abort_flag, a.gflags)) break;
@@ -521,25 +520,30 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             if (__any_sync(0xffffffffu, cnt == kCBuf))
               merge_candidates(reg, cbuf, m, kBM, cnt, thr_s, desc);
           }
-        } else if (KR == 0 && qvalid) {
+        } else if (KR == 0) {
+          // k > 32: a max-heap per query in shared memory (root = the worst
+          // key kept); a candidate replaces the root and sifts down.
+          const int64_t nvalid = a.N - (row0 + c * 32);
+          uint32_t mask = 0;
 #pragma unroll
           for (int j = 0; j < 32; ++j) {
-            const int64_t row = row0 + c * 32 + j;
-            if (row < a.N) {
-              const float rf = need_cc ? ccbuf[buf * kBN + c * 32 + j] : 0.0f;
-              const float sc = tile_score(a.metric, __uint_as_float(v[j]), fq, qq, rf);
-              const uint64_t key = make_key(sc, (uint32_t)row, desc);
-              if (key < thr) {
-                int p = k - 1;
-                while (p > 0) {
-                  const uint64_t prev = lists[(size_t)(p - 1) * kBM + m];
-                  if (prev <= key) break;
-                  lists[(size_t)p * kBM + m] = prev;
-                  --p;
-                }
-                lists[(size_t)p * kBM + m] = key;
-                thr = lists[(size_t)(k - 1) * kBM + m];
-              }
+            const float rf = need_cc ? ccbuf[buf * kBN + c * 32 + j] : 0.0f;
+            const float sc = tile_score(a.metric, __uint_as_float(v[j]), fq, qq, rf);
+            mask |= (uint32_t)(desc ? sc > thr_s : sc < thr_s) << j;
+          }
+          if (!qvalid || nvalid <= 0) mask = 0;
+          else if (nvalid < 32) mask &= (1u << nvalid) - 1u;
+          while (mask != 0) {
+            const int j = __ffs(mask) - 1;
+            mask &= mask - 1;
+            const float rf = need_cc ? ccbuf[buf * kBN + c * 32 + j] : 0.0f;
+            const float sc = tile_score(a.metric, __uint_as_float(select32(v, j)), fq, qq, rf);
+            const uint64_t key = make_key(sc, (uint32_t)(row0 + c * 32 + j), desc);
+            if (key < lists[m]) {
+              heap_replace_root(lists, k, kBM, m, key);
+              const uint64_t root = lists[m];
+              thr_s = root == kSentinel ? (desc ? -INFINITY : INFINITY)
+                                        : rank_key32_score((uint32_t)(root >> 32), desc);
             }
           }
         }
@@ -557,6 +561,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         for (int i = 0; i < RK; ++i)
           if (i >= RK - k) out[i - (RK - k)] = ((uint64_t)reg.key[i] << 32) | reg.id[i];
       } else {
+        heap_sort_ascending(lists, k, kBM, m);
         for (int i = 0; i < k; ++i) out[i] = lists[(size_t)i * kBM + m];
       }
     }
