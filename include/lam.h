@@ -63,7 +63,7 @@ int32_t lam_version(void);
 /* Static text for a status code. */
 const char *lam_status_string(int32_t status);
 
-/* Bytes of device workspace lam_quantize needs (a small status block). */
+/* Bytes of device workspace lam_quantize needs (a 32-byte status block). */
 size_t lam_quantize_workspace_size(void);
 
 /*
@@ -88,10 +88,15 @@ size_t lam_quantize_workspace_size(void);
  *            NULL): the width used, s = 2*eps, and the smallest and largest
  *            code.  They are written for LAM_OK and LAM_ERR_RANGE.
  *
+ * With LAM_WIDTH_AUTO one cooperative launch speculates the width from a
+ * 1/64 sample of x, quantizes at it while measuring the exact range, and
+ * quantizes again only if the exact range needs a wider type.
+ *
  * Synchronous on `stream`: the status block is read back, because the width
  * and the range are outputs.  Errors: LAM_ERR_NONFINITE (NaN/Inf in x),
  * LAM_ERR_RANGE (a forced width, or int32, cannot hold the codes),
- * LAM_ERR_WORKSPACE (codes_bytes or the workspace is too small), LAM_ERR_CUDA.
+ * LAM_ERR_WORKSPACE (codes_bytes or the workspace is too small), LAM_ERR_TIMEOUT
+ * (a bounded device wait gave up), LAM_ERR_CUDA.
  */
 lam_status lam_quantize(const float *x, int64_t n, float eps, int32_t width_req,
                         void *codes, size_t codes_bytes, void *workspace,

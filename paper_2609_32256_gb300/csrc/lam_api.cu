@@ -177,8 +177,7 @@ lam_status lam_quantize(const float *x, int64_t n, float eps, int32_t width_req,
   if (cudaMemsetAsync(dst, 0, sizeof(QuantStatus), st) != cudaSuccess) return LAM_ERR_CUDA;
   cudaError_t e = cudaSuccess;
   if (width_req == LAM_WIDTH_AUTO) {
-    e = launch_quant_range(x, n, dst, sms, st);
-    if (e == cudaSuccess) e = launch_quantize(x, n, s, LAM_WIDTH_AUTO, codes, codes_bytes, dst, sms, st);
+    e = launch_quantize_auto_coop(x, n, s, codes, codes_bytes, dst, sms, st);
   } else if (codes != nullptr) {
     e = launch_quantize(x, n, s, width_req, codes, codes_bytes, dst, sms, st);
   } else {
@@ -189,6 +188,7 @@ lam_status lam_quantize(const float *x, int64_t n, float eps, int32_t width_req,
   if (cudaMemcpyAsync(&h, dst, sizeof(h), cudaMemcpyDeviceToHost, st) != cudaSuccess)
     return LAM_ERR_CUDA;
   if (cudaStreamSynchronize(st) != cudaSuccess) return LAM_ERR_CUDA;
+  if (h.flags & kFlagTimeout) return LAM_ERR_TIMEOUT;
   if (h.flags & kFlagNonfinite) return LAM_ERR_NONFINITE;
   float rmin = 0.0f, rmax = 0.0f;
   if (h.neg_min != 0) {

@@ -23,12 +23,16 @@ constexpr int kHeaderBytes = 256;         // status block at the head of a works
 // Wait budget of every device-side spin: ~1 s of SM clock.
 constexpr long long kWaitCycles = 2000000000LL;
 
-// Status block of lam_quantize (16 bytes, zeroed before each call).
+// Status block of lam_quantize (32 bytes, zeroed before each call).
 struct QuantStatus {
   uint32_t neg_min;   // max over inputs of ~ord(x)   (0: no finite input seen)
   uint32_t max;       // max over inputs of ord(x)
   uint32_t flags;
   uint32_t width;     // width the AUTO kernel resolved
+  uint32_t bar;       // grid barrier arrivals (AUTO kernel)
+  uint32_t s_neg_min; // the same over the sample the AUTO kernel speculates from
+  uint32_t s_max;
+  uint32_t passes;    // quantize passes the AUTO kernel made (1 or 2)
 };
 
 // ----------------------------------------------------- ordered float keys --
@@ -147,6 +151,9 @@ cudaError_t launch_quantize(const float *x, int64_t n, float s, int width_req, v
                             cudaStream_t st);
 cudaError_t launch_dequantize(const void *codes, int width, int64_t n, float s, float *out,
                               int sms, cudaStream_t st);
+cudaError_t launch_quantize_auto_coop(const float *x, int64_t n, float s, void *codes,
+                                      size_t codes_bytes, QuantStatus *status, int sms,
+                                      cudaStream_t st);
 
 struct ScoreArgs {
   const float *queries;

@@ -186,6 +186,109 @@ __global__ void __launch_bounds__(kThreads) quantize_auto_kernel(const float *__
   else quantize_body<4, false, VEC>(x, n, s, codes, st);
 }
 
+// Bounded grid barrier for a cooperative launch (every block resident):
+// block leaders count arrivals up to `target`; a wait longer than
+// kWaitCycles records a timeout and lets the block go on.
+__device__ __forceinline__ void grid_barrier(uint32_t *count, uint32_t target, uint32_t *flags) {
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    __threadfence();
+    atomicAdd(count, 1u);
+    const long long t0 = clock64();
+    while (*(volatile uint32_t *)count < target) {
+      if (clock64() - t0 > kWaitCycles) {
+        atomicOr(flags, kFlagTimeout);
+        break;
+      }
+      __nanosleep(64);
+    }
+    __threadfence();
+  }
+  __syncthreads();
+}
+
+__device__ __forceinline__ int width_of_range(uint32_t neg_min, uint32_t mx, float s) {
+  if (neg_min == 0) return 1;
+  const float xmin = unord_f32(~neg_min), xmax = unord_f32(mx);
+  const float rmin = rintf(__fdiv_rn(xmin, s)), rmax = rintf(__fdiv_rn(xmax, s));
+  if (rmin >= -128.0f && rmax <= 127.0f) return 1;
+  if (rmin >= -32768.0f && rmax <= 32767.0f) return 2;
+  if (rmin >= -2147483648.0f && rmax < 2147483648.0f) return 4;
+  return 0;
+}
+
+// Narrowest-width Q_eps in one cooperative launch.  Phase 1 takes the range
+// of a strided 1/64 sample and speculates the width from it; phase 2
+// quantizes at that width while tracking the exact range; if the exact range
+// needs a wider type (the sample missed an extreme), phase 3 quantizes again
+// at the exact width.  The sample's range lies inside the exact one, so the
+// speculation is never wider than needed and the result is always the
+// narrowest width.
+template <bool VEC>
+__global__ void __launch_bounds__(kThreads) quantize_auto_coop_kernel(
+    const float *__restrict__ x, int64_t n, float s, void *__restrict__ codes,
+    unsigned long long codes_bytes, QuantStatus *st) {
+  const uint32_t G = gridDim.x;
+  {  // phase 1: sample range
+    Range rg;
+    const int64_t tid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    const int64_t nsamp = (n + 255) / 256;  // one 4-value group per 256 values
+    for (int64_t v = tid; v < nsamp; v += stride) {
+      const int64_t i = v * 256;
+      if (VEC && i + 3 < n) {
+        const float4 t = __ldg(reinterpret_cast<const float4 *>(x + i));
+        rg.add(t.x);
+        rg.add(t.y);
+        rg.add(t.z);
+        rg.add(t.w);
+      } else {
+        for (int64_t j = i; j < i + 4 && j < n; ++j) rg.add(x[j]);
+      }
+    }
+    for (int off = 16; off > 0; off >>= 1) {
+      rg.vmin = fminf(rg.vmin, __shfl_xor_sync(0xffffffffu, rg.vmin, off));
+      rg.vmax = fmaxf(rg.vmax, __shfl_xor_sync(0xffffffffu, rg.vmax, off));
+    }
+    if ((threadIdx.x & 31) == 0 && rg.vmin <= rg.vmax) {
+      atomicMax(&st->s_neg_min, ~ord_f32(rg.vmin));
+      atomicMax(&st->s_max, ord_f32(rg.vmax));
+    }
+  }
+  grid_barrier(&st->bar, G, &st->flags);
+  const int ws = width_of_range(*(volatile uint32_t *)&st->s_neg_min,
+                                *(volatile uint32_t *)&st->s_max, s);
+  const bool write1 = codes != nullptr && ws != 0 &&
+                      (unsigned long long)n * (unsigned long long)ws <= codes_bytes;
+  // phase 2: quantize at the speculated width, tracking the exact range
+  if (write1) {
+    if (ws == 1) quantize_body<1, true, VEC>(x, n, s, codes, st);
+    else if (ws == 2) quantize_body<2, true, VEC>(x, n, s, codes, st);
+    else quantize_body<4, true, VEC>(x, n, s, codes, st);
+  } else {
+    Range rg;
+    const int64_t tid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t i = tid; i < n; i += stride) rg.add(x[i]);
+    rg.flush(st);
+  }
+  grid_barrier(&st->bar, 2 * G, &st->flags);
+  if (*(volatile uint32_t *)&st->flags & kFlagNonfinite) return;
+  const int w = width_of_range(*(volatile uint32_t *)&st->neg_min, *(volatile uint32_t *)&st->max, s);
+  const bool fits = w != 0 && (unsigned long long)n * (unsigned long long)w <= codes_bytes;
+  if (blockIdx.x == 0 && threadIdx.x == 0) {
+    st->width = (uint32_t)w;
+    st->passes = (write1 && w == ws) ? 1u : 2u;
+    if (w == 0) atomicOr(&st->flags, kFlagRange);
+    else if (codes != nullptr && !fits) atomicOr(&st->flags, kFlagWorkspace);
+  }
+  // phase 3 (rare): the exact range needs a wider type than the sample said
+  if (codes == nullptr || !fits || (write1 && w == ws)) return;
+  if (w == 1) quantize_body<1, false, VEC>(x, n, s, codes, st);
+  else if (w == 2) quantize_body<2, false, VEC>(x, n, s, codes, st);
+  else quantize_body<4, false, VEC>(x, n, s, codes, st);
+}
+
 template <int W, bool VEC>
 __global__ void __launch_bounds__(kThreads) dequantize_kernel(const void *__restrict__ codes,
                                                               int64_t n, float s,
@@ -268,6 +371,26 @@ cudaError_t launch_quantize(const float *x, int64_t n, float s, int width_req, v
   else { LAM_Q(4) }
 #undef LAM_Q
   return cudaGetLastError();
+}
+
+cudaError_t launch_quantize_auto_coop(const float *x, int64_t n, float s, void *codes,
+                                      size_t codes_bytes, QuantStatus *status, int sms,
+                                      cudaStream_t st) {
+  const bool vec = aligned16(x) && (codes == nullptr || aligned16(codes));
+  const void *kern = vec ? (const void *)quantize_auto_coop_kernel<true>
+                         : (const void *)quantize_auto_coop_kernel<false>;
+  int per_sm = 0;
+  cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, 0);
+  if (e != cudaSuccess) return e;
+  if (per_sm > kBlocksPerSm) per_sm = kBlocksPerSm;
+  if (per_sm < 1) return cudaErrorInvalidConfiguration;
+  int64_t g = (int64_t)sms * per_sm;
+  const int64_t need = (n / 4 + kThreads - 1) / kThreads + 1;
+  if (g > need) g = need;
+  unsigned long long cb = codes_bytes;
+  void *args[] = {(void *)&x, (void *)&n, (void *)&s, (void *)&codes, (void *)&cb,
+                  (void *)&status};
+  return cudaLaunchCooperativeKernel(kern, dim3((unsigned)g), dim3(kThreads), args, 0, st);
 }
 
 cudaError_t launch_dequantize(const void *codes, int width, int64_t n, float s, float *out,

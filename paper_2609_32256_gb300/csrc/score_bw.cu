@@ -581,7 +581,7 @@ template <int HPL>
 static cudaError_t launch_kmerge_t(const ScoreArgs &a, cudaStream_t st) {
   const size_t per_q = (size_t)a.n_lists * a.k * 8;
   int64_t qpc = (int64_t)(kKmCandBytes / per_q);
-  if (qpc > 64) qpc = 64;
+  if (qpc > kKmWarps) qpc = kKmWarps;  // one query per warp: spread over the SMs
   if (qpc > a.B) qpc = a.B;
   const size_t smem = (size_t)qpc * per_q + (size_t)kKmWarps * next_pow2(a.k) * 8;
   auto kern = topk_kmerge_kernel<HPL>;

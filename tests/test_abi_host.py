@@ -44,7 +44,7 @@ def test_status_strings(lib):
     assert lam.lam_status_string(0) == "ok"
     assert "invalid" in lam.lam_status_string(1)
     assert lam.lam_version() >= 100
-    assert lam.lam_quantize_workspace_size() == 16
+    assert lam.lam_quantize_workspace_size() == 32
 
 
 @pytest.mark.parametrize("n,eps,width", [

@@ -27,7 +27,7 @@ def gpu_quantize(x_np, eps, width, dev, offset=0):
     xt = torch.zeros(n + offset, dtype=torch.float32, device=dev)
     xt[offset:] = torch.from_numpy(x_np.reshape(-1)).to(dev)
     x = xt[offset:]
-    ws = torch.zeros(16, dtype=torch.uint8, device=dev)
+    ws = torch.zeros(lam.lam_quantize_workspace_size(), dtype=torch.uint8, device=dev)
     wbytes = 4 if width == 0 else width
     cbuf = torch.zeros(n * wbytes + 4 * offset, dtype=torch.uint8, device=dev)
     codes = cbuf[4 * offset:]  # aligned to any width, not to 16 bytes
@@ -101,7 +101,7 @@ def test_forced_width_overflow_reports_range(dev):
 def test_auto_codes_buffer_too_small(dev):
     x = inputs.flat_values(1000, seed=2)
     xt = torch.from_numpy(x).to(dev)
-    ws = torch.zeros(16, dtype=torch.uint8, device=dev)
+    ws = torch.zeros(lam.lam_quantize_workspace_size(), dtype=torch.uint8, device=dev)
     codes = torch.zeros(1500, dtype=torch.uint8, device=dev)  # int16 needs 2000
     st, w, *_ = lam.lam_quantize(xt, 1e-4, 0, codes, ws, raise_on_error=False)
     assert st == lam.LAM_ERR_WORKSPACE and w == 2
@@ -111,7 +111,7 @@ def test_range_only_without_codes(dev):
     x = inputs.flat_values(100000, seed=3)
     _, rmin, rmax, _ = oracle.quantize(x, 1e-4)
     xt = torch.from_numpy(x).to(dev)
-    ws = torch.zeros(16, dtype=torch.uint8, device=dev)
+    ws = torch.zeros(lam.lam_quantize_workspace_size(), dtype=torch.uint8, device=dev)
     for width in (0, 2, 4):
         st, w, _, cmin, cmax = lam.lam_quantize(xt, 1e-4, width, None, ws)
         assert st == 0 and (cmin, cmax) == (int(rmin), int(rmax))
@@ -165,3 +165,16 @@ def test_planted_chunks_widths(dev):
         oc, rmin, rmax, _ = oracle.quantize(x, eps)
         assert w == want_w == oracle.width(rmin, rmax)
         assert digest(codes.cpu().numpy()) == digest(oc.astype(NP_DT[w]))
+
+
+@pytest.mark.parametrize("outlier,width", [(300.0, 2), (40000.0, 4)])
+def test_auto_width_outlier_missed_by_sample(dev, outlier, width):
+    # AUTO speculates the width from a 1/64 sample (the first 4 of every 256
+    # values); one outlier outside the sample forces the exact-width re-pass.
+    x = inputs.flat_values((1 << 20) + 7, seed=4)
+    x[1000 * 256 + 100] = np.float32(outlier * 2 * 1e-2)  # index not sampled
+    oc, rmin, rmax, _ = oracle.quantize(x, 1e-2)
+    assert oracle.width(rmin, rmax) == width
+    st, w, _, cmin, cmax, c = gpu_quantize(x, 1e-2, 0, dev)
+    assert st == 0 and w == width and (cmin, cmax) == (int(rmin), int(rmax))
+    assert digest(c) == digest(oc.astype(NP_DT[w]))

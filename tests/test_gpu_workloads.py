@@ -70,7 +70,7 @@ def test_mem_n8388608_l2_int8_slabs(dev):
     L2 top-100 over the whole resident code matrix."""
     N, D, slab, eps, k = 8388608, 768, 1 << 20, 1e-2, 100
     codes = torch.empty((N, D), dtype=torch.int8, device=dev)
-    ws = torch.zeros(16, dtype=torch.uint8, device=dev)
+    ws = torch.zeros(lam.lam_quantize_workspace_size(), dtype=torch.uint8, device=dev)
     rng = np.random.default_rng(11)
     bound = 0
     for j in range(N // slab):
