@@ -111,14 +111,14 @@ bool make_plan(int64_t B, int64_t N, int32_t D, int32_t k, int32_t width, int32_
   }
   p->path = path;
   if (path == kPathBandwidth) p->n_lists = bandwidth_ctas(N, D, width, sms);
-  else if (path == kPathTensor) p->n_lists = tensor_splits(B, N, sms);
+  else if (path == kPathTensor) p->n_lists = tensor_plan(B, N, D, k, sms).n_lists;
   else p->n_lists = generic_ctas(B, N, sms);
   p->Bpad = (B + 127) / 128 * 128;
   p->partial_off = kHeaderBytes;
   const size_t partial = (size_t)p->n_lists * (size_t)B * (size_t)k * 8;
   p->qprep_off = align_up(p->partial_off + partial, 256);
   p->total = p->qprep_off;
-  if (path == kPathTensor) p->total += align_up(tensor_qprep_bytes(p->Bpad, D), 256);
+  if (path == kPathTensor) p->total += align_up(tensor_plan(B, N, D, k, sms).bytes, 256);
   return true;
 }
 

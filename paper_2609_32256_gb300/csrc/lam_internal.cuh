@@ -186,7 +186,15 @@ enum Path { kPathBandwidth = 0, kPathTensor = 1, kPathGeneric = 2 };
 int bandwidth_ctas(int64_t N, int D, int width, int sms);
 int tensor_splits(int64_t B, int64_t N, int sms);
 bool tensor_fits(int width, int k);  // shared memory holds >= 2 stages
-size_t tensor_qprep_bytes(int64_t Bpad, int D);
+// Tensor-path workspace (after the partial lists): [query images][query info]
+// and, for two or more query blocks, [fp16 code slab][per-row factors].
+struct TensorPlan {
+  bool pre;            // codes converted to fp16 by a separate pass
+  int64_t slab_rows;   // rows per slab (pre), else N
+  int nslabs, nsplit, n_lists;
+  size_t qinfo_off, fp16_off, rowf_off, bytes;
+};
+TensorPlan tensor_plan(int64_t B, int64_t N, int D, int k, int sms);
 int generic_ctas(int64_t B, int64_t N, int sms);
 
 }  // namespace lam

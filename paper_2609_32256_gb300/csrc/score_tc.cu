@@ -160,6 +160,12 @@ __device__ __forceinline__ float tile_score(int metric, float acc, float fq, flo
   return fmaf(fq, acc, qq + rowf);
 }
 
+__device__ __forceinline__ float warp_sum_tc(float v) {
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+  return v;
+}
+
 // v[j] for a run-time j, by a tree of selects (no local-memory indexing).
 __device__ __forceinline__ uint32_t select32(const uint32_t (&v)[32], int j) {
   uint32_t t16[16], t8[8], t4[4], t2[2];
@@ -637,6 +643,309 @@ __global__ void __launch_bounds__(256) qprep_kernel(const float *__restrict__ q,
                      : make_float4(0.f, 0.f, 0.f, 0.f);
 }
 
+
+// ===========================================================================
+// Batched path for two or more query blocks.  A separate pass converts the
+// codes once per call into fp16 rows (and the per-row score factor), so the
+// scoring kernel is a plain TMA -> tcgen05 pipeline: no conversion sits in
+// its stage loop.  Rows are processed in slabs to bound the fp16 copy.
+// ===========================================================================
+constexpr int kTc2Threads = 192;  // warp 0 producer, warp 1 MMA, warps 2-5 epilogue
+
+// codes [row_base, row_base + nrows) -> the fp16 operand image of the scoring
+// kernel: for each tile of 256 rows and each 32-wide K chunk, one contiguous
+// 16 KB block of 64-byte rows in the 64-byte swizzle (16-byte piece j of row r
+// at piece j ^ ((r >> 1) & 3)), so that one bulk copy stages it.  Rows past
+// nrows and columns past D are zero.  Also the per-row factor rowf (1/||c|| for
+// cosine, s^2 ||c||^2 for L2).  One warp per row of the padded slab.
+template <int W>
+__global__ void __launch_bounds__(256) convert_codes_kernel(const void *__restrict__ codes,
+                                                            int64_t row_base, int64_t nrows,
+                                                            int64_t nrows_pad, int D,
+                                                            uint8_t *__restrict__ out,
+                                                            float *__restrict__ rowf, int metric,
+                                                            float s, uint32_t *gflags) {
+  const int64_t r = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (r >= nrows_pad) return;
+  const bool valid = r < nrows;
+  const int nk = (D + kBK - 1) / kBK;
+  const int rr = (int)(r % kBN);
+  const int sw = (rr >> 1) & 3;
+  uint8_t *dst = out + (size_t)(r / kBN) * nk * kB16Bytes + (size_t)rr * 64;
+  const uint8_t *src = static_cast<const uint8_t *>(codes) + (row_base + r) * (int64_t)D * W;
+  float cc = 0.0f, amax = 0.0f;
+  for (int ch = lane; ch < nk * (kBK / 8); ch += 32) {
+    const int d0 = ch * 8;
+    float f[8];
+#pragma unroll
+    for (int t = 0; t < 8; ++t) f[t] = 0.0f;
+    if (valid && d0 < D) {  // D is a multiple of 16: a chunk is all in or all out
+      if (W == 1) {
+        const uint2 v = *reinterpret_cast<const uint2 *>(src + d0);
+#pragma unroll
+        for (int t = 0; t < 8; ++t) f[t] = (float)(int8_t)((t < 4 ? v.x : v.y) >> (8 * (t & 3)));
+      } else {
+        const uint4 v = *reinterpret_cast<const uint4 *>(src + d0 * 2);
+        const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int t = 0; t < 8; ++t) f[t] = (float)(int16_t)(w[t >> 1] >> (16 * (t & 1)));
+      }
+    }
+    uint32_t o[4];
+#pragma unroll
+    for (int t = 0; t < 4; ++t) {
+      amax = fmaxf(amax, fmaxf(fabsf(f[2 * t]), fabsf(f[2 * t + 1])));
+      cc = fmaf(f[2 * t], f[2 * t], fmaf(f[2 * t + 1], f[2 * t + 1], cc));
+      o[t] = h2_as_u32(__floats2half2_rn(f[2 * t], f[2 * t + 1]));
+    }
+    *reinterpret_cast<uint4 *>(dst + (size_t)(ch >> 2) * kB16Bytes + (((ch & 3) ^ sw) << 4)) =
+        make_uint4(o[0], o[1], o[2], o[3]);
+  }
+  cc = warp_sum_tc(cc);
+  if (lane == 0 && valid && metric != LAM_METRIC_IP)
+    rowf[r] = metric == LAM_METRIC_COSINE ? (cc > 0.0f ? 1.0f / sqrtf(cc) : 0.0f) : s * s * cc;
+  if (W == 2 && amax > 2048.0f) atomicOr(gflags, kFlagRange);
+}
+
+struct Tc2Layout {
+  int ns;
+  size_t lists_off, cbuf_off, bar_off, smem_bytes;
+};
+
+inline Tc2Layout tc2_layout(int k) {
+  Tc2Layout L;
+  const size_t lists = k > 32 ? (size_t)kBM * k * 8 : 0;
+  const size_t cbuf = k > 32 ? 0 : (size_t)kCBuf * kBM * 8;
+  const size_t tailb = 64 * 8 + 1024;
+  int ns = (int)((kMaxDynSmem - lists - cbuf - tailb) / kStageBytes);
+  if (ns > 6) ns = 6;
+  L.ns = ns;
+  L.lists_off = (size_t)ns * kStageBytes;
+  L.cbuf_off = L.lists_off + lists;
+  L.bar_off = L.cbuf_off + cbuf;
+  L.smem_bytes = L.bar_off + tailb;
+  return L;
+}
+
+struct Tc2Geom {
+  int ns;
+  int lists_off, cbuf_off, bar_off;
+  int64_t row_base, nrows;  // the slab
+  int list_base;            // partial-list index of this slab's split 0
+  const uint8_t *b16;       // fp16 operand image of the slab
+  const float *rowf;        // per-row factors of the slab
+};
+
+template <int KR>
+__global__ void __launch_bounds__(kTc2Threads, 1)
+    score_tc2_kernel(ScoreArgs a, Tc2Geom g) {
+  extern __shared__ uint8_t tc_smem_raw[];
+  const uint32_t base_u32 = smem_u32(tc_smem_raw);
+  uint8_t *smem = tc_smem_raw + (((base_u32 + 1023u) & ~1023u) - base_u32);
+  const int ns = g.ns;
+  uint64_t *lists = reinterpret_cast<uint64_t *>(smem + g.lists_off);
+  uint2 *cbuf = reinterpret_cast<uint2 *>(smem + g.cbuf_off);
+  uint64_t *full = reinterpret_cast<uint64_t *>(smem + g.bar_off);
+  uint64_t *empty = full + ns;
+  uint64_t *accf = empty + ns;
+  uint64_t *acce = accf + 2;
+  uint64_t *done = acce + 2;
+  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(done + 1);
+  volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int qb = blockIdx.y;
+  const int64_t n_tiles = (g.nrows + kBN - 1) / kBN;
+  const int64_t tb = (int64_t)blockIdx.x * n_tiles / gridDim.x;
+  const int64_t te = (int64_t)(blockIdx.x + 1) * n_tiles / gridDim.x;
+  const int ntl = (int)(te - tb);
+  const int nk = (a.D + kBK - 1) / kBK;
+  const bool need_cc = a.metric != LAM_METRIC_IP;
+  const uint8_t *qA = static_cast<const uint8_t *>(a.qprep);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < ns; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&accf[b], 1);
+      mbar_init(&acce[b], 128);
+    }
+    mbar_init(done, 1);
+    *abort_flag = 0;
+    fence_barrier_init();
+    fence_proxy_async_smem();
+  }
+  if (warp == 1) tmem_alloc(tmem_slot, kTmemCols);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  if (warp == 0) {
+    // ------------------------------------------------ producer -----------
+    if (lane == 0) {
+      int it = 0, issued = 0;
+      bool ok = true;
+      for (int lt = 0; lt < ntl && ok; ++lt) {
+        const int tile = (int)(tb + lt);
+        for (int kc = 0; kc < nk; ++kc, ++it) {
+          const int s = it % ns, r = it / ns;
+          if (r > 0 && !mbar_wait(&empty[s], (r - 1) & 1, abort_flag, a.gflags)) {
+            ok = false;
+            break;
+          }
+          uint8_t *st = smem + (size_t)s * kStageBytes;
+          mbar_arrive_expect_tx(&full[s], kAStage + kB16Bytes);
+          bulk_g2s(st, qA + ((size_t)qb * nk + kc) * kAStage, kAStage, &full[s]);
+          bulk_g2s(st + kAStage, g.b16 + ((size_t)tile * nk + kc) * kB16Bytes, kB16Bytes, &full[s]);
+          issued = it + 1;
+        }
+      }
+      for (int t = max(0, issued - ns); t < issued; ++t) drain_wait_tc(&full[t % ns], (t / ns) & 1);
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------ MMA issuer ---------
+    if (lane == 0) {
+      int it = 0;
+      bool ok = true;
+      for (int lt = 0; lt < ntl && ok; ++lt) {
+        const int buf = lt & 1, u = lt >> 1;
+        if (u > 0 && !mbar_wait(&acce[buf], (u - 1) & 1, abort_flag, a.gflags)) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + (uint32_t)(buf * kBN);
+        for (int kc = 0; kc < nk; ++kc, ++it) {
+          const int s = it % ns, r = it / ns;
+          if (!mbar_wait(&full[s], r & 1, abort_flag, a.gflags)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t st = smem_u32(smem + (size_t)s * kStageBytes);
+          const uint64_t ahi = desc_sw64(st), alo = desc_sw64(st + kABytes),
+                         bd = desc_sw64(st + kAStage);
+#pragma unroll
+          for (int j = 0; j < kBK / kUmmaK; ++j) {
+            const uint64_t koff = (uint64_t)((j * kUmmaK * 2) >> 4);
+            umma_f16(d_tmem, ahi + koff, bd + koff, kIdesc, (kc > 0 || j > 0) ? 1u : 0u);
+            umma_f16(d_tmem, alo + koff, bd + koff, kIdesc, 1u);
+          }
+          umma_commit(&empty[s]);
+        }
+        if (ok) umma_commit(&accf[buf]);
+      }
+      umma_commit(done);
+      drain_wait_tc(done, 0);
+    }
+  } else {
+    // ------------------------------------------------ epilogue -----------
+    // (warps 2-5: warp w may read TMEM lanes 32 (w % 4) .. 32 (w % 4) + 31)
+    const int quad = warp & 3;
+    const int m = quad * 32 + lane;
+    const int64_t qidx = (int64_t)qb * kBM + m;
+    const bool qvalid = qidx < a.B;
+    const int k = a.k;
+    const bool desc = a.metric != LAM_METRIC_L2;
+    const float s = a.s;
+    float pw = 0.0f, qn = 0.0f, qq = 0.0f;
+    if (qvalid) {
+      const float4 qi = reinterpret_cast<const float4 *>(
+          qA + (size_t)(a.Bpad / kBM) * nk * kAStage)[qidx];
+      pw = qi.x;
+      qn = qi.y;
+      qq = qi.z;
+    }
+    const float fq = a.metric == LAM_METRIC_IP ? s * pw
+                     : a.metric == LAM_METRIC_COSINE ? (qn > 0.0f ? pw / qn : 0.0f)
+                                                     : -2.0f * s * pw;
+    constexpr int RK = KR > 0 ? KR : 1;
+    RegTopK<RK> reg;
+    reg.init(k);
+    float thr_s = desc ? -INFINITY : INFINITY;
+    int cnt = 0;
+    if (KR == 0)
+      for (int i = 0; i < k; ++i) lists[(size_t)i * kBM + m] = kSentinel;
+    for (int lt = 0; lt < ntl; ++lt) {
+      const int buf = lt & 1, u = lt >> 1;
+      const int64_t row0 = (tb + lt) * kBN;  // slab-local
+      if (!warp_wait(&accf[buf], u & 1, abort_flag, a.gflags)) break;
+      tc_fence_after();
+      const uint32_t taddr = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(buf * kBN);
+#pragma unroll 1
+      for (int c = 0; c < kBN / 32; ++c) {
+        uint32_t v[32];
+        const int64_t nvalid = g.nrows - (row0 + c * 32);
+        // lane j holds the factor of row j of this chunk
+        const float rfl = need_cc && lane < nvalid ? g.rowf[row0 + c * 32 + lane] : 0.0f;
+        tmem_ld32(taddr + c * 32, v);
+        uint32_t mask = 0;
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+          const float rf = __shfl_sync(0xffffffffu, rfl, j);
+          const float sc = tile_score(a.metric, __uint_as_float(v[j]), fq, qq, rf);
+          mask |= (uint32_t)(desc ? sc > thr_s : sc < thr_s) << j;
+        }
+        if (!qvalid || nvalid <= 0) mask = 0;
+        else if (nvalid < 32) mask &= (1u << nvalid) - 1u;
+        const uint32_t grow0 = (uint32_t)(g.row_base + row0 + c * 32);  // global row id
+        if (KR > 0) {
+          while (__any_sync(0xffffffffu, mask != 0)) {
+            const int j = mask != 0 ? __ffs(mask) - 1 : 0;
+            const float rf = __shfl_sync(0xffffffffu, rfl, j);
+            if (mask != 0) {
+              mask &= mask - 1;
+              const float sc = tile_score(a.metric, __uint_as_float(select32(v, j)), fq, qq, rf);
+              cbuf[(size_t)cnt * kBM + m] = make_uint2(rank_key32(sc, desc), grow0 + j);
+              ++cnt;
+            }
+            if (__any_sync(0xffffffffu, cnt == kCBuf))
+              merge_candidates(reg, cbuf, m, kBM, cnt, thr_s, desc);
+          }
+        } else {
+          while (__any_sync(0xffffffffu, mask != 0)) {
+            const int j = mask != 0 ? __ffs(mask) - 1 : 0;
+            const float rf = __shfl_sync(0xffffffffu, rfl, j);
+            if (mask == 0) continue;
+            mask &= mask - 1;
+            const float sc = tile_score(a.metric, __uint_as_float(select32(v, j)), fq, qq, rf);
+            const uint64_t key = make_key(sc, grow0 + j, desc);
+            if (key < lists[m]) {
+              heap_replace_root(lists, k, kBM, m, key);
+              const uint64_t root = lists[m];
+              thr_s = root == kSentinel ? (desc ? -INFINITY : INFINITY)
+                                        : rank_key32_score((uint32_t)(root >> 32), desc);
+            }
+          }
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(&acce[buf]);
+      if (KR > 0 && __any_sync(0xffffffffu, cnt > 0)) merge_candidates(reg, cbuf, m, kBM, cnt, thr_s, desc);
+    }
+    if (KR > 0 && __any_sync(0xffffffffu, cnt > 0)) merge_candidates(reg, cbuf, m, kBM, cnt, thr_s, desc);
+    if (qvalid) {
+      uint64_t *out = a.partial + ((size_t)(g.list_base + blockIdx.x) * a.B + qidx) * k;
+      if (KR > 0) {
+#pragma unroll
+        for (int i = 0; i < RK; ++i)
+          if (i >= RK - k) out[i - (RK - k)] = ((uint64_t)reg.key[i] << 32) | reg.id[i];
+      } else {
+        heap_sort_ascending(lists, k, kBM, m);
+        for (int i = 0; i < k; ++i) out[i] = lists[(size_t)i * kBM + m];
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, kTmemCols);
+  }
+}
+
 typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
                                   const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
                                   const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
@@ -683,7 +992,7 @@ int gcd_i(int x, int y) {
 
 bool tensor_fits(int width, int k) {
   if (k > kTcMaxK || (width != 1 && width != 2)) return false;
-  return tc_layout(width, k).ns >= 2;
+  return tc_layout(width, k).ns >= 2 && tc2_layout(k).ns >= 2;
 }
 
 int tensor_splits(int64_t B, int64_t N, int sms) {
@@ -696,51 +1005,115 @@ int tensor_splits(int64_t B, int64_t N, int sms) {
   return (int)ns;
 }
 
-size_t tensor_qprep_bytes(int64_t Bpad, int D) {
+TensorPlan tensor_plan(int64_t B, int64_t N, int D, int k, int sms) {
+  TensorPlan p;
+  const int64_t Bpad = (B + kBM - 1) / kBM * kBM;
   const int64_t nk = (D + kBK - 1) / kBK;
-  return (size_t)(Bpad / kBM) * nk * kAStage + (size_t)Bpad * 16;
+  p.pre = Bpad / kBM >= 2;
+  p.qinfo_off = (size_t)(Bpad / kBM) * nk * kAStage;
+  size_t off = p.qinfo_off + (size_t)Bpad * 16;
+  off = (off + 255) / 256 * 256;
+  if (!p.pre) {
+    p.slab_rows = N;
+    p.nslabs = 1;
+    p.nsplit = tensor_splits(B, N, sms);
+    p.fp16_off = p.rowf_off = off;
+    p.bytes = off;
+  } else {
+    int64_t cap = ((int64_t)1 << 30) / (nk * kBK * 2) / kBN * kBN;  // ~1 GiB of fp16 rows
+    if (cap < kBN) cap = kBN;
+    p.slab_rows = N < cap ? N : cap;
+    p.nslabs = (int)((N + p.slab_rows - 1) / p.slab_rows);
+    p.nsplit = tensor_splits(B, p.slab_rows, sms);
+    p.fp16_off = off;
+    p.rowf_off = p.fp16_off + (size_t)((p.slab_rows + kBN - 1) / kBN) * nk * kB16Bytes;
+    p.bytes = p.rowf_off + (size_t)p.slab_rows * 4;
+  }
+  p.n_lists = p.nslabs * p.nsplit;
+  return p;
 }
 
 cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st) {
   if (a.k > kTcMaxK || (a.width != 1 && a.width != 2)) return cudaErrorInvalidValue;
-  const TcLayout L = tc_layout(a.width, a.k);
-  if (L.ns < 2) return cudaErrorInvalidValue;
+  const TensorPlan P = tensor_plan(a.B, a.N, a.D, a.k, a.sms);
+  if (P.n_lists != a.n_lists) return cudaErrorInvalidValue;
   uint8_t *qA = static_cast<uint8_t *>(a.qprep);
   qprep_kernel<<<(unsigned)((a.Bpad + 7) / 8), 256, 0, st>>>(a.queries, a.B, a.D, a.Bpad, qA);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
 
-  CUtensorMap cmap;
-  if (!make_map_2d(&cmap,
-                   a.width == 1 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_UINT16,
-                   a.codes, (uint64_t)a.D, (uint64_t)a.N, (uint64_t)a.D * a.width,
-                   (uint32_t)(kRawRow / a.width), kBN, CU_TENSOR_MAP_SWIZZLE_128B))
-    return cudaErrorInvalidValue;
+  if (!P.pre) {
+    const TcLayout L = tc_layout(a.width, a.k);
+    if (L.ns < 2) return cudaErrorInvalidValue;
+    CUtensorMap cmap;
+    if (!make_map_2d(&cmap,
+                     a.width == 1 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_UINT16,
+                     a.codes, (uint64_t)a.D, (uint64_t)a.N, (uint64_t)a.D * a.width,
+                     (uint32_t)(kRawRow / a.width), kBN, CU_TENSOR_MAP_SWIZZLE_128B))
+      return cudaErrorInvalidValue;
+    TcGeom g;
+    g.ns = L.ns;
+    g.nr = L.nr;
+    g.raw_off = (int)L.raw_off;
+    g.lists_off = (int)L.lists_off;
+    g.cbuf_off = (int)L.cbuf_off;
+    g.cc_off = (int)L.cc_off;
+    g.bar_off = (int)L.bar_off;
+    const dim3 grid((unsigned)a.n_lists, (unsigned)(a.Bpad / kBM));
+    auto run = [&](auto kern) -> cudaError_t {
+      cudaError_t r = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           (int)L.smem_bytes);
+      if (r != cudaSuccess) return r;
+      kern<<<grid, kTcThreads, L.smem_bytes, st>>>(cmap, a, g);
+      return cudaGetLastError();
+    };
+    if (a.width == 1) {
+      if (a.k <= 16) return run(score_tc_kernel<1, 16>);
+      if (a.k <= 32) return run(score_tc_kernel<1, 32>);
+      return run(score_tc_kernel<1, 0>);
+    }
+    if (a.k <= 16) return run(score_tc_kernel<2, 16>);
+    if (a.k <= 32) return run(score_tc_kernel<2, 32>);
+    return run(score_tc_kernel<2, 0>);
+  }
 
-  TcGeom g;
+  // two or more query blocks: convert each slab once, then the pure MMA kernel
+  const Tc2Layout L = tc2_layout(a.k);
+  if (L.ns < 2) return cudaErrorInvalidValue;
+  uint8_t *f16 = static_cast<uint8_t *>(a.qprep) + P.fp16_off;
+  float *rowf = reinterpret_cast<float *>(static_cast<uint8_t *>(a.qprep) + P.rowf_off);
+  Tc2Geom g;
   g.ns = L.ns;
-  g.nr = L.nr;
-  g.raw_off = (int)L.raw_off;
   g.lists_off = (int)L.lists_off;
   g.cbuf_off = (int)L.cbuf_off;
-  g.cc_off = (int)L.cc_off;
   g.bar_off = (int)L.bar_off;
-  const dim3 grid((unsigned)a.n_lists, (unsigned)(a.Bpad / kBM));
-  auto run = [&](auto kern) -> cudaError_t {
-    cudaError_t r = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)L.smem_bytes);
-    if (r != cudaSuccess) return r;
-    kern<<<grid, kTcThreads, L.smem_bytes, st>>>(cmap, a, g);
-    return cudaGetLastError();
-  };
-  if (a.width == 1) {
-    if (a.k <= 16) return run(score_tc_kernel<1, 16>);
-    if (a.k <= 32) return run(score_tc_kernel<1, 32>);
-    return run(score_tc_kernel<1, 0>);
+  g.b16 = f16;
+  g.rowf = rowf;
+  auto kern = a.k <= 16 ? score_tc2_kernel<16> : a.k <= 32 ? score_tc2_kernel<32> : score_tc2_kernel<0>;
+  e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)L.smem_bytes);
+  if (e != cudaSuccess) return e;
+  const dim3 grid((unsigned)P.nsplit, (unsigned)(a.Bpad / kBM));
+  for (int j = 0; j < P.nslabs; ++j) {
+    const int64_t row_base = (int64_t)j * P.slab_rows;
+    const int64_t nrows = a.N - row_base < P.slab_rows ? a.N - row_base : P.slab_rows;
+    const int64_t nrows_pad = (nrows + kBN - 1) / kBN * kBN;
+    const unsigned cg = (unsigned)((nrows_pad + 7) / 8);
+    if (a.width == 1)
+      convert_codes_kernel<1><<<cg, 256, 0, st>>>(a.codes, row_base, nrows, nrows_pad, a.D, f16,
+                                                  rowf, a.metric, a.s, a.gflags);
+    else
+      convert_codes_kernel<2><<<cg, 256, 0, st>>>(a.codes, row_base, nrows, nrows_pad, a.D, f16,
+                                                  rowf, a.metric, a.s, a.gflags);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    g.row_base = row_base;
+    g.nrows = nrows;
+    g.list_base = j * P.nsplit;
+    kern<<<grid, kTc2Threads, L.smem_bytes, st>>>(a, g);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
   }
-  if (a.k <= 16) return run(score_tc_kernel<2, 16>);
-  if (a.k <= 32) return run(score_tc_kernel<2, 32>);
-  return run(score_tc_kernel<2, 0>);
+  return cudaSuccess;
 }
 
 }  // namespace lam

@@ -62,7 +62,7 @@ def test_bandwidth_path_other_dims(dev, score_path, D):
 
 @pytest.mark.parametrize("metric", METRICS)
 @pytest.mark.parametrize("width,eps", [(1, 1e-2), (2, 1e-3), (2, 1e-4)])
-@pytest.mark.parametrize("B", [3, 16, 130])
+@pytest.mark.parametrize("B", [3, 16, 130, 500])
 def test_tensor_path(dev, score_path, metric, width, eps, B):
     score_path("tensor")
     codes, bound = make_codes(3001, 768, eps, width, seed=B)
@@ -73,10 +73,11 @@ def test_tensor_path(dev, score_path, metric, width, eps, B):
 
 @pytest.mark.parametrize("D", [16, 48, 80, 1024])
 @pytest.mark.parametrize("k", [1, 16, 17, 32, 64, 112])
-def test_tensor_path_dims_and_k(dev, score_path, D, k):
+@pytest.mark.parametrize("B", [20, 300])  # one query block; several (codes pre-converted)
+def test_tensor_path_dims_and_k(dev, score_path, D, k, B):
     score_path("tensor")
     codes, bound = make_codes(700, D, 1e-2, 1, seed=D + k)
-    q = inputs.queries(20, D, seed=k)
+    q = inputs.queries(B, D, seed=k)
     for metric in METRICS:
         check(dev, q, codes, 1, 1e-2, k, metric, bound)
 
@@ -92,12 +93,12 @@ def test_generic_path(dev, score_path, width, eps, D):
             check(dev, q, codes, width, eps, k, metric, bound)
 
 
-@pytest.mark.parametrize("path", ["bandwidth", "tensor", "generic"])
-def test_exact_ties_rank_lower_id_first(dev, score_path, path):
+@pytest.mark.parametrize("path,B", [("bandwidth", 2), ("tensor", 8), ("tensor", 136),
+                                    ("generic", 8)])
+def test_exact_ties_rank_lower_id_first(dev, score_path, path, B):
     score_path(path)
     codes, bound = make_codes(2000, 768, 1e-2, 1, dup_every=97)  # rows 0,97,194,... identical
-    q = inputs.unit_rows(2000, 768, seed=0)[:2] if path == "bandwidth" else \
-        inputs.unit_rows(2000, 768, seed=0)[:8]
+    q = inputs.unit_rows(2000, 768, seed=0)[:B]
     for metric in METRICS:
         gs, gi, os_, oi = check(dev, q, codes, 1, 1e-2, 25, metric, bound)
         # query 0 equals row 0, so the 21 copies of it lead, in id order
@@ -129,11 +130,12 @@ def test_forced_path_unsupported(dev, score_path):
     assert e.value.status == lam.LAM_ERR_UNSUPPORTED
 
 
-def test_code_bound_violation_reported(dev, score_path):
+@pytest.mark.parametrize("B", [4, 200])
+def test_code_bound_violation_reported(dev, score_path, B):
     score_path("tensor")
     codes, _ = make_codes(600, 64, 1e-4, 2)
     codes[5, 3] = 3000  # beyond what the tensor path can hold exactly
-    q = inputs.queries(4, 64, seed=2)
+    q = inputs.queries(B, 64, seed=2)
     with pytest.raises(lam.LamError) as e:
         run(dev, q, codes, 2, 1e-4, 10, oracle.IP, 2048)
     assert e.value.status == lam.LAM_ERR_RANGE
@@ -148,10 +150,11 @@ def test_k_equals_n_and_single_row(dev):
                 check(dev, q, codes, 1, 1e-2, 128, metric, bound)
 
 
-def test_zero_rows_and_zero_query_cosine(dev):
+@pytest.mark.parametrize("B", [4, 140])
+def test_zero_rows_and_zero_query_cosine(dev, B):
     codes, bound = make_codes(500, 768, 1e-2, 1)
     codes[10:20] = 0
-    q = inputs.queries(4, 768, seed=5)
+    q = inputs.queries(B, 768, seed=5)
     q[1] = 0.0
     for metric in METRICS:
         check(dev, q, codes, 1, 1e-2, 30, metric, bound)
