@@ -31,10 +31,15 @@ UNIT = "memory vectors/s"
 L2_FLUSH_BYTES = 512 << 20
 
 # DRAM bytes (read + write) of one launch of the dominant kernel, from one ncu
-# capture (profiles/score_tc_kernel_chunks_n27986_ip.md).  Reported only while
-# the kernel source is the one the counters were taken on.
-TC_TRAFFIC = {"source_sha256_16": "7c88b5c46b34d835", "bytes": 24713728,
-              "launch": "int8 codes, eps=1e-2, 27,986 x 768, 1,024 queries"}
+# capture (the profiles/ summary of that kernel).  Reported only while the
+# kernel's source file is the one the counters were taken on.
+KERNEL_TRAFFIC = {
+    "score_tc2_kernel": {"source": "score_tc.cu", "source_sha256_16": "661386ac61808ab1",
+                         "bytes": 46529024,
+                         "launch": "ncu, cold caches: int16 codes at eps=1e-4 (the fp16 operand "
+                                   "image is the same for every width), 27,986 x 768, "
+                                   "1,024 queries"},
+}
 
 
 def parse():
@@ -173,13 +178,6 @@ class Pipeline:
             self.plan.append((w, bound, lam.lam_score_topk_path(self.B, self.N, self.D, k, w, bound)))
         self.sws = torch.empty(wsz, dtype=torch.uint8, device=dev)
 
-    def launches_per_step(self):
-        n = 0
-        for (_, _, path) in self.plan:
-            n += 2 + 1  # range + quantize, dequantize
-            n += 3 if path == self.lam.PATH_TENSOR else 2  # (qprep) + score + merge
-        return n
-
     def step(self, ev=None):
         lam = self.lam
         for j, e in enumerate(self.eps_list):
@@ -264,7 +262,29 @@ def run_lam(args):
             flush.fill_(float(i))  # L2 flush between timed steps (outside the events)
             pipe.step(evs[i])
         torch.cuda.synchronize(dev)
+        # Second timed pass of the same steps for the per-kernel figures: the
+        # library brackets each launch of its quantize, dequantize and score
+        # kernels with CUDA events on the launching stream and counts every
+        # launch (kept out of the first pass, whose host-side event records
+        # would otherwise widen the step).
+        timed_kinds = {"quantize": lam.LAM_TIME_QUANTIZE,
+                       "dequantize": lam.LAM_TIME_DEQUANTIZE, "score": lam.LAM_TIME_SCORE}
+        lam.lam_timing_begin(lam.LAM_TIME_QUANTIZE | lam.LAM_TIME_DEQUANTIZE |
+                             lam.LAM_TIME_SCORE, min(args.steps * len(wl.eps) * 8, 1 << 20))
+        for i in range(args.steps):
+            flush.fill_(float(i))
+            pipe.step()
+        torch.cuda.synchronize(dev)
     barrier(world)
+    kern = {}
+    n_launch = 0
+    for name, kind in list(timed_kinds.items()) + [("aux", lam.LAM_TIME_AUX)]:
+        tot, timed, launches = lam.lam_timing_read(kind)
+        n_launch += launches
+        if name != "aux":
+            kern[name] = {"ms_total": tot, "timed": timed, "launches": launches,
+                          "ms_per_launch": tot / timed if timed else None}
+    lam.lam_timing_end()
 
     t_q = t_d = t_s = 0.0
     for i in range(args.steps):
@@ -288,28 +308,38 @@ def run_lam(args):
     hbm_peak, tc_peak, peak_kind = load_peaks()
     path_names = {0: "bandwidth", 1: "tensor", 2: "generic"}
     paths = [path_names[p] for (_, _, p) in pipe.plan]
-    traffic = None
-    try:
-        import hashlib
-        with open(os.path.join(ROOT, "paper_2609_32256_gb300", "csrc", "score_tc.cu"), "rb") as f:
-            if hashlib.sha256(f.read()).hexdigest()[:16] == TC_TRAFFIC["source_sha256_16"]:
-                traffic = TC_TRAFFIC["bytes"]
-    except OSError:
-        pass
+    sk = kern["score"]
     if all(p == "tensor" for p in paths):
-        achieved = flops / (ms_s / 1e3) / 1e12
+        kname = "score_tc2_kernel" if B > 128 else "score_tc_kernel"
+        # algorithmic work of the score kernel: 2 N D B flops per eps (one
+        # launch per row slab; the hi/lo query split doubles the MMA issue)
+        achieved = flops * args.steps / (sk["ms_total"] / 1e3) / 1e12
         roofline = {"bound": "tensor", "achieved": round(achieved, 2), "peak": tc_peak,
-                    "unit": "TFLOP/s", "frac": round(achieved / tc_peak, 4), "traffic": traffic,
-                    "traffic_launch": TC_TRAFFIC["launch"] if traffic else None,
-                    "kernel": "score_tc_kernel (timed span: lam_score_topk = query prep + "
-                              "tcgen05 score + merge)", "peak_source": peak_kind + " bf16 dense burst "
-                              "(fp16 has the same nominal rate)"}
+                    "unit": "TFLOP/s", "frac": round(achieved / tc_peak, 4),
+                    "kernel": kname, "ms_per_launch": sk["ms_per_launch"],
+                    "launches": sk["timed"],
+                    "peak_source": peak_kind + " bf16 dense burst (fp16 has the same nominal "
+                                   "rate)"}
     else:
-        sb = sum(w * nd for w in widths)
-        achieved = sb / (ms_s / 1e3) / 1e9
+        kname = "score_bw_kernel" if all(p == "bandwidth" for p in paths) else "score"
+        sb = sum(w * nd for w in widths)  # the codes, read once per eps
+        achieved = sb * args.steps / (sk["ms_total"] / 1e3) / 1e9
         roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": hbm_peak,
-                    "unit": "GB/s", "frac": round(achieved / hbm_peak, 4), "traffic": None,
-                    "kernel": "score (lam_score_topk span)", "peak_source": peak_kind + " copy"}
+                    "unit": "GB/s", "frac": round(achieved / hbm_peak, 4), "kernel": kname,
+                    "ms_per_launch": sk["ms_per_launch"], "launches": sk["timed"],
+                    "peak_source": peak_kind + " copy"}
+    roofline["traffic"] = None
+    tr = KERNEL_TRAFFIC.get(kname)
+    if tr and tr["bytes"]:
+        try:
+            import hashlib
+            with open(os.path.join(ROOT, "paper_2609_32256_gb300", "csrc", tr["source"]),
+                      "rb") as f:
+                if hashlib.sha256(f.read()).hexdigest()[:16] == tr["source_sha256_16"]:
+                    roofline["traffic"] = tr["bytes"]
+                    roofline["traffic_launch"] = tr["launch"]
+        except OSError:
+            pass
 
     # end to end: host (pinned) inputs, copies inside the timed region
     x_h = x.cpu().pin_memory()
@@ -355,14 +385,24 @@ def run_lam(args):
                        "l2": "flushed between timed steps (512 MB write, outside the events)"},
             "breakdown": {
                 "quantize_ms": ms_q, "quantize_gbs_algorithmic": q_bytes / (ms_q / 1e3) / 1e9,
-                "quantize_note": "lam_quantize span: range pass + quantize + status read-back",
+                "quantize_note": "lam_quantize span: status clear + quantize + status read-back",
                 "dequantize_ms": ms_d, "dequantize_gbs": d_bytes / (ms_d / 1e3) / 1e9,
                 "score_ms": ms_s, "score_vectors_per_s": wl.n * ne / (ms_s / 1e3),
-                "score_tflops": flops / (ms_s / 1e3) / 1e12},
+                "score_tflops": flops / (ms_s / 1e3) / 1e12,
+                "kernels": {
+                    "quantize": dict(kern["quantize"], gbs_algorithmic=(
+                        q_bytes / (kern["quantize"]["ms_total"] / args.steps / 1e3) / 1e9
+                        if kern["quantize"]["ms_total"] else None)),
+                    "dequantize": dict(kern["dequantize"], gbs_algorithmic=(
+                        d_bytes / (kern["dequantize"]["ms_total"] / args.steps / 1e3) / 1e9
+                        if kern["dequantize"]["ms_total"] else None)),
+                    "score": kern["score"]}},
             "roofline": roofline,
             "cpu_baseline": cpu,
             "e2e": e2e,
-            "gpu_launches": pipe.launches_per_step() * args.steps,
+            "gpu_launches": n_launch,
+            "gpu_launches_note": "counted by the library over the K steps of the per-kernel "
+                                 "pass (the same launches as the headline pass)",
             "clocks": sampler.summary(),
         }
         print(json.dumps(out))

@@ -88,15 +88,16 @@ size_t lam_quantize_workspace_size(void);
  *            NULL): the width used, s = 2*eps, and the smallest and largest
  *            code.  They are written for LAM_OK and LAM_ERR_RANGE.
  *
- * With LAM_WIDTH_AUTO one cooperative launch speculates the width from a
- * 1/64 sample of x, quantizes at it while measuring the exact range, and
- * quantizes again only if the exact range needs a wider type.
+ * With LAM_WIDTH_AUTO one launch speculates the width from a fixed sample
+ * of x (four values at each of 64 evenly spaced positions), quantizes at
+ * it while measuring the exact range, and a second launch quantizes again
+ * only if the exact range needs a wider type.
  *
  * Synchronous on `stream`: the status block is read back, because the width
  * and the range are outputs.  Errors: LAM_ERR_NONFINITE (NaN/Inf in x),
  * LAM_ERR_RANGE (a forced width, or int32, cannot hold the codes),
- * LAM_ERR_WORKSPACE (codes_bytes or the workspace is too small), LAM_ERR_TIMEOUT
- * (a bounded device wait gave up), LAM_ERR_CUDA.
+ * LAM_ERR_WORKSPACE (codes_bytes or the workspace is too small), LAM_ERR_CUDA.
+ * (LAM_ERR_TIMEOUT is not returned by this call.)
  */
 lam_status lam_quantize(const float *x, int64_t n, float eps, int32_t width_req,
                         void *codes, size_t codes_bytes, void *workspace,
@@ -177,6 +178,41 @@ lam_status lam_score_topk_status(const void *workspace, lam_stream_t stream,
  */
 int32_t lam_score_topk_path(int64_t B, int64_t N, int32_t D, int32_t k,
                             int32_t width, int32_t code_bound);
+
+/*
+ * Kernel timing (measurement support, not part of the method).
+ *
+ * lam_timing_begin(mask, capacity) makes the library bracket each launch of
+ * the kernels selected by `mask` with a pair of CUDA events recorded on the
+ * launching stream, for at most `capacity` launches in total, and count every
+ * launch of its kernels by kind.  Kinds:
+ *   LAM_TIME_QUANTIZE    the Q_eps kernel of lam_quantize
+ *   LAM_TIME_DEQUANTIZE  the kernel of lam_dequantize
+ *   LAM_TIME_SCORE       the fused score + top-k kernel of lam_score_topk
+ *                        (one launch per row slab)
+ *   LAM_TIME_AUX         every other kernel (query preparation, operand
+ *                        conversion, range pass, list merge)
+ * The events are created here (no allocation happens later on the timed
+ * path).  Intended for one host thread driving one device; a later begin
+ * replaces the earlier state.  Errors: LAM_ERR_INVALID for mask outside
+ * 1..15 or capacity outside 0..1048576; LAM_ERR_CUDA if event creation fails.
+ *
+ * lam_timing_read(kind, total_ms, timed, launches) waits for the recorded
+ * events of one kind (a single bit of the mask) and returns the summed device
+ * time of its bracketed launches, how many were bracketed, and how many were
+ * launched since begin.  Any output pointer may be NULL.
+ *
+ * lam_timing_end() stops timing and destroys the events.
+ */
+#define LAM_TIME_QUANTIZE 1
+#define LAM_TIME_DEQUANTIZE 2
+#define LAM_TIME_SCORE 4
+#define LAM_TIME_AUX 8
+
+lam_status lam_timing_begin(int32_t mask, int64_t capacity);
+lam_status lam_timing_read(int32_t kind, double *total_ms, int64_t *timed,
+                           int64_t *launches);
+lam_status lam_timing_end(void);
 
 /*
  * lam_score_topk_noalloc -- lam_score_topk for callers that cannot allocate

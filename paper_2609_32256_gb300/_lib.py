@@ -56,6 +56,9 @@ def load():
         "lam_score_topk_path": (i32, [i64, i64, i32, i32, i32, i32]),
         "lam_score_topk_noalloc": (i32, [vp, i64, vp, i32, i64, i32, f32, i32, i32, i32, vp,
                                          vp, vp]),
+        "lam_timing_begin": (i32, [i32, i64]),
+        "lam_timing_read": (i32, [i32, P(ctypes.c_double), P(i64), P(i64)]),
+        "lam_timing_end": (i32, []),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -163,3 +166,24 @@ def lam_score_topk_noalloc(queries, codes, width, N, D, eps, code_bound, k, metr
                                        int(metric), _ptr(scores), _ptr(ids),
                                        _stream(stream, queries.device))
     _check(st, "lam_score_topk_noalloc")
+
+
+LAM_TIME_QUANTIZE, LAM_TIME_DEQUANTIZE, LAM_TIME_SCORE, LAM_TIME_AUX = 1, 2, 4, 8
+
+
+def lam_timing_begin(mask, capacity) -> None:
+    """Bracket launches of the kernel kinds in `mask` with CUDA events (at most
+    `capacity` launches) and count all launches by kind."""
+    _check(load().lam_timing_begin(int(mask), int(capacity)), "lam_timing_begin")
+
+
+def lam_timing_read(kind):
+    """(summed device ms of the bracketed launches, bracketed count, launch count)."""
+    tot, timed, launches = ctypes.c_double(0), ctypes.c_int64(0), ctypes.c_int64(0)
+    _check(load().lam_timing_read(int(kind), ctypes.byref(tot), ctypes.byref(timed),
+                                  ctypes.byref(launches)), "lam_timing_read")
+    return tot.value, timed.value, launches.value
+
+
+def lam_timing_end() -> None:
+    _check(load().lam_timing_end(), "lam_timing_end")

@@ -5,6 +5,9 @@
 #include <stdlib.h>
 #include <string.h>
 
+#include <mutex>
+#include <vector>
+
 #include "lam_internal.cuh"
 
 namespace {
@@ -124,6 +127,58 @@ bool make_plan(int64_t B, int64_t N, int32_t D, int32_t k, int32_t width, int32_
 
 }  // namespace
 
+namespace lam {
+namespace {
+
+// Event pairs around selected kernel launches (lam_timing_*).
+struct Timing {
+  std::mutex mu;
+  int mask = 0;
+  std::vector<cudaEvent_t> ev;  // 2 per bracketed launch
+  std::vector<int> kind;        // kind of each bracketed launch
+  int64_t cap = 0, used = 0;
+  int64_t launches[4] = {0, 0, 0, 0};
+  bool open = false;  // a begin without its end
+};
+Timing g_timing;
+
+int kind_index(int kind) {
+  return kind == LAM_TIME_QUANTIZE ? 0 : kind == LAM_TIME_DEQUANTIZE ? 1
+         : kind == LAM_TIME_SCORE  ? 2 : 3;
+}
+
+void timing_release() {
+  for (cudaEvent_t e : g_timing.ev) cudaEventDestroy(e);
+  g_timing.ev.clear();
+  g_timing.kind.clear();
+  g_timing.cap = g_timing.used = 0;
+  g_timing.mask = 0;
+  g_timing.open = false;
+  for (int64_t &c : g_timing.launches) c = 0;
+}
+
+}  // namespace
+
+void timing_launch_begin(int kind, cudaStream_t st) {
+  std::lock_guard<std::mutex> lk(g_timing.mu);
+  if (g_timing.mask == 0) return;
+  ++g_timing.launches[kind_index(kind)];
+  if (!(g_timing.mask & kind) || g_timing.used >= g_timing.cap) return;
+  cudaEventRecord(g_timing.ev[2 * g_timing.used], st);
+  g_timing.open = true;
+}
+
+void timing_launch_end(int kind, cudaStream_t st) {
+  std::lock_guard<std::mutex> lk(g_timing.mu);
+  if (!g_timing.open || !(g_timing.mask & kind)) return;
+  cudaEventRecord(g_timing.ev[2 * g_timing.used + 1], st);
+  g_timing.kind.push_back(kind);
+  ++g_timing.used;
+  g_timing.open = false;
+}
+
+}  // namespace lam
+
 extern "C" {
 
 int32_t lam_version(void) { return 100; }
@@ -176,18 +231,36 @@ lam_status lam_quantize(const float *x, int64_t n, float eps, int32_t width_req,
   QuantStatus *dst = static_cast<QuantStatus *>(workspace);
   if (cudaMemsetAsync(dst, 0, sizeof(QuantStatus), st) != cudaSuccess) return LAM_ERR_CUDA;
   cudaError_t e = cudaSuccess;
+  const int tkind = (width_req == LAM_WIDTH_AUTO || codes != nullptr) ? LAM_TIME_QUANTIZE
+                                                                       : LAM_TIME_AUX;
+  timing_launch_begin(tkind, st);
   if (width_req == LAM_WIDTH_AUTO) {
-    e = launch_quantize_auto_coop(x, n, s, codes, codes_bytes, dst, sms, st);
+    e = launch_quantize_auto(x, n, s, codes, codes_bytes, dst, sms, st);
   } else if (codes != nullptr) {
     e = launch_quantize(x, n, s, width_req, codes, codes_bytes, dst, sms, st);
   } else {
     e = launch_quant_range(x, n, dst, sms, st);
   }
+  timing_launch_end(tkind, st);
   if (e != cudaSuccess) return LAM_ERR_CUDA;
   QuantStatus h;
   if (cudaMemcpyAsync(&h, dst, sizeof(h), cudaMemcpyDeviceToHost, st) != cudaSuccess)
     return LAM_ERR_CUDA;
   if (cudaStreamSynchronize(st) != cudaSuccess) return LAM_ERR_CUDA;
+  if (width_req == LAM_WIDTH_AUTO && codes != nullptr && h.passes == 2 &&
+      !(h.flags & (kFlagTimeout | kFlagNonfinite | kFlagRange | kFlagWorkspace)) &&
+      (h.width == 1 || h.width == 2 || h.width == 4)) {
+    // the width speculated from the sample was too narrow: quantize again
+    timing_launch_begin(LAM_TIME_QUANTIZE, st);
+    e = launch_quantize(x, n, s, (int)h.width, codes, codes_bytes, dst, sms, st);
+    timing_launch_end(LAM_TIME_QUANTIZE, st);
+    if (e != cudaSuccess) return LAM_ERR_CUDA;
+    const uint32_t width_resolved = h.width;
+    if (cudaMemcpyAsync(&h, dst, sizeof(h), cudaMemcpyDeviceToHost, st) != cudaSuccess)
+      return LAM_ERR_CUDA;
+    if (cudaStreamSynchronize(st) != cudaSuccess) return LAM_ERR_CUDA;
+    h.width = width_resolved;
+  }
   if (h.flags & kFlagTimeout) return LAM_ERR_TIMEOUT;
   if (h.flags & kFlagNonfinite) return LAM_ERR_NONFINITE;
   float rmin = 0.0f, rmax = 0.0f;
@@ -223,10 +296,11 @@ lam_status lam_dequantize(const void *codes, int32_t width, int64_t n, float sca
     return LAM_ERR_INVALID;
   const int sms = device_sms();
   if (sms <= 0) return LAM_ERR_CUDA;
-  if (launch_dequantize(codes, width, n, scale, out, sms, reinterpret_cast<cudaStream_t>(stream)) !=
-      cudaSuccess)
-    return LAM_ERR_CUDA;
-  return LAM_OK;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  timing_launch_begin(LAM_TIME_DEQUANTIZE, st);
+  const cudaError_t e = launch_dequantize(codes, width, n, scale, out, sms, st);
+  timing_launch_end(LAM_TIME_DEQUANTIZE, st);
+  return e == cudaSuccess ? LAM_OK : LAM_ERR_CUDA;
 }
 
 size_t lam_score_topk_workspace_size(int64_t B, int64_t N, int32_t D, int32_t k, int32_t width,
@@ -319,6 +393,55 @@ lam_status lam_score_topk_status(const void *workspace, lam_stream_t stream, int
   if (flags & kFlagTimeout) *status_out = LAM_ERR_TIMEOUT;
   else if (flags & kFlagRange) *status_out = LAM_ERR_RANGE;
   else *status_out = LAM_OK;
+  return LAM_OK;
+}
+
+
+lam_status lam_timing_begin(int32_t mask, int64_t capacity) {
+  if (mask < 1 || mask > 15 || capacity < 0 || capacity > (1 << 20)) return LAM_ERR_INVALID;
+  std::lock_guard<std::mutex> lk(lam::g_timing.mu);
+  lam::timing_release();
+  lam::g_timing.ev.reserve((size_t)capacity * 2);
+  for (int64_t i = 0; i < capacity * 2; ++i) {
+    cudaEvent_t e = nullptr;
+    if (cudaEventCreate(&e) != cudaSuccess) {
+      lam::timing_release();
+      return LAM_ERR_CUDA;
+    }
+    lam::g_timing.ev.push_back(e);
+  }
+  lam::g_timing.kind.reserve((size_t)capacity);
+  lam::g_timing.cap = capacity;
+  lam::g_timing.mask = mask;
+  return LAM_OK;
+}
+
+lam_status lam_timing_read(int32_t kind, double *total_ms, int64_t *timed, int64_t *launches) {
+  if (kind != LAM_TIME_QUANTIZE && kind != LAM_TIME_DEQUANTIZE && kind != LAM_TIME_SCORE &&
+      kind != LAM_TIME_AUX)
+    return LAM_ERR_INVALID;
+  std::lock_guard<std::mutex> lk(lam::g_timing.mu);
+  double tot = 0.0;
+  int64_t cnt = 0;
+  for (int64_t i = 0; i < lam::g_timing.used; ++i) {
+    if (lam::g_timing.kind[(size_t)i] != kind) continue;
+    if (cudaEventSynchronize(lam::g_timing.ev[2 * i + 1]) != cudaSuccess) return LAM_ERR_CUDA;
+    float ms = 0.0f;
+    if (cudaEventElapsedTime(&ms, lam::g_timing.ev[2 * i], lam::g_timing.ev[2 * i + 1]) !=
+        cudaSuccess)
+      return LAM_ERR_CUDA;
+    tot += ms;
+    ++cnt;
+  }
+  if (total_ms) *total_ms = tot;
+  if (timed) *timed = cnt;
+  if (launches) *launches = lam::g_timing.launches[lam::kind_index(kind)];
+  return LAM_OK;
+}
+
+lam_status lam_timing_end(void) {
+  std::lock_guard<std::mutex> lk(lam::g_timing.mu);
+  lam::timing_release();
   return LAM_OK;
 }
 

@@ -29,10 +29,10 @@ struct QuantStatus {
   uint32_t max;       // max over inputs of ord(x)
   uint32_t flags;
   uint32_t width;     // width the AUTO kernel resolved
-  uint32_t bar;       // grid barrier arrivals (AUTO kernel)
-  uint32_t s_neg_min; // the same over the sample the AUTO kernel speculates from
-  uint32_t s_max;
-  uint32_t passes;    // quantize passes the AUTO kernel made (1 or 2)
+  uint32_t bar;       // blocks of the AUTO kernel that have finished
+  uint32_t s_neg_min; // (unused)
+  uint32_t s_max;     // width the AUTO kernel speculated from its sample
+  uint32_t passes;    // 1: codes written at the resolved width; 2: a second pass is needed
 };
 
 // ----------------------------------------------------- ordered float keys --
@@ -151,9 +151,11 @@ cudaError_t launch_quantize(const float *x, int64_t n, float s, int width_req, v
                             cudaStream_t st);
 cudaError_t launch_dequantize(const void *codes, int width, int64_t n, float s, float *out,
                               int sms, cudaStream_t st);
-cudaError_t launch_quantize_auto_coop(const float *x, int64_t n, float s, void *codes,
-                                      size_t codes_bytes, QuantStatus *status, int sms,
-                                      cudaStream_t st);
+// AUTO width: one launch; if the status ends with passes == 2 the caller
+// quantizes again with launch_quantize at the resolved width.
+cudaError_t launch_quantize_auto(const float *x, int64_t n, float s, void *codes,
+                                 size_t codes_bytes, QuantStatus *status, int sms,
+                                 cudaStream_t st);
 
 struct ScoreArgs {
   const float *queries;
@@ -195,6 +197,10 @@ struct TensorPlan {
   size_t qinfo_off, fp16_off, rowf_off, bytes;
 };
 TensorPlan tensor_plan(int64_t B, int64_t N, int D, int k, int sms);
+
+// Launch bracketing for lam_timing_* (no-ops unless timing is on for `kind`).
+void timing_launch_begin(int kind, cudaStream_t st);
+void timing_launch_end(int kind, cudaStream_t st);
 int generic_ctas(int64_t B, int64_t N, int sms);
 
 }  // namespace lam

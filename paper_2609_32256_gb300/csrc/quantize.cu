@@ -30,19 +30,44 @@ struct Range {
       nonfinite = 1;
     }
   }
-  // Warp-reduce, then one atomic per warp into the status block.
-  __device__ __forceinline__ void flush(QuantStatus *st) {
+  // Block-reduce (every thread of the block calls this), then one thread
+  // folds the block's range into the status block, with an atomic only where
+  // it would change it: thousands of blocks otherwise queue on two words.
+  __device__ __forceinline__ void flush(QuantStatus *st) { flush_to(&st->neg_min, &st->max, &st->flags); }
+  // The block's range, in thread 0 (every thread of the block calls this).
+  __device__ __forceinline__ void block_reduce() {
+    __shared__ float s_min[kThreads / 32], s_max[kThreads / 32];
+    __shared__ uint32_t s_nf[kThreads / 32];
     for (int off = 16; off > 0; off >>= 1) {
       vmin = fminf(vmin, __shfl_xor_sync(0xffffffffu, vmin, off));
       vmax = fmaxf(vmax, __shfl_xor_sync(0xffffffffu, vmax, off));
       nonfinite |= __shfl_xor_sync(0xffffffffu, nonfinite, off);
     }
+    const int w = threadIdx.x >> 5;
     if ((threadIdx.x & 31) == 0) {
-      if (vmin <= vmax) {
-        atomicMax(&st->neg_min, ~ord_f32(vmin));
-        atomicMax(&st->max, ord_f32(vmax));
+      s_min[w] = vmin;
+      s_max[w] = vmax;
+      s_nf[w] = nonfinite;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      for (int i = 1; i < (int)(blockDim.x >> 5); ++i) {
+        vmin = fminf(vmin, s_min[i]);
+        vmax = fmaxf(vmax, s_max[i]);
+        nonfinite |= s_nf[i];
       }
-      if (nonfinite) atomicOr(&st->flags, kFlagNonfinite);
+    }
+    __syncthreads();
+  }
+  __device__ __forceinline__ void flush_to(uint32_t *neg_min, uint32_t *mx, uint32_t *flags) {
+    block_reduce();
+    if (threadIdx.x == 0) {
+      if (vmin <= vmax) {
+        const uint32_t a = ~ord_f32(vmin), b = ord_f32(vmax);
+        if (a > *(volatile uint32_t *)neg_min) atomicMax(neg_min, a);
+        if (b > *(volatile uint32_t *)mx) atomicMax(mx, b);
+      }
+      if (nonfinite) atomicOr(flags, kFlagNonfinite);
     }
   }
 };
@@ -54,29 +79,53 @@ __device__ __forceinline__ void store_code(void *codes, int64_t i, int32_t c) {
   if (W == 4) reinterpret_cast<int32_t *>(codes)[i] = c;
 }
 
-// Packs 16/W codes into one 16-byte word (two's-complement truncation).
+// Four codes of width W packed into one W*4-byte word (two's complement).
 template <int W>
-__device__ __forceinline__ uint4 pack(const int32_t *c) {
-  uint4 o;
-  if (W == 1) {
-    uint32_t w[4];
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      uint32_t lo = __byte_perm(c[4 * j], c[4 * j + 1], 0x0040);
-      uint32_t hi = __byte_perm(c[4 * j + 2], c[4 * j + 3], 0x0040);
-      w[j] = __byte_perm(lo, hi, 0x5410);
-    }
-    o = make_uint4(w[0], w[1], w[2], w[3]);
-  } else if (W == 2) {
-    o = make_uint4(__byte_perm(c[0], c[1], 0x5410), __byte_perm(c[2], c[3], 0x5410),
-                   __byte_perm(c[4], c[5], 0x5410), __byte_perm(c[6], c[7], 0x5410));
-  } else {
-    o = make_uint4(c[0], c[1], c[2], c[3]);
+struct Pack4;
+template <>
+struct Pack4<1> {
+  using T = uint32_t;
+  __device__ __forceinline__ static T pack(const int32_t *c) {
+    return __byte_perm(__byte_perm(c[0], c[1], 0x0040), __byte_perm(c[2], c[3], 0x0040), 0x5410);
   }
-  return o;
-}
+  __device__ __forceinline__ static void unpack(T u, int32_t *c) {
+#pragma unroll
+    for (int e = 0; e < 4; ++e) c[e] = (int32_t)(int8_t)(u >> (8 * e));
+  }
+};
+template <>
+struct Pack4<2> {
+  using T = uint2;
+  __device__ __forceinline__ static T pack(const int32_t *c) {
+    return make_uint2(__byte_perm(c[0], c[1], 0x5410), __byte_perm(c[2], c[3], 0x5410));
+  }
+  __device__ __forceinline__ static void unpack(T u, int32_t *c) {
+    c[0] = (int32_t)(int16_t)u.x;
+    c[1] = (int32_t)(int16_t)(u.x >> 16);
+    c[2] = (int32_t)(int16_t)u.y;
+    c[3] = (int32_t)(int16_t)(u.y >> 16);
+  }
+};
+template <>
+struct Pack4<4> {
+  using T = uint4;
+  __device__ __forceinline__ static T pack(const int32_t *c) {
+    return make_uint4((uint32_t)c[0], (uint32_t)c[1], (uint32_t)c[2], (uint32_t)c[3]);
+  }
+  __device__ __forceinline__ static void unpack(T u, int32_t *c) {
+    c[0] = (int32_t)u.x;
+    c[1] = (int32_t)u.y;
+    c[2] = (int32_t)u.z;
+    c[3] = (int32_t)u.w;
+  }
+};
+
+constexpr int kUnroll = 4;  // independent 4-value groups in flight per thread
 
 // Quantizes x[0, n) into codes of width W.  VEC: x and codes 16-byte aligned.
+// Each thread takes groups of four values (one 16-byte load, one 4W-byte
+// store) and a warp kUnroll * 32 consecutive groups per iteration, so every
+// warp access is contiguous.
 template <int W, bool TRACK, bool VEC>
 __device__ __forceinline__ void quantize_body(const float *__restrict__ x, int64_t n, float s,
                                               void *__restrict__ codes, QuantStatus *st) {
@@ -85,29 +134,34 @@ __device__ __forceinline__ void quantize_body(const float *__restrict__ x, int64
   Range rg;
   int64_t done = 0;
   if (VEC) {
-    constexpr int EPT = 16 / W;  // elements per 16-byte store
-    const int64_t nvec = n / EPT;
+    using T = typename Pack4<W>::T;
+    const int64_t ng = n / 4;
     const float4 *xv = reinterpret_cast<const float4 *>(x);
-    uint4 *cv = reinterpret_cast<uint4 *>(codes);
-    for (int64_t v = tid; v < nvec; v += stride) {
-      float f[EPT];
+    T *cv = reinterpret_cast<T *>(codes);
+    // a warp takes kUnroll * 32 consecutive groups per iteration
+    const int lane = threadIdx.x & 31;
+    const int64_t gw = tid >> 5, nw = stride >> 5;
+    for (int64_t g0 = gw * (32 * kUnroll) + lane; g0 < ng; g0 += nw * (32 * kUnroll)) {
+      float4 t[kUnroll];
 #pragma unroll
-      for (int j = 0; j < EPT / 4; ++j) {
-        float4 t = __ldg(xv + v * (EPT / 4) + j);
-        f[4 * j] = t.x;
-        f[4 * j + 1] = t.y;
-        f[4 * j + 2] = t.z;
-        f[4 * j + 3] = t.w;
-      }
-      int32_t c[EPT];
+      for (int u = 0; u < kUnroll; ++u)
+        if (g0 + u * 32 < ng) t[u] = __ldg(xv + g0 + u * 32);
 #pragma unroll
-      for (int e = 0; e < EPT; ++e) {
-        c[e] = q_code(f[e], s);
-        if (TRACK) rg.add(f[e]);
+      for (int u = 0; u < kUnroll; ++u) {
+        const int64_t g = g0 + u * 32;
+        if (g < ng) {
+          const float f[4] = {t[u].x, t[u].y, t[u].z, t[u].w};
+          int32_t c[4];
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            c[e] = q_code(f[e], s);
+            if (TRACK) rg.add(f[e]);
+          }
+          cv[g] = Pack4<W>::pack(c);
+        }
       }
-      cv[v] = pack<W>(c);
     }
-    done = nvec * EPT;
+    done = ng * 4;
   }
   for (int64_t i = done + tid; i < n; i += stride) {
     float f = x[i];
@@ -155,58 +209,8 @@ __global__ void __launch_bounds__(kThreads) range_kernel(const float *__restrict
   rg.flush(st);
 }
 
-// Narrowest width from the range the range pass left in *st; 0 if not int32.
-__device__ __forceinline__ int resolve_width(const QuantStatus *st, float s) {
-  if (st->neg_min == 0) return 1;  // no finite value
-  float xmin = unord_f32(~st->neg_min), xmax = unord_f32(st->max);
-  float rmin = rintf(__fdiv_rn(xmin, s)), rmax = rintf(__fdiv_rn(xmax, s));
-  if (rmin >= -128.0f && rmax <= 127.0f) return 1;
-  if (rmin >= -32768.0f && rmax <= 32767.0f) return 2;
-  if (rmin >= -2147483648.0f && rmax < 2147483648.0f) return 4;
-  return 0;
-}
-
-template <bool VEC>
-__global__ void __launch_bounds__(kThreads) quantize_auto_kernel(const float *__restrict__ x,
-                                                                 int64_t n, float s,
-                                                                 void *__restrict__ codes,
-                                                                 unsigned long long codes_bytes,
-                                                                 QuantStatus *st) {
-  if (st->flags & kFlagNonfinite) return;
-  const int w = resolve_width(st, s);
-  const bool fits = w != 0 && (unsigned long long)n * (unsigned long long)w <= codes_bytes;
-  if (blockIdx.x == 0 && threadIdx.x == 0) {
-    st->width = (uint32_t)w;
-    if (w == 0) atomicOr(&st->flags, kFlagRange);
-    else if (codes != nullptr && !fits) atomicOr(&st->flags, kFlagWorkspace);
-  }
-  if (codes == nullptr || !fits) return;
-  if (w == 1) quantize_body<1, false, VEC>(x, n, s, codes, st);
-  else if (w == 2) quantize_body<2, false, VEC>(x, n, s, codes, st);
-  else quantize_body<4, false, VEC>(x, n, s, codes, st);
-}
-
-// Bounded grid barrier for a cooperative launch (every block resident):
-// block leaders count arrivals up to `target`; a wait longer than
-// kWaitCycles records a timeout and lets the block go on.
-__device__ __forceinline__ void grid_barrier(uint32_t *count, uint32_t target, uint32_t *flags) {
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    __threadfence();
-    atomicAdd(count, 1u);
-    const long long t0 = clock64();
-    while (*(volatile uint32_t *)count < target) {
-      if (clock64() - t0 > kWaitCycles) {
-        atomicOr(flags, kFlagTimeout);
-        break;
-      }
-      __nanosleep(64);
-    }
-    __threadfence();
-  }
-  __syncthreads();
-}
-
+// Narrowest code width for the range (neg_min, mx) of the status block
+// (neg_min == 0: nothing finite seen); 0 if not even int32 holds it.
 __device__ __forceinline__ int width_of_range(uint32_t neg_min, uint32_t mx, float s) {
   if (neg_min == 0) return 1;
   const float xmin = unord_f32(~neg_min), xmax = unord_f32(mx);
@@ -217,25 +221,27 @@ __device__ __forceinline__ int width_of_range(uint32_t neg_min, uint32_t mx, flo
   return 0;
 }
 
-// Narrowest-width Q_eps in one cooperative launch.  Phase 1 takes the range
-// of a strided 1/64 sample and speculates the width from it; phase 2
-// quantizes at that width while tracking the exact range; if the exact range
-// needs a wider type (the sample missed an extreme), phase 3 quantizes again
-// at the exact width.  The sample's range lies inside the exact one, so the
-// speculation is never wider than needed and the result is always the
-// narrowest width.
+// Narrowest-width Q_eps in one launch with no grid-wide wait.  Every block
+// first takes the range of the same fixed sample of x (kSample groups of four
+// values spread evenly over the array; small, because every block reads the
+// same lines), so all blocks speculate the same width; each then quantizes its share at that width while tracking the exact
+// range, and the last block to finish resolves the exact width.  The sample's
+// range lies inside the exact one, so the guess is never too wide; when it is
+// too narrow (the sample missed an extreme) the status says so (passes = 2)
+// and the host quantizes again at the exact width.
+constexpr int kSample = 64;
+
 template <bool VEC>
-__global__ void __launch_bounds__(kThreads) quantize_auto_coop_kernel(
+__global__ void __launch_bounds__(kThreads) quantize_auto_kernel(
     const float *__restrict__ x, int64_t n, float s, void *__restrict__ codes,
     unsigned long long codes_bytes, QuantStatus *st) {
-  const uint32_t G = gridDim.x;
-  {  // phase 1: sample range
+  __shared__ int s_ws;
+  __shared__ bool s_last;
+  {
     Range rg;
-    const int64_t tid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-    const int64_t nsamp = (n + 255) / 256;  // one 4-value group per 256 values
-    for (int64_t v = tid; v < nsamp; v += stride) {
-      const int64_t i = v * 256;
+    const int64_t groups = n / 4;
+    for (int j = threadIdx.x; j < kSample; j += blockDim.x) {
+      const int64_t i = 4 * (int64_t)((unsigned long long)j * (unsigned long long)groups / kSample);
       if (VEC && i + 3 < n) {
         const float4 t = __ldg(reinterpret_cast<const float4 *>(x + i));
         rg.add(t.x);
@@ -243,24 +249,17 @@ __global__ void __launch_bounds__(kThreads) quantize_auto_coop_kernel(
         rg.add(t.z);
         rg.add(t.w);
       } else {
-        for (int64_t j = i; j < i + 4 && j < n; ++j) rg.add(x[j]);
+        for (int64_t k = i; k < i + 4 && k < n; ++k) rg.add(x[k]);
       }
     }
-    for (int off = 16; off > 0; off >>= 1) {
-      rg.vmin = fminf(rg.vmin, __shfl_xor_sync(0xffffffffu, rg.vmin, off));
-      rg.vmax = fmaxf(rg.vmax, __shfl_xor_sync(0xffffffffu, rg.vmax, off));
-    }
-    if ((threadIdx.x & 31) == 0 && rg.vmin <= rg.vmax) {
-      atomicMax(&st->s_neg_min, ~ord_f32(rg.vmin));
-      atomicMax(&st->s_max, ord_f32(rg.vmax));
-    }
+    rg.block_reduce();
+    if (threadIdx.x == 0)
+      s_ws = rg.vmin <= rg.vmax ? width_of_range(~ord_f32(rg.vmin), ord_f32(rg.vmax), s) : 1;
+    __syncthreads();
   }
-  grid_barrier(&st->bar, G, &st->flags);
-  const int ws = width_of_range(*(volatile uint32_t *)&st->s_neg_min,
-                                *(volatile uint32_t *)&st->s_max, s);
+  const int ws = s_ws;
   const bool write1 = codes != nullptr && ws != 0 &&
                       (unsigned long long)n * (unsigned long long)ws <= codes_bytes;
-  // phase 2: quantize at the speculated width, tracking the exact range
   if (write1) {
     if (ws == 1) quantize_body<1, true, VEC>(x, n, s, codes, st);
     else if (ws == 2) quantize_body<2, true, VEC>(x, n, s, codes, st);
@@ -272,21 +271,23 @@ __global__ void __launch_bounds__(kThreads) quantize_auto_coop_kernel(
     for (int64_t i = tid; i < n; i += stride) rg.add(x[i]);
     rg.flush(st);
   }
-  grid_barrier(&st->bar, 2 * G, &st->flags);
-  if (*(volatile uint32_t *)&st->flags & kFlagNonfinite) return;
-  const int w = width_of_range(*(volatile uint32_t *)&st->neg_min, *(volatile uint32_t *)&st->max, s);
-  const bool fits = w != 0 && (unsigned long long)n * (unsigned long long)w <= codes_bytes;
-  if (blockIdx.x == 0 && threadIdx.x == 0) {
-    st->width = (uint32_t)w;
-    st->passes = (write1 && w == ws) ? 1u : 2u;
-    if (w == 0) atomicOr(&st->flags, kFlagRange);
-    else if (codes != nullptr && !fits) atomicOr(&st->flags, kFlagWorkspace);
+  // the block's range updates are in; count it, and let the last block resolve
+  if (threadIdx.x == 0) {
+    __threadfence();
+    s_last = atomicAdd(&st->bar, 1u) == gridDim.x - 1;
   }
-  // phase 3 (rare): the exact range needs a wider type than the sample said
-  if (codes == nullptr || !fits || (write1 && w == ws)) return;
-  if (w == 1) quantize_body<1, false, VEC>(x, n, s, codes, st);
-  else if (w == 2) quantize_body<2, false, VEC>(x, n, s, codes, st);
-  else quantize_body<4, false, VEC>(x, n, s, codes, st);
+  __syncthreads();
+  if (!s_last || threadIdx.x != 0) return;
+  __threadfence();
+  const uint32_t nm = *(volatile uint32_t *)&st->neg_min, mx = *(volatile uint32_t *)&st->max;
+  st->s_max = (uint32_t)ws;
+  if (*(volatile uint32_t *)&st->flags & kFlagNonfinite) return;
+  const int w = width_of_range(nm, mx, s);
+  st->width = (uint32_t)w;
+  st->passes = (write1 && w == ws) ? 1u : 2u;
+  if (w == 0) atomicOr(&st->flags, kFlagRange);
+  else if (codes != nullptr && (unsigned long long)n * (unsigned long long)w > codes_bytes)
+    atomicOr(&st->flags, kFlagWorkspace);
 }
 
 template <int W, bool VEC>
@@ -297,30 +298,30 @@ __global__ void __launch_bounds__(kThreads) dequantize_kernel(const void *__rest
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   int64_t done = 0;
   if (VEC) {
-    constexpr int EPT = 16 / W;
-    const int64_t nvec = n / EPT;
-    const uint4 *cv = reinterpret_cast<const uint4 *>(codes);
+    using T = typename Pack4<W>::T;
+    const int64_t ng = n / 4;
+    const T *cv = reinterpret_cast<const T *>(codes);
     float4 *ov = reinterpret_cast<float4 *>(out);
-    for (int64_t v = tid; v < nvec; v += stride) {
-      const uint4 u = __ldg(cv + v);
-      float f[EPT];
+    // a warp takes kUnroll * 32 consecutive groups per iteration
+    const int lane = threadIdx.x & 31;
+    const int64_t gw = tid >> 5, nw = stride >> 5;
+    for (int64_t g0 = gw * (32 * kUnroll) + lane; g0 < ng; g0 += nw * (32 * kUnroll)) {
+      T u4[kUnroll];
 #pragma unroll
-      for (int e = 0; e < EPT; ++e) {
-        constexpr int PER = 4 / W;  // codes per 32-bit word
-        const int j = e / PER;
-        const uint32_t wj = j == 0 ? u.x : (j == 1 ? u.y : (j == 2 ? u.z : u.w));
-        const int sh = (e % PER) * 8 * W;
-        int32_t c;
-        if (W == 1) c = (int32_t)(int8_t)(wj >> sh);
-        else if (W == 2) c = (int32_t)(int16_t)(wj >> sh);
-        else c = (int32_t)wj;
-        f[e] = __fmul_rn(s, (float)c);
+      for (int u = 0; u < kUnroll; ++u)
+        if (g0 + u * 32 < ng) u4[u] = __ldg(cv + g0 + u * 32);
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) {
+        const int64_t g = g0 + u * 32;
+        if (g < ng) {
+          int32_t c[4];
+          Pack4<W>::unpack(u4[u], c);
+          ov[g] = make_float4(__fmul_rn(s, (float)c[0]), __fmul_rn(s, (float)c[1]),
+                              __fmul_rn(s, (float)c[2]), __fmul_rn(s, (float)c[3]));
+        }
       }
-#pragma unroll
-      for (int j = 0; j < EPT / 4; ++j)
-        ov[v * (EPT / 4) + j] = make_float4(f[4 * j], f[4 * j + 1], f[4 * j + 2], f[4 * j + 3]);
     }
-    done = nvec * EPT;
+    done = ng * 4;
   }
   for (int64_t i = done + tid; i < n; i += stride) {
     int32_t c;
@@ -356,12 +357,7 @@ cudaError_t launch_quantize(const float *x, int64_t n, float s, int width_req, v
                             size_t codes_bytes, QuantStatus *status, int sms,
                             cudaStream_t st) {
   const bool vec = aligned16(x) && (codes == nullptr || aligned16(codes));
-  if (width_req == LAM_WIDTH_AUTO) {
-    const int g = grid_for(vec ? n / 4 + 1 : n, sms);
-    if (vec) quantize_auto_kernel<true><<<g, kThreads, 0, st>>>(x, n, s, codes, codes_bytes, status);
-    else quantize_auto_kernel<false><<<g, kThreads, 0, st>>>(x, n, s, codes, codes_bytes, status);
-    return cudaGetLastError();
-  }
+  if (width_req == LAM_WIDTH_AUTO) return cudaErrorInvalidValue;  // AUTO: launch_quantize_auto
   const int g = grid_for(vec ? n / (16 / width_req) + 1 : n, sms);
 #define LAM_Q(W)                                                                      \
   if (vec) quantize_forced_kernel<W, true><<<g, kThreads, 0, st>>>(x, n, s, codes, status); \
@@ -373,24 +369,15 @@ cudaError_t launch_quantize(const float *x, int64_t n, float s, int width_req, v
   return cudaGetLastError();
 }
 
-cudaError_t launch_quantize_auto_coop(const float *x, int64_t n, float s, void *codes,
-                                      size_t codes_bytes, QuantStatus *status, int sms,
-                                      cudaStream_t st) {
+cudaError_t launch_quantize_auto(const float *x, int64_t n, float s, void *codes,
+                                 size_t codes_bytes, QuantStatus *status, int sms,
+                                 cudaStream_t st) {
   const bool vec = aligned16(x) && (codes == nullptr || aligned16(codes));
-  const void *kern = vec ? (const void *)quantize_auto_coop_kernel<true>
-                         : (const void *)quantize_auto_coop_kernel<false>;
-  int per_sm = 0;
-  cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, 0);
-  if (e != cudaSuccess) return e;
-  if (per_sm > kBlocksPerSm) per_sm = kBlocksPerSm;
-  if (per_sm < 1) return cudaErrorInvalidConfiguration;
-  int64_t g = (int64_t)sms * per_sm;
-  const int64_t need = (n / 4 + kThreads - 1) / kThreads + 1;
-  if (g > need) g = need;
-  unsigned long long cb = codes_bytes;
-  void *args[] = {(void *)&x, (void *)&n, (void *)&s, (void *)&codes, (void *)&cb,
-                  (void *)&status};
-  return cudaLaunchCooperativeKernel(kern, dim3((unsigned)g), dim3(kThreads), args, 0, st);
+  const int g = grid_for(vec ? n / 4 + 1 : n, sms);
+  const unsigned long long cb = codes_bytes;
+  if (vec) quantize_auto_kernel<true><<<g, kThreads, 0, st>>>(x, n, s, codes, cb, status);
+  else quantize_auto_kernel<false><<<g, kThreads, 0, st>>>(x, n, s, codes, cb, status);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_dequantize(const void *codes, int width, int64_t n, float s, float *out,

@@ -549,7 +549,9 @@ static cudaError_t launch_bw_t(const ScoreArgs &a, const BwShape &sh, cudaStream
                                         : score_bw_kernel<W, QB, KPL, true>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
+  timing_launch_begin(LAM_TIME_SCORE, st);
   kern<<<a.n_lists, kBwThreads, smem, st>>>(a, sh.tr, sh.ns, sh.stage_bytes);
+  timing_launch_end(LAM_TIME_SCORE, st);
   return cudaGetLastError();
 }
 
@@ -573,7 +575,9 @@ cudaError_t launch_score_generic(const ScoreArgs &a, cudaStream_t st) {
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   dim3 grid(a.n_lists, (unsigned)(a.B < 65535 ? a.B : 65535));
+  timing_launch_begin(LAM_TIME_SCORE, st);
   score_generic_kernel<<<grid, kGenWarps * 32, smem, st>>>(a);
+  timing_launch_end(LAM_TIME_SCORE, st);
   return cudaGetLastError();
 }
 
@@ -587,7 +591,9 @@ static cudaError_t launch_kmerge_t(const ScoreArgs &a, cudaStream_t st) {
   auto kern = topk_kmerge_kernel<HPL>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
+  timing_launch_begin(LAM_TIME_AUX, st);
   kern<<<(unsigned)((a.B + qpc - 1) / qpc), kKmWarps * 32, smem, st>>>(a, (int)qpc);
+  timing_launch_end(LAM_TIME_AUX, st);
   return cudaGetLastError();
 }
 
@@ -608,7 +614,9 @@ cudaError_t launch_topk_merge(const ScoreArgs &a, cudaStream_t st) {
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   const int threads = P / 2 < 32 ? 32 : (P / 2 > kMergeThreads ? kMergeThreads : P / 2);
+  timing_launch_begin(LAM_TIME_AUX, st);
   topk_merge_kernel<<<(unsigned)a.B, threads, smem, st>>>(a, P);
+  timing_launch_end(LAM_TIME_AUX, st);
   return cudaGetLastError();
 }
 

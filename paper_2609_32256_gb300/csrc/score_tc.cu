@@ -1038,7 +1038,9 @@ cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st) {
   const TensorPlan P = tensor_plan(a.B, a.N, a.D, a.k, a.sms);
   if (P.n_lists != a.n_lists) return cudaErrorInvalidValue;
   uint8_t *qA = static_cast<uint8_t *>(a.qprep);
+  timing_launch_begin(LAM_TIME_AUX, st);
   qprep_kernel<<<(unsigned)((a.Bpad + 7) / 8), 256, 0, st>>>(a.queries, a.B, a.D, a.Bpad, qA);
+  timing_launch_end(LAM_TIME_AUX, st);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
 
@@ -1064,7 +1066,9 @@ cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st) {
       cudaError_t r = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                            (int)L.smem_bytes);
       if (r != cudaSuccess) return r;
+      timing_launch_begin(LAM_TIME_SCORE, st);
       kern<<<grid, kTcThreads, L.smem_bytes, st>>>(cmap, a, g);
+      timing_launch_end(LAM_TIME_SCORE, st);
       return cudaGetLastError();
     };
     if (a.width == 1) {
@@ -1098,18 +1102,22 @@ cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st) {
     const int64_t nrows = a.N - row_base < P.slab_rows ? a.N - row_base : P.slab_rows;
     const int64_t nrows_pad = (nrows + kBN - 1) / kBN * kBN;
     const unsigned cg = (unsigned)((nrows_pad + 7) / 8);
+    timing_launch_begin(LAM_TIME_AUX, st);
     if (a.width == 1)
       convert_codes_kernel<1><<<cg, 256, 0, st>>>(a.codes, row_base, nrows, nrows_pad, a.D, f16,
                                                   rowf, a.metric, a.s, a.gflags);
     else
       convert_codes_kernel<2><<<cg, 256, 0, st>>>(a.codes, row_base, nrows, nrows_pad, a.D, f16,
                                                   rowf, a.metric, a.s, a.gflags);
+    timing_launch_end(LAM_TIME_AUX, st);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     g.row_base = row_base;
     g.nrows = nrows;
     g.list_base = j * P.nsplit;
+    timing_launch_begin(LAM_TIME_SCORE, st);
     kern<<<grid, kTc2Threads, L.smem_bytes, st>>>(a, g);
+    timing_launch_end(LAM_TIME_SCORE, st);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }

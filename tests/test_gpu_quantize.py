@@ -169,8 +169,9 @@ def test_planted_chunks_widths(dev):
 
 @pytest.mark.parametrize("outlier,width", [(300.0, 2), (40000.0, 4)])
 def test_auto_width_outlier_missed_by_sample(dev, outlier, width):
-    # AUTO speculates the width from a 1/64 sample (the first 4 of every 256
-    # values); one outlier outside the sample forces the exact-width re-pass.
+    # AUTO speculates the width from a fixed sample (four values at each of
+    # 64 evenly spaced positions: here x[16384 j .. 16384 j + 3]); one outlier
+    # outside the sample forces the exact-width second pass.
     x = inputs.flat_values((1 << 20) + 7, seed=4)
     x[1000 * 256 + 100] = np.float32(outlier * 2 * 1e-2)  # index not sampled
     oc, rmin, rmax, _ = oracle.quantize(x, 1e-2)
