@@ -123,13 +123,16 @@ class ClockSampler:
                 "samples": len(rows)}
 
 
-def dist_setup(args):
+def dist_setup(args, backend=None):
+    """Rank geometry from the torchrun environment; joins the process group
+    when there is more than one rank (NCCL for the GPU arm, gloo otherwise)."""
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
     if world > 1:
         import torch.distributed as dist
-        backend = "nccl" if args.impl == "lam" else "gloo"
+        if backend is None:
+            backend = "nccl" if args.impl == "lam" else "gloo"
         dist.init_process_group(backend=backend)
     return world, rank, local
 
@@ -148,6 +151,14 @@ def barrier(world):
     if world > 1:
         import torch.distributed as dist
         dist.barrier()
+
+
+def aggregate_replicas(ms_step_local, units_per_step, world, device=None):
+    """Replicas only: every rank runs the whole workload on its own GPU, so the
+    job's step time is the slowest rank's and its throughput counts the units
+    of all ranks.  Returns (ms_per_step, units per second)."""
+    ms = max_over_ranks(ms_step_local, world, device)
+    return ms, units_per_step * world / (ms / 1e3)
 
 
 # ----------------------------------------------------------------- lam arm --
@@ -293,10 +304,8 @@ def run_lam(args):
             t_q += e[0].elapsed_time(e[1])
             t_d += e[1].elapsed_time(e[2])
             t_s += e[2].elapsed_time(e[3])
-    ms_step = (t_q + t_d + t_s) / args.steps
-    ms_step = max_over_ranks(ms_step, world, dev)
     units_per_step = wl.n * ne
-    value = units_per_step * world / (ms_step / 1e3)
+    ms_step, value = aggregate_replicas((t_q + t_d + t_s) / args.steps, units_per_step, world, dev)
 
     # per-stage figures (rank-local)
     nd = wl.n * wl.d
