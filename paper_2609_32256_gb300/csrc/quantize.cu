@@ -7,6 +7,9 @@
 // (__float2int_rn), the same operations the host uses to resolve the width.
 #include "lam_internal.cuh"
 
+#include <map>
+#include <mutex>
+
 namespace lam {
 
 namespace {
@@ -334,9 +337,28 @@ __global__ void __launch_bounds__(kThreads) dequantize_kernel(const void *__rest
 
 inline bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
-inline int grid_for(int64_t work_items, int sms) {
+// Resident blocks per SM of a kernel at kThreads threads (registers decide
+// it), looked up once per kernel.
+int resident_blocks(const void *kern) {
+  static std::mutex mu;
+  static std::map<const void *, int> cache;
+  std::lock_guard<std::mutex> lk(mu);
+  auto it = cache.find(kern);
+  if (it != cache.end()) return it->second;
+  int b = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&b, kern, kThreads, 0) != cudaSuccess || b < 1)
+    b = 1;
+  if (b > kBlocksPerSm) b = kBlocksPerSm;
+  cache[kern] = b;
+  return b;
+}
+
+// One wave of resident blocks (or fewer, for little work): the grid-stride
+// loops then split the array evenly with no second wave.
+template <typename K>
+int grid_for(K kern, int64_t work_items, int sms) {
   int64_t blocks = (work_items + kThreads - 1) / kThreads;
-  int64_t cap = (int64_t)sms * kBlocksPerSm;
+  const int64_t cap = (int64_t)sms * resident_blocks(reinterpret_cast<const void *>(kern));
   if (blocks > cap) blocks = cap;
   if (blocks < 1) blocks = 1;
   return (int)blocks;
@@ -347,9 +369,8 @@ inline int grid_for(int64_t work_items, int sms) {
 cudaError_t launch_quant_range(const float *x, int64_t n, QuantStatus *status, int sms,
                                cudaStream_t st) {
   const bool vec = aligned16(x);
-  const int g = grid_for(vec ? n / 16 + 1 : n, sms);
-  if (vec) range_kernel<true><<<g, kThreads, 0, st>>>(x, n, status);
-  else range_kernel<false><<<g, kThreads, 0, st>>>(x, n, status);
+  auto kern = vec ? range_kernel<true> : range_kernel<false>;
+  kern<<<grid_for(kern, vec ? n / 16 + 1 : n, sms), kThreads, 0, st>>>(x, n, status);
   return cudaGetLastError();
 }
 
@@ -358,14 +379,10 @@ cudaError_t launch_quantize(const float *x, int64_t n, float s, int width_req, v
                             cudaStream_t st) {
   const bool vec = aligned16(x) && (codes == nullptr || aligned16(codes));
   if (width_req == LAM_WIDTH_AUTO) return cudaErrorInvalidValue;  // AUTO: launch_quantize_auto
-  const int g = grid_for(vec ? n / (16 / width_req) + 1 : n, sms);
-#define LAM_Q(W)                                                                      \
-  if (vec) quantize_forced_kernel<W, true><<<g, kThreads, 0, st>>>(x, n, s, codes, status); \
-  else quantize_forced_kernel<W, false><<<g, kThreads, 0, st>>>(x, n, s, codes, status);
-  if (width_req == 1) { LAM_Q(1) }
-  else if (width_req == 2) { LAM_Q(2) }
-  else { LAM_Q(4) }
-#undef LAM_Q
+  auto kern = width_req == 1 ? (vec ? quantize_forced_kernel<1, true> : quantize_forced_kernel<1, false>)
+              : width_req == 2 ? (vec ? quantize_forced_kernel<2, true> : quantize_forced_kernel<2, false>)
+                               : (vec ? quantize_forced_kernel<4, true> : quantize_forced_kernel<4, false>);
+  kern<<<grid_for(kern, vec ? n / 4 + 1 : n, sms), kThreads, 0, st>>>(x, n, s, codes, status);
   return cudaGetLastError();
 }
 
@@ -373,24 +390,19 @@ cudaError_t launch_quantize_auto(const float *x, int64_t n, float s, void *codes
                                  size_t codes_bytes, QuantStatus *status, int sms,
                                  cudaStream_t st) {
   const bool vec = aligned16(x) && (codes == nullptr || aligned16(codes));
-  const int g = grid_for(vec ? n / 4 + 1 : n, sms);
+  auto kern = vec ? quantize_auto_kernel<true> : quantize_auto_kernel<false>;
   const unsigned long long cb = codes_bytes;
-  if (vec) quantize_auto_kernel<true><<<g, kThreads, 0, st>>>(x, n, s, codes, cb, status);
-  else quantize_auto_kernel<false><<<g, kThreads, 0, st>>>(x, n, s, codes, cb, status);
+  kern<<<grid_for(kern, vec ? n / 4 + 1 : n, sms), kThreads, 0, st>>>(x, n, s, codes, cb, status);
   return cudaGetLastError();
 }
 
 cudaError_t launch_dequantize(const void *codes, int width, int64_t n, float s, float *out,
                               int sms, cudaStream_t st) {
   const bool vec = aligned16(codes) && aligned16(out);
-  const int g = grid_for(vec ? n / (16 / width) + 1 : n, sms);
-#define LAM_D(W)                                                                   \
-  if (vec) dequantize_kernel<W, true><<<g, kThreads, 0, st>>>(codes, n, s, out);   \
-  else dequantize_kernel<W, false><<<g, kThreads, 0, st>>>(codes, n, s, out);
-  if (width == 1) { LAM_D(1) }
-  else if (width == 2) { LAM_D(2) }
-  else { LAM_D(4) }
-#undef LAM_D
+  auto kern = width == 1 ? (vec ? dequantize_kernel<1, true> : dequantize_kernel<1, false>)
+              : width == 2 ? (vec ? dequantize_kernel<2, true> : dequantize_kernel<2, false>)
+                           : (vec ? dequantize_kernel<4, true> : dequantize_kernel<4, false>);
+  kern<<<grid_for(kern, vec ? n / 4 + 1 : n, sms), kThreads, 0, st>>>(codes, n, s, out);
   return cudaGetLastError();
 }
 
