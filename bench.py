@@ -501,11 +501,13 @@ def run_kernels(args):
     codes = torch.empty(n * 4, dtype=torch.uint8, device=dev)
     out = torch.empty(n, dtype=torch.float32, device=dev)
 
-    def timed(fn):
+    def timed(fn, kind):
+        """(mean call span ms, mean device ms of the call's `kind` kernel launches)."""
         for i in range(3):
             flush.fill_(float(i))
             fn()
         tot = 0.0
+        lam.lam_timing_begin(kind, args.reps * 64)
         for i in range(args.reps):
             flush.fill_(float(i))
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -514,7 +516,9 @@ def run_kernels(args):
             e1.record()
             torch.cuda.synchronize(dev)
             tot += e0.elapsed_time(e1)
-        return tot / args.reps
+        k_ms, _, _ = lam.lam_timing_read(kind)
+        lam.lam_timing_end()
+        return tot / args.reps, k_ms / args.reps
 
     res = {"workload": wl.name, "n_values": n, "quantize": [], "dequantize": [], "score": []}
     hbm, tc_peak, kind = load_peaks()
@@ -524,17 +528,24 @@ def run_kernels(args):
         _, w, sc, cmin, cmax = lam.lam_quantize(x, e, 0, None, ws)
         wq = args.width if args.width > 0 else (wl.width or w)
         widths[e] = (wq, sc, max(-cmin, cmax))
-        ms_auto = timed(lambda: lam.lam_quantize(x, e, 0, codes, ws))
-        ms_forced = timed(lambda: lam.lam_quantize(x, e, wq, codes, ws))
-        gbs = (4 + wq) * n / (ms_forced / 1e3) / 1e9
+        ms_auto, k_auto = timed(lambda: lam.lam_quantize(x, e, 0, codes, ws),
+                                lam.LAM_TIME_QUANTIZE)
+        ms_forced, k_forced = timed(lambda: lam.lam_quantize(x, e, wq, codes, ws),
+                                    lam.LAM_TIME_QUANTIZE)
+        qb = (4 + wq) * n
         res["quantize"].append({"eps": e, "width": wq, "ms_auto_span": ms_auto,
-                                "ms_forced_span": ms_forced, "gbs_forced_span": gbs,
-                                "frac_of_hbm": gbs / hbm})
+                                "ms_auto_kernel": k_auto, "ms_forced_span": ms_forced,
+                                "ms_forced_kernel": k_forced,
+                                "gbs_auto_kernel": qb / (k_auto / 1e3) / 1e9,
+                                "frac_of_hbm_auto_kernel": qb / (k_auto / 1e3) / 1e9 / hbm,
+                                "gbs_forced_kernel": qb / (k_forced / 1e3) / 1e9,
+                                "frac_of_hbm_forced_kernel": qb / (k_forced / 1e3) / 1e9 / hbm})
         lam.lam_quantize(x, e, wq, codes, ws)
-        ms_d = timed(lambda: lam.lam_dequantize(codes, wq, n, sc, out))
-        gbd = (wq + 4) * n / (ms_d / 1e3) / 1e9
-        res["dequantize"].append({"eps": e, "width": wq, "ms": ms_d, "gbs": gbd,
-                                  "frac_of_hbm": gbd / hbm})
+        ms_d, k_d = timed(lambda: lam.lam_dequantize(codes, wq, n, sc, out),
+                          lam.LAM_TIME_DEQUANTIZE)
+        gbd = (wq + 4) * n / (k_d / 1e3) / 1e9
+        res["dequantize"].append({"eps": e, "width": wq, "ms_span": ms_d, "ms_kernel": k_d,
+                                  "gbs_kernel": gbd, "frac_of_hbm_kernel": gbd / hbm})
     if wl.batches and wl.d > 1:
         e = eps_list[0]
         wq, sc, bound = widths[e]
@@ -548,16 +559,18 @@ def run_kernels(args):
             s_ = torch.empty((B, wl.k), dtype=torch.float32, device=dev)
             i_ = torch.empty((B, wl.k), dtype=torch.int64, device=dev)
             path = lam.lam_score_topk_path(B, N, wl.d, wl.k, wq, bound)
-            ms = timed(lambda: lam.lam_score_topk(q, codes, wq, N, wl.d, e, bound, wl.k, wl.metric,
-                                                  s_, i_, sws))
+            ms, k_s = timed(lambda: lam.lam_score_topk(q, codes, wq, N, wl.d, e, bound, wl.k,
+                                                       wl.metric, s_, i_, sws),
+                            lam.LAM_TIME_SCORE)
             code_bytes = N * wl.d * wq
             fl = 2.0 * N * wl.d * B
             res["score"].append({"B": B, "path": ["bandwidth", "tensor", "generic"][path],
-                                 "ms_span": ms, "vectors_per_s": N / (ms / 1e3),
-                                 "code_gbs": code_bytes / (ms / 1e3) / 1e9,
-                                 "frac_of_hbm": code_bytes / (ms / 1e3) / 1e9 / hbm,
-                                 "tflops": fl / (ms / 1e3) / 1e12,
-                                 "frac_of_tensor": fl / (ms / 1e3) / 1e12 / tc_peak})
+                                 "ms_span": ms, "ms_kernel": k_s,
+                                 "vectors_per_s_span": N / (ms / 1e3),
+                                 "code_gbs_kernel": code_bytes / (k_s / 1e3) / 1e9,
+                                 "frac_of_hbm_kernel": code_bytes / (k_s / 1e3) / 1e9 / hbm,
+                                 "tflops_kernel": fl / (k_s / 1e3) / 1e12,
+                                 "frac_of_tensor_kernel": fl / (k_s / 1e3) / 1e12 / tc_peak})
     res["peaks"] = {"hbm_gbs": hbm, "bf16_tflops": tc_peak, "kind": kind}
     print(json.dumps(res))
 

@@ -118,6 +118,21 @@ __device__ __forceinline__ void merge_candidates(RegTopK<KR> &reg, const uint2 *
   thr_s = tk == 0xffffffffu ? (desc ? -INFINITY : INFINITY) : rank_key32_score(tk, desc);
 }
 
+// k-th largest of G register values (1 <= k <= G): the smallest value that
+// fewer than k values exceed.  O(G^2) compares, no stores into v.
+template <int G>
+__device__ __forceinline__ float kth_largest(const float (&v)[G], int k) {
+  float r = INFINITY;
+#pragma unroll
+  for (int i = 0; i < G; ++i) {
+    int above = 0;
+#pragma unroll
+    for (int j = 0; j < G; ++j) above += v[j] > v[i] ? 1 : 0;
+    if (above < k) r = fminf(r, v[i]);
+  }
+  return r;
+}
+
 // ---- per-thread max-heap of k keys in shared memory -------------------------
 // Entry i of this thread's heap is H[i * stride + slot]; the root (i = 0) is
 // the largest key, i.e. the worst of the k kept.

@@ -484,6 +484,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     RegTopK<RK> reg;
     reg.init(k);
     float thr_s = desc ? -INFINITY : INFINITY;  // score of the k-th best so far
+    float seed = desc ? -INFINITY : INFINITY;   // admission bound before the list fills
     int cnt = 0;                                // buffered candidates of this query
     if (KR == 0)
       for (int i = 0; i < k; ++i) lists[(size_t)i * kBM + m] = kSentinel;
@@ -494,6 +495,33 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       tc_fence_after();
       const int64_t row0 = (tb + lt) * kBN;
       const uint32_t taddr = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(buf * kBN);
+      if (KR > 0 && lt == 0 && row0 + kBN <= a.N) {
+        // First (full) tile: the k-th best of RK group bests bounds the k-th
+        // best score from below (as in the batched kernel).
+        constexpr int NG = KR > 0 ? KR : 1, GR = kBN / NG, P = 32 / GR;
+        float gb[NG];
+#pragma unroll 1
+        for (int c = 0; c < kBN / 32; ++c) {
+          uint32_t v[32];
+          tmem_ld32(taddr + c * 32, v);
+#pragma unroll
+          for (int i = 0; i < NG - P; ++i) gb[i] = gb[i + P];
+#pragma unroll
+          for (int h = 0; h < P; ++h) {
+            float best = -INFINITY;
+#pragma unroll
+            for (int j = h * GR; j < (h + 1) * GR; ++j) {
+              const float rf = need_cc ? ccbuf[buf * kBN + c * 32 + j] : 0.0f;
+              const float sc = tile_score(a.metric, __uint_as_float(v[j]), fq, qq, rf);
+              best = fmaxf(best, desc ? sc : -sc);
+            }
+            gb[NG - P + h] = best;
+          }
+        }
+        const float kth = kth_largest(gb, k);
+        seed = desc ? nextafterf(kth, -INFINITY) : nextafterf(-kth, INFINITY);
+      }
+      const float thr = desc ? fmaxf(thr_s, seed) : fminf(thr_s, seed);
 #pragma unroll 1
       for (int c = 0; c < kBN / 32; ++c) {
         uint32_t v[32];
@@ -504,12 +532,13 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           // marks them in a 32-bit mask; the warp then appends them to the
           // per-query buffers and merges all buffers when one is full.
           const int64_t nvalid = a.N - (row0 + c * 32);
+          const float thr_c = desc ? fmaxf(thr_s, thr) : fminf(thr_s, thr);
           uint32_t mask = 0;
 #pragma unroll
           for (int j = 0; j < 32; ++j) {
             const float rf = need_cc ? ccbuf[buf * kBN + c * 32 + j] : 0.0f;
             const float sc = tile_score(a.metric, __uint_as_float(v[j]), fq, qq, rf);
-            mask |= (uint32_t)(desc ? sc > thr_s : sc < thr_s) << j;
+            mask |= (uint32_t)(desc ? sc > thr_c : sc < thr_c) << j;
           }
           if (!qvalid || nvalid <= 0) mask = 0;
           else if (nvalid < 32) mask &= (1u << nvalid) - 1u;
@@ -864,6 +893,7 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
     RegTopK<RK> reg;
     reg.init(k);
     float thr_s = desc ? -INFINITY : INFINITY;
+    float seed = desc ? -INFINITY : INFINITY;  // admission bound before the list fills
     int cnt = 0;
     if (KR == 0)
       for (int i = 0; i < k; ++i) lists[(size_t)i * kBM + m] = kSentinel;
@@ -873,6 +903,37 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
       if (!warp_wait(&accf[buf], u & 1, abort_flag, a.gflags)) break;
       tc_fence_after();
       const uint32_t taddr = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(buf * kBN);
+      if (KR > 0 && lt == 0 && row0 + kBN <= g.nrows) {
+        // First (full) tile: the best score of each of RK row groups gives RK
+        // >= k distinct rows, so the k-th best of these group bests bounds the
+        // k-th best score from below; rows worse than it are never offered
+        // (equal ones are).  Saves most of the candidates of the empty list.
+        constexpr int GR = kBN / (KR > 0 ? KR : 1);  // rows per group
+        constexpr int NG = KR > 0 ? KR : 1, P = 32 / GR;  // groups, groups per chunk
+        float gb[NG];
+#pragma unroll 1
+        for (int c = 0; c < kBN / 32; ++c) {
+          uint32_t v[32];
+          const float rfl = need_cc ? g.rowf[row0 + c * 32 + lane] : 0.0f;
+          tmem_ld32(taddr + c * 32, v);
+          // shift register: the P bests of this chunk enter at the top
+#pragma unroll
+          for (int i = 0; i < NG - P; ++i) gb[i] = gb[i + P];
+#pragma unroll
+          for (int h = 0; h < P; ++h) {
+            float best = -INFINITY;
+#pragma unroll
+            for (int j = h * GR; j < (h + 1) * GR; ++j) {
+              const float sc = tile_score(a.metric, __uint_as_float(v[j]), fq, qq,
+                                          __shfl_sync(0xffffffffu, rfl, j));
+              best = fmaxf(best, desc ? sc : -sc);
+            }
+            gb[NG - P + h] = best;
+          }
+        }
+        const float kth = kth_largest(gb, k);  // in "larger is better" units
+        seed = desc ? nextafterf(kth, -INFINITY) : nextafterf(-kth, INFINITY);
+      }
 #pragma unroll 1
       for (int c = 0; c < kBN / 32; ++c) {
         uint32_t v[32];
@@ -880,12 +941,13 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
         // lane j holds the factor of row j of this chunk
         const float rfl = need_cc && lane < nvalid ? g.rowf[row0 + c * 32 + lane] : 0.0f;
         tmem_ld32(taddr + c * 32, v);
+        const float thr = desc ? fmaxf(thr_s, seed) : fminf(thr_s, seed);
         uint32_t mask = 0;
 #pragma unroll
         for (int j = 0; j < 32; ++j) {
           const float rf = __shfl_sync(0xffffffffu, rfl, j);
           const float sc = tile_score(a.metric, __uint_as_float(v[j]), fq, qq, rf);
-          mask |= (uint32_t)(desc ? sc > thr_s : sc < thr_s) << j;
+          mask |= (uint32_t)(desc ? sc > thr : sc < thr) << j;
         }
         if (!qvalid || nvalid <= 0) mask = 0;
         else if (nvalid < 32) mask &= (1u << nvalid) - 1u;
