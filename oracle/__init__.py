@@ -65,6 +65,8 @@ def _load():
         lib.lam_oracle_dequantize.argtypes = [i32p, ctypes.c_int64, ctypes.c_float,
                                               f32p]
         lib.lam_oracle_dequantize.restype = None
+        lib.lam_oracle_code_sqnorms.argtypes = [i32p, ctypes.c_int64, ctypes.c_int32, f32p]
+        lib.lam_oracle_code_sqnorms.restype = None
         lib.lam_oracle_scores.argtypes = [f32p, ctypes.c_int64, i32p, ctypes.c_int64,
                                           ctypes.c_int32, ctypes.c_float,
                                           ctypes.c_int32, f32p]
@@ -123,6 +125,15 @@ def dequantize(codes: np.ndarray, scale: float) -> np.ndarray:
                                   ctypes.c_float(np.float32(scale)),
                                   _ptr(out, ctypes.c_float))
     return out.reshape(np.shape(codes))
+
+
+def code_sqnorms(codes: np.ndarray) -> np.ndarray:
+    """fl32 of the exact sum of squares of each code row [N, D] -> [N]."""
+    c = np.ascontiguousarray(codes, dtype=np.int32)
+    N, D = c.shape
+    out = np.empty(N, dtype=np.float32)
+    _load().lam_oracle_code_sqnorms(_ptr(c, ctypes.c_int32), N, D, _ptr(out, ctypes.c_float))
+    return out
 
 
 def scores(queries: np.ndarray, codes: np.ndarray, eps: float, metric: int):

@@ -110,6 +110,23 @@ void lam_oracle_dequantize(const int32_t *codes, int64_t n, float scale,
   for (int64_t i = 0; i < n; ++i) out[i] = scale * (float)codes[i];
 }
 
+/* Squared norm of each code row, sum_d c_{i,d}^2: the exact integer sum
+ * (in int64; |c| <= 32767 for the 1- and 2-byte widths, so it cannot
+ * overflow for D < 2^33) rounded once to fp32.  This is the side array an
+ * exact scan can keep to score cosine and squared L2 on codes (Eq. 1 expands
+ * the L2 distance into the two norms and the inner product). */
+void lam_oracle_code_sqnorms(const int32_t *codes, int64_t N, int32_t D,
+                             float *out) {
+  for (int64_t i = 0; i < N; ++i) {
+    int64_t acc = 0;
+    for (int32_t d = 0; d < D; ++d) {
+      const int64_t c = codes[i * (int64_t)D + d];
+      acc += c * c;
+    }
+    out[i] = (float)acc; /* one round-to-nearest conversion */
+  }
+}
+
 /* Score of one query against one dequantised row, in double, rounded to fp32. */
 static float score_one(const float *q, const int32_t *c, int32_t D, float s,
                        int metric) {

@@ -248,3 +248,37 @@ def test_numpy_rint_cross_check():
         codes, *_ = oracle.quantize(x, eps)
         s = np.float32(2.0) * np.float32(eps)
         np.testing.assert_array_equal(codes, np.rint(x / s).astype(np.int32))
+
+
+def test_code_sqnorms_closed_forms_and_invariants():
+    # constant rows: D v^2 (the exact integer, rounded once to fp32)
+    for D in (1, 7, 768):
+        for v in (0, 1, -3, 127, -128, 2048, 32767, -32768):
+            got = oracle.code_sqnorms(np.full((1, D), v, dtype=np.int32))[0]
+            assert got == np.float32(float(D * v * v))
+    # one non-zero coordinate reads back its square wherever it sits
+    D = 33
+    basis = np.zeros((D, D), dtype=np.int32)
+    basis[np.arange(D), np.arange(D)] = np.arange(1, D + 1) * 7
+    np.testing.assert_array_equal(oracle.code_sqnorms(basis),
+                                  (np.arange(1, D + 1, dtype=np.float32) * 7) ** 2)
+    rng = np.random.default_rng(5)
+    c = rng.integers(-300, 300, size=(50, 96)).astype(np.int32)
+    base = oracle.code_sqnorms(c)
+    # sign and coordinate-order invariance
+    np.testing.assert_array_equal(oracle.code_sqnorms(-c), base)
+    np.testing.assert_array_equal(oracle.code_sqnorms(c[:, rng.permutation(96)]), base)
+    # additivity over a split of the coordinates (sums here stay exact in fp32)
+    np.testing.assert_array_equal(oracle.code_sqnorms(c[:, :40]) + oracle.code_sqnorms(c[:, 40:]),
+                                  base)
+
+
+def test_code_sqnorms_agree_with_the_l2_score_of_a_zero_query():
+    # ||0 - s c||^2 = s^2 sum c^2: the two oracle functions must agree to fp32 rounding
+    x = inputs.unit_rows(40, 64, seed=6)
+    codes, *_ = oracle.quantize(x, 1e-3)
+    codes = codes.reshape(x.shape)
+    s = float(oracle.step(1e-3))
+    l2 = oracle.scores(np.zeros((1, 64), np.float32), codes, 1e-3, oracle.L2)[0]
+    np.testing.assert_allclose(l2, s * s * oracle.code_sqnorms(codes).astype(np.float64),
+                               rtol=3e-7)
