@@ -180,6 +180,23 @@ int32_t lam_score_topk_path(int64_t B, int64_t N, int32_t D, int32_t k,
                             int32_t width, int32_t code_bound);
 
 /*
+ * lam_code_sqnorms -- sqnorm_out[i] = fl32(sum_d c_{i,d}^2) for each code row:
+ * the exact integer sum, rounded once to fp32.  It is the per-row side array
+ * an exact scan on codes can keep for cosine and squared L2 (Eq. 1 splits the
+ * L2 distance into the two norms and the inner product); lam_score_topk
+ * computes the same sums internally where it already reads the codes, so it
+ * does not take this array.
+ *
+ * codes       [N, D] row-major device codes of `width` bytes (1 or 2),
+ *             aligned to the width.
+ * sqnorm_out  [N] device fp32, 4-byte aligned.
+ * Asynchronous on `stream`.  Errors: LAM_ERR_INVALID (N < 0, D < 1, NULL or
+ * misaligned pointers, width not 1 or 2), LAM_ERR_CUDA.
+ */
+lam_status lam_code_sqnorms(const void *codes, int32_t width, int64_t N, int32_t D,
+                            float *sqnorm_out, lam_stream_t stream);
+
+/*
  * Kernel timing (measurement support, not part of the method).
  *
  * lam_timing_begin(mask, capacity) makes the library bracket each launch of

@@ -56,6 +56,7 @@ def load():
         "lam_score_topk_path": (i32, [i64, i64, i32, i32, i32, i32]),
         "lam_score_topk_noalloc": (i32, [vp, i64, vp, i32, i64, i32, f32, i32, i32, i32, vp,
                                          vp, vp]),
+        "lam_code_sqnorms": (i32, [vp, i32, i64, i32, vp, vp]),
         "lam_timing_begin": (i32, [i32, i64]),
         "lam_timing_read": (i32, [i32, P(ctypes.c_double), P(i64), P(i64)]),
         "lam_timing_end": (i32, []),
@@ -166,6 +167,13 @@ def lam_score_topk_noalloc(queries, codes, width, N, D, eps, code_bound, k, metr
                                        int(metric), _ptr(scores), _ptr(ids),
                                        _stream(stream, queries.device))
     _check(st, "lam_score_topk_noalloc")
+
+
+def lam_code_sqnorms(codes, width, N, D, sqnorm_out, stream=None) -> None:
+    """sqnorm_out[i] = fl32(exact sum of squares of code row i)."""
+    st = load().lam_code_sqnorms(_ptr(codes), int(width), int(N), int(D), _ptr(sqnorm_out),
+                                 _stream(stream, codes.device))
+    _check(st, "lam_code_sqnorms")
 
 
 LAM_TIME_QUANTIZE, LAM_TIME_DEQUANTIZE, LAM_TIME_SCORE, LAM_TIME_AUX = 1, 2, 4, 8

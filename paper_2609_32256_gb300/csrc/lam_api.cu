@@ -303,6 +303,23 @@ lam_status lam_dequantize(const void *codes, int32_t width, int64_t n, float sca
   return e == cudaSuccess ? LAM_OK : LAM_ERR_CUDA;
 }
 
+lam_status lam_code_sqnorms(const void *codes, int32_t width, int64_t N, int32_t D,
+                            float *sqnorm_out, lam_stream_t stream) {
+  if (N < 0 || D < 1 || (width != 1 && width != 2)) return LAM_ERR_INVALID;
+  if (N == 0) return LAM_OK;
+  if (codes == nullptr || sqnorm_out == nullptr) return LAM_ERR_INVALID;
+  if ((reinterpret_cast<uintptr_t>(codes) & (uintptr_t)(width - 1)) != 0 ||
+      (reinterpret_cast<uintptr_t>(sqnorm_out) & 3u) != 0)
+    return LAM_ERR_INVALID;
+  const int sms = device_sms();
+  if (sms <= 0) return LAM_ERR_CUDA;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  timing_launch_begin(LAM_TIME_AUX, st);
+  const cudaError_t e = launch_code_sqnorms(codes, width, N, D, sqnorm_out, sms, st);
+  timing_launch_end(LAM_TIME_AUX, st);
+  return e == cudaSuccess ? LAM_OK : LAM_ERR_CUDA;
+}
+
 size_t lam_score_topk_workspace_size(int64_t B, int64_t N, int32_t D, int32_t k, int32_t width,
                                      int32_t code_bound) {
   Plan p;

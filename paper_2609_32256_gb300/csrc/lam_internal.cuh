@@ -149,6 +149,8 @@ cudaError_t launch_quant_range(const float *x, int64_t n, QuantStatus *status, i
 cudaError_t launch_quantize(const float *x, int64_t n, float s, int width_req, void *codes,
                             size_t codes_bytes, QuantStatus *status, int sms,
                             cudaStream_t st);
+cudaError_t launch_code_sqnorms(const void *codes, int width, int64_t N, int D, float *out,
+                                int sms, cudaStream_t st);
 cudaError_t launch_dequantize(const void *codes, int width, int64_t n, float s, float *out,
                               int sms, cudaStream_t st);
 // AUTO width: one launch; if the status ends with passes == 2 the caller

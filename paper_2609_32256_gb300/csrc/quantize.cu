@@ -335,6 +335,29 @@ __global__ void __launch_bounds__(kThreads) dequantize_kernel(const void *__rest
   }
 }
 
+// One warp per code row: exact int64 sum of squares, rounded once to fp32.
+template <int W>
+__global__ void __launch_bounds__(kThreads) code_sqnorms_kernel(const void *__restrict__ codes,
+                                                                int64_t N, int D,
+                                                                float *__restrict__ out) {
+  const int lane = threadIdx.x & 31;
+  const int64_t nwarps = (int64_t)gridDim.x * (blockDim.x >> 5);
+  for (int64_t r = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); r < N;
+       r += nwarps) {
+    long long acc = 0;
+    if (W == 1) {
+      const int8_t *row = static_cast<const int8_t *>(codes) + r * (int64_t)D;
+      for (int d = lane; d < D; d += 32) acc += (int)row[d] * (int)row[d];
+    } else {
+      const int16_t *row = static_cast<const int16_t *>(codes) + r * (int64_t)D;
+      for (int d = lane; d < D; d += 32) acc += (long long)((int)row[d] * (int)row[d]);
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
+    if (lane == 0) out[r] = __ll2float_rn(acc);
+  }
+}
+
 inline bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 // Resident blocks per SM of a kernel at kThreads threads (registers decide
@@ -403,6 +426,14 @@ cudaError_t launch_dequantize(const void *codes, int width, int64_t n, float s, 
               : width == 2 ? (vec ? dequantize_kernel<2, true> : dequantize_kernel<2, false>)
                            : (vec ? dequantize_kernel<4, true> : dequantize_kernel<4, false>);
   kern<<<grid_for(kern, vec ? n / 4 + 1 : n, sms), kThreads, 0, st>>>(codes, n, s, out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_code_sqnorms(const void *codes, int width, int64_t N, int D, float *out,
+                                int sms, cudaStream_t st) {
+  auto kern = width == 1 ? code_sqnorms_kernel<1> : code_sqnorms_kernel<2>;
+  const int g = grid_for(kern, N * 32, sms);
+  kern<<<g, kThreads, 0, st>>>(codes, N, D, out);
   return cudaGetLastError();
 }
 

@@ -140,3 +140,12 @@ def test_timing_read_rejects_bad_kind_and_end_is_idempotent(lib):
     assert (tot, timed, launches) == (0.0, 0, 0)
     assert lib.lam_timing_end() == 0
     assert lib.lam_timing_end() == 0
+
+
+@pytest.mark.parametrize("width,N,D,codes,out", [(4, 10, 8, 256, 512), (3, 10, 8, 256, 512),
+                                                 (1, -1, 8, 256, 512), (1, 10, 0, 256, 512),
+                                                 (2, 10, 8, 257, 512), (1, 10, 8, 256, 514),
+                                                 (1, 10, 8, 0, 512)])
+def test_code_sqnorms_rejects_bad_arguments(lib, width, N, D, codes, out):
+    c = ctypes
+    assert lib.lam_code_sqnorms(c.c_void_p(codes), width, N, D, c.c_void_p(out), None) == 1

@@ -158,3 +158,17 @@ def test_zero_rows_and_zero_query_cosine(dev, B):
     q[1] = 0.0
     for metric in METRICS:
         check(dev, q, codes, 1, 1e-2, 30, metric, bound)
+
+
+@pytest.mark.parametrize("width", [1, 2])
+@pytest.mark.parametrize("N,D", [(1, 1), (1000, 33), (777, 768)])
+def test_code_sqnorms_bit_exact(dev, width, N, D):
+    rng = np.random.default_rng(N + D + width)
+    lo, hi = (-128, 128) if width == 1 else (-32768, 32768)
+    c = rng.integers(lo, hi, size=(N, D)).astype(NP_DT[width])
+    c[0, :] = lo  # the extreme code everywhere in one row
+    want = oracle.code_sqnorms(c.astype(np.int32))
+    ct = torch.from_numpy(c).to(dev)
+    out = torch.empty(N, dtype=torch.float32, device=dev)
+    lam.lam_code_sqnorms(ct, width, N, D, out)
+    np.testing.assert_array_equal(out.cpu().numpy().view(np.uint32), want.view(np.uint32))
