@@ -198,7 +198,8 @@ class Pipeline:
         self.codes = self.codes_e[0]
         self.deq = torch.empty_like(x)
         self.sq = torch.cuda.Stream(dev)  # quantize stream
-        self.ss = torch.cuda.Stream(dev)  # dequantize + score stream
+        self.sd = torch.cuda.Stream(dev)  # dequantize stream
+        self.ss = torch.cuda.Stream(dev)  # score stream
         self.qdone = [torch.cuda.Event() for _ in eps_list]
         self.qws = torch.zeros(64, dtype=torch.uint8, device=dev)
         self.scores = [torch.empty((self.B, k), dtype=torch.float32, device=dev) for _ in eps_list]
@@ -215,20 +216,23 @@ class Pipeline:
 
     def step_overlapped(self):
         """The step as a user would drive it: Q_eps of each eps on one stream
-        (synchronous: the width comes back to the host), dequantisation and
-        search of that eps on a second stream, so the search of eps j runs
-        while eps j+1 is quantized.  The same calls and work as step()."""
+        (synchronous: the width comes back to the host); the dequantisation
+        and the search of that eps, which only read its codes, each on a
+        stream of their own, so they overlap one another and the quantization
+        of the next eps.  The same calls and work as step()."""
         lam = self.lam
         n = self.x.numel()
         for j, e in enumerate(self.eps_list):
             st, w, s, cmin, cmax = lam.lam_quantize(self.x, e, 0, self.codes_e[j], self.qws,
                                                     stream=self.sq.cuda_stream)
             self.qdone[j].record(self.sq)
+            self.sd.wait_event(self.qdone[j])
             self.ss.wait_event(self.qdone[j])
-            lam.lam_dequantize(self.codes_e[j], w, n, s, self.deq, stream=self.ss.cuda_stream)
+            lam.lam_dequantize(self.codes_e[j], w, n, s, self.deq, stream=self.sd.cuda_stream)
             lam.lam_score_topk(self.q, self.codes_e[j], w, self.N, self.D, e, max(-cmin, cmax),
                                self.k, self.metric, self.scores[j], self.ids[j], self.sws,
                                stream=self.ss.cuda_stream)
+        self.ss.wait_stream(self.sd)  # the step ends when both have finished
 
     def step(self, ev=None):
         """The step with every call in order on the current stream (per-stage
@@ -305,6 +309,7 @@ def run_lam(args):
     def overlapped_step(i, e0, e1):
         # the previous step is finished and L2 is flushed before the step starts
         pipe.sq.wait_stream(pipe.ss)
+        pipe.sq.wait_stream(pipe.sd)
         pipe.sq.wait_stream(cur)
         with torch.cuda.stream(pipe.sq):
             flush(i)
@@ -460,8 +465,9 @@ def run_lam(args):
                        "l2": "flushed between timed steps (512 MB write then 512 MB read, outside "
                              "the events)",
                        "step": "per eps: lam_quantize (synchronous) on one stream, lam_dequantize "
-                               "+ lam_score_topk on a second; the search of eps j overlaps the "
-                               "quantization of eps j+1 (ms_per_step_serial: all on one stream)"},
+                               "and lam_score_topk of its codes on two more; they overlap each "
+                               "other and the quantization of the next eps "
+                               "(ms_per_step_serial: all on one stream)"},
             "breakdown": {
                 "quantize_ms": ms_q, "quantize_gbs_algorithmic": q_bytes / (ms_q / 1e3) / 1e9,
                 "quantize_note": "lam_quantize span: status clear + quantize + status read-back",
