@@ -419,10 +419,10 @@ __global__ void __launch_bounds__(kKmWarps * 32) topk_kmerge_kernel(ScoreArgs a,
   uint64_t *outk = cand + (size_t)qpc * L * k;                       // [kKmWarps][P2]
   const int P2 = next_pow2_dev(k);
   const int64_t b0 = (int64_t)blockIdx.x * qpc;
-  const int64_t per_q = (int64_t)L * k;
-  for (int64_t e = threadIdx.x; e < (int64_t)qpc * per_q; e += blockDim.x) {
-    const int64_t qi = e / per_q, rem = e - qi * per_q;
-    const int64_t l = rem / k, i = rem - l * k;
+  const int per_q = L * k;  // fits: the candidates of qpc queries fit in shared memory
+  for (int e = threadIdx.x; e < qpc * per_q; e += blockDim.x) {
+    const int qi = e / per_q, rem = e - qi * per_q;
+    const int l = rem / k, i = rem - l * k;
     const int64_t b = b0 + qi;
     cand[e] = b < a.B ? a.partial[((size_t)l * a.B + b) * k + i] : kSentinel;
   }

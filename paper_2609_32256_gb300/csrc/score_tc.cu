@@ -616,9 +616,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 // 64 bytes apart with the 16-byte chunks of row r XOR-ed by (r >> 1) & 3, the
 // 64-byte swizzle), zeros for padding rows and columns; then (2^-e, ||q||,
 // ||q||^2, 0) per query after the images.
-__global__ void __launch_bounds__(256) qprep_kernel(const float *__restrict__ q, int64_t B, int D,
-                                                    int64_t Bpad, uint8_t *__restrict__ qA) {
-  const int64_t b = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
+__device__ __forceinline__ void qprep_block(const float *__restrict__ q, int64_t B, int D,
+                                            int64_t Bpad, uint8_t *__restrict__ qA, int64_t blk) {
+  const int64_t b = blk * 8 + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (b >= Bpad) return;
   const int nk = (D + kBK - 1) / kBK;
@@ -672,6 +672,11 @@ __global__ void __launch_bounds__(256) qprep_kernel(const float *__restrict__ q,
                      : make_float4(0.f, 0.f, 0.f, 0.f);
 }
 
+__global__ void __launch_bounds__(256) qprep_kernel(const float *__restrict__ q, int64_t B, int D,
+                                                    int64_t Bpad, uint8_t *__restrict__ qA) {
+  qprep_block(q, B, D, Bpad, qA, blockIdx.x);
+}
+
 
 // ===========================================================================
 // Batched path for two or more query blocks.  A separate pass converts the
@@ -688,13 +693,12 @@ constexpr int kTc2Threads = 192;  // warp 0 producer, warp 1 MMA, warps 2-5 epil
 // nrows and columns past D are zero.  Also the per-row factor rowf (1/||c|| for
 // cosine, s^2 ||c||^2 for L2).  One warp per row of the padded slab.
 template <int W>
-__global__ void __launch_bounds__(256) convert_codes_kernel(const void *__restrict__ codes,
-                                                            int64_t row_base, int64_t nrows,
-                                                            int64_t nrows_pad, int D,
-                                                            uint8_t *__restrict__ out,
-                                                            float *__restrict__ rowf, int metric,
-                                                            float s, uint32_t *gflags) {
-  const int64_t r = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
+__device__ __forceinline__ void convert_block(const void *__restrict__ codes, int64_t row_base,
+                                              int64_t nrows, int64_t nrows_pad, int D,
+                                              uint8_t *__restrict__ out,
+                                              float *__restrict__ rowf, int metric, float s,
+                                              uint32_t *gflags, int64_t blk) {
+  const int64_t r = blk * 8 + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (r >= nrows_pad) return;
   const bool valid = r < nrows;
@@ -735,6 +739,30 @@ __global__ void __launch_bounds__(256) convert_codes_kernel(const void *__restri
   if (lane == 0 && valid && metric != LAM_METRIC_IP)
     rowf[r] = metric == LAM_METRIC_COSINE ? (cc > 0.0f ? 1.0f / sqrtf(cc) : 0.0f) : s * s * cc;
   if (W == 2 && amax > 2048.0f) atomicOr(gflags, kFlagRange);
+}
+
+template <int W>
+__global__ void __launch_bounds__(256) convert_codes_kernel(const void *__restrict__ codes,
+                                                            int64_t row_base, int64_t nrows,
+                                                            int64_t nrows_pad, int D,
+                                                            uint8_t *__restrict__ out,
+                                                            float *__restrict__ rowf, int metric,
+                                                            float s, uint32_t *gflags) {
+  convert_block<W>(codes, row_base, nrows, nrows_pad, D, out, rowf, metric, s, gflags, blockIdx.x);
+}
+
+// Query preparation and the first slab's conversion in one launch: blocks
+// [0, q_blocks) prepare queries, the rest convert code rows (independent work).
+template <int W>
+__global__ void __launch_bounds__(256) prep_convert_kernel(
+    const float *__restrict__ q, int64_t B, int D, int64_t Bpad, uint8_t *__restrict__ qA,
+    unsigned q_blocks, const void *__restrict__ codes, int64_t nrows, int64_t nrows_pad,
+    uint8_t *__restrict__ out, float *__restrict__ rowf, int metric, float s, uint32_t *gflags) {
+  if (blockIdx.x < q_blocks)
+    qprep_block(q, B, D, Bpad, qA, blockIdx.x);
+  else
+    convert_block<W>(codes, 0, nrows, nrows_pad, D, out, rowf, metric, s, gflags,
+                     blockIdx.x - q_blocks);
 }
 
 struct Tc2Layout {
@@ -1100,13 +1128,15 @@ cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st) {
   const TensorPlan P = tensor_plan(a.B, a.N, a.D, a.k, a.sms);
   if (P.n_lists != a.n_lists) return cudaErrorInvalidValue;
   uint8_t *qA = static_cast<uint8_t *>(a.qprep);
-  timing_launch_begin(LAM_TIME_AUX, st);
-  qprep_kernel<<<(unsigned)((a.Bpad + 7) / 8), 256, 0, st>>>(a.queries, a.B, a.D, a.Bpad, qA);
-  timing_launch_end(LAM_TIME_AUX, st);
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
+  const unsigned q_blocks = (unsigned)((a.Bpad + 7) / 8);
+  cudaError_t e = cudaSuccess;
 
   if (!P.pre) {
+    timing_launch_begin(LAM_TIME_AUX, st);
+    qprep_kernel<<<q_blocks, 256, 0, st>>>(a.queries, a.B, a.D, a.Bpad, qA);
+    timing_launch_end(LAM_TIME_AUX, st);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
     const TcLayout L = tc_layout(a.width, a.k);
     if (L.ns < 2) return cudaErrorInvalidValue;
     CUtensorMap cmap;
@@ -1165,12 +1195,22 @@ cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st) {
     const int64_t nrows_pad = (nrows + kBN - 1) / kBN * kBN;
     const unsigned cg = (unsigned)((nrows_pad + 7) / 8);
     timing_launch_begin(LAM_TIME_AUX, st);
-    if (a.width == 1)
+    if (j == 0) {  // the first slab's conversion shares a launch with the query prep
+      if (a.width == 1)
+        prep_convert_kernel<1><<<q_blocks + cg, 256, 0, st>>>(
+            a.queries, a.B, a.D, a.Bpad, qA, q_blocks, a.codes, nrows, nrows_pad, f16, rowf,
+            a.metric, a.s, a.gflags);
+      else
+        prep_convert_kernel<2><<<q_blocks + cg, 256, 0, st>>>(
+            a.queries, a.B, a.D, a.Bpad, qA, q_blocks, a.codes, nrows, nrows_pad, f16, rowf,
+            a.metric, a.s, a.gflags);
+    } else if (a.width == 1) {
       convert_codes_kernel<1><<<cg, 256, 0, st>>>(a.codes, row_base, nrows, nrows_pad, a.D, f16,
                                                   rowf, a.metric, a.s, a.gflags);
-    else
+    } else {
       convert_codes_kernel<2><<<cg, 256, 0, st>>>(a.codes, row_base, nrows, nrows_pad, a.D, f16,
                                                   rowf, a.metric, a.s, a.gflags);
+    }
     timing_launch_end(LAM_TIME_AUX, st);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
