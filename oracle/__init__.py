@@ -65,6 +65,13 @@ def _load():
         lib.lam_oracle_dequantize.argtypes = [i32p, ctypes.c_int64, ctypes.c_float,
                                               f32p]
         lib.lam_oracle_dequantize.restype = None
+        u8p = ctypes.POINTER(ctypes.c_uint8)
+        u64p = ctypes.POINTER(ctypes.c_uint64)
+        lib.lam_oracle_fnv1a64.argtypes = [u8p, ctypes.c_int64, ctypes.c_uint64]
+        lib.lam_oracle_fnv1a64.restype = ctypes.c_uint64
+        lib.lam_oracle_band_digests.argtypes = [i32p, ctypes.c_int64, ctypes.c_int32,
+                                                ctypes.c_int32, ctypes.c_int32, u64p]
+        lib.lam_oracle_band_digests.restype = None
         lib.lam_oracle_code_sqnorms.argtypes = [i32p, ctypes.c_int64, ctypes.c_int32, f32p]
         lib.lam_oracle_code_sqnorms.restype = None
         lib.lam_oracle_scores.argtypes = [f32p, ctypes.c_int64, i32p, ctypes.c_int64,
@@ -125,6 +132,26 @@ def dequantize(codes: np.ndarray, scale: float) -> np.ndarray:
                                   ctypes.c_float(np.float32(scale)),
                                   _ptr(out, ctypes.c_float))
     return out.reshape(np.shape(codes))
+
+
+FNV_OFFSET = 14695981039346656037
+
+
+def fnv1a64(data: bytes, h: int = FNV_OFFSET) -> int:
+    """64-bit FNV-1a of a byte string, continuing from state h."""
+    buf = np.frombuffer(bytes(data), dtype=np.uint8).copy()
+    return int(_load().lam_oracle_fnv1a64(_ptr(buf, ctypes.c_uint8), buf.size, h))
+
+
+def band_digests(codes: np.ndarray, r: int, width: int) -> np.ndarray:
+    """Digest of every r-coordinate band of every code row [N, D] -> uint64 [N, D // r]."""
+    c = np.ascontiguousarray(codes, dtype=np.int32)
+    N, D = c.shape
+    assert D % r == 0
+    out = np.empty((N, D // r), dtype=np.uint64)
+    _load().lam_oracle_band_digests(_ptr(c, ctypes.c_int32), N, D, r, width,
+                                    _ptr(out, ctypes.c_uint64))
+    return out
 
 
 def code_sqnorms(codes: np.ndarray) -> np.ndarray:

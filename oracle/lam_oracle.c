@@ -127,7 +127,46 @@ void lam_oracle_code_sqnorms(const int32_t *codes, int64_t N, int32_t D,
   }
 }
 
-/* Score of one query against one dequantised row, in double, rounded to fp32. */
+/*
+ * Band digests of quantized rows (Sec. 3.2, L1: "divide the vector into
+ * bands, and hash each band; records sharing a band digest are candidates";
+ * Algorithm 1, BandHash(Q_eps(e))).  The paper names no hash function; the
+ * reading taken here is 64-bit FNV-1a (Fowler, Noll, Vo: offset basis
+ * 14695981039346656037, prime 1099511628211, one xor then one multiply per
+ * byte) over
+ *   - the band's index within its row, as 2 little-endian bytes (so that
+ *     equal code patterns in different bands do not share a digest), then
+ *   - the band's r codes in coordinate order, each as its `width`
+ *     little-endian two's-complement bytes (the bytes the code array holds).
+ * Rows have D coordinates, D a multiple of r; digest[i * (D / r) + b] is band
+ * b of row i.
+ */
+uint64_t lam_oracle_fnv1a64(const uint8_t *bytes, int64_t n, uint64_t h) {
+  for (int64_t i = 0; i < n; ++i) {
+    h ^= (uint64_t)bytes[i];
+    h *= 1099511628211ULL;
+  }
+  return h;
+}
+
+void lam_oracle_band_digests(const int32_t *codes, int64_t N, int32_t D, int32_t r,
+                             int32_t width, uint64_t *digest) {
+  const int32_t nb = D / r;
+  for (int64_t i = 0; i < N; ++i) {
+    for (int32_t b = 0; b < nb; ++b) {
+      uint8_t idx[2] = {(uint8_t)(b & 0xff), (uint8_t)((b >> 8) & 0xff)};
+      uint64_t h = lam_oracle_fnv1a64(idx, 2, 14695981039346656037ULL);
+      for (int32_t d = b * r; d < (b + 1) * r; ++d) {
+        const uint32_t c = (uint32_t)codes[i * (int64_t)D + d];
+        uint8_t le[4] = {(uint8_t)c, (uint8_t)(c >> 8), (uint8_t)(c >> 16), (uint8_t)(c >> 24)};
+        h = lam_oracle_fnv1a64(le, width, h);
+      }
+      digest[i * nb + b] = h;
+    }
+  }
+}
+
+/* Score of one query against one dequantised row, in double, rounded to fp32. *//* Score of one query against one dequantised row, in double, rounded to fp32. */
 static float score_one(const float *q, const int32_t *c, int32_t D, float s,
                        int metric) {
   if (metric == ORACLE_IP) {

@@ -282,3 +282,45 @@ def test_code_sqnorms_agree_with_the_l2_score_of_a_zero_query():
     l2 = oracle.scores(np.zeros((1, 64), np.float32), codes, 1e-3, oracle.L2)[0]
     np.testing.assert_allclose(l2, s * s * oracle.code_sqnorms(codes).astype(np.float64),
                                rtol=3e-7)
+
+
+def test_fnv1a64_published_vectors():
+    for text, want in golden("fnv1a64_vectors.txt"):
+        data = b"" if text == "-" else text.encode("ascii")
+        assert oracle.fnv1a64(data) == int(want, 16), text
+
+
+def test_band_digests_depend_on_every_code_and_the_band_position():
+    rng = np.random.default_rng(12)
+    for r, width, (lo, hi) in ((2, 1, (-128, 128)), (4, 2, (-32768, 32768)), (32, 1, (-5, 6)),
+                               (8, 4, (-2**31, 2**31))):
+        D = 4 * r
+        row = rng.integers(lo, hi, size=(1, D)).astype(np.int64).astype(np.int32)
+        base = oracle.band_digests(row, r, width)
+        assert base.shape == (1, D // r)
+        # the same codes in every band still give a different digest per band
+        same = np.tile(row[:, :r], (1, D // r))
+        dig = oracle.band_digests(same, r, width)[0]
+        assert len(set(dig.tolist())) == D // r
+        # changing any one coordinate changes only its own band's digest
+        for d in range(D):
+            mod = row.copy()
+            mod[0, d] = mod[0, d] + 1 if mod[0, d] < hi - 1 else mod[0, d] - 1
+            got = oracle.band_digests(mod, r, width)[0]
+            changed = np.nonzero(got != base[0])[0].tolist()
+            assert changed == [d // r], (r, width, d)
+        # identical rows share every digest; rows are independent of each other
+        two = np.vstack([row, row[:, ::-1]])
+        dd = oracle.band_digests(two, r, width)
+        np.testing.assert_array_equal(dd[0], base[0])
+        np.testing.assert_array_equal(oracle.band_digests(two[1:], r, width)[0], dd[1])
+
+
+def test_band_digest_of_a_single_band_is_the_fnv_of_its_bytes():
+    # one band, one code: the digest is FNV-1a of the two index bytes then the
+    # code's little-endian bytes, checked through the published FNV function
+    for width, code in ((1, -3), (2, 1234), (4, -70000)):
+        got = oracle.band_digests(np.array([[code]], dtype=np.int32), 1, width)[0, 0]
+        want = oracle.fnv1a64(int(code).to_bytes(4, "little", signed=True)[:width],
+                              oracle.fnv1a64(b"\x00\x00"))
+        assert int(got) == want
