@@ -622,6 +622,24 @@ def run_kernels(args):
         gbd = (wq + 4) * n / (k_d / 1e3) / 1e9
         res["dequantize"].append({"eps": e, "width": wq, "ms_span": ms_d, "ms_kernel": k_d,
                                   "gbs_kernel": gbd, "frac_of_hbm_kernel": gbd / hbm})
+    if wl.d > 1:
+        # Q_eps fused with the band digests (r = 4 and 8, the paper's shipped and
+        # best band widths), codes written, AUTO width
+        res["bands"] = []
+        N = wl.n
+        for r in (4, 8):
+            dig = torch.empty((N, wl.d // r), dtype=torch.int64, device=dev)
+            for e in eps_list:
+                xr = x.view(N, wl.d)
+                st, w, *_ = lam.lam_quantize_bands(xr, e, 0, r, codes, dig, ws)
+                ms, k_ms = timed(lambda: lam.lam_quantize_bands(xr, e, 0, r, codes, dig, ws),
+                                 lam.LAM_TIME_QUANTIZE)
+                nbytes = (4 + w) * n + 8 * (n // r)
+                res["bands"].append({"r": r, "eps": e, "width": w, "ms_span": ms,
+                                     "ms_kernel": k_ms,
+                                     "gbs_kernel": nbytes / (k_ms / 1e3) / 1e9,
+                                     "frac_of_hbm_kernel": nbytes / (k_ms / 1e3) / 1e9 / hbm})
+            del dig
     if wl.batches and wl.d > 1:
         e = eps_list[0]
         wq, sc, bound = widths[e]

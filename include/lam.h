@@ -106,6 +106,35 @@ lam_status lam_quantize(const float *x, int64_t n, float eps, int32_t width_req,
                         int32_t *code_max_out, lam_stream_t stream);
 
 /*
+ * lam_quantize_bands -- Q_eps fused with the band digests of the quantized
+ * rows (Sec. 3.2, layer L1: quantize, divide each vector into bands of r
+ * coordinates and hash each band; records sharing a band digest are
+ * candidates.  Algorithm 1: B <- BandHash(Q_eps(e))).  One pass over x.
+ *
+ * x        [N, D] fp32 rows, device, 4-byte aligned; D a multiple of r and
+ *          D / r <= 65536.
+ * r        band width in coordinates (the paper sweeps 2, 4, 8, 16, 32).
+ * codes    as for lam_quantize (may be NULL: digests only).
+ * digests  [N, D / r] uint64, device, 8-byte aligned: digests[i * (D/r) + b]
+ *          is the 64-bit FNV-1a (offset basis 14695981039346656037, prime
+ *          1099511628211, one xor and one multiply per byte) of band b of
+ *          row i: the band index as 2 little-endian bytes, then the band's r
+ *          codes as their `width` little-endian two's-complement bytes.  The
+ *          paper names no hash; this reading is exact and portable.
+ * The width, workspace, outputs, synchrony and errors are those of
+ * lam_quantize (with AUTO, the digests use the resolved width); on an error
+ * the digests are undefined.  LAM_ERR_INVALID also for r outside 1..D, D not
+ * a multiple of r, or a misaligned digests pointer.
+ */
+lam_status lam_quantize_bands(const float *x, int64_t N, int32_t D, float eps,
+                              int32_t width_req, int32_t r, void *codes,
+                              size_t codes_bytes, uint64_t *digests,
+                              void *workspace, size_t workspace_bytes,
+                              int32_t *width_out, float *scale_out,
+                              int32_t *code_min_out, int32_t *code_max_out,
+                              lam_stream_t stream);
+
+/*
  * lam_dequantize -- xhat_i = fl32(scale * code_i), the inverse map of Q_eps
  * up to the cell half-width eps (|x - xhat| <= eps, Sec. 3.1).
  *

@@ -57,6 +57,8 @@ def load():
         "lam_score_topk_noalloc": (i32, [vp, i64, vp, i32, i64, i32, f32, i32, i32, i32, vp,
                                          vp, vp]),
         "lam_code_sqnorms": (i32, [vp, i32, i64, i32, vp, vp]),
+        "lam_quantize_bands": (i32, [vp, i64, i32, f32, i32, i32, vp, sz, vp, vp, sz, P(i32),
+                                     P(f32), P(i32), P(i32), vp]),
         "lam_timing_begin": (i32, [i32, i64]),
         "lam_timing_read": (i32, [i32, P(ctypes.c_double), P(i64), P(i64)]),
         "lam_timing_end": (i32, []),
@@ -167,6 +169,23 @@ def lam_score_topk_noalloc(queries, codes, width, N, D, eps, code_bound, k, metr
                                        int(metric), _ptr(scores), _ptr(ids),
                                        _stream(stream, queries.device))
     _check(st, "lam_score_topk_noalloc")
+
+
+def lam_quantize_bands(x, eps, width_req, r, codes, digests, workspace, stream=None,
+                       raise_on_error=True):
+    """Q_eps of the fp32 rows x [N, D] fused with the FNV-1a digest of every
+    r-coordinate band; digests is a [N, D // r] int64/uint64 CUDA tensor.
+    Returns (status, width, scale, code_min, code_max)."""
+    N, D = x.shape
+    w, sc, cmin, cmax = ctypes.c_int32(0), ctypes.c_float(0), ctypes.c_int32(0), ctypes.c_int32(0)
+    st = load().lam_quantize_bands(_ptr(x), int(N), int(D), ctypes.c_float(eps), int(width_req),
+                                   int(r), _ptr(codes), _nbytes(codes), _ptr(digests),
+                                   _ptr(workspace), _nbytes(workspace), ctypes.byref(w),
+                                   ctypes.byref(sc), ctypes.byref(cmin), ctypes.byref(cmax),
+                                   _stream(stream, x.device))
+    if raise_on_error:
+        _check(st, "lam_quantize_bands")
+    return st, w.value, sc.value, cmin.value, cmax.value
 
 
 def lam_code_sqnorms(codes, width, N, D, sqnorm_out, stream=None) -> None:

@@ -179,6 +179,40 @@ void timing_launch_end(int kind, cudaStream_t st) {
 
 }  // namespace lam
 
+namespace lam {
+namespace {
+// Host outputs and status of a finished Q_eps pass from its status block.
+lam_status decode_quant_status(const QuantStatus &h, int32_t width_req, float s,
+                               int32_t *width_out, float *scale_out, int32_t *code_min_out,
+                               int32_t *code_max_out) {
+  if (h.flags & kFlagTimeout) return LAM_ERR_TIMEOUT;
+  if (h.flags & kFlagNonfinite) return LAM_ERR_NONFINITE;
+  float rmin = 0.0f, rmax = 0.0f;
+  if (h.neg_min != 0) {
+    rmin = host_qround(unord_host(~h.neg_min), s);
+    rmax = host_qround(unord_host(h.max), s);
+  }
+  const int need = width_of(rmin, rmax);
+  const int w = width_req == LAM_WIDTH_AUTO ? need : width_req;
+  if (scale_out) *scale_out = s;
+  if (width_out) *width_out = w;
+  if (need != 0) {
+    if (code_min_out) *code_min_out = (int32_t)rmin;
+    if (code_max_out) *code_max_out = (int32_t)rmax;
+  } else {
+    if (code_min_out) *code_min_out = rmin < -2147483648.0f ? INT32_MIN : (int32_t)rmin;
+    if (code_max_out) *code_max_out = rmax >= 2147483648.0f ? INT32_MAX : (int32_t)rmax;
+  }
+  if (need == 0 || (h.flags & kFlagRange)) return LAM_ERR_RANGE;
+  if (width_req != LAM_WIDTH_AUTO && need > width_req) return LAM_ERR_RANGE;
+  if (width_req == LAM_WIDTH_AUTO && (int)h.width != need) return LAM_ERR_CUDA;  // must agree
+  if (h.flags & kFlagWorkspace) return LAM_ERR_WORKSPACE;
+  return LAM_OK;
+}
+
+}  // namespace
+}  // namespace lam
+
 extern "C" {
 
 int32_t lam_version(void) { return 100; }
@@ -261,29 +295,72 @@ lam_status lam_quantize(const float *x, int64_t n, float eps, int32_t width_req,
     if (cudaStreamSynchronize(st) != cudaSuccess) return LAM_ERR_CUDA;
     h.width = width_resolved;
   }
-  if (h.flags & kFlagTimeout) return LAM_ERR_TIMEOUT;
-  if (h.flags & kFlagNonfinite) return LAM_ERR_NONFINITE;
-  float rmin = 0.0f, rmax = 0.0f;
-  if (h.neg_min != 0) {
-    rmin = host_qround(unord_host(~h.neg_min), s);
-    rmax = host_qround(unord_host(h.max), s);
+  return lam::decode_quant_status(h, width_req, s, width_out, scale_out, code_min_out,
+                                  code_max_out);
+}
+
+lam_status lam_quantize_bands(const float *x, int64_t N, int32_t D, float eps, int32_t width_req,
+                              int32_t r, void *codes, size_t codes_bytes, uint64_t *digests,
+                              void *workspace, size_t workspace_bytes, int32_t *width_out,
+                              float *scale_out, int32_t *code_min_out, int32_t *code_max_out,
+                              lam_stream_t stream) {
+  if (N < 0 || D < 1 || r < 1 || r > D || D % r != 0 || D / r > 65536 || !valid_eps(eps))
+    return LAM_ERR_INVALID;
+  if (N > (1LL << 62) / D) return LAM_ERR_INVALID;
+  if (width_req != LAM_WIDTH_AUTO && !valid_width(width_req)) return LAM_ERR_INVALID;
+  const int64_t n = N * (int64_t)D;
+  if (n > 0 && (x == nullptr || digests == nullptr)) return LAM_ERR_INVALID;
+  if ((reinterpret_cast<uintptr_t>(x) & 3u) != 0 ||
+      (reinterpret_cast<uintptr_t>(digests) & 7u) != 0)
+    return LAM_ERR_INVALID;
+  const uintptr_t calign = width_req == LAM_WIDTH_AUTO ? 4u : (uintptr_t)width_req;
+  if (codes != nullptr && (reinterpret_cast<uintptr_t>(codes) & (calign - 1)) != 0)
+    return LAM_ERR_INVALID;
+  const float s = 2.0f * eps;
+  if (n == 0) {
+    if (width_out) *width_out = width_req == LAM_WIDTH_AUTO ? 1 : width_req;
+    if (scale_out) *scale_out = s;
+    if (code_min_out) *code_min_out = 0;
+    if (code_max_out) *code_max_out = 0;
+    return LAM_OK;
   }
-  const int need = width_of(rmin, rmax);
-  const int w = width_req == LAM_WIDTH_AUTO ? need : width_req;
-  if (scale_out) *scale_out = s;
-  if (width_out) *width_out = w;
-  if (need != 0) {
-    if (code_min_out) *code_min_out = (int32_t)rmin;
-    if (code_max_out) *code_max_out = (int32_t)rmax;
-  } else {
-    if (code_min_out) *code_min_out = rmin < -2147483648.0f ? INT32_MIN : (int32_t)rmin;
-    if (code_max_out) *code_max_out = rmax >= 2147483648.0f ? INT32_MAX : (int32_t)rmax;
+  if (workspace == nullptr || (reinterpret_cast<uintptr_t>(workspace) & 15u) != 0)
+    return LAM_ERR_INVALID;
+  if (workspace_bytes < sizeof(QuantStatus)) return LAM_ERR_WORKSPACE;
+  if (codes != nullptr && width_req != LAM_WIDTH_AUTO &&
+      (unsigned long long)n * (unsigned long long)width_req > codes_bytes)
+    return LAM_ERR_WORKSPACE;
+  const int sms = device_sms();
+  if (sms <= 0) return LAM_ERR_CUDA;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  QuantStatus *dst = static_cast<QuantStatus *>(workspace);
+  if (cudaMemsetAsync(dst, 0, sizeof(QuantStatus), st) != cudaSuccess) return LAM_ERR_CUDA;
+  timing_launch_begin(LAM_TIME_QUANTIZE, st);
+  cudaError_t e = launch_quantize_bands(x, N, D, r, s, width_req, codes, codes_bytes, digests,
+                                        dst, sms, st);
+  timing_launch_end(LAM_TIME_QUANTIZE, st);
+  if (e != cudaSuccess) return LAM_ERR_CUDA;
+  QuantStatus h;
+  if (cudaMemcpyAsync(&h, dst, sizeof(h), cudaMemcpyDeviceToHost, st) != cudaSuccess)
+    return LAM_ERR_CUDA;
+  if (cudaStreamSynchronize(st) != cudaSuccess) return LAM_ERR_CUDA;
+  if (width_req == LAM_WIDTH_AUTO && h.passes == 2 &&
+      !(h.flags & (kFlagTimeout | kFlagNonfinite | kFlagRange | kFlagWorkspace)) &&
+      (h.width == 1 || h.width == 2 || h.width == 4)) {
+    // the width speculated from the sample was too narrow: hash again at the exact one
+    timing_launch_begin(LAM_TIME_QUANTIZE, st);
+    e = launch_quantize_bands(x, N, D, r, s, (int)h.width, codes, codes_bytes, digests, dst, sms,
+                              st);
+    timing_launch_end(LAM_TIME_QUANTIZE, st);
+    if (e != cudaSuccess) return LAM_ERR_CUDA;
+    const uint32_t width_resolved = h.width;
+    if (cudaMemcpyAsync(&h, dst, sizeof(h), cudaMemcpyDeviceToHost, st) != cudaSuccess)
+      return LAM_ERR_CUDA;
+    if (cudaStreamSynchronize(st) != cudaSuccess) return LAM_ERR_CUDA;
+    h.width = width_resolved;
   }
-  if (need == 0 || (h.flags & kFlagRange)) return LAM_ERR_RANGE;
-  if (width_req != LAM_WIDTH_AUTO && need > width_req) return LAM_ERR_RANGE;
-  if (width_req == LAM_WIDTH_AUTO && (int)h.width != need) return LAM_ERR_CUDA;  // must agree
-  if (h.flags & kFlagWorkspace) return LAM_ERR_WORKSPACE;
-  return LAM_OK;
+  return lam::decode_quant_status(h, width_req, s, width_out, scale_out, code_min_out,
+                                  code_max_out);
 }
 
 lam_status lam_dequantize(const void *codes, int32_t width, int64_t n, float scale, float *out,

@@ -149,6 +149,11 @@ cudaError_t launch_quant_range(const float *x, int64_t n, QuantStatus *status, i
 cudaError_t launch_quantize(const float *x, int64_t n, float s, int width_req, void *codes,
                             size_t codes_bytes, QuantStatus *status, int sms,
                             cudaStream_t st);
+// Q_eps fused with the band digests (width_req 1/2/4 forced, 0 AUTO).
+cudaError_t launch_quantize_bands(const float *x, int64_t N, int D, int r, float s,
+                                  int width_req, void *codes, size_t codes_bytes,
+                                  uint64_t *digests, QuantStatus *st, int sms,
+                                  cudaStream_t stream);
 cudaError_t launch_code_sqnorms(const void *codes, int width, int64_t N, int D, float *out,
                                 int sms, cudaStream_t st);
 cudaError_t launch_dequantize(const void *codes, int width, int64_t n, float s, float *out,

@@ -149,3 +149,16 @@ def test_timing_read_rejects_bad_kind_and_end_is_idempotent(lib):
 def test_code_sqnorms_rejects_bad_arguments(lib, width, N, D, codes, out):
     c = ctypes
     assert lib.lam_code_sqnorms(c.c_void_p(codes), width, N, D, c.c_void_p(out), None) == 1
+
+
+@pytest.mark.parametrize("N,D,r,width,x,dig", [(4, 8, 3, 0, 256, 512), (4, 8, 0, 0, 256, 512),
+                                              (4, 8, 16, 0, 256, 512), (-1, 8, 2, 0, 256, 512),
+                                              (4, 8, 2, 3, 256, 512), (4, 8, 2, 0, 258, 512),
+                                              (4, 8, 2, 0, 256, 516), (4, 8, 2, 0, 0, 512),
+                                              (4, 8, 2, 0, 256, 0)])
+def test_quantize_bands_rejects_bad_arguments(lib, N, D, r, width, x, dig):
+    c = ctypes
+    st = lib.lam_quantize_bands(c.c_void_p(x), N, D, c.c_float(1e-3), width, r, None, 0,
+                                c.c_void_p(dig), c.c_void_p(1024), 64, None, None, None, None,
+                                None)
+    assert st == 1
