@@ -72,6 +72,11 @@ def _load():
         lib.lam_oracle_band_digests.argtypes = [i32p, ctypes.c_int64, ctypes.c_int32,
                                                 ctypes.c_int32, ctypes.c_int32, u64p]
         lib.lam_oracle_band_digests.restype = None
+        lib.lam_oracle_admit_batch.argtypes = [f32p, ctypes.c_int64, ctypes.c_int32, u64p,
+                                               ctypes.c_int32, ctypes.c_double, i32p,
+                                               ctypes.POINTER(ctypes.c_double),
+                                               ctypes.POINTER(ctypes.c_double)]
+        lib.lam_oracle_admit_batch.restype = ctypes.c_int64
         lib.lam_oracle_code_sqnorms.argtypes = [i32p, ctypes.c_int64, ctypes.c_int32, f32p]
         lib.lam_oracle_code_sqnorms.restype = None
         lib.lam_oracle_scores.argtypes = [f32p, ctypes.c_int64, i32p, ctypes.c_int64,
@@ -152,6 +157,23 @@ def band_digests(codes: np.ndarray, r: int, width: int) -> np.ndarray:
     _load().lam_oracle_band_digests(_ptr(c, ctypes.c_int32), N, D, r, width,
                                     _ptr(out, ctypes.c_uint64))
     return out
+
+
+def admit_batch(e: np.ndarray, digests: np.ndarray, delta: float):
+    """Batch admission (Algorithm 2) of the fp32 rows e [N, D] with band
+    digests [N, nb]: (rep int32 [N], dist float64 [N], delta_hat, n_retained)."""
+    x = np.ascontiguousarray(e, dtype=np.float32)
+    dg = np.ascontiguousarray(digests, dtype=np.uint64)
+    N, D = x.shape
+    nb = dg.shape[1]
+    rep = np.empty(N, dtype=np.int32)
+    dist = np.empty(N, dtype=np.float64)
+    dh = ctypes.c_double(0.0)
+    kept = _load().lam_oracle_admit_batch(_ptr(x, ctypes.c_float), N, D,
+                                          _ptr(dg, ctypes.c_uint64), nb, float(delta),
+                                          _ptr(rep, ctypes.c_int32),
+                                          _ptr(dist, ctypes.c_double), ctypes.byref(dh))
+    return rep, dist, dh.value, int(kept)
 
 
 def code_sqnorms(codes: np.ndarray) -> np.ndarray:

@@ -166,7 +166,90 @@ void lam_oracle_band_digests(const int32_t *codes, int64_t N, int32_t D, int32_t
   }
 }
 
-/* Score of one query against one dequantised row, in double, rounded to fp32. *//* Score of one query against one dequantised row, in double, rounded to fp32. */
+/*
+ * Batch form of the admission rule (Algorithm 2; Sec. 3.3 "The eps
+ * error-bounded test"): records 0..N-1 in order; record i's candidates are the
+ * retained records that share a band digest with it in the same band
+ * (BandHash(Q_eps(e_y)) and BandHash(Q_eps(e_i)) intersect; the band index
+ * holds retained records only); its representative is the lowest-indexed
+ * candidate within l2 distance delta (Eq. 2: delta = sqrt(2 - 2t) for merge
+ * threshold t), else it is retained and becomes its own representative.
+ * Distances are taken in full precision: the squared difference of each
+ * coordinate in double, summed in coordinate order, then one sqrt.
+ * Outputs: rep[i] (representative index, i itself when retained), dist[i]
+ * (distance to it, 0 when retained) and the measured bound delta_hat = the
+ * largest distance of a merge (0 when nothing merges).  Returns the number of
+ * retained records.
+ */
+static double l2_full(const float *a, const float *b, int32_t D) {
+  double acc = 0.0;
+  for (int32_t d = 0; d < D; ++d) {
+    const double t = (double)a[d] - (double)b[d];
+    acc += t * t;
+  }
+  return sqrt(acc);
+}
+
+int64_t lam_oracle_admit_batch(const float *e, int64_t N, int32_t D, const uint64_t *digests,
+                               int32_t nb, double delta, int32_t *rep, double *dist,
+                               double *delta_hat) {
+  /* per band: open-addressing table digest -> most recent retained id with it,
+   * and for every (band, retained id) the previous retained id with the same
+   * digest in that band (a linked list, newest first) */
+  int64_t cap = 16;
+  while (cap < 2 * N + 2) cap <<= 1;
+  int64_t *tab_key_id = (int64_t *)malloc(sizeof(int64_t) * (size_t)cap * (size_t)nb);
+  int32_t *prev = (int32_t *)malloc(sizeof(int32_t) * (size_t)N * (size_t)nb);
+  int64_t *seen = (int64_t *)malloc(sizeof(int64_t) * (size_t)(N > 0 ? N : 1));
+  for (int64_t i = 0; i < cap * nb; ++i) tab_key_id[i] = -1;
+  for (int64_t i = 0; i < N; ++i) seen[i] = -1;
+  int64_t retained = 0;
+  double dh = 0.0;
+  for (int64_t i = 0; i < N; ++i) {
+    int64_t best = -1;
+    double best_d = 0.0;
+    for (int32_t b = 0; b < nb; ++b) {
+      const uint64_t key = digests[i * nb + b];
+      int64_t *tab = tab_key_id + (size_t)b * (size_t)cap;
+      int64_t slot = (int64_t)(key & (uint64_t)(cap - 1));
+      while (tab[slot] >= 0 && digests[tab[slot] * nb + b] != key) slot = (slot + 1) & (cap - 1);
+      for (int64_t y = tab[slot]; y >= 0; y = prev[y * nb + b]) {
+        if (seen[y] == i) continue; /* already a candidate through another band */
+        seen[y] = i;
+        if (best >= 0 && y > best) continue; /* cannot lower the representative */
+        const double dd = l2_full(e + i * (int64_t)D, e + y * (int64_t)D, D);
+        if (dd <= delta && (best < 0 || y < best)) {
+          best = y;
+          best_d = dd;
+        }
+      }
+    }
+    if (best >= 0) {
+      rep[i] = (int32_t)best;
+      dist[i] = best_d;
+      if (best_d > dh) dh = best_d;
+    } else {
+      rep[i] = (int32_t)i;
+      dist[i] = 0.0;
+      ++retained;
+      for (int32_t b = 0; b < nb; ++b) {
+        const uint64_t key = digests[i * nb + b];
+        int64_t *tab = tab_key_id + (size_t)b * (size_t)cap;
+        int64_t slot = (int64_t)(key & (uint64_t)(cap - 1));
+        while (tab[slot] >= 0 && digests[tab[slot] * nb + b] != key) slot = (slot + 1) & (cap - 1);
+        prev[i * nb + b] = tab[slot] >= 0 ? (int32_t)tab[slot] : -1;
+        tab[slot] = i;
+      }
+    }
+  }
+  free(tab_key_id);
+  free(prev);
+  free(seen);
+  *delta_hat = dh;
+  return retained;
+}
+
+/* Score of one query against one dequantised row, in double, rounded to fp32. *//* Score of one query against one dequantised row, in double, rounded to fp32. *//* Score of one query against one dequantised row, in double, rounded to fp32. */
 static float score_one(const float *q, const int32_t *c, int32_t D, float s,
                        int metric) {
   if (metric == ORACLE_IP) {

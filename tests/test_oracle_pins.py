@@ -324,3 +324,68 @@ def test_band_digest_of_a_single_band_is_the_fnv_of_its_bytes():
         want = oracle.fnv1a64(int(code).to_bytes(4, "little", signed=True)[:width],
                               oracle.fnv1a64(b"\x00\x00"))
         assert int(got) == want
+
+
+def test_admit_batch_worked_line_cases():
+    for case, delta, pos, reps, dh in golden("admit_line.txt"):
+        x = np.array([[float(p), 0.0] for p in pos.split(",")], dtype=np.float32)
+        rep, dist, delta_hat, kept = oracle.admit_batch(x, np.zeros((len(x), 1), np.uint64),
+                                                        float(delta))
+        assert rep.tolist() == [int(v) for v in reps.split(",")], case
+        assert abs(delta_hat - float(dh)) < 1e-6, case
+        assert kept == len(set(rep.tolist()))
+
+
+def _lsh_rows(n, seed, dup_every=7):
+    x = inputs.unit_rows(n, 64, seed=seed)
+    rng = np.random.default_rng(seed)
+    for i in range(dup_every, n, dup_every):  # near-duplicates of earlier rows
+        j = int(rng.integers(0, i))
+        v = x[j] + rng.normal(0, 0.03, size=64).astype(np.float32)
+        x[i] = v / np.linalg.norm(v)
+    return x
+
+
+def test_admit_batch_cover_packing_and_lowest_index_with_all_pairs_candidates():
+    x = _lsh_rows(300, 21)
+    delta = float(np.sqrt(2 - 2 * 0.95))
+    rep, dist, dh, kept = oracle.admit_batch(x, np.zeros((300, 1), np.uint64), delta)
+    R = np.nonzero(rep == np.arange(300))[0]
+    d = np.linalg.norm(x[:, None, :].astype(np.float64) - x[None, :, :], axis=2)
+    # cover: every merged row lies within delta of an earlier retained row
+    for i in np.nonzero(rep != np.arange(300))[0]:
+        assert rep[i] < i and rep[rep[i]] == rep[i] and d[i, rep[i]] <= delta
+        # lowest index: no retained row below the representative is within delta
+        assert not np.any(d[i, R[R < rep[i]]] <= delta)
+    # packing: retained rows are pairwise farther apart than delta (Prop. 2)
+    dr = d[np.ix_(R, R)] + np.eye(len(R)) * 10
+    assert dr.min() > delta
+    assert kept == len(R) and dh == pytest.approx(max(dist.max(), 0.0))
+
+
+def test_admit_batch_score_deficit_bound_and_prefix_stability():
+    x = _lsh_rows(400, 22)
+    delta = float(np.sqrt(2 - 2 * 0.9))
+    oc, *_ = oracle.quantize(x, 0.05)
+    dig = oracle.band_digests(oc.reshape(x.shape), 4, oracle.width(*oracle.quantize(x, 0.05)[1:3]))
+    rep, dist, dh, kept = oracle.admit_batch(x, dig, delta)
+    R = np.nonzero(rep == np.arange(400))[0]
+    # Theorem 1: for unit queries 0 <= max_S q.x - max_R q.z <= delta_hat <= delta
+    q = inputs.queries(200, 64, seed=5).astype(np.float64)
+    gap = (q @ x.T.astype(np.float64)).max(1) - (q @ x[R].T.astype(np.float64)).max(1)
+    assert gap.min() >= 0 and gap.max() <= dh + 1e-12 and dh <= delta
+    # decisions are never revised: a prefix decides exactly as in the whole run
+    rep_p, *_ = oracle.admit_batch(x[:250], dig[:250], delta)
+    np.testing.assert_array_equal(rep_p, rep[:250])
+
+
+def test_admit_batch_only_band_candidates_merge():
+    # two identical rows with no digest in common are not candidates
+    x = np.array([[1.0, 0.0], [1.0, 0.0], [1.0, 0.0]], dtype=np.float32)
+    dig = np.array([[5], [6], [5]], dtype=np.uint64)
+    rep, dist, dh, kept = oracle.admit_batch(x, dig, 0.1)
+    assert rep.tolist() == [0, 1, 0] and kept == 2
+    # digests match only within the same band position
+    dig2 = np.array([[5, 9], [9, 5]], dtype=np.uint64)
+    rep, *_ = oracle.admit_batch(x[:2], dig2, 0.1)
+    assert rep.tolist() == [0, 1]
