@@ -640,6 +640,35 @@ def run_kernels(args):
                                      "gbs_kernel": nbytes / (k_ms / 1e3) / 1e9,
                                      "frac_of_hbm_kernel": nbytes / (k_ms / 1e3) / 1e9 / hbm})
             del dig
+    if wl.planted:
+        # batch admission (Algorithm 2) at cos >= 0.95 over band candidates at
+        # the paper's shipped (r = 4, eps = 0.2 sigma) and relaxed (r = 8, 0.3 sigma)
+        # operating points: digests from the fused pass, then lam_admit_batch
+        res["admit"] = []
+        N, sigma = wl.n, 1.0 / (wl.d ** 0.5)
+        delta = (2.0 - 2.0 * 0.95) ** 0.5
+        xr = x.view(N, wl.d)
+        for r, rel in ((4, 0.2), (8, 0.3)):
+            dig = torch.empty((N, wl.d // r), dtype=torch.int64, device=dev)
+            lam.lam_quantize_bands(xr, rel * sigma, 0, r, None, dig, ws)
+            rep = torch.empty(N, dtype=torch.int32, device=dev)
+            dist = torch.empty(N, dtype=torch.float64, device=dev)
+            mp = 1 << 20
+            while True:
+                aws = torch.empty(lam.lam_admit_batch_workspace_size(N, wl.d // r, mp),
+                                  dtype=torch.uint8, device=dev)
+                st, dh, kept, npairs = lam.lam_admit_batch(xr, dig, delta, rep, dist, aws, mp,
+                                                           raise_on_error=False)
+                if st == 0:
+                    break
+                mp = npairs
+                del aws
+            ms, _ = timed(lambda: lam.lam_admit_batch(xr, dig, delta, rep, dist, aws, mp),
+                          lam.LAM_TIME_AUX)
+            res["admit"].append({"r": r, "eps": rel * sigma, "t": 0.95, "ms_span": ms,
+                                 "records_per_s": N / (ms / 1e3), "candidate_pairs": npairs,
+                                 "retained": kept, "delta_hat": dh})
+            del aws, dig
     if wl.batches and wl.d > 1:
         e = eps_list[0]
         wq, sc, bound = widths[e]

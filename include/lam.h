@@ -135,6 +135,40 @@ lam_status lam_quantize_bands(const float *x, int64_t N, int32_t D, float eps,
                               lam_stream_t stream);
 
 /*
+ * lam_admit_batch -- the batch form of the admission rule (Algorithm 2;
+ * Sec. 3.3): records 0..N-1 in order; the candidates of record i are the
+ * retained records that share a band digest with it in the same band (the
+ * digests of lam_quantize_bands); its representative is the lowest-indexed
+ * candidate within l2 distance delta of it (delta = sqrt(2 - 2t) for merge
+ * threshold t, Eq. 2), else record i is retained.  Distances are taken in
+ * full precision: per coordinate the difference of the two fp32 values in
+ * double, squared, summed in coordinate order without fused multiply-adds,
+ * then one sqrt; a pair is within delta when that distance is <= delta.
+ *
+ * e         [N, D] fp32 embeddings, device, 4-byte aligned.
+ * digests   [N, nb] uint64 band digests, device, 8-byte aligned.
+ * rep       [N] int32 out: representative of each record (itself if retained).
+ * dist      [N] double out: distance to the representative (0 if retained).
+ * workspace >= lam_admit_batch_workspace_size(N, nb, max_pairs) bytes of
+ *           device memory, 256-byte aligned; max_pairs bounds the number of
+ *           (row, lower row) candidate pairs before de-duplication.
+ * delta_hat_out (host, may be NULL): the measured bound, the largest merge
+ *           distance (0 when nothing merges); n_retained_out: |R|;
+ *           n_pairs_out: candidate pairs found.
+ * Synchronous on `stream`.  Errors: LAM_ERR_INVALID (bad sizes, NULL or
+ * misaligned pointers, delta negative or not finite, N > 2^31 - 1, N * nb >=
+ * 2^32), LAM_ERR_WORKSPACE (workspace too small, or more candidate pairs than
+ * max_pairs: *n_pairs_out then holds the count needed), LAM_ERR_CUDA.
+ */
+size_t lam_admit_batch_workspace_size(int64_t N, int32_t nb, int64_t max_pairs);
+lam_status lam_admit_batch(const float *e, int64_t N, int32_t D,
+                           const uint64_t *digests, int32_t nb, double delta,
+                           int32_t *rep, double *dist, void *workspace,
+                           size_t workspace_bytes, int64_t max_pairs,
+                           double *delta_hat_out, int64_t *n_retained_out,
+                           int64_t *n_pairs_out, lam_stream_t stream);
+
+/*
  * lam_dequantize -- xhat_i = fl32(scale * code_i), the inverse map of Q_eps
  * up to the cell half-width eps (|x - xhat| <= eps, Sec. 3.1).
  *

@@ -57,6 +57,9 @@ def load():
         "lam_score_topk_noalloc": (i32, [vp, i64, vp, i32, i64, i32, f32, i32, i32, i32, vp,
                                          vp, vp]),
         "lam_code_sqnorms": (i32, [vp, i32, i64, i32, vp, vp]),
+        "lam_admit_batch_workspace_size": (sz, [i64, i32, i64]),
+        "lam_admit_batch": (i32, [vp, i64, i32, vp, i32, ctypes.c_double, vp, vp, vp, sz, i64,
+                                  P(ctypes.c_double), P(i64), P(i64), vp]),
         "lam_quantize_bands": (i32, [vp, i64, i32, f32, i32, i32, vp, sz, vp, vp, sz, P(i32),
                                      P(f32), P(i32), P(i32), vp]),
         "lam_timing_begin": (i32, [i32, i64]),
@@ -186,6 +189,27 @@ def lam_quantize_bands(x, eps, width_req, r, codes, digests, workspace, stream=N
     if raise_on_error:
         _check(st, "lam_quantize_bands")
     return st, w.value, sc.value, cmin.value, cmax.value
+
+
+def lam_admit_batch_workspace_size(N, nb, max_pairs) -> int:
+    return int(load().lam_admit_batch_workspace_size(int(N), int(nb), int(max_pairs)))
+
+
+def lam_admit_batch(e, digests, delta, rep, dist, workspace, max_pairs, stream=None,
+                    raise_on_error=True):
+    """Batch admission of the fp32 rows e [N, D] over their band digests
+    [N, nb]; fills rep (int32 [N]) and dist (float64 [N]).  Returns
+    (status, delta_hat, n_retained, n_pairs)."""
+    N, D = e.shape
+    nb = digests.shape[1]
+    dh, kept, np_ = ctypes.c_double(0), ctypes.c_int64(0), ctypes.c_int64(0)
+    st = load().lam_admit_batch(_ptr(e), int(N), int(D), _ptr(digests), int(nb),
+                                ctypes.c_double(delta), _ptr(rep), _ptr(dist), _ptr(workspace),
+                                _nbytes(workspace), int(max_pairs), ctypes.byref(dh),
+                                ctypes.byref(kept), ctypes.byref(np_), _stream(stream, e.device))
+    if raise_on_error:
+        _check(st, "lam_admit_batch")
+    return st, dh.value, kept.value, np_.value
 
 
 def lam_code_sqnorms(codes, width, N, D, sqnorm_out, stream=None) -> None:

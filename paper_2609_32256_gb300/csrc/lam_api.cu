@@ -363,6 +363,53 @@ lam_status lam_quantize_bands(const float *x, int64_t N, int32_t D, float eps, i
                                   code_max_out);
 }
 
+size_t lam_admit_batch_workspace_size(int64_t N, int32_t nb, int64_t max_pairs) {
+  if (N < 0 || N > INT32_MAX || nb < 1 || max_pairs < 0 || max_pairs > INT32_MAX ||
+      (N * (int64_t)nb) > (int64_t)UINT32_MAX)
+    return 0;
+  return admit_workspace_bytes(N, nb, max_pairs);
+}
+
+lam_status lam_admit_batch(const float *e, int64_t N, int32_t D, const uint64_t *digests,
+                           int32_t nb, double delta, int32_t *rep, double *dist,
+                           void *workspace, size_t workspace_bytes, int64_t max_pairs,
+                           double *delta_hat_out, int64_t *n_retained_out,
+                           int64_t *n_pairs_out, lam_stream_t stream) {
+  if (N < 0 || N > INT32_MAX || D < 1 || nb < 1 || max_pairs < 0 || max_pairs > INT32_MAX ||
+      !(delta >= 0.0) || !isfinite(delta) || (N * (int64_t)nb) > (int64_t)UINT32_MAX)
+    return LAM_ERR_INVALID;
+  if (n_pairs_out) *n_pairs_out = 0;
+  if (N == 0) {
+    if (delta_hat_out) *delta_hat_out = 0.0;
+    if (n_retained_out) *n_retained_out = 0;
+    return LAM_OK;
+  }
+  if (e == nullptr || digests == nullptr || rep == nullptr || dist == nullptr ||
+      workspace == nullptr)
+    return LAM_ERR_INVALID;
+  if ((reinterpret_cast<uintptr_t>(e) & 3u) || (reinterpret_cast<uintptr_t>(digests) & 7u) ||
+      (reinterpret_cast<uintptr_t>(rep) & 3u) || (reinterpret_cast<uintptr_t>(dist) & 7u) ||
+      (reinterpret_cast<uintptr_t>(workspace) & 255u))
+    return LAM_ERR_INVALID;
+  if (workspace_bytes < admit_workspace_bytes(N, nb, max_pairs)) return LAM_ERR_WORKSPACE;
+  const int sms = device_sms();
+  if (sms <= 0) return LAM_ERR_CUDA;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  int64_t np = 0, kept = 0;
+  double dh = 0.0;
+  bool overflow = false;
+  timing_launch_begin(LAM_TIME_AUX, st);
+  const cudaError_t err = launch_admit_batch(e, N, D, digests, nb, delta, rep, dist, workspace,
+                                             max_pairs, sms, st, &np, &dh, &kept, &overflow);
+  timing_launch_end(LAM_TIME_AUX, st);
+  if (err != cudaSuccess) return LAM_ERR_CUDA;
+  if (n_pairs_out) *n_pairs_out = np;
+  if (overflow) return LAM_ERR_WORKSPACE;
+  if (delta_hat_out) *delta_hat_out = dh;
+  if (n_retained_out) *n_retained_out = kept;
+  return LAM_OK;
+}
+
 lam_status lam_dequantize(const void *codes, int32_t width, int64_t n, float scale, float *out,
                           lam_stream_t stream) {
   if (n < 0 || !valid_width(width) || !isfinite(scale)) return LAM_ERR_INVALID;

@@ -154,6 +154,12 @@ cudaError_t launch_quantize_bands(const float *x, int64_t N, int D, int r, float
                                   int width_req, void *codes, size_t codes_bytes,
                                   uint64_t *digests, QuantStatus *st, int sms,
                                   cudaStream_t stream);
+// Batch admission (admit.cu).
+size_t admit_workspace_bytes(int64_t N, int nb, int64_t max_pairs);
+cudaError_t launch_admit_batch(const float *e, int64_t N, int D, const uint64_t *dig, int nb,
+                               double delta, int32_t *rep, double *dist, void *ws,
+                               int64_t max_pairs, int sms, cudaStream_t st, int64_t *n_pairs,
+                               double *delta_hat, int64_t *n_retained, bool *overflow);
 cudaError_t launch_code_sqnorms(const void *codes, int width, int64_t N, int D, float *out,
                                 int sms, cudaStream_t st);
 cudaError_t launch_dequantize(const void *codes, int width, int64_t n, float s, float *out,
