@@ -213,6 +213,10 @@ class Pipeline:
             wsz = max(wsz, lam.lam_score_topk_workspace_size(self.B, self.N, self.D, k, w, bound))
             self.plan.append((w, bound, lam.lam_score_topk_path(self.B, self.N, self.D, k, w, bound)))
         self.sws = torch.empty(wsz, dtype=torch.uint8, device=dev)
+        # a second search stream (and workspace): the short kernels of one
+        # search overlap the scoring kernel of the next
+        self.ss2 = torch.cuda.Stream(dev)
+        self.sws2 = torch.empty(wsz, dtype=torch.uint8, device=dev)
 
     def step_overlapped(self):
         """The step as a user would drive it: Q_eps of each eps on one stream
@@ -226,13 +230,15 @@ class Pipeline:
             st, w, s, cmin, cmax = lam.lam_quantize(self.x, e, 0, self.codes_e[j], self.qws,
                                                     stream=self.sq.cuda_stream)
             self.qdone[j].record(self.sq)
+            ss, sws = (self.ss, self.sws) if j % 2 == 0 else (self.ss2, self.sws2)
             self.sd.wait_event(self.qdone[j])
-            self.ss.wait_event(self.qdone[j])
+            ss.wait_event(self.qdone[j])
             lam.lam_dequantize(self.codes_e[j], w, n, s, self.deq, stream=self.sd.cuda_stream)
             lam.lam_score_topk(self.q, self.codes_e[j], w, self.N, self.D, e, max(-cmin, cmax),
-                               self.k, self.metric, self.scores[j], self.ids[j], self.sws,
-                               stream=self.ss.cuda_stream)
-        self.ss.wait_stream(self.sd)  # the step ends when both have finished
+                               self.k, self.metric, self.scores[j], self.ids[j], sws,
+                               stream=ss.cuda_stream)
+        self.ss.wait_stream(self.sd)  # the step ends when all have finished
+        self.ss.wait_stream(self.ss2)
 
     def step(self, ev=None):
         """The step with every call in order on the current stream (per-stage
@@ -309,6 +315,7 @@ def run_lam(args):
     def overlapped_step(i, e0, e1):
         # the previous step is finished and L2 is flushed before the step starts
         pipe.sq.wait_stream(pipe.ss)
+        pipe.sq.wait_stream(pipe.ss2)
         pipe.sq.wait_stream(pipe.sd)
         pipe.sq.wait_stream(cur)
         with torch.cuda.stream(pipe.sq):
@@ -432,6 +439,7 @@ def run_lam(args):
         pipe.ss.wait_event(e0)
         with torch.cuda.stream(pipe.ss):
             q.copy_(q_h, non_blocking=True)  # ordered before the searches on this stream
+        pipe.ss2.wait_stream(pipe.ss)         # and on the other search stream
         pipe.step_overlapped()
         with torch.cuda.stream(pipe.ss):
             for j in range(ne):
@@ -465,8 +473,8 @@ def run_lam(args):
                        "l2": "flushed between timed steps (512 MB write then 512 MB read, outside "
                              "the events)",
                        "step": "per eps: lam_quantize (synchronous) on one stream, lam_dequantize "
-                               "and lam_score_topk of its codes on two more; they overlap each "
-                               "other and the quantization of the next eps "
+                               "on a second and lam_score_topk on a third or fourth (alternating), "
+                               "so they overlap each other and the quantization of the next eps "
                                "(ms_per_step_serial: all on one stream)"},
             "breakdown": {
                 "quantize_ms": ms_q, "quantize_gbs_algorithmic": q_bytes / (ms_q / 1e3) / 1e9,
@@ -685,10 +693,17 @@ def run_kernels(args):
             ms, k_s = timed(lambda: lam.lam_score_topk(q, codes, wq, N, wl.d, e, bound, wl.k,
                                                        wl.metric, s_, i_, sws),
                             lam.LAM_TIME_SCORE)
+            _, k_m = timed(lambda: lam.lam_score_topk(q, codes, wq, N, wl.d, e, bound, wl.k,
+                                                      wl.metric, s_, i_, sws),
+                           lam.LAM_TIME_MERGE)
+            _, k_a = timed(lambda: lam.lam_score_topk(q, codes, wq, N, wl.d, e, bound, wl.k,
+                                                      wl.metric, s_, i_, sws),
+                           lam.LAM_TIME_AUX)
             code_bytes = N * wl.d * wq
             fl = 2.0 * N * wl.d * B
             res["score"].append({"B": B, "path": ["bandwidth", "tensor", "generic"][path],
-                                 "ms_span": ms, "ms_kernel": k_s,
+                                 "ms_span": ms, "ms_kernel": k_s, "ms_merge": k_m,
+                                 "ms_prep": k_a,
                                  "vectors_per_s_span": N / (ms / 1e3),
                                  "code_gbs_kernel": code_bytes / (k_s / 1e3) / 1e9,
                                  "frac_of_hbm_kernel": code_bytes / (k_s / 1e3) / 1e9 / hbm,

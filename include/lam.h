@@ -271,11 +271,12 @@ lam_status lam_code_sqnorms(const void *codes, int32_t width, int64_t N, int32_t
  *   LAM_TIME_SCORE       the fused score + top-k kernel of lam_score_topk
  *                        (one launch per row slab)
  *   LAM_TIME_AUX         every other kernel (query preparation, operand
- *                        conversion, range pass, list merge)
+ *                        conversion, range pass, admission)
+ *   LAM_TIME_MERGE       the merge of partial top-k lists of lam_score_topk
  * The events are created here (no allocation happens later on the timed
  * path).  Intended for one host thread driving one device; a later begin
  * replaces the earlier state.  Errors: LAM_ERR_INVALID for mask outside
- * 1..15 or capacity outside 0..1048576; LAM_ERR_CUDA if event creation fails.
+ * 1..31 or capacity outside 0..1048576; LAM_ERR_CUDA if event creation fails.
  *
  * lam_timing_read(kind, total_ms, timed, launches) waits for the recorded
  * events of one kind (a single bit of the mask) and returns the summed device
@@ -288,6 +289,7 @@ lam_status lam_code_sqnorms(const void *codes, int32_t width, int64_t N, int32_t
 #define LAM_TIME_DEQUANTIZE 2
 #define LAM_TIME_SCORE 4
 #define LAM_TIME_AUX 8
+#define LAM_TIME_MERGE 16
 
 lam_status lam_timing_begin(int32_t mask, int64_t capacity);
 lam_status lam_timing_read(int32_t kind, double *total_ms, int64_t *timed,

@@ -16,7 +16,7 @@ from ._lib import (LAM_ERR_CUDA, LAM_ERR_INVALID, LAM_ERR_NONFINITE, LAM_ERR_RAN
                    lam_dequantize, lam_quantize, lam_quantize_workspace_size,
                    lam_score_topk, lam_score_topk_path, lam_score_topk_status,
                    lam_score_topk_workspace_size, lam_status_string, lam_version, load,
-                   LAM_TIME_AUX, LAM_TIME_DEQUANTIZE, LAM_TIME_QUANTIZE, LAM_TIME_SCORE,
+                   LAM_TIME_AUX, LAM_TIME_MERGE, LAM_TIME_DEQUANTIZE, LAM_TIME_QUANTIZE, LAM_TIME_SCORE,
                    lam_timing_begin, lam_timing_end, lam_timing_read, lam_code_sqnorms,
                    lam_quantize_bands, lam_admit_batch, lam_admit_batch_workspace_size)
 

@@ -219,7 +219,7 @@ def lam_code_sqnorms(codes, width, N, D, sqnorm_out, stream=None) -> None:
     _check(st, "lam_code_sqnorms")
 
 
-LAM_TIME_QUANTIZE, LAM_TIME_DEQUANTIZE, LAM_TIME_SCORE, LAM_TIME_AUX = 1, 2, 4, 8
+LAM_TIME_QUANTIZE, LAM_TIME_DEQUANTIZE, LAM_TIME_SCORE, LAM_TIME_AUX, LAM_TIME_MERGE = 1, 2, 4, 8, 16
 
 
 def lam_timing_begin(mask, capacity) -> None:

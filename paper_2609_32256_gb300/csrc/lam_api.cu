@@ -137,14 +137,14 @@ struct Timing {
   std::vector<cudaEvent_t> ev;  // 2 per bracketed launch
   std::vector<int> kind;        // kind of each bracketed launch
   int64_t cap = 0, used = 0;
-  int64_t launches[4] = {0, 0, 0, 0};
+  int64_t launches[5] = {0, 0, 0, 0, 0};
   bool open = false;  // a begin without its end
 };
 Timing g_timing;
 
 int kind_index(int kind) {
   return kind == LAM_TIME_QUANTIZE ? 0 : kind == LAM_TIME_DEQUANTIZE ? 1
-         : kind == LAM_TIME_SCORE  ? 2 : 3;
+         : kind == LAM_TIME_SCORE  ? 2 : kind == LAM_TIME_MERGE ? 4 : 3;
 }
 
 void timing_release() {
@@ -539,7 +539,7 @@ lam_status lam_score_topk_status(const void *workspace, lam_stream_t stream, int
 
 
 lam_status lam_timing_begin(int32_t mask, int64_t capacity) {
-  if (mask < 1 || mask > 15 || capacity < 0 || capacity > (1 << 20)) return LAM_ERR_INVALID;
+  if (mask < 1 || mask > 31 || capacity < 0 || capacity > (1 << 20)) return LAM_ERR_INVALID;
   std::lock_guard<std::mutex> lk(lam::g_timing.mu);
   lam::timing_release();
   lam::g_timing.ev.reserve((size_t)capacity * 2);
@@ -559,7 +559,7 @@ lam_status lam_timing_begin(int32_t mask, int64_t capacity) {
 
 lam_status lam_timing_read(int32_t kind, double *total_ms, int64_t *timed, int64_t *launches) {
   if (kind != LAM_TIME_QUANTIZE && kind != LAM_TIME_DEQUANTIZE && kind != LAM_TIME_SCORE &&
-      kind != LAM_TIME_AUX)
+      kind != LAM_TIME_AUX && kind != LAM_TIME_MERGE)
     return LAM_ERR_INVALID;
   std::lock_guard<std::mutex> lk(lam::g_timing.mu);
   double tot = 0.0;

@@ -591,9 +591,9 @@ static cudaError_t launch_kmerge_t(const ScoreArgs &a, cudaStream_t st) {
   auto kern = topk_kmerge_kernel<HPL>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  timing_launch_begin(LAM_TIME_AUX, st);
+  timing_launch_begin(LAM_TIME_MERGE, st);
   kern<<<(unsigned)((a.B + qpc - 1) / qpc), kKmWarps * 32, smem, st>>>(a, (int)qpc);
-  timing_launch_end(LAM_TIME_AUX, st);
+  timing_launch_end(LAM_TIME_MERGE, st);
   return cudaGetLastError();
 }
 
@@ -614,9 +614,9 @@ cudaError_t launch_topk_merge(const ScoreArgs &a, cudaStream_t st) {
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   const int threads = P / 2 < 32 ? 32 : (P / 2 > kMergeThreads ? kMergeThreads : P / 2);
-  timing_launch_begin(LAM_TIME_AUX, st);
+  timing_launch_begin(LAM_TIME_MERGE, st);
   topk_merge_kernel<<<(unsigned)a.B, threads, smem, st>>>(a, P);
-  timing_launch_end(LAM_TIME_AUX, st);
+  timing_launch_end(LAM_TIME_MERGE, st);
   return cudaGetLastError();
 }
 

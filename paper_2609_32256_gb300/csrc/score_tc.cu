@@ -772,11 +772,13 @@ struct Tc2Layout {
 
 inline Tc2Layout tc2_layout(int k) {
   Tc2Layout L;
+  // (k <= 32 keeps its candidates in registers: no shared buffer, so that a
+  // seventh stage fits)
   const size_t lists = k > 32 ? (size_t)kBM * k * 8 : 0;
-  const size_t cbuf = k > 32 ? 0 : (size_t)kCBuf * kBM * 8;
+  const size_t cbuf = 0;
   const size_t tailb = 64 * 8 + 1024;
   int ns = (int)((kMaxDynSmem - lists - cbuf - tailb) / kStageBytes);
-  if (ns > 6) ns = 6;
+  if (ns > 7) ns = 7;
   L.ns = ns;
   L.lists_off = (size_t)ns * kStageBytes;
   L.cbuf_off = L.lists_off + lists;
@@ -802,7 +804,6 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
   uint8_t *smem = tc_smem_raw + (((base_u32 + 1023u) & ~1023u) - base_u32);
   const int ns = g.ns;
   uint64_t *lists = reinterpret_cast<uint64_t *>(smem + g.lists_off);
-  uint2 *cbuf = reinterpret_cast<uint2 *>(smem + g.cbuf_off);
   uint64_t *full = reinterpret_cast<uint64_t *>(smem + g.bar_off);
   uint64_t *empty = full + ns;
   uint64_t *accf = empty + ns;
@@ -922,7 +923,6 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
     reg.init(k);
     float thr_s = desc ? -INFINITY : INFINITY;
     float seed = desc ? -INFINITY : INFINITY;  // admission bound before the list fills
-    int cnt = 0;
     if (KR == 0)
       for (int i = 0; i < k; ++i) lists[(size_t)i * kBM + m] = kSentinel;
     for (int lt = 0; lt < ntl; ++lt) {
@@ -981,17 +981,23 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
         else if (nvalid < 32) mask &= (1u << nvalid) - 1u;
         const uint32_t grow0 = (uint32_t)(g.row_base + row0 + c * 32);  // global row id
         if (KR > 0) {
+          // one candidate per lane per step straight into the register list
+          // (re-tested against the threshold the earlier steps tightened)
           while (__any_sync(0xffffffffu, mask != 0)) {
             const int j = mask != 0 ? __ffs(mask) - 1 : 0;
             const float rf = __shfl_sync(0xffffffffu, rfl, j);
+            uint32_t kc = 0xffffffffu, ic = 0xffffffffu;
             if (mask != 0) {
               mask &= mask - 1;
               const float sc = tile_score(a.metric, __uint_as_float(select32(v, j)), fq, qq, rf);
-              cbuf[(size_t)cnt * kBM + m] = make_uint2(rank_key32(sc, desc), grow0 + j);
-              ++cnt;
+              if (desc ? sc > thr_s : sc < thr_s) {
+                kc = rank_key32(sc, desc);
+                ic = grow0 + j;
+              }
             }
-            if (__any_sync(0xffffffffu, cnt == kCBuf))
-              merge_candidates(reg, cbuf, m, kBM, cnt, thr_s, desc);
+            reg.insert(kc, ic);
+            const uint32_t tk = reg.key[RK - 1];
+            thr_s = tk == 0xffffffffu ? (desc ? -INFINITY : INFINITY) : rank_key32_score(tk, desc);
           }
         } else {
           while (__any_sync(0xffffffffu, mask != 0)) {
@@ -1012,9 +1018,7 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
       }
       tc_fence_before();
       mbar_arrive(&acce[buf]);
-      if (KR > 0 && __any_sync(0xffffffffu, cnt > 0)) merge_candidates(reg, cbuf, m, kBM, cnt, thr_s, desc);
     }
-    if (KR > 0 && __any_sync(0xffffffffu, cnt > 0)) merge_candidates(reg, cbuf, m, kBM, cnt, thr_s, desc);
     if (qvalid) {
       uint64_t *out = a.partial + ((size_t)(g.list_base + blockIdx.x) * a.B + qidx) * k;
       if (KR > 0) {

@@ -126,14 +126,14 @@ def test_misaligned_buffers_rejected(lib):
     assert lib.lam_score_topk(*base) == 1
 
 
-@pytest.mark.parametrize("mask,cap", [(0, 10), (16, 10), (-1, 10), (1, -1), (1, (1 << 20) + 1)])
+@pytest.mark.parametrize("mask,cap", [(0, 10), (32, 10), (-1, 10), (1, -1), (1, (1 << 20) + 1)])
 def test_timing_rejects_bad_arguments(lib, mask, cap):
     assert lib.lam_timing_begin(mask, cap) == 1
 
 
 def test_timing_read_rejects_bad_kind_and_end_is_idempotent(lib):
     import paper_2609_32256_gb300 as lam
-    for kind in (0, 3, 16):
+    for kind in (0, 3, 32):
         assert lib.lam_timing_read(kind, None, None, None) == 1
     assert lib.lam_timing_begin(lam.LAM_TIME_SCORE, 0) == 0  # no events to create
     tot, timed, launches = lam.lam_timing_read(lam.LAM_TIME_SCORE)
