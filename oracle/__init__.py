@@ -77,6 +77,11 @@ def _load():
                                                ctypes.POINTER(ctypes.c_double),
                                                ctypes.POINTER(ctypes.c_double)]
         lib.lam_oracle_admit_batch.restype = ctypes.c_int64
+        lib.lam_oracle_lamz_compress.argtypes = [f32p, ctypes.c_int64, ctypes.c_float, u8p,
+                                                 ctypes.c_int64]
+        lib.lam_oracle_lamz_compress.restype = ctypes.c_int64
+        lib.lam_oracle_lamz_decompress.argtypes = [u8p, ctypes.c_int64, f32p, ctypes.c_int64]
+        lib.lam_oracle_lamz_decompress.restype = ctypes.c_int32
         lib.lam_oracle_code_sqnorms.argtypes = [i32p, ctypes.c_int64, ctypes.c_int32, f32p]
         lib.lam_oracle_code_sqnorms.restype = None
         lib.lam_oracle_scores.argtypes = [f32p, ctypes.c_int64, i32p, ctypes.c_int64,
@@ -174,6 +179,30 @@ def admit_batch(e: np.ndarray, digests: np.ndarray, delta: float):
                                           _ptr(rep, ctypes.c_int32),
                                           _ptr(dist, ctypes.c_double), ctypes.byref(dh))
     return rep, dist, dh.value, int(kept)
+
+
+def lamz_compress(x: np.ndarray, rel: float) -> bytes:
+    """Error-bounded byte codec (bound rel * max|x|): the compressed bytes."""
+    v = np.ascontiguousarray(x, dtype=np.float32).reshape(-1)
+    lib = _load()
+    size = lib.lam_oracle_lamz_compress(_ptr(v, ctypes.c_float), v.size,
+                                        ctypes.c_float(np.float32(rel)), None, 0)
+    if size < 0:
+        raise ValueError("non-finite input")
+    out = np.empty(size, dtype=np.uint8)
+    lib.lam_oracle_lamz_compress(_ptr(v, ctypes.c_float), v.size, ctypes.c_float(np.float32(rel)),
+                                 _ptr(out, ctypes.c_uint8), size)
+    return out.tobytes()
+
+
+def lamz_decompress(data: bytes, n: int) -> np.ndarray:
+    buf = np.frombuffer(data, dtype=np.uint8).copy()
+    out = np.empty(n, dtype=np.float32)
+    st = _load().lam_oracle_lamz_decompress(_ptr(buf, ctypes.c_uint8), buf.size,
+                                            _ptr(out, ctypes.c_float), n)
+    if st != 0:
+        raise ValueError("malformed stream")
+    return out
 
 
 def code_sqnorms(codes: np.ndarray) -> np.ndarray:

@@ -249,7 +249,149 @@ int64_t lam_oracle_admit_batch(const float *e, int64_t N, int32_t D, const uint6
   return retained;
 }
 
-/* Score of one query against one dequantised row, in double, rounded to fp32. *//* Score of one query against one dequantised row, in double, rounded to fp32. *//* Score of one query against one dequantised row, in double, rounded to fp32. */
+/*
+ * Error-bounded byte codec for retained embeddings (Sec. 3.2, layer L2:
+ * "error-bounded byte compression" under a relative codec error bound; the
+ * deployed bound is 1% of max|x|).  The paper uses a third-party codec; this
+ * is a self-contained format of the same family, defined here:
+ *   eb = fl32(rel * max|x_i|), s = fl32(2 eb) (s = 1 when every x_i is 0);
+ *   q_i = Q(x_i) = rint_half_even(fl32(x_i / s)), exactly as the quantizer;
+ *   blocks of 32 values; inside a block the deltas d_0 = q_0, d_j = q_j - q_{j-1}
+ *   (a tail block is padded by repeating its last code, i.e. zero deltas);
+ *   per block L = bit length of max_j |d_j| (0..31);
+ *   layout: "LAMZ", n (int64 LE), s (fp32 LE), one byte L per block, zero
+ *   padding to a multiple of 4 bytes, then for every block with L > 0 in
+ *   order: a 32-bit sign word (bit j set when d_j < 0) and L 32-bit bit planes
+ *   (bit j of plane p is bit p of |d_j|), all little-endian.
+ * Decoding sums the deltas back into q and returns fl32(s * q): the error is
+ * that of Q_eps at eps = eb.
+ */
+static int32_t bitlen_u32(uint32_t v) {
+  int32_t b = 0;
+  while (v) {
+    ++b;
+    v >>= 1;
+  }
+  return b;
+}
+
+static void put_u32(uint8_t *p, uint32_t v) {
+  p[0] = (uint8_t)v;
+  p[1] = (uint8_t)(v >> 8);
+  p[2] = (uint8_t)(v >> 16);
+  p[3] = (uint8_t)(v >> 24);
+}
+
+static uint32_t get_u32(const uint8_t *p) {
+  return (uint32_t)p[0] | ((uint32_t)p[1] << 8) | ((uint32_t)p[2] << 16) | ((uint32_t)p[3] << 24);
+}
+
+/* Returns the compressed size; writes only when it fits in cap (out may be
+ * NULL to ask for the size).  Returns -1 for a non-finite input. */
+int64_t lam_oracle_lamz_compress(const float *x, int64_t n, float rel, uint8_t *out, int64_t cap) {
+  int old_mode = fegetround();
+  fesetround(FE_TONEAREST);
+  float mx = 0.0f;
+  for (int64_t i = 0; i < n; ++i) {
+    if (!isfinite(x[i])) {
+      fesetround(old_mode);
+      return -1;
+    }
+    const float a = fabsf(x[i]);
+    if (a > mx) mx = a;
+  }
+  const float eb = rel * mx;
+  const float s = mx > 0.0f ? 2.0f * eb : 1.0f;
+  const int64_t nb = (n + 31) / 32;
+  const int64_t head = 16 + ((nb + 3) / 4) * 4;
+  int64_t size = head;
+  int32_t q[32], d[32];
+  for (int pass = 0; pass < 2; ++pass) {
+    int64_t pos = head;
+    if (pass == 1) {
+      if (out == NULL || size > cap) break;
+      memset(out, 0, (size_t)head);
+      out[0] = 'L';
+      out[1] = 'A';
+      out[2] = 'M';
+      out[3] = 'Z';
+      for (int k = 0; k < 8; ++k) out[4 + k] = (uint8_t)((uint64_t)n >> (8 * k));
+      uint32_t sb;
+      memcpy(&sb, &s, 4);
+      put_u32(out + 12, sb);
+    }
+    for (int64_t b = 0; b < nb; ++b) {
+      uint32_t mag_max = 0;
+      for (int j = 0; j < 32; ++j) {
+        const int64_t i = b * 32 + j;
+        q[j] = i < n ? (int32_t)nearbyintf(x[i] / s) : q[j - 1];
+        d[j] = j == 0 ? q[0] : q[j] - q[j - 1];
+        const uint32_t m = (uint32_t)(d[j] < 0 ? -(int64_t)d[j] : d[j]);
+        if (m > mag_max) mag_max = m;
+      }
+      const int32_t L = bitlen_u32(mag_max);
+      if (pass == 0) {
+        if (L > 0) size += 4 + 4 * (int64_t)L;
+        continue;
+      }
+      out[16 + b] = (uint8_t)L;
+      if (L == 0) continue;
+      uint32_t sign = 0;
+      for (int j = 0; j < 32; ++j)
+        if (d[j] < 0) sign |= 1u << j;
+      put_u32(out + pos, sign);
+      pos += 4;
+      for (int p = 0; p < L; ++p) {
+        uint32_t plane = 0;
+        for (int j = 0; j < 32; ++j) {
+          const uint32_t m = (uint32_t)(d[j] < 0 ? -(int64_t)d[j] : d[j]);
+          if ((m >> p) & 1u) plane |= 1u << j;
+        }
+        put_u32(out + pos, plane);
+        pos += 4;
+      }
+    }
+  }
+  fesetround(old_mode);
+  return size;
+}
+
+/* Decodes n values; returns 0, or -1 for a malformed or truncated stream. */
+int32_t lam_oracle_lamz_decompress(const uint8_t *in, int64_t size, float *out, int64_t n) {
+  if (size < 16 || in[0] != 'L' || in[1] != 'A' || in[2] != 'M' || in[3] != 'Z') return -1;
+  uint64_t nn = 0;
+  for (int k = 0; k < 8; ++k) nn |= (uint64_t)in[4 + k] << (8 * k);
+  if ((int64_t)nn != n) return -1;
+  const uint32_t sb = get_u32(in + 12);
+  float s;
+  memcpy(&s, &sb, 4);
+  const int64_t nb = (n + 31) / 32;
+  const int64_t head = 16 + ((nb + 3) / 4) * 4;
+  if (size < head) return -1;
+  int64_t pos = head;
+  for (int64_t b = 0; b < nb; ++b) {
+    const int32_t L = in[16 + b];
+    if (L > 31 || pos + (L > 0 ? 4 + 4 * (int64_t)L : 0) > size) return -1;
+    uint32_t sign = 0, planes[32];
+    if (L > 0) {
+      sign = get_u32(in + pos);
+      pos += 4;
+      for (int p = 0; p < L; ++p, pos += 4) planes[p] = get_u32(in + pos);
+    }
+    int32_t qv = 0;
+    for (int j = 0; j < 32; ++j) {
+      uint32_t m = 0;
+      for (int p = 0; p < L; ++p) m |= ((planes[p] >> j) & 1u) << p;
+      const int32_t dj = ((sign >> j) & 1u) ? -(int32_t)m : (int32_t)m;
+      qv += dj;
+      const int64_t i = b * 32 + j;
+      if (i < n) out[i] = s * (float)qv;
+    }
+  }
+  return 0;
+}
+
+/* Score of one query against one dequantised row, in double, rounded to fp32. *//* Score of one query against one dequantised row, in double, rounded to fp32. *//* Score of one query against one dequantised row, in double, rounded to fp32. *//* Score of one query against one dequantised row, in double, rounded to fp32. */
 static float score_one(const float *q, const int32_t *c, int32_t D, float s,
                        int metric) {
   if (metric == ORACLE_IP) {

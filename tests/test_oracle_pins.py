@@ -389,3 +389,41 @@ def test_admit_batch_only_band_candidates_merge():
     dig2 = np.array([[5, 9], [9, 5]], dtype=np.uint64)
     rep, *_ = oracle.admit_batch(x[:2], dig2, 0.1)
     assert rep.tolist() == [0, 1]
+
+
+def test_lamz_worked_stream():
+    for vals, rel, hexs in golden("lamz_small.txt"):
+        x = np.array([float(v) for v in vals.split(",")], dtype=np.float32)
+        b = oracle.lamz_compress(x, float(rel))
+        assert b.hex() == hexs
+        np.testing.assert_array_equal(oracle.lamz_decompress(b, x.size), x)
+
+
+@pytest.mark.parametrize("rel", [1e-3, 1e-2, 3e-2])
+def test_lamz_round_trip_is_q_eps_at_the_codec_bound(rel):
+    x = inputs.flat_values((1 << 16) + 13, seed=8)  # ragged tail block
+    b = oracle.lamz_compress(x, rel)
+    y = oracle.lamz_decompress(b, x.size)
+    eb = np.float32(rel) * np.abs(x).max()
+    # the decoded values are exactly the quantizer's at eps = eb (an
+    # independent function: its own division, rounding and dequantisation)
+    codes, *_ = oracle.quantize(x, float(eb))
+    np.testing.assert_array_equal(y, oracle.dequantize(codes, oracle.step(float(eb))))
+    err = np.abs(x.astype(np.float64) - y)
+    assert np.all(err <= eb * (1 + 2.0 ** -23) + np.abs(x) * 2.0 ** -23)
+
+
+def test_lamz_sizes_of_zero_and_constant_inputs():
+    n = 1000
+    nb = (n + 31) // 32
+    head = 16 + (nb + 3) // 4 * 4
+    assert len(oracle.lamz_compress(np.zeros(n, np.float32), 0.01)) == head
+    # a constant c: one non-zero delta per block, c / s = 1 / (2 rel) = 50
+    b = oracle.lamz_compress(np.full(n, 0.37, np.float32), 0.01)
+    assert len(b) == head + nb * (4 + 4 * 6)  # |50| needs 6 bits
+    y = oracle.lamz_decompress(b, n)
+    assert np.all(y == y[0]) and abs(float(y[0]) - 0.37) <= 0.0037
+    with pytest.raises(ValueError):
+        oracle.lamz_compress(np.array([1.0, np.inf], np.float32), 0.01)
+    with pytest.raises(ValueError):
+        oracle.lamz_decompress(b[:-4], n)  # truncated
