@@ -648,6 +648,27 @@ def run_kernels(args):
                                      "gbs_kernel": nbytes / (k_ms / 1e3) / 1e9,
                                      "frac_of_hbm_kernel": nbytes / (k_ms / 1e3) / 1e9 / hbm})
             del dig
+    if wl.d == 1:
+        # the error-bounded byte codec at the paper's relative bounds (its
+        # deployed bound is 1% of max|x|), on the first 2^24 values and all
+        res["codec"] = []
+        for n_c in sorted({min(n, 1 << 24), n}):
+            xc = x[:n_c]
+            cbuf = torch.empty(lam.lam_lamz_bound(n_c), dtype=torch.uint8, device=dev)
+            cws = torch.empty(lam.lam_lamz_workspace_size(n_c), dtype=torch.uint8, device=dev)
+            yc = torch.empty(n_c, dtype=torch.float32, device=dev)
+            for rel in (1e-3, 1e-2, 3e-2):
+                st, nbytes = lam.lam_lamz_compress(xc, rel, cbuf, cws)
+                ms_c, _ = timed(lambda: lam.lam_lamz_compress(xc, rel, cbuf, cws),
+                                lam.LAM_TIME_AUX)
+                ms_d, _ = timed(lambda: lam.lam_lamz_decompress(cbuf, nbytes, yc, cws),
+                                lam.LAM_TIME_AUX)
+                res["codec"].append({"n": n_c, "rel": rel, "ratio": 4.0 * n_c / nbytes,
+                                     "compress_ms_span": ms_c,
+                                     "compress_gbs": 4.0 * n_c / (ms_c / 1e3) / 1e9,
+                                     "decompress_ms_span": ms_d,
+                                     "decompress_gbs": 4.0 * n_c / (ms_d / 1e3) / 1e9})
+            del cbuf, cws, yc
     if wl.planted:
         # batch admission (Algorithm 2) at cos >= 0.95 over band candidates at
         # the paper's shipped (r = 4, eps = 0.2 sigma) and relaxed (r = 8, 0.3 sigma)

@@ -169,6 +169,42 @@ lam_status lam_admit_batch(const float *e, int64_t N, int32_t D,
                            int64_t *n_pairs_out, lam_stream_t stream);
 
 /*
+ * Error-bounded byte codec for retained embeddings (Sec. 3.2, layer L2:
+ * "error-bounded byte compression" under a relative codec error bound; the
+ * paper deploys 1% of max|x|).  The paper uses a third-party codec; this is a
+ * self-contained format of the same family:
+ *   eb = fl32(rel * max|x|), s = fl32(2 eb) (s = 1 when every x is 0); the
+ *   codes are Q_eps at eps = eb (the quantizer's division and rounding);
+ *   blocks of 32 codes; inside a block the deltas d_0 = q_0, d_j = q_j -
+ *   q_{j-1} (a tail block repeats its last code); L = bit length of the
+ *   block's largest |d| (0..31).
+ * Stream (little-endian): "LAMZ", n (int64), s (fp32), one byte L per block,
+ * zero padding to a multiple of 4, then for each block with L > 0 a 32-bit
+ * sign word (bit j: d_j < 0) and L 32-bit bit planes (bit j of plane p: bit p
+ * of |d_j|).  Decoding returns fl32(s * q): |x - x_hat| <= eb (+ fp32
+ * rounding of the quotient and the product), exactly the error of Q_eps.
+ *
+ * lam_lamz_bound(n): the largest stream for n values.
+ * lam_lamz_workspace_size(n): device scratch for either direction.
+ * lam_lamz_compress: x [n] fp32 device (4-byte aligned), rel in [1e-6, 1],
+ *   out (device, 4-byte aligned) of out_capacity bytes, *out_bytes (host) the
+ *   stream size.  Synchronous.  Errors: LAM_ERR_INVALID, LAM_ERR_NONFINITE,
+ *   LAM_ERR_WORKSPACE (workspace too small, or the stream exceeds
+ *   out_capacity: *out_bytes then holds the size needed), LAM_ERR_CUDA.
+ * lam_lamz_decompress: the stream (device, in_bytes) into out [n] fp32
+ *   (device).  LAM_ERR_INVALID for a stream that is not LAMZ, has another n,
+ *   a bit length above 31, or is truncated.  Asynchronous after its checks.
+ */
+size_t lam_lamz_bound(int64_t n);
+size_t lam_lamz_workspace_size(int64_t n);
+lam_status lam_lamz_compress(const float *x, int64_t n, float rel, void *out,
+                             size_t out_capacity, size_t *out_bytes, void *workspace,
+                             size_t workspace_bytes, lam_stream_t stream);
+lam_status lam_lamz_decompress(const void *in, size_t in_bytes, float *out, int64_t n,
+                               void *workspace, size_t workspace_bytes,
+                               lam_stream_t stream);
+
+/*
  * lam_dequantize -- xhat_i = fl32(scale * code_i), the inverse map of Q_eps
  * up to the cell half-width eps (|x - xhat| <= eps, Sec. 3.1).
  *

@@ -18,7 +18,9 @@ from ._lib import (LAM_ERR_CUDA, LAM_ERR_INVALID, LAM_ERR_NONFINITE, LAM_ERR_RAN
                    lam_score_topk_workspace_size, lam_status_string, lam_version, load,
                    LAM_TIME_AUX, LAM_TIME_MERGE, LAM_TIME_DEQUANTIZE, LAM_TIME_QUANTIZE, LAM_TIME_SCORE,
                    lam_timing_begin, lam_timing_end, lam_timing_read, lam_code_sqnorms,
-                   lam_quantize_bands, lam_admit_batch, lam_admit_batch_workspace_size)
+                   lam_quantize_bands, lam_admit_batch, lam_admit_batch_workspace_size,
+                   lam_lamz_bound, lam_lamz_compress, lam_lamz_decompress,
+                   lam_lamz_workspace_size)
 
 CODE_DTYPES = {1: "int8", 2: "int16", 4: "int32"}
 

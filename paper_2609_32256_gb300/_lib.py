@@ -57,6 +57,10 @@ def load():
         "lam_score_topk_noalloc": (i32, [vp, i64, vp, i32, i64, i32, f32, i32, i32, i32, vp,
                                          vp, vp]),
         "lam_code_sqnorms": (i32, [vp, i32, i64, i32, vp, vp]),
+        "lam_lamz_bound": (sz, [i64]),
+        "lam_lamz_workspace_size": (sz, [i64]),
+        "lam_lamz_compress": (i32, [vp, i64, f32, vp, sz, P(sz), vp, sz, vp]),
+        "lam_lamz_decompress": (i32, [vp, sz, vp, i64, vp, sz, vp]),
         "lam_admit_batch_workspace_size": (sz, [i64, i32, i64]),
         "lam_admit_batch": (i32, [vp, i64, i32, vp, i32, ctypes.c_double, vp, vp, vp, sz, i64,
                                   P(ctypes.c_double), P(i64), P(i64), vp]),
@@ -210,6 +214,36 @@ def lam_admit_batch(e, digests, delta, rep, dist, workspace, max_pairs, stream=N
     if raise_on_error:
         _check(st, "lam_admit_batch")
     return st, dh.value, kept.value, np_.value
+
+
+def lam_lamz_bound(n) -> int:
+    return int(load().lam_lamz_bound(int(n)))
+
+
+def lam_lamz_workspace_size(n) -> int:
+    return int(load().lam_lamz_workspace_size(int(n)))
+
+
+def lam_lamz_compress(x, rel, out, workspace, stream=None, raise_on_error=True):
+    """Error-bounded compression of the fp32 CUDA tensor x into the uint8 CUDA
+    tensor out; returns (status, stream bytes)."""
+    nb = ctypes.c_size_t(0)
+    st = load().lam_lamz_compress(_ptr(x), int(x.numel()), ctypes.c_float(rel), _ptr(out),
+                                  _nbytes(out), ctypes.byref(nb), _ptr(workspace),
+                                  _nbytes(workspace), _stream(stream, x.device))
+    if raise_on_error:
+        _check(st, "lam_lamz_compress")
+    return st, nb.value
+
+
+def lam_lamz_decompress(stream_bytes, nbytes, out, workspace, stream=None, raise_on_error=True):
+    """Decodes the first nbytes of the uint8 CUDA tensor into out (fp32)."""
+    st = load().lam_lamz_decompress(_ptr(stream_bytes), int(nbytes), _ptr(out), int(out.numel()),
+                                    _ptr(workspace), _nbytes(workspace),
+                                    _stream(stream, out.device))
+    if raise_on_error:
+        _check(st, "lam_lamz_decompress")
+    return st
 
 
 def lam_code_sqnorms(codes, width, N, D, sqnorm_out, stream=None) -> None:

@@ -410,6 +410,58 @@ lam_status lam_admit_batch(const float *e, int64_t N, int32_t D, const uint64_t 
   return LAM_OK;
 }
 
+size_t lam_lamz_bound(int64_t n) { return n < 0 ? 0 : lamz_bound_bytes(n); }
+
+size_t lam_lamz_workspace_size(int64_t n) { return n < 0 ? 0 : lamz_workspace_bytes(n); }
+
+lam_status lam_lamz_compress(const float *x, int64_t n, float rel, void *out, size_t out_capacity,
+                             size_t *out_bytes, void *workspace, size_t workspace_bytes,
+                             lam_stream_t stream) {
+  if (n < 0 || n > (1LL << 40) || !(rel >= 1e-6f) || !(rel <= 1.0f)) return LAM_ERR_INVALID;
+  if (n > 0 && (x == nullptr || out == nullptr || workspace == nullptr)) return LAM_ERR_INVALID;
+  if ((reinterpret_cast<uintptr_t>(x) & 3u) || (reinterpret_cast<uintptr_t>(out) & 3u) ||
+      (reinterpret_cast<uintptr_t>(workspace) & 255u))
+    return LAM_ERR_INVALID;
+  if (workspace_bytes < lamz_workspace_bytes(n)) return LAM_ERR_WORKSPACE;
+  if (out_capacity < lamz_head_bytes(n)) {
+    if (out_bytes) *out_bytes = lamz_head_bytes(n);
+    return LAM_ERR_WORKSPACE;
+  }
+  const int sms = device_sms();
+  if (sms <= 0) return LAM_ERR_CUDA;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  size_t bytes = 0;
+  bool fits = false, nonfinite = false;
+  timing_launch_begin(LAM_TIME_AUX, st);
+  const cudaError_t e = launch_lamz_compress(x, n, rel, static_cast<uint8_t *>(out), out_capacity,
+                                             workspace, sms, st, &bytes, &fits, &nonfinite);
+  timing_launch_end(LAM_TIME_AUX, st);
+  if (e != cudaSuccess) return LAM_ERR_CUDA;
+  if (out_bytes) *out_bytes = bytes;
+  if (nonfinite) return LAM_ERR_NONFINITE;
+  return fits ? LAM_OK : LAM_ERR_WORKSPACE;
+}
+
+lam_status lam_lamz_decompress(const void *in, size_t in_bytes, float *out, int64_t n,
+                               void *workspace, size_t workspace_bytes, lam_stream_t stream) {
+  if (n < 0 || n > (1LL << 40)) return LAM_ERR_INVALID;
+  if (n > 0 && (in == nullptr || out == nullptr || workspace == nullptr)) return LAM_ERR_INVALID;
+  if ((reinterpret_cast<uintptr_t>(in) & 3u) || (reinterpret_cast<uintptr_t>(out) & 3u) ||
+      (reinterpret_cast<uintptr_t>(workspace) & 255u))
+    return LAM_ERR_INVALID;
+  if (workspace_bytes < lamz_workspace_bytes(n)) return LAM_ERR_WORKSPACE;
+  const int sms = device_sms();
+  if (sms <= 0) return LAM_ERR_CUDA;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  bool bad = true;
+  timing_launch_begin(LAM_TIME_AUX, st);
+  const cudaError_t e = launch_lamz_decompress(static_cast<const uint8_t *>(in), in_bytes, out, n,
+                                               workspace, sms, st, &bad);
+  timing_launch_end(LAM_TIME_AUX, st);
+  if (e != cudaSuccess) return LAM_ERR_CUDA;
+  return bad ? LAM_ERR_INVALID : LAM_OK;
+}
+
 lam_status lam_dequantize(const void *codes, int32_t width, int64_t n, float scale, float *out,
                           lam_stream_t stream) {
   if (n < 0 || !valid_width(width) || !isfinite(scale)) return LAM_ERR_INVALID;

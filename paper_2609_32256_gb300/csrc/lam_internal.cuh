@@ -160,6 +160,15 @@ cudaError_t launch_admit_batch(const float *e, int64_t N, int D, const uint64_t 
                                double delta, int32_t *rep, double *dist, void *ws,
                                int64_t max_pairs, int sms, cudaStream_t st, int64_t *n_pairs,
                                double *delta_hat, int64_t *n_retained, bool *overflow);
+// Error-bounded byte codec (lamz.cu).
+size_t lamz_head_bytes(int64_t n);
+size_t lamz_bound_bytes(int64_t n);
+size_t lamz_workspace_bytes(int64_t n);
+cudaError_t launch_lamz_compress(const float *x, int64_t n, float rel, uint8_t *out, size_t cap,
+                                 void *ws, int sms, cudaStream_t stream, size_t *bytes,
+                                 bool *fits, bool *nonfinite);
+cudaError_t launch_lamz_decompress(const uint8_t *in, size_t in_bytes, float *out, int64_t n,
+                                   void *ws, int sms, cudaStream_t stream, bool *bad);
 cudaError_t launch_code_sqnorms(const void *codes, int width, int64_t N, int D, float *out,
                                 int sms, cudaStream_t st);
 cudaError_t launch_dequantize(const void *codes, int width, int64_t n, float s, float *out,

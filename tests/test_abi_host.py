@@ -162,3 +162,20 @@ def test_quantize_bands_rejects_bad_arguments(lib, N, D, r, width, x, dig):
                                 c.c_void_p(dig), c.c_void_p(1024), 64, None, None, None, None,
                                 None)
     assert st == 1
+
+
+@pytest.mark.parametrize("n,rel", [(-1, 0.01), (10, 0.0), (10, 1e-7), (10, 2.0),
+                                   (10, float("nan"))])
+def test_lamz_compress_rejects_bad_arguments(lib, n, rel):
+    c = ctypes
+    nb = c.c_size_t(0)
+    st = lib.lam_lamz_compress(c.c_void_p(256), n, c.c_float(rel), c.c_void_p(512), 1 << 20,
+                               c.byref(nb), c.c_void_p(1024), 1 << 20, None)
+    assert st == 1
+
+
+def test_lamz_sizes(lib):
+    import paper_2609_32256_gb300 as lam
+    assert lam.lam_lamz_bound(0) == 16
+    assert lam.lam_lamz_bound(33) == 16 + 4 + 2 * (4 + 4 * 31)
+    assert lam.lam_lamz_workspace_size(1 << 20) > 0
