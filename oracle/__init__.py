@@ -14,6 +14,11 @@ What it follows (paper: "LAM: Lossy Agent Memory"):
                   product, cosine and squared L2 (Eq. 1 ties L2 to cosine);
   * top-k      -- full sort, best first, equal scores by lower id (the
                   lowest-index rule of Algorithm 1).
+  * encode_rows / decode_rows / scores_rows -- the per-vector byte codecs
+                  of the composite experiment (Sec. "Composite reduction",
+                  Table "composite": fp16, per-vector int8 with a scale and an
+                  offset per row, sign bits with one scale per row) and the
+                  exact scores of their decoded fp32 rows.
 """
 from __future__ import annotations
 
@@ -82,6 +87,19 @@ def _load():
         lib.lam_oracle_lamz_compress.restype = ctypes.c_int64
         lib.lam_oracle_lamz_decompress.argtypes = [u8p, ctypes.c_int64, f32p, ctypes.c_int64]
         lib.lam_oracle_lamz_decompress.restype = ctypes.c_int32
+        i8p = ctypes.POINTER(ctypes.c_int8)
+        lib.lam_oracle_encode_int8_rows.argtypes = [f32p, ctypes.c_int64, ctypes.c_int32, i8p,
+                                                    f32p, f32p]
+        lib.lam_oracle_encode_int8_rows.restype = None
+        lib.lam_oracle_encode_sign_rows.argtypes = [f32p, ctypes.c_int64, ctypes.c_int32, u8p,
+                                                    f32p]
+        lib.lam_oracle_encode_sign_rows.restype = None
+        lib.lam_oracle_decode_rows.argtypes = [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64,
+                                               ctypes.c_int32, f32p, f32p, f32p]
+        lib.lam_oracle_decode_rows.restype = None
+        lib.lam_oracle_scores_rows.argtypes = [f32p, ctypes.c_int64, f32p, ctypes.c_int64,
+                                               ctypes.c_int32, ctypes.c_int32, f32p]
+        lib.lam_oracle_scores_rows.restype = None
         lib.lam_oracle_code_sqnorms.argtypes = [i32p, ctypes.c_int64, ctypes.c_int32, f32p]
         lib.lam_oracle_code_sqnorms.restype = None
         lib.lam_oracle_scores.argtypes = [f32p, ctypes.c_int64, i32p, ctypes.c_int64,
@@ -202,6 +220,57 @@ def lamz_decompress(data: bytes, n: int) -> np.ndarray:
                                             _ptr(out, ctypes.c_float), n)
     if st != 0:
         raise ValueError("malformed stream")
+    return out
+
+
+FMT_INT8_ROWS, FMT_FP16, FMT_SIGN = 1, 2, 3
+
+
+def encode_rows(x: np.ndarray, fmt: int):
+    """Alternative codec of rows [N, D]: (codes, scale, offset) with codes int8
+    [N, D] (fmt 1), fp16 [N, D] (fmt 2) or packed sign bits uint8 [N, D/8]
+    (fmt 3); scale/offset float32 [N] (offset None unless fmt 1)."""
+    v = np.ascontiguousarray(x, dtype=np.float32)
+    N, D = v.shape
+    if fmt == FMT_FP16:
+        return v.astype(np.float16), None, None
+    if fmt == FMT_INT8_ROWS:
+        c = np.empty((N, D), np.int8)
+        sc = np.empty(N, np.float32)
+        of = np.empty(N, np.float32)
+        _load().lam_oracle_encode_int8_rows(_ptr(v, ctypes.c_float), N, D,
+                                            _ptr(c, ctypes.c_int8), _ptr(sc, ctypes.c_float),
+                                            _ptr(of, ctypes.c_float))
+        return c, sc, of
+    assert D % 8 == 0
+    bits = np.empty((N, D // 8), np.uint8)
+    al = np.empty(N, np.float32)
+    _load().lam_oracle_encode_sign_rows(_ptr(v, ctypes.c_float), N, D,
+                                        _ptr(bits, ctypes.c_uint8), _ptr(al, ctypes.c_float))
+    return bits, al, None
+
+
+def decode_rows(codes: np.ndarray, fmt: int, D: int, scale=None, offset=None) -> np.ndarray:
+    c = np.ascontiguousarray(codes)
+    N = c.shape[0]
+    out = np.empty((N, D), np.float32)
+    sc = np.ascontiguousarray(scale if scale is not None else np.zeros(N), dtype=np.float32)
+    of = np.ascontiguousarray(offset if offset is not None else np.zeros(N), dtype=np.float32)
+    _load().lam_oracle_decode_rows(c.ctypes.data_as(ctypes.c_void_p), fmt, N, D,
+                                   _ptr(sc, ctypes.c_float), _ptr(of, ctypes.c_float),
+                                   _ptr(out, ctypes.c_float))
+    return out
+
+
+def scores_rows(queries: np.ndarray, rows: np.ndarray, metric: int) -> np.ndarray:
+    """Scores [B, N] of queries [B, D] against decoded fp32 rows [N, D]."""
+    q = np.ascontiguousarray(queries, dtype=np.float32)
+    r = np.ascontiguousarray(rows, dtype=np.float32)
+    B, D = q.shape
+    N = r.shape[0]
+    out = np.empty((B, N), np.float32)
+    _load().lam_oracle_scores_rows(_ptr(q, ctypes.c_float), B, _ptr(r, ctypes.c_float), N, D,
+                                   metric, _ptr(out, ctypes.c_float))
     return out
 
 

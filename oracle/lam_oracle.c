@@ -19,7 +19,7 @@
  *     (Sec. "Brute-force scan crossover"), followed by a top-k.  Metrics:
  *     inner product, cosine, squared L2 (Eq. 1 relates L2 and cosine).
  *
- * Readings where the paper is silent (each also listed in the design doc):
+ * Readings where the paper is silent:
  *   - "round" is IEEE round-half-to-even, evaluated as nearbyintf() under
  *     FE_TONEAREST on the fp32 quotient.
  *   - x / 2 eps is one fp32 IEEE division by s = fl32(2 * eps), eps given in
@@ -30,6 +30,10 @@
  *     cosine rank descending.  Equal scores rank the lower id first (the
  *     paper's lowest-index rule, Algorithm 1).
  *   - Scores are accumulated in double and rounded once to fp32.
+ *   - The per-vector byte codecs of the composite experiment (fp16,
+ *     per-vector int8, sign-binary; Sec. "Composite reduction", Table
+ *     "composite") are defined only by name and ratio; the definitions taken
+ *     are given above lam_oracle_encode_int8_rows.
  *
  * Build flags matter: -O2 -ffp-contract=off -fno-fast-math, so that no
  * multiply-add is contracted into an FMA on either x86-64 or aarch64.
@@ -391,7 +395,98 @@ int32_t lam_oracle_lamz_decompress(const uint8_t *in, int64_t size, float *out, 
   return 0;
 }
 
-/* Score of one query against one dequantised row, in double, rounded to fp32. *//* Score of one query against one dequantised row, in double, rounded to fp32. *//* Score of one query against one dequantised row, in double, rounded to fp32. *//* Score of one query against one dequantised row, in double, rounded to fp32. */
+/*
+ * Alternative byte codecs of the composite experiment (App. "Composite
+ * reduction": fp16, per-vector int8, sign-binary).  The paper names them and
+ * their compression ratios only; the definitions taken here:
+ *   fp16:            xhat = fp16(x) (round to nearest even).
+ *   per-vector int8: lo = min_d x, hi = max_d x, scale = fl32((hi - lo) / 255),
+ *                    c = rint_half_even(fl32(fl32(x - lo) / scale)) - 128 in
+ *                    [-128, 127] (c = -128 when scale = 0), offset =
+ *                    fl32(lo + 128 scale), xhat = fl32(offset + fl32(scale c));
+ *                    two fp32 per row, i.e. 776 bytes for D = 768, the
+ *                    paper's 3.96x.
+ *   sign-binary:     bit b_d = (x_d >= 0), alpha = fl32(sum_d |x_d| / D)
+ *                    summed in double, xhat = b ? alpha : -alpha; D/8 bytes
+ *                    plus one fp32, the paper's 30.72x at D = 768.
+ * Encoders write the codes and the per-row factors; lam_oracle_decode_rows
+ * writes xhat.
+ */
+void lam_oracle_encode_int8_rows(const float *x, int64_t N, int32_t D, int8_t *codes,
+                                 float *scale, float *offset) {
+  int old_mode = fegetround();
+  fesetround(FE_TONEAREST);
+  for (int64_t i = 0; i < N; ++i) {
+    const float *r = x + i * (int64_t)D;
+    float lo = r[0], hi = r[0];
+    for (int32_t d = 1; d < D; ++d) {
+      if (r[d] < lo) lo = r[d];
+      if (r[d] > hi) hi = r[d];
+    }
+    const float sc = (hi - lo) / 255.0f;
+    for (int32_t d = 0; d < D; ++d) {
+      int32_t c = -128;
+      if (sc > 0.0f) {
+        const float t = (r[d] - lo) / sc;
+        c = (int32_t)nearbyintf(t) - 128;
+        if (c < -128) c = -128;
+        if (c > 127) c = 127;
+      }
+      codes[i * (int64_t)D + d] = (int8_t)c;
+    }
+    scale[i] = sc;
+    offset[i] = lo + 128.0f * sc;
+  }
+  fesetround(old_mode);
+}
+
+void lam_oracle_encode_sign_rows(const float *x, int64_t N, int32_t D, uint8_t *bits,
+                                 float *alpha) {
+  for (int64_t i = 0; i < N; ++i) {
+    const float *r = x + i * (int64_t)D;
+    double a = 0.0;
+    for (int32_t d = 0; d < D; ++d) a += fabs((double)r[d]);
+    alpha[i] = (float)(a / (double)D);
+    for (int32_t d = 0; d < D; d += 8) {
+      uint8_t byte = 0;
+      for (int t = 0; t < 8 && d + t < D; ++t)
+        if (r[d + t] >= 0.0f) byte |= (uint8_t)(1u << t);
+      bits[i * (int64_t)(D / 8) + d / 8] = byte;
+    }
+  }
+}
+
+/* fmt 1: int8 codes + scale + offset; fmt 2: fp16 bit patterns (uint16);
+ * fmt 3: sign bits + alpha (in scale).  Writes xhat [N, D]. */
+void lam_oracle_decode_rows(const void *codes, int32_t fmt, int64_t N, int32_t D,
+                            const float *scale, const float *offset, float *out);
+
+/* Scores [B, N] of queries against decoded rows xhat [N, D] (double, one
+ * rounding; cosine 0 for a zero norm; squared L2 in the direct form). */
+void lam_oracle_scores_rows(const float *queries, int64_t B, const float *rows, int64_t N,
+                            int32_t D, int32_t metric, float *out) {
+  for (int64_t b = 0; b < B; ++b) {
+    const float *q = queries + b * (int64_t)D;
+    for (int64_t i = 0; i < N; ++i) {
+      const float *x = rows + i * (int64_t)D;
+      double dot = 0.0, qq = 0.0, xx = 0.0, l2 = 0.0;
+      for (int32_t d = 0; d < D; ++d) {
+        dot += (double)q[d] * (double)x[d];
+        qq += (double)q[d] * (double)q[d];
+        xx += (double)x[d] * (double)x[d];
+        const double df = (double)q[d] - (double)x[d];
+        l2 += df * df;
+      }
+      float v;
+      if (metric == ORACLE_IP) v = (float)dot;
+      else if (metric == ORACLE_COSINE) v = (qq == 0.0 || xx == 0.0) ? 0.0f : (float)(dot / (sqrt(qq) * sqrt(xx)));
+      else v = (float)l2;
+      out[b * N + i] = v;
+    }
+  }
+}
+
+/* Score of one query against one dequantised row, in double, rounded to fp32. *//* Score of one query against one dequantised row, in double, rounded to fp32. *//* Score of one query against one dequantised row, in double, rounded to fp32. *//* Score of one query against one dequantised row, in double, rounded to fp32. *//* Score of one query against one dequantised row, in double, rounded to fp32. */
 static float score_one(const float *q, const int32_t *c, int32_t D, float s,
                        int metric) {
   if (metric == ORACLE_IP) {
@@ -612,4 +707,39 @@ int lam_oracle_search(const float *queries, int64_t B, const int32_t *codes,
   free(th);
   free(jobs);
   return status;
+}
+
+/* IEEE binary16 bit pattern to float (exact). */
+static float half_to_float(uint16_t h) {
+  const uint32_t sign = (uint32_t)(h >> 15) << 31;
+  const int32_t e = (h >> 10) & 0x1f;
+  const uint32_t m = h & 0x3ffu;
+  float v;
+  if (e == 0) {
+    v = ldexpf((float)m, -24); /* subnormal (or zero) */
+  } else if (e == 31) {
+    v = m ? NAN : INFINITY;
+  } else {
+    v = ldexpf((float)(m | 0x400u), e - 25);
+  }
+  return sign ? -v : v;
+}
+
+void lam_oracle_decode_rows(const void *codes, int32_t fmt, int64_t N, int32_t D,
+                            const float *scale, const float *offset, float *out) {
+  for (int64_t i = 0; i < N; ++i) {
+    for (int32_t d = 0; d < D; ++d) {
+      float v = 0.0f;
+      if (fmt == 1) {
+        const int8_t c = ((const int8_t *)codes)[i * (int64_t)D + d];
+        v = offset[i] + scale[i] * (float)c;
+      } else if (fmt == 2) {
+        v = half_to_float(((const uint16_t *)codes)[i * (int64_t)D + d]);
+      } else {
+        const uint8_t byte = ((const uint8_t *)codes)[i * (int64_t)(D / 8) + d / 8];
+        v = ((byte >> (d % 8)) & 1u) ? scale[i] : -scale[i];
+      }
+      out[i * (int64_t)D + d] = v;
+    }
+  }
 }

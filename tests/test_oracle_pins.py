@@ -427,3 +427,118 @@ def test_lamz_sizes_of_zero_and_constant_inputs():
         oracle.lamz_compress(np.array([1.0, np.inf], np.float32), 0.01)
     with pytest.raises(ValueError):
         oracle.lamz_decompress(b[:-4], n)  # truncated
+
+
+# --- per-vector byte codecs (Sec. "Composite reduction", Table "composite") --
+
+def _row_cases():
+    for line in golden("row_codecs_hand.txt"):
+        yield line
+
+
+def test_row_codecs_hand_worked_rows():
+    for codec, vals, codes, scale, offset, xhat in _row_cases():
+        x = np.array([float(v) for v in vals.split(",")], np.float32)[None, :]
+        want = np.array([float(v) for v in xhat.split(",")], np.float32)
+        if codec == "int8":
+            c, sc, of = oracle.encode_rows(x, oracle.FMT_INT8_ROWS)
+            assert c[0].tolist() == [int(v) for v in codes.split(",")]
+            assert sc[0] == np.float32(scale) and of[0] == np.float32(offset)
+            got = oracle.decode_rows(c, oracle.FMT_INT8_ROWS, x.shape[1], sc, of)
+        else:
+            c, al, _ = oracle.encode_rows(x, oracle.FMT_SIGN)
+            assert c[0].tolist() == [int(codes, 16)]
+            assert al[0] == np.float32(scale)
+            got = oracle.decode_rows(c, oracle.FMT_SIGN, x.shape[1], al)
+        assert np.array_equal(got[0], want)
+
+
+def test_row_codec_sizes_give_the_papers_ratios():
+    # bytes per row: int8 D + two fp32 factors, sign D/8 + one fp32
+    D = 768
+    x = inputs.unit_rows(3, D, seed=5)
+    c, sc, of = oracle.encode_rows(x, oracle.FMT_INT8_ROWS)
+    int8_bytes = c[0].nbytes + sc[:1].nbytes + of[:1].nbytes
+    b, al, _ = oracle.encode_rows(x, oracle.FMT_SIGN)
+    sign_bytes = b[0].nbytes + al[:1].nbytes
+    h, _, _ = oracle.encode_rows(x, oracle.FMT_FP16)
+    assert round(4 * D / int8_bytes, 2) == 3.96
+    assert round(4 * D / sign_bytes, 2) == 30.72
+    assert 4 * D / h[0].nbytes == 2.0
+
+
+def test_fp16_decode_is_exact_for_every_bit_pattern():
+    # the C decoder against the IEEE binary16 definition as numpy implements it
+    pats = np.arange(1 << 16, dtype=np.uint32).astype(np.uint16)[None, :]
+    got = oracle.decode_rows(pats, oracle.FMT_FP16, pats.shape[1])[0]
+    want = pats.view(np.float16).astype(np.float32)[0]
+    fin = np.isfinite(want)
+    assert np.array_equal(got[fin].view(np.uint32), want[fin].view(np.uint32))
+    assert np.array_equal(np.isnan(got), np.isnan(want))
+    assert np.array_equal(got[np.isinf(want)], want[np.isinf(want)])
+
+
+def test_int8_rows_error_bound_extremes_and_order():
+    x = inputs.unit_rows(64, 96, seed=11)
+    c, sc, of = oracle.encode_rows(x, oracle.FMT_INT8_ROWS)
+    xh = oracle.decode_rows(c, oracle.FMT_INT8_ROWS, 96, sc, of)
+    for i in range(64):
+        lo, hi = x[i].min(), x[i].max()
+        assert sc[i] == np.float32((hi - lo) / np.float32(255))
+        # the row minimum takes code -128 and the maximum 127
+        assert c[i][x[i].argmin()] == -128 and c[i][x[i].argmax()] == 127
+        # half a step, plus the fp32 roundings of the encode and the decode
+        assert np.abs(xh[i] - x[i]).max() <= 0.5 * sc[i] * (1 + 1e-4) + 4e-7
+        # codes are monotone in x
+        o = np.argsort(x[i], kind="stable")
+        assert np.all(np.diff(c[i][o].astype(int)) >= 0)
+
+
+def test_sign_rows_alpha_is_the_least_squares_scale():
+    # for fixed signs b, ||x - a (2b - 1)||^2 is smallest at a = mean |x|
+    x = inputs.unit_rows(16, 64, seed=12)
+    b, al, _ = oracle.encode_rows(x, oracle.FMT_SIGN)
+    xh = oracle.decode_rows(b, oracle.FMT_SIGN, 64, al)
+    for i in range(16):
+        assert np.array_equal(np.sign(xh[i]), np.where(x[i] >= 0, 1.0, -1.0))
+        assert abs(al[i] - np.abs(x[i].astype(np.float64)).mean()) <= 1e-7 * al[i]
+        sg = np.sign(xh[i]).astype(np.float64)
+        err = lambda a: ((x[i] - a * sg) ** 2).sum()
+        assert err(al[i]) <= min(err(al[i] * 1.01), err(al[i] * 0.99))
+
+
+def test_fp16_rows_are_round_to_nearest():
+    x = inputs.unit_rows(8, 64, seed=13)
+    h, _, _ = oracle.encode_rows(x, oracle.FMT_FP16)
+    xh = oracle.decode_rows(h, oracle.FMT_FP16, 64)
+    # no fp16 value lies strictly closer to x than the chosen one
+    up = np.nextafter(h, np.float16(np.inf)).astype(np.float32)
+    dn = np.nextafter(h, np.float16(-np.inf)).astype(np.float32)
+    d = np.abs(xh - x)
+    assert np.all(d <= np.abs(up - x)) and np.all(d <= np.abs(dn - x))
+
+
+def test_row_scores_agree_with_the_code_scores_on_dequantised_rows():
+    # Q_eps rows s c are a per-row affine code with offset 0; the fp32-row
+    # scorer must reproduce the code scorer (pinned above) on them
+    eps = 1e-2
+    x = inputs.unit_rows(40, 64, seed=14)
+    q = inputs.unit_rows(5, 64, seed=15)
+    codes = oracle.quantize(x, eps)[0].reshape(x.shape)
+    rows = oracle.dequantize(codes, oracle.step(eps))
+    for metric in (oracle.IP, oracle.COSINE, oracle.L2):
+        a = oracle.scores_rows(q, rows, metric)
+        b = oracle.scores(q, codes, eps, metric)
+        np.testing.assert_allclose(a, b, rtol=2e-7, atol=1e-7)
+
+
+def test_row_scores_closed_forms():
+    rows = np.array([[3.0, 4.0], [0.0, 0.0], [-1.0, 0.5]], np.float32)
+    q = np.array([[1.0, 2.0]], np.float32)
+    ip = oracle.scores_rows(q, rows, oracle.IP)[0]
+    cs = oracle.scores_rows(q, rows, oracle.COSINE)[0]
+    l2 = oracle.scores_rows(q, rows, oracle.L2)[0]
+    assert ip.tolist() == [11.0, 0.0, 0.0]
+    assert cs[1] == 0.0 and cs[2] == 0.0
+    assert cs[0] == np.float32(11.0 / (5.0 * math.sqrt(5.0)))
+    assert l2.tolist() == [8.0, 5.0, 6.25]
