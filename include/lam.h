@@ -264,6 +264,71 @@ lam_status lam_score_topk(const float *queries, int64_t B, const void *codes,
                           size_t workspace_bytes, lam_stream_t stream);
 
 /*
+ * Per-vector byte codecs of the composite-reduction experiment (Sec.
+ * "Composite reduction", Table "composite": fp16, per-vector int8 and
+ * sign-binary next to the error-bounded codec).  The paper names them with
+ * their ratios only (3.96x and 30.72x over fp32 at D = 768); the library's
+ * definitions, per row x of D values:
+ *
+ *   LAM_ROWS_INT8  lo = min x, hi = max x, scale = fl32((hi - lo) / 255),
+ *                  c_d = rint_half_even(fl32(fl32(x_d - lo) / scale)) - 128
+ *                  (-128 where scale = 0), offset = fl32(lo + 128 scale);
+ *                  xhat_d = fl32(offset + fl32(scale c_d)).  Codes int8
+ *                  [N, D], scale and offset fp32 [N]: D + 8 bytes a row.
+ *   LAM_ROWS_FP16  c_d = fp16(x_d), round to nearest even; xhat_d = c_d.
+ *                  Codes [N, D] binary16; scale and offset unused.
+ *   LAM_ROWS_SIGN  bit d of row byte d/8 at position d % 8 is (x_d >= 0);
+ *                  scale = alpha = fl32(sum_d |x_d| / D) with the sum in fp64
+ *                  (the least-squares scale for the signs); xhat_d = alpha or
+ *                  -alpha.  Codes uint8 [N, D/8] (D a multiple of 8), scale
+ *                  fp32 [N]: D/8 + 4 bytes a row.
+ *
+ * The alpha of a row may differ by one fp32 ulp from a sum in another order
+ * (the fp64 sum's own error is far below half an fp32 ulp); everything else
+ * is exact.
+ */
+enum { LAM_ROWS_INT8 = 1, LAM_ROWS_FP16 = 2, LAM_ROWS_SIGN = 3 };
+
+/*
+ * lam_encode_rows -- x [N, D] fp32 (device, 4-byte aligned) into the codes
+ * and per-row factors of `fmt` (layouts above; device buffers owned by the
+ * caller, codes aligned to their element, scale/offset 4-byte aligned, NULL
+ * where the codec has none).  Non-finite inputs give unspecified codes.
+ * Asynchronous on `stream`.  Errors: LAM_ERR_INVALID, LAM_ERR_CUDA.
+ *
+ * lam_decode_rows -- the codes back to xhat [N, D] fp32 (device).
+ * Asynchronous.  Errors: LAM_ERR_INVALID, LAM_ERR_CUDA.
+ */
+lam_status lam_encode_rows(const float *x, int64_t N, int32_t D, int32_t fmt, void *codes,
+                           float *scale, float *offset, lam_stream_t stream);
+lam_status lam_decode_rows(const void *codes, int32_t fmt, int64_t N, int32_t D,
+                           const float *scale, const float *offset, float *out,
+                           lam_stream_t stream);
+
+/*
+ * lam_score_topk_rows -- exact search over rows stored in a per-row codec:
+ * the scores of lam_score_topk on the decoded rows xhat (inner product,
+ * cosine with the norm of xhat, squared L2; same ordering and tie rule), with
+ * the decoding folded into the score.  For int8 rows
+ *   q . xhat = scale_i (q . c_i) + offset_i sum_d q_d,
+ * so the codes enter the tensor-core product as they are stored.
+ *
+ * codes, scale, offset as written by lam_encode_rows for `fmt` (a 16-byte
+ * aligned code base enables the tensor-core path).  Other arguments, the
+ * workspace rule, LAM_SCORE_PATH (tensor|generic here) and the status read
+ * (lam_score_topk_status) as for lam_score_topk.  Asynchronous.
+ * Errors: LAM_ERR_INVALID, LAM_ERR_WORKSPACE, LAM_ERR_UNSUPPORTED,
+ * LAM_ERR_CUDA.
+ */
+size_t lam_score_topk_rows_workspace_size(int64_t B, int64_t N, int32_t D, int32_t k,
+                                          int32_t fmt);
+int32_t lam_score_topk_rows_path(int64_t B, int64_t N, int32_t D, int32_t k, int32_t fmt);
+lam_status lam_score_topk_rows(const float *queries, int64_t B, const void *codes, int32_t fmt,
+                               const float *scale, const float *offset, int64_t N, int32_t D,
+                               int32_t k, int32_t metric, float *scores, int64_t *ids,
+                               void *workspace, size_t workspace_bytes, lam_stream_t stream);
+
+/*
  * Waits for `stream`, then reads the device status the last lam_score_topk
  * on this workspace recorded: LAM_OK, LAM_ERR_RANGE or LAM_ERR_TIMEOUT
  * (written to *status_out).  Returns LAM_ERR_CUDA if the read fails.

@@ -470,13 +470,19 @@ void lam_oracle_scores_rows(const float *queries, int64_t B, const float *rows, 
     for (int64_t i = 0; i < N; ++i) {
       const float *x = rows + i * (int64_t)D;
       double dot = 0.0, qq = 0.0, xx = 0.0, l2 = 0.0;
-      for (int32_t d = 0; d < D; ++d) {
-        dot += (double)q[d] * (double)x[d];
-        qq += (double)q[d] * (double)q[d];
-        xx += (double)x[d] * (double)x[d];
-        const double df = (double)q[d] - (double)x[d];
-        l2 += df * df;
+      if (metric == ORACLE_L2) {
+        for (int32_t d = 0; d < D; ++d) {
+          const double df = (double)q[d] - (double)x[d];
+          l2 += df * df;
+        }
+      } else {
+        for (int32_t d = 0; d < D; ++d) dot += (double)q[d] * (double)x[d];
       }
+      if (metric == ORACLE_COSINE)
+        for (int32_t d = 0; d < D; ++d) {
+          qq += (double)q[d] * (double)q[d];
+          xx += (double)x[d] * (double)x[d];
+        }
       float v;
       if (metric == ORACLE_IP) v = (float)dot;
       else if (metric == ORACLE_COSINE) v = (qq == 0.0 || xx == 0.0) ? 0.0f : (float)(dot / (sqrt(qq) * sqrt(xx)));

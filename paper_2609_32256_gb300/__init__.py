@@ -20,7 +20,9 @@ from ._lib import (LAM_ERR_CUDA, LAM_ERR_INVALID, LAM_ERR_NONFINITE, LAM_ERR_RAN
                    lam_timing_begin, lam_timing_end, lam_timing_read, lam_code_sqnorms,
                    lam_quantize_bands, lam_admit_batch, lam_admit_batch_workspace_size,
                    lam_lamz_bound, lam_lamz_compress, lam_lamz_decompress,
-                   lam_lamz_workspace_size)
+                   lam_lamz_workspace_size, LAM_ROWS_INT8, LAM_ROWS_FP16, LAM_ROWS_SIGN,
+                   lam_encode_rows, lam_decode_rows, lam_score_topk_rows,
+                   lam_score_topk_rows_path, lam_score_topk_rows_workspace_size)
 
 CODE_DTYPES = {1: "int8", 2: "int16", 4: "int32"}
 
@@ -76,4 +78,45 @@ def search(queries, codes, eps, k, metric=LAM_METRIC_IP, code_bound=0, stream=No
     st = lam_score_topk_status(ws, stream)
     if st != LAM_OK:
         raise LamError(st, "lam_score_topk")
+    return scores, ids
+
+
+def encode_rows(x, fmt, stream=None):
+    """Per-vector codec of CUDA fp32 rows x [N, D]: (codes, scale, offset),
+    scale/offset None where the codec has none."""
+    torch = _torch()
+    x = x.contiguous()
+    N, D = x.shape
+    dev = x.device
+    if fmt == LAM_ROWS_INT8:
+        codes = torch.empty((N, D), dtype=torch.int8, device=dev)
+    elif fmt == LAM_ROWS_FP16:
+        codes = torch.empty((N, D), dtype=torch.float16, device=dev)
+    else:
+        codes = torch.empty((N, D // 8), dtype=torch.uint8, device=dev)
+    scale = torch.empty(N, dtype=torch.float32, device=dev) if fmt != LAM_ROWS_FP16 else None
+    offset = torch.empty(N, dtype=torch.float32, device=dev) if fmt == LAM_ROWS_INT8 else None
+    lam_encode_rows(x, fmt, codes, scale, offset, stream)
+    return codes, scale, offset
+
+
+def search_rows(queries, codes, fmt, scale, offset, k, metric=LAM_METRIC_IP, D=None,
+                stream=None):
+    """Top-k of every query against rows in a per-vector codec."""
+    torch = _torch()
+    queries = queries.contiguous()
+    B, Dq = queries.shape
+    D = Dq if D is None else D
+    N = codes.shape[0]
+    nbytes = lam_score_topk_rows_workspace_size(B, N, D, k, fmt)
+    if nbytes == 0:
+        raise LamError(LAM_ERR_INVALID, "lam_score_topk_rows_workspace_size")
+    ws = torch.empty(nbytes, dtype=torch.uint8, device=queries.device)
+    scores = torch.empty((B, k), dtype=torch.float32, device=queries.device)
+    ids = torch.empty((B, k), dtype=torch.int64, device=queries.device)
+    lam_score_topk_rows(queries, codes, fmt, scale, offset, N, D, k, metric, scores, ids, ws,
+                        stream)
+    st = lam_score_topk_status(ws, stream)
+    if st != LAM_OK:
+        raise LamError(st, "lam_score_topk_rows")
     return scores, ids

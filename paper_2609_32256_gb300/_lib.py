@@ -66,6 +66,12 @@ def load():
                                   P(ctypes.c_double), P(i64), P(i64), vp]),
         "lam_quantize_bands": (i32, [vp, i64, i32, f32, i32, i32, vp, sz, vp, vp, sz, P(i32),
                                      P(f32), P(i32), P(i32), vp]),
+        "lam_encode_rows": (i32, [vp, i64, i32, i32, vp, vp, vp, vp]),
+        "lam_decode_rows": (i32, [vp, i32, i64, i32, vp, vp, vp, vp]),
+        "lam_score_topk_rows_workspace_size": (sz, [i64, i64, i32, i32, i32]),
+        "lam_score_topk_rows_path": (i32, [i64, i64, i32, i32, i32]),
+        "lam_score_topk_rows": (i32, [vp, i64, vp, i32, vp, vp, i64, i32, i32, i32, vp, vp, vp,
+                                      sz, vp]),
         "lam_timing_begin": (i32, [i32, i64]),
         "lam_timing_read": (i32, [i32, P(ctypes.c_double), P(i64), P(i64)]),
         "lam_timing_end": (i32, []),
@@ -156,6 +162,45 @@ def lam_score_topk(queries, codes, width, N, D, eps, code_bound, k, metric, scor
                                _ptr(scores), _ptr(ids), _ptr(workspace), _nbytes(workspace),
                                _stream(stream, queries.device))
     _check(st, "lam_score_topk")
+
+
+LAM_ROWS_INT8, LAM_ROWS_FP16, LAM_ROWS_SIGN = 1, 2, 3
+
+
+def lam_encode_rows(x, fmt, codes, scale=None, offset=None, stream=None):
+    """Per-vector codec of the fp32 rows x [N, D] into codes (int8 [N, D],
+    fp16 [N, D] or uint8 [N, D/8]) and per-row scale/offset (asynchronous)."""
+    N, D = x.shape
+    st = load().lam_encode_rows(_ptr(x), int(N), int(D), int(fmt), _ptr(codes), _ptr(scale),
+                                _ptr(offset), _stream(stream, x.device))
+    _check(st, "lam_encode_rows")
+
+
+def lam_decode_rows(codes, fmt, N, D, scale, offset, out, stream=None):
+    """xhat [N, D] fp32 of per-vector codes (asynchronous)."""
+    st = load().lam_decode_rows(_ptr(codes), int(fmt), int(N), int(D), _ptr(scale),
+                                _ptr(offset), _ptr(out), _stream(stream, out.device))
+    _check(st, "lam_decode_rows")
+
+
+def lam_score_topk_rows_workspace_size(B, N, D, k, fmt) -> int:
+    return int(load().lam_score_topk_rows_workspace_size(int(B), int(N), int(D), int(k),
+                                                         int(fmt)))
+
+
+def lam_score_topk_rows_path(B, N, D, k, fmt) -> int:
+    return int(load().lam_score_topk_rows_path(int(B), int(N), int(D), int(k), int(fmt)))
+
+
+def lam_score_topk_rows(queries, codes, fmt, scale, offset, N, D, k, metric, scores, ids,
+                        workspace, stream=None):
+    """Exact search over per-vector coded rows; writes scores/ids [B, k]."""
+    B = queries.shape[0]
+    st = load().lam_score_topk_rows(_ptr(queries), int(B), _ptr(codes), int(fmt), _ptr(scale),
+                                    _ptr(offset), int(N), int(D), int(k), int(metric),
+                                    _ptr(scores), _ptr(ids), _ptr(workspace), _nbytes(workspace),
+                                    _stream(stream, queries.device))
+    _check(st, "lam_score_topk_rows")
 
 
 def lam_score_topk_status(workspace, stream=None) -> int:

@@ -125,6 +125,39 @@ bool make_plan(int64_t B, int64_t N, int32_t D, int32_t k, int32_t width, int32_
   return true;
 }
 
+// Per-row codecs: shape checks and the plan (tensor path with the converting
+// pass, else the generic path; no bandwidth kernel).
+bool rows_shape_ok(int64_t B, int64_t N, int32_t D, int32_t k, int32_t fmt) {
+  if (fmt != LAM_ROWS_INT8 && fmt != LAM_ROWS_FP16 && fmt != LAM_ROWS_SIGN) return false;
+  if (fmt == LAM_ROWS_SIGN && D % 8 != 0) return false;
+  return shape_ok(B, N, D, k, 1, 0);
+}
+
+bool make_rows_plan(int64_t B, int64_t N, int32_t D, int32_t k, int32_t fmt, int sms, Plan *p) {
+  if (!rows_shape_ok(B, N, D, k, fmt) || sms <= 0) return false;
+  const bool tc = D % 16 == 0 && tensor_fits_pre(k) && B <= (1LL << 23);
+  const int f = forced_path();
+  if (f == -2) return false;
+  int path = tc ? kPathTensor : kPathGeneric;
+  if (f >= 0) {
+    if (f == kPathBandwidth || (f == kPathTensor && !tc)) {
+      p->path = -2;
+      return false;
+    }
+    path = f;
+  }
+  p->path = path;
+  p->n_lists = path == kPathTensor ? tensor_plan(B, N, D, k, sms, true).n_lists
+                                   : generic_ctas(B, N, sms);
+  p->Bpad = (B + 127) / 128 * 128;
+  p->partial_off = kHeaderBytes;
+  const size_t partial = (size_t)p->n_lists * (size_t)B * (size_t)k * 8;
+  p->qprep_off = align_up(p->partial_off + partial, 256);
+  p->total = p->qprep_off;
+  if (path == kPathTensor) p->total += align_up(tensor_plan(B, N, D, k, sms, true).bytes, 256);
+  return true;
+}
+
 }  // namespace
 
 namespace lam {
@@ -571,6 +604,137 @@ lam_status lam_score_topk(const float *queries, int64_t B, const void *codes, in
   if (p.path == kPathBandwidth) e = launch_score_bandwidth(a, st);
   else if (p.path == kPathTensor) e = launch_score_tensor(a, st);
   else e = launch_score_generic(a, st);
+  if (e != cudaSuccess) return LAM_ERR_CUDA;
+  if (launch_topk_merge(a, st) != cudaSuccess) return LAM_ERR_CUDA;
+  return LAM_OK;
+}
+
+lam_status lam_encode_rows(const float *x, int64_t N, int32_t D, int32_t fmt, void *codes,
+                           float *scale, float *offset, lam_stream_t stream) {
+  if (N < 0 || D < 1 || D > (1 << 20)) return LAM_ERR_INVALID;
+  if (fmt != LAM_ROWS_INT8 && fmt != LAM_ROWS_FP16 && fmt != LAM_ROWS_SIGN) return LAM_ERR_INVALID;
+  if (fmt == LAM_ROWS_SIGN && D % 8 != 0) return LAM_ERR_INVALID;
+  if (N >= (1LL << 40) / D) return LAM_ERR_INVALID;
+  if (N == 0) return LAM_OK;
+  if (x == nullptr || codes == nullptr) return LAM_ERR_INVALID;
+  if (fmt != LAM_ROWS_FP16 && scale == nullptr) return LAM_ERR_INVALID;
+  if (fmt == LAM_ROWS_INT8 && offset == nullptr) return LAM_ERR_INVALID;
+  if ((reinterpret_cast<uintptr_t>(x) & 3u) != 0 ||
+      (fmt == LAM_ROWS_FP16 && (reinterpret_cast<uintptr_t>(codes) & 1u) != 0) ||
+      (reinterpret_cast<uintptr_t>(scale) & 3u) != 0 ||
+      (reinterpret_cast<uintptr_t>(offset) & 3u) != 0)
+    return LAM_ERR_INVALID;
+  const int sms = device_sms();
+  if (sms <= 0) return LAM_ERR_CUDA;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  timing_launch_begin(LAM_TIME_QUANTIZE, st);
+  const cudaError_t e = launch_encode_rows(x, N, D, fmt, codes, scale, offset, sms, st);
+  timing_launch_end(LAM_TIME_QUANTIZE, st);
+  return e == cudaSuccess ? LAM_OK : LAM_ERR_CUDA;
+}
+
+lam_status lam_decode_rows(const void *codes, int32_t fmt, int64_t N, int32_t D,
+                           const float *scale, const float *offset, float *out,
+                           lam_stream_t stream) {
+  if (N < 0 || D < 1 || D > (1 << 20)) return LAM_ERR_INVALID;
+  if (fmt != LAM_ROWS_INT8 && fmt != LAM_ROWS_FP16 && fmt != LAM_ROWS_SIGN) return LAM_ERR_INVALID;
+  if (fmt == LAM_ROWS_SIGN && D % 8 != 0) return LAM_ERR_INVALID;
+  if (N >= (1LL << 40) / D) return LAM_ERR_INVALID;
+  if (N == 0) return LAM_OK;
+  if (codes == nullptr || out == nullptr) return LAM_ERR_INVALID;
+  if (fmt != LAM_ROWS_FP16 && scale == nullptr) return LAM_ERR_INVALID;
+  if (fmt == LAM_ROWS_INT8 && offset == nullptr) return LAM_ERR_INVALID;
+  if ((reinterpret_cast<uintptr_t>(out) & 3u) != 0 ||
+      (fmt == LAM_ROWS_FP16 && (reinterpret_cast<uintptr_t>(codes) & 1u) != 0) ||
+      (reinterpret_cast<uintptr_t>(scale) & 3u) != 0 ||
+      (reinterpret_cast<uintptr_t>(offset) & 3u) != 0)
+    return LAM_ERR_INVALID;
+  const int sms = device_sms();
+  if (sms <= 0) return LAM_ERR_CUDA;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  timing_launch_begin(LAM_TIME_DEQUANTIZE, st);
+  const cudaError_t e = launch_decode_rows(codes, fmt, N, D, scale, offset, out, sms, st);
+  timing_launch_end(LAM_TIME_DEQUANTIZE, st);
+  return e == cudaSuccess ? LAM_OK : LAM_ERR_CUDA;
+}
+
+size_t lam_score_topk_rows_workspace_size(int64_t B, int64_t N, int32_t D, int32_t k,
+                                          int32_t fmt) {
+  Plan p;
+  const int sms = device_sms();
+  if (!make_rows_plan(B, N, D, k, fmt, sms, &p)) return 0;
+  const size_t generic = align_up(kHeaderBytes + (size_t)generic_ctas(B, N, sms) * B * k * 8, 256);
+  return p.total > generic ? p.total : generic;
+}
+
+int32_t lam_score_topk_rows_path(int64_t B, int64_t N, int32_t D, int32_t k, int32_t fmt) {
+  Plan p;
+  if (!make_rows_plan(B, N, D, k, fmt, device_sms(), &p)) return -1;
+  return p.path;
+}
+
+lam_status lam_score_topk_rows(const float *queries, int64_t B, const void *codes, int32_t fmt,
+                               const float *scale, const float *offset, int64_t N, int32_t D,
+                               int32_t k, int32_t metric, float *scores, int64_t *ids,
+                               void *workspace, size_t workspace_bytes, lam_stream_t stream) {
+  if (queries == nullptr || codes == nullptr || scores == nullptr || ids == nullptr ||
+      workspace == nullptr)
+    return LAM_ERR_INVALID;
+  if (metric != LAM_METRIC_IP && metric != LAM_METRIC_COSINE && metric != LAM_METRIC_L2)
+    return LAM_ERR_INVALID;
+  if (!rows_shape_ok(B, N, D, k, fmt)) return LAM_ERR_INVALID;
+  if (fmt != LAM_ROWS_FP16 && scale == nullptr) return LAM_ERR_INVALID;
+  if (fmt == LAM_ROWS_INT8 && offset == nullptr) return LAM_ERR_INVALID;
+  if ((reinterpret_cast<uintptr_t>(workspace) & 255u) != 0) return LAM_ERR_INVALID;
+  if ((fmt == LAM_ROWS_FP16 && (reinterpret_cast<uintptr_t>(codes) & 1u) != 0) ||
+      (reinterpret_cast<uintptr_t>(scale) & 3u) != 0 ||
+      (reinterpret_cast<uintptr_t>(offset) & 3u) != 0 ||
+      (reinterpret_cast<uintptr_t>(queries) & 3u) != 0 ||
+      (reinterpret_cast<uintptr_t>(scores) & 3u) != 0 || (reinterpret_cast<uintptr_t>(ids) & 7u) != 0)
+    return LAM_ERR_INVALID;
+  const int sms = device_sms();
+  if (sms <= 0) return LAM_ERR_CUDA;
+  Plan p;
+  if (!make_rows_plan(B, N, D, k, fmt, sms, &p))
+    return p.path == -2 ? LAM_ERR_UNSUPPORTED : LAM_ERR_INVALID;
+  // the converting pass reads 8- or 16-byte code vectors: a 16-byte aligned base
+  const bool aligned = (reinterpret_cast<uintptr_t>(codes) & 15u) == 0;
+  if (!aligned && p.path != kPathGeneric) {
+    if (forced_path() >= 0) return LAM_ERR_UNSUPPORTED;
+    p.path = kPathGeneric;
+    p.n_lists = generic_ctas(B, N, sms);
+    p.qprep_off = align_up(p.partial_off + (size_t)p.n_lists * B * k * 8, 256);
+    p.total = p.qprep_off;
+  }
+  if (workspace_bytes < p.total) return LAM_ERR_WORKSPACE;
+
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  uint8_t *ws = static_cast<uint8_t *>(workspace);
+  if (cudaMemsetAsync(ws, 0, kHeaderBytes, st) != cudaSuccess) return LAM_ERR_CUDA;
+  ScoreArgs a{};
+  a.queries = queries;
+  a.B = B;
+  a.codes = codes;
+  a.width = 1;
+  a.N = N;
+  a.D = D;
+  a.s = 1.0f;
+  a.code_bound = 0;
+  a.k = k;
+  a.metric = metric;
+  a.scores = scores;
+  a.ids = ids;
+  a.gflags = reinterpret_cast<uint32_t *>(ws);
+  a.partial = reinterpret_cast<uint64_t *>(ws + p.partial_off);
+  a.n_lists = p.n_lists;
+  a.qprep = ws + p.qprep_off;
+  a.Bpad = p.Bpad;
+  a.sms = sms;
+  a.fmt = fmt;
+  a.row_scale = scale;
+  a.row_offset = offset;
+  const cudaError_t e =
+      p.path == kPathTensor ? launch_score_tensor(a, st) : launch_score_generic(a, st);
   if (e != cudaSuccess) return LAM_ERR_CUDA;
   if (launch_topk_merge(a, st) != cudaSuccess) return LAM_ERR_CUDA;
   return LAM_OK;

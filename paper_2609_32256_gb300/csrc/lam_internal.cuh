@@ -198,7 +198,30 @@ struct ScoreArgs {
   void *qprep;          // tensor path: fp16 [2*Bpad][D] then float4 [Bpad]
   int64_t Bpad;
   int sms;
+  // Per-row codecs (lam_score_topk_rows): LAM_ROWS_* (0: Q_eps codes, the
+  // fields above), per-row scale and offset.
+  int fmt = 0;
+  const float *row_scale = nullptr;
+  const float *row_offset = nullptr;
 };
+
+// Decoded value xhat_d of row `row` of a per-row codec, evaluated exactly as
+// lam_decode_rows writes it.
+__device__ __forceinline__ float row_value(const ScoreArgs &a, int64_t row, int d) {
+  if (a.fmt == LAM_ROWS_INT8)
+    return __fadd_rn(a.row_offset[row],
+                     __fmul_rn(a.row_scale[row],
+                               (float)static_cast<const int8_t *>(a.codes)[row * a.D + d]));
+  if (a.fmt == LAM_ROWS_FP16)
+    return __half2float(static_cast<const __half *>(a.codes)[row * a.D + d]);
+  const uint8_t byte = static_cast<const uint8_t *>(a.codes)[row * (a.D / 8) + d / 8];
+  return ((byte >> (d & 7)) & 1u) ? a.row_scale[row] : -a.row_scale[row];
+}
+
+cudaError_t launch_encode_rows(const float *x, int64_t N, int D, int fmt, void *codes,
+                               float *scale, float *offset, int sms, cudaStream_t st);
+cudaError_t launch_decode_rows(const void *codes, int fmt, int64_t N, int D, const float *scale,
+                               const float *offset, float *out, int sms, cudaStream_t st);
 
 cudaError_t launch_score_bandwidth(const ScoreArgs &a, cudaStream_t st);
 cudaError_t launch_score_generic(const ScoreArgs &a, cudaStream_t st);
@@ -210,15 +233,17 @@ enum Path { kPathBandwidth = 0, kPathTensor = 1, kPathGeneric = 2 };
 int bandwidth_ctas(int64_t N, int D, int width, int sms);
 int tensor_splits(int64_t B, int64_t N, int sms);
 bool tensor_fits(int width, int k);  // shared memory holds >= 2 stages
+bool tensor_fits_pre(int k);         // the same for the converting-pass kernel alone
 // Tensor-path workspace (after the partial lists): [query images][query info]
 // and, for two or more query blocks, [fp16 code slab][per-row factors].
 struct TensorPlan {
   bool pre;            // codes converted to fp16 by a separate pass
   int64_t slab_rows;   // rows per slab (pre), else N
   int nslabs, nsplit, n_lists;
-  size_t qinfo_off, fp16_off, rowf_off, bytes;
+  size_t qinfo_off, fp16_off, rowf_off, bytes;  // rowf: 16 bytes per slab row
 };
-TensorPlan tensor_plan(int64_t B, int64_t N, int D, int k, int sms);
+// (force_pre: the per-row codecs always take the converting pass)
+TensorPlan tensor_plan(int64_t B, int64_t N, int D, int k, int sms, bool force_pre = false);
 
 // Launch bracketing for lam_timing_* (no-ops unless timing is on for `kind`).
 void timing_launch_begin(int kind, cudaStream_t st);

@@ -284,7 +284,8 @@ __global__ void __launch_bounds__(kGenWarps * 32) score_generic_kernel(ScoreArgs
   for (int d = lane; d < D; d += 32) part = fmaf(q[d], q[d], part);
   const float qq = warp_sum(part), qn = sqrtf(qq);
   const bool desc = a.metric != LAM_METRIC_L2;
-  const float s = a.s, s2 = a.s * a.s;
+  // per-row codecs score the decoded rows themselves (unit step)
+  const float s = a.fmt ? 1.0f : a.s, s2 = s * s;
 
   const int64_t r0 = (int64_t)blockIdx.x * a.N / gridDim.x;
   const int64_t r1 = (int64_t)(blockIdx.x + 1) * a.N / gridDim.x;
@@ -292,7 +293,7 @@ __global__ void __launch_bounds__(kGenWarps * 32) score_generic_kernel(ScoreArgs
     float acc = 0.0f, cc = 0.0f;
     const int64_t base = row * D;
     for (int d = lane; d < D; d += 32) {
-      const float c = (float)load_code(a.codes, a.width, base + d);
+      const float c = a.fmt ? row_value(a, row, d) : (float)load_code(a.codes, a.width, base + d);
       acc = fmaf(q[d], c, acc);
       cc = fmaf(c, c, cc);
     }
@@ -380,7 +381,9 @@ __global__ void __launch_bounds__(kMergeThreads) topk_merge_kernel(ScoreArgs a, 
       float acc = 0.0f;
       if (row < a.N) {
         for (int d = lane; d < a.D; d += 32) {
-          const float xh = __fmul_rn(a.s, (float)load_code(a.codes, a.width, (int64_t)row * a.D + d));
+          const float xh = a.fmt ? row_value(a, row, d)
+                                 : __fmul_rn(a.s, (float)load_code(a.codes, a.width,
+                                                                   (int64_t)row * a.D + d));
           const float df = __fsub_rn(q[d], xh);
           acc = fmaf(df, df, acc);
         }
@@ -476,7 +479,9 @@ __global__ void __launch_bounds__(kKmWarps * 32) topk_kmerge_kernel(ScoreArgs a,
         float acc = 0.0f;
         if (row < a.N) {
           for (int d = lane; d < a.D; d += 32) {
-            const float xh = __fmul_rn(a.s, (float)load_code(a.codes, a.width, (int64_t)row * a.D + d));
+            const float xh = a.fmt ? row_value(a, row, d)
+                                 : __fmul_rn(a.s, (float)load_code(a.codes, a.width,
+                                                                   (int64_t)row * a.D + d));
             const float df = __fsub_rn(q[d], xh);
             acc = fmaf(df, df, acc);
           }

@@ -615,7 +615,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 // stages load (per query block and 32-wide K slice: [hi 128 x 64 B | lo], rows
 // 64 bytes apart with the 16-byte chunks of row r XOR-ed by (r >> 1) & 3, the
 // 64-byte swizzle), zeros for padding rows and columns; then (2^-e, ||q||,
-// ||q||^2, 0) per query after the images.
+// ||q||^2, sum_d q_d) per query after the images.
 __device__ __forceinline__ void qprep_block(const float *__restrict__ q, int64_t B, int D,
                                             int64_t Bpad, uint8_t *__restrict__ qA, int64_t blk) {
   const int64_t b = blk * 8 + (threadIdx.x >> 5);
@@ -627,17 +627,19 @@ __device__ __forceinline__ void qprep_block(const float *__restrict__ q, int64_t
   float4 *qinfo = reinterpret_cast<float4 *>(qA + (size_t)(Bpad / kBM) * nk * kAStage);
   const bool valid = b < B;
   const float *qr = q + b * D;
-  float mx = 0.0f, qq = 0.0f;
+  float mx = 0.0f, qq = 0.0f, qs = 0.0f;
   if (valid) {
     for (int d = lane; d < D; d += 32) {
       const float v = qr[d];
       mx = fmaxf(mx, fabsf(v));
       qq = fmaf(v, v, qq);
+      qs += v;
     }
   }
   for (int off = 16; off > 0; off >>= 1) {
     mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
     qq += __shfl_xor_sync(0xffffffffu, qq, off);
+    qs += __shfl_xor_sync(0xffffffffu, qs, off);
   }
   int e = 0;
   if (mx > 0.0f) {
@@ -668,7 +670,7 @@ __device__ __forceinline__ void qprep_block(const float *__restrict__ q, int64_t
     *reinterpret_cast<uint4 *>(qA + off + kABytes) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
   }
   if (lane == 0)
-    qinfo[b] = valid ? make_float4(ldexpf(1.0f, -e), sqrtf(qq), qq, 0.0f)
+    qinfo[b] = valid ? make_float4(ldexpf(1.0f, -e), sqrtf(qq), qq, qs)
                      : make_float4(0.f, 0.f, 0.f, 0.f);
 }
 
@@ -765,6 +767,114 @@ __global__ void __launch_bounds__(256) prep_convert_kernel(
                      blockIdx.x - q_blocks);
 }
 
+// Per-row codecs: the stored codes become the fp16 operand image as they are
+// (int8 codes c, fp16 values, sign bits as +-1), and the decoding moves into
+// per-row factors (u, w, z) of the score
+//   q . xhat = pw (q 2^e) . c * a + (sum q) * o      (a, o: scale, offset)
+//   inner product / squared L2   u = a, w = o, z = ||xhat||^2
+//   cosine                       u = a / ||xhat||, w = o / ||xhat||
+// with ||xhat||^2 summed over xhat_d exactly as the decoder forms it.
+template <int FMT>
+__device__ __forceinline__ void convert_rows_block(const void *__restrict__ codes,
+                                                   const float *__restrict__ rscale,
+                                                   const float *__restrict__ roff,
+                                                   int64_t row_base, int64_t nrows,
+                                                   int64_t nrows_pad, int D,
+                                                   uint8_t *__restrict__ out,
+                                                   float4 *__restrict__ rowf4, int metric,
+                                                   int64_t blk) {
+  const int64_t r = blk * 8 + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (r >= nrows_pad) return;
+  const bool valid = r < nrows;
+  const int nk = (D + kBK - 1) / kBK;
+  const int rr = (int)(r % kBN);
+  const int sw = (rr >> 1) & 3;
+  uint8_t *dst = out + (size_t)(r / kBN) * nk * kB16Bytes + (size_t)rr * 64;
+  const int64_t grow = row_base + r;
+  float sa = 1.0f, so = 0.0f;
+  if (valid && FMT != LAM_ROWS_FP16) sa = rscale[grow];
+  if (valid && FMT == LAM_ROWS_INT8) so = roff[grow];
+  float xx = 0.0f;
+  for (int ch = lane; ch < nk * (kBK / 8); ch += 32) {
+    const int d0 = ch * 8;
+    uint32_t o[4] = {0u, 0u, 0u, 0u};
+    if (valid && d0 < D) {  // D is a multiple of 16: a chunk is all in or all out
+      if (FMT == LAM_ROWS_INT8) {
+        const uint2 v = *reinterpret_cast<const uint2 *>(static_cast<const int8_t *>(codes) +
+                                                         grow * D + d0);
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+          const uint32_t wv = t < 2 ? v.x : v.y;
+          const float c0 = (float)(int8_t)(wv >> (16 * (t & 1)));
+          const float c1 = (float)(int8_t)(wv >> (16 * (t & 1) + 8));
+          const float x0 = __fadd_rn(so, __fmul_rn(sa, c0));
+          const float x1 = __fadd_rn(so, __fmul_rn(sa, c1));
+          xx = fmaf(x0, x0, fmaf(x1, x1, xx));
+          o[t] = h2_as_u32(__floats2half2_rn(c0, c1));
+        }
+      } else if (FMT == LAM_ROWS_FP16) {
+        const uint4 v = *reinterpret_cast<const uint4 *>(static_cast<const __half *>(codes) +
+                                                         grow * D + d0);
+        o[0] = v.x;
+        o[1] = v.y;
+        o[2] = v.z;
+        o[3] = v.w;
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+          __half2 h;
+          memcpy(&h, &o[t], 4);
+          const float2 f = __half22float2(h);
+          xx = fmaf(f.x, f.x, fmaf(f.y, f.y, xx));
+        }
+      } else {
+        const uint32_t byte = static_cast<const uint8_t *>(codes)[grow * (D / 8) + ch];
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {  // +1 = 0x3C00, -1 = 0xBC00 in binary16
+          const uint32_t lo = ((byte >> (2 * t)) & 1u) ? 0x3C00u : 0xBC00u;
+          const uint32_t hi = ((byte >> (2 * t + 1)) & 1u) ? 0x3C00u : 0xBC00u;
+          o[t] = lo | (hi << 16);
+          xx = fmaf(sa, sa, fmaf(sa, sa, xx));
+        }
+      }
+    }
+    *reinterpret_cast<uint4 *>(dst + (size_t)(ch >> 2) * kB16Bytes + (((ch & 3) ^ sw) << 4)) =
+        make_uint4(o[0], o[1], o[2], o[3]);
+  }
+  xx = warp_sum_tc(xx);
+  if (lane == 0 && valid) {
+    float u = sa, w = so;
+    if (metric == LAM_METRIC_COSINE) {
+      const float inv = xx > 0.0f ? 1.0f / sqrtf(xx) : 0.0f;
+      u = sa * inv;
+      w = so * inv;
+    }
+    rowf4[r] = make_float4(u, w, xx, 0.0f);
+  }
+}
+
+template <int FMT>
+__global__ void __launch_bounds__(256) convert_rows_kernel(
+    const void *__restrict__ codes, const float *__restrict__ rscale,
+    const float *__restrict__ roff, int64_t row_base, int64_t nrows, int64_t nrows_pad, int D,
+    uint8_t *__restrict__ out, float4 *__restrict__ rowf4, int metric) {
+  convert_rows_block<FMT>(codes, rscale, roff, row_base, nrows, nrows_pad, D, out, rowf4, metric,
+                          blockIdx.x);
+}
+
+template <int FMT>
+__global__ void __launch_bounds__(256) prep_convert_rows_kernel(
+    const float *__restrict__ q, int64_t B, int D, int64_t Bpad, uint8_t *__restrict__ qA,
+    unsigned q_blocks, const void *__restrict__ codes, const float *__restrict__ rscale,
+    const float *__restrict__ roff, int64_t nrows, int64_t nrows_pad, uint8_t *__restrict__ out,
+    float4 *__restrict__ rowf4, int metric) {
+  if (blockIdx.x < q_blocks)
+    qprep_block(q, B, D, Bpad, qA, blockIdx.x);
+  else
+    convert_rows_block<FMT>(codes, rscale, roff, 0, nrows, nrows_pad, D, out, rowf4, metric,
+                            blockIdx.x - q_blocks);
+}
+
 struct Tc2Layout {
   int ns;
   size_t lists_off, cbuf_off, bar_off, smem_bytes;
@@ -793,10 +903,57 @@ struct Tc2Geom {
   int64_t row_base, nrows;  // the slab
   int list_base;            // partial-list index of this slab's split 0
   const uint8_t *b16;       // fp16 operand image of the slab
-  const float *rowf;        // per-row factors of the slab
+  const float *rowf;        // per-row factors of the slab (Q_eps codes)
+  const float4 *rowf4;      // per-row (u, w, z) of the slab (per-row codecs)
 };
 
-template <int KR>
+// Per-row score factors of one 32-row chunk, one row per lane, and their
+// broadcast for row j (all lanes must call at()).
+template <bool RC>
+struct RowFac;
+template <>
+struct RowFac<false> {
+  float r;
+  __device__ __forceinline__ void load(const Tc2Geom &g, int64_t i, bool ok, bool need) {
+    r = need && ok ? g.rowf[i] : 0.0f;
+  }
+  __device__ __forceinline__ RowFac at(int j, bool) const {
+    RowFac f;
+    f.r = __shfl_sync(0xffffffffu, r, j);
+    return f;
+  }
+};
+template <>
+struct RowFac<true> {
+  float u, w, z;
+  __device__ __forceinline__ void load(const Tc2Geom &g, int64_t i, bool ok, bool) {
+    const float4 v = ok ? g.rowf4[i] : make_float4(0.f, 0.f, 0.f, 0.f);
+    u = v.x;
+    w = v.y;
+    z = v.z;
+  }
+  __device__ __forceinline__ RowFac at(int j, bool l2) const {
+    RowFac f;
+    f.u = __shfl_sync(0xffffffffu, u, j);
+    f.w = __shfl_sync(0xffffffffu, w, j);
+    f.z = l2 ? __shfl_sync(0xffffffffu, z, j) : 0.0f;
+    return f;
+  }
+};
+// Per-query factors: fq multiplies the accumulator, fs the row offset term.
+struct QFac {
+  float fq, fs, qq;
+  int metric;
+};
+__device__ __forceinline__ float fac_score(const RowFac<false> &f, float acc, const QFac &q) {
+  return tile_score(q.metric, acc, q.fq, q.qq, f.r);
+}
+__device__ __forceinline__ float fac_score(const RowFac<true> &f, float acc, const QFac &q) {
+  const float dot = fmaf(q.fq * f.u, acc, q.fs * f.w);
+  return q.metric == LAM_METRIC_L2 ? fmaf(-2.0f, dot, q.qq + f.z) : dot;
+}
+
+template <int KR, bool RC>
 __global__ void __launch_bounds__(kTc2Threads, 1)
     score_tc2_kernel(ScoreArgs a, Tc2Geom g) {
   extern __shared__ uint8_t tc_smem_raw[];
@@ -819,7 +976,7 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
   const int64_t te = (int64_t)(blockIdx.x + 1) * n_tiles / gridDim.x;
   const int ntl = (int)(te - tb);
   const int nk = (a.D + kBK - 1) / kBK;
-  const bool need_cc = a.metric != LAM_METRIC_IP;
+  const bool need_cc = RC || a.metric != LAM_METRIC_IP;
   const uint8_t *qA = static_cast<const uint8_t *>(a.qprep);
 
   if (threadIdx.x == 0) {
@@ -907,17 +1064,29 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
     const int k = a.k;
     const bool desc = a.metric != LAM_METRIC_L2;
     const float s = a.s;
-    float pw = 0.0f, qn = 0.0f, qq = 0.0f;
+    float pw = 0.0f, qn = 0.0f, qq = 0.0f, qs = 0.0f;
     if (qvalid) {
       const float4 qi = reinterpret_cast<const float4 *>(
           qA + (size_t)(a.Bpad / kBM) * nk * kAStage)[qidx];
       pw = qi.x;
       qn = qi.y;
       qq = qi.z;
+      qs = qi.w;
     }
-    const float fq = a.metric == LAM_METRIC_IP ? s * pw
-                     : a.metric == LAM_METRIC_COSINE ? (qn > 0.0f ? pw / qn : 0.0f)
-                                                     : -2.0f * s * pw;
+    QFac qf;
+    qf.metric = a.metric;
+    qf.qq = qq;
+    qf.fs = 0.0f;
+    if (RC) {
+      const float inv = a.metric == LAM_METRIC_COSINE ? (qn > 0.0f ? 1.0f / qn : 0.0f) : 1.0f;
+      qf.fq = pw * inv;
+      qf.fs = qs * inv;
+    } else {
+      qf.fq = a.metric == LAM_METRIC_IP ? s * pw
+              : a.metric == LAM_METRIC_COSINE ? (qn > 0.0f ? pw / qn : 0.0f)
+                                              : -2.0f * s * pw;
+    }
+    const bool l2 = a.metric == LAM_METRIC_L2;
     constexpr int RK = KR > 0 ? KR : 1;
     RegTopK<RK> reg;
     reg.init(k);
@@ -942,7 +1111,8 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
 #pragma unroll 1
         for (int c = 0; c < kBN / 32; ++c) {
           uint32_t v[32];
-          const float rfl = need_cc ? g.rowf[row0 + c * 32 + lane] : 0.0f;
+          RowFac<RC> rl;
+          rl.load(g, row0 + c * 32 + lane, true, need_cc);
           tmem_ld32(taddr + c * 32, v);
           // shift register: the P bests of this chunk enter at the top
 #pragma unroll
@@ -952,8 +1122,7 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
             float best = -INFINITY;
 #pragma unroll
             for (int j = h * GR; j < (h + 1) * GR; ++j) {
-              const float sc = tile_score(a.metric, __uint_as_float(v[j]), fq, qq,
-                                          __shfl_sync(0xffffffffu, rfl, j));
+              const float sc = fac_score(rl.at(j, l2), __uint_as_float(v[j]), qf);
               best = fmaxf(best, desc ? sc : -sc);
             }
             gb[NG - P + h] = best;
@@ -966,15 +1135,15 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
       for (int c = 0; c < kBN / 32; ++c) {
         uint32_t v[32];
         const int64_t nvalid = g.nrows - (row0 + c * 32);
-        // lane j holds the factor of row j of this chunk
-        const float rfl = need_cc && lane < nvalid ? g.rowf[row0 + c * 32 + lane] : 0.0f;
+        // lane j holds the factors of row j of this chunk
+        RowFac<RC> rl;
+        rl.load(g, row0 + c * 32 + lane, lane < nvalid, need_cc);
         tmem_ld32(taddr + c * 32, v);
         const float thr = desc ? fmaxf(thr_s, seed) : fminf(thr_s, seed);
         uint32_t mask = 0;
 #pragma unroll
         for (int j = 0; j < 32; ++j) {
-          const float rf = __shfl_sync(0xffffffffu, rfl, j);
-          const float sc = tile_score(a.metric, __uint_as_float(v[j]), fq, qq, rf);
+          const float sc = fac_score(rl.at(j, l2), __uint_as_float(v[j]), qf);
           mask |= (uint32_t)(desc ? sc > thr : sc < thr) << j;
         }
         if (!qvalid || nvalid <= 0) mask = 0;
@@ -985,11 +1154,11 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
           // (re-tested against the threshold the earlier steps tightened)
           while (__any_sync(0xffffffffu, mask != 0)) {
             const int j = mask != 0 ? __ffs(mask) - 1 : 0;
-            const float rf = __shfl_sync(0xffffffffu, rfl, j);
+            const RowFac<RC> rf = rl.at(j, l2);
             uint32_t kc = 0xffffffffu, ic = 0xffffffffu;
             if (mask != 0) {
               mask &= mask - 1;
-              const float sc = tile_score(a.metric, __uint_as_float(select32(v, j)), fq, qq, rf);
+              const float sc = fac_score(rf, __uint_as_float(select32(v, j)), qf);
               if (desc ? sc > thr_s : sc < thr_s) {
                 kc = rank_key32(sc, desc);
                 ic = grow0 + j;
@@ -1002,10 +1171,10 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
         } else {
           while (__any_sync(0xffffffffu, mask != 0)) {
             const int j = mask != 0 ? __ffs(mask) - 1 : 0;
-            const float rf = __shfl_sync(0xffffffffu, rfl, j);
+            const RowFac<RC> rf = rl.at(j, l2);
             if (mask == 0) continue;
             mask &= mask - 1;
-            const float sc = tile_score(a.metric, __uint_as_float(select32(v, j)), fq, qq, rf);
+            const float sc = fac_score(rf, __uint_as_float(select32(v, j)), qf);
             const uint64_t key = make_key(sc, grow0 + j, desc);
             if (key < lists[m]) {
               heap_replace_root(lists, k, kBM, m, key);
@@ -1089,6 +1258,8 @@ bool tensor_fits(int width, int k) {
   return tc_layout(width, k).ns >= 2 && tc2_layout(k).ns >= 2;
 }
 
+bool tensor_fits_pre(int k) { return k <= kTcMaxK && tc2_layout(k).ns >= 2; }
+
 int tensor_splits(int64_t B, int64_t N, int sms) {
   const int64_t nqb = (B + kBM - 1) / kBM;
   const int64_t n_tiles = (N + kBN - 1) / kBN;
@@ -1099,11 +1270,11 @@ int tensor_splits(int64_t B, int64_t N, int sms) {
   return (int)ns;
 }
 
-TensorPlan tensor_plan(int64_t B, int64_t N, int D, int k, int sms) {
+TensorPlan tensor_plan(int64_t B, int64_t N, int D, int k, int sms, bool force_pre) {
   TensorPlan p;
   const int64_t Bpad = (B + kBM - 1) / kBM * kBM;
   const int64_t nk = (D + kBK - 1) / kBK;
-  p.pre = Bpad / kBM >= 2;
+  p.pre = force_pre || Bpad / kBM >= 2;
   p.qinfo_off = (size_t)(Bpad / kBM) * nk * kAStage;
   size_t off = p.qinfo_off + (size_t)Bpad * 16;
   off = (off + 255) / 256 * 256;
@@ -1121,15 +1292,16 @@ TensorPlan tensor_plan(int64_t B, int64_t N, int D, int k, int sms) {
     p.nsplit = tensor_splits(B, p.slab_rows, sms);
     p.fp16_off = off;
     p.rowf_off = p.fp16_off + (size_t)((p.slab_rows + kBN - 1) / kBN) * nk * kB16Bytes;
-    p.bytes = p.rowf_off + (size_t)p.slab_rows * 4;
+    p.bytes = p.rowf_off + (size_t)p.slab_rows * 16;
   }
   p.n_lists = p.nslabs * p.nsplit;
   return p;
 }
 
 cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st) {
-  if (a.k > kTcMaxK || (a.width != 1 && a.width != 2)) return cudaErrorInvalidValue;
-  const TensorPlan P = tensor_plan(a.B, a.N, a.D, a.k, a.sms);
+  const bool rc = a.fmt != 0;
+  if (a.k > kTcMaxK || (!rc && a.width != 1 && a.width != 2)) return cudaErrorInvalidValue;
+  const TensorPlan P = tensor_plan(a.B, a.N, a.D, a.k, a.sms, rc);
   if (P.n_lists != a.n_lists) return cudaErrorInvalidValue;
   uint8_t *qA = static_cast<uint8_t *>(a.qprep);
   const unsigned q_blocks = (unsigned)((a.Bpad + 7) / 8);
@@ -1189,7 +1361,13 @@ cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st) {
   g.bar_off = (int)L.bar_off;
   g.b16 = f16;
   g.rowf = rowf;
-  auto kern = a.k <= 16 ? score_tc2_kernel<16> : a.k <= 32 ? score_tc2_kernel<32> : score_tc2_kernel<0>;
+  g.rowf4 = reinterpret_cast<const float4 *>(rowf);
+  auto kern = rc ? (a.k <= 16   ? score_tc2_kernel<16, true>
+                    : a.k <= 32 ? score_tc2_kernel<32, true>
+                                : score_tc2_kernel<0, true>)
+                 : (a.k <= 16   ? score_tc2_kernel<16, false>
+                    : a.k <= 32 ? score_tc2_kernel<32, false>
+                                : score_tc2_kernel<0, false>);
   e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)L.smem_bytes);
   if (e != cudaSuccess) return e;
   const dim3 grid((unsigned)P.nsplit, (unsigned)(a.Bpad / kBM));
@@ -1199,7 +1377,24 @@ cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st) {
     const int64_t nrows_pad = (nrows + kBN - 1) / kBN * kBN;
     const unsigned cg = (unsigned)((nrows_pad + 7) / 8);
     timing_launch_begin(LAM_TIME_AUX, st);
-    if (j == 0) {  // the first slab's conversion shares a launch with the query prep
+    float4 *rowf4 = reinterpret_cast<float4 *>(rowf);
+    if (rc) {
+      auto conv = [&](auto first, auto rest) {
+        if (j == 0)
+          first<<<q_blocks + cg, 256, 0, st>>>(a.queries, a.B, a.D, a.Bpad, qA, q_blocks, a.codes,
+                                               a.row_scale, a.row_offset, nrows, nrows_pad, f16,
+                                               rowf4, a.metric);
+        else
+          rest<<<cg, 256, 0, st>>>(a.codes, a.row_scale, a.row_offset, row_base, nrows,
+                                   nrows_pad, a.D, f16, rowf4, a.metric);
+      };
+      if (a.fmt == LAM_ROWS_INT8)
+        conv(prep_convert_rows_kernel<LAM_ROWS_INT8>, convert_rows_kernel<LAM_ROWS_INT8>);
+      else if (a.fmt == LAM_ROWS_FP16)
+        conv(prep_convert_rows_kernel<LAM_ROWS_FP16>, convert_rows_kernel<LAM_ROWS_FP16>);
+      else
+        conv(prep_convert_rows_kernel<LAM_ROWS_SIGN>, convert_rows_kernel<LAM_ROWS_SIGN>);
+    } else if (j == 0) {  // the first slab's conversion shares a launch with the query prep
       if (a.width == 1)
         prep_convert_kernel<1><<<q_blocks + cg, 256, 0, st>>>(
             a.queries, a.B, a.D, a.Bpad, qA, q_blocks, a.codes, nrows, nrows_pad, f16, rowf,

@@ -28,6 +28,14 @@ def check_topk(g_scores, g_ids, queries, codes_i32, eps, metric, o_scores, o_ids
 
     codes_i32: the [N, D] codes (int32) the ids index (ids - row_offset).
     """
+    def score_at(b, ids):
+        return oracle.scores(queries[b:b + 1], codes_i32[ids - row_offset], eps, metric)[0]
+    check_topk_fn(g_scores, g_ids, score_at, codes_i32.shape[0], metric, o_scores, o_ids,
+                  row_offset)
+
+
+def check_topk_fn(g_scores, g_ids, score_at, n_rows, metric, o_scores, o_ids, row_offset=0):
+    """check_topk with the oracle's score of (query b, ids) given by score_at."""
     g_scores = np.asarray(g_scores, dtype=np.float32)
     g_ids = np.asarray(g_ids, dtype=np.int64)
     B, k = g_scores.shape
@@ -36,8 +44,8 @@ def check_topk(g_scores, g_ids, queries, codes_i32, eps, metric, o_scores, o_ids
         ids = g_ids[b]
         sc = g_scores[b]
         assert len(set(ids.tolist())) == k, "duplicate ids in query %d" % b
-        assert ids.min() >= row_offset and ids.max() < row_offset + codes_i32.shape[0]
-        o_at = oracle.scores(queries[b:b + 1], codes_i32[ids - row_offset], eps, metric)[0]
+        assert ids.min() >= row_offset and ids.max() < row_offset + n_rows
+        o_at = score_at(b, ids)
         err = np.abs(sc.astype(np.float64) - o_at.astype(np.float64))
         bad = np.nonzero(err > tol(o_at))[0]
         assert bad.size == 0, "query %d: score of id %d is %r, oracle %r" % (

@@ -179,3 +179,45 @@ def test_lamz_sizes(lib):
     assert lam.lam_lamz_bound(0) == 16
     assert lam.lam_lamz_bound(33) == 16 + 4 + 2 * (4 + 4 * 31)
     assert lam.lam_lamz_workspace_size(1 << 20) > 0
+
+
+# fmt, N, D, codes, scale, offset: each case is invalid before any device work
+ROWS_BAD = [(0, 4, 16, 256, 512, 768), (4, 4, 16, 256, 512, 768), (3, 4, 12, 256, 512, 768),
+            (1, -1, 16, 256, 512, 768), (1, 4, 0, 256, 512, 768), (1, 4, 16, None, 512, 768),
+            (1, 4, 16, 256, None, 768), (1, 4, 16, 256, 512, None), (3, 4, 16, 256, None, None),
+            (2, 4, 16, 257, None, None), (1, 4, 16, 256, 514, 768)]
+
+
+@pytest.mark.parametrize("fmt,N,D,codes,scale,offset", ROWS_BAD)
+def test_row_codecs_reject_bad_arguments(lib, fmt, N, D, codes, scale, offset):
+    c = ctypes
+    p = lambda v: None if v is None else c.c_void_p(v)
+    assert lib.lam_encode_rows(c.c_void_p(1024), N, D, fmt, p(codes), p(scale), p(offset),
+                               None) == 1
+    assert lib.lam_decode_rows(p(codes), fmt, N, D, p(scale), p(offset), c.c_void_p(1024),
+                               None) == 1
+
+
+def test_row_codecs_empty_needs_no_device(lib):
+    c = ctypes
+    assert lib.lam_encode_rows(None, 0, 16, 1, None, None, None, None) == 0
+    assert lib.lam_decode_rows(None, 2, 0, 16, None, None, None, None) == 0
+
+
+def test_score_rows_rejects_bad_arguments(lib):
+    c = ctypes
+    v = c.c_void_p
+    ok = dict(q=v(1024), B=4, codes=v(4096), fmt=1, scale=v(512), offset=v(768), N=100, D=32,
+              k=10, metric=0, scores=v(8192), ids=v(16384), ws=v(1 << 20), wsb=1 << 30)
+
+    def call(**kw):
+        a = dict(ok, **kw)
+        return lib.lam_score_topk_rows(a["q"], a["B"], a["codes"], a["fmt"], a["scale"],
+                                       a["offset"], a["N"], a["D"], a["k"], a["metric"],
+                                       a["scores"], a["ids"], a["ws"], a["wsb"], None)
+    for bad in (dict(fmt=5), dict(fmt=3, D=20), dict(k=0), dict(k=101), dict(metric=3),
+                dict(scale=None), dict(offset=None), dict(q=None), dict(ws=v(1 << 20 | 8)),
+                dict(scale=v(514)), dict(B=0), dict(ids=v(16388))):
+        assert call(**bad) == 1, bad
+    assert lib.lam_score_topk_rows_workspace_size(4, 100, 32, 10, 9) == 0
+    assert lib.lam_score_topk_rows_path(4, 100, 20, 10, 3) == -1
