@@ -52,8 +52,8 @@ class L2Flush:
 # capture (the profiles/ summary of that kernel).  Reported only while the
 # kernel's source file is the one the counters were taken on.
 KERNEL_TRAFFIC = {
-    "score_tc2_kernel": {"source": "score_tc.cu", "source_sha256_16": "97194a3bf5ec2385",
-                         "bytes": 46579200,
+    "score_tc2_kernel": {"source": "score_tc.cu", "source_sha256_16": "3c8535db739de982",
+                         "bytes": 46622720,
                          "launch": "ncu, cold caches: int16 codes at eps=1e-4 (the fp16 operand "
                                    "image is the same for every width), 27,986 x 768, "
                                    "1,024 queries"},
@@ -730,6 +730,46 @@ def run_kernels(args):
                                  "frac_of_hbm_kernel": code_bytes / (k_s / 1e3) / 1e9 / hbm,
                                  "tflops_kernel": fl / (k_s / 1e3) / 1e12,
                                  "frac_of_tensor_kernel": fl / (k_s / 1e3) / 1e12 / tc_peak})
+    if wl.batches and wl.d > 1:
+        # the per-vector byte codecs of the composite experiment: encode, and
+        # exact search over the coded rows (decoding folded into the score)
+        res["rows"] = []
+        N, D = wl.n, wl.d
+        xr = x.view(N, D)
+        batches = [args.batch] if args.batch else list(wl.batches)
+        names = {lam.LAM_ROWS_INT8: "int8/vector", lam.LAM_ROWS_FP16: "fp16",
+                 lam.LAM_ROWS_SIGN: "sign"}
+        row_bytes = {lam.LAM_ROWS_INT8: D + 8, lam.LAM_ROWS_FP16: 2 * D,
+                     lam.LAM_ROWS_SIGN: D // 8 + 4}
+        for fmt in (lam.LAM_ROWS_INT8, lam.LAM_ROWS_FP16, lam.LAM_ROWS_SIGN):
+            rc, rs, ro = lam.encode_rows(xr, fmt)
+            ms_e, k_e = timed(lambda: lam.lam_encode_rows(xr, fmt, rc, rs, ro),
+                              lam.LAM_TIME_QUANTIZE)
+            eb = N * (4 * D + row_bytes[fmt])
+            for B in batches:
+                q = torch.from_numpy(inputs.queries(B, D, seed=1)).to(dev)
+                nb = lam.lam_score_topk_rows_workspace_size(B, N, D, wl.k, fmt)
+                sws = torch.empty(nb, dtype=torch.uint8, device=dev)
+                s_ = torch.empty((B, wl.k), dtype=torch.float32, device=dev)
+                i_ = torch.empty((B, wl.k), dtype=torch.int64, device=dev)
+                path = lam.lam_score_topk_rows_path(B, N, D, wl.k, fmt)
+                call = lambda: lam.lam_score_topk_rows(q, rc, fmt, rs, ro, N, D, wl.k, wl.metric,
+                                                       s_, i_, sws)
+                ms, k_s = timed(call, lam.LAM_TIME_SCORE)
+                _, k_m = timed(call, lam.LAM_TIME_MERGE)
+                _, k_a = timed(call, lam.LAM_TIME_AUX)
+                fl = 2.0 * N * D * B
+                res["rows"].append({"codec": names[fmt], "ratio_vs_fp32": 4.0 * D / row_bytes[fmt],
+                                    "encode_ms_kernel": k_e,
+                                    "encode_gbs_kernel": eb / (k_e / 1e3) / 1e9,
+                                    "B": B, "path": ["bandwidth", "tensor", "generic"][path],
+                                    "ms_span": ms, "ms_kernel": k_s, "ms_merge": k_m,
+                                    "ms_prep": k_a,
+                                    "vectors_per_s_span": N / (ms / 1e3),
+                                    "tflops_kernel": fl / (k_s / 1e3) / 1e12,
+                                    "frac_of_tensor_kernel": fl / (k_s / 1e3) / 1e12 / tc_peak})
+                del sws
+            del rc, rs, ro
     res["peaks"] = {"hbm_gbs": hbm, "bf16_tflops": tc_peak, "kind": kind}
     print(json.dumps(res))
 

@@ -731,12 +731,13 @@ lam_status lam_score_topk_rows(const float *queries, int64_t B, const void *code
   a.Bpad = p.Bpad;
   a.sms = sms;
   a.fmt = fmt;
-  a.row_scale = scale;
-  a.row_offset = offset;
+  RowPtrs rp;
+  rp.scale = scale;
+  rp.offset = offset;
   const cudaError_t e =
-      p.path == kPathTensor ? launch_score_tensor(a, st) : launch_score_generic(a, st);
+      p.path == kPathTensor ? launch_score_tensor(a, st, rp) : launch_score_generic(a, st, rp);
   if (e != cudaSuccess) return LAM_ERR_CUDA;
-  if (launch_topk_merge(a, st) != cudaSuccess) return LAM_ERR_CUDA;
+  if (launch_topk_merge(a, st, rp) != cudaSuccess) return LAM_ERR_CUDA;
   return LAM_OK;
 }
 

@@ -198,24 +198,30 @@ struct ScoreArgs {
   void *qprep;          // tensor path: fp16 [2*Bpad][D] then float4 [Bpad]
   int64_t Bpad;
   int sms;
-  // Per-row codecs (lam_score_topk_rows): LAM_ROWS_* (0: Q_eps codes, the
-  // fields above), per-row scale and offset.
+  // Per-row codecs (lam_score_topk_rows): LAM_ROWS_*, 0 for Q_eps codes.
+  // (It sits in the struct's tail padding: a larger kernel parameter block
+  // costs the tensor-core kernel registers and time.)
   int fmt = 0;
-  const float *row_scale = nullptr;
-  const float *row_offset = nullptr;
+};
+
+// Per-row factors of a per-row codec, passed beside ScoreArgs.
+struct RowPtrs {
+  const float *scale = nullptr;
+  const float *offset = nullptr;
 };
 
 // Decoded value xhat_d of row `row` of a per-row codec, evaluated exactly as
 // lam_decode_rows writes it.
-__device__ __forceinline__ float row_value(const ScoreArgs &a, int64_t row, int d) {
+__device__ __forceinline__ float row_value(const ScoreArgs &a, const RowPtrs &rp, int64_t row,
+                                           int d) {
   if (a.fmt == LAM_ROWS_INT8)
-    return __fadd_rn(a.row_offset[row],
-                     __fmul_rn(a.row_scale[row],
+    return __fadd_rn(rp.offset[row],
+                     __fmul_rn(rp.scale[row],
                                (float)static_cast<const int8_t *>(a.codes)[row * a.D + d]));
   if (a.fmt == LAM_ROWS_FP16)
     return __half2float(static_cast<const __half *>(a.codes)[row * a.D + d]);
   const uint8_t byte = static_cast<const uint8_t *>(a.codes)[row * (a.D / 8) + d / 8];
-  return ((byte >> (d & 7)) & 1u) ? a.row_scale[row] : -a.row_scale[row];
+  return ((byte >> (d & 7)) & 1u) ? rp.scale[row] : -rp.scale[row];
 }
 
 cudaError_t launch_encode_rows(const float *x, int64_t N, int D, int fmt, void *codes,
@@ -224,9 +230,11 @@ cudaError_t launch_decode_rows(const void *codes, int fmt, int64_t N, int D, con
                                const float *offset, float *out, int sms, cudaStream_t st);
 
 cudaError_t launch_score_bandwidth(const ScoreArgs &a, cudaStream_t st);
-cudaError_t launch_score_generic(const ScoreArgs &a, cudaStream_t st);
-cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st);
-cudaError_t launch_topk_merge(const ScoreArgs &a, cudaStream_t st);
+cudaError_t launch_score_generic(const ScoreArgs &a, cudaStream_t st,
+                                 const RowPtrs &rp = RowPtrs());
+cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st,
+                                const RowPtrs &rp = RowPtrs());
+cudaError_t launch_topk_merge(const ScoreArgs &a, cudaStream_t st, const RowPtrs &rp = RowPtrs());
 
 // Planning shared by the workspace-size query and the launch.
 enum Path { kPathBandwidth = 0, kPathTensor = 1, kPathGeneric = 2 };

@@ -268,7 +268,7 @@ __device__ __forceinline__ int32_t load_code(const void *codes, int width, int64
   return reinterpret_cast<const int32_t *>(codes)[i];
 }
 
-__global__ void __launch_bounds__(kGenWarps * 32) score_generic_kernel(ScoreArgs a) {
+__global__ void __launch_bounds__(kGenWarps * 32) score_generic_kernel(ScoreArgs a, RowPtrs rp) {
   extern __shared__ __align__(16) uint8_t gsmem[];
   uint64_t *lists = reinterpret_cast<uint64_t *>(gsmem);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -293,7 +293,7 @@ __global__ void __launch_bounds__(kGenWarps * 32) score_generic_kernel(ScoreArgs
     float acc = 0.0f, cc = 0.0f;
     const int64_t base = row * D;
     for (int d = lane; d < D; d += 32) {
-      const float c = a.fmt ? row_value(a, row, d) : (float)load_code(a.codes, a.width, base + d);
+      const float c = a.fmt ? row_value(a, rp, row, d) : (float)load_code(a.codes, a.width, base + d);
       acc = fmaf(q[d], c, acc);
       cc = fmaf(c, c, cc);
     }
@@ -341,7 +341,8 @@ __device__ void bitonic_sort(uint64_t *buf, int P) {
   }
 }
 
-__global__ void __launch_bounds__(kMergeThreads) topk_merge_kernel(ScoreArgs a, int P) {
+__global__ void __launch_bounds__(kMergeThreads) topk_merge_kernel(ScoreArgs a, int P,
+                                                                   RowPtrs rp) {
   extern __shared__ __align__(16) uint8_t msmem[];
   uint64_t *buf = reinterpret_cast<uint64_t *>(msmem);
   const int64_t b = blockIdx.x;
@@ -381,7 +382,7 @@ __global__ void __launch_bounds__(kMergeThreads) topk_merge_kernel(ScoreArgs a, 
       float acc = 0.0f;
       if (row < a.N) {
         for (int d = lane; d < a.D; d += 32) {
-          const float xh = a.fmt ? row_value(a, row, d)
+          const float xh = a.fmt ? row_value(a, rp, row, d)
                                  : __fmul_rn(a.s, (float)load_code(a.codes, a.width,
                                                                    (int64_t)row * a.D + d));
           const float df = __fsub_rn(q[d], xh);
@@ -415,7 +416,8 @@ __global__ void __launch_bounds__(kMergeThreads) topk_merge_kernel(ScoreArgs a, 
 constexpr int kKmWarps = 8;
 
 template <int HPL>
-__global__ void __launch_bounds__(kKmWarps * 32) topk_kmerge_kernel(ScoreArgs a, int qpc) {
+__global__ void __launch_bounds__(kKmWarps * 32) topk_kmerge_kernel(ScoreArgs a, int qpc,
+                                                                    RowPtrs rp) {
   extern __shared__ __align__(16) uint8_t ksmem[];
   const int L = a.n_lists, k = a.k;
   uint64_t *cand = reinterpret_cast<uint64_t *>(ksmem);            // [qpc][L][k]
@@ -479,7 +481,7 @@ __global__ void __launch_bounds__(kKmWarps * 32) topk_kmerge_kernel(ScoreArgs a,
         float acc = 0.0f;
         if (row < a.N) {
           for (int d = lane; d < a.D; d += 32) {
-            const float xh = a.fmt ? row_value(a, row, d)
+            const float xh = a.fmt ? row_value(a, rp, row, d)
                                  : __fmul_rn(a.s, (float)load_code(a.codes, a.width,
                                                                    (int64_t)row * a.D + d));
             const float df = __fsub_rn(q[d], xh);
@@ -574,20 +576,20 @@ cudaError_t launch_score_bandwidth(const ScoreArgs &a, cudaStream_t st) {
   return a.B == 1 ? launch_bw_k<2, 1>(a, sh, st) : launch_bw_k<2, 2>(a, sh, st);
 }
 
-cudaError_t launch_score_generic(const ScoreArgs &a, cudaStream_t st) {
+cudaError_t launch_score_generic(const ScoreArgs &a, cudaStream_t st, const RowPtrs &rp) {
   const size_t smem = (size_t)kGenWarps * a.k * sizeof(uint64_t);
   cudaError_t e = cudaFuncSetAttribute(score_generic_kernel,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   dim3 grid(a.n_lists, (unsigned)(a.B < 65535 ? a.B : 65535));
   timing_launch_begin(LAM_TIME_SCORE, st);
-  score_generic_kernel<<<grid, kGenWarps * 32, smem, st>>>(a);
+  score_generic_kernel<<<grid, kGenWarps * 32, smem, st>>>(a, rp);
   timing_launch_end(LAM_TIME_SCORE, st);
   return cudaGetLastError();
 }
 
 template <int HPL>
-static cudaError_t launch_kmerge_t(const ScoreArgs &a, cudaStream_t st) {
+static cudaError_t launch_kmerge_t(const ScoreArgs &a, cudaStream_t st, const RowPtrs &rp) {
   const size_t per_q = (size_t)a.n_lists * a.k * 8;
   int64_t qpc = (int64_t)(kKmCandBytes / per_q);
   if (qpc > kKmWarps) qpc = kKmWarps;  // one query per warp: spread over the SMs
@@ -597,19 +599,19 @@ static cudaError_t launch_kmerge_t(const ScoreArgs &a, cudaStream_t st) {
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   timing_launch_begin(LAM_TIME_MERGE, st);
-  kern<<<(unsigned)((a.B + qpc - 1) / qpc), kKmWarps * 32, smem, st>>>(a, (int)qpc);
+  kern<<<(unsigned)((a.B + qpc - 1) / qpc), kKmWarps * 32, smem, st>>>(a, (int)qpc, rp);
   timing_launch_end(LAM_TIME_MERGE, st);
   return cudaGetLastError();
 }
 
-cudaError_t launch_topk_merge(const ScoreArgs &a, cudaStream_t st) {
+cudaError_t launch_topk_merge(const ScoreArgs &a, cudaStream_t st, const RowPtrs &rp) {
   // warp k-way merge when one query's candidates fit the shared-memory budget
   if ((size_t)a.n_lists * a.k * 8 <= kKmCandBytes && a.n_lists <= 512) {
-    if (a.n_lists <= 32) return launch_kmerge_t<1>(a, st);
-    if (a.n_lists <= 64) return launch_kmerge_t<2>(a, st);
-    if (a.n_lists <= 128) return launch_kmerge_t<4>(a, st);
-    if (a.n_lists <= 256) return launch_kmerge_t<8>(a, st);
-    return launch_kmerge_t<16>(a, st);
+    if (a.n_lists <= 32) return launch_kmerge_t<1>(a, st, rp);
+    if (a.n_lists <= 64) return launch_kmerge_t<2>(a, st, rp);
+    if (a.n_lists <= 128) return launch_kmerge_t<4>(a, st, rp);
+    if (a.n_lists <= 256) return launch_kmerge_t<8>(a, st, rp);
+    return launch_kmerge_t<16>(a, st, rp);
   }
   const int64_t total = (int64_t)a.n_lists * a.k;
   int P = total <= kMergeCap ? next_pow2(total) : kMergeCap;
@@ -620,7 +622,7 @@ cudaError_t launch_topk_merge(const ScoreArgs &a, cudaStream_t st) {
   if (e != cudaSuccess) return e;
   const int threads = P / 2 < 32 ? 32 : (P / 2 > kMergeThreads ? kMergeThreads : P / 2);
   timing_launch_begin(LAM_TIME_MERGE, st);
-  topk_merge_kernel<<<(unsigned)a.B, threads, smem, st>>>(a, P);
+  topk_merge_kernel<<<(unsigned)a.B, threads, smem, st>>>(a, P, rp);
   timing_launch_end(LAM_TIME_MERGE, st);
   return cudaGetLastError();
 }

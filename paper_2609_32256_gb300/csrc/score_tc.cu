@@ -907,21 +907,14 @@ struct Tc2Geom {
   const float4 *rowf4;      // per-row (u, w, z) of the slab (per-row codecs)
 };
 
-// Per-row score factors of one 32-row chunk, one row per lane, and their
-// broadcast for row j (all lanes must call at()).
+// Per-row score factors of the per-row codecs for one 32-row chunk, one row
+// per lane, and their broadcast for row j (all lanes must call at()).
 template <bool RC>
 struct RowFac;
 template <>
-struct RowFac<false> {
-  float r;
-  __device__ __forceinline__ void load(const Tc2Geom &g, int64_t i, bool ok, bool need) {
-    r = need && ok ? g.rowf[i] : 0.0f;
-  }
-  __device__ __forceinline__ RowFac at(int j, bool) const {
-    RowFac f;
-    f.r = __shfl_sync(0xffffffffu, r, j);
-    return f;
-  }
+struct RowFac<false> {  // (the Q_eps path keeps its single factor in `rfl`)
+  __device__ __forceinline__ void load(const Tc2Geom &, int64_t, bool, bool) {}
+  __device__ __forceinline__ RowFac at(int, bool) const { return *this; }
 };
 template <>
 struct RowFac<true> {
@@ -945,8 +938,8 @@ struct QFac {
   float fq, fs, qq;
   int metric;
 };
-__device__ __forceinline__ float fac_score(const RowFac<false> &f, float acc, const QFac &q) {
-  return tile_score(q.metric, acc, q.fq, q.qq, f.r);
+__device__ __forceinline__ float fac_score(const RowFac<false> &, float, const QFac &) {
+  return 0.0f;
 }
 __device__ __forceinline__ float fac_score(const RowFac<true> &f, float acc, const QFac &q) {
   const float dot = fmaf(q.fq * f.u, acc, q.fs * f.w);
@@ -1073,18 +1066,16 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
       qq = qi.z;
       qs = qi.w;
     }
-    QFac qf;
-    qf.metric = a.metric;
-    qf.qq = qq;
-    qf.fs = 0.0f;
-    if (RC) {
+    const float fq = a.metric == LAM_METRIC_IP ? s * pw
+                     : a.metric == LAM_METRIC_COSINE ? (qn > 0.0f ? pw / qn : 0.0f)
+                                                     : -2.0f * s * pw;
+    QFac qf;  // per-row codecs
+    {
       const float inv = a.metric == LAM_METRIC_COSINE ? (qn > 0.0f ? 1.0f / qn : 0.0f) : 1.0f;
       qf.fq = pw * inv;
       qf.fs = qs * inv;
-    } else {
-      qf.fq = a.metric == LAM_METRIC_IP ? s * pw
-              : a.metric == LAM_METRIC_COSINE ? (qn > 0.0f ? pw / qn : 0.0f)
-                                              : -2.0f * s * pw;
+      qf.qq = qq;
+      qf.metric = a.metric;
     }
     const bool l2 = a.metric == LAM_METRIC_L2;
     constexpr int RK = KR > 0 ? KR : 1;
@@ -1113,6 +1104,7 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
           uint32_t v[32];
           RowFac<RC> rl;
           rl.load(g, row0 + c * 32 + lane, true, need_cc);
+          const float rfl = RC ? 0.0f : need_cc ? g.rowf[row0 + c * 32 + lane] : 0.0f;
           tmem_ld32(taddr + c * 32, v);
           // shift register: the P bests of this chunk enter at the top
 #pragma unroll
@@ -1122,7 +1114,10 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
             float best = -INFINITY;
 #pragma unroll
             for (int j = h * GR; j < (h + 1) * GR; ++j) {
-              const float sc = fac_score(rl.at(j, l2), __uint_as_float(v[j]), qf);
+              const float sc =
+                  RC ? fac_score(rl.at(j, l2), __uint_as_float(v[j]), qf)
+                     : tile_score(a.metric, __uint_as_float(v[j]), fq, qq,
+                                  __shfl_sync(0xffffffffu, rfl, j));
               best = fmaxf(best, desc ? sc : -sc);
             }
             gb[NG - P + h] = best;
@@ -1138,12 +1133,20 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
         // lane j holds the factors of row j of this chunk
         RowFac<RC> rl;
         rl.load(g, row0 + c * 32 + lane, lane < nvalid, need_cc);
+        const float rfl =
+            RC ? 0.0f : need_cc && lane < nvalid ? g.rowf[row0 + c * 32 + lane] : 0.0f;
         tmem_ld32(taddr + c * 32, v);
         const float thr = desc ? fmaxf(thr_s, seed) : fminf(thr_s, seed);
         uint32_t mask = 0;
 #pragma unroll
         for (int j = 0; j < 32; ++j) {
-          const float sc = fac_score(rl.at(j, l2), __uint_as_float(v[j]), qf);
+          float sc;
+          if constexpr (RC) {
+            sc = fac_score(rl.at(j, l2), __uint_as_float(v[j]), qf);
+          } else {
+            const float rf = __shfl_sync(0xffffffffu, rfl, j);
+            sc = tile_score(a.metric, __uint_as_float(v[j]), fq, qq, rf);
+          }
           mask |= (uint32_t)(desc ? sc > thr : sc < thr) << j;
         }
         if (!qvalid || nvalid <= 0) mask = 0;
@@ -1154,11 +1157,14 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
           // (re-tested against the threshold the earlier steps tightened)
           while (__any_sync(0xffffffffu, mask != 0)) {
             const int j = mask != 0 ? __ffs(mask) - 1 : 0;
-            const RowFac<RC> rf = rl.at(j, l2);
+            const RowFac<RC> rfc = RC ? rl.at(j, l2) : rl;
+            const float rf = RC ? 0.0f : __shfl_sync(0xffffffffu, rfl, j);
             uint32_t kc = 0xffffffffu, ic = 0xffffffffu;
             if (mask != 0) {
               mask &= mask - 1;
-              const float sc = fac_score(rf, __uint_as_float(select32(v, j)), qf);
+              const float sc = RC ? fac_score(rfc, __uint_as_float(select32(v, j)), qf)
+                                  : tile_score(a.metric, __uint_as_float(select32(v, j)), fq,
+                                               qq, rf);
               if (desc ? sc > thr_s : sc < thr_s) {
                 kc = rank_key32(sc, desc);
                 ic = grow0 + j;
@@ -1171,10 +1177,13 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
         } else {
           while (__any_sync(0xffffffffu, mask != 0)) {
             const int j = mask != 0 ? __ffs(mask) - 1 : 0;
-            const RowFac<RC> rf = rl.at(j, l2);
+            const RowFac<RC> rfc = RC ? rl.at(j, l2) : rl;
+            const float rf = RC ? 0.0f : __shfl_sync(0xffffffffu, rfl, j);
             if (mask == 0) continue;
             mask &= mask - 1;
-            const float sc = fac_score(rf, __uint_as_float(select32(v, j)), qf);
+            const float sc = RC ? fac_score(rfc, __uint_as_float(select32(v, j)), qf)
+                                : tile_score(a.metric, __uint_as_float(select32(v, j)), fq, qq,
+                                             rf);
             const uint64_t key = make_key(sc, grow0 + j, desc);
             if (key < lists[m]) {
               heap_replace_root(lists, k, kBM, m, key);
@@ -1298,7 +1307,7 @@ TensorPlan tensor_plan(int64_t B, int64_t N, int D, int k, int sms, bool force_p
   return p;
 }
 
-cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st) {
+cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st, const RowPtrs &rp) {
   const bool rc = a.fmt != 0;
   if (a.k > kTcMaxK || (!rc && a.width != 1 && a.width != 2)) return cudaErrorInvalidValue;
   const TensorPlan P = tensor_plan(a.B, a.N, a.D, a.k, a.sms, rc);
@@ -1382,10 +1391,10 @@ cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st) {
       auto conv = [&](auto first, auto rest) {
         if (j == 0)
           first<<<q_blocks + cg, 256, 0, st>>>(a.queries, a.B, a.D, a.Bpad, qA, q_blocks, a.codes,
-                                               a.row_scale, a.row_offset, nrows, nrows_pad, f16,
+                                               rp.scale, rp.offset, nrows, nrows_pad, f16,
                                                rowf4, a.metric);
         else
-          rest<<<cg, 256, 0, st>>>(a.codes, a.row_scale, a.row_offset, row_base, nrows,
+          rest<<<cg, 256, 0, st>>>(a.codes, rp.scale, rp.offset, row_base, nrows,
                                    nrows_pad, a.D, f16, rowf4, a.metric);
       };
       if (a.fmt == LAM_ROWS_INT8)
