@@ -15,8 +15,7 @@
  * Conventions shared by every call:
  *   - Every array argument is a DEVICE pointer on the current CUDA device,
  *     allocated and owned by the caller.  The library allocates no memory.
- *     Only the scalar outputs of lam_quantize and lam_score_topk_status are
- *     host pointers.
+ *     Only the scalar outputs of the synchronous calls are host pointers.
  *   - Arrays are dense and row-major.  Codes are two's-complement integers of
  *     1, 2 or 4 bytes ("width").
  *   - `stream` is a cudaStream_t (NULL = the legacy default stream).  Work is

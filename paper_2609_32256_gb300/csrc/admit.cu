@@ -362,9 +362,7 @@ cudaError_t launch_admit_batch(const float *e, int64_t N, int D, const uint64_t 
   err = scan_u32(U(L.cnt), m, U(L.sums), stat32 + 0, st);
   if (err != cudaSuccess) return err;
   uint32_t np = 0;
-  err = cudaMemcpyAsync(&np, stat32, 4, cudaMemcpyDeviceToHost, st);
-  if (err != cudaSuccess) return err;
-  err = cudaStreamSynchronize(st);
+  err = read_back(&np, stat32, 4, st);
   if (err != cudaSuccess) return err;
   *n_pairs = np;
   if ((int64_t)np > max_pairs) {
@@ -400,9 +398,7 @@ cudaError_t launch_admit_batch(const float *e, int64_t N, int D, const uint64_t 
   resolve_kernel<<<1, 1024, 0, st>>>(N, U(L.rowc), U(L.elo), Dp(L.edist), w + L.state, rep, dist,
                                      stat64);
   double h[2];
-  err = cudaMemcpyAsync(h, stat64, 16, cudaMemcpyDeviceToHost, st);
-  if (err != cudaSuccess) return err;
-  err = cudaStreamSynchronize(st);
+  err = read_back(h, stat64, 16, st);
   if (err != cudaSuccess) return err;
   *delta_hat = h[0];
   *n_retained = (int64_t)h[1];

@@ -161,6 +161,13 @@ bool make_rows_plan(int64_t B, int64_t N, int32_t D, int32_t k, int32_t fmt, int
 }  // namespace
 
 namespace lam {
+
+cudaError_t read_back(void *dst, const void *src, size_t n, cudaStream_t st) {
+  cudaError_t e = cudaMemcpyAsync(dst, src, n, cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  return e;
+}
+
 namespace {
 
 // Event pairs around selected kernel launches (lam_timing_*).
@@ -311,9 +318,7 @@ lam_status lam_quantize(const float *x, int64_t n, float eps, int32_t width_req,
   timing_launch_end(tkind, st);
   if (e != cudaSuccess) return LAM_ERR_CUDA;
   QuantStatus h;
-  if (cudaMemcpyAsync(&h, dst, sizeof(h), cudaMemcpyDeviceToHost, st) != cudaSuccess)
-    return LAM_ERR_CUDA;
-  if (cudaStreamSynchronize(st) != cudaSuccess) return LAM_ERR_CUDA;
+  if (read_back(&h, dst, sizeof(h), st) != cudaSuccess) return LAM_ERR_CUDA;
   if (width_req == LAM_WIDTH_AUTO && codes != nullptr && h.passes == 2 &&
       !(h.flags & (kFlagTimeout | kFlagNonfinite | kFlagRange | kFlagWorkspace)) &&
       (h.width == 1 || h.width == 2 || h.width == 4)) {
@@ -323,9 +328,7 @@ lam_status lam_quantize(const float *x, int64_t n, float eps, int32_t width_req,
     timing_launch_end(LAM_TIME_QUANTIZE, st);
     if (e != cudaSuccess) return LAM_ERR_CUDA;
     const uint32_t width_resolved = h.width;
-    if (cudaMemcpyAsync(&h, dst, sizeof(h), cudaMemcpyDeviceToHost, st) != cudaSuccess)
-      return LAM_ERR_CUDA;
-    if (cudaStreamSynchronize(st) != cudaSuccess) return LAM_ERR_CUDA;
+    if (read_back(&h, dst, sizeof(h), st) != cudaSuccess) return LAM_ERR_CUDA;
     h.width = width_resolved;
   }
   return lam::decode_quant_status(h, width_req, s, width_out, scale_out, code_min_out,
@@ -374,9 +377,7 @@ lam_status lam_quantize_bands(const float *x, int64_t N, int32_t D, float eps, i
   timing_launch_end(LAM_TIME_QUANTIZE, st);
   if (e != cudaSuccess) return LAM_ERR_CUDA;
   QuantStatus h;
-  if (cudaMemcpyAsync(&h, dst, sizeof(h), cudaMemcpyDeviceToHost, st) != cudaSuccess)
-    return LAM_ERR_CUDA;
-  if (cudaStreamSynchronize(st) != cudaSuccess) return LAM_ERR_CUDA;
+  if (read_back(&h, dst, sizeof(h), st) != cudaSuccess) return LAM_ERR_CUDA;
   if (width_req == LAM_WIDTH_AUTO && h.passes == 2 &&
       !(h.flags & (kFlagTimeout | kFlagNonfinite | kFlagRange | kFlagWorkspace)) &&
       (h.width == 1 || h.width == 2 || h.width == 4)) {
@@ -387,9 +388,7 @@ lam_status lam_quantize_bands(const float *x, int64_t N, int32_t D, float eps, i
     timing_launch_end(LAM_TIME_QUANTIZE, st);
     if (e != cudaSuccess) return LAM_ERR_CUDA;
     const uint32_t width_resolved = h.width;
-    if (cudaMemcpyAsync(&h, dst, sizeof(h), cudaMemcpyDeviceToHost, st) != cudaSuccess)
-      return LAM_ERR_CUDA;
-    if (cudaStreamSynchronize(st) != cudaSuccess) return LAM_ERR_CUDA;
+    if (read_back(&h, dst, sizeof(h), st) != cudaSuccess) return LAM_ERR_CUDA;
     h.width = width_resolved;
   }
   return lam::decode_quant_status(h, width_req, s, width_out, scale_out, code_min_out,
@@ -745,9 +744,7 @@ lam_status lam_score_topk_status(const void *workspace, lam_stream_t stream, int
   if (workspace == nullptr || status_out == nullptr) return LAM_ERR_INVALID;
   uint32_t flags = 0;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  if (cudaMemcpyAsync(&flags, workspace, 4, cudaMemcpyDeviceToHost, st) != cudaSuccess)
-    return LAM_ERR_CUDA;
-  if (cudaStreamSynchronize(st) != cudaSuccess) return LAM_ERR_CUDA;
+  if (read_back(&flags, workspace, 4, st) != cudaSuccess) return LAM_ERR_CUDA;
   if (flags & kFlagTimeout) *status_out = LAM_ERR_TIMEOUT;
   else if (flags & kFlagRange) *status_out = LAM_ERR_RANGE;
   else *status_out = LAM_OK;

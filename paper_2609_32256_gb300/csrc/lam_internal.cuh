@@ -253,6 +253,10 @@ struct TensorPlan {
 // (force_pre: the per-row codecs always take the converting pass)
 TensorPlan tensor_plan(int64_t B, int64_t N, int D, int k, int sms, bool force_pre = false);
 
+// Synchronous read-back of a small device status block into host memory:
+// queued on `st`, then waits for `st`.
+cudaError_t read_back(void *dst, const void *src, size_t n, cudaStream_t st);
+
 // Launch bracketing for lam_timing_* (no-ops unless timing is on for `kind`).
 void timing_launch_begin(int kind, cudaStream_t st);
 void timing_launch_end(int kind, cudaStream_t st);

@@ -241,9 +241,7 @@ cudaError_t launch_lamz_compress(const float *x, int64_t n, float rel, uint8_t *
   e = scan_u32(sizes, nb, sums, &st->total, stream);
   if (e != cudaSuccess) return e;
   CodecStatus h;
-  e = cudaMemcpyAsync(&h, st, sizeof(h), cudaMemcpyDeviceToHost, stream);
-  if (e != cudaSuccess) return e;
-  e = cudaStreamSynchronize(stream);
+  e = read_back(&h, st, sizeof(h), stream);
   if (e != cudaSuccess) return e;
   *nonfinite = (h.flags & kFlagNonfinite) != 0;
   *bytes = head + h.total;
@@ -278,7 +276,7 @@ cudaError_t launch_lamz_decompress(const uint8_t *in, size_t in_bytes, float *ou
   *bad = true;
   if (in_bytes < head) return cudaSuccess;
   uint8_t fixed[16];
-  cudaError_t e = cudaMemcpyAsync(fixed, in, 16, cudaMemcpyDeviceToHost, stream);
+  cudaError_t e = read_back(fixed, in, 16, stream);
   if (e != cudaSuccess) return e;
   e = cudaMemsetAsync(st, 0, sizeof(CodecStatus), stream);
   if (e != cudaSuccess) return e;
@@ -286,9 +284,7 @@ cudaError_t launch_lamz_decompress(const uint8_t *in, size_t in_bytes, float *ou
   e = scan_u32(sizes, nb, sums, &st->total, stream);
   if (e != cudaSuccess) return e;
   CodecStatus h;
-  e = cudaMemcpyAsync(&h, st, sizeof(h), cudaMemcpyDeviceToHost, stream);
-  if (e != cudaSuccess) return e;
-  e = cudaStreamSynchronize(stream);
+  e = read_back(&h, st, sizeof(h), stream);
   if (e != cudaSuccess) return e;
   uint64_t nn = 0;
   for (int k = 0; k < 8; ++k) nn |= (uint64_t)fixed[4 + k] << (8 * k);

@@ -592,8 +592,12 @@ template <int HPL>
 static cudaError_t launch_kmerge_t(const ScoreArgs &a, cudaStream_t st, const RowPtrs &rp) {
   const size_t per_q = (size_t)a.n_lists * a.k * 8;
   int64_t qpc = (int64_t)(kKmCandBytes / per_q);
-  if (qpc > kKmWarps) qpc = kKmWarps;  // one query per warp: spread over the SMs
+  if (qpc > kKmWarps) qpc = kKmWarps;  // one query per warp
+  // at least ~2 CTAs per SM when the batch allows: the merge is latency-bound
+  const int64_t spread = (a.B + 2LL * a.sms - 1) / (2LL * a.sms);
+  if (qpc > spread) qpc = spread;
   if (qpc > a.B) qpc = a.B;
+  if (qpc < 1) qpc = 1;
   const size_t smem = (size_t)qpc * per_q + (size_t)kKmWarps * next_pow2(a.k) * 8;
   auto kern = topk_kmerge_kernel<HPL>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
