@@ -74,6 +74,10 @@ def parse():
     p.add_argument("--reps", type=int, default=20)
     p.add_argument("--eps", type=float, default=0.0, help="(--kernels) one eps instead of the sweep")
     p.add_argument("--width", type=int, default=-1, help="(--kernels) forced code width")
+    p.add_argument("--rows", type=int, default=0,
+                   help="(--kernels) a smaller memory of the same workload (profiling captures)")
+    p.add_argument("--only", default="",
+                   help="(--kernels) comma list of parts: quantize,bands,codec,admit,score,rows")
     return p.parse_args()
 
 
@@ -571,6 +575,12 @@ def run_kernels(args):
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
     wl = inputs.WORKLOADS[args.workload]
+    if args.rows:
+        import dataclasses
+        wl = dataclasses.replace(wl, n=args.rows,
+                                 slab_rows=min(wl.slab_rows, args.rows) if wl.slab_rows else 0)
+    parts = set(args.only.split(",")) if args.only else {"quantize", "bands", "codec", "admit",
+                                                         "score", "rows"}
     if wl.d == 1:
         x = torch.from_numpy(inputs.flat_values(wl.n, seed=0)).to(dev)
     elif wl.slab_rows:
@@ -612,6 +622,8 @@ def run_kernels(args):
         _, w, sc, cmin, cmax = lam.lam_quantize(x, e, 0, None, ws)
         wq = args.width if args.width > 0 else (wl.width or w)
         widths[e] = (wq, sc, max(-cmin, cmax))
+        if "quantize" not in parts:
+            continue
         ms_auto, k_auto = timed(lambda: lam.lam_quantize(x, e, 0, codes, ws),
                                 lam.LAM_TIME_QUANTIZE)
         ms_forced, k_forced = timed(lambda: lam.lam_quantize(x, e, wq, codes, ws),
@@ -630,7 +642,7 @@ def run_kernels(args):
         gbd = (wq + 4) * n / (k_d / 1e3) / 1e9
         res["dequantize"].append({"eps": e, "width": wq, "ms_span": ms_d, "ms_kernel": k_d,
                                   "gbs_kernel": gbd, "frac_of_hbm_kernel": gbd / hbm})
-    if wl.d > 1:
+    if wl.d > 1 and "bands" in parts:
         # Q_eps fused with the band digests (r = 4 and 8, the paper's shipped and
         # best band widths), codes written, AUTO width
         res["bands"] = []
@@ -648,7 +660,7 @@ def run_kernels(args):
                                      "gbs_kernel": nbytes / (k_ms / 1e3) / 1e9,
                                      "frac_of_hbm_kernel": nbytes / (k_ms / 1e3) / 1e9 / hbm})
             del dig
-    if wl.d == 1:
+    if wl.d == 1 and "codec" in parts:
         # the error-bounded byte codec at the paper's relative bounds (its
         # deployed bound is 1% of max|x|), on the first 2^24 values and all
         res["codec"] = []
@@ -669,7 +681,7 @@ def run_kernels(args):
                                      "decompress_ms_span": ms_d,
                                      "decompress_gbs": 4.0 * n_c / (ms_d / 1e3) / 1e9})
             del cbuf, cws, yc
-    if wl.planted:
+    if wl.planted and "admit" in parts:
         # batch admission (Algorithm 2) at cos >= 0.95 over band candidates at
         # the paper's shipped (r = 4, eps = 0.2 sigma) and relaxed (r = 8, 0.3 sigma)
         # operating points: digests from the fused pass, then lam_admit_batch
@@ -698,7 +710,7 @@ def run_kernels(args):
                                  "records_per_s": N / (ms / 1e3), "candidate_pairs": npairs,
                                  "retained": kept, "delta_hat": dh})
             del aws, dig
-    if wl.batches and wl.d > 1:
+    if wl.batches and wl.d > 1 and "score" in parts:
         e = eps_list[0]
         wq, sc, bound = widths[e]
         lam.lam_quantize(x, e, wq, codes, ws)
@@ -730,7 +742,7 @@ def run_kernels(args):
                                  "frac_of_hbm_kernel": code_bytes / (k_s / 1e3) / 1e9 / hbm,
                                  "tflops_kernel": fl / (k_s / 1e3) / 1e12,
                                  "frac_of_tensor_kernel": fl / (k_s / 1e3) / 1e12 / tc_peak})
-    if wl.batches and wl.d > 1:
+    if wl.batches and wl.d > 1 and "rows" in parts:
         # the per-vector byte codecs of the composite experiment: encode, and
         # exact search over the coded rows (decoding folded into the score)
         res["rows"] = []

@@ -86,7 +86,7 @@ bool bandwidth_ok(int64_t B, int32_t D, int32_t k, int32_t width) {
 bool tensor_ok(int64_t B, int64_t N, int32_t D, int32_t k, int32_t width, int32_t code_bound) {
   (void)N;
   const bool codes_exact = width == 1 || (width == 2 && code_bound > 0 && code_bound <= 2048);
-  return codes_exact && D % 16 == 0 && tensor_fits(width, k) && B <= (1LL << 23);
+  return codes_exact && D % 16 == 0 && tensor_fits(width, k, B) && B <= (1LL << 23);
 }
 
 // Chooses the path (or honours LAM_SCORE_PATH) and lays out the workspace:
@@ -600,11 +600,12 @@ lam_status lam_score_topk(const float *queries, int64_t B, const void *codes, in
   a.Bpad = p.Bpad;
   a.sms = sms;
   cudaError_t e;
+  ScoreArgs m = a;  // the final merge's lists
   if (p.path == kPathBandwidth) e = launch_score_bandwidth(a, st);
-  else if (p.path == kPathTensor) e = launch_score_tensor(a, st);
+  else if (p.path == kPathTensor) e = launch_score_tensor(a, st, RowPtrs(), &m);
   else e = launch_score_generic(a, st);
   if (e != cudaSuccess) return LAM_ERR_CUDA;
-  if (launch_topk_merge(a, st) != cudaSuccess) return LAM_ERR_CUDA;
+  if (launch_topk_merge(m, st) != cudaSuccess) return LAM_ERR_CUDA;
   return LAM_OK;
 }
 
@@ -733,10 +734,11 @@ lam_status lam_score_topk_rows(const float *queries, int64_t B, const void *code
   RowPtrs rp;
   rp.scale = scale;
   rp.offset = offset;
-  const cudaError_t e =
-      p.path == kPathTensor ? launch_score_tensor(a, st, rp) : launch_score_generic(a, st, rp);
+  ScoreArgs m = a;  // the final merge's lists
+  const cudaError_t e = p.path == kPathTensor ? launch_score_tensor(a, st, rp, &m)
+                                              : launch_score_generic(a, st, rp);
   if (e != cudaSuccess) return LAM_ERR_CUDA;
-  if (launch_topk_merge(a, st, rp) != cudaSuccess) return LAM_ERR_CUDA;
+  if (launch_topk_merge(m, st, rp) != cudaSuccess) return LAM_ERR_CUDA;
   return LAM_OK;
 }
 

@@ -232,15 +232,22 @@ cudaError_t launch_decode_rows(const void *codes, int fmt, int64_t N, int D, con
 cudaError_t launch_score_bandwidth(const ScoreArgs &a, cudaStream_t st);
 cudaError_t launch_score_generic(const ScoreArgs &a, cudaStream_t st,
                                  const RowPtrs &rp = RowPtrs());
+// `merge` (optional) receives the arguments of the final merge: a search of
+// several slabs leaves one merged list per slab in its workspace.
 cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st,
-                                const RowPtrs &rp = RowPtrs());
+                                const RowPtrs &rp = RowPtrs(), ScoreArgs *merge = nullptr);
 cudaError_t launch_topk_merge(const ScoreArgs &a, cudaStream_t st, const RowPtrs &rp = RowPtrs());
+// Multi-slab searches: the partial lists [list0, list0 + n_lists) of one slab
+// merged into slab `slab` of `out` ([nslabs][B][k] keys); with `seed`, also
+// per query the ranking-form score of the slab's k-th best key.
+cudaError_t launch_slab_merge(const ScoreArgs &a, int list0, int n_lists, int slab, uint64_t *out,
+                              float *seed, cudaStream_t st);
 
 // Planning shared by the workspace-size query and the launch.
 enum Path { kPathBandwidth = 0, kPathTensor = 1, kPathGeneric = 2 };
 int bandwidth_ctas(int64_t N, int D, int width, int sms);
 int tensor_splits(int64_t B, int64_t N, int sms);
-bool tensor_fits(int width, int k);  // shared memory holds >= 2 stages
+bool tensor_fits(int width, int k, int64_t B);  // shared memory holds >= 2 stages
 bool tensor_fits_pre(int k);         // the same for the converting-pass kernel alone
 // Tensor-path workspace (after the partial lists): [query images][query info]
 // and, for two or more query blocks, [fp16 code slab][per-row factors].
@@ -248,7 +255,9 @@ struct TensorPlan {
   bool pre;            // codes converted to fp16 by a separate pass
   int64_t slab_rows;   // rows per slab (pre), else N
   int nslabs, nsplit, n_lists;
-  size_t qinfo_off, fp16_off, rowf_off, bytes;  // rowf: 16 bytes per slab row
+  // rowf: 16 bytes per slab row; seed: 4 bytes per query; slab lists: the
+  // merged list of each slab, nslabs x B x k keys (several slabs only)
+  size_t qinfo_off, fp16_off, rowf_off, seed_off, slabl_off, bytes;
 };
 // (force_pre: the per-row codecs always take the converting pass)
 TensorPlan tensor_plan(int64_t B, int64_t N, int D, int k, int sms, bool force_pre = false);

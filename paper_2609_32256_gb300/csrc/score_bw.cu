@@ -411,8 +411,8 @@ __global__ void __launch_bounds__(kMergeThreads) topk_merge_kernel(ScoreArgs a, 
 // copies the candidate lists of its qpc queries to shared memory; lane l then
 // owns lists l, l + 32, ... and keeps their heads in registers; each of the k
 // steps takes the warp-wide smallest head and advances that list.  Squared L2
-// survivors are rescored in the direct form and re-sorted, as in the
-// block-sort merge above.
+// survivors are rescored in the direct form (all warps of the CTA share the
+// rows of its queries) and re-sorted, as in the block-sort merge above.
 constexpr int kKmWarps = 8;
 
 template <int HPL>
@@ -434,10 +434,12 @@ __global__ void __launch_bounds__(kKmWarps * 32) topk_kmerge_kernel(ScoreArgs a,
   __syncthreads();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const bool desc = a.metric != LAM_METRIC_L2;
+  // qpc <= kKmWarps: warp qi owns query b0 + qi
+  const int qi = warp;
+  const int64_t b = b0 + qi;
+  const bool mine = qi < qpc && b < a.B;
   uint64_t *O = outk + (size_t)warp * P2;
-  for (int qi = warp; qi < qpc; qi += kKmWarps) {
-    const int64_t b = b0 + qi;
-    if (b >= a.B) break;
+  if (mine) {
     const uint64_t *C = cand + (size_t)qi * per_q;
     int pos[HPL];
     uint64_t head[HPL];
@@ -473,26 +475,33 @@ __global__ void __launch_bounds__(kKmWarps * 32) topk_kmerge_kernel(ScoreArgs a,
       }
       if (lane == 0) O[i] = gm;
     }
-    __syncwarp();
-    if (!desc) {
-      const float *q = a.queries + b * a.D;
-      for (int i = 0; i < k; ++i) {
-        const uint32_t row = (uint32_t)(O[i] & 0xffffffffu);
-        float acc = 0.0f;
-        if (row < a.N) {
-          for (int d = lane; d < a.D; d += 32) {
-            const float xh = a.fmt ? row_value(a, rp, row, d)
+  }
+  if (!desc) {
+    // every warp rescores survivors of every query of the CTA
+    __syncthreads();
+    for (int t = warp; t < qpc * k; t += kKmWarps) {
+      const int tq = t / k, i = t - tq * k;
+      const int64_t tb = b0 + tq;
+      if (tb >= a.B) continue;
+      uint64_t *Ot = outk + (size_t)tq * P2;
+      const uint32_t row = (uint32_t)(Ot[i] & 0xffffffffu);
+      const float *q = a.queries + tb * a.D;
+      float acc = 0.0f;
+      if (row < a.N) {
+#pragma unroll 4
+        for (int d = lane; d < a.D; d += 32) {
+          const float xh = a.fmt ? row_value(a, rp, row, d)
                                  : __fmul_rn(a.s, (float)load_code(a.codes, a.width,
                                                                    (int64_t)row * a.D + d));
-            const float df = __fsub_rn(q[d], xh);
-            acc = fmaf(df, df, acc);
-          }
+          const float df = __fsub_rn(q[d], xh);
+          acc = fmaf(df, df, acc);
         }
-        acc = warp_sum(acc);
-        __syncwarp();
-        if (lane == 0) O[i] = row < a.N ? make_key(acc, row, false) : kSentinel;
-        __syncwarp();
       }
+      acc = warp_sum(acc);
+      if (lane == 0) Ot[i] = row < a.N ? make_key(acc, row, false) : kSentinel;
+    }
+    __syncthreads();
+    if (mine) {
       for (int i = k + lane; i < P2; i += 32) O[i] = kSentinel;
       __syncwarp();
       for (int size = 2; size <= P2; size <<= 1) {
@@ -511,6 +520,9 @@ __global__ void __launch_bounds__(kKmWarps * 32) topk_kmerge_kernel(ScoreArgs a,
         }
       }
     }
+  }
+  __syncwarp();
+  if (mine) {
     for (int i = lane; i < k; i += 32) {
       const uint64_t key = O[i];
       uint32_t o = (uint32_t)(key >> 32);
@@ -518,7 +530,95 @@ __global__ void __launch_bounds__(kKmWarps * 32) topk_kmerge_kernel(ScoreArgs a,
       a.scores[b * k + i] = unord_f32(o);
       a.ids[b * k + i] = (int64_t)(uint32_t)(key & 0xffffffffu);
     }
-    __syncwarp();
+  }
+}
+
+// Per-slab merge of a multi-slab search: per query the nsplit partial lists
+// of one slab (lists list0 .. list0 + n_lists - 1) become one sorted list of
+// k keys, slab `slab` of `out` ([nslabs][B][k], the partial-list layout), so
+// the final merge sees one list per slab.  With `seed` it also writes the
+// ranking-form score of the k-th key (+-inf when the slab holds fewer than k
+// rows): the first slab's k-th best bounds what the later slabs may offer.
+// One warp per query, lists staged in shared memory when they fit; the merge
+// stops at the first sentinel (later slabs offer few rows).
+constexpr int kSmWarps = 8;
+
+template <int HPL>
+__global__ void __launch_bounds__(kSmWarps * 32)
+    slab_merge_kernel(ScoreArgs a, int list0, int n_lists, int qpc, bool staged, int slab,
+                      uint64_t *__restrict__ out, float *__restrict__ seed) {
+  extern __shared__ __align__(16) uint8_t smsmem[];
+  uint64_t *cand = reinterpret_cast<uint64_t *>(smsmem);  // [qpc][n_lists][k]
+  const int k = a.k;
+  const int per_q = n_lists * k;
+  const int64_t b0 = (int64_t)blockIdx.x * qpc;
+  if (staged) {
+    for (int e = threadIdx.x; e < qpc * per_q; e += blockDim.x) {
+      const int qi = e / per_q, rem = e - qi * per_q;
+      const int l = rem / k, i = rem - l * k;
+      const int64_t b = b0 + qi;
+      cand[e] = b < a.B ? a.partial[((size_t)(list0 + l) * a.B + b) * k + i] : kSentinel;
+    }
+    __syncthreads();
+  }
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const bool desc = a.metric != LAM_METRIC_L2;
+  for (int qi = warp; qi < qpc; qi += kSmWarps) {
+    const int64_t b = b0 + qi;
+    if (b >= a.B) break;
+    // key i of list l of this query
+    auto at = [&](int l, int i) -> uint64_t {
+      return staged ? cand[(size_t)qi * per_q + (size_t)l * k + i]
+                    : a.partial[((size_t)(list0 + l) * a.B + b) * k + i];
+    };
+    int pos[HPL];
+    uint64_t head[HPL];
+#pragma unroll
+    for (int h = 0; h < HPL; ++h) {
+      const int l = lane + 32 * h;
+      pos[h] = 0;
+      head[h] = l < n_lists ? at(l, 0) : kSentinel;
+    }
+    uint64_t *o = out + ((size_t)slab * a.B + b) * k;
+    uint64_t gm = kSentinel;
+    int i = 0;
+    for (; i < k; ++i) {
+      uint64_t m = head[0];
+      int mh = 0;
+#pragma unroll
+      for (int h = 1; h < HPL; ++h)
+        if (head[h] < m) {
+          m = head[h];
+          mh = h;
+        }
+      gm = m;
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) {
+        const uint64_t v = __shfl_xor_sync(0xffffffffu, gm, off);
+        gm = v < gm ? v : gm;
+      }
+      if (gm == kSentinel) break;  // every list is exhausted
+      if (lane == 0) o[i] = gm;
+      const unsigned bal = __ballot_sync(0xffffffffu, m == gm);
+      if (lane == __ffs(bal) - 1) {
+#pragma unroll
+        for (int h = 0; h < HPL; ++h)
+          if (h == mh) {
+            ++pos[h];
+            head[h] = pos[h] < k ? at(lane + 32 * h, pos[h]) : kSentinel;
+          }
+      }
+    }
+    for (int j = i + lane; j < k; j += 32) o[j] = kSentinel;
+    if (seed != nullptr && lane == 0) {
+      float v = desc ? -INFINITY : INFINITY;
+      if (i == k) {
+        uint32_t ok = (uint32_t)(gm >> 32);
+        if (desc) ok = ~ok;
+        v = unord_f32(ok);
+      }
+      seed[b] = v;
+    }
   }
 }
 
@@ -606,6 +706,34 @@ static cudaError_t launch_kmerge_t(const ScoreArgs &a, cudaStream_t st, const Ro
   kern<<<(unsigned)((a.B + qpc - 1) / qpc), kKmWarps * 32, smem, st>>>(a, (int)qpc, rp);
   timing_launch_end(LAM_TIME_MERGE, st);
   return cudaGetLastError();
+}
+
+template <int HPL>
+static cudaError_t launch_slab_merge_t(const ScoreArgs &a, int list0, int n_lists, int slab,
+                                      uint64_t *out, float *seed, cudaStream_t st) {
+  const size_t per_q = (size_t)n_lists * a.k * 8;
+  const bool staged = per_q <= kKmCandBytes;
+  int64_t qpc = staged ? (int64_t)(kKmCandBytes / per_q) : kSmWarps;
+  if (qpc > kSmWarps) qpc = kSmWarps;
+  const int64_t spread = (a.B + 2LL * a.sms - 1) / (2LL * a.sms);
+  if (qpc > spread) qpc = spread;
+  if (qpc < 1) qpc = 1;
+  const size_t smem = staged ? (size_t)qpc * per_q : 0;
+  auto kern = slab_merge_kernel<HPL>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  kern<<<(unsigned)((a.B + qpc - 1) / qpc), kSmWarps * 32, smem, st>>>(a, list0, n_lists, (int)qpc,
+                                                                      staged, slab, out, seed);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_slab_merge(const ScoreArgs &a, int list0, int n_lists, int slab, uint64_t *out,
+                              float *seed, cudaStream_t st) {
+  if (n_lists <= 32) return launch_slab_merge_t<1>(a, list0, n_lists, slab, out, seed, st);
+  if (n_lists <= 64) return launch_slab_merge_t<2>(a, list0, n_lists, slab, out, seed, st);
+  if (n_lists <= 128) return launch_slab_merge_t<4>(a, list0, n_lists, slab, out, seed, st);
+  if (n_lists <= 256) return launch_slab_merge_t<8>(a, list0, n_lists, slab, out, seed, st);
+  return cudaErrorInvalidValue;
 }
 
 cudaError_t launch_topk_merge(const ScoreArgs &a, cudaStream_t st, const RowPtrs &rp) {

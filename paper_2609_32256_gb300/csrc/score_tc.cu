@@ -903,6 +903,7 @@ struct Tc2Geom {
   int64_t row_base, nrows;  // the slab
   int list_base;            // partial-list index of this slab's split 0
   const uint8_t *b16;       // fp16 operand image of the slab
+  const float *seed;        // later slabs: per query, the first slab's k-th best score
   const float *rowf;        // per-row factors of the slab (Q_eps codes)
   const float4 *rowf4;      // per-row (u, w, z) of the slab (per-row codecs)
 };
@@ -1083,6 +1084,12 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
     reg.init(k);
     float thr_s = desc ? -INFINITY : INFINITY;
     float seed = desc ? -INFINITY : INFINITY;  // admission bound before the list fills
+    if (g.seed != nullptr && qvalid) {
+      // rows worse than the first slab's k-th best cannot enter the final top-k
+      // (equal ones are still offered)
+      const float t = g.seed[qidx];
+      seed = desc ? nextafterf(t, -INFINITY) : nextafterf(t, INFINITY);
+    }
     if (KR == 0)
       for (int i = 0; i < k; ++i) lists[(size_t)i * kBM + m] = kSentinel;
     for (int lt = 0; lt < ntl; ++lt) {
@@ -1124,7 +1131,8 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
           }
         }
         const float kth = kth_largest(gb, k);  // in "larger is better" units
-        seed = desc ? nextafterf(kth, -INFINITY) : nextafterf(-kth, INFINITY);
+        seed = desc ? fmaxf(seed, nextafterf(kth, -INFINITY))
+                    : fminf(seed, nextafterf(-kth, INFINITY));
       }
 #pragma unroll 1
       for (int c = 0; c < kBN / 32; ++c) {
@@ -1262,9 +1270,17 @@ int gcd_i(int x, int y) {
 
 }  // namespace
 
-bool tensor_fits(int width, int k) {
+// Four or more query blocks: the codes are converted once per call (each
+// code tile would otherwise be converted once per query block); one to three
+// blocks convert in the stage loop.  Measured: B = 256 over 8.4M int8 rows
+// takes 8.3 ms in the stage loop against 9.4 ms with the conversion pass (3.1
+// of them); B = 1,024 over 27,986 rows 88 us against 72 + 12.
+constexpr int64_t kPreBlocks = 4;
+
+bool tensor_fits(int width, int k, int64_t B) {
   if (k > kTcMaxK || (width != 1 && width != 2)) return false;
-  return tc_layout(width, k).ns >= 2 && tc2_layout(k).ns >= 2;
+  if ((B + kBM - 1) / kBM >= kPreBlocks) return tc2_layout(k).ns >= 2;
+  return tc_layout(width, k).ns >= 2;
 }
 
 bool tensor_fits_pre(int k) { return k <= kTcMaxK && tc2_layout(k).ns >= 2; }
@@ -1283,7 +1299,7 @@ TensorPlan tensor_plan(int64_t B, int64_t N, int D, int k, int sms, bool force_p
   TensorPlan p;
   const int64_t Bpad = (B + kBM - 1) / kBM * kBM;
   const int64_t nk = (D + kBK - 1) / kBK;
-  p.pre = force_pre || Bpad / kBM >= 2;
+  p.pre = force_pre || Bpad / kBM >= kPreBlocks;
   p.qinfo_off = (size_t)(Bpad / kBM) * nk * kAStage;
   size_t off = p.qinfo_off + (size_t)Bpad * 16;
   off = (off + 255) / 256 * 256;
@@ -1291,7 +1307,7 @@ TensorPlan tensor_plan(int64_t B, int64_t N, int D, int k, int sms, bool force_p
     p.slab_rows = N;
     p.nslabs = 1;
     p.nsplit = tensor_splits(B, N, sms);
-    p.fp16_off = p.rowf_off = off;
+    p.fp16_off = p.rowf_off = p.seed_off = p.slabl_off = off;
     p.bytes = off;
   } else {
     int64_t cap = ((int64_t)1 << 30) / (nk * kBK * 2) / kBN * kBN;  // ~1 GiB of fp16 rows
@@ -1301,13 +1317,17 @@ TensorPlan tensor_plan(int64_t B, int64_t N, int D, int k, int sms, bool force_p
     p.nsplit = tensor_splits(B, p.slab_rows, sms);
     p.fp16_off = off;
     p.rowf_off = p.fp16_off + (size_t)((p.slab_rows + kBN - 1) / kBN) * nk * kB16Bytes;
-    p.bytes = p.rowf_off + (size_t)p.slab_rows * 16;
+    p.seed_off = p.rowf_off + (size_t)p.slab_rows * 16;
+    p.slabl_off = (p.seed_off + (size_t)Bpad * 4 + 255) / 256 * 256;
+    p.bytes = p.slabl_off + (p.nslabs > 1 ? (size_t)p.nslabs * B * k * 8 : 0);
   }
   p.n_lists = p.nslabs * p.nsplit;
   return p;
 }
 
-cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st, const RowPtrs &rp) {
+cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st, const RowPtrs &rp,
+                                ScoreArgs *merge) {
+  if (merge != nullptr) *merge = a;
   const bool rc = a.fmt != 0;
   if (a.k > kTcMaxK || (!rc && a.width != 1 && a.width != 2)) return cudaErrorInvalidValue;
   const TensorPlan P = tensor_plan(a.B, a.N, a.D, a.k, a.sms, rc);
@@ -1371,6 +1391,12 @@ cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st, const RowPt
   g.b16 = f16;
   g.rowf = rowf;
   g.rowf4 = reinterpret_cast<const float4 *>(rowf);
+  g.seed = nullptr;
+  float *seed = reinterpret_cast<float *>(static_cast<uint8_t *>(a.qprep) + P.seed_off);
+  uint64_t *slabl = reinterpret_cast<uint64_t *>(static_cast<uint8_t *>(a.qprep) + P.slabl_off);
+  // several slabs: each slab's lists are merged into one, and the first slab's
+  // k-th best bounds what the later slabs may offer
+  const bool per_slab = P.nslabs > 1 && P.nsplit <= 256;
   auto kern = rc ? (a.k <= 16   ? score_tc2_kernel<16, true>
                     : a.k <= 32 ? score_tc2_kernel<32, true>
                                 : score_tc2_kernel<0, true>)
@@ -1430,6 +1456,17 @@ cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st, const RowPt
     timing_launch_end(LAM_TIME_SCORE, st);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
+    if (per_slab) {
+      timing_launch_begin(LAM_TIME_MERGE, st);
+      e = launch_slab_merge(a, j * P.nsplit, P.nsplit, j, slabl, j == 0 ? seed : nullptr, st);
+      timing_launch_end(LAM_TIME_MERGE, st);
+      if (e != cudaSuccess) return e;
+      if (j == 0) g.seed = seed;
+    }
+  }
+  if (per_slab && merge != nullptr) {
+    merge->partial = slabl;
+    merge->n_lists = P.nslabs;
   }
   return cudaSuccess;
 }

@@ -163,3 +163,25 @@ def test_workload_size_sampled(dev, fmt):
     full = oracle.scores_rows(q[sample], rows, oracle.IP)
     os_, oi = oracle.topk(full, k, oracle.IP)
     check_topk_fn(gs[sample], gi[sample], lambda b, ids: full[b, ids], n, oracle.IP, os_, oi)
+
+
+def test_two_slabs_with_first_slab_bound(dev):
+    """Per-vector int8 rows over two fp16 slabs (750,000 x 768), L2 top-100:
+    the second slab offers only rows at least as good as the first slab's
+    k-th best; sampled queries against the oracle."""
+    n, d, k = 750000, 768, 100
+    x = inputs.unit_rows_device(n, d, seed=78, device=dev)
+    x[700100:700140] = x[0:40]
+    codes, scale, offset = lam.encode_rows(x, lam.LAM_ROWS_INT8)
+    q = inputs.queries(200, d, seed=6)
+    q[7] = x[30].cpu().numpy()
+    del x
+    gs, gi = lam.search_rows(torch.from_numpy(q).to(dev), codes, lam.LAM_ROWS_INT8, scale,
+                             offset, k, oracle.L2)
+    gs, gi = gs.cpu().numpy(), gi.cpu().numpy()
+    rows = oracle.decode_rows(codes.cpu().numpy(), oracle.FMT_INT8_ROWS, d,
+                              scale.cpu().numpy(), offset.cpu().numpy())
+    sel = np.array([0, 7, 128, 199])
+    full = oracle.scores_rows(q[sel], rows, oracle.L2)
+    os_, oi = oracle.topk(full, k, oracle.L2)
+    check_topk_fn(gs[sel], gi[sel], lambda b, ids: full[b, ids], n, oracle.L2, os_, oi)

@@ -73,7 +73,7 @@ def test_tensor_path(dev, score_path, metric, width, eps, B):
 
 @pytest.mark.parametrize("D", [16, 48, 80, 1024])
 @pytest.mark.parametrize("k", [1, 16, 17, 32, 64, 112])
-@pytest.mark.parametrize("B", [20, 300])  # one query block; several (codes pre-converted)
+@pytest.mark.parametrize("B", [20, 300, 520])  # 1 and 3 query blocks (stage-loop conversion); 5 (conversion pass)
 def test_tensor_path_dims_and_k(dev, score_path, D, k, B):
     score_path("tensor")
     codes, bound = make_codes(700, D, 1e-2, 1, seed=D + k)
@@ -172,3 +172,42 @@ def test_code_sqnorms_bit_exact(dev, width, N, D):
     out = torch.empty(N, dtype=torch.float32, device=dev)
     lam.lam_code_sqnorms(ct, width, N, D, out)
     np.testing.assert_array_equal(out.cpu().numpy().view(np.uint32), want.view(np.uint32))
+
+
+@pytest.mark.parametrize("metric,k", [(oracle.IP, 10), (oracle.L2, 100), (oracle.COSINE, 128)])
+def test_tensor_two_slabs_with_first_slab_bound(dev, score_path, metric, k):
+    """750,000 rows take two fp16 slabs: the second slab only offers rows at
+    least as good as the first slab's k-th best.  Duplicated rows across the
+    slab boundary tie exactly; sampled queries against the oracle."""
+    score_path("tensor")
+    n, d, eps = 750000, 768, 1e-2
+    x = inputs.unit_rows_device(n, d, seed=77, device=dev)
+    x[720000:720050] = x[10:60]  # second-slab copies of first-slab rows
+    codes = torch.empty((n, d), dtype=torch.int8, device=dev)
+    ws = torch.zeros(64, dtype=torch.uint8, device=dev)
+    st, w, scale, cmin, cmax = lam.lam_quantize(x, eps, 1, codes, ws)
+    assert st == 0 and w == 1
+    del x
+    q = inputs.queries(520, d, seed=5)  # five query blocks: the conversion pass, in slabs
+    # plant queries equal to duplicated rows so that the ties reach the top-k
+    q[3] = (codes[20].float() * scale).cpu().numpy()
+    q[129] = (codes[45].float() * scale).cpu().numpy()
+    gs, gi = lam.search(torch.from_numpy(q).to(dev), codes, eps, k, metric,
+                        code_bound=max(-cmin, cmax))
+    gs, gi = gs.cpu().numpy(), gi.cpu().numpy()
+    sel = np.array([0, 3, 129, 257, 519])
+    oc = codes.cpu().numpy().astype(np.int32)
+    os_, oi = oracle_topk(q[sel], oc, eps, metric, k)
+    check_topk(gs[sel], gi[sel], q[sel], oc, eps, metric, os_, oi)
+
+
+def test_tensor_k128_needs_the_conversion_pass(dev, score_path):
+    """k = 128 fits the conversion-pass kernel only: five query blocks take the
+    tensor path, one block the generic path."""
+    codes, bound = make_codes(2000, 768, 1e-2, 1, seed=128)
+    assert lam.lam_score_topk_path(520, 2000, 768, 128, 1, bound) == lam.PATH_TENSOR
+    assert lam.lam_score_topk_path(100, 2000, 768, 128, 1, bound) == lam.PATH_GENERIC
+    score_path("tensor")
+    q = inputs.queries(520, 768, seed=128)
+    for metric in METRICS:
+        check(dev, q, codes, 1, 1e-2, 128, metric, bound)
