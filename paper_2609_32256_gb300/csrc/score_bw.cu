@@ -61,6 +61,12 @@ __device__ __forceinline__ float warp_sum(float v) {
   return v;
 }
 
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, off));
+  return v;
+}
+
 // Sums a over the lanes 0-15 and b over the lanes 16-31 with one shared
 // butterfly: lanes 0-15 end with sum(a), lanes 16-31 with sum(b).
 __device__ __forceinline__ float pair_sum(float a, float b, int lane) {
@@ -171,6 +177,56 @@ __global__ void __launch_bounds__(kBwThreads, 1)
       qq[q] = warp_sum(part);
       qn[q] = sqrtf(qq[q]);
     }
+    // int8 codes: the query as signed base-256 digits of round(q 2^e) with
+    // max|q| 2^e in [2^21, 2^22), so that the products with the codes are
+    // integer dot products (__dp4a) summed exactly per digit plane; the
+    // query's rounding, |q 2^e - round(q 2^e)| <= 1/2, is the only error
+    // besides the final fp32 sums (the tensor path's hi/lo split has 2^-22)
+    uint32_t qdig[W == 1 ? QB : 1][W == 1 ? kNchMax : 1][3][2];
+    float qinv[QB];
+#pragma unroll
+    for (int q = 0; q < QB; ++q) qinv[q] = 1.0f;
+    if constexpr (W == 1) {
+#pragma unroll
+      for (int q = 0; q < QB; ++q) {
+        float mx = 0.0f;
+#pragma unroll
+        for (int j = 0; j < kNchMax; ++j)
+#pragma unroll
+          for (int t = 0; t < 4; ++t)
+            mx = fmaxf(mx, fmaxf(fabsf(qreg[q][j][t].x), fabsf(qreg[q][j][t].y)));
+        mx = warp_max(mx);
+        int e = 0;
+        if (mx > 0.0f) {
+          int ex;
+          frexpf(mx, &ex);  // mx = f 2^ex, f in [0.5, 1)
+          e = max(-126, min(126, 22 - ex));
+        }
+        const float sc = ldexpf(1.0f, e);
+        qinv[q] = ldexpf(1.0f, -e);
+#pragma unroll
+        for (int j = 0; j < kNchMax; ++j)
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            uint32_t w0 = 0, w1 = 0, w2 = 0;
+#pragma unroll
+            for (int t = 0; t < 4; ++t) {
+              const float2 pr = qreg[q][j][2 * h + (t >> 1)];
+              const int qi = __float2int_rn((t & 1) ? pr.y * sc : pr.x * sc);
+              const int d2 = ((qi + 128) & 255) - 128;
+              const int r1 = (qi - d2) >> 8;
+              const int d1 = ((r1 + 128) & 255) - 128;
+              const int d0 = (r1 - d1) >> 8;
+              w0 |= ((uint32_t)d0 & 0xffu) << (8 * t);
+              w1 |= ((uint32_t)d1 & 0xffu) << (8 * t);
+              w2 |= ((uint32_t)d2 & 0xffu) << (8 * t);
+            }
+            qdig[q][j][0][h] = w0;
+            qdig[q][j][1][h] = w1;
+            qdig[q][j][2][h] = w2;
+          }
+      }
+    }
     const bool desc = a.metric != LAM_METRIC_L2;
     const float s = a.s, s2 = a.s * a.s;
     float thr_s[QB];  // score of each list's k-th entry; rows come in increasing
@@ -193,8 +249,48 @@ __global__ void __launch_bounds__(kBwThreads, 1)
 #pragma unroll
         for (int q = 0; q < QB; ++q) acc_a[q] = acc_b[q] = make_float2(0.0f, 0.0f);
         float2 cc_a = make_float2(0.0f, 0.0f), cc_b = make_float2(0.0f, 0.0f);
+        if constexpr (W == 1) {
+          // integer dot products per digit plane, exact in int32
+          int ia[QB][3], ib[QB][3], ca = 0, cb = 0;
 #pragma unroll
-        for (int j = 0; j < kNchMax; ++j) {
+          for (int q = 0; q < QB; ++q)
+#pragma unroll
+            for (int p = 0; p < 3; ++p) ia[q][p] = ib[q][p] = 0;
+#pragma unroll
+          for (int j = 0; j < kNchMax; ++j) {
+            const int e0 = (j * 32 + lane) * 8;
+            if (j < nch && e0 < D) {
+              const uint2 wa = *reinterpret_cast<const uint2 *>(pa + e0);
+              const uint2 wb = *reinterpret_cast<const uint2 *>(pb + e0);
+#pragma unroll
+              for (int q = 0; q < QB; ++q)
+#pragma unroll
+                for (int p = 0; p < 3; ++p) {
+                  ia[q][p] = __dp4a((int)wa.x, (int)qdig[q][j][p][0], ia[q][p]);
+                  ia[q][p] = __dp4a((int)wa.y, (int)qdig[q][j][p][1], ia[q][p]);
+                  ib[q][p] = __dp4a((int)wb.x, (int)qdig[q][j][p][0], ib[q][p]);
+                  ib[q][p] = __dp4a((int)wb.y, (int)qdig[q][j][p][1], ib[q][p]);
+                }
+              if (CC) {
+                ca = __dp4a((int)wa.x, (int)wa.x, ca);
+                ca = __dp4a((int)wa.y, (int)wa.y, ca);
+                cb = __dp4a((int)wb.x, (int)wb.x, cb);
+                cb = __dp4a((int)wb.y, (int)wb.y, cb);
+              }
+            }
+          }
+#pragma unroll
+          for (int q = 0; q < QB; ++q) {
+            acc_a[q].x = fmaf((float)ia[q][0], 65536.0f, fmaf((float)ia[q][1], 256.0f,
+                                                              (float)ia[q][2]));
+            acc_b[q].x = fmaf((float)ib[q][0], 65536.0f, fmaf((float)ib[q][1], 256.0f,
+                                                              (float)ib[q][2]));
+          }
+          cc_a.x = (float)ca;
+          cc_b.x = (float)cb;
+        }
+#pragma unroll
+        for (int j = 0; j < (W == 1 ? 0 : kNchMax); ++j) {
           const int e0 = (j * 32 + lane) * 8;
           if (j < nch && e0 < D) {
             float2 fa[4], fb[4];
@@ -218,7 +314,8 @@ __global__ void __launch_bounds__(kBwThreads, 1)
         const float cc = CC ? pair_sum(cc_a.x + cc_a.y, cc_b.x + cc_b.y, lane) : 0.0f;
 #pragma unroll
         for (int q = 0; q < QB; ++q) {
-          const float acc = pair_sum(acc_a[q].x + acc_a[q].y, acc_b[q].x + acc_b[q].y, lane);
+          const float acc =
+              pair_sum(acc_a[q].x + acc_a[q].y, acc_b[q].x + acc_b[q].y, lane) * qinv[q];
           // lanes 0-15 hold row rr, lanes 16-31 row rb
           const float sc = finish_score(a.metric, acc, cc, s, s2, qq[q], qn[q]);
           const float sa = __shfl_sync(0xffffffffu, sc, 0);
