@@ -313,9 +313,11 @@ lam_status lam_decode_rows(const void *codes, int32_t fmt, int64_t N, int32_t D,
  * so the codes enter the tensor-core product as they are stored.
  *
  * codes, scale, offset as written by lam_encode_rows for `fmt` (a 16-byte
- * aligned code base enables the tensor-core path).  Other arguments, the
- * workspace rule, LAM_SCORE_PATH (tensor|generic here) and the status read
- * (lam_score_topk_status) as for lam_score_topk.  Asynchronous.
+ * aligned code base enables the bulk-copy and tensor-core paths: B <= 2 takes
+ * the bandwidth kernel when D <= 1024, k <= 128 and a row is a multiple of 16
+ * bytes, larger batches the tensor cores).  Other arguments, the workspace
+ * rule, LAM_SCORE_PATH and the status read (lam_score_topk_status) as for
+ * lam_score_topk.  Asynchronous.
  * Errors: LAM_ERR_INVALID, LAM_ERR_WORKSPACE, LAM_ERR_UNSUPPORTED,
  * LAM_ERR_CUDA.
  */

@@ -136,19 +136,22 @@ bool rows_shape_ok(int64_t B, int64_t N, int32_t D, int32_t k, int32_t fmt) {
 bool make_rows_plan(int64_t B, int64_t N, int32_t D, int32_t k, int32_t fmt, int sms, Plan *p) {
   if (!rows_shape_ok(B, N, D, k, fmt) || sms <= 0) return false;
   const bool tc = D % 16 == 0 && tensor_fits_pre(k) && B <= (1LL << 23);
+  const int row_bytes = fmt == LAM_ROWS_INT8 ? D : fmt == LAM_ROWS_FP16 ? 2 * D : D / 8;
+  const bool bw = B <= 2 && k <= 128 && D <= 1024 && D % 8 == 0 && row_bytes % 16 == 0;
   const int f = forced_path();
   if (f == -2) return false;
-  int path = tc ? kPathTensor : kPathGeneric;
+  int path = bw ? kPathBandwidth : tc ? kPathTensor : kPathGeneric;
   if (f >= 0) {
-    if (f == kPathBandwidth || (f == kPathTensor && !tc)) {
+    if ((f == kPathBandwidth && !bw) || (f == kPathTensor && !tc)) {
       p->path = -2;
       return false;
     }
     path = f;
   }
   p->path = path;
-  p->n_lists = path == kPathTensor ? tensor_plan(B, N, D, k, sms, true).n_lists
-                                   : generic_ctas(B, N, sms);
+  p->n_lists = path == kPathTensor      ? tensor_plan(B, N, D, k, sms, true).n_lists
+               : path == kPathBandwidth ? bandwidth_rows_ctas(N, fmt, D, sms)
+                                        : generic_ctas(B, N, sms);
   p->Bpad = (B + 127) / 128 * 128;
   p->partial_off = kHeaderBytes;
   const size_t partial = (size_t)p->n_lists * (size_t)B * (size_t)k * 8;
@@ -735,8 +738,9 @@ lam_status lam_score_topk_rows(const float *queries, int64_t B, const void *code
   rp.scale = scale;
   rp.offset = offset;
   ScoreArgs m = a;  // the final merge's lists
-  const cudaError_t e = p.path == kPathTensor ? launch_score_tensor(a, st, rp, &m)
-                                              : launch_score_generic(a, st, rp);
+  const cudaError_t e = p.path == kPathTensor      ? launch_score_tensor(a, st, rp, &m)
+                        : p.path == kPathBandwidth ? launch_score_bandwidth_rows(a, rp, st)
+                                                   : launch_score_generic(a, st, rp);
   if (e != cudaSuccess) return LAM_ERR_CUDA;
   if (launch_topk_merge(m, st, rp) != cudaSuccess) return LAM_ERR_CUDA;
   return LAM_OK;

@@ -230,6 +230,9 @@ cudaError_t launch_decode_rows(const void *codes, int fmt, int64_t N, int D, con
                                const float *offset, float *out, int sms, cudaStream_t st);
 
 cudaError_t launch_score_bandwidth(const ScoreArgs &a, cudaStream_t st);
+// Per-vector codecs, B <= 2: row bytes (D, 2D or D/8) a multiple of 16, D <= 1024, k <= 128.
+cudaError_t launch_score_bandwidth_rows(const ScoreArgs &a, const RowPtrs &rp, cudaStream_t st);
+int bandwidth_rows_ctas(int64_t N, int fmt, int D, int sms);
 cudaError_t launch_score_generic(const ScoreArgs &a, cudaStream_t st,
                                  const RowPtrs &rp = RowPtrs());
 // `merge` (optional) receives the arguments of the final merge: a search of

@@ -354,6 +354,331 @@ __global__ void __launch_bounds__(kBwThreads, 1)
 }
 
 // ---------------------------------------------------------------------------
+// Per-vector codecs for B <= 2: the same pipeline over the stored rows (int8
+// codes with a scale and an offset per row, fp16 values, or sign bits with a
+// scale per row).  The decoding moves into the per-row finish:
+//   int8   q.xhat = scale (q.c) + offset sum(q),
+//          ||xhat||^2 = D offset^2 + 2 scale offset sum(c) + scale^2 sum(c^2)
+//          (q.c by __dp4a against the query's base-256 digits, as for Q_eps
+//          int8 codes; sum(c) and sum(c^2) by __dp4a as well)
+//   fp16   q.xhat with the values widened to fp32, ||xhat||^2 summed alongside
+//   sign   q.xhat = alpha (2 sum_{bit set} q - sum(q)), ||xhat||^2 = D alpha^2
+template <int FMT>
+__host__ __device__ constexpr int rows_bytes_per_dim8() {  // bytes per 8 coordinates
+  return FMT == LAM_ROWS_INT8 ? 8 : FMT == LAM_ROWS_FP16 ? 16 : 1;
+}
+
+template <int FMT, int QB, int KPL, bool CC>
+__global__ void __launch_bounds__(kBwThreads, 1)
+    score_bw_rows_kernel(ScoreArgs a, RowPtrs rp, int tr, int ns, int stage_bytes) {
+  extern __shared__ __align__(1024) uint8_t smem[];
+  uint64_t *full = reinterpret_cast<uint64_t *>(smem + (size_t)ns * stage_bytes);
+  uint64_t *empty = full + ns;
+  volatile int *abort_flag = reinterpret_cast<volatile int *>(empty + ns);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t N = a.N;
+  const int D = a.D;
+  const int64_t r0 = (int64_t)blockIdx.x * N / gridDim.x;
+  const int64_t r1 = (int64_t)(blockIdx.x + 1) * N / gridDim.x;
+  const int64_t nrows = r1 - r0;
+  const int ntiles = (int)((nrows + tr - 1) / tr);
+  constexpr int B8 = rows_bytes_per_dim8<FMT>();
+  const size_t row_bytes = (size_t)(D / 8) * B8;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < ns; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], kBwWarps);
+    }
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  __syncthreads();
+
+  WarpList<KPL> lists[QB];
+#pragma unroll
+  for (int q = 0; q < QB; ++q) lists[q].init();
+
+  if (warp == kBwWarps) {
+    if (lane == 0) {
+      int issued = 0;
+      for (int t = 0; t < ntiles; ++t) {
+        const int s = t % ns, r = t / ns;
+        if (r > 0 && !mbar_wait(&empty[s], (r - 1) & 1, abort_flag, a.gflags)) break;
+        const int64_t nr = min((int64_t)tr, nrows - (int64_t)t * tr);
+        const uint32_t bytes = (uint32_t)(nr * row_bytes);
+        mbar_arrive_expect_tx(&full[s], bytes);
+        bulk_g2s(smem + (size_t)s * stage_bytes,
+                 static_cast<const uint8_t *>(a.codes) + (r0 + (int64_t)t * tr) * row_bytes,
+                 bytes, &full[s]);
+        issued = t + 1;
+      }
+      for (int t = max(0, issued - ns); t < issued; ++t) drain_wait(&full[t % ns], (t / ns) & 1);
+    }
+  } else {
+    const int nch = (D + 255) / 256;
+    float2 qreg[QB][kNchMax][4];
+    float qq[QB], qn[QB], qs[QB];
+#pragma unroll
+    for (int q = 0; q < QB; ++q) {
+      const bool qv = q < a.B;
+      float part = 0.0f, sum = 0.0f;
+#pragma unroll
+      for (int j = 0; j < kNchMax; ++j) {
+        const int e0 = (j * 32 + lane) * 8;
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+          const int d = e0 + 2 * t;
+          const float v0 = (qv && j < nch && d < D) ? a.queries[(int64_t)q * D + d] : 0.0f;
+          const float v1 = (qv && j < nch && d + 1 < D) ? a.queries[(int64_t)q * D + d + 1] : 0.0f;
+          qreg[q][j][t] = make_float2(v0, v1);
+          part = fmaf(v0, v0, fmaf(v1, v1, part));
+          sum += v0 + v1;
+        }
+      }
+      qq[q] = warp_sum(part);
+      qn[q] = sqrtf(qq[q]);
+      qs[q] = warp_sum(sum);
+    }
+    uint32_t qdig[FMT == LAM_ROWS_INT8 ? QB : 1][FMT == LAM_ROWS_INT8 ? kNchMax : 1][3][2];
+    float qinv[QB];
+#pragma unroll
+    for (int q = 0; q < QB; ++q) qinv[q] = 1.0f;
+    if constexpr (FMT == LAM_ROWS_INT8) {
+#pragma unroll
+      for (int q = 0; q < QB; ++q) {
+        float mx = 0.0f;
+#pragma unroll
+        for (int j = 0; j < kNchMax; ++j)
+#pragma unroll
+          for (int t = 0; t < 4; ++t)
+            mx = fmaxf(mx, fmaxf(fabsf(qreg[q][j][t].x), fabsf(qreg[q][j][t].y)));
+        mx = warp_max(mx);
+        int e = 0;
+        if (mx > 0.0f) {
+          int ex;
+          frexpf(mx, &ex);
+          e = max(-126, min(126, 22 - ex));
+        }
+        const float sc = ldexpf(1.0f, e);
+        qinv[q] = ldexpf(1.0f, -e);
+#pragma unroll
+        for (int j = 0; j < kNchMax; ++j)
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            uint32_t w0 = 0, w1 = 0, w2 = 0;
+#pragma unroll
+            for (int t = 0; t < 4; ++t) {
+              const float2 pr = qreg[q][j][2 * h + (t >> 1)];
+              const int qi = __float2int_rn((t & 1) ? pr.y * sc : pr.x * sc);
+              const int d2 = ((qi + 128) & 255) - 128;
+              const int r1 = (qi - d2) >> 8;
+              const int d1 = ((r1 + 128) & 255) - 128;
+              const int d0 = (r1 - d1) >> 8;
+              w0 |= ((uint32_t)d0 & 0xffu) << (8 * t);
+              w1 |= ((uint32_t)d1 & 0xffu) << (8 * t);
+              w2 |= ((uint32_t)d2 & 0xffu) << (8 * t);
+            }
+            qdig[q][j][0][h] = w0;
+            qdig[q][j][1][h] = w1;
+            qdig[q][j][2][h] = w2;
+          }
+      }
+    }
+    const bool desc = a.metric != LAM_METRIC_L2;
+    float thr_s[QB];
+#pragma unroll
+    for (int q = 0; q < QB; ++q) thr_s[q] = desc ? -INFINITY : INFINITY;
+    // Per-row factors one row pair ahead: lanes 0-15 finish rows r0 + warp +
+    // 32 i, lanes 16-31 rows r0 + warp + 16 + 32 i (tiles hold a multiple of
+    // 32 rows), so the next factors are those of the row 32 further on.
+    int64_t frow = r0 + warp + (lane >= 16 ? kBwWarps : 0);
+    float f_sr = 1.0f, f_or = 0.0f;
+    if (FMT != LAM_ROWS_FP16 && frow < r1) f_sr = rp.scale[frow];
+    if (FMT == LAM_ROWS_INT8 && frow < r1) f_or = rp.offset[frow];
+
+    for (int t = 0; t < ntiles; ++t) {
+      const int st = t % ns, r = t / ns;
+      if (!mbar_wait(&full[st], r & 1, abort_flag, a.gflags)) break;
+      const int nr = (int)min((int64_t)tr, nrows - (int64_t)t * tr);
+      const uint8_t *stage = smem + (size_t)st * stage_bytes;
+      for (int rr = warp; rr < nr; rr += 2 * kBwWarps) {
+        const int rb = rr + kBwWarps;
+        const bool has_b = rb < nr;
+        const uint8_t *pa = stage + (size_t)rr * row_bytes;
+        const uint8_t *pb = stage + (size_t)(has_b ? rb : rr) * row_bytes;
+        const float sr = f_sr, orr = f_or;
+        frow += 2 * kBwWarps;
+        if (FMT != LAM_ROWS_FP16 && frow < r1) f_sr = rp.scale[frow];
+        if (FMT == LAM_ROWS_INT8 && frow < r1) f_or = rp.offset[frow];
+        float pa_acc[QB], pb_acc[QB], pa_c1 = 0.0f, pb_c1 = 0.0f, pa_c2 = 0.0f, pb_c2 = 0.0f;
+        if constexpr (FMT == LAM_ROWS_INT8) {
+          int ia[QB][3], ib[QB][3], sa1 = 0, sb1 = 0, sa2 = 0, sb2 = 0;
+#pragma unroll
+          for (int q = 0; q < QB; ++q)
+#pragma unroll
+            for (int p = 0; p < 3; ++p) ia[q][p] = ib[q][p] = 0;
+#pragma unroll
+          for (int j = 0; j < kNchMax; ++j) {
+            const int e0 = (j * 32 + lane) * 8;
+            if (j < nch && e0 < D) {
+              const uint2 wa = *reinterpret_cast<const uint2 *>(pa + e0);
+              const uint2 wb = *reinterpret_cast<const uint2 *>(pb + e0);
+#pragma unroll
+              for (int q = 0; q < QB; ++q)
+#pragma unroll
+                for (int p = 0; p < 3; ++p) {
+                  ia[q][p] = __dp4a((int)wa.x, (int)qdig[q][j][p][0], ia[q][p]);
+                  ia[q][p] = __dp4a((int)wa.y, (int)qdig[q][j][p][1], ia[q][p]);
+                  ib[q][p] = __dp4a((int)wb.x, (int)qdig[q][j][p][0], ib[q][p]);
+                  ib[q][p] = __dp4a((int)wb.y, (int)qdig[q][j][p][1], ib[q][p]);
+                }
+              if (CC) {
+                sa1 = __dp4a((int)wa.x, 0x01010101, __dp4a((int)wa.y, 0x01010101, sa1));
+                sb1 = __dp4a((int)wb.x, 0x01010101, __dp4a((int)wb.y, 0x01010101, sb1));
+                sa2 = __dp4a((int)wa.x, (int)wa.x, __dp4a((int)wa.y, (int)wa.y, sa2));
+                sb2 = __dp4a((int)wb.x, (int)wb.x, __dp4a((int)wb.y, (int)wb.y, sb2));
+              }
+            }
+          }
+#pragma unroll
+          for (int q = 0; q < QB; ++q) {
+            pa_acc[q] = fmaf((float)ia[q][0], 65536.0f, fmaf((float)ia[q][1], 256.0f,
+                                                              (float)ia[q][2]));
+            pb_acc[q] = fmaf((float)ib[q][0], 65536.0f, fmaf((float)ib[q][1], 256.0f,
+                                                              (float)ib[q][2]));
+          }
+          pa_c1 = (float)sa1;
+          pb_c1 = (float)sb1;
+          pa_c2 = (float)sa2;
+          pb_c2 = (float)sb2;
+        } else if constexpr (FMT == LAM_ROWS_FP16) {
+          float2 aa[QB], ab[QB], ca = make_float2(0.f, 0.f), cb = make_float2(0.f, 0.f);
+#pragma unroll
+          for (int q = 0; q < QB; ++q) aa[q] = ab[q] = make_float2(0.f, 0.f);
+#pragma unroll
+          for (int j = 0; j < kNchMax; ++j) {
+            const int e0 = (j * 32 + lane) * 8;
+            if (j < nch && e0 < D) {
+              const uint4 va = *reinterpret_cast<const uint4 *>(pa + (size_t)e0 * 2);
+              const uint4 vb = *reinterpret_cast<const uint4 *>(pb + (size_t)e0 * 2);
+              const uint32_t wa[4] = {va.x, va.y, va.z, va.w}, wb[4] = {vb.x, vb.y, vb.z, vb.w};
+#pragma unroll
+              for (int u = 0; u < 4; ++u) {
+                __half2 ha, hb;
+                memcpy(&ha, &wa[u], 4);
+                memcpy(&hb, &wb[u], 4);
+                const float2 fa = __half22float2(ha), fb = __half22float2(hb);
+#pragma unroll
+                for (int q = 0; q < QB; ++q) {
+                  aa[q] = __ffma2_rn(qreg[q][j][u], fa, aa[q]);
+                  ab[q] = __ffma2_rn(qreg[q][j][u], fb, ab[q]);
+                }
+                if (CC) {
+                  ca = __ffma2_rn(fa, fa, ca);
+                  cb = __ffma2_rn(fb, fb, cb);
+                }
+              }
+            }
+          }
+#pragma unroll
+          for (int q = 0; q < QB; ++q) {
+            pa_acc[q] = aa[q].x + aa[q].y;
+            pb_acc[q] = ab[q].x + ab[q].y;
+          }
+          pa_c2 = ca.x + ca.y;
+          pb_c2 = cb.x + cb.y;
+        } else {
+          // sign bits: the sum of q over the set bits
+          float2 aa[QB], ab[QB];
+#pragma unroll
+          for (int q = 0; q < QB; ++q) aa[q] = ab[q] = make_float2(0.f, 0.f);
+#pragma unroll
+          for (int j = 0; j < kNchMax; ++j) {
+            const int e0 = (j * 32 + lane) * 8;
+            if (j < nch && e0 < D) {
+              const uint32_t ba = pa[e0 / 8], bb = pb[e0 / 8];
+#pragma unroll
+              for (int u = 0; u < 4; ++u) {
+                const float2 ma = make_float2((float)((ba >> (2 * u)) & 1u),
+                                             (float)((ba >> (2 * u + 1)) & 1u));
+                const float2 mb = make_float2((float)((bb >> (2 * u)) & 1u),
+                                             (float)((bb >> (2 * u + 1)) & 1u));
+#pragma unroll
+                for (int q = 0; q < QB; ++q) {
+                  aa[q] = __ffma2_rn(qreg[q][j][u], ma, aa[q]);
+                  ab[q] = __ffma2_rn(qreg[q][j][u], mb, ab[q]);
+                }
+              }
+            }
+          }
+#pragma unroll
+          for (int q = 0; q < QB; ++q) {
+            pa_acc[q] = aa[q].x + aa[q].y;
+            pb_acc[q] = ab[q].x + ab[q].y;
+          }
+        }
+        // lanes 0-15 finish row rr, lanes 16-31 row rb (its factors are unused
+        // when the pair has no second row)
+        const float c1 = (FMT == LAM_ROWS_INT8 && CC) ? pair_sum(pa_c1, pb_c1, lane) : 0.0f;
+        const float c2 = (FMT != LAM_ROWS_SIGN && CC) ? pair_sum(pa_c2, pb_c2, lane) : 0.0f;
+        float xx = 0.0f;
+        if (CC) {
+          if (FMT == LAM_ROWS_INT8)
+            xx = fmaf(sr * sr, c2, fmaf(2.0f * sr * orr, c1, (float)D * orr * orr));
+          else if (FMT == LAM_ROWS_FP16)
+            xx = c2;
+          else
+            xx = (float)D * sr * sr;
+        }
+#pragma unroll
+        for (int q = 0; q < QB; ++q) {
+          const float acc = pair_sum(pa_acc[q], pb_acc[q], lane) * qinv[q];
+          float dot;
+          if (FMT == LAM_ROWS_INT8) dot = fmaf(sr, acc, orr * qs[q]);
+          else if (FMT == LAM_ROWS_FP16) dot = acc;
+          else dot = sr * fmaf(2.0f, acc, -qs[q]);
+          float sc;
+          if (a.metric == LAM_METRIC_IP) sc = dot;
+          else if (a.metric == LAM_METRIC_COSINE)
+            sc = (qn[q] == 0.0f || xx == 0.0f) ? 0.0f : dot / (qn[q] * sqrtf(xx));
+          else sc = fmaf(-2.0f, dot, qq[q] + xx);
+          const float sa = __shfl_sync(0xffffffffu, sc, 0);
+          const float sb = __shfl_sync(0xffffffffu, sc, 16);
+          if (q >= a.B) continue;
+          if (desc ? sa > thr_s[q] : sa < thr_s[q]) {
+            lists[q].insert(make_key(sa, (uint32_t)(r0 + (int64_t)t * tr + rr), desc), lane);
+            const uint64_t kk = lists[q].kth(a.k);
+            thr_s[q] = kk == kSentinel ? (desc ? -INFINITY : INFINITY)
+                                       : rank_key32_score((uint32_t)(kk >> 32), desc);
+          }
+          if (has_b && (desc ? sb > thr_s[q] : sb < thr_s[q])) {
+            lists[q].insert(make_key(sb, (uint32_t)(r0 + (int64_t)t * tr + rb), desc), lane);
+            const uint64_t kk = lists[q].kth(a.k);
+            thr_s[q] = kk == kSentinel ? (desc ? -INFINITY : INFINITY)
+                                       : rank_key32_score((uint32_t)(kk >> 32), desc);
+          }
+        }
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&empty[st]);
+    }
+  }
+  __syncthreads();
+  uint64_t *cand = reinterpret_cast<uint64_t *>(smem);
+  if (warp < kBwWarps) {
+#pragma unroll
+    for (int q = 0; q < QB; ++q)
+      lists[q].store(cand + ((size_t)q * kBwWarps + warp) * a.k, a.k, lane);
+  }
+  __syncthreads();
+  for (int q = 0; q < QB && q < a.B; ++q)
+    rank_merge(cand + (size_t)q * kBwWarps * a.k, kBwWarps, a.k,
+               a.partial + ((size_t)blockIdx.x * a.B + q) * a.k, threadIdx.x, kBwThreads);
+}
+
+// ---------------------------------------------------------------------------
 // Generic path: any D, width 1/2/4, k <= 1024, any batch.  Grid (ctas, B):
 // a CTA scores one query against a range of rows, warp per row with plain
 // global loads, per-warp top-k lists in shared memory, then a rank merge.
@@ -771,6 +1096,46 @@ cudaError_t launch_score_bandwidth(const ScoreArgs &a, cudaStream_t st) {
   if ((size_t)2 * kBwWarps * a.k * 8 > (size_t)sh.ns * sh.stage_bytes) return cudaErrorInvalidValue;
   if (a.width == 1) return a.B == 1 ? launch_bw_k<1, 1>(a, sh, st) : launch_bw_k<1, 2>(a, sh, st);
   return a.B == 1 ? launch_bw_k<2, 1>(a, sh, st) : launch_bw_k<2, 2>(a, sh, st);
+}
+
+template <int FMT, int QB, int KPL>
+static cudaError_t launch_bw_rows_t(const ScoreArgs &a, const RowPtrs &rp, const BwShape &sh,
+                                   cudaStream_t st) {
+  const size_t smem = (size_t)sh.ns * sh.stage_bytes + 2 * sh.ns * sizeof(uint64_t) + 16;
+  auto kern = a.metric == LAM_METRIC_IP ? score_bw_rows_kernel<FMT, QB, KPL, false>
+                                        : score_bw_rows_kernel<FMT, QB, KPL, true>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  timing_launch_begin(LAM_TIME_SCORE, st);
+  kern<<<a.n_lists, kBwThreads, smem, st>>>(a, rp, sh.tr, sh.ns, sh.stage_bytes);
+  timing_launch_end(LAM_TIME_SCORE, st);
+  return cudaGetLastError();
+}
+
+template <int FMT>
+static cudaError_t launch_bw_rows_f(const ScoreArgs &a, const RowPtrs &rp, const BwShape &sh,
+                                   cudaStream_t st) {
+  if (a.B == 1)
+    return a.k <= 32 ? launch_bw_rows_t<FMT, 1, 1>(a, rp, sh, st)
+                     : launch_bw_rows_t<FMT, 1, 4>(a, rp, sh, st);
+  return a.k <= 32 ? launch_bw_rows_t<FMT, 2, 1>(a, rp, sh, st)
+                   : launch_bw_rows_t<FMT, 2, 4>(a, rp, sh, st);
+}
+
+int rows_row_bytes(int fmt, int D) {
+  return fmt == LAM_ROWS_INT8 ? D : fmt == LAM_ROWS_FP16 ? 2 * D : D / 8;
+}
+
+int bandwidth_rows_ctas(int64_t N, int fmt, int D, int sms) {
+  return bandwidth_ctas(N, rows_row_bytes(fmt, D), 1, sms);
+}
+
+cudaError_t launch_score_bandwidth_rows(const ScoreArgs &a, const RowPtrs &rp, cudaStream_t st) {
+  const BwShape sh = bw_shape(rows_row_bytes(a.fmt, a.D), 1);
+  if ((size_t)2 * kBwWarps * a.k * 8 > (size_t)sh.ns * sh.stage_bytes) return cudaErrorInvalidValue;
+  if (a.fmt == LAM_ROWS_INT8) return launch_bw_rows_f<LAM_ROWS_INT8>(a, rp, sh, st);
+  if (a.fmt == LAM_ROWS_FP16) return launch_bw_rows_f<LAM_ROWS_FP16>(a, rp, sh, st);
+  return launch_bw_rows_f<LAM_ROWS_SIGN>(a, rp, sh, st);
 }
 
 cudaError_t launch_score_generic(const ScoreArgs &a, cudaStream_t st, const RowPtrs &rp) {

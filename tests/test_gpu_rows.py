@@ -185,3 +185,32 @@ def test_two_slabs_with_first_slab_bound(dev):
     full = oracle.scores_rows(q[sel], rows, oracle.L2)
     os_, oi = oracle.topk(full, k, oracle.L2)
     check_topk_fn(gs[sel], gi[sel], lambda b, ids: full[b, ids], n, oracle.L2, os_, oi)
+
+
+@pytest.mark.parametrize("metric", METRICS)
+@pytest.mark.parametrize("fmt", FMTS)
+@pytest.mark.parametrize("B", [1, 2])
+@pytest.mark.parametrize("k", [1, 10, 100, 128])
+def test_bandwidth_path(dev, score_path, fmt, metric, B, k):
+    score_path("bandwidth")
+    assert lam.lam_score_topk_rows_path(B, 5003, 768, k, fmt) == lam.PATH_BANDWIDTH
+    rows_case(dev, fmt, 5003, 768, B, k, metric, seed=B + k)
+
+
+@pytest.mark.parametrize("fmt", FMTS)
+@pytest.mark.parametrize("d", [128, 256, 1024])
+def test_bandwidth_path_dims(dev, score_path, fmt, d):
+    score_path("bandwidth")
+    for metric in METRICS:
+        rows_case(dev, fmt, 777, d, 2, 10, metric, seed=d)
+
+
+def test_bandwidth_path_routing(dev):
+    # small batches go to the bandwidth kernel when a row is a multiple of 16
+    # bytes; otherwise to the tensor cores or the generic kernel
+    assert lam.lam_score_topk_rows_path(1, 1000, 768, 10, lam.LAM_ROWS_SIGN) == lam.PATH_BANDWIDTH
+    assert lam.lam_score_topk_rows_path(1, 1000, 64, 10, lam.LAM_ROWS_SIGN) == lam.PATH_TENSOR
+    assert lam.lam_score_topk_rows_path(1, 1000, 24, 10, lam.LAM_ROWS_FP16) == lam.PATH_BANDWIDTH
+    assert lam.lam_score_topk_rows_path(1, 1000, 24, 10, lam.LAM_ROWS_INT8) == lam.PATH_GENERIC
+    assert lam.lam_score_topk_rows_path(3, 1000, 768, 10, lam.LAM_ROWS_INT8) == lam.PATH_TENSOR
+    assert lam.lam_score_topk_rows_path(2, 1000, 768, 200, lam.LAM_ROWS_INT8) == lam.PATH_GENERIC
