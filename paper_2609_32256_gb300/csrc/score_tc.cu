@@ -48,6 +48,7 @@ constexpr int kStageBytes = kAStage + kB16Bytes;  // one MMA stage: 32 KB
 constexpr int kRawRow = 128;              // bytes of one code row per raw stage
 constexpr int kRawBytes = kBN * kRawRow;  // one raw stage: 32 KB
 constexpr int kCBuf = 16;                 // epilogue candidate buffer per query
+constexpr int kTcChunks = 2;              // K chunks per MMA stage of the stage-loop kernel
 constexpr uint32_t kTmemCols = 512;       // two 256-column accumulators
 constexpr int kMaxDynSmem = 232448;       // 227 KB
 constexpr int kTcMaxK = 128;
@@ -181,7 +182,7 @@ __device__ __forceinline__ uint32_t select32(const uint32_t (&v)[32], int j) {
 }
 
 struct TcLayout {
-  int ns, nr;  // MMA stages, raw stages
+  int ns, nr, chunks;  // MMA stages, raw stages, K chunks per MMA stage
   size_t raw_off, lists_off, cbuf_off, cc_off, bar_off, smem_bytes;
 };
 
@@ -195,8 +196,11 @@ inline TcLayout tc_layout(int width, int k) {
   const size_t cc = 2 * kBN * 4;
   const size_t tailb = 64 * 8 + 1024;  // barriers, slots, alignment slack
   const size_t avail = kMaxDynSmem - lists - cbuf - cc - tailb;
-  int ns = 4, nr = 2;
-  while ((size_t)ns * kStageBytes + (size_t)nr * kRawBytes > avail) {
+  // two K chunks per MMA stage (one 32 KB copy of the query blocks, 8 MMAs
+  // per barrier round trip) when two such stages and two raw stages fit
+  L.chunks = (size_t)2 * kTcChunks * kStageBytes + (size_t)2 * kRawBytes <= avail ? kTcChunks : 1;
+  int ns = L.chunks > 1 ? 2 : 4, nr = 2;
+  while ((size_t)ns * L.chunks * kStageBytes + (size_t)nr * kRawBytes > avail) {
     if (ns > 2) {
       --ns;
     } else if (nr > 1) {
@@ -208,7 +212,7 @@ inline TcLayout tc_layout(int width, int k) {
   }
   L.ns = ns;
   L.nr = nr;
-  L.raw_off = (size_t)ns * kStageBytes;
+  L.raw_off = (size_t)ns * L.chunks * kStageBytes;
   L.lists_off = L.raw_off + (size_t)nr * kRawBytes;
   L.cbuf_off = L.lists_off + lists;
   L.cc_off = L.cbuf_off + cbuf;
@@ -218,7 +222,7 @@ inline TcLayout tc_layout(int width, int k) {
 }
 
 struct TcGeom {
-  int ns, nr;
+  int ns, nr, chunks;  // MMA stages, raw stages, 32-wide K chunks per MMA stage
   int raw_off, lists_off, cbuf_off, cc_off, bar_off;
 };
 
@@ -229,7 +233,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   // 1024-byte alignment for the swizzled tiles (address bits drive the swizzle)
   const uint32_t base_u32 = smem_u32(tc_smem_raw);
   uint8_t *smem = tc_smem_raw + (((base_u32 + 1023u) & ~1023u) - base_u32);
-  const int ns = g.ns, nr = g.nr;
+  const int ns = g.ns, nr = g.nr, C = g.chunks;
+  const size_t stage_stride = (size_t)C * kStageBytes;  // [C query blocks][C code blocks]
   uint8_t *raw_ring = smem + g.raw_off;
   uint64_t *lists = reinterpret_cast<uint64_t *>(smem + g.lists_off);
   uint2 *cbuf = reinterpret_cast<uint2 *>(smem + g.cbuf_off);
@@ -292,7 +297,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       bool ok = true;
       for (int lt = 0; lt < ntl && ok; ++lt) {
         const int tile = (int)(tb + lt);
-        for (int kc = 0; kc < nk; ++kc, ++it) {
+        for (int kc = 0; kc < nk; ++kc) {
           if (kc % R == 0) {
             const int rs = gr % nr, rr = gr / nr;
             if (rr > 0 && !mbar_wait(&rempty[rs], (rr - 1) & 1, abort_flag, a.gflags)) {
@@ -304,15 +309,17 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                         tile * kBN, &rfull[rs]);
             r_issued = ++gr;
           }
+          if (kc % C != 0) continue;  // the stage's query blocks came with its first chunk
           const int s = it % ns, r = it / ns;
+          const int nc = nk - kc < C ? nk - kc : C;
           if (r > 0 && !mbar_wait(&empty[s], (r - 1) & 1, abort_flag, a.gflags)) {
             ok = false;
             break;
           }
-          mbar_arrive_expect_tx(&afull[s], kAStage);
-          bulk_g2s(smem + (size_t)s * kStageBytes, qA + ((size_t)qb * nk + kc) * kAStage, kAStage,
-                   &afull[s]);
-          a_issued = it + 1;
+          mbar_arrive_expect_tx(&afull[s], (uint32_t)nc * kAStage);
+          bulk_g2s(smem + (size_t)s * stage_stride, qA + ((size_t)qb * nk + kc) * kAStage,
+                   (uint32_t)nc * kAStage, &afull[s]);
+          a_issued = ++it;
         }
       }
       for (int t = max(0, a_issued - ns); t < a_issued; ++t) drain_wait_tc(&afull[t % ns], (t / ns) & 1);
@@ -328,22 +335,26 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         if (u > 0 && !mbar_wait(&acce[buf], (u - 1) & 1, abort_flag, a.gflags)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(buf * kBN);
-        for (int kc = 0; kc < nk; ++kc, ++it) {
+        for (int kc = 0; kc < nk; kc += C, ++it) {
           const int s = it % ns, r = it / ns;
+          const int nc = nk - kc < C ? nk - kc : C;
           if (!mbar_wait(&afull[s], r & 1, abort_flag, a.gflags) ||
               !mbar_wait(&conv[s], r & 1, abort_flag, a.gflags)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t st = smem_u32(smem + (size_t)s * kStageBytes);
-          const uint64_t ahi = desc_sw64(st), alo = desc_sw64(st + kABytes),
-                         bd = desc_sw64(st + kAStage);
+          const uint32_t st = smem_u32(smem + (size_t)s * stage_stride);
+          for (int c = 0; c < nc; ++c) {
+            const uint64_t ahi = desc_sw64(st + c * kAStage),
+                           alo = desc_sw64(st + c * kAStage + kABytes),
+                           bd = desc_sw64(st + C * kAStage + c * kB16Bytes);
 #pragma unroll
-          for (int j = 0; j < kBK / kUmmaK; ++j) {
-            const uint64_t koff = (uint64_t)((j * kUmmaK * 2) >> 4);
-            umma_f16(d_tmem, ahi + koff, bd + koff, kIdesc, (kc > 0 || j > 0) ? 1u : 0u);
-            umma_f16(d_tmem, alo + koff, bd + koff, kIdesc, 1u);
+            for (int j = 0; j < kBK / kUmmaK; ++j) {
+              const uint64_t koff = (uint64_t)((j * kUmmaK * 2) >> 4);
+              umma_f16(d_tmem, ahi + koff, bd + koff, kIdesc, (kc + c > 0 || j > 0) ? 1u : 0u);
+              umma_f16(d_tmem, alo + koff, bd + koff, kIdesc, 1u);
+            }
           }
           umma_commit(&empty[s]);
         }
@@ -365,19 +376,20 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       float ccp[kTasks];
 #pragma unroll
       for (int i = 0; i < kTasks; ++i) ccp[i] = 0.0f;
-      for (int kc = 0; kc < nk; ++kc, ++it) {
+      for (int kc = 0; kc < nk; ++kc) {
         const int rs = gr % nr;
         if (kc % R == 0 && !mbar_wait(&rfull[rs], (gr / nr) & 1, abort_flag, a.gflags)) {
           ok = false;
           break;
         }
         const int s = it % ns, r = it / ns;
-        if (r > 0 && !mbar_wait(&empty[s], (r - 1) & 1, abort_flag, a.gflags)) {
+        if (kc % C == 0 && r > 0 && !mbar_wait(&empty[s], (r - 1) & 1, abort_flag, a.gflags)) {
           ok = false;
           break;
         }
         const uint8_t *__restrict__ raw = raw_ring + (size_t)rs * kRawBytes;
-        uint8_t *__restrict__ b16 = smem + (size_t)s * kStageBytes + kAStage;
+        uint8_t *__restrict__ b16 =
+            smem + (size_t)s * stage_stride + (size_t)C * kAStage + (size_t)(kc % C) * kB16Bytes;
         const int j0 = (kc % R) * (kBK * W / 16);  // first 16-byte chunk of this K slice
         // All loads first: the stores below could alias them as far as the
         // compiler knows, which would otherwise serialise the tasks.
@@ -432,8 +444,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             if (need_cc) ccp[i] += c2;
           }
         }
-        fence_proxy_async_smem();
-        mbar_arrive(&conv[s]);
+        if (kc % C == C - 1 || kc == nk - 1) {  // the stage's chunks are all converted
+          fence_proxy_async_smem();
+          mbar_arrive(&conv[s]);
+          ++it;
+        }
         if (kc % R == R - 1 || kc == nk - 1) {
           mbar_arrive(&rempty[rs]);
           ++gr;
@@ -1368,6 +1383,7 @@ cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st, const RowPt
     TcGeom g;
     g.ns = L.ns;
     g.nr = L.nr;
+    g.chunks = L.chunks;
     g.raw_off = (int)L.raw_off;
     g.lists_off = (int)L.lists_off;
     g.cbuf_off = (int)L.cbuf_off;
