@@ -161,6 +161,23 @@ __device__ __forceinline__ float tile_score(int metric, float acc, float fq, flo
   return fmaf(fq, acc, qq + rowf);
 }
 
+// k > 32 heaps: candidates that beat the heap root are buffered per query
+// (cbn slots per query in shared memory, stride kBM) and poured into the heaps
+// when one query's buffer is full, so the lanes of a warp sift together
+// instead of one at a time (sparse candidates otherwise leave 31 lanes idle
+// for every insertion).
+__device__ __forceinline__ void heap_pour(uint64_t *lists, int k, const uint64_t *hb, int m,
+                                          int &cnt, float &thr_s, bool desc) {
+  for (int i = 0; i < cnt; ++i) {
+    const uint64_t key = hb[(size_t)i * kBM + m];
+    if (key < lists[m]) heap_replace_root(lists, k, kBM, m, key);
+  }
+  cnt = 0;
+  const uint64_t root = lists[m];
+  thr_s = root == kSentinel ? (desc ? -INFINITY : INFINITY)
+                            : rank_key32_score((uint32_t)(root >> 32), desc);
+}
+
 __device__ __forceinline__ float warp_sum_tc(float v) {
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
@@ -186,15 +203,24 @@ struct TcLayout {
   size_t raw_off, lists_off, cbuf_off, cc_off, bar_off, smem_bytes;
 };
 
-// Shared memory: [MMA stages][raw stages][k > 32: per-query lists | k <= 32:
-// candidate buffers][c^2 per row, 2 tiles][barriers, TMEM slot, abort flag].
+// Shared memory: [MMA stages][raw stages][k > 32: per-query heaps][candidate
+// buffers][c^2 per row, 2 tiles][barriers, TMEM slot, abort flag].  The heaps'
+// buffers take up to kCBuf slots per query, as many as leave room for two
+// single-chunk MMA stages and one raw stage (the kernel reads the depth back
+// from the offsets).
 inline TcLayout tc_layout(int width, int k) {
   (void)width;
   TcLayout L;
   const size_t lists = k > 32 ? (size_t)kBM * k * 8 : 0;
-  const size_t cbuf = k > 32 ? 0 : (size_t)kCBuf * kBM * 8;
   const size_t cc = 2 * kBN * 4;
   const size_t tailb = 64 * 8 + 1024;  // barriers, slots, alignment slack
+  size_t cbuf = (size_t)kCBuf * kBM * 8;
+  if (k > 32) {
+    const size_t room = kMaxDynSmem - lists - cc - tailb;
+    const size_t need = 2 * (size_t)kStageBytes + kRawBytes;
+    const size_t slots = room > need ? (room - need) / ((size_t)kBM * 8) : 0;
+    cbuf = (slots < (size_t)kCBuf ? slots : (size_t)kCBuf) * kBM * 8;
+  }
   const size_t avail = kMaxDynSmem - lists - cbuf - cc - tailb;
   // two K chunks per MMA stage (one 32 KB copy of the query blocks, 8 MMAs
   // per barrier round trip) when two such stages and two raw stages fit
@@ -501,6 +527,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     float thr_s = desc ? -INFINITY : INFINITY;  // score of the k-th best so far
     float seed = desc ? -INFINITY : INFINITY;   // admission bound before the list fills
     int cnt = 0;                                // buffered candidates of this query
+    // k > 32: the heaps' candidate buffers (depth from the layout)
+    uint64_t *hb = reinterpret_cast<uint64_t *>(cbuf);
+    const int hbn = KR == 0 ? (g.cc_off - g.cbuf_off) / (kBM * 8) : 0;
+    int hcnt = 0;
     if (KR == 0)
       for (int i = 0; i < k; ++i) lists[(size_t)i * kBM + m] = kSentinel;
     for (int lt = 0; lt < ntl; ++lt) {
@@ -583,17 +613,32 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           }
           if (!qvalid || nvalid <= 0) mask = 0;
           else if (nvalid < 32) mask &= (1u << nvalid) - 1u;
-          while (mask != 0) {
-            const int j = __ffs(mask) - 1;
-            mask &= mask - 1;
-            const float rf = need_cc ? ccbuf[buf * kBN + c * 32 + j] : 0.0f;
-            const float sc = tile_score(a.metric, __uint_as_float(select32(v, j)), fq, qq, rf);
-            const uint64_t key = make_key(sc, (uint32_t)(row0 + c * 32 + j), desc);
-            if (key < lists[m]) {
-              heap_replace_root(lists, k, kBM, m, key);
-              const uint64_t root = lists[m];
-              thr_s = root == kSentinel ? (desc ? -INFINITY : INFINITY)
-                                        : rank_key32_score((uint32_t)(root >> 32), desc);
+          if (hbn > 0) {
+            while (__any_sync(0xffffffffu, mask != 0)) {
+              if (mask != 0) {
+                const int j = __ffs(mask) - 1;
+                mask &= mask - 1;
+                const float rf = need_cc ? ccbuf[buf * kBN + c * 32 + j] : 0.0f;
+                const float sc =
+                    tile_score(a.metric, __uint_as_float(select32(v, j)), fq, qq, rf);
+                const uint64_t key = make_key(sc, (uint32_t)(row0 + c * 32 + j), desc);
+                if (key < lists[m]) hb[(size_t)(hcnt++) * kBM + m] = key;
+              }
+              if (__any_sync(0xffffffffu, hcnt == hbn)) heap_pour(lists, k, hb, m, hcnt, thr_s, desc);
+            }
+          } else {
+            while (mask != 0) {
+              const int j = __ffs(mask) - 1;
+              mask &= mask - 1;
+              const float rf = need_cc ? ccbuf[buf * kBN + c * 32 + j] : 0.0f;
+              const float sc = tile_score(a.metric, __uint_as_float(select32(v, j)), fq, qq, rf);
+              const uint64_t key = make_key(sc, (uint32_t)(row0 + c * 32 + j), desc);
+              if (key < lists[m]) {
+                heap_replace_root(lists, k, kBM, m, key);
+                const uint64_t root = lists[m];
+                thr_s = root == kSentinel ? (desc ? -INFINITY : INFINITY)
+                                          : rank_key32_score((uint32_t)(root >> 32), desc);
+              }
             }
           }
         }
@@ -611,6 +656,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         for (int i = 0; i < RK; ++i)
           if (i >= RK - k) out[i - (RK - k)] = ((uint64_t)reg.key[i] << 32) | reg.id[i];
       } else {
+        if (hcnt > 0) heap_pour(lists, k, hb, m, hcnt, thr_s, desc);
         heap_sort_ascending(lists, k, kBM, m);
         for (int i = 0; i < k; ++i) out[i] = lists[(size_t)i * kBM + m];
       }
@@ -906,8 +952,14 @@ inline Tc2Layout tc2_layout(int k) {
   // shared memory; stages of kTc2Chunks chunks while two of them fit beside
   // the heaps, else single-chunk stages)
   const size_t lists = k > 32 ? (size_t)kBM * k * 8 : 0;
-  const size_t cbuf = 0;
   const size_t tailb = 64 * 8 + 1024;
+  size_t cbuf = 0;  // k > 32: the heaps' candidate buffers (as in the stage-loop kernel)
+  if (k > 32) {
+    const size_t room = kMaxDynSmem - lists - tailb;
+    const size_t need = 2 * (size_t)kStageBytes;
+    const size_t slots = room > need ? (room - need) / ((size_t)kBM * 8) : 0;
+    cbuf = (slots < (size_t)kCBuf ? slots : (size_t)kCBuf) * kBM * 8;
+  }
   const size_t avail = kMaxDynSmem - lists - cbuf - tailb;
   L.chunks = avail / ((size_t)kTc2Chunks * kStageBytes) >= 2 ? kTc2Chunks : 1;
   int ns = (int)(avail / ((size_t)L.chunks * kStageBytes));
@@ -1120,6 +1172,10 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
       const float t = g.seed[qidx];
       seed = desc ? nextafterf(t, -INFINITY) : nextafterf(t, INFINITY);
     }
+    // k > 32: the heaps' candidate buffers (depth from the layout)
+    uint64_t *hb = reinterpret_cast<uint64_t *>(smem + g.cbuf_off);
+    const int hbn = KR == 0 ? (g.bar_off - g.cbuf_off) / (kBM * 8) : 0;
+    int hcnt = 0;
     if (KR == 0)
       for (int i = 0; i < k; ++i) lists[(size_t)i * kBM + m] = kSentinel;
     for (int lt = 0; lt < ntl; ++lt) {
@@ -1212,6 +1268,21 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
             const uint32_t tk = reg.key[RK - 1];
             thr_s = tk == 0xffffffffu ? (desc ? -INFINITY : INFINITY) : rank_key32_score(tk, desc);
           }
+        } else if (hbn > 0) {
+          while (__any_sync(0xffffffffu, mask != 0)) {
+            const int j = mask != 0 ? __ffs(mask) - 1 : 0;
+            const RowFac<RC> rfc = RC ? rl.at(j, l2) : rl;
+            const float rf = RC ? 0.0f : __shfl_sync(0xffffffffu, rfl, j);
+            if (mask != 0) {
+              mask &= mask - 1;
+              const float sc = RC ? fac_score(rfc, __uint_as_float(select32(v, j)), qf)
+                                  : tile_score(a.metric, __uint_as_float(select32(v, j)), fq,
+                                               qq, rf);
+              const uint64_t key = make_key(sc, grow0 + j, desc);
+              if (key < lists[m]) hb[(size_t)(hcnt++) * kBM + m] = key;
+            }
+            if (__any_sync(0xffffffffu, hcnt == hbn)) heap_pour(lists, k, hb, m, hcnt, thr_s, desc);
+          }
         } else {
           while (__any_sync(0xffffffffu, mask != 0)) {
             const int j = mask != 0 ? __ffs(mask) - 1 : 0;
@@ -1242,6 +1313,7 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
         for (int i = 0; i < RK; ++i)
           if (i >= RK - k) out[i - (RK - k)] = ((uint64_t)reg.key[i] << 32) | reg.id[i];
       } else {
+        if (hcnt > 0) heap_pour(lists, k, hb, m, hcnt, thr_s, desc);
         heap_sort_ascending(lists, k, kBM, m);
         for (int i = 0; i < k; ++i) out[i] = lists[(size_t)i * kBM + m];
       }
