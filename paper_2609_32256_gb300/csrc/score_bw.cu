@@ -67,6 +67,16 @@ __device__ __forceinline__ float warp_max(float v) {
   return v;
 }
 
+// Power of two that brings the largest |q| near 1, so that a query's squared
+// norm neither underflows nor overflows in fp32 while it is summed (the norm
+// itself is then rescaled exactly).
+__device__ __forceinline__ float norm_scale(float mx) {
+  if (!(mx > 0.0f) || !isfinite(mx)) return 1.0f;
+  int ex;
+  frexpf(mx, &ex);
+  return ldexpf(1.0f, max(-126, min(126, -ex)));
+}
+
 // Sums a over the lanes 0-15 and b over the lanes 16-31 with one shared
 // butterfly: lanes 0-15 end with sum(a), lanes 16-31 with sum(b).
 __device__ __forceinline__ float pair_sum(float a, float b, int lane) {
@@ -174,8 +184,24 @@ __global__ void __launch_bounds__(kBwThreads, 1)
           part = fmaf(v0, v0, fmaf(v1, v1, part));
         }
       }
-      qq[q] = warp_sum(part);
-      qn[q] = sqrtf(qq[q]);
+      // the norm from the scaled query (range-safe), then ||q||^2
+      float mx = 0.0f;
+#pragma unroll
+      for (int j = 0; j < kNchMax; ++j)
+#pragma unroll
+        for (int t = 0; t < 4; ++t)
+          mx = fmaxf(mx, fmaxf(fabsf(qreg[q][j][t].x), fabsf(qreg[q][j][t].y)));
+      const float ns = norm_scale(warp_max(mx));
+      part = 0.0f;
+#pragma unroll
+      for (int j = 0; j < kNchMax; ++j)
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+          const float u0 = qreg[q][j][t].x * ns, u1 = qreg[q][j][t].y * ns;
+          part = fmaf(u0, u0, fmaf(u1, u1, part));
+        }
+      qn[q] = sqrtf(warp_sum(part)) / ns;
+      qq[q] = qn[q] * qn[q];
     }
     // int8 codes: the query as signed base-256 digits of round(q 2^e) with
     // max|q| 2^e in [2^21, 2^22), so that the products with the codes are
@@ -437,8 +463,24 @@ __global__ void __launch_bounds__(kBwThreads, 1)
           sum += v0 + v1;
         }
       }
-      qq[q] = warp_sum(part);
-      qn[q] = sqrtf(qq[q]);
+      // the norm from the scaled query (range-safe), then ||q||^2
+      float mx = 0.0f;
+#pragma unroll
+      for (int j = 0; j < kNchMax; ++j)
+#pragma unroll
+        for (int t = 0; t < 4; ++t)
+          mx = fmaxf(mx, fmaxf(fabsf(qreg[q][j][t].x), fabsf(qreg[q][j][t].y)));
+      const float ns = norm_scale(warp_max(mx));
+      part = 0.0f;
+#pragma unroll
+      for (int j = 0; j < kNchMax; ++j)
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+          const float u0 = qreg[q][j][t].x * ns, u1 = qreg[q][j][t].y * ns;
+          part = fmaf(u0, u0, fmaf(u1, u1, part));
+        }
+      qn[q] = sqrtf(warp_sum(part)) / ns;
+      qq[q] = qn[q] * qn[q];
       qs[q] = warp_sum(sum);
     }
     uint32_t qdig[FMT == LAM_ROWS_INT8 ? QB : 1][FMT == LAM_ROWS_INT8 ? kNchMax : 1][3][2];
@@ -703,8 +745,11 @@ __global__ void __launch_bounds__(kGenWarps * 32) score_generic_kernel(ScoreArgs
   uint64_t thr = kSentinel;
 
   float part = 0.0f;
-  for (int d = lane; d < D; d += 32) part = fmaf(q[d], q[d], part);
-  const float qq = warp_sum(part), qn = sqrtf(qq);
+  float mx = 0.0f;
+  for (int d = lane; d < D; d += 32) mx = fmaxf(mx, fabsf(q[d]));
+  const float ns = norm_scale(warp_max(mx));
+  for (int d = lane; d < D; d += 32) part = fmaf(q[d] * ns, q[d] * ns, part);
+  const float qn = sqrtf(warp_sum(part)) / ns, qq = qn * qn;
   const bool desc = a.metric != LAM_METRIC_L2;
   // per-row codecs score the decoded rows themselves (unit step)
   const float s = a.fmt ? 1.0f : a.s, s2 = s * s;

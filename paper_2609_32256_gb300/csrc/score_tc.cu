@@ -688,28 +688,32 @@ __device__ __forceinline__ void qprep_block(const float *__restrict__ q, int64_t
   float4 *qinfo = reinterpret_cast<float4 *>(qA + (size_t)(Bpad / kBM) * nk * kAStage);
   const bool valid = b < B;
   const float *qr = q + b * D;
-  float mx = 0.0f, qq = 0.0f, qs = 0.0f;
+  float mx = 0.0f, qs = 0.0f;
   if (valid) {
     for (int d = lane; d < D; d += 32) {
       const float v = qr[d];
       mx = fmaxf(mx, fabsf(v));
-      qq = fmaf(v, v, qq);
       qs += v;
     }
   }
   for (int off = 16; off > 0; off >>= 1) {
     mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-    qq += __shfl_xor_sync(0xffffffffu, qq, off);
     qs += __shfl_xor_sync(0xffffffffu, qs, off);
   }
-  int e = 0;
+  int e = 0, ex = 0;
   if (mx > 0.0f) {
-    int ex;
     frexpf(mx, &ex);  // mx = f * 2^ex, f in [0.5, 1)
     e = 15 - ex;      // mx * 2^e in [2^14, 2^15)
     e = max(-126, min(126, e));
   }
   const float sc = ldexpf(1.0f, e);
+  // ||q|| from the query scaled near 1 (no under- or overflow of the squares)
+  const float ns = mx > 0.0f ? ldexpf(1.0f, max(-126, min(126, -ex))) : 1.0f;
+  float ss = 0.0f;
+  if (valid)
+    for (int d = lane; d < D; d += 32) ss = fmaf(qr[d] * ns, qr[d] * ns, ss);
+  for (int off = 16; off > 0; off >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, off);
+  const float qn = sqrtf(ss) / ns, qq = qn * qn;
   // lane writes whole 16-byte chunks (8 fp16) of the hi and lo images
   for (int ch = lane; ch < nk * (kBK / 8); ch += 32) {
     const int d0 = ch * 8, kc = d0 / kBK, c16 = (d0 % kBK) / 8;
@@ -731,7 +735,7 @@ __device__ __forceinline__ void qprep_block(const float *__restrict__ q, int64_t
     *reinterpret_cast<uint4 *>(qA + off + kABytes) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
   }
   if (lane == 0)
-    qinfo[b] = valid ? make_float4(ldexpf(1.0f, -e), sqrtf(qq), qq, qs)
+    qinfo[b] = valid ? make_float4(ldexpf(1.0f, -e), qn, qq, qs)
                      : make_float4(0.f, 0.f, 0.f, 0.f);
 }
 

@@ -211,3 +211,18 @@ def test_tensor_k128_needs_the_conversion_pass(dev, score_path):
     q = inputs.queries(520, 768, seed=128)
     for metric in METRICS:
         check(dev, q, codes, 1, 1e-2, 128, metric, bound)
+
+
+@pytest.mark.parametrize("path", ["bandwidth", "tensor", "generic"])
+@pytest.mark.parametrize("qscale", [1e-30, 1e-3, 1e20])
+def test_query_scale_extremes(dev, score_path, path, qscale):
+    """Queries far from unit norm: the integer-digit (int8, bandwidth) and
+    split-fp16 (tensor) encodings of the query rescale by a power of two, so
+    inner-product and cosine scores keep their relative accuracy."""
+    score_path(path)
+    codes, bound = make_codes(1500, 768, 1e-2, 1, seed=31)
+    B = 2 if path == "bandwidth" else 130
+    q = (inputs.queries(B, 768, seed=32).astype(np.float64) * qscale).astype(np.float32)
+    q[1, 5:] = 0.0  # one query with a few coordinates only
+    for metric in (oracle.IP, oracle.COSINE):
+        check(dev, q, codes, 1, 1e-2, 10, metric, bound)
