@@ -204,6 +204,54 @@ lam_status lam_lamz_decompress(const void *in, size_t in_bytes, float *out, int6
                                lam_stream_t stream);
 
 /*
+ * Device-resident form of the same steps, for pipelines that must not wait
+ * for the host: lam_quantize_async queues Q_eps exactly as lam_quantize
+ * computes it (same codes, same AUTO width) but reads nothing back.  The
+ * outcome stays in the workspace's 32-byte status block: the width, the code
+ * range, the errors.  lam_dequantize_from and lam_score_topk_from take the
+ * codes' width from that block on the device, so quantize -> dequantize ->
+ * search can be queued back to back on streams (or captured in a CUDA graph)
+ * with no host round trip; lam_quantize_result reads the block when the host
+ * needs it.
+ *
+ * lam_quantize_async: arguments as for lam_quantize without the host
+ *   outputs.  AUTO writes the codes at the narrowest width; when the width
+ *   it speculated from a sample was too narrow, a second pass on the device
+ *   rewrites them (the codes buffer must hold n times that width).  A forced
+ *   width too narrow for the codes is recorded as a range error.  Keep the
+ *   workspace (and codes) alive and unchanged until their consumers ran.
+ *   Asynchronous.  Errors now: LAM_ERR_INVALID, LAM_ERR_WORKSPACE (workspace
+ *   below 32 bytes, or codes_bytes < n * forced width), LAM_ERR_CUDA.
+ * lam_quantize_result: waits for `stream` and decodes the status block of
+ *   the workspace as lam_quantize reports it (same eps and width_req as the
+ *   call; outputs and errors as for lam_quantize).
+ * lam_dequantize_from: xhat = fl32(2 eps * code) at the width in the status
+ *   block `quant_workspace` (codes and out 4-byte aligned).  Nothing is
+ *   written when the status holds an error.  Asynchronous.
+ * lam_score_topk_from: lam_score_topk with the width and validity taken from
+ *   `quant_workspace` (widths 1 and 2; eps the quantizer's).  The path is
+ *   chosen without the width, from shapes that both widths take; the tensor
+ *   cores take int16 codes up to +-2048 only, larger ones give LAM_ERR_RANGE
+ *   from lam_score_topk_status.  A status with an error, or width 4, gives
+ *   LAM_ERR_UNSUPPORTED there (the scores are then undefined).  Workspace
+ *   size and path queries as for lam_score_topk.  Asynchronous.
+ */
+lam_status lam_quantize_async(const float *x, int64_t n, float eps, int32_t width_req,
+                              void *codes, size_t codes_bytes, void *workspace,
+                              size_t workspace_bytes, lam_stream_t stream);
+lam_status lam_quantize_result(const void *workspace, float eps, int32_t width_req,
+                               lam_stream_t stream, int32_t *width_out, float *scale_out,
+                               int32_t *code_min_out, int32_t *code_max_out);
+lam_status lam_dequantize_from(const void *codes, const void *quant_workspace, int64_t n,
+                               float eps, float *out, lam_stream_t stream);
+size_t lam_score_topk_from_workspace_size(int64_t B, int64_t N, int32_t D, int32_t k);
+int32_t lam_score_topk_from_path(int64_t B, int64_t N, int32_t D, int32_t k);
+lam_status lam_score_topk_from(const float *queries, int64_t B, const void *codes,
+                               const void *quant_workspace, int64_t N, int32_t D, float eps,
+                               int32_t k, int32_t metric, float *scores, int64_t *ids,
+                               void *workspace, size_t workspace_bytes, lam_stream_t stream);
+
+/*
  * lam_dequantize -- xhat_i = fl32(scale * code_i), the inverse map of Q_eps
  * up to the cell half-width eps (|x - xhat| <= eps, Sec. 3.1).
  *

@@ -22,7 +22,10 @@ from ._lib import (LAM_ERR_CUDA, LAM_ERR_INVALID, LAM_ERR_NONFINITE, LAM_ERR_RAN
                    lam_lamz_bound, lam_lamz_compress, lam_lamz_decompress,
                    lam_lamz_workspace_size, LAM_ROWS_INT8, LAM_ROWS_FP16, LAM_ROWS_SIGN,
                    lam_encode_rows, lam_decode_rows, lam_score_topk_rows,
-                   lam_score_topk_rows_path, lam_score_topk_rows_workspace_size)
+                   lam_score_topk_rows_path, lam_score_topk_rows_workspace_size,
+                   lam_quantize_async, lam_quantize_result, lam_dequantize_from,
+                   lam_score_topk_from, lam_score_topk_from_path,
+                   lam_score_topk_from_workspace_size)
 
 CODE_DTYPES = {1: "int8", 2: "int16", 4: "int32"}
 

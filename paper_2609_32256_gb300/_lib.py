@@ -66,6 +66,13 @@ def load():
                                   P(ctypes.c_double), P(i64), P(i64), vp]),
         "lam_quantize_bands": (i32, [vp, i64, i32, f32, i32, i32, vp, sz, vp, vp, sz, P(i32),
                                      P(f32), P(i32), P(i32), vp]),
+        "lam_quantize_async": (i32, [vp, i64, f32, i32, vp, sz, vp, sz, vp]),
+        "lam_quantize_result": (i32, [vp, f32, i32, vp, P(i32), P(f32), P(i32), P(i32)]),
+        "lam_dequantize_from": (i32, [vp, vp, i64, f32, vp, vp]),
+        "lam_score_topk_from_workspace_size": (sz, [i64, i64, i32, i32]),
+        "lam_score_topk_from_path": (i32, [i64, i64, i32, i32]),
+        "lam_score_topk_from": (i32, [vp, i64, vp, vp, i64, i32, f32, i32, i32, vp, vp, vp, sz,
+                                      vp]),
         "lam_encode_rows": (i32, [vp, i64, i32, i32, vp, vp, vp, vp]),
         "lam_decode_rows": (i32, [vp, i32, i64, i32, vp, vp, vp, vp]),
         "lam_score_topk_rows_workspace_size": (sz, [i64, i64, i32, i32, i32]),
@@ -162,6 +169,53 @@ def lam_score_topk(queries, codes, width, N, D, eps, code_bound, k, metric, scor
                                _ptr(scores), _ptr(ids), _ptr(workspace), _nbytes(workspace),
                                _stream(stream, queries.device))
     _check(st, "lam_score_topk")
+
+
+def lam_quantize_async(x, eps, width_req, codes, workspace, stream=None):
+    """Q_eps of x queued on the stream; the outcome stays in `workspace`."""
+    st = load().lam_quantize_async(_ptr(x), x.numel(), ctypes.c_float(eps), int(width_req),
+                                   _ptr(codes), _nbytes(codes), _ptr(workspace),
+                                   _nbytes(workspace), _stream(stream, x.device))
+    _check(st, "lam_quantize_async")
+
+
+def lam_quantize_result(workspace, eps, width_req=LAM_WIDTH_AUTO, stream=None,
+                        raise_on_error=True):
+    """(status, width, scale, code_min, code_max) of an asynchronous Q_eps."""
+    w = ctypes.c_int32(0)
+    s = ctypes.c_float(0)
+    cmin = ctypes.c_int32(0)
+    cmax = ctypes.c_int32(0)
+    st = load().lam_quantize_result(_ptr(workspace), ctypes.c_float(eps), int(width_req),
+                                    _stream(stream, workspace.device), ctypes.byref(w),
+                                    ctypes.byref(s), ctypes.byref(cmin), ctypes.byref(cmax))
+    if raise_on_error and st != LAM_OK:
+        raise LamError(st, "lam_quantize_result")
+    return int(st), w.value, s.value, cmin.value, cmax.value
+
+
+def lam_dequantize_from(codes, quant_workspace, n, eps, out, stream=None):
+    st = load().lam_dequantize_from(_ptr(codes), _ptr(quant_workspace), int(n),
+                                    ctypes.c_float(eps), _ptr(out), _stream(stream, out.device))
+    _check(st, "lam_dequantize_from")
+
+
+def lam_score_topk_from_workspace_size(B, N, D, k) -> int:
+    return int(load().lam_score_topk_from_workspace_size(int(B), int(N), int(D), int(k)))
+
+
+def lam_score_topk_from_path(B, N, D, k) -> int:
+    return int(load().lam_score_topk_from_path(int(B), int(N), int(D), int(k)))
+
+
+def lam_score_topk_from(queries, codes, quant_workspace, N, D, eps, k, metric, scores, ids,
+                        workspace, stream=None):
+    B = queries.shape[0]
+    st = load().lam_score_topk_from(_ptr(queries), int(B), _ptr(codes), _ptr(quant_workspace),
+                                    int(N), int(D), ctypes.c_float(eps), int(k), int(metric),
+                                    _ptr(scores), _ptr(ids), _ptr(workspace), _nbytes(workspace),
+                                    _stream(stream, queries.device))
+    _check(st, "lam_score_topk_from")
 
 
 LAM_ROWS_INT8, LAM_ROWS_FP16, LAM_ROWS_SIGN = 1, 2, 3

@@ -125,6 +125,36 @@ bool make_plan(int64_t B, int64_t N, int32_t D, int32_t k, int32_t width, int32_
   return true;
 }
 
+// Status-driven search (codes' width on the device, 1 or 2): the path cannot
+// depend on the width, so each test holds for both.
+bool make_from_plan(int64_t B, int64_t N, int32_t D, int32_t k, int sms, Plan *p) {
+  if (!shape_ok(B, N, D, k, 2, 0) || sms <= 0) return false;
+  const bool bw = bandwidth_ok(B, D, k, 1) && bandwidth_ok(B, D, k, 2);
+  const bool tc = D % 16 == 0 && tensor_fits(1, k, B) && tensor_fits(2, k, B) &&
+                  B <= (1LL << 23);
+  const int f = forced_path();
+  if (f == -2) return false;
+  int path = bw ? kPathBandwidth : tc ? kPathTensor : kPathGeneric;
+  if (f >= 0) {
+    if ((f == kPathBandwidth && !bw) || (f == kPathTensor && !tc)) {
+      p->path = -2;
+      return false;
+    }
+    path = f;
+  }
+  p->path = path;
+  p->n_lists = path == kPathBandwidth ? bandwidth_ctas(N, D, 2, sms)
+               : path == kPathTensor  ? tensor_plan(B, N, D, k, sms).n_lists
+                                      : generic_ctas(B, N, sms);
+  p->Bpad = (B + 127) / 128 * 128;
+  p->partial_off = kHeaderBytes;
+  const size_t partial = (size_t)p->n_lists * (size_t)B * (size_t)k * 8;
+  p->qprep_off = align_up(p->partial_off + partial, 256);
+  p->total = p->qprep_off;
+  if (path == kPathTensor) p->total += align_up(tensor_plan(B, N, D, k, sms).bytes, 256);
+  return true;
+}
+
 // Per-row codecs: shape checks and the plan (tensor path with the converting
 // pass, else the generic path; no bandwidth kernel).
 bool rows_shape_ok(int64_t B, int64_t N, int32_t D, int32_t k, int32_t fmt) {
@@ -746,12 +776,164 @@ lam_status lam_score_topk_rows(const float *queries, int64_t B, const void *code
   return LAM_OK;
 }
 
+lam_status lam_quantize_async(const float *x, int64_t n, float eps, int32_t width_req, void *codes,
+                              size_t codes_bytes, void *workspace, size_t workspace_bytes,
+                              lam_stream_t stream) {
+  if (n < 0 || n >= (1LL << 62) || !valid_eps(eps)) return LAM_ERR_INVALID;
+  if (width_req != LAM_WIDTH_AUTO && !valid_width(width_req)) return LAM_ERR_INVALID;
+  if (n > 0 && x == nullptr) return LAM_ERR_INVALID;
+  if ((reinterpret_cast<uintptr_t>(x) & 3u) != 0) return LAM_ERR_INVALID;
+  const uintptr_t calign = width_req == LAM_WIDTH_AUTO ? 4u : (uintptr_t)width_req;
+  if (codes != nullptr && (reinterpret_cast<uintptr_t>(codes) & (calign - 1)) != 0)
+    return LAM_ERR_INVALID;
+  if (workspace == nullptr || (reinterpret_cast<uintptr_t>(workspace) & 15u) != 0)
+    return LAM_ERR_INVALID;
+  if (workspace_bytes < sizeof(QuantStatus)) return LAM_ERR_WORKSPACE;
+  if (codes != nullptr && width_req != LAM_WIDTH_AUTO &&
+      (unsigned long long)n * (unsigned long long)width_req > codes_bytes)
+    return LAM_ERR_WORKSPACE;
+  const int sms = device_sms();
+  if (sms <= 0) return LAM_ERR_CUDA;
+  const float s = 2.0f * eps;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  QuantStatus *dst = static_cast<QuantStatus *>(workspace);
+  if (cudaMemsetAsync(dst, 0, sizeof(QuantStatus), st) != cudaSuccess) return LAM_ERR_CUDA;
+  cudaError_t e = cudaSuccess;
+  if (n > 0) {
+    timing_launch_begin(LAM_TIME_QUANTIZE, st);
+    if (width_req == LAM_WIDTH_AUTO) e = launch_quantize_auto(x, n, s, codes, codes_bytes, dst, sms, st);
+    else if (codes != nullptr) e = launch_quantize(x, n, s, width_req, codes, codes_bytes, dst, sms, st);
+    else e = launch_quant_range(x, n, dst, sms, st);
+    timing_launch_end(LAM_TIME_QUANTIZE, st);
+    if (e != cudaSuccess) return LAM_ERR_CUDA;
+  }
+  // settle on the device: the forced width and its range check, or AUTO's
+  // second pass (n == 0: the width alone)
+  timing_launch_begin(LAM_TIME_AUX, st);
+  e = launch_quantize_settle(x, n, s, width_req, codes, codes_bytes, dst, sms, st);
+  timing_launch_end(LAM_TIME_AUX, st);
+  return e == cudaSuccess ? LAM_OK : LAM_ERR_CUDA;
+}
+
+lam_status lam_quantize_result(const void *workspace, float eps, int32_t width_req,
+                               lam_stream_t stream, int32_t *width_out, float *scale_out,
+                               int32_t *code_min_out, int32_t *code_max_out) {
+  if (workspace == nullptr || !valid_eps(eps)) return LAM_ERR_INVALID;
+  if (width_req != LAM_WIDTH_AUTO && !valid_width(width_req)) return LAM_ERR_INVALID;
+  QuantStatus h;
+  if (read_back(&h, workspace, sizeof(h), reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess)
+    return LAM_ERR_CUDA;
+  return lam::decode_quant_status(h, width_req, 2.0f * eps, width_out, scale_out, code_min_out,
+                                  code_max_out);
+}
+
+lam_status lam_dequantize_from(const void *codes, const void *quant_workspace, int64_t n,
+                               float eps, float *out, lam_stream_t stream) {
+  if (n < 0 || !valid_eps(eps)) return LAM_ERR_INVALID;
+  if (n == 0) return LAM_OK;
+  if (codes == nullptr || out == nullptr || quant_workspace == nullptr) return LAM_ERR_INVALID;
+  // any width may come back: 4-byte alignment covers them all
+  if ((reinterpret_cast<uintptr_t>(codes) & 3u) != 0 ||
+      (reinterpret_cast<uintptr_t>(out) & 3u) != 0 ||
+      (reinterpret_cast<uintptr_t>(quant_workspace) & 15u) != 0)
+    return LAM_ERR_INVALID;
+  const int sms = device_sms();
+  if (sms <= 0) return LAM_ERR_CUDA;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  timing_launch_begin(LAM_TIME_DEQUANTIZE, st);
+  const cudaError_t e = launch_dequantize_from(
+      codes, static_cast<const QuantStatus *>(quant_workspace), n, 2.0f * eps, out, sms, st);
+  timing_launch_end(LAM_TIME_DEQUANTIZE, st);
+  return e == cudaSuccess ? LAM_OK : LAM_ERR_CUDA;
+}
+
+size_t lam_score_topk_from_workspace_size(int64_t B, int64_t N, int32_t D, int32_t k) {
+  Plan p;
+  const int sms = device_sms();
+  if (!make_from_plan(B, N, D, k, sms, &p)) return 0;
+  const size_t generic = align_up(kHeaderBytes + (size_t)generic_ctas(B, N, sms) * B * k * 8, 256);
+  return p.total > generic ? p.total : generic;
+}
+
+int32_t lam_score_topk_from_path(int64_t B, int64_t N, int32_t D, int32_t k) {
+  Plan p;
+  if (!make_from_plan(B, N, D, k, device_sms(), &p)) return -1;
+  return p.path;
+}
+
+lam_status lam_score_topk_from(const float *queries, int64_t B, const void *codes,
+                               const void *quant_workspace, int64_t N, int32_t D, float eps,
+                               int32_t k, int32_t metric, float *scores, int64_t *ids,
+                               void *workspace, size_t workspace_bytes, lam_stream_t stream) {
+  if (queries == nullptr || codes == nullptr || quant_workspace == nullptr || scores == nullptr ||
+      ids == nullptr || workspace == nullptr)
+    return LAM_ERR_INVALID;
+  if (metric != LAM_METRIC_IP && metric != LAM_METRIC_COSINE && metric != LAM_METRIC_L2)
+    return LAM_ERR_INVALID;
+  if (!valid_eps(eps) || !shape_ok(B, N, D, k, 2, 0)) return LAM_ERR_INVALID;
+  if ((reinterpret_cast<uintptr_t>(workspace) & 255u) != 0 ||
+      (reinterpret_cast<uintptr_t>(quant_workspace) & 15u) != 0)
+    return LAM_ERR_INVALID;
+  if ((reinterpret_cast<uintptr_t>(codes) & 1u) != 0 ||
+      (reinterpret_cast<uintptr_t>(queries) & 3u) != 0 ||
+      (reinterpret_cast<uintptr_t>(scores) & 3u) != 0 || (reinterpret_cast<uintptr_t>(ids) & 7u) != 0)
+    return LAM_ERR_INVALID;
+  const int sms = device_sms();
+  if (sms <= 0) return LAM_ERR_CUDA;
+  Plan p;
+  if (!make_from_plan(B, N, D, k, sms, &p))
+    return p.path == -2 ? LAM_ERR_UNSUPPORTED : LAM_ERR_INVALID;
+  const bool aligned = (reinterpret_cast<uintptr_t>(codes) & 15u) == 0;
+  if (!aligned && p.path != kPathGeneric) {
+    if (forced_path() >= 0) return LAM_ERR_UNSUPPORTED;
+    p.path = kPathGeneric;
+    p.n_lists = generic_ctas(B, N, sms);
+    p.qprep_off = align_up(p.partial_off + (size_t)p.n_lists * B * k * 8, 256);
+    p.total = p.qprep_off;
+  }
+  if (workspace_bytes < p.total) return LAM_ERR_WORKSPACE;
+
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  uint8_t *ws = static_cast<uint8_t *>(workspace);
+  if (cudaMemsetAsync(ws, 0, kHeaderBytes, st) != cudaSuccess) return LAM_ERR_CUDA;
+  ScoreArgs a;
+  a.queries = queries;
+  a.B = B;
+  a.codes = codes;
+  a.width = 1;  // unused: the kernels take the width from the status
+  a.N = N;
+  a.D = D;
+  a.s = 2.0f * eps;
+  a.code_bound = 0;
+  a.k = k;
+  a.metric = metric;
+  a.scores = scores;
+  a.ids = ids;
+  a.gflags = reinterpret_cast<uint32_t *>(ws);
+  a.partial = reinterpret_cast<uint64_t *>(ws + p.partial_off);
+  a.n_lists = p.n_lists;
+  a.qprep = ws + p.qprep_off;
+  a.Bpad = p.Bpad;
+  a.sms = sms;
+  RowPtrs rp;
+  rp.qst = static_cast<const QuantStatus *>(quant_workspace);
+  ScoreArgs m = a;  // the final merge's lists
+  cudaError_t e;
+  if (p.path == kPathBandwidth) e = launch_score_bandwidth(a, st, rp.qst);
+  else if (p.path == kPathTensor) e = launch_score_tensor(a, st, rp, &m);
+  else e = launch_score_generic(a, st, rp);
+  if (e != cudaSuccess) return LAM_ERR_CUDA;
+  if (launch_topk_merge(m, st, rp) != cudaSuccess) return LAM_ERR_CUDA;
+  return LAM_OK;
+}
+
 lam_status lam_score_topk_status(const void *workspace, lam_stream_t stream, int32_t *status_out) {
   if (workspace == nullptr || status_out == nullptr) return LAM_ERR_INVALID;
   uint32_t flags = 0;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   if (read_back(&flags, workspace, 4, st) != cudaSuccess) return LAM_ERR_CUDA;
   if (flags & kFlagTimeout) *status_out = LAM_ERR_TIMEOUT;
+  else if (flags & kFlagInput) *status_out = LAM_ERR_UNSUPPORTED;
   else if (flags & kFlagRange) *status_out = LAM_ERR_RANGE;
   else *status_out = LAM_OK;
   return LAM_OK;

@@ -16,6 +16,8 @@ constexpr uint32_t kFlagNonfinite = 1u;   // quantize: NaN/Inf seen
 constexpr uint32_t kFlagRange = 2u;       // codes beyond a width / code bound
 constexpr uint32_t kFlagWorkspace = 4u;   // codes buffer too small (AUTO)
 constexpr uint32_t kFlagTimeout = 8u;     // a bounded wait gave up
+constexpr uint32_t kFlagInput = 16u;      // the codes' quantize status reports an error
+                                          // or a width the call does not take
 
 constexpr int kMaxK = 1024;
 constexpr int kHeaderBytes = 256;         // status block at the head of a workspace
@@ -178,6 +180,13 @@ cudaError_t launch_dequantize(const void *codes, int width, int64_t n, float s, 
 cudaError_t launch_quantize_auto(const float *x, int64_t n, float s, void *codes,
                                  size_t codes_bytes, QuantStatus *status, int sms,
                                  cudaStream_t st);
+// Asynchronous quantization: settles the status on the device after the AUTO
+// or forced kernel (range error for a forced width, AUTO's second pass).
+cudaError_t launch_quantize_settle(const float *x, int64_t n, float s, int width_req, void *codes,
+                                   size_t codes_bytes, QuantStatus *status, int sms,
+                                   cudaStream_t st);
+cudaError_t launch_dequantize_from(const void *codes, const QuantStatus *status, int64_t n,
+                                   float s, float *out, int sms, cudaStream_t st);
 
 struct ScoreArgs {
   const float *queries;
@@ -204,11 +213,27 @@ struct ScoreArgs {
   int fmt = 0;
 };
 
-// Per-row factors of a per-row codec, passed beside ScoreArgs.
+// Per-row factors of a per-row codec, passed beside ScoreArgs; for the
+// status-driven calls (lam_score_topk_from) the quantize status that holds
+// the codes' width (a.width is then ignored).
 struct RowPtrs {
   const float *scale = nullptr;
   const float *offset = nullptr;
+  const QuantStatus *qst = nullptr;
 };
+
+// A quantize status that finished without error.
+__device__ __forceinline__ bool status_ok(const QuantStatus *st) {
+  const uint32_t f = *(volatile const uint32_t *)&st->flags;
+  return !(f & (kFlagNonfinite | kFlagRange | kFlagWorkspace | kFlagTimeout));
+}
+__device__ __forceinline__ uint32_t status_width(const QuantStatus *st) {
+  return *(volatile const uint32_t *)&st->width;
+}
+// Width of the codes: from the status when there is one.
+__device__ __forceinline__ int codes_width(const ScoreArgs &a, const RowPtrs &rp) {
+  return rp.qst != nullptr ? (int)status_width(rp.qst) : a.width;
+}
 
 // Decoded value xhat_d of row `row` of a per-row codec, evaluated exactly as
 // lam_decode_rows writes it.
@@ -229,7 +254,9 @@ cudaError_t launch_encode_rows(const float *x, int64_t N, int D, int fmt, void *
 cudaError_t launch_decode_rows(const void *codes, int fmt, int64_t N, int D, const float *scale,
                                const float *offset, float *out, int sms, cudaStream_t st);
 
-cudaError_t launch_score_bandwidth(const ScoreArgs &a, cudaStream_t st);
+// `qst` (status-driven calls): the codes' width is read on the device.
+cudaError_t launch_score_bandwidth(const ScoreArgs &a, cudaStream_t st,
+                                   const QuantStatus *qst = nullptr);
 // Per-vector codecs, B <= 2: row bytes (D, 2D or D/8) a multiple of 16, D <= 1024, k <= 128.
 cudaError_t launch_score_bandwidth_rows(const ScoreArgs &a, const RowPtrs &rp, cudaStream_t st);
 int bandwidth_rows_ctas(int64_t N, int fmt, int D, int sms);

@@ -294,9 +294,8 @@ __global__ void __launch_bounds__(kThreads) quantize_auto_kernel(
 }
 
 template <int W, bool VEC>
-__global__ void __launch_bounds__(kThreads) dequantize_kernel(const void *__restrict__ codes,
-                                                              int64_t n, float s,
-                                                              float *__restrict__ out) {
+__device__ __forceinline__ void dequantize_body(const void *__restrict__ codes, int64_t n, float s,
+                                                float *__restrict__ out) {
   const int64_t tid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   int64_t done = 0;
@@ -333,6 +332,61 @@ __global__ void __launch_bounds__(kThreads) dequantize_kernel(const void *__rest
     else c = reinterpret_cast<const int32_t *>(codes)[i];
     out[i] = __fmul_rn(s, (float)c);
   }
+}
+
+template <int W, bool VEC>
+__global__ void __launch_bounds__(kThreads) dequantize_kernel(const void *__restrict__ codes,
+                                                              int64_t n, float s,
+                                                              float *__restrict__ out) {
+  dequantize_body<W, VEC>(codes, n, s, out);
+}
+
+// Status-driven forms (lam_quantize_async and its consumers): the width comes
+// from the quantize status block on the device, so no host round trip sits
+// between quantizing and using the codes.
+template <bool VEC>
+__global__ void __launch_bounds__(kThreads) dequantize_from_kernel(const void *__restrict__ codes,
+                                                                   int64_t n, float s,
+                                                                   const QuantStatus *st,
+                                                                   float *__restrict__ out) {
+  if (!status_ok(st)) return;
+  const uint32_t w = *(volatile const uint32_t *)&st->width;
+  if (w == 1) dequantize_body<1, VEC>(codes, n, s, out);
+  else if (w == 2) dequantize_body<2, VEC>(codes, n, s, out);
+  else if (w == 4) dequantize_body<4, VEC>(codes, n, s, out);
+}
+
+// Settles an asynchronous quantization on the device.  Forced width: one
+// thread records the width and flags a range error when the exact range
+// needs a wider type.  AUTO:
+// the AUTO kernel resolved the width; when its speculation was too narrow
+// (passes == 2) every block quantizes again at the resolved width.
+template <bool VEC>
+__global__ void __launch_bounds__(kThreads) quantize_settle_kernel(
+    const float *__restrict__ x, int64_t n, float s, void *__restrict__ codes,
+    unsigned long long codes_bytes, int width_req, QuantStatus *st) {
+  if (n == 0) {  // nothing was quantized: the width alone
+    if (blockIdx.x == 0 && threadIdx.x == 0)
+      st->width = width_req != LAM_WIDTH_AUTO ? (uint32_t)width_req : 1u;
+    return;
+  }
+  const uint32_t f = *(volatile const uint32_t *)&st->flags;
+  if (width_req != LAM_WIDTH_AUTO) {
+    if (blockIdx.x == 0 && threadIdx.x == 0) st->width = (uint32_t)width_req;
+    if (blockIdx.x == 0 && threadIdx.x == 0 && !(f & (kFlagNonfinite | kFlagTimeout))) {
+      const int need = width_of_range(*(volatile const uint32_t *)&st->neg_min,
+                                      *(volatile const uint32_t *)&st->max, s);
+      if (need == 0 || need > width_req) atomicOr(&st->flags, kFlagRange);
+    }
+    return;
+  }
+  if (f & (kFlagNonfinite | kFlagRange | kFlagWorkspace | kFlagTimeout)) return;
+  if (*(volatile const uint32_t *)&st->passes != 2u || codes == nullptr) return;
+  const uint32_t w = *(volatile const uint32_t *)&st->width;
+  if ((unsigned long long)n * w > codes_bytes) return;
+  if (w == 1) quantize_body<1, true, VEC>(x, n, s, codes, st);
+  else if (w == 2) quantize_body<2, true, VEC>(x, n, s, codes, st);
+  else if (w == 4) quantize_body<4, true, VEC>(x, n, s, codes, st);
 }
 
 // One warp per code row: exact int64 sum of squares, rounded once to fp32.
@@ -416,6 +470,26 @@ cudaError_t launch_quantize_auto(const float *x, int64_t n, float s, void *codes
   auto kern = vec ? quantize_auto_kernel<true> : quantize_auto_kernel<false>;
   const unsigned long long cb = codes_bytes;
   kern<<<grid_for(kern, vec ? n / 4 + 1 : n, sms), kThreads, 0, st>>>(x, n, s, codes, cb, status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_quantize_settle(const float *x, int64_t n, float s, int width_req, void *codes,
+                                   size_t codes_bytes, QuantStatus *status, int sms,
+                                   cudaStream_t st) {
+  const bool vec = aligned16(x) && (codes == nullptr || aligned16(codes));
+  auto kern = vec ? quantize_settle_kernel<true> : quantize_settle_kernel<false>;
+  unsigned grid = width_req == LAM_WIDTH_AUTO && n > 0 ? grid_for(kern, vec ? n / 4 + 1 : n, sms) : 1;
+  if (grid < 1) grid = 1;
+  kern<<<grid, kThreads, 0, st>>>(x, n, s, codes, (unsigned long long)codes_bytes, width_req,
+                                  status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_dequantize_from(const void *codes, const QuantStatus *status, int64_t n,
+                                   float s, float *out, int sms, cudaStream_t st) {
+  const bool vec = aligned16(codes) && aligned16(out);
+  auto kern = vec ? dequantize_from_kernel<true> : dequantize_from_kernel<false>;
+  kern<<<grid_for(kern, vec ? n / 4 + 1 : n, sms), kThreads, 0, st>>>(codes, n, s, status, out);
   return cudaGetLastError();
 }
 

@@ -117,7 +117,9 @@ inline BwShape bw_shape(int D, int width) {
 
 template <int W, int QB, int KPL, bool CC>
 __global__ void __launch_bounds__(kBwThreads, 1)
-    score_bw_kernel(ScoreArgs a, int tr, int ns, int stage_bytes) {
+    score_bw_kernel(ScoreArgs a, int tr, int ns, int stage_bytes, const QuantStatus *qst) {
+  // status-driven call: only the variant of the codes' width runs
+  if (qst != nullptr && (!status_ok(qst) || status_width(qst) != (uint32_t)W)) return;
   extern __shared__ __align__(1024) uint8_t smem[];
   uint64_t *full = reinterpret_cast<uint64_t *>(smem + (size_t)ns * stage_bytes);
   uint64_t *empty = full + ns;
@@ -733,6 +735,8 @@ __device__ __forceinline__ int32_t load_code(const void *codes, int width, int64
 }
 
 __global__ void __launch_bounds__(kGenWarps * 32) score_generic_kernel(ScoreArgs a, RowPtrs rp) {
+  const int width = codes_width(a, rp);
+  if (rp.qst != nullptr && (!status_ok(rp.qst) || (width != 1 && width != 2))) return;
   extern __shared__ __align__(16) uint8_t gsmem[];
   uint64_t *lists = reinterpret_cast<uint64_t *>(gsmem);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -760,7 +764,7 @@ __global__ void __launch_bounds__(kGenWarps * 32) score_generic_kernel(ScoreArgs
     float acc = 0.0f, cc = 0.0f;
     const int64_t base = row * D;
     for (int d = lane; d < D; d += 32) {
-      const float c = a.fmt ? row_value(a, rp, row, d) : (float)load_code(a.codes, a.width, base + d);
+      const float c = a.fmt ? row_value(a, rp, row, d) : (float)load_code(a.codes, width, base + d);
       acc = fmaf(q[d], c, acc);
       cc = fmaf(c, c, cc);
     }
@@ -810,6 +814,11 @@ __device__ void bitonic_sort(uint64_t *buf, int P) {
 
 __global__ void __launch_bounds__(kMergeThreads) topk_merge_kernel(ScoreArgs a, int P,
                                                                    RowPtrs rp) {
+  if (rp.qst != nullptr && (!status_ok(rp.qst) || (status_width(rp.qst) != 1 &&
+                                                   status_width(rp.qst) != 2))) {
+    if (blockIdx.x == 0 && threadIdx.x == 0) atomicOr(a.gflags, kFlagInput);
+    return;
+  }
   extern __shared__ __align__(16) uint8_t msmem[];
   uint64_t *buf = reinterpret_cast<uint64_t *>(msmem);
   const int64_t b = blockIdx.x;
@@ -850,7 +859,7 @@ __global__ void __launch_bounds__(kMergeThreads) topk_merge_kernel(ScoreArgs a, 
       if (row < a.N) {
         for (int d = lane; d < a.D; d += 32) {
           const float xh = a.fmt ? row_value(a, rp, row, d)
-                                 : __fmul_rn(a.s, (float)load_code(a.codes, a.width,
+                                 : __fmul_rn(a.s, (float)load_code(a.codes, codes_width(a, rp),
                                                                    (int64_t)row * a.D + d));
           const float df = __fsub_rn(q[d], xh);
           acc = fmaf(df, df, acc);
@@ -885,6 +894,11 @@ constexpr int kKmWarps = 8;
 template <int HPL>
 __global__ void __launch_bounds__(kKmWarps * 32) topk_kmerge_kernel(ScoreArgs a, int qpc,
                                                                     RowPtrs rp) {
+  if (rp.qst != nullptr && (!status_ok(rp.qst) || (status_width(rp.qst) != 1 &&
+                                                   status_width(rp.qst) != 2))) {
+    if (blockIdx.x == 0 && threadIdx.x == 0) atomicOr(a.gflags, kFlagInput);
+    return;
+  }
   extern __shared__ __align__(16) uint8_t ksmem[];
   const int L = a.n_lists, k = a.k;
   uint64_t *cand = reinterpret_cast<uint64_t *>(ksmem);            // [qpc][L][k]
@@ -958,7 +972,7 @@ __global__ void __launch_bounds__(kKmWarps * 32) topk_kmerge_kernel(ScoreArgs a,
 #pragma unroll 4
         for (int d = lane; d < a.D; d += 32) {
           const float xh = a.fmt ? row_value(a, rp, row, d)
-                                 : __fmul_rn(a.s, (float)load_code(a.codes, a.width,
+                                 : __fmul_rn(a.s, (float)load_code(a.codes, codes_width(a, rp),
                                                                    (int64_t)row * a.D + d));
           const float df = __fsub_rn(q[d], xh);
           acc = fmaf(df, df, acc);
@@ -1117,30 +1131,40 @@ int generic_ctas(int64_t B, int64_t N, int sms) {
 }
 
 template <int W, int QB, int KPL>
-static cudaError_t launch_bw_t(const ScoreArgs &a, const BwShape &sh, cudaStream_t st) {
+static cudaError_t launch_bw_t(const ScoreArgs &a, const BwShape &sh, const QuantStatus *qst,
+                               cudaStream_t st) {
   const size_t smem = (size_t)sh.ns * sh.stage_bytes + 2 * sh.ns * sizeof(uint64_t) + 16;
   auto kern = a.metric == LAM_METRIC_IP ? score_bw_kernel<W, QB, KPL, false>
                                         : score_bw_kernel<W, QB, KPL, true>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   timing_launch_begin(LAM_TIME_SCORE, st);
-  kern<<<a.n_lists, kBwThreads, smem, st>>>(a, sh.tr, sh.ns, sh.stage_bytes);
+  kern<<<a.n_lists, kBwThreads, smem, st>>>(a, sh.tr, sh.ns, sh.stage_bytes, qst);
   timing_launch_end(LAM_TIME_SCORE, st);
   return cudaGetLastError();
 }
 
 template <int W, int QB>
-static cudaError_t launch_bw_k(const ScoreArgs &a, const BwShape &sh, cudaStream_t st) {
-  if (a.k <= 32) return launch_bw_t<W, QB, 1>(a, sh, st);
-  return launch_bw_t<W, QB, 4>(a, sh, st);
+static cudaError_t launch_bw_k(const ScoreArgs &a, const BwShape &sh, const QuantStatus *qst,
+                               cudaStream_t st) {
+  if (a.k <= 32) return launch_bw_t<W, QB, 1>(a, sh, qst, st);
+  return launch_bw_t<W, QB, 4>(a, sh, qst, st);
 }
 
-cudaError_t launch_score_bandwidth(const ScoreArgs &a, cudaStream_t st) {
-  const BwShape sh = bw_shape(a.D, a.width);
+template <int W>
+static cudaError_t launch_bw_w(const ScoreArgs &a, const QuantStatus *qst, cudaStream_t st) {
+  const BwShape sh = bw_shape(a.D, W);
   // merge scratch (QB * 8 warps * k keys) must fit in the stage buffers
   if ((size_t)2 * kBwWarps * a.k * 8 > (size_t)sh.ns * sh.stage_bytes) return cudaErrorInvalidValue;
-  if (a.width == 1) return a.B == 1 ? launch_bw_k<1, 1>(a, sh, st) : launch_bw_k<1, 2>(a, sh, st);
-  return a.B == 1 ? launch_bw_k<2, 1>(a, sh, st) : launch_bw_k<2, 2>(a, sh, st);
+  return a.B == 1 ? launch_bw_k<W, 1>(a, sh, qst, st) : launch_bw_k<W, 2>(a, sh, qst, st);
+}
+
+cudaError_t launch_score_bandwidth(const ScoreArgs &a, cudaStream_t st, const QuantStatus *qst) {
+  if (qst != nullptr) {  // width on the device: both variants, one runs
+    const cudaError_t e = launch_bw_w<1>(a, qst, st);
+    return e != cudaSuccess ? e : launch_bw_w<2>(a, qst, st);
+  }
+  return a.width == 1 ? launch_bw_w<1>(a, nullptr, st) : launch_bw_w<2>(a, nullptr, st);
 }
 
 template <int FMT, int QB, int KPL>

@@ -250,11 +250,14 @@ inline TcLayout tc_layout(int width, int k) {
 struct TcGeom {
   int ns, nr, chunks;  // MMA stages, raw stages, 32-wide K chunks per MMA stage
   int raw_off, lists_off, cbuf_off, cc_off, bar_off;
+  const QuantStatus *qst;  // status-driven calls: the codes' width is read here
 };
 
 template <int W, int KR>
 __global__ void __launch_bounds__(kTcThreads, 1)
     score_tc_kernel(const __grid_constant__ CUtensorMap cmap, ScoreArgs a, TcGeom g) {
+  // status-driven call: only the variant of the codes' width runs
+  if (g.qst != nullptr && (!status_ok(g.qst) || status_width(g.qst) != (uint32_t)W)) return;
   extern __shared__ uint8_t tc_smem_raw[];
   // 1024-byte alignment for the swizzled tiles (address bits drive the swizzle)
   const uint32_t base_u32 = smem_u32(tc_smem_raw);
@@ -813,13 +816,20 @@ __device__ __forceinline__ void convert_block(const void *__restrict__ codes, in
   if (W == 2 && amax > 2048.0f) atomicOr(gflags, kFlagRange);
 }
 
+// (qst: status-driven calls launch both widths; only the codes' width converts)
+__device__ __forceinline__ bool width_gate(const QuantStatus *qst, int W) {
+  return qst == nullptr || (status_ok(qst) && status_width(qst) == (uint32_t)W);
+}
+
 template <int W>
 __global__ void __launch_bounds__(256) convert_codes_kernel(const void *__restrict__ codes,
                                                             int64_t row_base, int64_t nrows,
                                                             int64_t nrows_pad, int D,
                                                             uint8_t *__restrict__ out,
                                                             float *__restrict__ rowf, int metric,
-                                                            float s, uint32_t *gflags) {
+                                                            float s, uint32_t *gflags,
+                                                            const QuantStatus *qst) {
+  if (!width_gate(qst, W)) return;
   convert_block<W>(codes, row_base, nrows, nrows_pad, D, out, rowf, metric, s, gflags, blockIdx.x);
 }
 
@@ -829,10 +839,11 @@ template <int W>
 __global__ void __launch_bounds__(256) prep_convert_kernel(
     const float *__restrict__ q, int64_t B, int D, int64_t Bpad, uint8_t *__restrict__ qA,
     unsigned q_blocks, const void *__restrict__ codes, int64_t nrows, int64_t nrows_pad,
-    uint8_t *__restrict__ out, float *__restrict__ rowf, int metric, float s, uint32_t *gflags) {
+    uint8_t *__restrict__ out, float *__restrict__ rowf, int metric, float s, uint32_t *gflags,
+    const QuantStatus *qst) {
   if (blockIdx.x < q_blocks)
     qprep_block(q, B, D, Bpad, qA, blockIdx.x);
-  else
+  else if (width_gate(qst, W))
     convert_block<W>(codes, 0, nrows, nrows_pad, D, out, rowf, metric, s, gflags,
                      blockIdx.x - q_blocks);
 }
@@ -1435,7 +1446,9 @@ cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st, const RowPt
                                 ScoreArgs *merge) {
   if (merge != nullptr) *merge = a;
   const bool rc = a.fmt != 0;
-  if (a.k > kTcMaxK || (!rc && a.width != 1 && a.width != 2)) return cudaErrorInvalidValue;
+  // status-driven call (codes' width on the device): both widths launch, one works
+  const QuantStatus *qst = rc ? nullptr : rp.qst;
+  if (a.k > kTcMaxK || (!rc && !qst && a.width != 1 && a.width != 2)) return cudaErrorInvalidValue;
   const TensorPlan P = tensor_plan(a.B, a.N, a.D, a.k, a.sms, rc);
   if (P.n_lists != a.n_lists) return cudaErrorInvalidValue;
   uint8_t *qA = static_cast<uint8_t *>(a.qprep);
@@ -1450,13 +1463,18 @@ cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st, const RowPt
     if (e != cudaSuccess) return e;
     const TcLayout L = tc_layout(a.width, a.k);
     if (L.ns < 2) return cudaErrorInvalidValue;
-    CUtensorMap cmap;
-    if (!make_map_2d(&cmap,
-                     a.width == 1 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_UINT16,
-                     a.codes, (uint64_t)a.D, (uint64_t)a.N, (uint64_t)a.D * a.width,
-                     (uint32_t)(kRawRow / a.width), kBN, CU_TENSOR_MAP_SWIZZLE_128B))
+    CUtensorMap cmap1, cmap2;  // the codes as int8 and as int16 rows
+    if ((qst || a.width == 1) &&
+        !make_map_2d(&cmap1, CU_TENSOR_MAP_DATA_TYPE_UINT8, a.codes, (uint64_t)a.D, (uint64_t)a.N,
+                     (uint64_t)a.D, (uint32_t)kRawRow, kBN, CU_TENSOR_MAP_SWIZZLE_128B))
+      return cudaErrorInvalidValue;
+    if ((qst || a.width == 2) &&
+        !make_map_2d(&cmap2, CU_TENSOR_MAP_DATA_TYPE_UINT16, a.codes, (uint64_t)a.D,
+                     (uint64_t)a.N, (uint64_t)a.D * 2, (uint32_t)(kRawRow / 2), kBN,
+                     CU_TENSOR_MAP_SWIZZLE_128B))
       return cudaErrorInvalidValue;
     TcGeom g;
+    g.qst = qst;
     g.ns = L.ns;
     g.nr = L.nr;
     g.chunks = L.chunks;
@@ -1466,7 +1484,7 @@ cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st, const RowPt
     g.cc_off = (int)L.cc_off;
     g.bar_off = (int)L.bar_off;
     const dim3 grid((unsigned)a.n_lists, (unsigned)(a.Bpad / kBM));
-    auto run = [&](auto kern) -> cudaError_t {
+    auto run = [&](auto kern, const CUtensorMap &cmap) -> cudaError_t {
       cudaError_t r = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                            (int)L.smem_bytes);
       if (r != cudaSuccess) return r;
@@ -1475,14 +1493,21 @@ cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st, const RowPt
       timing_launch_end(LAM_TIME_SCORE, st);
       return cudaGetLastError();
     };
-    if (a.width == 1) {
-      if (a.k <= 16) return run(score_tc_kernel<1, 16>);
-      if (a.k <= 32) return run(score_tc_kernel<1, 32>);
-      return run(score_tc_kernel<1, 0>);
+    auto run1 = [&]() -> cudaError_t {
+      if (a.k <= 16) return run(score_tc_kernel<1, 16>, cmap1);
+      if (a.k <= 32) return run(score_tc_kernel<1, 32>, cmap1);
+      return run(score_tc_kernel<1, 0>, cmap1);
+    };
+    auto run2 = [&]() -> cudaError_t {
+      if (a.k <= 16) return run(score_tc_kernel<2, 16>, cmap2);
+      if (a.k <= 32) return run(score_tc_kernel<2, 32>, cmap2);
+      return run(score_tc_kernel<2, 0>, cmap2);
+    };
+    if (qst) {
+      e = run1();
+      return e != cudaSuccess ? e : run2();
     }
-    if (a.k <= 16) return run(score_tc_kernel<2, 16>);
-    if (a.k <= 32) return run(score_tc_kernel<2, 32>);
-    return run(score_tc_kernel<2, 0>);
+    return a.width == 1 ? run1() : run2();
   }
 
   // two or more query blocks: convert each slab once, then the pure MMA kernel
@@ -1538,20 +1563,25 @@ cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st, const RowPt
       else
         conv(prep_convert_rows_kernel<LAM_ROWS_SIGN>, convert_rows_kernel<LAM_ROWS_SIGN>);
     } else if (j == 0) {  // the first slab's conversion shares a launch with the query prep
-      if (a.width == 1)
+      // (status-driven: the int8 launch also prepares the queries, the int16
+      // one only converts; whichever matches the codes' width does the work)
+      if (qst || a.width == 1)
         prep_convert_kernel<1><<<q_blocks + cg, 256, 0, st>>>(
             a.queries, a.B, a.D, a.Bpad, qA, q_blocks, a.codes, nrows, nrows_pad, f16, rowf,
-            a.metric, a.s, a.gflags);
-      else
-        prep_convert_kernel<2><<<q_blocks + cg, 256, 0, st>>>(
-            a.queries, a.B, a.D, a.Bpad, qA, q_blocks, a.codes, nrows, nrows_pad, f16, rowf,
-            a.metric, a.s, a.gflags);
-    } else if (a.width == 1) {
-      convert_codes_kernel<1><<<cg, 256, 0, st>>>(a.codes, row_base, nrows, nrows_pad, a.D, f16,
-                                                  rowf, a.metric, a.s, a.gflags);
+            a.metric, a.s, a.gflags, qst);
+      if (qst || a.width == 2) {
+        const unsigned qb2 = qst ? 0u : q_blocks;
+        prep_convert_kernel<2><<<qb2 + cg, 256, 0, st>>>(
+            a.queries, a.B, a.D, a.Bpad, qA, qb2, a.codes, nrows, nrows_pad, f16, rowf,
+            a.metric, a.s, a.gflags, qst);
+      }
     } else {
-      convert_codes_kernel<2><<<cg, 256, 0, st>>>(a.codes, row_base, nrows, nrows_pad, a.D, f16,
-                                                  rowf, a.metric, a.s, a.gflags);
+      if (qst || a.width == 1)
+        convert_codes_kernel<1><<<cg, 256, 0, st>>>(a.codes, row_base, nrows, nrows_pad, a.D,
+                                                    f16, rowf, a.metric, a.s, a.gflags, qst);
+      if (qst || a.width == 2)
+        convert_codes_kernel<2><<<cg, 256, 0, st>>>(a.codes, row_base, nrows, nrows_pad, a.D,
+                                                    f16, rowf, a.metric, a.s, a.gflags, qst);
     }
     timing_launch_end(LAM_TIME_AUX, st);
     e = cudaGetLastError();

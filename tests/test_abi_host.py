@@ -221,3 +221,31 @@ def test_score_rows_rejects_bad_arguments(lib):
         assert call(**bad) == 1, bad
     assert lib.lam_score_topk_rows_workspace_size(4, 100, 32, 10, 9) == 0
     assert lib.lam_score_topk_rows_path(4, 100, 20, 10, 3) == -1
+
+
+def test_async_calls_reject_bad_arguments(lib):
+    c = ctypes
+    v = c.c_void_p
+    # quantize: bad eps, bad width, null workspace, misaligned workspace
+    assert lib.lam_quantize_async(v(1024), 16, c.c_float(0.0), 0, v(2048), 64, v(4096), 256,
+                                  None) == 1
+    assert lib.lam_quantize_async(v(1024), 16, c.c_float(1e-2), 3, v(2048), 64, v(4096), 256,
+                                  None) == 1
+    assert lib.lam_quantize_async(v(1024), 16, c.c_float(1e-2), 0, v(2048), 64, None, 256,
+                                  None) == 1
+    assert lib.lam_quantize_async(v(1024), 16, c.c_float(1e-2), 0, v(2048), 64, v(4104), 256,
+                                  None) == 1
+    # result: null workspace
+    w = c.c_int32()
+    assert lib.lam_quantize_result(None, c.c_float(1e-2), 0, None, c.byref(w), None, None,
+                                   None) == 1
+    # dequantize_from: misaligned status, null codes
+    assert lib.lam_dequantize_from(v(1024), v(4104), 16, c.c_float(1e-2), v(2048), None) == 1
+    assert lib.lam_dequantize_from(None, v(4096), 16, c.c_float(1e-2), v(2048), None) == 1
+    # score_from: bad metric, null status, k > N
+    assert lib.lam_score_topk_from(v(1024), 2, v(4096), v(8192), 100, 64, c.c_float(1e-2), 10, 5,
+                                   v(16384), v(32768), v(1 << 20), 1 << 30, None) == 1
+    assert lib.lam_score_topk_from(v(1024), 2, v(4096), None, 100, 64, c.c_float(1e-2), 10, 0,
+                                   v(16384), v(32768), v(1 << 20), 1 << 30, None) == 1
+    assert lib.lam_score_topk_from(v(1024), 2, v(4096), v(8192), 5, 64, c.c_float(1e-2), 10, 0,
+                                   v(16384), v(32768), v(1 << 20), 1 << 30, None) == 1
