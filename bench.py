@@ -221,6 +221,34 @@ class Pipeline:
         # search overlap the scoring kernel of the next
         self.ss2 = torch.cuda.Stream(dev)
         self.sws2 = torch.empty(wsz, dtype=torch.uint8, device=dev)
+        # device-resident pipeline: one quantize status per eps, read by the
+        # dequantisation and the search on the device
+        self.qws_e = [torch.zeros(256, dtype=torch.uint8, device=dev) for _ in eps_list]
+        fsz = lam.lam_score_topk_from_workspace_size(self.B, self.N, self.D, k)
+        self.swsf = [torch.empty(fsz, dtype=torch.uint8, device=dev) for _ in range(2)]
+
+    def step_device(self):
+        """The step with no host round trip: each eps is quantized on one
+        stream (lam_quantize_async), its dequantisation and search take the
+        width from the quantize status on the device (lam_dequantize_from,
+        lam_score_topk_from) on streams of their own; the same work and
+        results as step()."""
+        lam = self.lam
+        n = self.x.numel()
+        for j, e in enumerate(self.eps_list):
+            lam.lam_quantize_async(self.x, e, 0, self.codes_e[j], self.qws_e[j],
+                                   stream=self.sq.cuda_stream)
+            self.qdone[j].record(self.sq)
+            ss, sws = (self.ss, self.swsf[0]) if j % 2 == 0 else (self.ss2, self.swsf[1])
+            self.sd.wait_event(self.qdone[j])
+            ss.wait_event(self.qdone[j])
+            lam.lam_dequantize_from(self.codes_e[j], self.qws_e[j], n, e, self.deq,
+                                    stream=self.sd.cuda_stream)
+            lam.lam_score_topk_from(self.q, self.codes_e[j], self.qws_e[j], self.N, self.D, e,
+                                    self.k, self.metric, self.scores[j], self.ids[j], sws,
+                                    stream=ss.cuda_stream)
+        self.ss.wait_stream(self.sd)  # the step ends when all have finished
+        self.ss.wait_stream(self.ss2)
 
     def step_overlapped(self):
         """The step as a user would drive it: Q_eps of each eps on one stream
@@ -316,7 +344,7 @@ def run_lam(args):
 
     cur = torch.cuda.current_stream(dev)
 
-    def overlapped_step(i, e0, e1):
+    def overlapped_step(i, e0, e1, device=True):
         # the previous step is finished and L2 is flushed before the step starts
         pipe.sq.wait_stream(pipe.ss)
         pipe.sq.wait_stream(pipe.ss2)
@@ -325,7 +353,10 @@ def run_lam(args):
         with torch.cuda.stream(pipe.sq):
             flush(i)
         e0.record(pipe.sq)
-        pipe.step_overlapped()
+        if device:
+            pipe.step_device()
+        else:
+            pipe.step_overlapped()
         e1.record(pipe.ss)
 
     for i in range(args.warmup):
@@ -333,7 +364,17 @@ def run_lam(args):
         pipe.step()
         overlapped_step(i, torch.cuda.Event(enable_timing=True),
                         torch.cuda.Event(enable_timing=True))
+        overlapped_step(i, torch.cuda.Event(enable_timing=True),
+                        torch.cuda.Event(enable_timing=True), device=False)
     torch.cuda.synchronize(dev)
+    # the device-resident step gives the synchronous calls' results
+    overlapped_step(0, torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+    torch.cuda.synchronize(dev)
+    dev_res = [(s_.clone(), i_.clone()) for s_, i_ in zip(pipe.scores, pipe.ids)]
+    pipe.step()
+    torch.cuda.synchronize(dev)
+    for (s_d, i_d), s_, i_ in zip(dev_res, pipe.scores, pipe.ids):
+        assert torch.equal(s_d, s_) and torch.equal(i_d, i_)
 
     ne = len(wl.eps)
     step_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
@@ -342,11 +383,19 @@ def run_lam(args):
            for _ in range(args.steps)]
     barrier(world)
     torch.cuda.synchronize(dev)
+    sync_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(args.steps)]
     sampler = ClockSampler(local)
     with sampler:
-        # headline pass: the step as a user drives it (two streams)
+        # headline pass: the step as a throughput user drives it, queued with
+        # no host round trip (the width stays on the device)
         for i in range(args.steps):
             overlapped_step(i, *step_ev[i])
+        torch.cuda.synchronize(dev)
+        # the same step through the synchronous lam_quantize (the host reads
+        # each width back before it launches that eps's search)
+        for i in range(args.steps):
+            overlapped_step(i, *sync_ev[i], device=False)
         torch.cuda.synchronize(dev)
         # Second pass, every call in order on one stream: per-stage spans and,
         # from the library, CUDA events around each launch of its quantize,
@@ -380,6 +429,7 @@ def run_lam(args):
             t_s += e[2].elapsed_time(e[3])
     units_per_step = wl.n * ne
     ms_local = sum(a.elapsed_time(b) for a, b in step_ev) / args.steps
+    ms_sync = sum(a.elapsed_time(b) for a, b in sync_ev) / args.steps
     ms_step, value = aggregate_replicas(ms_local, units_per_step, world, dev)
     ms_serial = (t_q + t_d + t_s) / args.steps
 
@@ -444,7 +494,7 @@ def run_lam(args):
         with torch.cuda.stream(pipe.ss):
             q.copy_(q_h, non_blocking=True)  # ordered before the searches on this stream
         pipe.ss2.wait_stream(pipe.ss)         # and on the other search stream
-        pipe.step_overlapped()
+        pipe.step_device()
         with torch.cuda.stream(pipe.ss):
             for j in range(ne):
                 res_h[j][0].copy_(pipe.scores[j], non_blocking=True)
@@ -468,6 +518,7 @@ def run_lam(args):
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
             "ms_per_step_serial": ms_serial,
+            "ms_per_step_host_sync": ms_sync,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "f32 in, int%d codes, fp16x2-split tensor / fp32 accumulate" % (8 * max(widths)),
             "data": "synthetic (seeded unit-Gaussian rows shaped like bge-base D=768 embeddings)",
@@ -476,10 +527,13 @@ def run_lam(args):
                        "widths": widths, "paths": paths, "parallelism": "replicas only",
                        "l2": "flushed between timed steps (512 MB write then 512 MB read, outside "
                              "the events)",
-                       "step": "per eps: lam_quantize (synchronous) on one stream, lam_dequantize "
-                               "on a second and lam_score_topk on a third or fourth (alternating), "
-                               "so they overlap each other and the quantization of the next eps "
-                               "(ms_per_step_serial: all on one stream)"},
+                       "step": "per eps: lam_quantize_async (AUTO width) on one stream, "
+                               "lam_dequantize_from on a second and lam_score_topk_from on a "
+                               "third or fourth (alternating), the width read from the quantize "
+                               "status on the device, so nothing waits for the host "
+                               "(ms_per_step_host_sync: the same with the synchronous "
+                               "lam_quantize / lam_dequantize / lam_score_topk; "
+                               "ms_per_step_serial: those all on one stream)"},
             "breakdown": {
                 "quantize_ms": ms_q, "quantize_gbs_algorithmic": q_bytes / (ms_q / 1e3) / 1e9,
                 "quantize_note": "lam_quantize span: status clear + quantize + status read-back",

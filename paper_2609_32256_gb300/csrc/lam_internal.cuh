@@ -222,13 +222,17 @@ struct RowPtrs {
   const QuantStatus *qst = nullptr;
 };
 
-// A quantize status that finished without error.
+// A quantize status that finished without error.  The consumers run after
+// the quantize kernels in stream order and nothing writes the block while
+// they read it, so every thread may take it through the read-only cache (one
+// address read by every thread of a grid: a coherent load per thread would
+// queue on that one L2 line).
 __device__ __forceinline__ bool status_ok(const QuantStatus *st) {
-  const uint32_t f = *(volatile const uint32_t *)&st->flags;
+  const uint32_t f = __ldg(&st->flags);
   return !(f & (kFlagNonfinite | kFlagRange | kFlagWorkspace | kFlagTimeout));
 }
 __device__ __forceinline__ uint32_t status_width(const QuantStatus *st) {
-  return *(volatile const uint32_t *)&st->width;
+  return __ldg(&st->width);
 }
 // Width of the codes: from the status when there is one.
 __device__ __forceinline__ int codes_width(const ScoreArgs &a, const RowPtrs &rp) {

@@ -350,7 +350,7 @@ __global__ void __launch_bounds__(kThreads) dequantize_from_kernel(const void *_
                                                                    const QuantStatus *st,
                                                                    float *__restrict__ out) {
   if (!status_ok(st)) return;
-  const uint32_t w = *(volatile const uint32_t *)&st->width;
+  const uint32_t w = status_width(st);
   if (w == 1) dequantize_body<1, VEC>(codes, n, s, out);
   else if (w == 2) dequantize_body<2, VEC>(codes, n, s, out);
   else if (w == 4) dequantize_body<4, VEC>(codes, n, s, out);
@@ -370,7 +370,11 @@ __global__ void __launch_bounds__(kThreads) quantize_settle_kernel(
       st->width = width_req != LAM_WIDTH_AUTO ? (uint32_t)width_req : 1u;
     return;
   }
-  const uint32_t f = *(volatile const uint32_t *)&st->flags;
+  // (the block is read as the earlier kernels left it: in AUTO mode the
+  // second pass only re-adds the same range, in forced mode one thread reads
+  // and writes it)
+  const uint32_t f = width_req == LAM_WIDTH_AUTO ? __ldg(&st->flags)
+                                                 : *(volatile const uint32_t *)&st->flags;
   if (width_req != LAM_WIDTH_AUTO) {
     if (blockIdx.x == 0 && threadIdx.x == 0) st->width = (uint32_t)width_req;
     if (blockIdx.x == 0 && threadIdx.x == 0 && !(f & (kFlagNonfinite | kFlagTimeout))) {
@@ -381,8 +385,8 @@ __global__ void __launch_bounds__(kThreads) quantize_settle_kernel(
     return;
   }
   if (f & (kFlagNonfinite | kFlagRange | kFlagWorkspace | kFlagTimeout)) return;
-  if (*(volatile const uint32_t *)&st->passes != 2u || codes == nullptr) return;
-  const uint32_t w = *(volatile const uint32_t *)&st->width;
+  if (__ldg(&st->passes) != 2u || codes == nullptr) return;
+  const uint32_t w = __ldg(&st->width);
   if ((unsigned long long)n * w > codes_bytes) return;
   if (w == 1) quantize_body<1, true, VEC>(x, n, s, codes, st);
   else if (w == 2) quantize_body<2, true, VEC>(x, n, s, codes, st);
@@ -478,7 +482,10 @@ cudaError_t launch_quantize_settle(const float *x, int64_t n, float s, int width
                                    cudaStream_t st) {
   const bool vec = aligned16(x) && (codes == nullptr || aligned16(codes));
   auto kern = vec ? quantize_settle_kernel<true> : quantize_settle_kernel<false>;
+  // (AUTO rarely needs the second pass: one block per SM keeps the idle
+  // launch short and still streams when it does)
   unsigned grid = width_req == LAM_WIDTH_AUTO && n > 0 ? grid_for(kern, vec ? n / 4 + 1 : n, sms) : 1;
+  if (grid > (unsigned)sms) grid = (unsigned)sms;
   if (grid < 1) grid = 1;
   kern<<<grid, kThreads, 0, st>>>(x, n, s, codes, (unsigned long long)codes_bytes, width_req,
                                   status);

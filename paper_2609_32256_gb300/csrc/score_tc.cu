@@ -848,6 +848,33 @@ __global__ void __launch_bounds__(256) prep_convert_kernel(
                      blockIdx.x - q_blocks);
 }
 
+// Status-driven calls: one launch converts at the width the quantize status
+// holds (a launch per width would schedule a whole grid of idle blocks).
+__global__ void __launch_bounds__(256) convert_codes_from_kernel(
+    const void *__restrict__ codes, int64_t row_base, int64_t nrows, int64_t nrows_pad, int D,
+    uint8_t *__restrict__ out, float *__restrict__ rowf, int metric, float s, uint32_t *gflags,
+    const QuantStatus *qst) {
+  if (width_gate(qst, 1))
+    convert_block<1>(codes, row_base, nrows, nrows_pad, D, out, rowf, metric, s, gflags, blockIdx.x);
+  else if (width_gate(qst, 2))
+    convert_block<2>(codes, row_base, nrows, nrows_pad, D, out, rowf, metric, s, gflags, blockIdx.x);
+}
+
+__global__ void __launch_bounds__(256) prep_convert_from_kernel(
+    const float *__restrict__ q, int64_t B, int D, int64_t Bpad, uint8_t *__restrict__ qA,
+    unsigned q_blocks, const void *__restrict__ codes, int64_t nrows, int64_t nrows_pad,
+    uint8_t *__restrict__ out, float *__restrict__ rowf, int metric, float s, uint32_t *gflags,
+    const QuantStatus *qst) {
+  if (blockIdx.x < q_blocks)
+    qprep_block(q, B, D, Bpad, qA, blockIdx.x);
+  else if (width_gate(qst, 1))
+    convert_block<1>(codes, 0, nrows, nrows_pad, D, out, rowf, metric, s, gflags,
+                     blockIdx.x - q_blocks);
+  else if (width_gate(qst, 2))
+    convert_block<2>(codes, 0, nrows, nrows_pad, D, out, rowf, metric, s, gflags,
+                     blockIdx.x - q_blocks);
+}
+
 // Per-row codecs: the stored codes become the fp16 operand image as they are
 // (int8 codes c, fp16 values, sign bits as +-1), and the decoding moves into
 // per-row factors (u, w, z) of the score
@@ -1562,26 +1589,29 @@ cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st, const RowPt
         conv(prep_convert_rows_kernel<LAM_ROWS_FP16>, convert_rows_kernel<LAM_ROWS_FP16>);
       else
         conv(prep_convert_rows_kernel<LAM_ROWS_SIGN>, convert_rows_kernel<LAM_ROWS_SIGN>);
-    } else if (j == 0) {  // the first slab's conversion shares a launch with the query prep
-      // (status-driven: the int8 launch also prepares the queries, the int16
-      // one only converts; whichever matches the codes' width does the work)
-      if (qst || a.width == 1)
-        prep_convert_kernel<1><<<q_blocks + cg, 256, 0, st>>>(
+    } else if (qst) {  // status-driven: the width is read on the device
+      if (j == 0)
+        prep_convert_from_kernel<<<q_blocks + cg, 256, 0, st>>>(
             a.queries, a.B, a.D, a.Bpad, qA, q_blocks, a.codes, nrows, nrows_pad, f16, rowf,
             a.metric, a.s, a.gflags, qst);
-      if (qst || a.width == 2) {
-        const unsigned qb2 = qst ? 0u : q_blocks;
-        prep_convert_kernel<2><<<qb2 + cg, 256, 0, st>>>(
-            a.queries, a.B, a.D, a.Bpad, qA, qb2, a.codes, nrows, nrows_pad, f16, rowf,
-            a.metric, a.s, a.gflags, qst);
-      }
+      else
+        convert_codes_from_kernel<<<cg, 256, 0, st>>>(a.codes, row_base, nrows, nrows_pad, a.D,
+                                                      f16, rowf, a.metric, a.s, a.gflags, qst);
+    } else if (j == 0) {  // the first slab's conversion shares a launch with the query prep
+      if (a.width == 1)
+        prep_convert_kernel<1><<<q_blocks + cg, 256, 0, st>>>(
+            a.queries, a.B, a.D, a.Bpad, qA, q_blocks, a.codes, nrows, nrows_pad, f16, rowf,
+            a.metric, a.s, a.gflags, nullptr);
+      else
+        prep_convert_kernel<2><<<q_blocks + cg, 256, 0, st>>>(
+            a.queries, a.B, a.D, a.Bpad, qA, q_blocks, a.codes, nrows, nrows_pad, f16, rowf,
+            a.metric, a.s, a.gflags, nullptr);
+    } else if (a.width == 1) {
+      convert_codes_kernel<1><<<cg, 256, 0, st>>>(a.codes, row_base, nrows, nrows_pad, a.D, f16,
+                                                  rowf, a.metric, a.s, a.gflags, nullptr);
     } else {
-      if (qst || a.width == 1)
-        convert_codes_kernel<1><<<cg, 256, 0, st>>>(a.codes, row_base, nrows, nrows_pad, a.D,
-                                                    f16, rowf, a.metric, a.s, a.gflags, qst);
-      if (qst || a.width == 2)
-        convert_codes_kernel<2><<<cg, 256, 0, st>>>(a.codes, row_base, nrows, nrows_pad, a.D,
-                                                    f16, rowf, a.metric, a.s, a.gflags, qst);
+      convert_codes_kernel<2><<<cg, 256, 0, st>>>(a.codes, row_base, nrows, nrows_pad, a.D, f16,
+                                                  rowf, a.metric, a.s, a.gflags, nullptr);
     }
     timing_launch_end(LAM_TIME_AUX, st);
     e = cudaGetLastError();
