@@ -76,6 +76,8 @@ def parse():
     p.add_argument("--width", type=int, default=-1, help="(--kernels) forced code width")
     p.add_argument("--rows", type=int, default=0,
                    help="(--kernels) a smaller memory of the same workload (profiling captures)")
+    p.add_argument("--no-graph", action="store_true",
+                   help="time the device-resident step eagerly instead of replaying its CUDA graph")
     p.add_argument("--only", default="",
                    help="(--kernels) comma list of parts: quantize,bands,codec,admit,score,rows")
     return p.parse_args()
@@ -344,7 +346,9 @@ def run_lam(args):
 
     cur = torch.cuda.current_stream(dev)
 
-    def overlapped_step(i, e0, e1, device=True):
+    graph = None  # the device-resident step captured once, replayed per step
+
+    def overlapped_step(i, e0, e1, device=True, use_graph=False):
         # the previous step is finished and L2 is flushed before the step starts
         pipe.sq.wait_stream(pipe.ss)
         pipe.sq.wait_stream(pipe.ss2)
@@ -353,6 +357,11 @@ def run_lam(args):
         with torch.cuda.stream(pipe.sq):
             flush(i)
         e0.record(pipe.sq)
+        if use_graph:
+            with torch.cuda.stream(pipe.sq):
+                graph.replay()
+            e1.record(pipe.sq)
+            return
         if device:
             pipe.step_device()
         else:
@@ -367,8 +376,26 @@ def run_lam(args):
         overlapped_step(i, torch.cuda.Event(enable_timing=True),
                         torch.cuda.Event(enable_timing=True), device=False)
     torch.cuda.synchronize(dev)
+    if not args.no_graph:
+        # capture the device-resident step (its four streams fork from and
+        # join the capture stream); every replay runs all of its launches
+        gs = torch.cuda.Stream(dev)
+        gs.wait_stream(cur)
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=gs):
+            for st_ in (pipe.sq, pipe.sd, pipe.ss, pipe.ss2):
+                st_.wait_stream(gs)
+            pipe.step_device()
+            for st_ in (pipe.sq, pipe.sd, pipe.ss, pipe.ss2):
+                gs.wait_stream(st_)
+        torch.cuda.synchronize(dev)
+        for i in range(args.warmup):
+            overlapped_step(i, torch.cuda.Event(enable_timing=True),
+                            torch.cuda.Event(enable_timing=True), use_graph=True)
+        torch.cuda.synchronize(dev)
     # the device-resident step gives the synchronous calls' results
-    overlapped_step(0, torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+    overlapped_step(0, torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
+                    use_graph=graph is not None)
     torch.cuda.synchronize(dev)
     dev_res = [(s_.clone(), i_.clone()) for s_, i_ in zip(pipe.scores, pipe.ids)]
     pipe.step()
@@ -385,12 +412,19 @@ def run_lam(args):
     torch.cuda.synchronize(dev)
     sync_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
                for _ in range(args.steps)]
+    eager_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                for _ in range(args.steps)]
     sampler = ClockSampler(local)
     with sampler:
         # headline pass: the step as a throughput user drives it, queued with
-        # no host round trip (the width stays on the device)
+        # no host round trip (the width stays on the device), replayed from
+        # its CUDA graph
         for i in range(args.steps):
-            overlapped_step(i, *step_ev[i])
+            overlapped_step(i, *step_ev[i], use_graph=graph is not None)
+        torch.cuda.synchronize(dev)
+        # the same calls launched one by one
+        for i in range(args.steps):
+            overlapped_step(i, *eager_ev[i])
         torch.cuda.synchronize(dev)
         # the same step through the synchronous lam_quantize (the host reads
         # each width back before it launches that eps's search)
@@ -430,6 +464,7 @@ def run_lam(args):
     units_per_step = wl.n * ne
     ms_local = sum(a.elapsed_time(b) for a, b in step_ev) / args.steps
     ms_sync = sum(a.elapsed_time(b) for a, b in sync_ev) / args.steps
+    ms_eager = sum(a.elapsed_time(b) for a, b in eager_ev) / args.steps
     ms_step, value = aggregate_replicas(ms_local, units_per_step, world, dev)
     ms_serial = (t_q + t_d + t_s) / args.steps
 
@@ -518,6 +553,7 @@ def run_lam(args):
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
             "ms_per_step_serial": ms_serial,
+            "ms_per_step_eager": ms_eager,
             "ms_per_step_host_sync": ms_sync,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "f32 in, int%d codes, fp16x2-split tensor / fp32 accumulate" % (8 * max(widths)),
@@ -530,10 +566,12 @@ def run_lam(args):
                        "step": "per eps: lam_quantize_async (AUTO width) on one stream, "
                                "lam_dequantize_from on a second and lam_score_topk_from on a "
                                "third or fourth (alternating), the width read from the quantize "
-                               "status on the device, so nothing waits for the host "
-                               "(ms_per_step_host_sync: the same with the synchronous "
-                               "lam_quantize / lam_dequantize / lam_score_topk; "
-                               "ms_per_step_serial: those all on one stream)"},
+                               "status on the device, so nothing waits for the host; the step "
+                               "is captured once in a CUDA graph and replayed (ms_per_step_eager: "
+                               "the same calls launched one by one; ms_per_step_host_sync: with "
+                               "the synchronous lam_quantize / lam_dequantize / lam_score_topk; "
+                               "ms_per_step_serial: those all on one stream)",
+                       "graph": graph is not None},
             "breakdown": {
                 "quantize_ms": ms_q, "quantize_gbs_algorithmic": q_bytes / (ms_q / 1e3) / 1e9,
                 "quantize_note": "lam_quantize span: status clear + quantize + status read-back",
