@@ -393,6 +393,17 @@ def run_lam(args):
             overlapped_step(i, torch.cuda.Event(enable_timing=True),
                             torch.cuda.Event(enable_timing=True), use_graph=True)
         torch.cuda.synchronize(dev)
+    # launches of one device-resident step (the graph replays the same ones),
+    # counted by the library over one eager step
+    all_kinds = (lam.LAM_TIME_QUANTIZE | lam.LAM_TIME_DEQUANTIZE | lam.LAM_TIME_SCORE |
+                 lam.LAM_TIME_AUX | lam.LAM_TIME_MERGE)
+    lam.lam_timing_begin(all_kinds, 1024)
+    pipe.step_device()
+    torch.cuda.synchronize(dev)
+    launches_per_step = sum(lam.lam_timing_read(kd)[2] for kd in
+                            (lam.LAM_TIME_QUANTIZE, lam.LAM_TIME_DEQUANTIZE, lam.LAM_TIME_SCORE,
+                             lam.LAM_TIME_AUX, lam.LAM_TIME_MERGE))
+    lam.lam_timing_end()
     # the device-resident step gives the synchronous calls' results
     overlapped_step(0, torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
                     use_graph=graph is not None)
@@ -589,9 +600,12 @@ def run_lam(args):
             "roofline": roofline,
             "cpu_baseline": cpu,
             "e2e": e2e,
-            "gpu_launches": n_launch,
-            "gpu_launches_note": "counted by the library over the K steps of the per-kernel "
-                                 "pass (the same launches as the headline pass)",
+            "gpu_launches": launches_per_step * args.steps,
+            "gpu_launches_note": "kernel launches of the library in the K headline steps: %d per "
+                                 "step, counted by the library over one eagerly launched step "
+                                 "(the graph replays the same launches); the per-kernel pass of "
+                                 "the synchronous calls launched %d" % (launches_per_step,
+                                                                         n_launch),
             "clocks": sampler.summary(),
         }
         print(json.dumps(out))
