@@ -105,10 +105,22 @@ __global__ void __launch_bounds__(kCodecThreads) lamz_size_kernel(const float *_
   }
 }
 
+// Writes the stream when the sizing pass found it finite and within `cap`
+// bytes: block 0 the fixed header (magic, n, step s), every warp its blocks'
+// sign words and planes.  (The decision is read from the status on the device,
+// so the host waits once, after this kernel.)
 __global__ void __launch_bounds__(kCodecThreads) lamz_write_kernel(
     const float *__restrict__ x, int64_t n, float rel, const CodecStatus *st,
-    const uint32_t *offs, int64_t nb, uint32_t *payload) {
+    const uint32_t *offs, int64_t nb, uint32_t *payload, uint32_t *out, uint64_t head,
+    uint64_t cap) {
+  if ((__ldg(&st->flags) & kFlagNonfinite) || head + __ldg(&st->total) > cap) return;
   const float s = codec_step(st, rel);
+  if (blockIdx.x == 0 && threadIdx.x == 0) {
+    out[0] = 0x5A4D414Cu;  // "LAMZ" little-endian
+    out[1] = (uint32_t)((uint64_t)n & 0xffffffffu);
+    out[2] = (uint32_t)((uint64_t)n >> 32);
+    out[3] = __float_as_uint(s);
+  }
   const int lane = threadIdx.x & 31;
   const int64_t gw = (int64_t)blockIdx.x * (kCodecThreads / 32) + (threadIdx.x >> 5);
   const int64_t nw = (int64_t)gridDim.x * (kCodecThreads / 32);
@@ -240,28 +252,18 @@ cudaError_t launch_lamz_compress(const float *x, int64_t n, float rel, uint8_t *
                                                                       sizes, nb);
   e = scan_u32(sizes, nb, sums, &st->total, stream);
   if (e != cudaSuccess) return e;
-  CodecStatus h;
+  lamz_write_kernel<<<codec_grid(nb, sms), kCodecThreads, 0, stream>>>(
+      x, n, rel, st, sizes, nb, reinterpret_cast<uint32_t *>(out + head),
+      reinterpret_cast<uint32_t *>(out), (uint64_t)head, (uint64_t)cap);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  CodecStatus h;  // one wait, after the stream is written
   e = read_back(&h, st, sizeof(h), stream);
   if (e != cudaSuccess) return e;
   *nonfinite = (h.flags & kFlagNonfinite) != 0;
   *bytes = head + h.total;
   *fits = *bytes <= cap;
-  if (*nonfinite || !*fits) return cudaSuccess;
-  // fixed header: magic, n, s
-  uint8_t fixed[16] = {'L', 'A', 'M', 'Z'};
-  for (int k = 0; k < 8; ++k) fixed[4 + k] = (uint8_t)((uint64_t)n >> (8 * k));
-  float mx;
-  memcpy(&mx, &h.amax, 4);
-  const float eb = rel * mx;  // fp32 multiply, as on the device
-  const float s = mx > 0.0f ? 2.0f * eb : 1.0f;
-  memcpy(fixed + 12, &s, 4);
-  e = cudaMemcpyAsync(out, fixed, 16, cudaMemcpyHostToDevice, stream);
-  if (e != cudaSuccess) return e;
-  lamz_write_kernel<<<codec_grid(nb, sms), kCodecThreads, 0, stream>>>(
-      x, n, rel, st, sizes, nb, reinterpret_cast<uint32_t *>(out + head));
-  e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
-  return cudaStreamSynchronize(stream);  // `fixed` lives on this stack frame
+  return cudaSuccess;
 }
 
 cudaError_t launch_lamz_decompress(const uint8_t *in, size_t in_bytes, float *out, int64_t n,
