@@ -140,10 +140,17 @@ __global__ void unique_flags_kernel(const uint32_t *hi, const uint32_t *lo, int6
     flag[p] = (p == 0 || hi[p] != hi[p - 1] || lo[p] != lo[p - 1]) ? 1u : 0u;
 }
 
-// Distance of each pair in full precision; keep[p] = 1 within delta.
+// Distance of each pair in full precision; keep[p] = 1 within delta.  The
+// partial sums of squares never decrease (each rounded addition of a
+// non-negative term is at least the running sum), so a pair is rejected as
+// soon as its partial sum passes delta^2 (1 + 2^-40), which puts even the
+// rounded square root above delta; the distances of the kept pairs are
+// summed in full, in coordinate order.  (Most band candidates are far apart
+// and leave after the first 64 coordinates.)
 __global__ void verify_kernel(const float *__restrict__ e, int D, const uint32_t *hi,
                               const uint32_t *lo, const uint32_t *uflag, int64_t n, double delta,
                               double *dist, uint32_t *keep) {
+  const double over = __dmul_rn(__dmul_rn(delta, delta), 1.0 + 0x1p-40);
   for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < n;
        p += (int64_t)gridDim.x * blockDim.x) {
     uint32_t k = 0;
@@ -151,11 +158,16 @@ __global__ void verify_kernel(const float *__restrict__ e, int D, const uint32_t
     if (uflag[p]) {
       const float *a = e + (int64_t)hi[p] * D, *b = e + (int64_t)lo[p] * D;
       double acc = 0.0;
-      for (int d = 0; d < D; ++d) {
-        const double t = __dsub_rn((double)__ldg(a + d), (double)__ldg(b + d));
-        acc = __dadd_rn(acc, __dmul_rn(t, t));
+      bool far = false;
+      for (int d0 = 0; d0 < D && !far; d0 += 64) {
+        const int d1 = d0 + 64 < D ? d0 + 64 : D;
+        for (int d = d0; d < d1; ++d) {
+          const double t = __dsub_rn((double)__ldg(a + d), (double)__ldg(b + d));
+          acc = __dadd_rn(acc, __dmul_rn(t, t));
+        }
+        far = acc > over;
       }
-      dd = sqrt(acc);
+      dd = far ? INFINITY : sqrt(acc);
       k = dd <= delta ? 1u : 0u;
     }
     dist[p] = dd;
