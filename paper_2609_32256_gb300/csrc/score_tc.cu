@@ -13,19 +13,22 @@
 //
 // CTA: 128 queries (MMA M) x a contiguous range of 256-row tiles (MMA N).
 // Two shared-memory rings:
-//   MMA stages (K = 32): the query block's hi/lo tiles, laid out by the query
-//     preparation kernel exactly as the 64-byte-swizzled UMMA operand, so one
-//     16 KB bulk copy fills them; and the fp16 code tile the converters write;
-//   raw stages: 256 code rows x 128 bytes (K = 128 int8 / 64 int16, four or
-//     two MMA stages' worth) by one 2-D TMA load with the 128-byte swizzle.
-// Warp roles (320 threads):
-//   warp 0      producer: raw-code TMA loads and query bulk copies;
+//   MMA stages (two K = 32 chunks): the query block's hi/lo tiles, laid out by
+//     the query preparation kernel exactly as the 64-byte-swizzled UMMA
+//     operand, so one 32 KB bulk copy fills them; and the fp16 code tiles the
+//     converters write;
+//   raw stages (two to four): 256 code rows x 128 bytes (K = 128 int8 / 64
+//     int16) by one 2-D TMA load with the 128-byte swizzle.
+// Warp roles (352 threads; warp w runs on SM sub-partition w % 4):
+//   warp 0      producer of the raw-code TMA loads;
 //   warp 1      TMEM allocation; one lane issues tcgen05.mma (2 K-steps x
-//               hi/lo per stage) and commits stage/accumulator barriers;
+//               hi/lo per chunk) and commits stage/accumulator barriers;
 //   warps 2-5   convert raw int8/int16 codes to fp16 in the UMMA K-major
 //               64B-swizzled layout, and sum c^2 per row for cosine / L2;
 //   warps 6-9   epilogue: tcgen05.ld of the 128x256 fp32 accumulator (double
-//               buffered, 2 x 256 TMEM columns), scores, per-query top-k.
+//               buffered, 2 x 256 TMEM columns), scores, per-query top-k; a
+//               warp whose 32 MMA rows hold no query sits out;
+//   warp 10     producer of the query-block bulk copies.
 // Every wait is bounded; a timeout records LAM_ERR_TIMEOUT and unwinds.
 #include "score_common.cuh"
 
@@ -39,7 +42,7 @@ constexpr int kBM = 128;        // queries per CTA (MMA M)
 constexpr int kBN = 256;        // code rows per tile (MMA N)
 constexpr int kBK = 32;         // fp16 per stage along D (64-byte rows)
 constexpr int kUmmaK = 16;      // K of one kind::f16 MMA
-constexpr int kTcThreads = 320;  // 10 warps, roles below
+constexpr int kTcThreads = 352;  // 11 warps, roles below
 constexpr int kConvThreads = 128;
 constexpr int kABytes = kBM * kBK * 2;    // one of hi / lo: 8 KB
 constexpr int kAStage = 2 * kABytes;      // hi + lo, one bulk copy: 16 KB
@@ -47,7 +50,8 @@ constexpr int kB16Bytes = kBN * kBK * 2;  // converted codes: 16 KB
 constexpr int kStageBytes = kAStage + kB16Bytes;  // one MMA stage: 32 KB
 constexpr int kRawRow = 128;              // bytes of one code row per raw stage
 constexpr int kRawBytes = kBN * kRawRow;  // one raw stage: 32 KB
-constexpr int kCBuf = 16;                 // epilogue candidate buffer per query
+constexpr int kRawMax = 4;                // raw stages at most
+constexpr int kCBuf = 16;                 // k > 32: heap candidate buffer depth at most
 constexpr int kTcChunks = 2;              // K chunks per MMA stage of the stage-loop kernel
 constexpr uint32_t kTmemCols = 512;       // two 256-column accumulators
 constexpr int kMaxDynSmem = 232448;       // 227 KB
@@ -161,6 +165,34 @@ __device__ __forceinline__ float tile_score(int metric, float acc, float fq, flo
   return fmaf(fq, acc, qq + rowf);
 }
 
+// Candidate mask of one 32-column chunk: bit j is set when column j's score
+// (tile_score, the same roundings) beats thr: greater for inner product and
+// cosine, smaller for L2.  rf(j) gives column j's row factor.  The metric is a
+// template argument so that the 32-wide loop carries no per-element dispatch.
+template <int MET, typename RF>
+__device__ __forceinline__ uint32_t chunk_mask_m(const uint32_t (&v)[32], float fq, float qq,
+                                                 float thr, RF rf) {
+  uint32_t mask = 0;
+#pragma unroll
+  for (int j = 0; j < 32; ++j) {
+    const float acc = __uint_as_float(v[j]);
+    float sc;
+    if constexpr (MET == LAM_METRIC_IP) sc = fq * acc;
+    else if constexpr (MET == LAM_METRIC_COSINE) sc = (fq * acc) * rf(j);
+    else sc = fmaf(fq, acc, qq + rf(j));
+    const bool beat = MET == LAM_METRIC_L2 ? sc < thr : sc > thr;
+    mask |= (uint32_t)beat << j;
+  }
+  return mask;
+}
+template <typename RF>
+__device__ __forceinline__ uint32_t chunk_mask(int metric, const uint32_t (&v)[32], float fq,
+                                               float qq, float thr, RF rf) {
+  if (metric == LAM_METRIC_IP) return chunk_mask_m<LAM_METRIC_IP>(v, fq, qq, thr, rf);
+  if (metric == LAM_METRIC_COSINE) return chunk_mask_m<LAM_METRIC_COSINE>(v, fq, qq, thr, rf);
+  return chunk_mask_m<LAM_METRIC_L2>(v, fq, qq, thr, rf);
+}
+
 // k > 32 heaps: candidates that beat the heap root are buffered per query
 // (cbn slots per query in shared memory, stride kBM) and poured into the heaps
 // when one query's buffer is full, so the lanes of a warp sift together
@@ -184,6 +216,33 @@ __device__ __forceinline__ float warp_sum_tc(float v) {
   return v;
 }
 
+// Converter thread -> (tile row, 16-byte piece) of its i-th task, chosen so
+// that each quarter-warp's 16-byte accesses fall in distinct banks both when
+// reading the raw rows (128 bytes, piece ^ row & 7) and when writing the fp16
+// rows (64 bytes, piece ^ (row >> 1) & 3).  int16: a quarter-warp takes rows
+// {j, j ^ 5} of an 8-row block (four pieces each); int8: rows {0, 2, 5, 7} or
+// {1, 3, 4, 6} of the block (two pieces each).  Lanes of one row differ in
+// the low bits of the thread index (for the c^2 shuffles).
+template <int W>
+__device__ __forceinline__ int conv_row(int ct, int i) {
+  const int q = ct >> 3, e = ct & 7;
+  if (W == 2) {
+    const int j = q & 3;
+    return 32 * i + 8 * (q >> 2) + ((e >> 2) ? (j ^ 5) : j);
+  }
+  const int slot = e >> 1;
+  return 64 * i + 8 * (q >> 1) + ((2 * slot + (slot >> 1)) ^ (q & 1));
+}
+template <int W>
+__device__ __forceinline__ int conv_sub(int ct) {
+  return W == 2 ? ct & 3 : ct & 1;
+}
+
+template <bool B>
+struct BoolTag {
+  static constexpr bool value = B;
+};
+
 // v[j] for a run-time j, by a tree of selects (no local-memory indexing).
 __device__ __forceinline__ uint32_t select32(const uint32_t (&v)[32], int j) {
   uint32_t t16[16], t8[8], t4[4], t2[2];
@@ -203,18 +262,21 @@ struct TcLayout {
   size_t raw_off, lists_off, cbuf_off, cc_off, bar_off, smem_bytes;
 };
 
-// Shared memory: [MMA stages][raw stages][k > 32: per-query heaps][candidate
-// buffers][c^2 per row, 2 tiles][barriers, TMEM slot, abort flag].  The heaps'
-// buffers take up to kCBuf slots per query, as many as leave room for two
-// single-chunk MMA stages and one raw stage (the kernel reads the depth back
-// from the offsets).
-inline TcLayout tc_layout(int width, int k) {
+// Shared memory: [MMA stages][raw stages][k > 32: per-query heaps and their
+// candidate buffers][cosine / L2: c^2 per row, 2 tiles][barriers, TMEM slot,
+// abort flag].  The heaps' buffers take up to kCBuf slots per query, as many
+// as leave room for two single-chunk MMA stages and one raw stage (the kernel
+// reads the depth back from the offsets).  Raw stages fill what is left, up to
+// kRawMax: the deeper the ring, the more code bytes are in flight while the
+// converters work.  (The inner-product layout, without the c^2 buffers, fits
+// a third raw stage beside two double-chunk MMA stages.)
+inline TcLayout tc_layout(int width, int k, bool cc_rows = true) {
   (void)width;
   TcLayout L;
   const size_t lists = k > 32 ? (size_t)kBM * k * 8 : 0;
-  const size_t cc = 2 * kBN * 4;
+  const size_t cc = cc_rows ? 2 * kBN * 4 : 0;
   const size_t tailb = 64 * 8 + 1024;  // barriers, slots, alignment slack
-  size_t cbuf = (size_t)kCBuf * kBM * 8;
+  size_t cbuf = 0;
   if (k > 32) {
     const size_t room = kMaxDynSmem - lists - cc - tailb;
     const size_t need = 2 * (size_t)kStageBytes + kRawBytes;
@@ -225,17 +287,14 @@ inline TcLayout tc_layout(int width, int k) {
   // two K chunks per MMA stage (one 32 KB copy of the query blocks, 8 MMAs
   // per barrier round trip) when two such stages and two raw stages fit
   L.chunks = (size_t)2 * kTcChunks * kStageBytes + (size_t)2 * kRawBytes <= avail ? kTcChunks : 1;
-  int ns = L.chunks > 1 ? 2 : 4, nr = 2;
-  while ((size_t)ns * L.chunks * kStageBytes + (size_t)nr * kRawBytes > avail) {
-    if (ns > 2) {
-      --ns;
-    } else if (nr > 1) {
-      --nr;
-    } else {
-      ns = 0;
-      break;
-    }
+  int ns = L.chunks > 1 ? 2 : 3, nr = 0;
+  for (;; --ns) {
+    const size_t mma = (size_t)ns * L.chunks * kStageBytes;
+    nr = mma < avail ? (int)((avail - mma) / kRawBytes) : 0;
+    if (nr > kRawMax) nr = kRawMax;
+    if (nr >= 2 || ns == 2) break;
   }
+  if (nr < 1) ns = 0;
   L.ns = ns;
   L.nr = nr;
   L.raw_off = (size_t)ns * L.chunks * kStageBytes;
@@ -250,6 +309,7 @@ inline TcLayout tc_layout(int width, int k) {
 struct TcGeom {
   int ns, nr, chunks;  // MMA stages, raw stages, 32-wide K chunks per MMA stage
   int raw_off, lists_off, cbuf_off, cc_off, bar_off;
+  int qoff;  // MMA row of the block's first query (64 for one block of <= 64)
   const QuantStatus *qst;  // status-driven calls: the codes' width is read here
 };
 
@@ -266,7 +326,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   const size_t stage_stride = (size_t)C * kStageBytes;  // [C query blocks][C code blocks]
   uint8_t *raw_ring = smem + g.raw_off;
   uint64_t *lists = reinterpret_cast<uint64_t *>(smem + g.lists_off);
-  uint2 *cbuf = reinterpret_cast<uint2 *>(smem + g.cbuf_off);
+  uint8_t *cbuf = smem + g.cbuf_off;  // k > 32: the heaps' candidate buffers
   float *ccbuf = reinterpret_cast<float *>(smem + g.cc_off);
   uint64_t *afull = reinterpret_cast<uint64_t *>(smem + g.bar_off);
   uint64_t *conv = afull + ns;
@@ -288,9 +348,15 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   const int64_t te = (int64_t)(blockIdx.x + 1) * n_tiles / gridDim.x;
   const int ntl = (int)(te - tb);
   const int nk = (a.D + kBK - 1) / kBK;
-  constexpr int R = kRawRow / (kBK * W);  // MMA stages per raw stage: 4 (int8), 2 (int16)
+  constexpr int R = kRawRow / (kBK * W);  // K chunks per raw stage: 4 (int8), 2 (int16)
   const bool need_cc = a.metric != LAM_METRIC_IP;
   const uint8_t *qA = static_cast<const uint8_t *>(a.qprep);
+  // Epilogue warps whose 32 MMA rows hold queries; the others sit out (the
+  // query rows are g.qoff .. row_end - 1 of the block).
+  const int64_t q_left = a.B - (int64_t)qb * kBM;
+  const int row_end = g.qoff + (int)(q_left < kBM - g.qoff ? q_left : kBM - g.qoff);
+  auto quad_used = [&](int q) { return 32 * q < row_end && 32 * q + 32 > g.qoff; };
+  const uint32_t n_epi = 32u * (uint32_t)(quad_used(0) + quad_used(1) + quad_used(2) + quad_used(3));
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < ns; ++s) {
@@ -304,9 +370,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&accf[b], 1);
-      mbar_init(&acce[b], 128);
+      mbar_init(&acce[b], n_epi);
       mbar_init(&ccf[b], kConvThreads);
-      mbar_init(&cce[b], 128);
+      mbar_init(&cce[b], n_epi);
     }
     mbar_init(done, 1);
     *abort_flag = 0;
@@ -322,37 +388,19 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   if (warp == 0) {
     // ------------------------------------------------ producer -----------
     if (lane == 0) {
-      int it = 0, gr = 0, a_issued = 0, r_issued = 0;
-      bool ok = true;
-      for (int lt = 0; lt < ntl && ok; ++lt) {
-        const int tile = (int)(tb + lt);
-        for (int kc = 0; kc < nk; ++kc) {
-          if (kc % R == 0) {
-            const int rs = gr % nr, rr = gr / nr;
-            if (rr > 0 && !mbar_wait(&rempty[rs], (rr - 1) & 1, abort_flag, a.gflags)) {
-              ok = false;
-              break;
-            }
-            mbar_arrive_expect_tx(&rfull[rs], kRawBytes);
-            tma_load_2d(raw_ring + (size_t)rs * kRawBytes, &cmap, (kc / R) * (kRawRow / W),
-                        tile * kBN, &rfull[rs]);
-            r_issued = ++gr;
-          }
-          if (kc % C != 0) continue;  // the stage's query blocks came with its first chunk
-          const int s = it % ns, r = it / ns;
-          const int nc = nk - kc < C ? nk - kc : C;
-          if (r > 0 && !mbar_wait(&empty[s], (r - 1) & 1, abort_flag, a.gflags)) {
-            ok = false;
-            break;
-          }
-          mbar_arrive_expect_tx(&afull[s], (uint32_t)nc * kAStage);
-          bulk_g2s(smem + (size_t)s * stage_stride, qA + ((size_t)qb * nk + kc) * kAStage,
-                   (uint32_t)nc * kAStage, &afull[s]);
-          a_issued = ++it;
-        }
+      // raw code stages, freed by the converters
+      const int rpt = (nk + R - 1) / R;  // raw stages per tile
+      const int r_total = ntl * rpt;
+      int gr = 0;
+      for (; gr < r_total; ++gr) {
+        const int rs = gr % nr, rr = gr / nr;
+        if (rr > 0 && !mbar_wait(&rempty[rs], (rr - 1) & 1, abort_flag, a.gflags)) break;
+        const int lt = gr / rpt, j = gr - lt * rpt;
+        mbar_arrive_expect_tx(&rfull[rs], kRawBytes);
+        tma_load_2d(raw_ring + (size_t)rs * kRawBytes, &cmap, j * (kRawRow / W),
+                    (int)(tb + lt) * kBN, &rfull[rs]);
       }
-      for (int t = max(0, a_issued - ns); t < a_issued; ++t) drain_wait_tc(&afull[t % ns], (t / ns) & 1);
-      for (int t = max(0, r_issued - nr); t < r_issued; ++t) drain_wait_tc(&rfull[t % nr], (t / nr) & 1);
+      for (int t = max(0, gr - nr); t < gr; ++t) drain_wait_tc(&rfull[t % nr], (t / nr) & 1);
     }
   } else if (warp == 1) {
     // ------------------------------------------------ MMA issuer ---------
@@ -394,120 +442,196 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     }
   } else if (warp < 6) {
     // ------------------------------------------------ converters ---------
-    const int ct = threadIdx.x - 64;  // 0 .. 127
-    constexpr int kTasks = (W == 1 ? 512 : 1024) / kConvThreads;  // 16-byte chunks per thread
-    const __half2 bias = __float2half2_rn(1152.0f);
-    int it = 0, gr = 0;
-    bool ok = true;
-    float amax = 0.0f;
-    for (int lt = 0; lt < ntl && ok; ++lt) {
-      const int buf = lt & 1, u = lt >> 1;
-      float ccp[kTasks];
+    // (CC: the row's sum of c^2 is needed, cosine and L2)
+    auto converters = [&](auto cc_tag) {
+      constexpr bool CC = decltype(cc_tag)::value;
+      const int ct = threadIdx.x - 64;  // 0 .. 127
+      constexpr int kTasks = (W == 1 ? 512 : 1024) / kConvThreads;  // 16-byte chunks per thread
+      const __half2 bias = __float2half2_rn(1152.0f);
+      int it = 0, gr = 0;
+      bool ok = true;
+      float amax = 0.0f;
+      for (int lt = 0; lt < ntl && ok; ++lt) {
+        const int buf = lt & 1, u = lt >> 1;
+        float ccp[kTasks];
 #pragma unroll
-      for (int i = 0; i < kTasks; ++i) ccp[i] = 0.0f;
-      for (int kc = 0; kc < nk; ++kc) {
-        const int rs = gr % nr;
-        if (kc % R == 0 && !mbar_wait(&rfull[rs], (gr / nr) & 1, abort_flag, a.gflags)) {
-          ok = false;
-          break;
-        }
-        const int s = it % ns, r = it / ns;
-        if (kc % C == 0 && r > 0 && !mbar_wait(&empty[s], (r - 1) & 1, abort_flag, a.gflags)) {
-          ok = false;
-          break;
-        }
-        const uint8_t *__restrict__ raw = raw_ring + (size_t)rs * kRawBytes;
-        uint8_t *__restrict__ b16 =
-            smem + (size_t)s * stage_stride + (size_t)C * kAStage + (size_t)(kc % C) * kB16Bytes;
-        const int j0 = (kc % R) * (kBK * W / 16);  // first 16-byte chunk of this K slice
-        // All loads first: the stores below could alias them as far as the
-        // compiler knows, which would otherwise serialise the tasks.
-        uint4 rv[kTasks];
+        for (int i = 0; i < kTasks; ++i) ccp[i] = 0.0f;
+        for (int kc = 0; kc < nk; ++kc) {
+          const int rs = gr % nr;
+          if (kc % R == 0 && !mbar_wait(&rfull[rs], (gr / nr) & 1, abort_flag, a.gflags)) {
+            ok = false;
+            break;
+          }
+          const int s = it % ns, r = it / ns;
+          if (kc % C == 0 && r > 0 && !mbar_wait(&empty[s], (r - 1) & 1, abort_flag, a.gflags)) {
+            ok = false;
+            break;
+          }
+          const uint8_t *__restrict__ raw = raw_ring + (size_t)rs * kRawBytes;
+          uint8_t *__restrict__ b16 =
+              smem + (size_t)s * stage_stride + (size_t)C * kAStage + (size_t)(kc % C) * kB16Bytes;
+          const int j0 = (kc % R) * (kBK * W / 16);  // first 16-byte chunk of this K slice
+          // All loads first: the stores below could alias them as far as the
+          // compiler knows, which would otherwise serialise the tasks.  Raw rows
+          // are 128 bytes in the 128-byte swizzle (chunk ^ row & 7).
+          uint4 rv[kTasks];
 #pragma unroll
-        for (int i = 0; i < kTasks; ++i) {
-          const int task = ct + kConvThreads * i;
-          const int row = (W == 1) ? task >> 1 : task >> 2;
-          const int sub = (W == 1) ? task & 1 : task & 3;
-          rv[i] = *reinterpret_cast<const uint4 *>(raw + row * kRawRow + (((j0 + sub) ^ (row & 7)) << 4));
-        }
+          for (int i = 0; i < kTasks; ++i) {
+            const int row = conv_row<W>(ct, i), sub = conv_sub<W>(ct);
+            rv[i] = *reinterpret_cast<const uint4 *>(raw + row * kRawRow +
+                                                     (((j0 + sub) ^ (row & 7)) << 4));
+          }
+          if constexpr (W == 1) {
 #pragma unroll
-        for (int i = 0; i < kTasks; ++i) {
-          const int task = ct + kConvThreads * i;
-          if (W == 1) {
-            const int row = task >> 1, h = task & 1;
-            const uint32_t w[4] = {rv[i].x, rv[i].y, rv[i].z, rv[i].w};
-            uint32_t o[8];
+            for (int i = 0; i < kTasks; ++i) {
+              const int row = conv_row<W>(ct, i), h = conv_sub<W>(ct);
+              const uint32_t w[4] = {rv[i].x, rv[i].y, rv[i].z, rv[i].w};
+              uint32_t o[8];
 #pragma unroll
-            for (int j = 0; j < 4; ++j) {
-              const uint32_t x = w[j] ^ 0x80808080u;
-              // fp16 bits 0x64uu = 1024 + u with u = code + 128; minus 1152 = code
-              o[2 * j] = h2_as_u32(__hsub2(u32_as_h2(__byte_perm(x, 0x64646464u, 0x5140)), bias));
-              o[2 * j + 1] = h2_as_u32(__hsub2(u32_as_h2(__byte_perm(x, 0x64646464u, 0x7362)), bias));
-            }
-            const int sw = (row >> 1) & 3;
-            uint8_t *rowp = b16 + row * 64;
-            *reinterpret_cast<uint4 *>(rowp + (((2 * h) ^ sw) << 4)) = make_uint4(o[0], o[1], o[2], o[3]);
-            *reinterpret_cast<uint4 *>(rowp + (((2 * h + 1) ^ sw) << 4)) = make_uint4(o[4], o[5], o[6], o[7]);
-            if (need_cc) {
-              int c2 = 0;
+              for (int j = 0; j < 4; ++j) {
+                const uint32_t x = w[j] ^ 0x80808080u;
+                // fp16 bits 0x64uu = 1024 + u with u = code + 128; minus 1152 = code
+                o[2 * j] = h2_as_u32(__hsub2(u32_as_h2(__byte_perm(x, 0x64646464u, 0x5140)), bias));
+                o[2 * j + 1] =
+                    h2_as_u32(__hsub2(u32_as_h2(__byte_perm(x, 0x64646464u, 0x7362)), bias));
+              }
+              const int sw = (row >> 1) & 3;
+              uint8_t *rowp = b16 + row * 64;
+              *reinterpret_cast<uint4 *>(rowp + (((2 * h) ^ sw) << 4)) = make_uint4(o[0], o[1], o[2], o[3]);
+              *reinterpret_cast<uint4 *>(rowp + (((2 * h + 1) ^ sw) << 4)) =
+                  make_uint4(o[4], o[5], o[6], o[7]);
+              if (CC) {
+                int c2 = 0;
 #pragma unroll
-              for (int j = 0; j < 4; ++j) c2 = __dp4a((int)w[j], (int)w[j], c2);
-              ccp[i] += (float)c2;
+                for (int j = 0; j < 4; ++j) c2 = __dp4a((int)w[j], (int)w[j], c2);
+                ccp[i] += (float)c2;
+              }
             }
           } else {
-            const int row = task >> 2, qt = task & 3;
-            const uint32_t w[4] = {rv[i].x ^ 0x80008000u, rv[i].y ^ 0x80008000u,
-                                   rv[i].z ^ 0x80008000u, rv[i].w ^ 0x80008000u};
-            uint32_t o[4];
-            float c2 = 0.0f;
+            // Each 16-bit half biased to c + 0x8080 (no carry between the
+            // halves while c is small): its high byte is 0x80 exactly when c
+            // lies in [-128, 127], and its low byte is then c + 128.  One vote
+            // per chunk picks the path for all of the warp's tasks, so that
+            // the tasks stay independent and interleave.
+            uint32_t xb[kTasks][4], tor = 0;
 #pragma unroll
-            for (int j = 0; j < 4; ++j) {
-              const float f0 = __int_as_float(__byte_perm(w[j], 0x4B000000u, 0x7410)) - 8421376.0f;
-              const float f1 = __int_as_float(__byte_perm(w[j], 0x4B000000u, 0x7432)) - 8421376.0f;
-              amax = fmaxf(amax, fmaxf(fabsf(f0), fabsf(f1)));
-              c2 = fmaf(f0, f0, fmaf(f1, f1, c2));
-              o[j] = h2_as_u32(__floats2half2_rn(f0, f1));
+            for (int i = 0; i < kTasks; ++i) {
+              const uint32_t w[4] = {rv[i].x, rv[i].y, rv[i].z, rv[i].w};
+#pragma unroll
+              for (int j = 0; j < 4; ++j) {
+                xb[i][j] = (w[j] ^ 0x80008000u) + 0x00800080u;
+                tor |= xb[i][j] ^ 0x80008000u;
+              }
             }
-            const int sw = (row >> 1) & 3;
-            *reinterpret_cast<uint4 *>(b16 + row * 64 + ((qt ^ sw) << 4)) = make_uint4(o[0], o[1], o[2], o[3]);
-            if (need_cc) ccp[i] += c2;
+            if (__all_sync(0xffffffffu, (tor & 0xff00ff00u) == 0u)) {
+              // the int8 conversion on the low bytes
+#pragma unroll
+              for (int i = 0; i < kTasks; ++i) {
+                const int row = conv_row<W>(ct, i), qt = conv_sub<W>(ct);
+                uint32_t o[4];
+#pragma unroll
+                for (int j = 0; j < 4; ++j)
+                  o[j] = h2_as_u32(__hsub2(u32_as_h2(__byte_perm(xb[i][j], 0x64646464u, 0x4240)), bias));
+                *reinterpret_cast<uint4 *>(b16 + row * 64 + ((qt ^ ((row >> 1) & 3)) << 4)) =
+                    make_uint4(o[0], o[1], o[2], o[3]);
+                if (CC) {
+                  const int p0 = (int)__byte_perm(rv[i].x, rv[i].y, 0x6420);
+                  const int p1 = (int)__byte_perm(rv[i].z, rv[i].w, 0x6420);
+                  ccp[i] += (float)__dp4a(p1, p1, __dp4a(p0, p0, 0));
+                }
+              }
+            } else {
+#pragma unroll
+              for (int i = 0; i < kTasks; ++i) {
+                const int row = conv_row<W>(ct, i), qt = conv_sub<W>(ct);
+                const uint32_t w[4] = {rv[i].x, rv[i].y, rv[i].z, rv[i].w};
+                uint32_t o[4];
+                float c2 = 0.0f;
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                  const uint32_t x = w[j] ^ 0x80008000u;
+                  const float f0 = __int_as_float(__byte_perm(x, 0x4B000000u, 0x7410)) - 8421376.0f;
+                  const float f1 = __int_as_float(__byte_perm(x, 0x4B000000u, 0x7432)) - 8421376.0f;
+                  amax = fmaxf(amax, fmaxf(fabsf(f0), fabsf(f1)));
+                  if (CC) c2 = fmaf(f0, f0, fmaf(f1, f1, c2));
+                  o[j] = h2_as_u32(__floats2half2_rn(f0, f1));
+                }
+                *reinterpret_cast<uint4 *>(b16 + row * 64 + ((qt ^ ((row >> 1) & 3)) << 4)) =
+                    make_uint4(o[0], o[1], o[2], o[3]);
+                if (CC) ccp[i] += c2;
+              }
+            }
+          }
+          if (kc % C == C - 1 || kc == nk - 1) {  // the stage's chunks are all converted
+            fence_proxy_async_smem();
+            mbar_arrive(&conv[s]);
+            ++it;
+          }
+          if (kc % R == R - 1 || kc == nk - 1) {
+            mbar_arrive(&rempty[rs]);
+            ++gr;
           }
         }
-        if (kc % C == C - 1 || kc == nk - 1) {  // the stage's chunks are all converted
-          fence_proxy_async_smem();
-          mbar_arrive(&conv[s]);
-          ++it;
-        }
-        if (kc % R == R - 1 || kc == nk - 1) {
-          mbar_arrive(&rempty[rs]);
-          ++gr;
-        }
-      }
-      if (!ok) break;
-      if (need_cc) {
-        if (u > 0 && !mbar_wait(&cce[buf], (u - 1) & 1, abort_flag, a.gflags)) break;
+        if (!ok) break;
+        if (CC) {
+          if (u > 0 && !mbar_wait(&cce[buf], (u - 1) & 1, abort_flag, a.gflags)) break;
 #pragma unroll
-        for (int i = 0; i < kTasks; ++i) {
-          const int task = ct + kConvThreads * i;
-          float t = ccp[i] + __shfl_xor_sync(0xffffffffu, ccp[i], 1);
-          if (W == 2) t += __shfl_xor_sync(0xffffffffu, t, 2);
-          const bool writer = (W == 1) ? ((task & 1) == 0) : ((task & 3) == 0);
-          // per-row factor of the score: 1/||c|| for cosine, s^2 ||c||^2 for L2
-          const float rowf = a.metric == LAM_METRIC_COSINE ? (t > 0.0f ? 1.0f / sqrtf(t) : 0.0f)
-                                                          : a.s * a.s * t;
-          if (writer) ccbuf[buf * kBN + (W == 1 ? task >> 1 : task >> 2)] = rowf;
+          for (int i = 0; i < kTasks; ++i) {
+            float t = ccp[i] + __shfl_xor_sync(0xffffffffu, ccp[i], 1);
+            if (W == 2) t += __shfl_xor_sync(0xffffffffu, t, 2);
+            const bool writer = conv_sub<W>(ct) == 0;
+            // per-row factor of the score: 1/||c|| for cosine, s^2 ||c||^2 for L2
+            const float rowf = a.metric == LAM_METRIC_COSINE ? (t > 0.0f ? 1.0f / sqrtf(t) : 0.0f)
+                                                            : a.s * a.s * t;
+            if (writer) ccbuf[buf * kBN + conv_row<W>(ct, i)] = rowf;
+          }
+          mbar_arrive(&ccf[buf]);
         }
-        mbar_arrive(&ccf[buf]);
       }
+      if (W == 2 && amax > 2048.0f) atomicOr(a.gflags, kFlagRange);
+    };
+    if (need_cc)
+      converters(BoolTag<true>{});
+    else
+      converters(BoolTag<false>{});
+  } else if (warp == 10) {
+    // ------------------------------------------------ query producer -----
+    if (lane == 0) {
+      // the query blocks of the MMA stages, freed by the MMAs
+      const int spt = (nk + C - 1) / C;  // MMA stages per tile
+      const int a_total = ntl * spt;
+      int it = 0;
+      for (; it < a_total; ++it) {
+        const int s = it % ns, r = it / ns;
+        if (r > 0 && !mbar_wait(&empty[s], (r - 1) & 1, abort_flag, a.gflags)) break;
+        const int kc = (it % spt) * C;
+        const int nc = nk - kc < C ? nk - kc : C;
+        uint8_t *dst = smem + (size_t)s * stage_stride;
+        const uint8_t *src = qA + ((size_t)qb * nk + kc) * kAStage;
+        if (g.qoff == 0) {
+          mbar_arrive_expect_tx(&afull[s], (uint32_t)nc * kAStage);
+          bulk_g2s(dst, src, (uint32_t)nc * kAStage, &afull[s]);
+        } else {
+          // queries in MMA rows 64 .. 127 only: the hi and lo rows 0 .. 63
+          // (64-byte rows, the first 4 KB of each 8 KB tile) feed TMEM lanes
+          // that no epilogue warp reads, so they are not copied
+          mbar_arrive_expect_tx(&afull[s], (uint32_t)nc * kABytes);
+          for (int c = 0; c < nc; ++c)
+            for (int h = 0; h < 2; ++h) {
+              const size_t off = (size_t)c * kAStage + (size_t)h * kABytes + kABytes / 2;
+              bulk_g2s(dst + off, src + off, kABytes / 2, &afull[s]);
+            }
+        }
+      }
+      for (int t = max(0, it - ns); t < it; ++t) drain_wait_tc(&afull[t % ns], (t / ns) & 1);
     }
-    if (W == 2 && amax > 2048.0f) atomicOr(a.gflags, kFlagRange);
-  } else {
+  } else if (quad_used(warp & 3)) {
     // ------------------------------------------------ epilogue -----------
     // (warp w may read TMEM lanes 32 (w % 4) .. 32 (w % 4) + 31)
     const int quad = warp & 3;
-    const int m = quad * 32 + lane;  // TMEM lane = query within the block
-    const int64_t qidx = (int64_t)qb * kBM + m;
-    const bool qvalid = qidx < a.B;
+    const int m = quad * 32 + lane;  // TMEM lane = MMA row of the query block
+    const int64_t qidx = (int64_t)qb * kBM + m - g.qoff;
+    const bool qvalid = m >= g.qoff && qidx < a.B;
     const int k = a.k;
     const bool desc = a.metric != LAM_METRIC_L2;
     const float s = a.s;
@@ -529,7 +653,6 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     reg.init(k);
     float thr_s = desc ? -INFINITY : INFINITY;  // score of the k-th best so far
     float seed = desc ? -INFINITY : INFINITY;   // admission bound before the list fills
-    int cnt = 0;                                // buffered candidates of this query
     // k > 32: the heaps' candidate buffers (depth from the layout)
     uint64_t *hb = reinterpret_cast<uint64_t *>(cbuf);
     const int hbn = KR == 0 ? (g.cc_off - g.cbuf_off) / (kBM * 8) : 0;
@@ -577,43 +700,37 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         if (KR > 0) {
           // Candidates must beat the k-th score strictly (rows arrive in
           // increasing order, so an equal score ranks later).  A compact pass
-          // marks them in a 32-bit mask; the warp then appends them to the
-          // per-query buffers and merges all buffers when one is full.
+          // marks them in a 32-bit mask; the warp then inserts them into the
+          // register lists, one per lane per step, each re-tested against the
+          // threshold the earlier steps tightened.
           const int64_t nvalid = a.N - (row0 + c * 32);
           const float thr_c = desc ? fmaxf(thr_s, thr) : fminf(thr_s, thr);
-          uint32_t mask = 0;
-#pragma unroll
-          for (int j = 0; j < 32; ++j) {
-            const float rf = need_cc ? ccbuf[buf * kBN + c * 32 + j] : 0.0f;
-            const float sc = tile_score(a.metric, __uint_as_float(v[j]), fq, qq, rf);
-            mask |= (uint32_t)(desc ? sc > thr_c : sc < thr_c) << j;
-          }
+          const float *ccc = ccbuf + buf * kBN + c * 32;
+          uint32_t mask = chunk_mask(a.metric, v, fq, qq, thr_c, [&](int j) { return ccc[j]; });
           if (!qvalid || nvalid <= 0) mask = 0;
           else if (nvalid < 32) mask &= (1u << nvalid) - 1u;
           while (__any_sync(0xffffffffu, mask != 0)) {
+            uint32_t kc = 0xffffffffu, ic = 0xffffffffu;
             if (mask != 0) {
               const int j = __ffs(mask) - 1;
               mask &= mask - 1;
-              const float rf = need_cc ? ccbuf[buf * kBN + c * 32 + j] : 0.0f;
+              const float rf = need_cc ? ccc[j] : 0.0f;
               const float sc = tile_score(a.metric, __uint_as_float(select32(v, j)), fq, qq, rf);
-              cbuf[(size_t)cnt * kBM + m] =
-                  make_uint2(rank_key32(sc, desc), (uint32_t)(row0 + c * 32 + j));
-              ++cnt;
+              if (desc ? sc > thr_s : sc < thr_s) {
+                kc = rank_key32(sc, desc);
+                ic = (uint32_t)(row0 + c * 32 + j);
+              }
             }
-            if (__any_sync(0xffffffffu, cnt == kCBuf))
-              merge_candidates(reg, cbuf, m, kBM, cnt, thr_s, desc);
+            reg.insert(kc, ic);
+            const uint32_t tk = reg.key[RK - 1];
+            thr_s = tk == 0xffffffffu ? (desc ? -INFINITY : INFINITY) : rank_key32_score(tk, desc);
           }
         } else if (KR == 0) {
           // k > 32: a max-heap per query in shared memory (root = the worst
           // key kept); a candidate replaces the root and sifts down.
           const int64_t nvalid = a.N - (row0 + c * 32);
-          uint32_t mask = 0;
-#pragma unroll
-          for (int j = 0; j < 32; ++j) {
-            const float rf = need_cc ? ccbuf[buf * kBN + c * 32 + j] : 0.0f;
-            const float sc = tile_score(a.metric, __uint_as_float(v[j]), fq, qq, rf);
-            mask |= (uint32_t)(desc ? sc > thr_s : sc < thr_s) << j;
-          }
+          const float *ccc = ccbuf + buf * kBN + c * 32;
+          uint32_t mask = chunk_mask(a.metric, v, fq, qq, thr_s, [&](int j) { return ccc[j]; });
           if (!qvalid || nvalid <= 0) mask = 0;
           else if (nvalid < 32) mask &= (1u << nvalid) - 1u;
           if (hbn > 0) {
@@ -649,9 +766,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       tc_fence_before();
       mbar_arrive(&acce[buf]);
       if (need_cc) mbar_arrive(&cce[buf]);
-      if (KR > 0 && __any_sync(0xffffffffu, cnt > 0)) merge_candidates(reg, cbuf, m, kBM, cnt, thr_s, desc);
     }
-    if (KR > 0 && __any_sync(0xffffffffu, cnt > 0)) merge_candidates(reg, cbuf, m, kBM, cnt, thr_s, desc);
     if (qvalid) {
       uint64_t *out = a.partial + ((size_t)blockIdx.x * a.B + qidx) * k;
       if (KR > 0) {
@@ -681,16 +796,18 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 // 64-byte swizzle), zeros for padding rows and columns; then (2^-e, ||q||,
 // ||q||^2, sum_d q_d) per query after the images.
 __device__ __forceinline__ void qprep_block(const float *__restrict__ q, int64_t B, int D,
-                                            int64_t Bpad, uint8_t *__restrict__ qA, int64_t blk) {
-  const int64_t b = blk * 8 + (threadIdx.x >> 5);
+                                            int64_t Bpad, uint8_t *__restrict__ qA, int64_t blk,
+                                            int qoff = 0) {
+  const int64_t b = blk * 8 + (threadIdx.x >> 5);  // MMA row over all query blocks
   const int lane = threadIdx.x & 31;
   if (b >= Bpad) return;
   const int nk = (D + kBK - 1) / kBK;
   const int64_t qb = b / kBM;
   const int r = (int)(b % kBM);
   float4 *qinfo = reinterpret_cast<float4 *>(qA + (size_t)(Bpad / kBM) * nk * kAStage);
-  const bool valid = b < B;
-  const float *qr = q + b * D;
+  const int64_t qi = b - qoff;  // the query of this row (qoff > 0 only with one block)
+  const bool valid = qi >= 0 && qi < B;
+  const float *qr = valid ? q + qi * D : q;
   float mx = 0.0f, qs = 0.0f;
   if (valid) {
     for (int d = lane; d < D; d += 32) {
@@ -737,14 +854,15 @@ __device__ __forceinline__ void qprep_block(const float *__restrict__ q, int64_t
     *reinterpret_cast<uint4 *>(qA + off) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
     *reinterpret_cast<uint4 *>(qA + off + kABytes) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
   }
-  if (lane == 0)
-    qinfo[b] = valid ? make_float4(ldexpf(1.0f, -e), qn, qq, qs)
-                     : make_float4(0.f, 0.f, 0.f, 0.f);
+  if (lane == 0 && qi >= 0)
+    qinfo[qi] = valid ? make_float4(ldexpf(1.0f, -e), qn, qq, qs)
+                      : make_float4(0.f, 0.f, 0.f, 0.f);
 }
 
 __global__ void __launch_bounds__(256) qprep_kernel(const float *__restrict__ q, int64_t B, int D,
-                                                    int64_t Bpad, uint8_t *__restrict__ qA) {
-  qprep_block(q, B, D, Bpad, qA, blockIdx.x);
+                                                    int64_t Bpad, uint8_t *__restrict__ qA,
+                                                    int qoff) {
+  qprep_block(q, B, D, Bpad, qA, blockIdx.x, qoff);
 }
 
 
@@ -1274,16 +1392,15 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
         tmem_ld32(taddr + c * 32, v);
         const float thr = desc ? fmaxf(thr_s, seed) : fminf(thr_s, seed);
         uint32_t mask = 0;
+        if constexpr (RC) {
 #pragma unroll
-        for (int j = 0; j < 32; ++j) {
-          float sc;
-          if constexpr (RC) {
-            sc = fac_score(rl.at(j, l2), __uint_as_float(v[j]), qf);
-          } else {
-            const float rf = __shfl_sync(0xffffffffu, rfl, j);
-            sc = tile_score(a.metric, __uint_as_float(v[j]), fq, qq, rf);
+          for (int j = 0; j < 32; ++j) {
+            const float sc = fac_score(rl.at(j, l2), __uint_as_float(v[j]), qf);
+            mask |= (uint32_t)(desc ? sc > thr : sc < thr) << j;
           }
-          mask |= (uint32_t)(desc ? sc > thr : sc < thr) << j;
+        } else {
+          mask = chunk_mask(a.metric, v, fq, qq, thr,
+                            [&](int j) { return __shfl_sync(0xffffffffu, rfl, j); });
         }
         if (!qvalid || nvalid <= 0) mask = 0;
         else if (nvalid < 32) mask &= (1u << nvalid) - 1u;
@@ -1484,11 +1601,15 @@ cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st, const RowPt
 
   if (!P.pre) {
     timing_launch_begin(LAM_TIME_AUX, st);
-    qprep_kernel<<<q_blocks, 256, 0, st>>>(a.queries, a.B, a.D, a.Bpad, qA);
+    // one block of at most 64 queries: they take MMA rows 64 .. 127, read by
+    // the epilogue warps that share the SM sub-partitions of the converters
+    // only (the producer and MMA warps sit on the other two)
+    const int qoff = a.Bpad == kBM && a.B <= kBM / 2 ? kBM / 2 : 0;
+    qprep_kernel<<<q_blocks, 256, 0, st>>>(a.queries, a.B, a.D, a.Bpad, qA, qoff);
     timing_launch_end(LAM_TIME_AUX, st);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    const TcLayout L = tc_layout(a.width, a.k);
+    const TcLayout L = tc_layout(a.width, a.k, a.metric != LAM_METRIC_IP);
     if (L.ns < 2) return cudaErrorInvalidValue;
     CUtensorMap cmap1, cmap2;  // the codes as int8 and as int16 rows
     if ((qst || a.width == 1) &&
@@ -1502,6 +1623,7 @@ cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st, const RowPt
       return cudaErrorInvalidValue;
     TcGeom g;
     g.qst = qst;
+    g.qoff = qoff;
     g.ns = L.ns;
     g.nr = L.nr;
     g.chunks = L.chunks;

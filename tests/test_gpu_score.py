@@ -62,7 +62,7 @@ def test_bandwidth_path_other_dims(dev, score_path, D):
 
 @pytest.mark.parametrize("metric", METRICS)
 @pytest.mark.parametrize("width,eps", [(1, 1e-2), (2, 1e-3), (2, 1e-4)])
-@pytest.mark.parametrize("B", [3, 16, 130, 500])
+@pytest.mark.parametrize("B", [3, 16, 64, 65, 130, 500])
 def test_tensor_path(dev, score_path, metric, width, eps, B):
     score_path("tensor")
     codes, bound = make_codes(3001, 768, eps, width, seed=B)
