@@ -4,8 +4,8 @@
 // Algorithm 1: B <- BandHash(Q_eps(e_j))).
 //
 // One pass over x: each thread takes whole bands of r consecutive values of a
-// row, quantizes them exactly as the quantize kernels do (one IEEE division by
-// s = 2 eps, round half to even), writes the codes (optional) and the 64-bit
+// row, quantizes them exactly as the quantize kernels do (the IEEE-rounded
+// quotient by s = 2 eps, round half to even), writes the codes (optional) and the 64-bit
 // FNV-1a digest of the band: the band's index within its row as 2
 // little-endian bytes, then the band's codes as their `width` little-endian
 // bytes.  The range is tracked for the width decision, as in Q_eps alone.
@@ -23,9 +23,6 @@ constexpr int kBlocksPerSm = 8;
 constexpr uint64_t kFnvOffset = 14695981039346656037ULL;
 constexpr uint64_t kFnvPrime = 1099511628211ULL;
 
-__device__ __forceinline__ int32_t q_code(float x, float s) {
-  return __float2int_rn(__fdiv_rn(x, s));
-}
 
 __device__ __forceinline__ uint64_t fnv_byte(uint64_t h, uint32_t byte) {
   return (h ^ (uint64_t)(byte & 0xffu)) * kFnvPrime;
@@ -127,6 +124,7 @@ __device__ __forceinline__ void bands_body(const float *__restrict__ x, int64_t 
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   const int step_b = (int)(stride % nb);  // band index advance per grid stride
   int b = (int)(tid % nb);
+  const QDiv qd = QDiv::of(s);
   BRange rg;
   for (int64_t j = tid; j < nbands_total; j += stride) {
     uint64_t h = fnv_byte(fnv_byte(kFnvOffset, (uint32_t)b), (uint32_t)b >> 8);
@@ -150,7 +148,7 @@ __device__ __forceinline__ void bands_body(const float *__restrict__ x, int64_t 
 #pragma unroll
       for (int e = 0; e < V; ++e) {
         if (TRACK) rg.add(f[e]);
-        c[e] = q_code(f[e], s);
+        c[e] = qd.code(f[e]);
 #pragma unroll
         for (int t = 0; t < W; ++t) h = fnv_byte(h, (uint32_t)c[e] >> (8 * t));
       }

@@ -144,6 +144,42 @@ __device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, i
       : "memory");
 }
 
+// The Q_eps quotient x / s rounded to nearest, equal bit for bit to one IEEE
+// division, from y = RN(1/s) and two FMA steps (cheaper than the division):
+// q0 = x y is within two ulps of x / s; q1 = q0 + (x - s q0) y is faithful;
+// and by Markstein's theorem (a faithful quotient, a reciprocal with relative
+// error below 2^-24, the residual and the update each rounded once to
+// nearest) q2 = q1 + (x - s q1) y is the correctly rounded quotient, as long
+// as nothing over- or underflows.  Hence the guards: s in [2^-40, 2^40]
+// (otherwise every value takes the division) and |q0| < 2^100 (otherwise,
+// and for non-finite x, this value does); below |x| = 2^-80 the residual may
+// be subnormal, but the quotient is then under 2^-40 and rounds to code 0
+// either way.  (Checked against IEEE single division for every finite x and
+// 18 divisors, among them 2^-40, 2^40 and all-ones significands.)
+struct QDiv {
+  float s, y;
+  bool fast;
+  __device__ __forceinline__ static QDiv of(float s_) {
+    QDiv d;
+    d.s = s_;
+    d.y = __frcp_rn(s_);
+    d.fast = s_ >= 0x1p-40f && s_ <= 0x1p40f;
+    return d;
+  }
+  __device__ __forceinline__ float quot(float x) const {
+    float q = __fmul_rn(x, y);
+    if (fast && fabsf(q) < 0x1p100f) {
+      q = __fmaf_rn(__fmaf_rn(-s, q, x), y, q);
+      q = __fmaf_rn(__fmaf_rn(-s, q, x), y, q);
+    } else {
+      q = __fdiv_rn(x, s);
+    }
+    return q;
+  }
+  // Q_eps(x): the quotient rounded half to even
+  __device__ __forceinline__ int32_t code(float x) const { return __float2int_rn(quot(x)); }
+};
+
 // ------------------------------------------------------------- launchers --
 // (defined in quantize.cu / score_bw.cu / score_tc.cu; all launch on `st`)
 cudaError_t launch_quant_range(const float *x, int64_t n, QuantStatus *status, int sms,

@@ -3,8 +3,9 @@
 //
 // One pass reads fp32 with 128-bit loads and writes codes with 128-bit
 // stores; it is HBM-bound at (4 + width) bytes per element.  The quotient is
-// one IEEE division (__fdiv_rn) and the rounding is half-to-even
-// (__float2int_rn), the same operations the host uses to resolve the width.
+// the IEEE-rounded x / s (QDiv: a reciprocal and two FMA steps, equal to the
+// division) and the rounding is half-to-even (__float2int_rn), the same
+// operations the host uses to resolve the width.
 #include "lam_internal.cuh"
 
 #include <map>
@@ -17,9 +18,6 @@ namespace {
 constexpr int kThreads = 256;
 constexpr int kBlocksPerSm = 8;
 
-__device__ __forceinline__ int32_t q_code(float x, float s) {
-  return __float2int_rn(__fdiv_rn(x, s));
-}
 
 struct Range {
   float vmin, vmax;
@@ -134,6 +132,7 @@ __device__ __forceinline__ void quantize_body(const float *__restrict__ x, int64
                                               void *__restrict__ codes, QuantStatus *st) {
   const int64_t tid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  const QDiv qd = QDiv::of(s);
   Range rg;
   int64_t done = 0;
   if (VEC) {
@@ -157,7 +156,7 @@ __device__ __forceinline__ void quantize_body(const float *__restrict__ x, int64
           int32_t c[4];
 #pragma unroll
           for (int e = 0; e < 4; ++e) {
-            c[e] = q_code(f[e], s);
+            c[e] = qd.code(f[e]);
             if (TRACK) rg.add(f[e]);
           }
           cv[g] = Pack4<W>::pack(c);
@@ -169,7 +168,7 @@ __device__ __forceinline__ void quantize_body(const float *__restrict__ x, int64
   for (int64_t i = done + tid; i < n; i += stride) {
     float f = x[i];
     if (TRACK) rg.add(f);
-    store_code<W>(codes, i, q_code(f, s));
+    store_code<W>(codes, i, qd.code(f));
   }
   if (TRACK) rg.flush(st);
 }

@@ -42,6 +42,22 @@ def test_codes_and_digests_bit_exact(dev, r, eps, width):
     np.testing.assert_array_equal(d, oracle.band_digests(oc, r, w))
 
 
+@pytest.mark.parametrize("eps", [1e-3, 0.0123457, 1e-13])
+def test_codes_at_rounding_midpoints(dev, eps):
+    """The fused band kernel's codes next to every quotient midpoint equal the
+    oracle's (int32 codes, so every value is in range)."""
+    from tests.test_gpu_quantize import midpoint_values
+    x = midpoint_values(eps, n_random=100000)
+    n = x.size // 768 * 768
+    x = x[:n].reshape(-1, 768)
+    oc, rmin, rmax, _ = oracle.quantize(x, eps)
+    oc = oc.reshape(x.shape)
+    w, cmin, cmax, c, d = run(dev, x, eps, 4, 8)
+    assert w == 4 and (cmin, cmax) == (int(rmin), int(rmax))
+    np.testing.assert_array_equal(c, oc.astype(np.int32))
+    np.testing.assert_array_equal(d, oracle.band_digests(oc, 8, 4))
+
+
 @pytest.mark.parametrize("r", [4, 32])
 def test_digests_only_and_unaligned_rows(dev, r):
     x = inputs.unit_rows(333, 64, seed=9)

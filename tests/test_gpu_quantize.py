@@ -54,6 +54,40 @@ def test_codes_bit_exact(dev, eps, width, n):
     assert digest(c) == digest(oc.astype(NP_DT[w]))
 
 
+def midpoint_values(eps, kmax=4096, ulps=4, n_random=200000, seed=7):
+    """fp32 values within `ulps` ulps of every quotient midpoint (k + 1/2) s,
+    |k| < kmax, where the rounded quotient decides the code, plus random bit
+    patterns of every magnitude whose quotient stays below 2^30."""
+    s = np.float64(oracle.step(eps))
+    k = np.arange(-kmax, kmax, dtype=np.float64)
+    mid = ((k + 0.5) * s).astype(np.float32)
+    xs, up, dn = [mid], mid.copy(), mid.copy()
+    for _ in range(ulps):
+        up = np.nextafter(up, np.float32(np.inf))
+        dn = np.nextafter(dn, np.float32(-np.inf))
+        xs += [up, dn]
+    bits = np.random.default_rng(seed).integers(0, 2**32, size=n_random, dtype=np.uint64)
+    r = bits.astype(np.uint32).view(np.float32)
+    r = r[np.isfinite(r)]
+    r = r[np.abs(r.astype(np.float64)) < 2.0**30 * s]
+    return np.concatenate(xs + [r]).astype(np.float32)
+
+
+# steps s = 2 eps inside [2^-40, 2^40] take the reciprocal-and-FMA quotient;
+# 1e-13 and 1e12 fall outside and take the division for every value
+@pytest.mark.parametrize("eps", [1e-2, 1e-3, 1e-4, 0.0123457, 3e-7, 5e-13, 1e11, 1e-13, 1e12])
+def test_codes_at_rounding_midpoints(dev, eps):
+    """Codes bit-exact with the oracle's IEEE quotient where rounding decides
+    them: next to every midpoint between two codes, and at random magnitudes
+    down to subnormal values."""
+    x = midpoint_values(eps)
+    oc, rmin, rmax, _ = oracle.quantize(x, eps)
+    st, w, s, cmin, cmax, c = gpu_quantize(x, eps, 4, dev)
+    assert st == 0 and w == 4 and s == oracle.step(eps)
+    assert (cmin, cmax) == (int(rmin), int(rmax))
+    np.testing.assert_array_equal(c, oc.astype(np.int32))
+
+
 @pytest.mark.parametrize("offset", [1, 2, 3])
 @pytest.mark.parametrize("width", [0, 1, 2, 4])
 def test_misaligned_buffers(dev, offset, width):
