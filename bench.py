@@ -735,11 +735,12 @@ def run_kernels(args):
         ms_forced, k_forced = timed(lambda: lam.lam_quantize(x, e, wq, codes, ws),
                                     lam.LAM_TIME_QUANTIZE)
         qb = (4 + wq) * n
-        res["quantize"].append({"eps": e, "width": wq, "ms_auto_span": ms_auto,
+        qa = (4 + w) * n  # AUTO writes the resolved width
+        res["quantize"].append({"eps": e, "width": wq, "width_auto": w, "ms_auto_span": ms_auto,
                                 "ms_auto_kernel": k_auto, "ms_forced_span": ms_forced,
                                 "ms_forced_kernel": k_forced,
-                                "gbs_auto_kernel": qb / (k_auto / 1e3) / 1e9,
-                                "frac_of_hbm_auto_kernel": qb / (k_auto / 1e3) / 1e9 / hbm,
+                                "gbs_auto_kernel": qa / (k_auto / 1e3) / 1e9,
+                                "frac_of_hbm_auto_kernel": qa / (k_auto / 1e3) / 1e9 / hbm,
                                 "gbs_forced_kernel": qb / (k_forced / 1e3) / 1e9,
                                 "frac_of_hbm_forced_kernel": qb / (k_forced / 1e3) / 1e9 / hbm})
         lam.lam_quantize(x, e, wq, codes, ws)
