@@ -45,11 +45,12 @@ __global__ void __launch_bounds__(kRowWarps * 32)
     lo = warp_min(lo);
     hi = warp_max(hi);
     const float sc = __fdiv_rn(__fsub_rn(hi, lo), 255.0f);
+    const QDiv qd = QDiv::of(sc);  // the IEEE quotient by sc, as a division gives it
     int8_t *cr = codes + r * D;
     for (int d = lane; d < D; d += 32) {
       int c = -128;
       if (sc > 0.0f) {
-        c = __float2int_rn(__fdiv_rn(__fsub_rn(xr[d], lo), sc)) - 128;
+        c = qd.code(__fsub_rn(xr[d], lo)) - 128;
         c = c < -128 ? -128 : (c > 127 ? 127 : c);
       }
       cr[d] = (int8_t)c;
@@ -86,6 +87,7 @@ __global__ void __launch_bounds__(kRowWarps * 32)
     lo = warp_min(lo);
     hi = warp_max(hi);
     const float sc = __fdiv_rn(__fsub_rn(hi, lo), 255.0f);
+    const QDiv qd = QDiv::of(sc);
     uint32_t *cr = reinterpret_cast<uint32_t *>(codes + r * D);
 #pragma unroll
     for (int j = 0; j < NCH; ++j) {
@@ -97,7 +99,7 @@ __global__ void __launch_bounds__(kRowWarps * 32)
       for (int t = 0; t < 4; ++t) {
         int c = -128;
         if (sc > 0.0f) {
-          c = __float2int_rn(__fdiv_rn(__fsub_rn(e[t], lo), sc)) - 128;
+          c = qd.code(__fsub_rn(e[t], lo)) - 128;
           c = c < -128 ? -128 : (c > 127 ? 127 : c);
         }
         packed |= ((uint32_t)c & 0xffu) << (8 * t);
