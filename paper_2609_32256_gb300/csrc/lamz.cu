@@ -61,11 +61,11 @@ constexpr int kUnrollBlocks = 8;  // blocks a warp loads ahead (memory-level par
 
 // Codes, deltas and |deltas| of the warp's block b from its value xv (lane's
 // element, loaded by the caller); returns L (0..31).
-__device__ __forceinline__ int block_deltas(float xv, int64_t n, int64_t b, float s, int lane,
+__device__ __forceinline__ int block_deltas(float xv, int64_t n, int64_t b, const QDiv &qd, int lane,
                                             int32_t &d, uint32_t &m) {
   const int64_t i = b * 32 + lane;
   const int valid = (int)min((int64_t)32, n - b * 32);
-  int32_t q = i < n ? __float2int_rn(__fdiv_rn(xv, s)) : 0;
+  int32_t q = i < n ? qd.code(xv) : 0;
   q = __shfl_sync(0xffffffffu, q, lane < valid ? lane : valid - 1);  // pad: repeat the last code
   const int32_t prev = __shfl_up_sync(0xffffffffu, q, 1);
   d = lane == 0 ? q : q - prev;
@@ -80,6 +80,7 @@ __global__ void __launch_bounds__(kCodecThreads) lamz_size_kernel(const float *_
                                                                  uint8_t *hdr, uint32_t *sizes,
                                                                  int64_t nb) {
   const float s = codec_step(st, rel);
+  const QDiv qd = QDiv::of(s);
   const int lane = threadIdx.x & 31;
   const int64_t gw = (int64_t)blockIdx.x * (kCodecThreads / 32) + (threadIdx.x >> 5);
   const int64_t nw = (int64_t)gridDim.x * (kCodecThreads / 32);
@@ -96,7 +97,7 @@ __global__ void __launch_bounds__(kCodecThreads) lamz_size_kernel(const float *_
       if (b >= nb) break;
       int32_t d;
       uint32_t m;
-      const int L = block_deltas(xv[u], n, b, s, lane, d, m);
+      const int L = block_deltas(xv[u], n, b, qd, lane, d, m);
       if (lane == 0) {
         hdr[b] = (uint8_t)L;
         sizes[b] = L > 0 ? 4u + 4u * (uint32_t)L : 0u;
@@ -115,6 +116,7 @@ __global__ void __launch_bounds__(kCodecThreads) lamz_write_kernel(
     uint64_t cap) {
   if ((__ldg(&st->flags) & kFlagNonfinite) || head + __ldg(&st->total) > cap) return;
   const float s = codec_step(st, rel);
+  const QDiv qd = QDiv::of(s);
   if (blockIdx.x == 0 && threadIdx.x == 0) {
     out[0] = 0x5A4D414Cu;  // "LAMZ" little-endian
     out[1] = (uint32_t)((uint64_t)n & 0xffffffffu);
@@ -137,7 +139,7 @@ __global__ void __launch_bounds__(kCodecThreads) lamz_write_kernel(
     if (b >= nb) break;
     int32_t d;
     uint32_t m;
-    const int L = block_deltas(xv[u], n, b, s, lane, d, m);
+    const int L = block_deltas(xv[u], n, b, qd, lane, d, m);
     if (L == 0) continue;
     uint32_t *w = payload + offs[b] / 4;
     const uint32_t sign = __ballot_sync(0xffffffffu, d < 0);

@@ -102,22 +102,6 @@ __device__ __forceinline__ float rank_key32_score(uint32_t key, bool desc) {
   return unord_f32(desc ? ~key : key);
 }
 
-// Merges `cnt` buffered candidates (entry i of this thread at buf[i * stride +
-// slot]) into the register list, every lane of the warp in step (lanes with
-// fewer candidates insert nothing), then refreshes the k-th score threshold.
-template <int KR>
-__device__ __forceinline__ void merge_candidates(RegTopK<KR> &reg, const uint2 *buf, int slot,
-                                                 int stride, int &cnt, float &thr_s, bool desc) {
-  const int mx = __reduce_max_sync(0xffffffffu, cnt);
-  for (int i = 0; i < mx; ++i) {
-    const uint2 e = i < cnt ? buf[(size_t)i * stride + slot] : make_uint2(0xffffffffu, 0xffffffffu);
-    reg.insert(e.x, e.y);
-  }
-  cnt = 0;
-  const uint32_t tk = reg.key[KR - 1];
-  thr_s = tk == 0xffffffffu ? (desc ? -INFINITY : INFINITY) : rank_key32_score(tk, desc);
-}
-
 // k-th largest of G register values (1 <= k <= G): the smallest value that
 // fewer than k values exceed.  O(G^2) compares, no stores into v.
 template <int G>
