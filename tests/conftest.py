@@ -43,3 +43,18 @@ def score_path(monkeypatch):
     def force(name):
         monkeypatch.setenv("LAM_SCORE_PATH", name)
     return force
+
+
+def pytest_terminal_summary(terminalreporter):
+    """Prints, per parity test, the largest |gpu - oracle| / tolerance of its
+    scores (1.0 would be at the tolerance)."""
+    try:
+        from tests.parity import WORST
+    except Exception:
+        return
+    if not WORST:
+        return
+    tr = terminalreporter
+    tr.section("score margin: max |gpu - oracle| / (1e-6 + 1e-5 |oracle|) per test")
+    for name, r in sorted(WORST.items(), key=lambda kv: -kv[1]):
+        tr.write_line("%8.4f  %s" % (r, name))

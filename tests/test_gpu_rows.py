@@ -174,13 +174,20 @@ def test_two_slabs_with_first_slab_bound(dev):
     x[700100:700140] = x[0:40]
     codes, scale, offset = lam.encode_rows(x, lam.LAM_ROWS_INT8)
     q = inputs.queries(200, d, seed=6)
-    q[7] = x[30].cpu().numpy()
+    x_np = x.cpu().numpy()
+    q[7] = x_np[30]
     del x
+    # the oracle encodes the same rows: codes and factors bit-exact, and its
+    # own rows feed its scores
+    oc, osc, oof = oracle.encode_rows(x_np, oracle.FMT_INT8_ROWS)
+    del x_np
+    assert np.array_equal(codes.cpu().numpy(), oc)
+    assert np.array_equal(scale.cpu().numpy().view(np.uint32), osc.view(np.uint32))
+    assert np.array_equal(offset.cpu().numpy().view(np.uint32), oof.view(np.uint32))
     gs, gi = lam.search_rows(torch.from_numpy(q).to(dev), codes, lam.LAM_ROWS_INT8, scale,
                              offset, k, oracle.L2)
     gs, gi = gs.cpu().numpy(), gi.cpu().numpy()
-    rows = oracle.decode_rows(codes.cpu().numpy(), oracle.FMT_INT8_ROWS, d,
-                              scale.cpu().numpy(), offset.cpu().numpy())
+    rows = oracle.decode_rows(oc, oracle.FMT_INT8_ROWS, d, osc, oof)
     sel = np.array([0, 7, 128, 199])
     full = oracle.scores_rows(q[sel], rows, oracle.L2)
     os_, oi = oracle.topk(full, k, oracle.L2)
