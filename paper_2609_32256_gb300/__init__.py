@@ -63,14 +63,21 @@ def dequantize(codes, scale, stream=None):
     return out
 
 
-def search(queries, codes, eps, k, metric=LAM_METRIC_IP, code_bound=0, stream=None):
-    """Top-k of every query against every code row: (scores [B,k] f32, ids [B,k] i64)."""
+def search(queries, codes, eps, k, metric=LAM_METRIC_IP, code_bound=None, stream=None):
+    """Top-k of every query against every code row: (scores [B,k] f32, ids [B,k] i64).
+
+    code_bound: the largest |code| (max(-code_min, code_max) from quantize),
+    or None.  Every int8 code is bounded by 128; for int16 codes, None means
+    unknown, and the tensor cores then score the codes split as 256 h + l
+    (exact for every int16 code, twice the tensor work of a bound <= 2048)."""
     torch = _torch()
     queries = queries.contiguous()
     codes = codes.contiguous()
     B, D = queries.shape
     N = codes.shape[0]
     w = codes.element_size()
+    if code_bound is None:
+        code_bound = 128 if w == 1 else 0
     nbytes = lam_score_topk_workspace_size(B, N, D, k, w, code_bound)
     if nbytes == 0:
         raise LamError(LAM_ERR_INVALID, "lam_score_topk_workspace_size")

@@ -83,10 +83,44 @@ bool bandwidth_ok(int64_t B, int32_t D, int32_t k, int32_t width) {
          D <= 1024 && k <= 128;
 }
 
+// int8 codes and int16 codes within +-2048 are exact fp16 operands; other
+// int16 codes take the split (256 h + l) through the converting pass.
 bool tensor_ok(int64_t B, int64_t N, int32_t D, int32_t k, int32_t width, int32_t code_bound) {
   (void)N;
-  const bool codes_exact = width == 1 || (width == 2 && code_bound > 0 && code_bound <= 2048);
-  return codes_exact && D % 16 == 0 && tensor_fits(width, k, B) && B <= (1LL << 23);
+  if (width != 1 && width != 2) return false;
+  const bool fits = tensor_wide(width, code_bound) ? tensor_fits_pre(k) : tensor_fits(width, k, B);
+  return D % 16 == 0 && fits && B <= (1LL << 23);
+}
+
+TensorPlan tensor_plan_for(int64_t B, int64_t N, int32_t D, int32_t k, int32_t width,
+                           int32_t code_bound, int sms) {
+  return tensor_wide(width, code_bound) ? tensor_plan(B, N, tensor_k_extent(D, true), k, sms, true)
+                                        : tensor_plan(B, N, D, k, sms);
+}
+
+// Test hooks of the timeout path, read from the environment at every search
+// (unset in normal use): LAM_TEST_WAIT_CYCLES=<n> gives the search's device
+// waits a budget of n SM cycles instead of ~1 s, LAM_TEST_STALL=1 makes its
+// copy producers issue nothing, so that every consumer's wait runs out.
+}  // namespace
+
+namespace lam {
+__global__ void set_test_words_kernel(uint32_t *hdr, uint32_t wait_cycles, uint32_t stall) {
+  hdr[kHdrWaitCycles] = wait_cycles;
+  hdr[kHdrStall] = stall;
+}
+}  // namespace lam
+
+namespace {
+
+cudaError_t apply_test_hooks(void *ws, cudaStream_t st) {
+  const char *w = getenv("LAM_TEST_WAIT_CYCLES");
+  const char *z = getenv("LAM_TEST_STALL");
+  const uint32_t wait_cycles = (w && *w) ? (uint32_t)strtoul(w, nullptr, 10) : 0u;
+  const uint32_t stall = (z && strcmp(z, "1") == 0) ? 1u : 0u;
+  if (wait_cycles == 0 && stall == 0) return cudaSuccess;
+  set_test_words_kernel<<<1, 1, 0, st>>>(static_cast<uint32_t *>(ws), wait_cycles, stall);
+  return cudaGetLastError();
 }
 
 // Chooses the path (or honours LAM_SCORE_PATH) and lays out the workspace:
@@ -114,14 +148,16 @@ bool make_plan(int64_t B, int64_t N, int32_t D, int32_t k, int32_t width, int32_
   }
   p->path = path;
   if (path == kPathBandwidth) p->n_lists = bandwidth_ctas(N, D, width, sms);
-  else if (path == kPathTensor) p->n_lists = tensor_plan(B, N, D, k, sms).n_lists;
+  else if (path == kPathTensor)
+    p->n_lists = tensor_plan_for(B, N, D, k, width, code_bound, sms).n_lists;
   else p->n_lists = generic_ctas(B, N, sms);
   p->Bpad = (B + 127) / 128 * 128;
   p->partial_off = kHeaderBytes;
   const size_t partial = (size_t)p->n_lists * (size_t)B * (size_t)k * 8;
   p->qprep_off = align_up(p->partial_off + partial, 256);
   p->total = p->qprep_off;
-  if (path == kPathTensor) p->total += align_up(tensor_plan(B, N, D, k, sms).bytes, 256);
+  if (path == kPathTensor)
+    p->total += align_up(tensor_plan_for(B, N, D, k, width, code_bound, sms).bytes, 256);
   return true;
 }
 
@@ -613,6 +649,7 @@ lam_status lam_score_topk(const float *queries, int64_t B, const void *codes, in
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   uint8_t *ws = static_cast<uint8_t *>(workspace);
   if (cudaMemsetAsync(ws, 0, kHeaderBytes, st) != cudaSuccess) return LAM_ERR_CUDA;
+  if (apply_test_hooks(ws, st) != cudaSuccess) return LAM_ERR_CUDA;
   ScoreArgs a;
   a.queries = queries;
   a.B = B;
@@ -744,6 +781,7 @@ lam_status lam_score_topk_rows(const float *queries, int64_t B, const void *code
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   uint8_t *ws = static_cast<uint8_t *>(workspace);
   if (cudaMemsetAsync(ws, 0, kHeaderBytes, st) != cudaSuccess) return LAM_ERR_CUDA;
+  if (apply_test_hooks(ws, st) != cudaSuccess) return LAM_ERR_CUDA;
   ScoreArgs a{};
   a.queries = queries;
   a.B = B;
@@ -896,6 +934,7 @@ lam_status lam_score_topk_from(const float *queries, int64_t B, const void *code
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   uint8_t *ws = static_cast<uint8_t *>(workspace);
   if (cudaMemsetAsync(ws, 0, kHeaderBytes, st) != cudaSuccess) return LAM_ERR_CUDA;
+  if (apply_test_hooks(ws, st) != cudaSuccess) return LAM_ERR_CUDA;
   ScoreArgs a;
   a.queries = queries;
   a.B = B;

@@ -25,6 +25,14 @@ constexpr int kHeaderBytes = 256;         // status block at the head of a works
 // Wait budget of every device-side spin: ~1 s of SM clock.
 constexpr long long kWaitCycles = 2000000000LL;
 
+// 32-bit words of a search's status header (zeroed by every call): the flags
+// above, and two test hooks the host sets only when asked to (the tests of
+// the timeout path): a wait budget in SM cycles (0: kWaitCycles) and a stall
+// word that makes the copy producers issue nothing.
+constexpr int kHdrFlags = 0;
+constexpr int kHdrWaitCycles = 2;
+constexpr int kHdrStall = 3;
+
 // Status block of lam_quantize (32 bytes, zeroed before each call).
 struct QuantStatus {
   uint32_t neg_min;   // max over inputs of ~ord(x)   (0: no finite input seen)
@@ -106,16 +114,29 @@ __device__ __forceinline__ bool mbar_try_wait_sleep(uint64_t *bar, uint32_t pari
       : "memory");
   return ok != 0;
 }
-// Bounded wait for phase `parity` of `bar`.  Gives up after kWaitCycles or as
+// The wait budget of a search: its header's test word, else kWaitCycles.
+__device__ __forceinline__ long long wait_budget(const uint32_t *gflags) {
+  const uint32_t v = gflags ? *reinterpret_cast<const volatile uint32_t *>(gflags + kHdrWaitCycles)
+                            : 0u;
+  return v ? (long long)v : kWaitCycles;
+}
+// Whether the copy producers of a search must issue nothing (test hook).
+__device__ __forceinline__ bool producers_stalled(const uint32_t *gflags) {
+  return gflags && *reinterpret_cast<const volatile uint32_t *>(gflags + kHdrStall) != 0u;
+}
+// Bounded wait for phase `parity` of `bar`.  Gives up after the search's wait
+// budget (read only once the wait has slept; ~1 s unless a test set it) or as
 // soon as *abort is set; on giving up sets *abort and the timeout flag.
 __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity,
                                           volatile int *abort, uint32_t *gflags) {
   if (mbar_try_wait(bar, parity)) return true;
   long long t0 = clock64();
+  long long budget = -1;
   while (true) {
     if (mbar_try_wait_sleep(bar, parity)) return true;
     if (*abort) return false;
-    if (clock64() - t0 > kWaitCycles) {
+    if (budget < 0) budget = wait_budget(gflags);
+    if (clock64() - t0 > budget) {
       *abort = 1;
       if (gflags) atomicOr(gflags, kFlagTimeout);
       return false;
@@ -331,6 +352,15 @@ struct TensorPlan {
 };
 // (force_pre: the per-row codecs always take the converting pass)
 TensorPlan tensor_plan(int64_t B, int64_t N, int D, int k, int sms, bool force_pre = false);
+// int16 codes the fp16 operands cannot hold exactly (a bound above 2048, or
+// no bound given): the tensor path splits each code as 256 h + l, two exact
+// fp16 values, and converts with the separate pass over 2 D image columns.
+inline bool tensor_wide(int width, int code_bound) {
+  return width == 2 && !(code_bound > 0 && code_bound <= 2048);
+}
+// K extent of the tensor path's operand images: D, or for the split two
+// image chunks per 32-wide K chunk of the codes (D rounded up to 32, doubled).
+inline int tensor_k_extent(int D, bool wide) { return wide ? 2 * ((D + 31) / 32 * 32) : D; }
 
 // Synchronous read-back of a small device status block into host memory:
 // queued on `st`, then waits for `st`.

@@ -152,7 +152,8 @@ __global__ void __launch_bounds__(kBwThreads, 1)
     // ---------------- producer: one lane issues the bulk copies ----------
     if (lane == 0) {
       int issued = 0;
-      for (int t = 0; t < ntiles; ++t) {
+      const int nt = producers_stalled(a.gflags) ? 0 : ntiles;
+      for (int t = 0; t < nt; ++t) {
         const int s = t % ns, r = t / ns;
         if (r > 0 && !mbar_wait(&empty[s], (r - 1) & 1, abort_flag, a.gflags)) break;
         const int64_t nr = min((int64_t)tr, nrows - (int64_t)t * tr);
@@ -431,7 +432,8 @@ __global__ void __launch_bounds__(kBwThreads, 1)
   if (warp == kBwWarps) {
     if (lane == 0) {
       int issued = 0;
-      for (int t = 0; t < ntiles; ++t) {
+      const int nt = producers_stalled(a.gflags) ? 0 : ntiles;
+      for (int t = 0; t < nt; ++t) {
         const int s = t % ns, r = t / ns;
         if (r > 0 && !mbar_wait(&empty[s], (r - 1) & 1, abort_flag, a.gflags)) break;
         const int64_t nr = min((int64_t)tr, nrows - (int64_t)t * tr);

@@ -41,6 +41,7 @@ namespace {
 constexpr int kBM = 128;        // queries per CTA (MMA M)
 constexpr int kBN = 256;        // code rows per tile (MMA N)
 constexpr int kBK = 32;         // fp16 per stage along D (64-byte rows)
+static_assert(kBK == 32, "tensor_k_extent (lam_internal.cuh) rounds D to 32-wide K chunks");
 constexpr int kUmmaK = 16;      // K of one kind::f16 MMA
 constexpr int kTcThreads = 352;  // 11 warps, roles below
 constexpr int kConvThreads = 128;
@@ -390,7 +391,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     if (lane == 0) {
       // raw code stages, freed by the converters
       const int rpt = (nk + R - 1) / R;  // raw stages per tile
-      const int r_total = ntl * rpt;
+      const int r_total = producers_stalled(a.gflags) ? 0 : ntl * rpt;
       int gr = 0;
       for (; gr < r_total; ++gr) {
         const int rs = gr % nr, rr = gr / nr;
@@ -599,7 +600,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     if (lane == 0) {
       // the query blocks of the MMA stages, freed by the MMAs
       const int spt = (nk + C - 1) / C;  // MMA stages per tile
-      const int a_total = ntl * spt;
+      const int a_total = producers_stalled(a.gflags) ? 0 : ntl * spt;
       int it = 0;
       for (; it < a_total; ++it) {
         const int s = it % ns, r = it / ns;
@@ -794,14 +795,16 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 // stages load (per query block and 32-wide K slice: [hi 128 x 64 B | lo], rows
 // 64 bytes apart with the 16-byte chunks of row r XOR-ed by (r >> 1) & 3, the
 // 64-byte swizzle), zeros for padding rows and columns; then (2^-e, ||q||,
-// ||q||^2, sum_d q_d) per query after the images.
+// ||q||^2, sum_d q_d) per query after the images.  With dup = 2 (int16 codes
+// split as 256 h + l, two K chunks per 32 coordinates) every K slice of the
+// query is written twice, as image chunks 2 j and 2 j + 1.
 __device__ __forceinline__ void qprep_block(const float *__restrict__ q, int64_t B, int D,
                                             int64_t Bpad, uint8_t *__restrict__ qA, int64_t blk,
-                                            int qoff = 0) {
+                                            int qoff = 0, int dup = 1) {
   const int64_t b = blk * 8 + (threadIdx.x >> 5);  // MMA row over all query blocks
   const int lane = threadIdx.x & 31;
   if (b >= Bpad) return;
-  const int nk = (D + kBK - 1) / kBK;
+  const int nk = (D + kBK - 1) / kBK * dup;
   const int64_t qb = b / kBM;
   const int r = (int)(b % kBM);
   float4 *qinfo = reinterpret_cast<float4 *>(qA + (size_t)(Bpad / kBM) * nk * kAStage);
@@ -836,7 +839,8 @@ __device__ __forceinline__ void qprep_block(const float *__restrict__ q, int64_t
   const float qn = sqrtf(ss) / ns, qq = qn * qn;
   // lane writes whole 16-byte chunks (8 fp16) of the hi and lo images
   for (int ch = lane; ch < nk * (kBK / 8); ch += 32) {
-    const int d0 = ch * 8, kc = d0 / kBK, c16 = (d0 % kBK) / 8;
+    const int kc = ch / (kBK / 8), c16 = ch % (kBK / 8);
+    const int d0 = (kc / dup) * kBK + c16 * 8;  // the query coordinates of this piece
     uint32_t hw[4], lw[4];
 #pragma unroll
     for (int t = 0; t < 4; ++t) {
@@ -885,12 +889,20 @@ constexpr int kTc2Chunks = 2;
 // at piece j ^ ((r >> 1) & 3)), so that one bulk copy stages it.  Rows past
 // nrows and columns past D are zero.  Also the per-row factor rowf (1/||c|| for
 // cosine, s^2 ||c||^2 for L2).  One warp per row of the padded slab.
+//
+// Wide (int16 codes beyond +-2048, or no known bound): each code is split as
+// c = 256 h + l with h = c >> 8 in [-128, 127] and l = c & 255 in [0, 255];
+// 256 h and l are both exact in fp16.  K chunk j of the codes becomes image
+// chunks 2 j (the 256 h values) and 2 j + 1 (the l values), and the query
+// image repeats each K slice (qprep_block with dup = 2), so the scoring
+// kernel runs unchanged over 2 D columns: q . c = q . (256 h) + q . l, every
+// product exact in fp32 (11 x 8 significant bits at most).
 template <int W>
 __device__ __forceinline__ void convert_block(const void *__restrict__ codes, int64_t row_base,
                                               int64_t nrows, int64_t nrows_pad, int D,
                                               uint8_t *__restrict__ out,
                                               float *__restrict__ rowf, int metric, float s,
-                                              uint32_t *gflags, int64_t blk) {
+                                              uint32_t *gflags, int64_t blk, bool wide = false) {
   const int64_t r = blk * 8 + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (r >= nrows_pad) return;
@@ -898,7 +910,7 @@ __device__ __forceinline__ void convert_block(const void *__restrict__ codes, in
   const int nk = (D + kBK - 1) / kBK;
   const int rr = (int)(r % kBN);
   const int sw = (rr >> 1) & 3;
-  uint8_t *dst = out + (size_t)(r / kBN) * nk * kB16Bytes + (size_t)rr * 64;
+  uint8_t *dst = out + (size_t)(r / kBN) * nk * (wide ? 2 : 1) * kB16Bytes + (size_t)rr * 64;
   const uint8_t *src = static_cast<const uint8_t *>(codes) + (row_base + r) * (int64_t)D * W;
   float cc = 0.0f, amax = 0.0f;
   for (int ch = lane; ch < nk * (kBK / 8); ch += 32) {
@@ -919,19 +931,34 @@ __device__ __forceinline__ void convert_block(const void *__restrict__ codes, in
       }
     }
     uint32_t o[4];
+    const size_t piece = (size_t)(((ch & 3) ^ sw) << 4);
+    if (W == 2 && wide) {
+      uint32_t ol[4];
+#pragma unroll
+      for (int t = 0; t < 4; ++t) {
+        cc = fmaf(f[2 * t], f[2 * t], fmaf(f[2 * t + 1], f[2 * t + 1], cc));
+        const int c0 = (int)f[2 * t], c1 = (int)f[2 * t + 1];
+        o[t] = h2_as_u32(__floats2half2_rn((float)((c0 >> 8) * 256), (float)((c1 >> 8) * 256)));
+        ol[t] = h2_as_u32(__floats2half2_rn((float)(c0 & 255), (float)(c1 & 255)));
+      }
+      uint8_t *d2 = dst + (size_t)(ch >> 2) * 2 * kB16Bytes + piece;
+      *reinterpret_cast<uint4 *>(d2) = make_uint4(o[0], o[1], o[2], o[3]);
+      *reinterpret_cast<uint4 *>(d2 + kB16Bytes) = make_uint4(ol[0], ol[1], ol[2], ol[3]);
+      continue;
+    }
 #pragma unroll
     for (int t = 0; t < 4; ++t) {
       amax = fmaxf(amax, fmaxf(fabsf(f[2 * t]), fabsf(f[2 * t + 1])));
       cc = fmaf(f[2 * t], f[2 * t], fmaf(f[2 * t + 1], f[2 * t + 1], cc));
       o[t] = h2_as_u32(__floats2half2_rn(f[2 * t], f[2 * t + 1]));
     }
-    *reinterpret_cast<uint4 *>(dst + (size_t)(ch >> 2) * kB16Bytes + (((ch & 3) ^ sw) << 4)) =
+    *reinterpret_cast<uint4 *>(dst + (size_t)(ch >> 2) * kB16Bytes + piece) =
         make_uint4(o[0], o[1], o[2], o[3]);
   }
   cc = warp_sum_tc(cc);
   if (lane == 0 && valid && metric != LAM_METRIC_IP)
     rowf[r] = metric == LAM_METRIC_COSINE ? (cc > 0.0f ? 1.0f / sqrtf(cc) : 0.0f) : s * s * cc;
-  if (W == 2 && amax > 2048.0f) atomicOr(gflags, kFlagRange);
+  if (W == 2 && !wide && amax > 2048.0f) atomicOr(gflags, kFlagRange);
 }
 
 // (qst: status-driven calls launch both widths; only the codes' width converts)
@@ -946,9 +973,11 @@ __global__ void __launch_bounds__(256) convert_codes_kernel(const void *__restri
                                                             uint8_t *__restrict__ out,
                                                             float *__restrict__ rowf, int metric,
                                                             float s, uint32_t *gflags,
-                                                            const QuantStatus *qst) {
+                                                            const QuantStatus *qst,
+                                                            int wide = 0) {
   if (!width_gate(qst, W)) return;
-  convert_block<W>(codes, row_base, nrows, nrows_pad, D, out, rowf, metric, s, gflags, blockIdx.x);
+  convert_block<W>(codes, row_base, nrows, nrows_pad, D, out, rowf, metric, s, gflags, blockIdx.x,
+                   wide != 0);
 }
 
 // Query preparation and the first slab's conversion in one launch: blocks
@@ -958,12 +987,12 @@ __global__ void __launch_bounds__(256) prep_convert_kernel(
     const float *__restrict__ q, int64_t B, int D, int64_t Bpad, uint8_t *__restrict__ qA,
     unsigned q_blocks, const void *__restrict__ codes, int64_t nrows, int64_t nrows_pad,
     uint8_t *__restrict__ out, float *__restrict__ rowf, int metric, float s, uint32_t *gflags,
-    const QuantStatus *qst) {
+    const QuantStatus *qst, int wide = 0) {
   if (blockIdx.x < q_blocks)
-    qprep_block(q, B, D, Bpad, qA, blockIdx.x);
+    qprep_block(q, B, D, Bpad, qA, blockIdx.x, 0, wide ? 2 : 1);
   else if (width_gate(qst, W))
     convert_block<W>(codes, 0, nrows, nrows_pad, D, out, rowf, metric, s, gflags,
-                     blockIdx.x - q_blocks);
+                     blockIdx.x - q_blocks, wide != 0);
 }
 
 // Status-driven calls: one launch converts at the width the quantize status
@@ -1232,7 +1261,7 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
     // ------------------------------------------------ producer -----------
     if (lane == 0) {
       int it = 0, issued = 0;
-      bool ok = true;
+      bool ok = !producers_stalled(a.gflags);
       for (int lt = 0; lt < ntl && ok; ++lt) {
         const int tile = (int)(tb + lt);
         for (int kc = 0; kc < nk; kc += C, ++it) {
@@ -1593,7 +1622,10 @@ cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st, const RowPt
   // status-driven call (codes' width on the device): both widths launch, one works
   const QuantStatus *qst = rc ? nullptr : rp.qst;
   if (a.k > kTcMaxK || (!rc && !qst && a.width != 1 && a.width != 2)) return cudaErrorInvalidValue;
-  const TensorPlan P = tensor_plan(a.B, a.N, a.D, a.k, a.sms, rc);
+  // int16 codes split as 256 h + l: the operand images span 2 D columns
+  const bool wide = !rc && !qst && tensor_wide(a.width, a.code_bound);
+  const int Dk = tensor_k_extent(a.D, wide);
+  const TensorPlan P = tensor_plan(a.B, a.N, Dk, a.k, a.sms, rc || wide);
   if (P.n_lists != a.n_lists) return cudaErrorInvalidValue;
   uint8_t *qA = static_cast<uint8_t *>(a.qprep);
   const unsigned q_blocks = (unsigned)((a.Bpad + 7) / 8);
@@ -1727,13 +1759,14 @@ cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st, const RowPt
       else
         prep_convert_kernel<2><<<q_blocks + cg, 256, 0, st>>>(
             a.queries, a.B, a.D, a.Bpad, qA, q_blocks, a.codes, nrows, nrows_pad, f16, rowf,
-            a.metric, a.s, a.gflags, nullptr);
+            a.metric, a.s, a.gflags, nullptr, wide ? 1 : 0);
     } else if (a.width == 1) {
       convert_codes_kernel<1><<<cg, 256, 0, st>>>(a.codes, row_base, nrows, nrows_pad, a.D, f16,
                                                   rowf, a.metric, a.s, a.gflags, nullptr);
     } else {
       convert_codes_kernel<2><<<cg, 256, 0, st>>>(a.codes, row_base, nrows, nrows_pad, a.D, f16,
-                                                  rowf, a.metric, a.s, a.gflags, nullptr);
+                                                  rowf, a.metric, a.s, a.gflags, nullptr,
+                                                  wide ? 1 : 0);
     }
     timing_launch_end(LAM_TIME_AUX, st);
     e = cudaGetLastError();
@@ -1742,7 +1775,9 @@ cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st, const RowPt
     g.nrows = nrows;
     g.list_base = j * P.nsplit;
     timing_launch_begin(LAM_TIME_SCORE, st);
-    kern<<<grid, kTc2Threads, L.smem_bytes, st>>>(a, g);
+    ScoreArgs ak = a;  // the kernel sees the K extent of the operand images
+    ak.D = Dk;
+    kern<<<grid, kTc2Threads, L.smem_bytes, st>>>(ak, g);
     timing_launch_end(LAM_TIME_SCORE, st);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;

@@ -1,6 +1,8 @@
 """Exact search on the codes (dequantisation fused into the score, then top-k)
 against the CPU oracle, per kernel path, metric, width and shape, including
 ragged tiles, ragged query blocks, planted exact ties and error statuses."""
+import hashlib
+
 import numpy as np
 import pytest
 import torch
@@ -8,7 +10,7 @@ import torch
 import oracle
 import paper_2609_32256_gb300 as lam
 from paper_2609_32256_gb300 import inputs
-from tests.parity import check_topk, oracle_topk
+from tests.parity import check_topk, oracle_topk, quantize_rows
 
 pytestmark = pytest.mark.gpu
 METRICS = (oracle.IP, oracle.COSINE, oracle.L2)
@@ -110,10 +112,48 @@ def test_exact_ties_rank_lower_id_first(dev, score_path, path, B):
 def test_auto_selects_paths(dev):
     assert lam.lam_score_topk_path(1, 361802, 768, 10, 2, 120) == lam.PATH_BANDWIDTH
     assert lam.lam_score_topk_path(64, 361802, 768, 10, 2, 120) == lam.PATH_TENSOR
-    assert lam.lam_score_topk_path(64, 361802, 768, 10, 2, 0) == lam.PATH_GENERIC
-    assert lam.lam_score_topk_path(64, 361802, 768, 10, 2, 4000) == lam.PATH_GENERIC
+    # int16 codes with no bound, or beyond 2048, take the split (256 h + l) tensor path
+    assert lam.lam_score_topk_path(64, 361802, 768, 10, 2, 0) == lam.PATH_TENSOR
+    assert lam.lam_score_topk_path(64, 361802, 768, 10, 2, 4000) == lam.PATH_TENSOR
+    assert lam.lam_score_topk_path(64, 361802, 768, 10, 4, 0) == lam.PATH_GENERIC
+    assert (lam.lam_score_topk_workspace_size(64, 361802, 768, 10, 2, 4000) >
+            lam.lam_score_topk_workspace_size(64, 361802, 768, 10, 2, 120))
     assert lam.lam_score_topk_path(256, 8388608, 768, 100, 1, 0) == lam.PATH_TENSOR
     assert lam.lam_score_topk_path(4, 1000, 768, 500, 1, 0) == lam.PATH_GENERIC
+
+
+@pytest.mark.parametrize("metric", METRICS)
+@pytest.mark.parametrize("B", [3, 64, 130, 520])
+@pytest.mark.parametrize("eps,known", [(2e-5, True), (2e-5, False), (1e-3, False)])
+def test_tensor_path_int16_split(dev, score_path, metric, B, eps, known):
+    """int16 codes the fp16 operands cannot hold (|c| up to ~8,000 at eps=2e-5),
+    or with no bound given: the tensor path splits each code as 256 h + l."""
+    score_path("tensor")
+    codes, bound = make_codes(2500, 768, eps, 2, seed=B + 7)
+    assert (bound > 2048) == (eps == 2e-5)
+    cb = bound if known else 0
+    assert lam.lam_score_topk_path(B, 2500, 768, 10, 2, cb) == lam.PATH_TENSOR
+    q = inputs.queries(B, 768, seed=B + 8)
+    check(dev, q, codes, 2, eps, 10, metric, cb)
+
+
+@pytest.mark.parametrize("k", [1, 32, 100])
+def test_tensor_path_int16_full_range(dev, score_path, k):
+    """Codes spanning the whole int16 range (the largest |c| = 32767 and
+    -32768), ragged tile and query block, D not a multiple of 32."""
+    score_path("tensor")
+    n, d = 1300, 272
+    x = inputs.unit_rows(n, d, seed=k)
+    x[5, 7] = 0.999
+    x[9, 3] = -0.999
+    eps = float(np.float32(0.999 / 2 / 32767.4))
+    oc, rmin, rmax, _ = oracle.quantize(x, eps)
+    assert oracle.width(rmin, rmax) == 2 and max(-rmin, rmax) >= 32767
+    codes = oc.reshape(n, d)
+    codes[11, :] = -32768
+    q = inputs.queries(140, d, seed=k + 1)
+    for metric in METRICS:
+        check(dev, q, codes, 2, eps, k, metric, 0)
 
 
 def test_forced_path_unsupported(dev, score_path):
@@ -187,16 +227,21 @@ def test_tensor_two_slabs_with_first_slab_bound(dev, score_path, metric, k):
     ws = torch.zeros(64, dtype=torch.uint8, device=dev)
     st, w, scale, cmin, cmax = lam.lam_quantize(x, eps, 1, codes, ws)
     assert st == 0 and w == 1
+    # the oracle quantizes the same rows: every code bit-exact, and its own
+    # codes feed its search
+    oc, rmin, rmax, nnf = quantize_rows(x.cpu().numpy(), eps)
     del x
+    assert nnf == 0 and (cmin, cmax) == (int(rmin), int(rmax))
+    assert hashlib.sha256(codes.cpu().numpy().tobytes()).hexdigest() == \
+        hashlib.sha256(oc.astype(np.int8).tobytes()).hexdigest()
     q = inputs.queries(520, d, seed=5)  # five query blocks: the conversion pass, in slabs
     # plant queries equal to duplicated rows so that the ties reach the top-k
-    q[3] = (codes[20].float() * scale).cpu().numpy()
-    q[129] = (codes[45].float() * scale).cpu().numpy()
+    q[3] = oracle.dequantize(oc[20], scale)
+    q[129] = oracle.dequantize(oc[45], scale)
     gs, gi = lam.search(torch.from_numpy(q).to(dev), codes, eps, k, metric,
                         code_bound=max(-cmin, cmax))
     gs, gi = gs.cpu().numpy(), gi.cpu().numpy()
     sel = np.array([0, 3, 129, 257, 519])
-    oc = codes.cpu().numpy().astype(np.int32)
     os_, oi = oracle_topk(q[sel], oc, eps, metric, k)
     check_topk(gs[sel], gi[sel], q[sel], oc, eps, metric, os_, oi)
 
