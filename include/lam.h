@@ -379,8 +379,10 @@ lam_status lam_score_topk_rows(const float *queries, int64_t B, const void *code
 
 /*
  * Waits for `stream`, then reads the device status the last lam_score_topk
- * on this workspace recorded: LAM_OK, LAM_ERR_RANGE or LAM_ERR_TIMEOUT
- * (written to *status_out).  Returns LAM_ERR_CUDA if the read fails.
+ * on this workspace recorded: LAM_OK, LAM_ERR_RANGE, LAM_ERR_TIMEOUT, or
+ * LAM_ERR_UNSUPPORTED when a lam_score_topk_from found an error or width 4 in
+ * its quantize status (written to *status_out).  Returns LAM_ERR_CUDA if the
+ * read fails.
  */
 lam_status lam_score_topk_status(const void *workspace, lam_stream_t stream,
                                  int32_t *status_out);
@@ -461,18 +463,24 @@ lam_status lam_timing_end(void);
  * other allocating routine.
  *
  * Limits and behaviour:
- *   - Shapes whose lam_score_topk_workspace_size exceeds 16 MiB (16777216
- *     bytes) return LAM_ERR_WORKSPACE without queuing anything.
- *   - The first call on a device looks up the array's device address (once
- *     per device, with that device current); make that first call before any
- *     stream capture begins.
+ *   - Arguments, the path forced by LAM_SCORE_PATH and the shape are checked
+ *     exactly as lam_score_topk checks them, with the same statuses
+ *     (LAM_ERR_INVALID, LAM_ERR_UNSUPPORTED, LAM_ERR_CUDA).  Shapes whose
+ *     search needs more than 16 MiB (16777216 bytes) of scratch return
+ *     LAM_ERR_WORKSPACE; in every such case nothing is queued.
+ *   - The scratch belongs to the current device: `stream` must be a stream of
+ *     the current device (or NULL).
+ *   - The array's device address is looked up (cudaGetSymbolAddress, with the
+ *     device current) on the first call in each CUDA context on a device, and
+ *     again after that context changed (e.g. cudaDeviceReset); make the first
+ *     call on a device before any stream capture begins.
  *   - All calls share the one array, which keeps the last call's contents;
  *     the status word is cleared at the start of every call.  Calls that
  *     overlap on the GPU (other streams, other host threads) race on it and
  *     must be serialised by the caller.
  *   - Synchronous on `stream`: it waits for the search and returns the device
- *     status (LAM_ERR_RANGE or LAM_ERR_TIMEOUT as lam_score_topk_status would
- *     report them) as its own return value.
+ *     status as its own return value: LAM_ERR_RANGE, LAM_ERR_TIMEOUT or
+ *     LAM_ERR_UNSUPPORTED as lam_score_topk_status would report them.
  */
 lam_status lam_score_topk_noalloc(const float *queries, int64_t B,
                                   const void *codes, int32_t width, int64_t N,

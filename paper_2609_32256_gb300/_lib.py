@@ -269,11 +269,13 @@ def lam_score_topk_noalloc(queries, codes, width, N, D, eps, code_bound, k, metr
                            stream=None):
     """lam_score_topk for callers that cannot allocate: scratch lives in a fixed
     16 MiB device array inside the library (synchronous; see include/lam.h)."""
+    import torch
     B = queries.shape[0]
-    st = load().lam_score_topk_noalloc(_ptr(queries), int(B), _ptr(codes), int(width), int(N),
-                                       int(D), ctypes.c_float(eps), int(code_bound), int(k),
-                                       int(metric), _ptr(scores), _ptr(ids),
-                                       _stream(stream, queries.device))
+    with torch.cuda.device(queries.device):  # the scratch is the current device's
+        st = load().lam_score_topk_noalloc(_ptr(queries), int(B), _ptr(codes), int(width),
+                                           int(N), int(D), ctypes.c_float(eps), int(code_bound),
+                                           int(k), int(metric), _ptr(scores), _ptr(ids),
+                                           _stream(stream, queries.device))
     _check(st, "lam_score_topk_noalloc")
 
 
