@@ -492,7 +492,7 @@ void lam_oracle_scores_rows(const float *queries, int64_t B, const float *rows, 
   }
 }
 
-/* Score of one query against one dequantised row, in double, rounded to fp32. *//* Score of one query against one dequantised row, in double, rounded to fp32. *//* Score of one query against one dequantised row, in double, rounded to fp32. *//* Score of one query against one dequantised row, in double, rounded to fp32. *//* Score of one query against one dequantised row, in double, rounded to fp32. */
+/* Score of one query against one dequantised row, in double, rounded to fp32. */
 static float score_one(const float *q, const int32_t *c, int32_t D, float s,
                        int metric) {
   if (metric == ORACLE_IP) {
