@@ -21,6 +21,7 @@ namespace {
 constexpr int kBwWarps = 16;  // consumer warps; each scores two rows at a time
 constexpr int kBwThreads = (kBwWarps + 1) * 32;
 constexpr int kNchMax = 4;  // 8-coordinate vectors per lane per row: D <= 1024
+constexpr int kRg = 4;      // rows per warp pass of the int8 single-query consumer
 constexpr int kBwStageTarget = 48 * 1024;
 constexpr int kBwSmemBudget = 200 * 1024;
 
@@ -86,6 +87,34 @@ __device__ __forceinline__ float pair_sum(float a, float b, int lane) {
 #pragma unroll
   for (int off = 8; off > 0; off >>= 1) keep += __shfl_xor_sync(0xffffffffu, keep, off);
   return keep;
+}
+
+// Warp sums of V values at once (V a power of two, <= 32): at each butterfly
+// step a lane keeps one half of its values and sends the other half, so the
+// V sums cost V - 1 + (5 - log2 V) shuffles instead of 5 V.  Afterwards lane L
+// holds the warp total of value L >> (5 - log2 V).
+template <int V>
+__device__ __forceinline__ float warp_sums_transposed(float (&v)[V], int lane) {
+  int n = V;
+#pragma unroll
+  for (int o = 16; o >= 1; o >>= 1) {
+    if (n > 1) {
+      const int h = n / 2;
+      const bool up = (lane & o) != 0;
+#pragma unroll
+      for (int i = 0; i < V / 2; ++i) {
+        if (i < h) {
+          const float send = up ? v[i] : v[i + h];
+          const float keep = up ? v[i + h] : v[i];
+          v[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+        }
+      }
+      n = h;
+    } else {
+      v[0] += __shfl_xor_sync(0xffffffffu, v[0], o);
+    }
+  }
+  return v[0];
 }
 
 // Waits (bounded, ignoring the abort flag) until a phase that is known to be
@@ -268,6 +297,67 @@ __global__ void __launch_bounds__(kBwThreads, 1)
       if (!mbar_wait(&full[st], r & 1, abort_flag, a.gflags)) break;
       const int nr = (int)min((int64_t)tr, nrows - (int64_t)t * tr);
       const uint8_t *stage = smem + (size_t)st * stage_bytes;
+      if constexpr (W == 1 && QB == 1) {
+        // int8 codes, one query: kRg consecutive rows per warp pass.  All
+        // their code words are loaded first, each lane sums its integer dot
+        // products per row, and one transposed butterfly gives every row's
+        // totals (and sum c^2) to its own lanes, which finish the scores in
+        // parallel; one ballot then admits rows into the warp's list in row
+        // order.
+        constexpr int V = CC ? 2 * kRg : kRg;
+        constexpr int lsh = CC ? 2 : 3;  // lane L ends with value L >> lsh
+        for (int g0 = warp * kRg; g0 < nr; g0 += kBwWarps * kRg) {
+          uint2 cw[kRg][kNchMax];
+#pragma unroll
+          for (int i = 0; i < kRg; ++i) {
+            const uint8_t *pr = stage + (size_t)min(g0 + i, nr - 1) * row_bytes;
+#pragma unroll
+            for (int j = 0; j < kNchMax; ++j) {
+              const int e0 = (j * 32 + lane) * 8;
+              cw[i][j] = (j < nch && e0 < D) ? *reinterpret_cast<const uint2 *>(pr + e0)
+                                             : make_uint2(0u, 0u);
+            }
+          }
+          float v[V];
+#pragma unroll
+          for (int i = 0; i < kRg; ++i) {
+            int d0 = 0, d1 = 0, d2 = 0, cc = 0;
+#pragma unroll
+            for (int j = 0; j < kNchMax; ++j) {
+              if (j < nch) {  // (warp-uniform)
+                const int wx = (int)cw[i][j].x, wy = (int)cw[i][j].y;
+                d0 = __dp4a(wx, (int)qdig[0][j][0][0], __dp4a(wy, (int)qdig[0][j][0][1], d0));
+                d1 = __dp4a(wx, (int)qdig[0][j][1][0], __dp4a(wy, (int)qdig[0][j][1][1], d1));
+                d2 = __dp4a(wx, (int)qdig[0][j][2][0], __dp4a(wy, (int)qdig[0][j][2][1], d2));
+                if constexpr (CC) cc = __dp4a(wx, wx, __dp4a(wy, wy, cc));
+              }
+            }
+            v[i] = fmaf((float)d0, 65536.0f, fmaf((float)d1, 256.0f, (float)d2));
+            if constexpr (CC) v[kRg + i] = (float)cc;
+          }
+          const float tot = warp_sums_transposed<V>(v, lane);
+          const int i_row = (lane >> lsh) & (kRg - 1);
+          const float cc = CC ? __shfl_xor_sync(0xffffffffu, tot, 16) : 0.0f;
+          const float sc = finish_score(a.metric, tot * qinv[0], cc, s, s2, qq[0], qn[0]);
+          const bool leader = (lane & ((1 << lsh) - 1)) == 0 && (!CC || lane < 16);
+          unsigned pass = __ballot_sync(0xffffffffu, leader && g0 + i_row < nr &&
+                                                         (desc ? sc > thr_s[0] : sc < thr_s[0]));
+          while (pass) {
+            const int l = __ffs(pass) - 1;
+            pass &= pass - 1;
+            const float sl = __shfl_sync(0xffffffffu, sc, l);
+            if (!(desc ? sl > thr_s[0] : sl < thr_s[0])) continue;  // the list moved on
+            const int64_t row = r0 + (int64_t)t * tr + g0 + ((l >> lsh) & (kRg - 1));
+            lists[0].insert(make_key(sl, (uint32_t)row, desc), lane);
+            const uint64_t kk = lists[0].kth(a.k);
+            thr_s[0] = kk == kSentinel ? (desc ? -INFINITY : INFINITY)
+                                       : rank_key32_score((uint32_t)(kk >> 32), desc);
+          }
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&empty[st]);
+        continue;
+      }
       for (int rr = warp; rr < nr; rr += 2 * kBwWarps) {
         const int rb = rr + kBwWarps;
         const bool has_b = rb < nr;
