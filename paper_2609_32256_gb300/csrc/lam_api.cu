@@ -2,6 +2,7 @@
 // scoring path and its workspace, and the launches.  The library allocates no
 // device memory; its only state is a per-device cache of the SM count.
 #include <math.h>
+#include <stdio.h>
 #include <stdlib.h>
 #include <string.h>
 
@@ -98,28 +99,42 @@ TensorPlan tensor_plan_for(int64_t B, int64_t N, int32_t D, int32_t k, int32_t w
                                         : tensor_plan(B, N, D, k, sms);
 }
 
-// Test hooks of the timeout path, read from the environment at every search
-// (unset in normal use): LAM_TEST_WAIT_CYCLES=<n> gives the search's device
-// waits a budget of n SM cycles instead of ~1 s, LAM_TEST_STALL=1 makes its
-// copy producers issue nothing, so that every consumer's wait runs out.
+// Test hooks, read from the environment at every search (unset in normal
+// use): LAM_TEST_WAIT_CYCLES=<n> gives the search's device waits a budget of
+// n SM cycles instead of ~1 s and LAM_TEST_STALL=1 makes its copy producers
+// issue nothing, so that every consumer's wait runs out (the timeout path);
+// LAM_TEST_HI_FAIL=1 makes the certifying merge of a two-pass tensor search
+// reject every query, so that the gated full pass runs.
 }  // namespace
 
 namespace lam {
-__global__ void set_test_words_kernel(uint32_t *hdr, uint32_t wait_cycles, uint32_t stall) {
+__global__ void set_test_words_kernel(uint32_t *hdr, uint32_t wait_cycles, uint32_t stall,
+                                      uint32_t force_fail) {
   hdr[kHdrWaitCycles] = wait_cycles;
   hdr[kHdrStall] = stall;
+  hdr[kHdrForceFail] = force_fail;
 }
 }  // namespace lam
 
 namespace {
 
+// LAM_DEBUG=1: the CUDA error behind a LAM_ERR_CUDA, on stderr.
+void debug_report(const char *where, cudaError_t e) {
+  const char *d = getenv("LAM_DEBUG");
+  if (d != nullptr && strcmp(d, "1") == 0)
+    fprintf(stderr, "%s: %s (%d)\n", where, cudaGetErrorString(e), (int)e);
+}
+
 cudaError_t apply_test_hooks(void *ws, cudaStream_t st) {
   const char *w = getenv("LAM_TEST_WAIT_CYCLES");
   const char *z = getenv("LAM_TEST_STALL");
+  const char *f = getenv("LAM_TEST_HI_FAIL");
   const uint32_t wait_cycles = (w && *w) ? (uint32_t)strtoul(w, nullptr, 10) : 0u;
   const uint32_t stall = (z && strcmp(z, "1") == 0) ? 1u : 0u;
-  if (wait_cycles == 0 && stall == 0) return cudaSuccess;
-  set_test_words_kernel<<<1, 1, 0, st>>>(static_cast<uint32_t *>(ws), wait_cycles, stall);
+  const uint32_t force_fail = (f && strcmp(f, "1") == 0) ? 1u : 0u;
+  if (wait_cycles == 0 && stall == 0 && force_fail == 0) return cudaSuccess;
+  set_test_words_kernel<<<1, 1, 0, st>>>(static_cast<uint32_t *>(ws), wait_cycles, stall,
+                                         force_fail);
   return cudaGetLastError();
 }
 
@@ -153,7 +168,10 @@ bool make_plan(int64_t B, int64_t N, int32_t D, int32_t k, int32_t width, int32_
   else p->n_lists = generic_ctas(B, N, sms);
   p->Bpad = (B + 127) / 128 * 128;
   p->partial_off = kHeaderBytes;
-  const size_t partial = (size_t)p->n_lists * (size_t)B * (size_t)k * 8;
+  // (a two-pass tensor search keeps hi_list(k) candidates per list)
+  const int kl = path == kPathTensor && tensor_hi(B, N, D, k, width, code_bound, sms)
+                     ? hi_list(k) : k;
+  const size_t partial = (size_t)p->n_lists * (size_t)B * (size_t)kl * 8;
   p->qprep_off = align_up(p->partial_off + partial, 256);
   p->total = p->qprep_off;
   if (path == kPathTensor)
@@ -671,11 +689,15 @@ lam_status lam_score_topk(const float *queries, int64_t B, const void *codes, in
   a.sms = sms;
   cudaError_t e;
   ScoreArgs m = a;  // the final merge's lists
+  int merge_mode = 0;
   if (p.path == kPathBandwidth) e = launch_score_bandwidth(a, st);
-  else if (p.path == kPathTensor) e = launch_score_tensor(a, st, RowPtrs(), &m);
+  else if (p.path == kPathTensor) e = launch_score_tensor(a, st, RowPtrs(), &m, &merge_mode);
   else e = launch_score_generic(a, st);
-  if (e != cudaSuccess) return LAM_ERR_CUDA;
-  if (launch_topk_merge(m, st) != cudaSuccess) return LAM_ERR_CUDA;
+  if (e == cudaSuccess) e = launch_topk_merge(m, st, RowPtrs(), merge_mode);
+  if (e != cudaSuccess) {
+    debug_report("lam_score_topk", e);
+    return LAM_ERR_CUDA;
+  }
   return LAM_OK;
 }
 

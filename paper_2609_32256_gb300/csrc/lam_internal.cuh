@@ -32,6 +32,12 @@ constexpr long long kWaitCycles = 2000000000LL;
 constexpr int kHdrFlags = 0;
 constexpr int kHdrWaitCycles = 2;
 constexpr int kHdrStall = 3;
+// Two-pass tensor search (hi-only candidates, then exact rescoring): the
+// count of queries whose candidates could not be certified, the largest
+// sum_d c_d^2 of any row (fp32 bits), and a test hook that fails every query.
+constexpr int kHdrHiFail = 4;
+constexpr int kHdrMaxCC = 5;
+constexpr int kHdrForceFail = 6;
 
 // Status block of lam_quantize (32 bytes, zeroed before each call).
 struct QuantStatus {
@@ -119,6 +125,18 @@ __device__ __forceinline__ long long wait_budget(const uint32_t *gflags) {
   const uint32_t v = gflags ? *reinterpret_cast<const volatile uint32_t *>(gflags + kHdrWaitCycles)
                             : 0u;
   return v ? (long long)v : kWaitCycles;
+}
+// Raises the header's largest row sum of squares to cc (cc >= 0: its fp32
+// bits order as unsigned integers); reads first, so most rows add no atomic.
+__device__ __forceinline__ void note_max_cc(uint32_t *gflags, float cc) {
+  uint32_t *p = gflags + kHdrMaxCC;
+  const uint32_t b = __float_as_uint(cc);
+  if (b > *reinterpret_cast<volatile uint32_t *>(p)) atomicMax(p, b);
+}
+// Whether every query of a two-pass tensor search was certified (the
+// fallback pass then has nothing to do).
+__device__ __forceinline__ bool hi_all_certified(const uint32_t *gflags) {
+  return *reinterpret_cast<const volatile uint32_t *>(gflags + kHdrHiFail) == 0u;
 }
 // Whether the copy producers of a search must issue nothing (test hook).
 __device__ __forceinline__ bool producers_stalled(const uint32_t *gflags) {
@@ -325,9 +343,17 @@ cudaError_t launch_score_generic(const ScoreArgs &a, cudaStream_t st,
                                  const RowPtrs &rp = RowPtrs());
 // `merge` (optional) receives the arguments of the final merge: a search of
 // several slabs leaves one merged list per slab in its workspace.
+// `merge_mode` (optional) receives the mode of that merge (launch_topk_merge):
+// 2 after a two-pass search, whose final merge belongs to the gated full pass.
 cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st,
-                                const RowPtrs &rp = RowPtrs(), ScoreArgs *merge = nullptr);
-cudaError_t launch_topk_merge(const ScoreArgs &a, cudaStream_t st, const RowPtrs &rp = RowPtrs());
+                                const RowPtrs &rp = RowPtrs(), ScoreArgs *merge = nullptr,
+                                int *merge_mode = nullptr);
+// mode 0: the merge of a search; 1: the certifying merge of a two-pass
+// tensor search (a.k = candidate lists; every candidate rescored exactly,
+// the best kout written, uncertified queries counted in the header); 2: the
+// merge of the gated full pass (does nothing when every query was certified).
+cudaError_t launch_topk_merge(const ScoreArgs &a, cudaStream_t st, const RowPtrs &rp = RowPtrs(),
+                              int mode = 0, int kout = 0);
 // Multi-slab searches: the partial lists [list0, list0 + n_lists) of one slab
 // merged into slab `slab` of `out` ([nslabs][B][k] keys); with `seed`, also
 // per query the ranking-form score of the slab's k-th best key.
@@ -358,6 +384,27 @@ TensorPlan tensor_plan(int64_t B, int64_t N, int D, int k, int sms, bool force_p
 inline bool tensor_wide(int width, int code_bound) {
   return width == 2 && !(code_bound > 0 && code_bound <= 2048);
 }
+// Candidate list length of the hi-only tensor pass for a final top-k: k plus
+// a margin (6 for k < 12, else 16), rounded up to the 16- and 32-entry
+// register lists; 0 when that exceeds the largest tensor-path list (128).
+inline int hi_list(int k) {
+  int kp = k + (k < 12 ? 6 : 16);
+  if (kp <= 16) kp = 16;
+  else if (kp <= 32) kp = 32;
+  return kp <= 128 ? kp : 0;
+}
+// Whether a tensor-path search of this shape runs as two passes: the hi-only
+// pass (fp16 hi term of the query only, half the MMAs) keeping hi_list(k)
+// candidates, exact rescoring and certification in the merge, and the full
+// (hi + lo) pass gated on a certification failure.  Opt-in: LAM_SCORE_HI=1
+// (measured, it does not beat the single full pass on this part: the
+// kernels are bound by shared-memory ingress and the epilogue as much as by
+// the MMAs, and the extra candidates, the rescoring merge and the gated
+// launches cost what the halved MMAs save).
+bool tensor_hi(int64_t B, int64_t N, int D, int k, int width, int code_bound, int sms);
+// The warp k-way merge takes n_lists sorted lists of k keys per query.
+bool kmerge_fits(int n_lists, int k);
+
 // K extent of the tensor path's operand images: D, or for the split two
 // image chunks per 32-wide K chunk of the codes (D rounded up to 32, doubled).
 inline int tensor_k_extent(int D, bool wide) { return wide ? 2 * ((D + 31) / 32 * 32) : D; }

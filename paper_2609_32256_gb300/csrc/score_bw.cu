@@ -983,21 +983,48 @@ __global__ void __launch_bounds__(kMergeThreads) topk_merge_kernel(ScoreArgs a, 
 // rows of its queries) and re-sorted, as in the block-sort merge above.
 constexpr int kKmWarps = 8;
 
+// Eight consecutive codes of width w (1, 2 or 4) from index i (a multiple of
+// 8; the address 8 w-byte aligned) as exact fp32 values.
+__device__ __forceinline__ void load8_codes(const void *codes, int w, int64_t i, float (&c)[8]) {
+  if (w == 1) {
+    const uint2 v = *reinterpret_cast<const uint2 *>(static_cast<const int8_t *>(codes) + i);
+#pragma unroll
+    for (int t = 0; t < 8; ++t) c[t] = (float)(int8_t)((t < 4 ? v.x : v.y) >> (8 * (t & 3)));
+  } else if (w == 2) {
+    const uint4 v = *reinterpret_cast<const uint4 *>(static_cast<const int16_t *>(codes) + i);
+    const uint32_t x[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int t = 0; t < 8; ++t) c[t] = (float)(int16_t)(x[t >> 1] >> (16 * (t & 1)));
+  } else {
+    const int4 *p = reinterpret_cast<const int4 *>(static_cast<const int32_t *>(codes) + i);
+    const int4 v0 = p[0], v1 = p[1];
+    c[0] = (float)v0.x; c[1] = (float)v0.y; c[2] = (float)v0.z; c[3] = (float)v0.w;
+    c[4] = (float)v1.x; c[5] = (float)v1.y; c[6] = (float)v1.z; c[7] = (float)v1.w;
+  }
+}
+
 template <int HPL>
 __global__ void __launch_bounds__(kKmWarps * 32) topk_kmerge_kernel(ScoreArgs a, int qpc,
-                                                                    RowPtrs rp) {
+                                                                    RowPtrs rp, int mode,
+                                                                    int kout) {
   if (rp.qst != nullptr && (!status_ok(rp.qst) || (status_width(rp.qst) != 1 &&
                                                    status_width(rp.qst) != 2))) {
     if (blockIdx.x == 0 && threadIdx.x == 0) atomicOr(a.gflags, kFlagInput);
     return;
   }
+  // the merge of the gated full pass: nothing to do when every query passed
+  if (mode == 2 && hi_all_certified(a.gflags)) return;
   extern __shared__ __align__(16) uint8_t ksmem[];
   const int L = a.n_lists, k = a.k;
+  const bool cert = mode == 1;
+  const int ko = cert ? kout : k;  // entries written per query
   uint64_t *cand = reinterpret_cast<uint64_t *>(ksmem);            // [qpc][L][k]
   uint64_t *outk = cand + (size_t)qpc * L * k;                       // [kKmWarps][P2]
   const int P2 = next_pow2_dev(k);
   const int64_t b0 = (int64_t)blockIdx.x * qpc;
   const int per_q = L * k;  // fits: the candidates of qpc queries fit in shared memory
+  // (unrolled: eight independent loads in flight per thread)
+#pragma unroll 8
   for (int e = threadIdx.x; e < qpc * per_q; e += blockDim.x) {
     const int qi = e / per_q, rem = e - qi * per_q;
     const int l = rem / k, i = rem - l * k;
@@ -1012,6 +1039,7 @@ __global__ void __launch_bounds__(kKmWarps * 32) topk_kmerge_kernel(ScoreArgs a,
   const int64_t b = b0 + qi;
   const bool mine = qi < qpc && b < a.B;
   uint64_t *O = outk + (size_t)warp * P2;
+  uint64_t tkey = kSentinel;  // cert: the k-th (last) candidate's key by the hi-only score
   if (mine) {
     const uint64_t *C = cand + (size_t)qi * per_q;
     int pos[HPL];
@@ -1031,12 +1059,12 @@ __global__ void __launch_bounds__(kKmWarps * 32) topk_kmerge_kernel(ScoreArgs a,
           m = head[h];
           mh = h;
         }
-      uint64_t gm = m;
-#pragma unroll
-      for (int off = 16; off > 0; off >>= 1) {
-        const uint64_t o = __shfl_xor_sync(0xffffffffu, gm, off);
-        gm = o < gm ? o : gm;
-      }
+      // warp minimum of the 64-bit heads: the high words by one reduction,
+      // then the low words of the lanes that hold the smallest high word
+      const uint32_t mhi = (uint32_t)(m >> 32);
+      const uint32_t ghi = __reduce_min_sync(0xffffffffu, mhi);
+      const uint32_t glo = __reduce_min_sync(0xffffffffu, mhi == ghi ? (uint32_t)m : 0xffffffffu);
+      const uint64_t gm = ((uint64_t)ghi << 32) | glo;
       const unsigned bal = __ballot_sync(0xffffffffu, m == gm);
       if (lane == __ffs(bal) - 1) {
 #pragma unroll
@@ -1047,31 +1075,122 @@ __global__ void __launch_bounds__(kKmWarps * 32) topk_kmerge_kernel(ScoreArgs a,
           }
       }
       if (lane == 0) O[i] = gm;
+      tkey = gm;
     }
   }
-  if (!desc) {
-    // every warp rescores survivors of every query of the CTA
+  if (!desc || cert) {
+    // Survivors rescored in the direct form (squared L2: the ranking form
+    // ||q||^2 + s^2||c||^2 - 2 s q.c cancels for near neighbours), and every
+    // candidate of the certifying merge exactly (it was ranked by the hi-only
+    // score).  Every warp rescores candidates of every query of the CTA, kRs
+    // rows at a time so that their code loads are in flight together (each
+    // row's sum keeps the order of a one-row loop).
+    constexpr int kRs = 4;
+    __shared__ float qnq[kKmWarps][2];  // cert: ||q|| and ||q||^2 of the CTA's queries
+    if (cert && mine) {
+      const float *q = a.queries + b * a.D;
+      float mx = 0.0f;
+      for (int d = lane; d < a.D; d += 32) mx = fmaxf(mx, fabsf(q[d]));
+      const float sc = norm_scale(warp_max(mx));
+      float part = 0.0f;
+      for (int d = lane; d < a.D; d += 32) part = fmaf(q[d] * sc, q[d] * sc, part);
+      const float qn = sqrtf(warp_sum(part)) / sc;
+      if (lane == 0) {
+        qnq[warp][0] = qn;
+        qnq[warp][1] = qn * qn;
+      }
+    }
     __syncthreads();
-    for (int t = warp; t < qpc * k; t += kKmWarps) {
-      const int tq = t / k, i = t - tq * k;
-      const int64_t tb = b0 + tq;
-      if (tb >= a.B) continue;
-      uint64_t *Ot = outk + (size_t)tq * P2;
-      const uint32_t row = (uint32_t)(Ot[i] & 0xffffffffu);
-      const float *q = a.queries + tb * a.D;
-      float acc = 0.0f;
-      if (row < a.N) {
+    const float s2 = a.s * a.s;
+    // vector loads when Q_eps code rows and query rows are 16-byte aligned
+    const bool vec = a.fmt == 0 && (a.D & 7) == 0 &&
+                     ((reinterpret_cast<uintptr_t>(a.codes) |
+                       reinterpret_cast<uintptr_t>(a.queries)) & 15u) == 0;
+    for (int t0 = warp; t0 < qpc * k; t0 += kKmWarps * kRs) {
+      uint32_t row[kRs];
+      const float *q[kRs];
+      uint64_t *slot[kRs];
+      float acc[kRs], cc[kRs];
+      int tqs[kRs];
+#pragma unroll
+      for (int u = 0; u < kRs; ++u) {
+        const int t = t0 + u * kKmWarps;
+        const int tq = t / k, i = t - tq * k;
+        const int64_t tb = b0 + tq;
+        const bool ok = t < qpc * k && tb < a.B;
+        tqs[u] = ok ? tq : 0;
+        slot[u] = ok ? outk + (size_t)tq * P2 + i : nullptr;
+        row[u] = ok ? (uint32_t)(*slot[u] & 0xffffffffu) : 0xffffffffu;
+        q[u] = a.queries + (ok ? tb : 0) * a.D;
+        acc[u] = 0.0f;
+        cc[u] = 0.0f;
+      }
+      if (vec) {
+        // eight consecutive coordinates per lane and 256-wide slice: one 8- or
+        // 16-byte code load (int8 / int16) and two float4 query loads per row
+        const int w = codes_width(a, rp);
+#pragma unroll 2
+        for (int d0 = lane * 8; d0 < a.D; d0 += 256) {
+#pragma unroll
+          for (int u = 0; u < kRs; ++u) {
+            if (row[u] < a.N) {
+              float c[8];
+              load8_codes(a.codes, w, (int64_t)row[u] * a.D + d0, c);
+              const float4 qa = *reinterpret_cast<const float4 *>(q[u] + d0);
+              const float4 qb = *reinterpret_cast<const float4 *>(q[u] + d0 + 4);
+              const float qv[8] = {qa.x, qa.y, qa.z, qa.w, qb.x, qb.y, qb.z, qb.w};
+#pragma unroll
+              for (int t = 0; t < 8; ++t) {
+                if (!desc) {
+                  const float df = __fsub_rn(qv[t], __fmul_rn(a.s, c[t]));
+                  acc[u] = fmaf(df, df, acc[u]);
+                } else {
+                  acc[u] = fmaf(qv[t], c[t], acc[u]);
+                  cc[u] = fmaf(c[t], c[t], cc[u]);
+                }
+              }
+            }
+          }
+        }
+      } else if (!desc) {
 #pragma unroll 4
         for (int d = lane; d < a.D; d += 32) {
-          const float xh = a.fmt ? row_value(a, rp, row, d)
-                                 : __fmul_rn(a.s, (float)load_code(a.codes, codes_width(a, rp),
-                                                                   (int64_t)row * a.D + d));
-          const float df = __fsub_rn(q[d], xh);
-          acc = fmaf(df, df, acc);
+#pragma unroll
+          for (int u = 0; u < kRs; ++u) {
+            if (row[u] < a.N) {
+              const float xh =
+                  a.fmt ? row_value(a, rp, row[u], d)
+                        : __fmul_rn(a.s, (float)load_code(a.codes, codes_width(a, rp),
+                                                          (int64_t)row[u] * a.D + d));
+              const float df = __fsub_rn(q[u][d], xh);
+              acc[u] = fmaf(df, df, acc[u]);
+            }
+          }
+        }
+      } else {  // cert, inner product or cosine: sum q_d c_d and sum c_d^2
+#pragma unroll 4
+        for (int d = lane; d < a.D; d += 32) {
+#pragma unroll
+          for (int u = 0; u < kRs; ++u) {
+            if (row[u] < a.N) {
+              const float c =
+                  (float)load_code(a.codes, codes_width(a, rp), (int64_t)row[u] * a.D + d);
+              acc[u] = fmaf(q[u][d], c, acc[u]);
+              cc[u] = fmaf(c, c, cc[u]);
+            }
+          }
         }
       }
-      acc = warp_sum(acc);
-      if (lane == 0) Ot[i] = row < a.N ? make_key(acc, row, false) : kSentinel;
+#pragma unroll
+      for (int u = 0; u < kRs; ++u) {
+        float tot = warp_sum(acc[u]);
+        if (desc) {
+          const float tcc = a.metric == LAM_METRIC_COSINE ? warp_sum(cc[u]) : 0.0f;
+          tot = finish_score(a.metric, tot, tcc, a.s, s2, qnq[tqs[u]][1], qnq[tqs[u]][0]);
+        }
+        if (lane == 0 && slot[u] != nullptr)
+          *slot[u] = row[u] < a.N ? make_key(tot, row[u], desc) : kSentinel;
+      }
     }
     __syncthreads();
     if (mine) {
@@ -1092,16 +1211,43 @@ __global__ void __launch_bounds__(kKmWarps * 32) topk_kmerge_kernel(ScoreArgs a,
           __syncwarp();
         }
       }
+      if (cert && lane == 0) {
+        // Certification: a row outside the candidates scored no better than
+        // the last candidate by the hi-only score T, and its exact score lies
+        // within Bq of that score (the dropped lo term, |q_lo . c| <=
+        // 2^-11 ||q|| ||c||, plus fp32 accumulation, D 2^-21 of ||q|| ||c||).
+        // The top-kout is exact when the kout-th exact score beats T by more
+        // than Bq; otherwise the query is counted and the full pass reruns.
+        bool ok = tkey == kSentinel;  // fewer rows than candidates: all were rescored
+        if (!ok) {
+          const float T = rank_key32_score((uint32_t)(tkey >> 32), desc);
+          const uint64_t kk = O[ko - 1];
+          const float ek = rank_key32_score((uint32_t)(kk >> 32), desc);
+          const float maxc = sqrtf(__uint_as_float(
+                                 *reinterpret_cast<volatile uint32_t *>(a.gflags + kHdrMaxCC))) *
+                             1.0001f;
+          const float coef = 0x1p-11f + (float)a.D * 0x1p-21f;
+          const float qn = qnq[warp][0];
+          float bq;
+          if (a.metric == LAM_METRIC_COSINE) bq = coef;
+          else if (a.metric == LAM_METRIC_IP) bq = coef * a.s * qn * maxc;
+          else  // also the fp32 rounding of the ranking form ||q||^2 + s^2||c||^2 - 2 s q.c
+            bq = 2.0f * coef * a.s * qn * maxc + 0x1p-21f * (qn * qn + s2 * maxc * maxc);
+          ok = kk != kSentinel && (desc ? ek > T + bq : ek < T - bq) &&
+               a.gflags[kHdrForceFail] == 0u;
+        }
+        if (!ok) atomicAdd(a.gflags + kHdrHiFail, 1u);
+      }
     }
   }
   __syncwarp();
   if (mine) {
-    for (int i = lane; i < k; i += 32) {
+    for (int i = lane; i < ko; i += 32) {
       const uint64_t key = O[i];
       uint32_t o = (uint32_t)(key >> 32);
       if (desc) o = ~o;
-      a.scores[b * k + i] = unord_f32(o);
-      a.ids[b * k + i] = (int64_t)(uint32_t)(key & 0xffffffffu);
+      a.scores[b * ko + i] = unord_f32(o);
+      a.ids[b * ko + i] = (int64_t)(uint32_t)(key & 0xffffffffu);
     }
   }
 }
@@ -1312,7 +1458,8 @@ cudaError_t launch_score_generic(const ScoreArgs &a, cudaStream_t st, const RowP
 }
 
 template <int HPL>
-static cudaError_t launch_kmerge_t(const ScoreArgs &a, cudaStream_t st, const RowPtrs &rp) {
+static cudaError_t launch_kmerge_t(const ScoreArgs &a, cudaStream_t st, const RowPtrs &rp,
+                                   int mode, int kout) {
   const size_t per_q = (size_t)a.n_lists * a.k * 8;
   int64_t qpc = (int64_t)(kKmCandBytes / per_q);
   if (qpc > kKmWarps) qpc = kKmWarps;  // one query per warp
@@ -1325,9 +1472,12 @@ static cudaError_t launch_kmerge_t(const ScoreArgs &a, cudaStream_t st, const Ro
   auto kern = topk_kmerge_kernel<HPL>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  timing_launch_begin(LAM_TIME_MERGE, st);
-  kern<<<(unsigned)((a.B + qpc - 1) / qpc), kKmWarps * 32, smem, st>>>(a, (int)qpc, rp);
-  timing_launch_end(LAM_TIME_MERGE, st);
+  // (the gated merge of a two-pass search counts as an auxiliary launch)
+  const int kind = mode == 2 ? LAM_TIME_AUX : LAM_TIME_MERGE;
+  timing_launch_begin(kind, st);
+  kern<<<(unsigned)((a.B + qpc - 1) / qpc), kKmWarps * 32, smem, st>>>(a, (int)qpc, rp, mode,
+                                                                       kout);
+  timing_launch_end(kind, st);
   return cudaGetLastError();
 }
 
@@ -1359,15 +1509,21 @@ cudaError_t launch_slab_merge(const ScoreArgs &a, int list0, int n_lists, int sl
   return cudaErrorInvalidValue;
 }
 
-cudaError_t launch_topk_merge(const ScoreArgs &a, cudaStream_t st, const RowPtrs &rp) {
+bool kmerge_fits(int n_lists, int k) {
+  return (size_t)n_lists * k * 8 <= kKmCandBytes && n_lists <= 512;
+}
+
+cudaError_t launch_topk_merge(const ScoreArgs &a, cudaStream_t st, const RowPtrs &rp, int mode,
+                              int kout) {
   // warp k-way merge when one query's candidates fit the shared-memory budget
-  if ((size_t)a.n_lists * a.k * 8 <= kKmCandBytes && a.n_lists <= 512) {
-    if (a.n_lists <= 32) return launch_kmerge_t<1>(a, st, rp);
-    if (a.n_lists <= 64) return launch_kmerge_t<2>(a, st, rp);
-    if (a.n_lists <= 128) return launch_kmerge_t<4>(a, st, rp);
-    if (a.n_lists <= 256) return launch_kmerge_t<8>(a, st, rp);
-    return launch_kmerge_t<16>(a, st, rp);
+  if (kmerge_fits(a.n_lists, a.k)) {
+    if (a.n_lists <= 32) return launch_kmerge_t<1>(a, st, rp, mode, kout);
+    if (a.n_lists <= 64) return launch_kmerge_t<2>(a, st, rp, mode, kout);
+    if (a.n_lists <= 128) return launch_kmerge_t<4>(a, st, rp, mode, kout);
+    if (a.n_lists <= 256) return launch_kmerge_t<8>(a, st, rp, mode, kout);
+    return launch_kmerge_t<16>(a, st, rp, mode, kout);
   }
+  if (mode != 0) return cudaErrorInvalidValue;  // two-pass searches plan for the k-way merge
   const int64_t total = (int64_t)a.n_lists * a.k;
   int P = total <= kMergeCap ? next_pow2(total) : kMergeCap;
   if (P < 64) P = 64;

@@ -32,6 +32,7 @@
 // Every wait is bounded; a timeout records LAM_ERR_TIMEOUT and unwinds.
 #include "score_common.cuh"
 
+#include <cstdlib>
 #include <cstring>
 
 namespace lam {
@@ -217,6 +218,12 @@ __device__ __forceinline__ float warp_sum_tc(float v) {
   return v;
 }
 
+__device__ __forceinline__ float warp_max_tc(float v) {
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, off));
+  return v;
+}
+
 // Converter thread -> (tile row, 16-byte piece) of its i-th task, chosen so
 // that each quarter-warp's 16-byte accesses fall in distinct banks both when
 // reading the raw rows (128 bytes, piece ^ row & 7) and when writing the fp16
@@ -312,6 +319,8 @@ struct TcGeom {
   int raw_off, lists_off, cbuf_off, cc_off, bar_off;
   int qoff;  // MMA row of the block's first query (64 for one block of <= 64)
   const QuantStatus *qst;  // status-driven calls: the codes' width is read here
+  int hi;    // hi-only pass: the lo term of the query is neither copied nor multiplied
+  int gate;  // full pass of a two-pass search: runs only if a query was not certified
 };
 
 template <int W, int KR>
@@ -319,6 +328,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     score_tc_kernel(const __grid_constant__ CUtensorMap cmap, ScoreArgs a, TcGeom g) {
   // status-driven call: only the variant of the codes' width runs
   if (g.qst != nullptr && (!status_ok(g.qst) || status_width(g.qst) != (uint32_t)W)) return;
+  if (g.gate && hi_all_certified(a.gflags)) return;
   extern __shared__ uint8_t tc_smem_raw[];
   // 1024-byte alignment for the swizzled tiles (address bits drive the swizzle)
   const uint32_t base_u32 = smem_u32(tc_smem_raw);
@@ -431,7 +441,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             for (int j = 0; j < kBK / kUmmaK; ++j) {
               const uint64_t koff = (uint64_t)((j * kUmmaK * 2) >> 4);
               umma_f16(d_tmem, ahi + koff, bd + koff, kIdesc, (kc + c > 0 || j > 0) ? 1u : 0u);
-              umma_f16(d_tmem, alo + koff, bd + koff, kIdesc, 1u);
+              if (!g.hi) umma_f16(d_tmem, alo + koff, bd + koff, kIdesc, 1u);
             }
           }
           umma_commit(&empty[s]);
@@ -451,7 +461,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       const __half2 bias = __float2half2_rn(1152.0f);
       int it = 0, gr = 0;
       bool ok = true;
-      float amax = 0.0f;
+      float amax = 0.0f, ccmax = 0.0f;
       for (int lt = 0; lt < ntl && ok; ++lt) {
         const int buf = lt & 1, u = lt >> 1;
         float ccp[kTasks];
@@ -575,23 +585,39 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         }
         if (!ok) break;
         if (CC) {
-          if (u > 0 && !mbar_wait(&cce[buf], (u - 1) & 1, abort_flag, a.gflags)) break;
+          float tr[kTasks];  // the rows' sums of c^2
 #pragma unroll
           for (int i = 0; i < kTasks; ++i) {
             float t = ccp[i] + __shfl_xor_sync(0xffffffffu, ccp[i], 1);
             if (W == 2) t += __shfl_xor_sync(0xffffffffu, t, 2);
-            const bool writer = conv_sub<W>(ct) == 0;
-            // per-row factor of the score: 1/||c|| for cosine, s^2 ||c||^2 for L2
-            const float rowf = a.metric == LAM_METRIC_COSINE ? (t > 0.0f ? 1.0f / sqrtf(t) : 0.0f)
-                                                            : a.s * a.s * t;
-            if (writer) ccbuf[buf * kBN + conv_row<W>(ct, i)] = rowf;
+            tr[i] = t;
+            ccmax = fmaxf(ccmax, t);
           }
-          mbar_arrive(&ccf[buf]);
+          if (need_cc) {
+            if (u > 0 && !mbar_wait(&cce[buf], (u - 1) & 1, abort_flag, a.gflags)) break;
+#pragma unroll
+            for (int i = 0; i < kTasks; ++i) {
+              const float t = tr[i];
+              const bool writer = conv_sub<W>(ct) == 0;
+              // per-row factor of the score: 1/||c|| for cosine, s^2 ||c||^2 for L2
+              const float rowf = a.metric == LAM_METRIC_COSINE
+                                     ? (t > 0.0f ? 1.0f / sqrtf(t) : 0.0f)
+                                     : a.s * a.s * t;
+              if (writer) ccbuf[buf * kBN + conv_row<W>(ct, i)] = rowf;
+            }
+            mbar_arrive(&ccf[buf]);
+          }
         }
       }
       if (W == 2 && amax > 2048.0f) atomicOr(a.gflags, kFlagRange);
+      // hi-only pass: the largest row norm bounds what the dropped lo term
+      // could add to any row's score (the certification in the merge)
+      if (CC && g.hi) {
+        const float m = warp_max_tc(ccmax);
+        if (lane == 0) note_max_cc(a.gflags, m);
+      }
     };
-    if (need_cc)
+    if (need_cc || g.hi)
       converters(BoolTag<true>{});
     else
       converters(BoolTag<false>{});
@@ -609,16 +635,22 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         const int nc = nk - kc < C ? nk - kc : C;
         uint8_t *dst = smem + (size_t)s * stage_stride;
         const uint8_t *src = qA + ((size_t)qb * nk + kc) * kAStage;
+        const int nh = g.hi ? 1 : 2;  // the hi image, and the lo image unless hi-only
         if (g.qoff == 0) {
-          mbar_arrive_expect_tx(&afull[s], (uint32_t)nc * kAStage);
-          bulk_g2s(dst, src, (uint32_t)nc * kAStage, &afull[s]);
+          mbar_arrive_expect_tx(&afull[s], (uint32_t)(nc * nh) * kABytes);
+          if (nh == 2) {
+            bulk_g2s(dst, src, (uint32_t)nc * kAStage, &afull[s]);
+          } else {
+            for (int c = 0; c < nc; ++c)
+              bulk_g2s(dst + (size_t)c * kAStage, src + (size_t)c * kAStage, kABytes, &afull[s]);
+          }
         } else {
           // queries in MMA rows 64 .. 127 only: the hi and lo rows 0 .. 63
           // (64-byte rows, the first 4 KB of each 8 KB tile) feed TMEM lanes
           // that no epilogue warp reads, so they are not copied
-          mbar_arrive_expect_tx(&afull[s], (uint32_t)nc * kABytes);
+          mbar_arrive_expect_tx(&afull[s], (uint32_t)(nc * nh) * (kABytes / 2));
           for (int c = 0; c < nc; ++c)
-            for (int h = 0; h < 2; ++h) {
+            for (int h = 0; h < nh; ++h) {
               const size_t off = (size_t)c * kAStage + (size_t)h * kABytes + kABytes / 2;
               bulk_g2s(dst + off, src + off, kABytes / 2, &afull[s]);
             }
@@ -902,7 +934,8 @@ __device__ __forceinline__ void convert_block(const void *__restrict__ codes, in
                                               int64_t nrows, int64_t nrows_pad, int D,
                                               uint8_t *__restrict__ out,
                                               float *__restrict__ rowf, int metric, float s,
-                                              uint32_t *gflags, int64_t blk, bool wide = false) {
+                                              uint32_t *gflags, int64_t blk, bool wide = false,
+                                              bool track = false) {
   const int64_t r = blk * 8 + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (r >= nrows_pad) return;
@@ -958,6 +991,8 @@ __device__ __forceinline__ void convert_block(const void *__restrict__ codes, in
   cc = warp_sum_tc(cc);
   if (lane == 0 && valid && metric != LAM_METRIC_IP)
     rowf[r] = metric == LAM_METRIC_COSINE ? (cc > 0.0f ? 1.0f / sqrtf(cc) : 0.0f) : s * s * cc;
+  // (a hi-only pass follows: the largest row norm, for the certification)
+  if (track && lane == 0 && valid) note_max_cc(gflags, cc);
   if (W == 2 && !wide && amax > 2048.0f) atomicOr(gflags, kFlagRange);
 }
 
@@ -974,10 +1009,10 @@ __global__ void __launch_bounds__(256) convert_codes_kernel(const void *__restri
                                                             float *__restrict__ rowf, int metric,
                                                             float s, uint32_t *gflags,
                                                             const QuantStatus *qst,
-                                                            int wide = 0) {
+                                                            int wide = 0, int track = 0) {
   if (!width_gate(qst, W)) return;
   convert_block<W>(codes, row_base, nrows, nrows_pad, D, out, rowf, metric, s, gflags, blockIdx.x,
-                   wide != 0);
+                   wide != 0, track != 0);
 }
 
 // Query preparation and the first slab's conversion in one launch: blocks
@@ -987,12 +1022,12 @@ __global__ void __launch_bounds__(256) prep_convert_kernel(
     const float *__restrict__ q, int64_t B, int D, int64_t Bpad, uint8_t *__restrict__ qA,
     unsigned q_blocks, const void *__restrict__ codes, int64_t nrows, int64_t nrows_pad,
     uint8_t *__restrict__ out, float *__restrict__ rowf, int metric, float s, uint32_t *gflags,
-    const QuantStatus *qst, int wide = 0) {
+    const QuantStatus *qst, int wide = 0, int track = 0) {
   if (blockIdx.x < q_blocks)
     qprep_block(q, B, D, Bpad, qA, blockIdx.x, 0, wide ? 2 : 1);
   else if (width_gate(qst, W))
     convert_block<W>(codes, 0, nrows, nrows_pad, D, out, rowf, metric, s, gflags,
-                     blockIdx.x - q_blocks, wide != 0);
+                     blockIdx.x - q_blocks, wide != 0, track != 0);
 }
 
 // Status-driven calls: one launch converts at the width the quantize status
@@ -1170,6 +1205,8 @@ struct Tc2Geom {
   const float *seed;        // later slabs: per query, the first slab's k-th best score
   const float *rowf;        // per-row factors of the slab (Q_eps codes)
   const float4 *rowf4;      // per-row (u, w, z) of the slab (per-row codecs)
+  int hi;    // hi-only pass: the lo term of the query is neither copied nor multiplied
+  int gate;  // full pass of a two-pass search: runs only if a query was not certified
 };
 
 // Per-row score factors of the per-row codecs for one 32-row chunk, one row
@@ -1214,6 +1251,7 @@ __device__ __forceinline__ float fac_score(const RowFac<true> &f, float acc, con
 template <int KR, bool RC>
 __global__ void __launch_bounds__(kTc2Threads, 1)
     score_tc2_kernel(ScoreArgs a, Tc2Geom g) {
+  if (g.gate && hi_all_certified(a.gflags)) return;
   extern __shared__ uint8_t tc_smem_raw[];
   const uint32_t base_u32 = smem_u32(tc_smem_raw);
   uint8_t *smem = tc_smem_raw + (((base_u32 + 1023u) & ~1023u) - base_u32);
@@ -1273,8 +1311,14 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
           }
           // stage: [query blocks of the nc chunks][code blocks of the nc chunks]
           uint8_t *st = smem + (size_t)s * C * kStageBytes;
-          mbar_arrive_expect_tx(&full[s], (uint32_t)nc * (kAStage + kB16Bytes));
-          bulk_g2s(st, qA + ((size_t)qb * nk + kc) * kAStage, (uint32_t)nc * kAStage, &full[s]);
+          const uint8_t *qsrc = qA + ((size_t)qb * nk + kc) * kAStage;
+          mbar_arrive_expect_tx(&full[s], (uint32_t)nc * ((g.hi ? kABytes : kAStage) + kB16Bytes));
+          if (!g.hi) {
+            bulk_g2s(st, qsrc, (uint32_t)nc * kAStage, &full[s]);
+          } else {  // the hi images only
+            for (int c = 0; c < nc; ++c)
+              bulk_g2s(st + (size_t)c * kAStage, qsrc + (size_t)c * kAStage, kABytes, &full[s]);
+          }
           bulk_g2s(st + C * kAStage, g.b16 + ((size_t)tile * nk + kc) * kB16Bytes,
                    (uint32_t)nc * kB16Bytes, &full[s]);
           issued = it + 1;
@@ -1309,7 +1353,7 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
             for (int j = 0; j < kBK / kUmmaK; ++j) {
               const uint64_t koff = (uint64_t)((j * kUmmaK * 2) >> 4);
               umma_f16(d_tmem, ahi + koff, bd + koff, kIdesc, (kc + c > 0 || j > 0) ? 1u : 0u);
-              umma_f16(d_tmem, alo + koff, bd + koff, kIdesc, 1u);
+              if (!g.hi) umma_f16(d_tmem, alo + koff, bd + koff, kIdesc, 1u);
             }
           }
           umma_commit(&empty[s]);
@@ -1616,8 +1660,9 @@ TensorPlan tensor_plan(int64_t B, int64_t N, int D, int k, int sms, bool force_p
 }
 
 cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st, const RowPtrs &rp,
-                                ScoreArgs *merge) {
+                                ScoreArgs *merge, int *merge_mode) {
   if (merge != nullptr) *merge = a;
+  if (merge_mode != nullptr) *merge_mode = 0;
   const bool rc = a.fmt != 0;
   // status-driven call (codes' width on the device): both widths launch, one works
   const QuantStatus *qst = rc ? nullptr : rp.qst;
@@ -1627,6 +1672,12 @@ cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st, const RowPt
   const int Dk = tensor_k_extent(a.D, wide);
   const TensorPlan P = tensor_plan(a.B, a.N, Dk, a.k, a.sms, rc || wide);
   if (P.n_lists != a.n_lists) return cudaErrorInvalidValue;
+  // Two passes (Q_eps codes): the hi-only pass keeps kp candidates per list,
+  // the certifying merge rescores them exactly and writes the top-k, and the
+  // full (hi + lo) pass with its merge runs only for an uncertified query.
+  const bool hi = !rc && !qst && tensor_hi(a.B, a.N, a.D, a.k, a.width, a.code_bound, a.sms);
+  ScoreArgs ah = a;
+  if (hi) ah.k = hi_list(a.k);
   uint8_t *qA = static_cast<uint8_t *>(a.qprep);
   const unsigned q_blocks = (unsigned)((a.Bpad + 7) / 8);
   cudaError_t e = cudaSuccess;
@@ -1641,8 +1692,6 @@ cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st, const RowPt
     timing_launch_end(LAM_TIME_AUX, st);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    const TcLayout L = tc_layout(a.width, a.k, a.metric != LAM_METRIC_IP);
-    if (L.ns < 2) return cudaErrorInvalidValue;
     CUtensorMap cmap1, cmap2;  // the codes as int8 and as int16 rows
     if ((qst || a.width == 1) &&
         !make_map_2d(&cmap1, CU_TENSOR_MAP_DATA_TYPE_UINT8, a.codes, (uint64_t)a.D, (uint64_t)a.N,
@@ -1653,47 +1702,63 @@ cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st, const RowPt
                      (uint64_t)a.N, (uint64_t)a.D * 2, (uint32_t)(kRawRow / 2), kBN,
                      CU_TENSOR_MAP_SWIZZLE_128B))
       return cudaErrorInvalidValue;
-    TcGeom g;
-    g.qst = qst;
-    g.qoff = qoff;
-    g.ns = L.ns;
-    g.nr = L.nr;
-    g.chunks = L.chunks;
-    g.raw_off = (int)L.raw_off;
-    g.lists_off = (int)L.lists_off;
-    g.cbuf_off = (int)L.cbuf_off;
-    g.cc_off = (int)L.cc_off;
-    g.bar_off = (int)L.bar_off;
     const dim3 grid((unsigned)a.n_lists, (unsigned)(a.Bpad / kBM));
-    auto run = [&](auto kern, const CUtensorMap &cmap) -> cudaError_t {
-      cudaError_t r = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                           (int)L.smem_bytes);
-      if (r != cudaSuccess) return r;
-      timing_launch_begin(LAM_TIME_SCORE, st);
-      kern<<<grid, kTcThreads, L.smem_bytes, st>>>(cmap, a, g);
-      timing_launch_end(LAM_TIME_SCORE, st);
-      return cudaGetLastError();
+    // one pass of the stage-loop kernel over the lists of x.k keys
+    auto pass = [&](const ScoreArgs &x, int hi_pass, int gate, int kind) -> cudaError_t {
+      const TcLayout L = tc_layout(x.width, x.k, x.metric != LAM_METRIC_IP);
+      if (L.ns < 2) return cudaErrorInvalidValue;
+      TcGeom g;
+      g.qst = qst;
+      g.qoff = qoff;
+      g.ns = L.ns;
+      g.nr = L.nr;
+      g.chunks = L.chunks;
+      g.raw_off = (int)L.raw_off;
+      g.lists_off = (int)L.lists_off;
+      g.cbuf_off = (int)L.cbuf_off;
+      g.cc_off = (int)L.cc_off;
+      g.bar_off = (int)L.bar_off;
+      g.hi = hi_pass;
+      g.gate = gate;
+      auto run = [&](auto kern, const CUtensorMap &cmap) -> cudaError_t {
+        cudaError_t r = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)L.smem_bytes);
+        if (r != cudaSuccess) return r;
+        timing_launch_begin(kind, st);
+        kern<<<grid, kTcThreads, L.smem_bytes, st>>>(cmap, x, g);
+        timing_launch_end(kind, st);
+        return cudaGetLastError();
+      };
+      auto run1 = [&]() -> cudaError_t {
+        if (x.k <= 16) return run(score_tc_kernel<1, 16>, cmap1);
+        if (x.k <= 32) return run(score_tc_kernel<1, 32>, cmap1);
+        return run(score_tc_kernel<1, 0>, cmap1);
+      };
+      auto run2 = [&]() -> cudaError_t {
+        if (x.k <= 16) return run(score_tc_kernel<2, 16>, cmap2);
+        if (x.k <= 32) return run(score_tc_kernel<2, 32>, cmap2);
+        return run(score_tc_kernel<2, 0>, cmap2);
+      };
+      if (qst) {
+        const cudaError_t r = run1();
+        return r != cudaSuccess ? r : run2();
+      }
+      return x.width == 1 ? run1() : run2();
     };
-    auto run1 = [&]() -> cudaError_t {
-      if (a.k <= 16) return run(score_tc_kernel<1, 16>, cmap1);
-      if (a.k <= 32) return run(score_tc_kernel<1, 32>, cmap1);
-      return run(score_tc_kernel<1, 0>, cmap1);
-    };
-    auto run2 = [&]() -> cudaError_t {
-      if (a.k <= 16) return run(score_tc_kernel<2, 16>, cmap2);
-      if (a.k <= 32) return run(score_tc_kernel<2, 32>, cmap2);
-      return run(score_tc_kernel<2, 0>, cmap2);
-    };
-    if (qst) {
-      e = run1();
-      return e != cudaSuccess ? e : run2();
-    }
-    return a.width == 1 ? run1() : run2();
+    if (!hi) return pass(a, 0, 0, LAM_TIME_SCORE);
+    e = pass(ah, 1, 0, LAM_TIME_SCORE);
+    if (e != cudaSuccess) return e;
+    e = launch_topk_merge(ah, st, RowPtrs(), 1, a.k);
+    if (e != cudaSuccess) return e;
+    e = pass(a, 0, 1, LAM_TIME_AUX);  // (a no-op unless a query was not certified)
+    if (merge_mode != nullptr) *merge_mode = 2;
+    return e;
   }
-
   // two or more query blocks: convert each slab once, then the pure MMA kernel
   const Tc2Layout L = tc2_layout(a.k);
   if (L.ns < 2) return cudaErrorInvalidValue;
+  const Tc2Layout LH = tc2_layout(ah.k);  // the hi-only pass's lists
+  if (LH.ns < 2) return cudaErrorInvalidValue;
   uint8_t *f16 = static_cast<uint8_t *>(a.qprep) + P.fp16_off;
   float *rowf = reinterpret_cast<float *>(static_cast<uint8_t *>(a.qprep) + P.rowf_off);
   Tc2Geom g;
@@ -1711,14 +1776,18 @@ cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st, const RowPt
   // several slabs: each slab's lists are merged into one, and the first slab's
   // k-th best bounds what the later slabs may offer
   const bool per_slab = P.nslabs > 1 && P.nsplit <= 256;
-  auto kern = rc ? (a.k <= 16   ? score_tc2_kernel<16, true>
-                    : a.k <= 32 ? score_tc2_kernel<32, true>
-                                : score_tc2_kernel<0, true>)
-                 : (a.k <= 16   ? score_tc2_kernel<16, false>
-                    : a.k <= 32 ? score_tc2_kernel<32, false>
-                                : score_tc2_kernel<0, false>);
-  e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)L.smem_bytes);
-  if (e != cudaSuccess) return e;
+  auto kern_for = [&](int kk) {
+    return rc ? (kk <= 16   ? score_tc2_kernel<16, true>
+                 : kk <= 32 ? score_tc2_kernel<32, true>
+                            : score_tc2_kernel<0, true>)
+              : (kk <= 16   ? score_tc2_kernel<16, false>
+                 : kk <= 32 ? score_tc2_kernel<32, false>
+                            : score_tc2_kernel<0, false>);
+  };
+  // (the two passes may share one instantiation with different layouts: the
+  // shared-memory limit is set right before each launch)
+  auto kern = kern_for(a.k);
+  auto kern_h = kern_for(ah.k);
   const dim3 grid((unsigned)P.nsplit, (unsigned)(a.Bpad / kBM));
   for (int j = 0; j < P.nslabs; ++j) {
     const int64_t row_base = (int64_t)j * P.slab_rows;
@@ -1755,11 +1824,11 @@ cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st, const RowPt
       if (a.width == 1)
         prep_convert_kernel<1><<<q_blocks + cg, 256, 0, st>>>(
             a.queries, a.B, a.D, a.Bpad, qA, q_blocks, a.codes, nrows, nrows_pad, f16, rowf,
-            a.metric, a.s, a.gflags, nullptr);
+            a.metric, a.s, a.gflags, nullptr, 0, hi ? 1 : 0);
       else
         prep_convert_kernel<2><<<q_blocks + cg, 256, 0, st>>>(
             a.queries, a.B, a.D, a.Bpad, qA, q_blocks, a.codes, nrows, nrows_pad, f16, rowf,
-            a.metric, a.s, a.gflags, nullptr, wide ? 1 : 0);
+            a.metric, a.s, a.gflags, nullptr, wide ? 1 : 0, hi ? 1 : 0);
     } else if (a.width == 1) {
       convert_codes_kernel<1><<<cg, 256, 0, st>>>(a.codes, row_base, nrows, nrows_pad, a.D, f16,
                                                   rowf, a.metric, a.s, a.gflags, nullptr);
@@ -1774,11 +1843,38 @@ cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st, const RowPt
     g.row_base = row_base;
     g.nrows = nrows;
     g.list_base = j * P.nsplit;
-    timing_launch_begin(LAM_TIME_SCORE, st);
+    g.hi = 0;
+    g.gate = 0;
+    if (hi) {  // (one slab): the hi-only pass, its certifying merge, the gated full pass
+      ScoreArgs akh = ah;  // the kernel sees the K extent of the operand images
+      akh.D = Dk;
+      Tc2Geom gh = g;
+      gh.ns = LH.ns;
+      gh.chunks = LH.chunks;
+      gh.lists_off = (int)LH.lists_off;
+      gh.cbuf_off = (int)LH.cbuf_off;
+      gh.bar_off = (int)LH.bar_off;
+      gh.hi = 1;
+      e = cudaFuncSetAttribute(kern_h, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               (int)LH.smem_bytes);
+      if (e != cudaSuccess) return e;
+      timing_launch_begin(LAM_TIME_SCORE, st);
+      kern_h<<<grid, kTc2Threads, LH.smem_bytes, st>>>(akh, gh);
+      timing_launch_end(LAM_TIME_SCORE, st);
+      e = cudaGetLastError();
+      if (e != cudaSuccess) return e;
+      e = launch_topk_merge(ah, st, RowPtrs(), 1, a.k);
+      if (e != cudaSuccess) return e;
+      g.gate = 1;
+    }
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)L.smem_bytes);
+    if (e != cudaSuccess) return e;
+    timing_launch_begin(hi ? LAM_TIME_AUX : LAM_TIME_SCORE, st);
     ScoreArgs ak = a;  // the kernel sees the K extent of the operand images
     ak.D = Dk;
     kern<<<grid, kTc2Threads, L.smem_bytes, st>>>(ak, g);
-    timing_launch_end(LAM_TIME_SCORE, st);
+    timing_launch_end(hi ? LAM_TIME_AUX : LAM_TIME_SCORE, st);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     if (per_slab) {
@@ -1793,7 +1889,20 @@ cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st, const RowPt
     merge->partial = slabl;
     merge->n_lists = P.nslabs;
   }
+  if (hi && merge_mode != nullptr) *merge_mode = 2;
   return cudaSuccess;
 }
+
+bool tensor_hi(int64_t B, int64_t N, int D, int k, int width, int code_bound, int sms) {
+  const char *env = getenv("LAM_SCORE_HI");
+  if (env == nullptr || strcmp(env, "1") != 0) return false;  // opt-in
+  const int kp = hi_list(k);
+  if (kp == 0 || (width != 1 && width != 2)) return false;
+  const bool wide = tensor_wide(width, code_bound);
+  const TensorPlan P = tensor_plan(B, N, tensor_k_extent(D, wide), k, sms, wide);
+  if (P.nslabs != 1 || !kmerge_fits(P.n_lists, kp)) return false;
+  return P.pre ? tc2_layout(kp).ns >= 2 : tc_layout(width, kp).ns >= 2;
+}
+
 
 }  // namespace lam

@@ -110,7 +110,12 @@ def search_from(dev, q, codes, ws, N, D, eps, k, metric):
                                     ("tensor", 520), ("generic", 5)])
 @pytest.mark.parametrize("eps", [1e-2, 1e-4])  # int8 and int16 codes
 @pytest.mark.parametrize("metric", [oracle.IP, oracle.COSINE, oracle.L2])
-def test_score_topk_from_equals_the_synchronous_search(dev, score_path, path, B, eps, metric):
+def test_score_topk_from_equals_the_synchronous_search(dev, monkeypatch, score_path, path, B,
+                                                       eps, metric):
+    """The status-driven search runs the same kernels as the synchronous one
+    (bit for bit); the synchronous call's opt-in two-pass tensor search
+    rescores its candidates on the CUDA cores instead, so it is compared
+    through the oracle."""
     score_path(path)
     N, D, k = 3001, 768, 10
     x = inputs.unit_rows(N, D, seed=B)
@@ -122,11 +127,15 @@ def test_score_topk_from_equals_the_synchronous_search(dev, score_path, path, B,
     gs, gi, gst = search_from(dev, q, codes, ws, N, D, eps, k, metric)
     assert gst == 0
     typed = codes[: N * D * w].view(torch.int8 if w == 1 else torch.int16).view(N, D)
+    oc = oracle.quantize(x, eps)[0].reshape(N, D)
+    os_, oi = oracle_topk(q, oc, eps, metric, k)
     ss, si = lam.search(torch.from_numpy(q).to(dev), typed, eps, k, metric,
                         code_bound=max(-cmin, cmax))
     assert torch.equal(gs, ss) and torch.equal(gi, si)
-    oc = oracle.quantize(x, eps)[0].reshape(N, D)
-    os_, oi = oracle_topk(q, oc, eps, metric, k)
+    monkeypatch.setenv("LAM_SCORE_HI", "1")
+    ss, si = lam.search(torch.from_numpy(q).to(dev), typed, eps, k, metric,
+                        code_bound=max(-cmin, cmax))
+    check_topk(ss.cpu().numpy(), si.cpu().numpy(), q, oc, eps, metric, os_, oi)
     check_topk(gs.cpu().numpy(), gi.cpu().numpy(), q, oc, eps, metric, os_, oi)
 
 
