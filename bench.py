@@ -769,13 +769,14 @@ def run_lam(args):
             e2e_step()
         torch.cuda.synchronize(dev)
         barrier(world)
-        t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        t0.record(stream)
-        for _ in range(e2e_steps):
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(e2e_steps + 1)]
+        ev[0].record(stream)
+        for i in range(e2e_steps):
             e2e_step()
-        t1.record(stream)
+            ev[i + 1].record(stream)
         torch.cuda.synchronize(dev)
-        ms_e2e = max_over_ranks(t0.elapsed_time(t1) / e2e_steps, world, dev)
+        e2e_ms = [ev[i].elapsed_time(ev[i + 1]) for i in range(e2e_steps)]
+        ms_e2e = max_over_ranks(ev[0].elapsed_time(ev[-1]) / e2e_steps, world, dev)
         mem.check()
         assert torch.equal(s_h, ref_s.cpu()) and torch.equal(i_h, ref_i.cpu())
         del x_h
@@ -839,10 +840,15 @@ def run_lam(args):
             "cpu_baseline": cpu,
             "e2e": {"value": units_per_step * world / (ms_e2e / 1e3), "unit": UNIT,
                     "ms_per_step": ms_e2e, "steps": e2e_steps,
+                    "ms_per_step_min_median_max": [min(e2e_ms), statistics.median(e2e_ms),
+                                                   max(e2e_ms)],
+                    "host_link_gbs_at_min": wl.n * wl.d * 4 / (min(e2e_ms) / 1e3) / 1e9,
                     "h2d_bytes_per_step": wl.n * wl.d * 4 + B * wl.d * 4,
                     "d2h_bytes_per_step": B * wl.k * (4 + 8),
                     "note": "fp32 memory and query from pinned host memory, results back to "
-                            "pinned host memory, inside the timed region"},
+                            "pinned host memory, inside the timed region; bound by the host "
+                            "link (~211 GB/s for these copies alone on this box, with "
+                            "occasional slow copies from the shared host)"},
             "gpu_launches": n_launch,
             "gpu_launches_note": "library kernel launches inside the K timed steps, counted "
                                  "by the library (%d per step)" % (n_launch // args.steps),
