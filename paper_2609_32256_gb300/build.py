@@ -18,7 +18,7 @@ BUILD = os.path.join(HERE, "_build")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC",
               "-Xptxas", "-warn-spills"]
-SOURCES = ["lam_api.cu", "quantize.cu", "bands.cu", "admit.cu", "lamz.cu", "rows.cu", "score_bw.cu", "score_tc.cu", "score_noalloc.cu"]
+SOURCES = ["lam_api.cu", "quantize.cu", "bands.cu", "admit.cu", "lamz.cu", "rows.cu", "score_bw.cu", "score_tc.cu", "score_tm.cu", "score_noalloc.cu"]
 
 
 def _nvcc() -> str:

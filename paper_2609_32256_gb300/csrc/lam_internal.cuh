@@ -402,6 +402,16 @@ inline int hi_list(int k) {
 // the MMAs, and the extra candidates, the rescoring merge and the gated
 // launches cost what the halved MMAs save).
 bool tensor_hi(int64_t B, int64_t N, int D, int k, int width, int code_bound, int sms);
+// Small query batches on the tensor cores with the codes in the MMA M
+// dimension (score_tm.cu): whether the kernel takes B queries and top-k, and
+// its launch over a.n_lists CTAs of 256-row tiles.  The query images are the
+// tensor path's (one block, queries from MMA row 0); cmap1 / cmap2 map the
+// codes as int8 / int16 rows (boxes of 128 bytes x tm_box_rows() rows,
+// 128-byte swizzle).
+bool tm_fits(int64_t B, int D, int k);
+int tm_box_rows();
+cudaError_t launch_score_tm(const ScoreArgs &a, const QuantStatus *qst, const CUtensorMap &cmap1,
+                            const CUtensorMap &cmap2, cudaStream_t st);
 // The warp k-way merge takes n_lists sorted lists of k keys per query.
 bool kmerge_fits(int n_lists, int k);
 

@@ -31,6 +31,7 @@
 //   warp 10     producer of the query-block bulk copies.
 // Every wait is bounded; a timeout records LAM_ERR_TIMEOUT and unwinds.
 #include "score_common.cuh"
+#include "tc_common.cuh"
 
 #include <cstdlib>
 #include <cstring>
@@ -58,114 +59,8 @@ constexpr int kTcChunks = 2;              // K chunks per MMA stage of the stage
 constexpr uint32_t kTmemCols = 512;       // two 256-column accumulators
 constexpr int kMaxDynSmem = 232448;       // 227 KB
 constexpr int kTcMaxK = 128;
-
-// ---------------------------------------------------------- tcgen05 PTX --
-__device__ __forceinline__ void tmem_alloc(uint32_t *slot, uint32_t ncols) {
-  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
-                   smem_u32(slot)),
-               "r"(ncols)
-               : "memory");
-  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
-}
-__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
-  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
-               : "memory");
-}
-__device__ __forceinline__ void tc_fence_before() {
-  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-}
-__device__ __forceinline__ void tc_fence_after() {
-  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-}
-// D[tmem] (+)= A[smem] * B[smem]^T, fp16 inputs, fp32 accumulate.
-__device__ __forceinline__ void umma_f16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
-                                         uint32_t idesc, uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
-      : "memory");
-}
-// Arrive on `bar` once every MMA this thread issued so far has completed.
-__device__ __forceinline__ void umma_commit(uint64_t *bar) {
-  asm volatile(
-      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
-          smem_u32(bar))
-      : "memory");
-}
-// 32 consecutive fp32 columns of this warp's 32 TMEM lanes.
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t *v) {
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
-      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
-      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
-      : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]),
-        "=r"(v[7]), "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]),
-        "=r"(v[13]), "=r"(v[14]), "=r"(v[15]), "=r"(v[16]), "=r"(v[17]), "=r"(v[18]),
-        "=r"(v[19]), "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]), "=r"(v[24]),
-        "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]),
-        "=r"(v[31])
-      : "r"(taddr)
-      : "memory");
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-}
-
-__device__ __forceinline__ __half2 u32_as_h2(uint32_t u) {
-  __half2 h;
-  *reinterpret_cast<uint32_t *>(&h) = u;
-  return h;
-}
-__device__ __forceinline__ uint32_t h2_as_u32(__half2 h) { return *reinterpret_cast<uint32_t *>(&h); }
-
-// Shared-memory matrix descriptor: K-major operand, rows of 64 bytes in the
-// 64-byte swizzle, 8-row groups 512 bytes apart (SBO); LBO unused.
-__device__ __forceinline__ uint64_t desc_sw64(uint32_t saddr) {
-  uint64_t d = 0;
-  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);  // start address
-  d |= (uint64_t)1 << 16;                     // leading byte offset (unused)
-  d |= (uint64_t)(512 >> 4) << 32;            // stride byte offset
-  d |= (uint64_t)1 << 46;                     // descriptor version
-  d |= (uint64_t)4 << 61;                     // 64-byte swizzle
-  return d;
-}
-// Instruction descriptor, kind::f16: fp32 accumulate, fp16 A and B, both
-// K-major, N = 256, M = 128.
-constexpr uint32_t kIdesc = (1u << 4) | (0u << 7) | (0u << 10) | ((uint32_t)(kBN >> 3) << 17) |
-                            ((uint32_t)(kBM >> 4) << 24);
-
-// Warp-uniform bounded wait: lane 0 waits, the verdict is broadcast, and every
-// lane then observes the completed phase itself.
-__device__ __forceinline__ bool warp_wait(uint64_t *bar, uint32_t parity, volatile int *abort,
-                                          uint32_t *gflags) {
-  int ok = 0;
-  if ((threadIdx.x & 31) == 0) ok = mbar_wait(bar, parity, abort, gflags) ? 1 : 0;
-  ok = __shfl_sync(0xffffffffu, ok, 0);
-  if (ok)
-    while (!mbar_try_wait(bar, parity)) {
-    }
-  return ok != 0;
-}
-
-__device__ __forceinline__ void drain_wait_tc(uint64_t *bar, uint32_t parity) {
-  long long t0 = clock64();
-  while (!mbar_try_wait(bar, parity))
-    if (clock64() - t0 > kWaitCycles) break;
-}
-
-
-// Score from the raw accumulator (2^e q.c), a per-query factor fq and a
-// per-row factor rowf (written by the converters at the end of each tile):
-//   inner product  fq acc                 fq = s 2^-e
-//   cosine         fq acc rowf            fq = 2^-e / ||q||, rowf = 1/||c||
-//   squared L2     fq acc + ||q||^2 + rowf    fq = -2 s 2^-e, rowf = s^2 ||c||^2
-// (the k L2 survivors are rescored in the direct form by the merge).
-__device__ __forceinline__ float tile_score(int metric, float acc, float fq, float qq,
-                                            float rowf) {
-  if (metric == LAM_METRIC_IP) return fq * acc;
-  if (metric == LAM_METRIC_COSINE) return (fq * acc) * rowf;
-  return fmaf(fq, acc, qq + rowf);
-}
+// M = 128 queries, N = 256 code rows
+constexpr uint32_t kIdesc = idesc_f16(kBM, kBN);
 
 // Candidate mask of one 32-column chunk: bit j is set when column j's score
 // (tile_score, the same roundings) beats thr: greater for inner product and
@@ -250,20 +145,6 @@ template <bool B>
 struct BoolTag {
   static constexpr bool value = B;
 };
-
-// v[j] for a run-time j, by a tree of selects (no local-memory indexing).
-__device__ __forceinline__ uint32_t select32(const uint32_t (&v)[32], int j) {
-  uint32_t t16[16], t8[8], t4[4], t2[2];
-#pragma unroll
-  for (int i = 0; i < 16; ++i) t16[i] = (j & 1) ? v[2 * i + 1] : v[2 * i];
-#pragma unroll
-  for (int i = 0; i < 8; ++i) t8[i] = (j & 2) ? t16[2 * i + 1] : t16[2 * i];
-#pragma unroll
-  for (int i = 0; i < 4; ++i) t4[i] = (j & 4) ? t8[2 * i + 1] : t8[2 * i];
-#pragma unroll
-  for (int i = 0; i < 2; ++i) t2[i] = (j & 8) ? t4[2 * i + 1] : t4[2 * i];
-  return (j & 16) ? t2[1] : t2[0];
-}
 
 struct TcLayout {
   int ns, nr, chunks;  // MMA stages, raw stages, K chunks per MMA stage
@@ -433,17 +314,15 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           }
           tc_fence_after();
           const uint32_t st = smem_u32(smem + (size_t)s * stage_stride);
-          for (int c = 0; c < nc; ++c) {
-            const uint64_t ahi = desc_sw64(st + c * kAStage),
-                           alo = desc_sw64(st + c * kAStage + kABytes),
-                           bd = desc_sw64(st + C * kAStage + c * kB16Bytes);
+          // the stage's MMAs from one asm block (see umma_chunks)
+          uint64_t ahi[2], alo[2], bd[2];
 #pragma unroll
-            for (int j = 0; j < kBK / kUmmaK; ++j) {
-              const uint64_t koff = (uint64_t)((j * kUmmaK * 2) >> 4);
-              umma_f16(d_tmem, ahi + koff, bd + koff, kIdesc, (kc + c > 0 || j > 0) ? 1u : 0u);
-              if (!g.hi) umma_f16(d_tmem, alo + koff, bd + koff, kIdesc, 1u);
-            }
+          for (int c = 0; c < 2; ++c) {
+            ahi[c] = desc_sw64(st + c * kAStage);
+            alo[c] = desc_sw64(st + c * kAStage + kABytes);
+            bd[c] = desc_sw64(st + C * kAStage + c * kB16Bytes);
           }
+          umma_chunks(d_tmem, nc, ahi, alo, bd, g.hi != 0, kIdesc, kc > 0 ? 1u : 0u);
           umma_commit(&empty[s]);
         }
         if (ok) umma_commit(&accf[buf]);
@@ -1345,17 +1224,15 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
           }
           tc_fence_after();
           const uint32_t st = smem_u32(smem + (size_t)s * C * kStageBytes);
-          for (int c = 0; c < nc; ++c) {
-            const uint64_t ahi = desc_sw64(st + c * kAStage),
-                           alo = desc_sw64(st + c * kAStage + kABytes),
-                           bd = desc_sw64(st + C * kAStage + c * kB16Bytes);
+          // the stage's MMAs from one asm block (see umma_chunks)
+          uint64_t ahi[2], alo[2], bd[2];
 #pragma unroll
-            for (int j = 0; j < kBK / kUmmaK; ++j) {
-              const uint64_t koff = (uint64_t)((j * kUmmaK * 2) >> 4);
-              umma_f16(d_tmem, ahi + koff, bd + koff, kIdesc, (kc + c > 0 || j > 0) ? 1u : 0u);
-              if (!g.hi) umma_f16(d_tmem, alo + koff, bd + koff, kIdesc, 1u);
-            }
+          for (int c = 0; c < 2; ++c) {
+            ahi[c] = desc_sw64(st + c * kAStage);
+            alo[c] = desc_sw64(st + c * kAStage + kABytes);
+            bd[c] = desc_sw64(st + C * kAStage + c * kB16Bytes);
           }
+          umma_chunks(d_tmem, nc, ahi, alo, bd, g.hi != 0, kIdesc, kc > 0 ? 1u : 0u);
           umma_commit(&empty[s]);
         }
         if (ok) umma_commit(&accf[buf]);
@@ -1611,6 +1488,17 @@ int gcd_i(int x, int y) {
 // of them); B = 1,024 over 27,986 rows 88 us against 72 + 12.
 constexpr int64_t kPreBlocks = 4;
 
+// Opt-in (LAM_SCORE_TM=1): the small-batch kernel with the codes in the MMA M
+// dimension.  Measured against the stage-loop kernel over 361,802 int16 rows:
+// 145 / 155 / 170 / 172 / 230 us at B = 3 / 8 / 16 / 32 / 64 against 153 /
+// 157 / 159 / 162 / 162 us, and slower on int8 codes; both are bound by the
+// raw-code supply of 128-byte row segments and their hand-offs, not by the
+// MMAs.
+bool tm_enabled() {
+  const char *e = getenv("LAM_SCORE_TM");
+  return e != nullptr && strcmp(e, "1") == 0;
+}
+
 bool tensor_fits(int width, int k, int64_t B) {
   if (k > kTcMaxK || (width != 1 && width != 2)) return false;
   if ((B + kBM - 1) / kBM >= kPreBlocks) return tc2_layout(k).ns >= 2;
@@ -1687,21 +1575,26 @@ cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st, const RowPt
     // one block of at most 64 queries: they take MMA rows 64 .. 127, read by
     // the epilogue warps that share the SM sub-partitions of the converters
     // only (the producer and MMA warps sit on the other two)
-    const int qoff = a.Bpad == kBM && a.B <= kBM / 2 ? kBM / 2 : 0;
+    // Opt-in: up to 64 queries with k <= 32 on the kernel with the codes in
+    // the MMA M dimension (queries from MMA row 0 of the image).
+    const bool tm = !hi && !rc && tm_fits(a.B, a.D, a.k) && tm_enabled();
+    const int qoff = !tm && a.Bpad == kBM && a.B <= kBM / 2 ? kBM / 2 : 0;
     qprep_kernel<<<q_blocks, 256, 0, st>>>(a.queries, a.B, a.D, a.Bpad, qA, qoff);
     timing_launch_end(LAM_TIME_AUX, st);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     CUtensorMap cmap1, cmap2;  // the codes as int8 and as int16 rows
+    const uint32_t box_rows = tm ? (uint32_t)tm_box_rows() : (uint32_t)kBN;
     if ((qst || a.width == 1) &&
         !make_map_2d(&cmap1, CU_TENSOR_MAP_DATA_TYPE_UINT8, a.codes, (uint64_t)a.D, (uint64_t)a.N,
-                     (uint64_t)a.D, (uint32_t)kRawRow, kBN, CU_TENSOR_MAP_SWIZZLE_128B))
+                     (uint64_t)a.D, (uint32_t)kRawRow, box_rows, CU_TENSOR_MAP_SWIZZLE_128B))
       return cudaErrorInvalidValue;
     if ((qst || a.width == 2) &&
         !make_map_2d(&cmap2, CU_TENSOR_MAP_DATA_TYPE_UINT16, a.codes, (uint64_t)a.D,
-                     (uint64_t)a.N, (uint64_t)a.D * 2, (uint32_t)(kRawRow / 2), kBN,
+                     (uint64_t)a.N, (uint64_t)a.D * 2, (uint32_t)(kRawRow / 2), box_rows,
                      CU_TENSOR_MAP_SWIZZLE_128B))
       return cudaErrorInvalidValue;
+    if (tm) return launch_score_tm(a, qst, cmap1, cmap2, st);
     const dim3 grid((unsigned)a.n_lists, (unsigned)(a.Bpad / kBM));
     // one pass of the stage-loop kernel over the lists of x.k keys
     auto pass = [&](const ScoreArgs &x, int hi_pass, int gate, int kind) -> cudaError_t {
