@@ -579,6 +579,8 @@ def measure_calls(lam, torch, dev, wl, parts, reps, batches=None, eps_list=None,
                                     "ms_span": ms, "ms_kernel": k_s, "ms_merge": k_m,
                                     "ms_prep": k_a,
                                     "vectors_per_s_span": N / (ms / 1e3),
+                                    "code_gbs_kernel": N * row_bytes[fmt] / (k_s / 1e3) / 1e9,
+                                    "frac_of_hbm_kernel": N * row_bytes[fmt] / (k_s / 1e3) / 1e9 / hbm,
                                     "tflops_kernel": fl / (k_s / 1e3) / 1e12,
                                     "frac_of_tensor_kernel": fl / (k_s / 1e3) / 1e12 / tc_peak})
                 del sws

@@ -14,6 +14,8 @@
 // instructions, so the kernel is bound by HBM at width bytes per element.
 #include "score_common.cuh"
 
+#include <type_traits>
+
 namespace lam {
 
 namespace {
@@ -815,6 +817,190 @@ __global__ void __launch_bounds__(kBwThreads, 1)
 }
 
 // ---------------------------------------------------------------------------
+// Sign-bit rows (per-vector codec), B <= 2: one lane per row.  The dot product
+// with the query is q . xhat = alpha (2 S - sum(q)), S = the sum of q_d over
+// the row's set bits.  S is gathered four bits at a time from per-query nibble
+// tables in shared memory, T[q][p][v] = sum of q_{4p + b} over the set bits b
+// of v (b = 0 .. 3, in that order), so a 768-bit row costs 192 table reads and
+// adds instead of 768 masked multiply-adds.  All lanes read the same nibble
+// position of their own rows at once, so a read touches at most 16 distinct
+// words of one 64-byte table row: no bank conflicts.  Stages hold contiguous
+// rows (bulk copies); warp w scores rows 32 w .. 32 w + 31 of each stage, and
+// one ballot per query admits candidates into the warp's register top-k in
+// row order.
+template <int QB, int KPL, bool CC, int NCH>
+__global__ void __launch_bounds__(kBwThreads, 1)
+    score_bw_sign_kernel(ScoreArgs a, RowPtrs rp, int tr, int ns, int stage_bytes) {
+  extern __shared__ __align__(1024) uint8_t smem[];
+  const int D = a.D;
+  const int npos = D / 4;  // nibbles per row
+  float *tab = reinterpret_cast<float *>(smem + (size_t)ns * stage_bytes);  // [QB][npos][16]
+  float *qstat = tab + (size_t)QB * npos * 16;                               // [QB][3]
+  uint64_t *full = reinterpret_cast<uint64_t *>(qstat + 4 * QB);
+  uint64_t *empty = full + ns;
+  volatile int *abort_flag = reinterpret_cast<volatile int *>(empty + ns);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t N = a.N;
+  const int64_t r0 = (int64_t)blockIdx.x * N / gridDim.x;
+  const int64_t r1 = (int64_t)(blockIdx.x + 1) * N / gridDim.x;
+  const int64_t nrows = r1 - r0;
+  const int ntiles = (int)((nrows + tr - 1) / tr);
+  const size_t row_bytes = (size_t)D / 8;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < ns; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], kBwWarps);
+    }
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  // the nibble tables
+  for (int e = threadIdx.x; e < QB * npos * 16; e += blockDim.x) {
+    const int q = e / (npos * 16), pv = e - q * npos * 16, pos = pv >> 4, v = pv & 15;
+    float t = 0.0f;
+    if (q < a.B) {
+      const float *qr = a.queries + (int64_t)q * D + 4 * pos;
+#pragma unroll
+      for (int b = 0; b < 4; ++b)
+        if (v & (1 << b)) t += qr[b];
+    }
+    tab[e] = t;
+  }
+  // sum(q), ||q|| and ||q||^2 per query (the norm from the query scaled near 1)
+  if (warp < QB) {
+    const int q = warp;
+    float sum = 0.0f, mx = 0.0f;
+    if (q < a.B)
+      for (int d = lane; d < D; d += 32) {
+        const float v = a.queries[(int64_t)q * D + d];
+        sum += v;
+        mx = fmaxf(mx, fabsf(v));
+      }
+    const float nsc = norm_scale(warp_max(mx));
+    float part = 0.0f;
+    if (q < a.B)
+      for (int d = lane; d < D; d += 32) {
+        const float u = a.queries[(int64_t)q * D + d] * nsc;
+        part = fmaf(u, u, part);
+      }
+    sum = warp_sum(sum);
+    const float qn = sqrtf(warp_sum(part)) / nsc;
+    if (lane == 0) {
+      qstat[3 * q] = sum;
+      qstat[3 * q + 1] = qn;
+      qstat[3 * q + 2] = qn * qn;
+    }
+  }
+  __syncthreads();
+
+  WarpList<KPL> lists[QB];
+#pragma unroll
+  for (int q = 0; q < QB; ++q) lists[q].init();
+
+  if (warp == kBwWarps) {
+    if (lane == 0) {
+      int issued = 0;
+      const int nt = producers_stalled(a.gflags) ? 0 : ntiles;
+      for (int t = 0; t < nt; ++t) {
+        const int s = t % ns, r = t / ns;
+        if (r > 0 && !mbar_wait(&empty[s], (r - 1) & 1, abort_flag, a.gflags)) break;
+        const int64_t nr = min((int64_t)tr, nrows - (int64_t)t * tr);
+        const uint32_t bytes = (uint32_t)(nr * row_bytes);
+        mbar_arrive_expect_tx(&full[s], bytes);
+        bulk_g2s(smem + (size_t)s * stage_bytes,
+                 static_cast<const uint8_t *>(a.codes) + (r0 + (int64_t)t * tr) * row_bytes,
+                 bytes, &full[s]);
+        issued = t + 1;
+      }
+      for (int t = max(0, issued - ns); t < issued; ++t) drain_wait(&full[t % ns], (t / ns) & 1);
+    }
+  } else {
+    const bool desc = a.metric != LAM_METRIC_L2;
+    float qs[QB], qn[QB], qq[QB], thr_s[QB];
+#pragma unroll
+    for (int q = 0; q < QB; ++q) {
+      qs[q] = qstat[3 * q];
+      qn[q] = qstat[3 * q + 1];
+      qq[q] = qstat[3 * q + 2];
+      thr_s[q] = desc ? -INFINITY : INFINITY;
+    }
+    // 16-byte pieces per row (128 bits); NCH > 0: that count, fully unrolled
+    const int nchunk = NCH > 0 ? NCH : (int)(row_bytes / 16);
+    for (int t = 0; t < ntiles; ++t) {
+      const int st = t % ns, r = t / ns;
+      if (!mbar_wait(&full[st], r & 1, abort_flag, a.gflags)) break;
+      const int nr = (int)min((int64_t)tr, nrows - (int64_t)t * tr);
+      const uint8_t *stage = smem + (size_t)st * stage_bytes;
+      for (int rb = warp * 32; rb < nr; rb += kBwWarps * 32) {
+        const int rr = rb + lane;
+        const bool valid = rr < nr;
+        const int64_t row = r0 + (int64_t)t * tr + rr;
+        const float alpha = valid ? rp.scale[row] : 0.0f;
+        const uint8_t *rowp = stage + (size_t)(valid ? rr : 0) * row_bytes;
+        float acc[QB][2];
+#pragma unroll
+        for (int q = 0; q < QB; ++q) acc[q][0] = acc[q][1] = 0.0f;
+#pragma unroll (NCH > 0 ? NCH : 1)
+        for (int c = 0; c < nchunk; ++c) {
+          const uint4 v = *reinterpret_cast<const uint4 *>(rowp + (size_t)c * 16);
+          const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            const int pos0 = (c * 4 + u) * 8;  // first nibble position of this word
+#pragma unroll
+            for (int n = 0; n < 8; ++n) {
+              const uint32_t nib = (w4[u] >> (4 * n)) & 15u;
+#pragma unroll
+              for (int q = 0; q < QB; ++q)
+                acc[q][n & 1] += tab[((size_t)q * npos + pos0 + n) * 16 + nib];
+            }
+          }
+        }
+        const float xx = CC ? (float)D * alpha * alpha : 0.0f;
+#pragma unroll
+        for (int q = 0; q < QB; ++q) {
+          const float S = acc[q][0] + acc[q][1];
+          const float dot = alpha * fmaf(2.0f, S, -qs[q]);
+          float sc;
+          if (a.metric == LAM_METRIC_IP) sc = dot;
+          else if (a.metric == LAM_METRIC_COSINE)
+            sc = (qn[q] == 0.0f || xx == 0.0f) ? 0.0f : dot / (qn[q] * sqrtf(xx));
+          else sc = fmaf(-2.0f, dot, qq[q] + xx);
+          if (q >= a.B) continue;
+          uint32_t m = __ballot_sync(0xffffffffu, valid && (desc ? sc > thr_s[q] : sc < thr_s[q]));
+          while (m != 0) {
+            const int l = __ffs(m) - 1;
+            m &= m - 1;
+            const float sl = __shfl_sync(0xffffffffu, sc, l);
+            if (desc ? sl > thr_s[q] : sl < thr_s[q]) {
+              lists[q].insert(make_key(sl, (uint32_t)(r0 + (int64_t)t * tr + rb + l), desc), lane);
+              const uint64_t kk = lists[q].kth(a.k);
+              thr_s[q] = kk == kSentinel ? (desc ? -INFINITY : INFINITY)
+                                         : rank_key32_score((uint32_t)(kk >> 32), desc);
+            }
+          }
+        }
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&empty[st]);
+    }
+  }
+  __syncthreads();
+  uint64_t *cand = reinterpret_cast<uint64_t *>(smem);
+  if (warp < kBwWarps) {
+#pragma unroll
+    for (int q = 0; q < QB; ++q)
+      lists[q].store(cand + ((size_t)q * kBwWarps + warp) * a.k, a.k, lane);
+  }
+  __syncthreads();
+  for (int q = 0; q < QB && q < a.B; ++q)
+    rank_merge(cand + (size_t)q * kBwWarps * a.k, kBwWarps, a.k,
+               a.partial + ((size_t)blockIdx.x * a.B + q) * a.k, threadIdx.x, kBwThreads);
+}
+
+// ---------------------------------------------------------------------------
 // Generic path: any D, width 1/2/4, k <= 1024, any batch.  Grid (ctas, B):
 // a CTA scores one query against a range of rows, warp per row with plain
 // global loads, per-warp top-k lists in shared memory, then a rank merge.
@@ -1429,6 +1615,34 @@ static cudaError_t launch_bw_rows_f(const ScoreArgs &a, const RowPtrs &rp, const
                    : launch_bw_rows_t<FMT, 2, 4>(a, rp, sh, st);
 }
 
+template <int QB, int KPL>
+static cudaError_t launch_bw_sign_t(const ScoreArgs &a, const RowPtrs &rp, const BwShape &sh,
+                                   cudaStream_t st) {
+  const size_t smem = (size_t)sh.ns * sh.stage_bytes + (size_t)QB * (a.D / 4) * 16 * 4 +
+                      16 * QB + 2 * sh.ns * sizeof(uint64_t) + 16;
+  auto pick = [&](auto cc) {
+    constexpr bool CC = decltype(cc)::value;
+    return a.D == 768    ? score_bw_sign_kernel<QB, KPL, CC, 6>
+           : a.D == 1024 ? score_bw_sign_kernel<QB, KPL, CC, 8>
+                         : score_bw_sign_kernel<QB, KPL, CC, 0>;
+  };
+  auto kern = a.metric == LAM_METRIC_IP ? pick(std::integral_constant<bool, false>{})
+                                        : pick(std::integral_constant<bool, true>{});
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  timing_launch_begin(LAM_TIME_SCORE, st);
+  kern<<<a.n_lists, kBwThreads, smem, st>>>(a, rp, sh.tr, sh.ns, sh.stage_bytes);
+  timing_launch_end(LAM_TIME_SCORE, st);
+  return cudaGetLastError();
+}
+
+static cudaError_t launch_bw_sign(const ScoreArgs &a, const RowPtrs &rp, const BwShape &sh,
+                                  cudaStream_t st) {
+  if (a.B == 1)
+    return a.k <= 32 ? launch_bw_sign_t<1, 1>(a, rp, sh, st) : launch_bw_sign_t<1, 4>(a, rp, sh, st);
+  return a.k <= 32 ? launch_bw_sign_t<2, 1>(a, rp, sh, st) : launch_bw_sign_t<2, 4>(a, rp, sh, st);
+}
+
 int rows_row_bytes(int fmt, int D) {
   return fmt == LAM_ROWS_INT8 ? D : fmt == LAM_ROWS_FP16 ? 2 * D : D / 8;
 }
@@ -1442,7 +1656,7 @@ cudaError_t launch_score_bandwidth_rows(const ScoreArgs &a, const RowPtrs &rp, c
   if ((size_t)2 * kBwWarps * a.k * 8 > (size_t)sh.ns * sh.stage_bytes) return cudaErrorInvalidValue;
   if (a.fmt == LAM_ROWS_INT8) return launch_bw_rows_f<LAM_ROWS_INT8>(a, rp, sh, st);
   if (a.fmt == LAM_ROWS_FP16) return launch_bw_rows_f<LAM_ROWS_FP16>(a, rp, sh, st);
-  return launch_bw_rows_f<LAM_ROWS_SIGN>(a, rp, sh, st);
+  return launch_bw_sign(a, rp, sh, st);
 }
 
 cudaError_t launch_score_generic(const ScoreArgs &a, cudaStream_t st, const RowPtrs &rp) {
