@@ -635,12 +635,110 @@ __global__ void __launch_bounds__(kBwThreads, 1)
     float f_sr = 1.0f, f_or = 0.0f;
     if (FMT != LAM_ROWS_FP16 && frow < r1) f_sr = rp.scale[frow];
     if (FMT == LAM_ROWS_INT8 && frow < r1) f_or = rp.offset[frow];
+    // int8 rows, one query: the factors of the row this lane finishes in its
+    // warp's next group of kRg rows (lane L finishes row (L >> lsh) % kRg)
+    constexpr int kLsh = CC ? 1 : 3;
+    const int g_row = (lane >> kLsh) & (kRg - 1);
+    float p_sr = 1.0f, p_or = 0.0f;
+    if (FMT == LAM_ROWS_INT8 && QB == 1) {
+      const int64_t row = r0 + warp * kRg + g_row;
+      if (row < r1) {
+        p_sr = rp.scale[row];
+        p_or = rp.offset[row];
+      }
+    }
 
     for (int t = 0; t < ntiles; ++t) {
       const int st = t % ns, r = t / ns;
       if (!mbar_wait(&full[st], r & 1, abort_flag, a.gflags)) break;
       const int nr = (int)min((int64_t)tr, nrows - (int64_t)t * tr);
       const uint8_t *stage = smem + (size_t)st * stage_bytes;
+      if constexpr (FMT == LAM_ROWS_INT8 && QB == 1) {
+        // As the Q_eps int8 single-query consumer: kRg consecutive rows per
+        // warp pass, all code words loaded first, per lane the integer dot
+        // products against the query's digit planes (and sum c, sum c^2 for
+        // cosine / L2), one transposed butterfly for every row's totals, the
+        // rows' scale and offset prefetched one group ahead, one ballot.
+        constexpr int V = CC ? 4 * kRg : kRg;  // dot, sum c, sum c^2, padding
+        for (int g0 = warp * kRg; g0 < nr; g0 += kBwWarps * kRg) {
+          const float sr = p_sr, orr = p_or;
+          {
+            const int ng = g0 + kBwWarps * kRg;
+            const int64_t nrow = ng < nr ? r0 + (int64_t)t * tr + ng + g_row
+                                         : r0 + (int64_t)(t + 1) * tr + warp * kRg + g_row;
+            if (nrow < r1) {
+              p_sr = rp.scale[nrow];
+              p_or = rp.offset[nrow];
+            }
+          }
+          uint2 cw[kRg][kNchMax];
+#pragma unroll
+          for (int i = 0; i < kRg; ++i) {
+            const uint8_t *pr = stage + (size_t)min(g0 + i, nr - 1) * row_bytes;
+#pragma unroll
+            for (int j = 0; j < kNchMax; ++j) {
+              const int e0 = (j * 32 + lane) * 8;
+              cw[i][j] = (j < nch && e0 < D) ? *reinterpret_cast<const uint2 *>(pr + e0)
+                                             : make_uint2(0u, 0u);
+            }
+          }
+          float v[V];
+#pragma unroll
+          for (int i = 0; i < kRg; ++i) {
+            int d0 = 0, d1 = 0, d2 = 0, c1 = 0, c2 = 0;
+#pragma unroll
+            for (int j = 0; j < kNchMax; ++j) {
+              if (j < nch) {  // (warp-uniform)
+                const int wx = (int)cw[i][j].x, wy = (int)cw[i][j].y;
+                d0 = __dp4a(wx, (int)qdig[0][j][0][0], __dp4a(wy, (int)qdig[0][j][0][1], d0));
+                d1 = __dp4a(wx, (int)qdig[0][j][1][0], __dp4a(wy, (int)qdig[0][j][1][1], d1));
+                d2 = __dp4a(wx, (int)qdig[0][j][2][0], __dp4a(wy, (int)qdig[0][j][2][1], d2));
+                if constexpr (CC) {
+                  c1 = __dp4a(wx, 0x01010101, __dp4a(wy, 0x01010101, c1));
+                  c2 = __dp4a(wx, wx, __dp4a(wy, wy, c2));
+                }
+              }
+            }
+            v[i] = fmaf((float)d0, 65536.0f, fmaf((float)d1, 256.0f, (float)d2));
+            if constexpr (CC) {
+              v[kRg + i] = (float)c1;
+              v[2 * kRg + i] = (float)c2;
+              v[3 * kRg + i] = 0.0f;
+            }
+          }
+          // lane L: the total of value L >> kLsh (CC: dot of row L / 2 on lanes
+          // 0-7, its sum c 8 lanes and its sum c^2 16 lanes further on)
+          const float tot = warp_sums_transposed<V>(v, lane);
+          const float c1 = CC ? __shfl_down_sync(0xffffffffu, tot, 8) : 0.0f;
+          const float c2 = CC ? __shfl_down_sync(0xffffffffu, tot, 16) : 0.0f;
+          const float acc = tot * qinv[0];
+          const float dot = fmaf(sr, acc, orr * qs[0]);
+          const float xx = CC ? fmaf(sr * sr, c2, fmaf(2.0f * sr * orr, c1, (float)D * orr * orr))
+                              : 0.0f;
+          float sc;
+          if (a.metric == LAM_METRIC_IP) sc = dot;
+          else if (a.metric == LAM_METRIC_COSINE)
+            sc = (qn[0] == 0.0f || xx == 0.0f) ? 0.0f : dot / (qn[0] * sqrtf(xx));
+          else sc = fmaf(-2.0f, dot, qq[0] + xx);
+          const bool leader = CC ? (lane < 2 * kRg && (lane & 1) == 0) : (lane & 7) == 0;
+          unsigned pass = __ballot_sync(0xffffffffu, leader && g0 + g_row < nr &&
+                                                         (desc ? sc > thr_s[0] : sc < thr_s[0]));
+          while (pass) {
+            const int l = __ffs(pass) - 1;
+            pass &= pass - 1;
+            const float sl = __shfl_sync(0xffffffffu, sc, l);
+            if (!(desc ? sl > thr_s[0] : sl < thr_s[0])) continue;  // the list moved on
+            const int64_t row = r0 + (int64_t)t * tr + g0 + ((l >> kLsh) & (kRg - 1));
+            lists[0].insert(make_key(sl, (uint32_t)row, desc), lane);
+            const uint64_t kk = lists[0].kth(a.k);
+            thr_s[0] = kk == kSentinel ? (desc ? -INFINITY : INFINITY)
+                                       : rank_key32_score((uint32_t)(kk >> 32), desc);
+          }
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&empty[st]);
+        continue;
+      }
       for (int rr = warp; rr < nr; rr += 2 * kBwWarps) {
         const int rb = rr + kBwWarps;
         const bool has_b = rb < nr;
