@@ -954,35 +954,35 @@ __global__ void __launch_bounds__(kBwThreads, 1)
     *abort_flag = 0;
     fence_barrier_init();
   }
-  // the nibble tables
+  // the nibble tables, from a copy of the queries in the first (still empty) stage
+  float *qsm = reinterpret_cast<float *>(smem);
+  for (int e = threadIdx.x; e < QB * D; e += blockDim.x)
+    qsm[e] = e < a.B * D ? a.queries[e] : 0.0f;
+  __syncthreads();
   for (int e = threadIdx.x; e < QB * npos * 16; e += blockDim.x) {
     const int q = e / (npos * 16), pv = e - q * npos * 16, pos = pv >> 4, v = pv & 15;
+    const float *qr = qsm + q * D + 4 * pos;
     float t = 0.0f;
-    if (q < a.B) {
-      const float *qr = a.queries + (int64_t)q * D + 4 * pos;
 #pragma unroll
-      for (int b = 0; b < 4; ++b)
-        if (v & (1 << b)) t += qr[b];
-    }
+    for (int b = 0; b < 4; ++b)
+      if (v & (1 << b)) t += qr[b];
     tab[e] = t;
   }
   // sum(q), ||q|| and ||q||^2 per query (the norm from the query scaled near 1)
   if (warp < QB) {
     const int q = warp;
     float sum = 0.0f, mx = 0.0f;
-    if (q < a.B)
-      for (int d = lane; d < D; d += 32) {
-        const float v = a.queries[(int64_t)q * D + d];
-        sum += v;
-        mx = fmaxf(mx, fabsf(v));
-      }
+    for (int d = lane; d < D; d += 32) {
+      const float v = qsm[q * D + d];
+      sum += v;
+      mx = fmaxf(mx, fabsf(v));
+    }
     const float nsc = norm_scale(warp_max(mx));
     float part = 0.0f;
-    if (q < a.B)
-      for (int d = lane; d < D; d += 32) {
-        const float u = a.queries[(int64_t)q * D + d] * nsc;
-        part = fmaf(u, u, part);
-      }
+    for (int d = lane; d < D; d += 32) {
+      const float u = qsm[q * D + d] * nsc;
+      part = fmaf(u, u, part);
+    }
     sum = warp_sum(sum);
     const float qn = sqrtf(warp_sum(part)) / nsc;
     if (lane == 0) {
@@ -1026,6 +1026,13 @@ __global__ void __launch_bounds__(kBwThreads, 1)
     }
     // 16-byte pieces per row (128 bits); NCH > 0: that count, fully unrolled
     const int nchunk = NCH > 0 ? NCH : (int)(row_bytes / 16);
+    // the row scale one pass ahead (the warp's passes are 32 kBwWarps rows
+    // apart, or start the next tile at the same offset)
+    float p_alpha = 0.0f;
+    {
+      const int64_t row = r0 + warp * 32 + lane;
+      if (warp * 32 < tr && row < r1) p_alpha = rp.scale[row];
+    }
     for (int t = 0; t < ntiles; ++t) {
       const int st = t % ns, r = t / ns;
       if (!mbar_wait(&full[st], r & 1, abort_flag, a.gflags)) break;
@@ -1034,8 +1041,13 @@ __global__ void __launch_bounds__(kBwThreads, 1)
       for (int rb = warp * 32; rb < nr; rb += kBwWarps * 32) {
         const int rr = rb + lane;
         const bool valid = rr < nr;
-        const int64_t row = r0 + (int64_t)t * tr + rr;
-        const float alpha = valid ? rp.scale[row] : 0.0f;
+        const float alpha = valid ? p_alpha : 0.0f;
+        {
+          const int nb = rb + kBwWarps * 32;
+          const int64_t nrow = nb < nr ? r0 + (int64_t)t * tr + nb + lane
+                                       : r0 + (int64_t)(t + 1) * tr + warp * 32 + lane;
+          if (nrow < r1) p_alpha = rp.scale[nrow];
+        }
         const uint8_t *rowp = stage + (size_t)(valid ? rr : 0) * row_bytes;
         float acc[QB][2];
 #pragma unroll
