@@ -116,10 +116,82 @@ __device__ __forceinline__ void put_codes(void *codes, int64_t i, const int32_t 
 // Quantizes and hashes every band of x (nbands_total = N * D / r bands, band j
 // covering x[j r, j r + r)); V values per load (r a multiple of V, x 4V-byte
 // aligned).  Codes are written when `codes` is not NULL.
+// Bands of exactly LB loads of V values (r = LB V), U bands per thread and
+// iteration (bands j, j + stride, ...): every load of the U bands is issued
+// before any of them is quantized, so a thread keeps U LB loads in flight.
+template <int W, int V, bool TRACK, int U, int LB>
+__device__ __forceinline__ void bands_body_u(const float *__restrict__ x, int64_t nbands_total,
+                                             int nb, float s, void *__restrict__ codes,
+                                             uint64_t *__restrict__ digests, QuantStatus *st) {
+  constexpr int r = LB * V;
+  const int64_t tid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  const int step_b = (int)(stride % nb);  // band index advance per grid stride
+  int b = (int)(tid % nb);
+  const QDiv qd = QDiv::of(s);
+  BRange rg;
+  for (int64_t j0 = tid; j0 < nbands_total; j0 += (int64_t)U * stride) {
+    float f[U][r];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int64_t j = j0 + (int64_t)u * stride;
+#pragma unroll
+      for (int l = 0; l < LB; ++l) {
+        const int64_t i = j * r + l * V;
+        if (j < nbands_total) {
+          if (V == 4) {
+            const float4 t = __ldg(reinterpret_cast<const float4 *>(x + i));
+            f[u][l * V] = t.x;
+            f[u][(l * V + 1) % r] = t.y;
+            f[u][(l * V + 2) % r] = t.z;
+            f[u][(l * V + 3) % r] = t.w;
+          } else if (V == 2) {
+            const float2 t = __ldg(reinterpret_cast<const float2 *>(x + i));
+            f[u][l * V] = t.x;
+            f[u][(l * V + 1) % r] = t.y;
+          } else {
+            f[u][l * V] = __ldg(x + i);
+          }
+        }
+      }
+    }
+    int bu = b;
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int64_t j = j0 + (int64_t)u * stride;
+      if (j < nbands_total) {
+        uint64_t h = fnv_byte(fnv_byte(kFnvOffset, (uint32_t)bu), (uint32_t)bu >> 8);
+#pragma unroll
+        for (int l = 0; l < LB; ++l) {
+          int32_t c[V];
+#pragma unroll
+          for (int e = 0; e < V; ++e) {
+            const float fe = f[u][l * V + e];
+            if (TRACK) rg.add(fe);
+            c[e] = qd.code(fe);
+#pragma unroll
+            for (int t = 0; t < W; ++t) h = fnv_byte(h, (uint32_t)c[e] >> (8 * t));
+          }
+          if (codes != nullptr) put_codes<W, V>(codes, j * r + l * V, c);
+        }
+        digests[j] = h;
+      }
+      bu += step_b;
+      if (bu >= nb) bu -= nb;
+    }
+    b = bu;
+  }
+  if (TRACK) rg.flush(st);
+}
+
 template <int W, int V, bool TRACK>
 __device__ __forceinline__ void bands_body(const float *__restrict__ x, int64_t nbands_total,
                                            int r, int nb, float s, void *__restrict__ codes,
                                            uint64_t *__restrict__ digests, QuantStatus *st) {
+  // one load per band: four bands per thread and iteration; two loads per band:
+  // both issued before the band is quantized (measured best of 1/2/4/8 bands)
+  if (r == V) return bands_body_u<W, V, TRACK, 4, 1>(x, nbands_total, nb, s, codes, digests, st);
+  if (r == 2 * V) return bands_body_u<W, V, TRACK, 1, 2>(x, nbands_total, nb, s, codes, digests, st);
   const int64_t tid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   const int step_b = (int)(stride % nb);  // band index advance per grid stride

@@ -206,10 +206,21 @@ def test_bandwidth_path(dev, score_path, fmt, metric, B, k):
 
 @pytest.mark.parametrize("fmt", FMTS)
 @pytest.mark.parametrize("d", [128, 256, 1024])
-def test_bandwidth_path_dims(dev, score_path, fmt, d):
+@pytest.mark.parametrize("B", [1, 2])
+def test_bandwidth_path_dims(dev, score_path, fmt, d, B):
     score_path("bandwidth")
     for metric in METRICS:
-        rows_case(dev, fmt, 777, d, 2, 10, metric, seed=d)
+        rows_case(dev, fmt, 777, d, B, 10, metric, seed=d + B)
+
+
+@pytest.mark.parametrize("fmt", FMTS)
+@pytest.mark.parametrize("n", [1, 5, 63, 64, 65, 1029])
+def test_bandwidth_path_ragged_rows(dev, score_path, fmt, n):
+    # fewer rows than one stage or one warp group, and ragged last stages: the
+    # one-query paths prefetch row factors across groups and stages
+    score_path("bandwidth")
+    for metric in METRICS:
+        rows_case(dev, fmt, n, 768, 1, min(10, n), metric, seed=n)
 
 
 def test_bandwidth_path_routing(dev):
