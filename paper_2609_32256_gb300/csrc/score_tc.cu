@@ -33,6 +33,7 @@
 #include "score_common.cuh"
 #include "tc_common.cuh"
 
+#include <cstdio>
 #include <cstdlib>
 #include <cstring>
 
@@ -44,7 +45,6 @@ constexpr int kBM = 128;        // queries per CTA (MMA M)
 constexpr int kBN = 256;        // code rows per tile (MMA N)
 constexpr int kBK = 32;         // fp16 per stage along D (64-byte rows)
 static_assert(kBK == 32, "tensor_k_extent (lam_internal.cuh) rounds D to 32-wide K chunks");
-constexpr int kUmmaK = 16;      // K of one kind::f16 MMA
 constexpr int kTcThreads = 352;  // 11 warps, roles below
 constexpr int kConvThreads = 128;
 constexpr int kABytes = kBM * kBK * 2;    // one of hi / lo: 8 KB
@@ -61,6 +61,7 @@ constexpr int kMaxDynSmem = 232448;       // 227 KB
 constexpr int kTcMaxK = 128;
 // M = 128 queries, N = 256 code rows
 constexpr uint32_t kIdesc = idesc_f16(kBM, kBN);
+constexpr uint32_t kIdescPair = idesc_f16(2 * kBM, kBN);  // a CTA pair: M = 256
 
 // Candidate mask of one 32-column chunk: bit j is set when column j's score
 // (tile_score, the same roundings) beats thr: greater for inner product and
@@ -1049,8 +1050,10 @@ struct Tc2Layout {
   size_t lists_off, cbuf_off, bar_off, smem_bytes;
 };
 
-inline Tc2Layout tc2_layout(int k) {
+inline Tc2Layout tc2_layout(int k, bool pair = false) {
   Tc2Layout L;
+  // (pair: each CTA of a 2-CTA cluster stages half of each chunk's code rows)
+  const size_t stage = (size_t)kAStage + (pair ? kB16Bytes / 2 : kB16Bytes);
   // (k <= 32 keeps its candidates in registers, k > 32 a heap per query in
   // shared memory; stages of kTc2Chunks chunks while two of them fit beside
   // the heaps, else single-chunk stages)
@@ -1059,16 +1062,16 @@ inline Tc2Layout tc2_layout(int k) {
   size_t cbuf = 0;  // k > 32: the heaps' candidate buffers (as in the stage-loop kernel)
   if (k > 32) {
     const size_t room = kMaxDynSmem - lists - tailb;
-    const size_t need = 2 * (size_t)kStageBytes;
+    const size_t need = 2 * stage;
     const size_t slots = room > need ? (room - need) / ((size_t)kBM * 8) : 0;
     cbuf = (slots < (size_t)kCBuf ? slots : (size_t)kCBuf) * kBM * 8;
   }
   const size_t avail = kMaxDynSmem - lists - cbuf - tailb;
-  L.chunks = avail / ((size_t)kTc2Chunks * kStageBytes) >= 2 ? kTc2Chunks : 1;
-  int ns = (int)(avail / ((size_t)L.chunks * kStageBytes));
+  L.chunks = avail / ((size_t)kTc2Chunks * stage) >= 2 ? kTc2Chunks : 1;
+  int ns = (int)(avail / ((size_t)L.chunks * stage));
   if (ns > 8) ns = 8;
   L.ns = ns;
-  L.lists_off = (size_t)ns * L.chunks * kStageBytes;
+  L.lists_off = (size_t)ns * L.chunks * stage;
   L.cbuf_off = L.lists_off + lists;
   L.bar_off = L.cbuf_off + cbuf;
   L.smem_bytes = L.bar_off + tailb;
@@ -1127,10 +1130,19 @@ __device__ __forceinline__ float fac_score(const RowFac<true> &f, float acc, con
   return q.metric == LAM_METRIC_L2 ? fmaf(-2.0f, dot, q.qq + f.z) : dot;
 }
 
-template <int KR, bool RC>
+// PAIR: the CTAs of a 2-CTA cluster take query blocks 2j and 2j + 1 over the
+// same code tiles.  Each stages its 128 queries and half of each chunk's 256
+// code rows (the even CTA rows 0-127, the odd one rows 128-255); the even
+// CTA's issuer waits for both halves (the odd CTA's MMA warp relays "stage s
+// landed" by a remote arrive) and issues M = 256 MMAs, so each accumulator
+// holds its CTA's 128 queries x all 256 rows while each SM takes in 24 KB per
+// chunk instead of 32 KB.  Its commits free the stage and fill the
+// accumulator in both CTAs; the accumulator is free again when the epilogue
+// threads of both CTAs arrived.  Two-pass (hi / gated) launches are not pairs.
+template <int KR, bool RC, bool PAIR = false>
 __global__ void __launch_bounds__(kTc2Threads, 1)
     score_tc2_kernel(ScoreArgs a, Tc2Geom g) {
-  if (g.gate && hi_all_certified(a.gflags)) return;
+  if (!PAIR && g.gate && hi_all_certified(a.gflags)) return;
   extern __shared__ uint8_t tc_smem_raw[];
   const uint32_t base_u32 = smem_u32(tc_smem_raw);
   uint8_t *smem = tc_smem_raw + (((base_u32 + 1023u) & ~1023u) - base_u32);
@@ -1141,14 +1153,21 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
   uint64_t *accf = empty + ns;
   uint64_t *acce = accf + 2;
   uint64_t *done = acce + 2;
-  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(done + 1);
+  uint64_t *pfull = done + 1;  // PAIR, even CTA: the odd CTA's stage s landed
+  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(pfull + ns);
   volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
+  constexpr int kBSlot = PAIR ? kB16Bytes / 2 : kB16Bytes;  // code bytes per chunk staged here
+  const size_t stage_bytes = (size_t)kAStage + kBSlot;
+  const uint32_t rank = PAIR ? cluster_rank() : 0u;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int qb = blockIdx.y;
+  // grid: (splits of the code tiles, query blocks); pairs take (query blocks,
+  // splits), the pair along the cluster's x dimension as the MMA pair needs
+  const int qb = PAIR ? blockIdx.x : blockIdx.y;
+  const int split = PAIR ? blockIdx.y : blockIdx.x, nsplit = PAIR ? gridDim.y : gridDim.x;
   const int64_t n_tiles = (g.nrows + kBN - 1) / kBN;
-  const int64_t tb = (int64_t)blockIdx.x * n_tiles / gridDim.x;
-  const int64_t te = (int64_t)(blockIdx.x + 1) * n_tiles / gridDim.x;
+  const int64_t tb = (int64_t)split * n_tiles / nsplit;
+  const int64_t te = (int64_t)(split + 1) * n_tiles / nsplit;
   const int ntl = (int)(te - tb);
   const int nk = (a.D + kBK - 1) / kBK;
   const bool need_cc = RC || a.metric != LAM_METRIC_IP;
@@ -1161,16 +1180,24 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&accf[b], 1);
-      mbar_init(&acce[b], 128);
+      mbar_init(&acce[b], PAIR ? 256 : 128);
     }
     mbar_init(done, 1);
+    if (PAIR)
+      for (int s = 0; s < ns; ++s) mbar_init(&pfull[s], 1);
     *abort_flag = 0;
     fence_barrier_init();
     fence_proxy_async_smem();
   }
-  if (warp == 1) tmem_alloc(tmem_slot, kTmemCols);
-  tc_fence_before();
-  __syncthreads();
+  if constexpr (PAIR) {
+    if (warp == 1) tmem_alloc_pair(tmem_slot, kTmemCols);
+    tc_fence_before();
+    cluster_sync_all();  // (both CTAs' barriers initialised before any remote arrive)
+  } else {
+    if (warp == 1) tmem_alloc(tmem_slot, kTmemCols);
+    tc_fence_before();
+    __syncthreads();
+  }
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
@@ -1189,55 +1216,89 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
             break;
           }
           // stage: [query blocks of the nc chunks][code blocks of the nc chunks]
-          uint8_t *st = smem + (size_t)s * C * kStageBytes;
+          uint8_t *st = smem + (size_t)s * C * stage_bytes;
           const uint8_t *qsrc = qA + ((size_t)qb * nk + kc) * kAStage;
-          mbar_arrive_expect_tx(&full[s], (uint32_t)nc * ((g.hi ? kABytes : kAStage) + kB16Bytes));
+          mbar_arrive_expect_tx(&full[s], (uint32_t)nc * ((g.hi ? kABytes : kAStage) + kBSlot));
           if (!g.hi) {
             bulk_g2s(st, qsrc, (uint32_t)nc * kAStage, &full[s]);
           } else {  // the hi images only
             for (int c = 0; c < nc; ++c)
               bulk_g2s(st + (size_t)c * kAStage, qsrc + (size_t)c * kAStage, kABytes, &full[s]);
           }
-          bulk_g2s(st + C * kAStage, g.b16 + ((size_t)tile * nk + kc) * kB16Bytes,
-                   (uint32_t)nc * kB16Bytes, &full[s]);
+          if constexpr (PAIR) {  // this CTA's 128 of each chunk's 256 code rows
+            for (int c = 0; c < nc; ++c)
+              bulk_g2s(st + C * kAStage + c * kBSlot,
+                       g.b16 + ((size_t)tile * nk + kc + c) * kB16Bytes + rank * kBSlot, kBSlot,
+                       &full[s]);
+          } else {
+            bulk_g2s(st + C * kAStage, g.b16 + ((size_t)tile * nk + kc) * kB16Bytes,
+                     (uint32_t)nc * kB16Bytes, &full[s]);
+          }
           issued = it + 1;
         }
       }
       for (int t = max(0, issued - ns); t < issued; ++t) drain_wait_tc(&full[t % ns], (t / ns) & 1);
     }
   } else if (warp == 1) {
-    // ------------------------------------------------ MMA issuer ---------
-    if (lane == 0) {
+    if (PAIR && rank == 1) {
+      // ---------------------------------- odd CTA of a pair: stage relay ---
+      if (lane == 0) {
+        int it = 0;
+        bool ok = true;
+        for (int lt = 0; lt < ntl && ok; ++lt)
+          for (int kc = 0; kc < nk; kc += C, ++it) {
+            const int s = it % ns, r = it / ns;
+            if (!mbar_wait(&full[s], r & 1, abort_flag, a.gflags)) {
+              ok = false;
+              break;
+            }
+            mbar_arrive_peer(&pfull[s], 0);
+          }
+      }
+    } else if (lane == 0) {
+      // ------------------------------------------------ MMA issuer ---------
       int it = 0;
       bool ok = true;
       for (int lt = 0; lt < ntl && ok; ++lt) {
         const int buf = lt & 1, u = lt >> 1;
-        if (u > 0 && !mbar_wait(&acce[buf], (u - 1) & 1, abort_flag, a.gflags)) break;
+        if (u > 0 && !(PAIR ? mbar_wait_cl(&acce[buf], (u - 1) & 1, abort_flag, a.gflags)
+                            : mbar_wait(&acce[buf], (u - 1) & 1, abort_flag, a.gflags)))
+          break;
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(buf * kBN);
         for (int kc = 0; kc < nk; kc += C, ++it) {
           const int s = it % ns, r = it / ns;
           const int nc = nk - kc < C ? nk - kc : C;
-          if (!mbar_wait(&full[s], r & 1, abort_flag, a.gflags)) {
+          if (!mbar_wait(&full[s], r & 1, abort_flag, a.gflags) ||
+              (PAIR && !mbar_wait_cl(&pfull[s], r & 1, abort_flag, a.gflags))) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t st = smem_u32(smem + (size_t)s * C * kStageBytes);
+          const uint32_t st = smem_u32(smem + (size_t)s * C * stage_bytes);
           // the stage's MMAs from one asm block (see umma_chunks)
           uint64_t ahi[2], alo[2], bd[2];
 #pragma unroll
           for (int c = 0; c < 2; ++c) {
             ahi[c] = desc_sw64(st + c * kAStage);
             alo[c] = desc_sw64(st + c * kAStage + kABytes);
-            bd[c] = desc_sw64(st + C * kAStage + c * kB16Bytes);
+            bd[c] = desc_sw64(st + C * kAStage + c * kBSlot);
           }
-          umma_chunks(d_tmem, nc, ahi, alo, bd, g.hi != 0, kIdesc, kc > 0 ? 1u : 0u);
-          umma_commit(&empty[s]);
+          if constexpr (PAIR) {
+            umma_chunks<2>(d_tmem, nc, ahi, alo, bd, g.hi != 0, kIdescPair, kc > 0 ? 1u : 0u);
+            umma_commit_pair(&empty[s], 3);
+          } else {
+            umma_chunks(d_tmem, nc, ahi, alo, bd, g.hi != 0, kIdesc, kc > 0 ? 1u : 0u);
+            umma_commit(&empty[s]);
+          }
         }
-        if (ok) umma_commit(&accf[buf]);
+        if (ok) {
+          if constexpr (PAIR) umma_commit_pair(&accf[buf], 3);
+          else umma_commit(&accf[buf]);
+        }
       }
-      umma_commit(done);
+      if constexpr (PAIR) umma_commit_pair(done, 1);
+      else umma_commit(done);
       drain_wait_tc(done, 0);
     }
   } else {
@@ -1413,10 +1474,11 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
         }
       }
       tc_fence_before();
-      mbar_arrive(&acce[buf]);
+      if (PAIR && rank == 1) mbar_arrive_peer(&acce[buf], 0);  // (the even CTA's issuer)
+      else mbar_arrive(&acce[buf]);
     }
     if (qvalid) {
-      uint64_t *out = a.partial + ((size_t)(g.list_base + blockIdx.x) * a.B + qidx) * k;
+      uint64_t *out = a.partial + ((size_t)(g.list_base + split) * a.B + qidx) * k;
       if (KR > 0) {
 #pragma unroll
         for (int i = 0; i < RK; ++i)
@@ -1430,10 +1492,20 @@ __global__ void __launch_bounds__(kTc2Threads, 1)
   }
 
   tc_fence_before();
-  __syncthreads();
-  if (warp == 1) {
-    tc_fence_after();
-    tmem_dealloc(tmem_base, kTmemCols);
+  if constexpr (PAIR) {
+    // (the even CTA's MMAs, which read this CTA's stages, have drained)
+    cluster_sync_all();
+    if (warp == 1) {
+      tc_fence_after();
+      tmem_dealloc_pair(tmem_base, kTmemCols);
+    }
+    cluster_sync_all();
+  } else {
+    __syncthreads();
+    if (warp == 1) {
+      tc_fence_after();
+      tmem_dealloc(tmem_base, kTmemCols);
+    }
   }
 }
 
@@ -1497,6 +1569,60 @@ constexpr int64_t kPreBlocks = 4;
 bool tm_enabled() {
   const char *e = getenv("LAM_SCORE_TM");
   return e != nullptr && strcmp(e, "1") == 0;
+}
+
+// Opt-in (LAM_SCORE_PAIR=1): CTA pairs for the batched kernel (an even number
+// of query blocks, one pass).  Measured: 77.7 against 68.0 us at 27,986 rows x
+// 1,024 queries, 2.82 against 2.37 ms at 361,802 x 4,096, results bit-identical.
+// A pair MMA (M = 256, N = 256) runs at the single-CTA rate per SM (128.7 cycles,
+// twice the work) and each SM stages 24 instead of 32 KB per chunk, but these
+// shapes are bound by the stage hand-offs and the epilogue, which the pair
+// couples across two SMs (spinning instead of sleeping waits changed nothing).
+bool pair_enabled() {
+  const char *e = getenv("LAM_SCORE_PAIR");
+  return e != nullptr && strcmp(e, "1") == 0;
+}
+
+// One launch of the batched kernel over grid (splits, query blocks); pairs as
+// 2-CTA clusters of query blocks 2j, 2j + 1 (an even count), launched over
+// (query blocks, splits): the driver takes an MMA pair only along the
+// cluster's x dimension (a cluster of 1 x 2 is refused at launch).
+cudaError_t launch_tc2(void (*kern)(ScoreArgs, Tc2Geom), dim3 grid, size_t smem,
+                       cudaStream_t st, bool pair, const ScoreArgs &x, const Tc2Geom &g) {
+  if (!pair) {
+    kern<<<grid, kTc2Threads, smem, st>>>(x, g);
+    return cudaGetLastError();
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid.y, grid.x);  // (query blocks, splits): the pair along x
+  cfg.blockDim = dim3(kTc2Threads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeClusterDimension;
+  at[0].val.clusterDim.x = 2;
+  at[0].val.clusterDim.y = 1;
+  at[0].val.clusterDim.z = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, kern, x, g);
+  if (e != cudaSuccess && getenv("LAM_DEBUG") != nullptr) {
+    int nc = -1, cs = -1;
+    const cudaError_t e1 = cudaOccupancyMaxActiveClusters(&nc, kern, &cfg);
+    cfg.numAttrs = 0;
+    const cudaError_t e2 = cudaOccupancyMaxPotentialClusterSize(&cs, kern, &cfg);
+    cudaFuncAttributes fa;
+    cudaFuncGetAttributes(&fa, kern);
+    fprintf(stderr,
+            "pair launch: grid (%u, %u) smem %zu: %s; max active clusters %d (%s), potential "
+            "cluster size %d (%s); regs %d, static smem %zu, max dyn smem %d, cluster dims "
+            "required %d, non-portable %d\n",
+            grid.x, grid.y, smem, cudaGetErrorString(e), nc, cudaGetErrorString(e1), cs,
+            cudaGetErrorString(e2), fa.numRegs, fa.sharedSizeBytes,
+            fa.maxDynamicSharedSizeBytes, fa.requiredClusterWidth,
+            fa.nonPortableClusterSizeAllowed);
+  }
+  return e;
 }
 
 bool tensor_fits(int width, int k, int64_t B) {
@@ -1648,7 +1774,8 @@ cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st, const RowPt
     return e;
   }
   // two or more query blocks: convert each slab once, then the pure MMA kernel
-  const Tc2Layout L = tc2_layout(a.k);
+  const bool pair = !hi && (a.Bpad / kBM) % 2 == 0 && pair_enabled();
+  const Tc2Layout L = tc2_layout(a.k, pair);
   if (L.ns < 2) return cudaErrorInvalidValue;
   const Tc2Layout LH = tc2_layout(ah.k);  // the hi-only pass's lists
   if (LH.ns < 2) return cudaErrorInvalidValue;
@@ -1669,7 +1796,14 @@ cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st, const RowPt
   // several slabs: each slab's lists are merged into one, and the first slab's
   // k-th best bounds what the later slabs may offer
   const bool per_slab = P.nslabs > 1 && P.nsplit <= 256;
-  auto kern_for = [&](int kk) {
+  auto kern_for = [&](int kk, bool pr) {
+    if (pr)
+      return rc ? (kk <= 16   ? score_tc2_kernel<16, true, true>
+                   : kk <= 32 ? score_tc2_kernel<32, true, true>
+                              : score_tc2_kernel<0, true, true>)
+                : (kk <= 16   ? score_tc2_kernel<16, false, true>
+                   : kk <= 32 ? score_tc2_kernel<32, false, true>
+                              : score_tc2_kernel<0, false, true>);
     return rc ? (kk <= 16   ? score_tc2_kernel<16, true>
                  : kk <= 32 ? score_tc2_kernel<32, true>
                             : score_tc2_kernel<0, true>)
@@ -1679,8 +1813,8 @@ cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st, const RowPt
   };
   // (the two passes may share one instantiation with different layouts: the
   // shared-memory limit is set right before each launch)
-  auto kern = kern_for(a.k);
-  auto kern_h = kern_for(ah.k);
+  auto kern = kern_for(a.k, pair);
+  auto kern_h = kern_for(ah.k, false);
   const dim3 grid((unsigned)P.nsplit, (unsigned)(a.Bpad / kBM));
   for (int j = 0; j < P.nslabs; ++j) {
     const int64_t row_base = (int64_t)j * P.slab_rows;
@@ -1766,9 +1900,9 @@ cudaError_t launch_score_tensor(const ScoreArgs &a, cudaStream_t st, const RowPt
     timing_launch_begin(hi ? LAM_TIME_AUX : LAM_TIME_SCORE, st);
     ScoreArgs ak = a;  // the kernel sees the K extent of the operand images
     ak.D = Dk;
-    kern<<<grid, kTc2Threads, L.smem_bytes, st>>>(ak, g);
+    e = launch_tc2(kern, grid, L.smem_bytes, st, pair, ak, g);
     timing_launch_end(hi ? LAM_TIME_AUX : LAM_TIME_SCORE, st);
-    e = cudaGetLastError();
+    if (e == cudaSuccess) e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     if (per_slab) {
       timing_launch_begin(LAM_TIME_MERGE, st);

@@ -140,6 +140,13 @@ __device__ __forceinline__ uint32_t select32(const uint32_t (&v)[32], int j) {
 namespace lam {
 namespace {
 
+// MMA instruction text per CTA group: 1, this SM; 2, the CTA pair of a
+// 2-CTA cluster, issued by its even CTA (M = 256 split 128 / 128 over the
+// pair's accumulators, B's N rows split half / half over the pair's shared
+// memories, both at the same offsets).
+#define LAM_MMA1 "tcgen05.mma.cta_group::1.kind::f16 "
+#define LAM_MMA2 "tcgen05.mma.cta_group::2.kind::f16 "
+
 // Back-to-back MMAs into one accumulator, issued from one asm block.  An
 // issued tcgen05.mma keeps its source registers (descriptors and the
 // enable-input predicate) for about 200 cycles; an instruction that rewrites
@@ -150,54 +157,57 @@ namespace {
 // is computed before the block, only the first MMA reads the predicate
 // (`accumulate`: 0 overwrites the accumulator), the others always accumulate.
 // MMA i multiplies a[i] by b[i].
+#define LAM_UMMA_X2(I)                                                               \
+  asm volatile("{\n\t.reg .pred p;\n\t"                                              \
+               "setp.ne.b32 p, %6, 0;\n\t" I "[%0], %1, %3, %5, p;\n\t" I            \
+               "[%0], %2, %4, %5, 1;\n\t}" ::"r"(d),                                 \
+               "l"(a[0]), "l"(a[1]), "l"(b[0]), "l"(b[1]), "r"(idesc), "r"(accumulate) \
+               : "memory")
+#define LAM_UMMA_X4(I)                                                                  \
+  asm volatile("{\n\t.reg .pred p;\n\t"                                                 \
+               "setp.ne.b32 p, %10, 0;\n\t" I "[%0], %1, %5, %9, p;\n\t" I              \
+               "[%0], %2, %6, %9, 1;\n\t" I "[%0], %3, %7, %9, 1;\n\t" I                \
+               "[%0], %4, %8, %9, 1;\n\t}" ::"r"(d),                                    \
+               "l"(a[0]), "l"(a[1]), "l"(a[2]), "l"(a[3]), "l"(b[0]), "l"(b[1]),        \
+               "l"(b[2]), "l"(b[3]), "r"(idesc), "r"(accumulate)                        \
+               : "memory")
+#define LAM_UMMA_X8(I)                                                                   \
+  asm volatile("{\n\t.reg .pred p;\n\t"                                                  \
+               "setp.ne.b32 p, %18, 0;\n\t" I "[%0], %1, %9, %17, p;\n\t" I              \
+               "[%0], %2, %10, %17, 1;\n\t" I "[%0], %3, %11, %17, 1;\n\t" I             \
+               "[%0], %4, %12, %17, 1;\n\t" I "[%0], %5, %13, %17, 1;\n\t" I             \
+               "[%0], %6, %14, %17, 1;\n\t" I "[%0], %7, %15, %17, 1;\n\t" I             \
+               "[%0], %8, %16, %17, 1;\n\t}" ::"r"(d),                                   \
+               "l"(a[0]), "l"(a[1]), "l"(a[2]), "l"(a[3]), "l"(a[4]), "l"(a[5]),         \
+               "l"(a[6]), "l"(a[7]), "l"(b[0]), "l"(b[1]), "l"(b[2]), "l"(b[3]),         \
+               "l"(b[4]), "l"(b[5]), "l"(b[6]), "l"(b[7]), "r"(idesc), "r"(accumulate)   \
+               : "memory")
+template <int CG = 1>
 __device__ __forceinline__ void umma_f16_x2(uint32_t d, const uint64_t (&a)[2],
                                             const uint64_t (&b)[2], uint32_t idesc,
                                             uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "setp.ne.b32 p, %6, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %3, %5, p;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %2, %4, %5, 1;\n\t}" ::"r"(d),
-      "l"(a[0]), "l"(a[1]), "l"(b[0]), "l"(b[1]), "r"(idesc), "r"(accumulate)
-      : "memory");
+  if constexpr (CG == 2) LAM_UMMA_X2(LAM_MMA2);
+  else LAM_UMMA_X2(LAM_MMA1);
 }
+template <int CG = 1>
 __device__ __forceinline__ void umma_f16_x4(uint32_t d, const uint64_t (&a)[4],
                                             const uint64_t (&b)[4], uint32_t idesc,
                                             uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "setp.ne.b32 p, %10, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %5, %9, p;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %2, %6, %9, 1;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %3, %7, %9, 1;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %4, %8, %9, 1;\n\t}" ::"r"(d),
-      "l"(a[0]), "l"(a[1]), "l"(a[2]), "l"(a[3]), "l"(b[0]), "l"(b[1]), "l"(b[2]), "l"(b[3]),
-      "r"(idesc), "r"(accumulate)
-      : "memory");
+  if constexpr (CG == 2) LAM_UMMA_X4(LAM_MMA2);
+  else LAM_UMMA_X4(LAM_MMA1);
 }
+template <int CG = 1>
 __device__ __forceinline__ void umma_f16_x8(uint32_t d, const uint64_t (&a)[8],
                                             const uint64_t (&b)[8], uint32_t idesc,
                                             uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "setp.ne.b32 p, %18, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %9, %17, p;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %2, %10, %17, 1;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %3, %11, %17, 1;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %4, %12, %17, 1;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %5, %13, %17, 1;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %6, %14, %17, 1;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %7, %15, %17, 1;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %8, %16, %17, 1;\n\t}" ::"r"(d),
-      "l"(a[0]), "l"(a[1]), "l"(a[2]), "l"(a[3]), "l"(a[4]), "l"(a[5]), "l"(a[6]), "l"(a[7]),
-      "l"(b[0]), "l"(b[1]), "l"(b[2]), "l"(b[3]), "l"(b[4]), "l"(b[5]), "l"(b[6]), "l"(b[7]),
-      "r"(idesc), "r"(accumulate)
-      : "memory");
+  if constexpr (CG == 2) LAM_UMMA_X8(LAM_MMA2);
+  else LAM_UMMA_X8(LAM_MMA1);
 }
 
 // The MMAs of `nc` (1 or 2) 32-wide K chunks of the query-block x code-tile
 // product: per chunk c and K step j (two of 16), hi * codes then (unless
 // hi-only) lo * codes.  ahi / alo / bd: the chunks' operand descriptors.
+template <int CG = 1>
 __device__ __forceinline__ void umma_chunks(uint32_t d, int nc, const uint64_t (&ahi)[2],
                                             const uint64_t (&alo)[2], const uint64_t (&bd)[2],
                                             bool hi_only, uint32_t idesc, uint32_t accumulate) {
@@ -206,22 +216,92 @@ __device__ __forceinline__ void umma_chunks(uint32_t d, int nc, const uint64_t (
     if (nc == 2) {
       const uint64_t a[4] = {ahi[0], ahi[0] + k1, ahi[1], ahi[1] + k1};
       const uint64_t b[4] = {bd[0], bd[0] + k1, bd[1], bd[1] + k1};
-      umma_f16_x4(d, a, b, idesc, accumulate);
+      umma_f16_x4<CG>(d, a, b, idesc, accumulate);
     } else {
       const uint64_t a[2] = {ahi[0], ahi[0] + k1};
       const uint64_t b[2] = {bd[0], bd[0] + k1};
-      umma_f16_x2(d, a, b, idesc, accumulate);
+      umma_f16_x2<CG>(d, a, b, idesc, accumulate);
     }
   } else if (nc == 2) {
     const uint64_t a[8] = {ahi[0], alo[0], ahi[0] + k1, alo[0] + k1,
                            ahi[1], alo[1], ahi[1] + k1, alo[1] + k1};
     const uint64_t b[8] = {bd[0], bd[0], bd[0] + k1, bd[0] + k1,
                            bd[1], bd[1], bd[1] + k1, bd[1] + k1};
-    umma_f16_x8(d, a, b, idesc, accumulate);
+    umma_f16_x8<CG>(d, a, b, idesc, accumulate);
   } else {
     const uint64_t a[4] = {ahi[0], alo[0], ahi[0] + k1, alo[0] + k1};
     const uint64_t b[4] = {bd[0], bd[0], bd[0] + k1, bd[0] + k1};
-    umma_f16_x4(d, a, b, idesc, accumulate);
+    umma_f16_x4<CG>(d, a, b, idesc, accumulate);
+  }
+}
+
+// ------------------------------------------- CTA pairs (cta_group::2) --
+// A 2-CTA cluster whose even CTA issues M = 256 MMAs for both.  Tensor memory
+// is allocated and freed collectively by one warp of each CTA; the commits of
+// the issuing CTA arrive on the barrier at the same offset in each CTA of
+// `mask`.  Every tcgen05 instruction of such a kernel names the pair.
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+// All threads of both CTAs (also orders this CTA's threads, as __syncthreads).
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::
+                   : "memory");
+}
+__device__ __forceinline__ void tmem_alloc_pair(uint32_t *slot, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                   smem_u32(slot)),
+               "r"(ncols)
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+               : "memory");
+}
+// Arrive on `bar` in every CTA of `mask` once the pair MMAs issued so far completed.
+__device__ __forceinline__ void umma_commit_pair(uint64_t *bar, uint16_t mask) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 "
+      "[%0], %1;" ::"r"(smem_u32(bar)),
+      "h"(mask)
+      : "memory");
+}
+// Arrive (release, cluster scope) on the barrier at this barrier's offset in CTA `rank`.
+__device__ __forceinline__ void mbar_arrive_peer(uint64_t *bar, uint32_t rank) {
+  uint32_t remote;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(bar)), "r"(rank));
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(remote)
+               : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait_cl(uint64_t *bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2, %3;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity), "r"(1000000u)
+      : "memory");
+  return ok != 0;
+}
+// mbar_wait for a barrier the other CTA of the pair arrives on (acquire at
+// cluster scope); the same budget, abort flag and timeout report.
+__device__ __forceinline__ bool mbar_wait_cl(uint64_t *bar, uint32_t parity,
+                                             volatile int *abort, uint32_t *gflags) {
+  long long t0 = clock64();
+  long long budget = -1;
+  while (true) {
+    if (mbar_try_wait_cl(bar, parity)) return true;
+    if (*abort) return false;
+    if (budget < 0) budget = wait_budget(gflags);
+    if (clock64() - t0 > budget) {
+      *abort = 1;
+      if (gflags) atomicOr(gflags, kFlagTimeout);
+      return false;
+    }
   }
 }
 
