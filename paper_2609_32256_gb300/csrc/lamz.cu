@@ -57,23 +57,69 @@ __device__ __forceinline__ float codec_step(const CodecStatus *st, float rel) {
   return mx > 0.0f ? 2.0f * __fmul_rn(rel, mx) : 1.0f;
 }
 
-constexpr int kUnrollBlocks = 8;  // blocks a warp loads ahead (memory-level parallelism)
+// Transpose of the 8 x 8 bit matrix held in x, bit (r, c) at position 8 r + c
+// (row r in byte r, column c from the least significant bit): three rounds of
+// swaps between the bits 7, 14 and 28 positions apart (the recursive 2 x 2
+// block transpose; Hacker's Delight, section 7-3).  Its own inverse.
+__device__ __forceinline__ uint64_t transpose8x8(uint64_t x) {
+  x = (x & 0xAA55AA55AA55AA55ull) | ((x & 0x00AA00AA00AA00AAull) << 7) |
+      ((x >> 7) & 0x00AA00AA00AA00AAull);
+  x = (x & 0xCCCC3333CCCC3333ull) | ((x & 0x0000CCCC0000CCCCull) << 14) |
+      ((x >> 14) & 0x0000CCCC0000CCCCull);
+  x = (x & 0xF0F0F0F00F0F0F0Full) | ((x & 0x00000000F0F0F0F0ull) << 28) |
+      ((x >> 28) & 0x00000000F0F0F0F0ull);
+  return x;
+}
 
-// Codes, deltas and |deltas| of the warp's block b from its value xv (lane's
-// element, loaded by the caller); returns L (0..31).
-__device__ __forceinline__ int block_deltas(float xv, int64_t n, int64_t b, const QDiv &qd, int lane,
-                                            int32_t &d, uint32_t &m) {
-  const int64_t i = b * 32 + lane;
-  const int valid = (int)min((int64_t)32, n - b * 32);
-  int32_t q = i < n ? qd.code(xv) : 0;
-  q = __shfl_sync(0xffffffffu, q, lane < valid ? lane : valid - 1);  // pad: repeat the last code
-  const int32_t prev = __shfl_up_sync(0xffffffffu, q, 1);
-  d = lane == 0 ? q : q - prev;
-  m = d < 0 ? (uint32_t)(-(int64_t)d) : (uint32_t)d;
-  const uint32_t mx = __reduce_max_sync(0xffffffffu, m);
+// Byte k of each of a, b, c, d, as one word (a's byte lowest).
+__device__ __forceinline__ uint32_t gather_bytes(uint32_t a, uint32_t b, uint32_t c, uint32_t d,
+                                                 int k) {
+  const uint32_t sel = (uint32_t)k | ((uint32_t)(4 + k) << 4);
+  return __byte_perm(__byte_perm(a, b, sel), __byte_perm(c, d, sel), 0x5410);
+}
+
+constexpr int kWarps = kCodecThreads / 32;
+
+// One lane, one block b: the block's codes (a tail block repeats its last
+// code), the magnitudes m of its deltas, their sign word, and L.  VEC: x is
+// 16-byte aligned, so a full block loads as eight 16-byte vectors.
+template <bool VEC>
+__device__ __forceinline__ int lane_block(const float *__restrict__ x, int64_t n, int64_t b,
+                                          const QDiv &qd, uint32_t (&m)[32], uint32_t &sign) {
+  const int64_t base = b * 32;
+  const int valid = (int)min((int64_t)32, n - base);
+  float v[32];
+  if (VEC && valid == 32) {
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      const float4 t = __ldg(reinterpret_cast<const float4 *>(x + base) + k);
+      v[4 * k] = t.x;
+      v[4 * k + 1] = t.y;
+      v[4 * k + 2] = t.z;
+      v[4 * k + 3] = t.w;
+    }
+  } else {
+#pragma unroll
+    for (int i = 0; i < 32; ++i) v[i] = i < valid ? __ldg(x + base + i) : 0.0f;
+  }
+  int32_t prev = 0;
+  uint32_t mx = 0;
+  sign = 0;
+#pragma unroll
+  for (int i = 0; i < 32; ++i) {
+    const int32_t q = i < valid ? qd.code(v[i]) : prev;
+    const int32_t d = i == 0 ? q : (int32_t)((uint32_t)q - (uint32_t)prev);
+    m[i] = d < 0 ? (uint32_t)(-(int64_t)d) : (uint32_t)d;
+    sign |= (uint32_t)(d < 0) << i;
+    mx = max(mx, m[i]);
+    prev = q;
+  }
   return 32 - __clz(mx);
 }
 
+// Sizing pass: a thread per block writes L into the header and the payload
+// size (a sign word and L planes) for the scan.
+template <bool VEC>
 __global__ void __launch_bounds__(kCodecThreads) lamz_size_kernel(const float *__restrict__ x,
                                                                  int64_t n, float rel,
                                                                  const CodecStatus *st,
@@ -81,39 +127,30 @@ __global__ void __launch_bounds__(kCodecThreads) lamz_size_kernel(const float *_
                                                                  int64_t nb) {
   const float s = codec_step(st, rel);
   const QDiv qd = QDiv::of(s);
-  const int lane = threadIdx.x & 31;
-  const int64_t gw = (int64_t)blockIdx.x * (kCodecThreads / 32) + (threadIdx.x >> 5);
-  const int64_t nw = (int64_t)gridDim.x * (kCodecThreads / 32);
-  for (int64_t b0 = gw * kUnrollBlocks; b0 < nb; b0 += nw * kUnrollBlocks) {
-    float xv[kUnrollBlocks];
-#pragma unroll
-    for (int u = 0; u < kUnrollBlocks; ++u) {
-      const int64_t i = (b0 + u) * 32 + lane;
-      xv[u] = i < n ? __ldg(x + i) : 0.0f;
-    }
-#pragma unroll
-    for (int u = 0; u < kUnrollBlocks; ++u) {
-      const int64_t b = b0 + u;
-      if (b >= nb) break;
-      int32_t d;
-      uint32_t m;
-      const int L = block_deltas(xv[u], n, b, qd, lane, d, m);
-      if (lane == 0) {
-        hdr[b] = (uint8_t)L;
-        sizes[b] = L > 0 ? 4u + 4u * (uint32_t)L : 0u;
-      }
-    }
+  for (int64_t b = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; b < nb;
+       b += (int64_t)gridDim.x * blockDim.x) {
+    uint32_t m[32], sign;
+    const int L = lane_block<VEC>(x, n, b, qd, m, sign);
+    hdr[b] = (uint8_t)L;
+    sizes[b] = L > 0 ? 4u + 4u * (uint32_t)L : 0u;
   }
 }
 
 // Writes the stream when the sizing pass found it finite and within `cap`
-// bytes: block 0 the fixed header (magic, n, step s), every warp its blocks'
-// sign words and planes.  (The decision is read from the status on the device,
-// so the host waits once, after this kernel.)
+// bytes: block 0 the fixed header (magic, n, step s); lane j of a warp block
+// b0 + j, its sign word and planes built by 8 x 8 bit transposes (byte 8g + ..
+// of the values 8t .. 8t + 7 transposed into byte t of planes 8g .. 8g + 7)
+// and staged in shared memory, so that the warp stores its 32 blocks' words
+// (one contiguous stretch of the payload) in coalesced rows.  (The decision
+// is read from the status on the device, so the host waits once, after this
+// kernel.)
+template <bool VEC>
 __global__ void __launch_bounds__(kCodecThreads) lamz_write_kernel(
     const float *__restrict__ x, int64_t n, float rel, const CodecStatus *st,
     const uint32_t *offs, int64_t nb, uint32_t *payload, uint32_t *out, uint64_t head,
     uint64_t cap) {
+  // (a block takes 1 + L <= 33 words: L = 32 only when a delta reaches 2^31)
+  __shared__ uint32_t stage[kWarps][32 * 33];
   if ((__ldg(&st->flags) & kFlagNonfinite) || head + __ldg(&st->total) > cap) return;
   const float s = codec_step(st, rel);
   const QDiv qd = QDiv::of(s);
@@ -123,35 +160,42 @@ __global__ void __launch_bounds__(kCodecThreads) lamz_write_kernel(
     out[2] = (uint32_t)((uint64_t)n >> 32);
     out[3] = __float_as_uint(s);
   }
-  const int lane = threadIdx.x & 31;
-  const int64_t gw = (int64_t)blockIdx.x * (kCodecThreads / 32) + (threadIdx.x >> 5);
-  const int64_t nw = (int64_t)gridDim.x * (kCodecThreads / 32);
-  for (int64_t b0 = gw * kUnrollBlocks; b0 < nb; b0 += nw * kUnrollBlocks) {
-   float xv[kUnrollBlocks];
+  const int lane = threadIdx.x & 31, wi = threadIdx.x >> 5;
+  uint32_t *U = stage[wi];
+  const int64_t gw = (int64_t)blockIdx.x * kWarps + wi;
+  const int64_t nw = (int64_t)gridDim.x * kWarps;
+  for (int64_t b0 = gw * 32; b0 < nb; b0 += nw * 32) {
+    const int64_t b = b0 + lane;
+    const bool has = b < nb;
+    uint32_t m[32], sign = 0;
+    int L = 0;
+    if (has) L = lane_block<VEC>(x, n, b, qd, m, sign);
+    const uint32_t w0 = __ldg(offs + b0) / 4;      // the warp's first payload word
+    const uint32_t mw = has ? __ldg(offs + b) / 4 - w0 : 0u;  // this block's, in the stage
+    if (L > 0) {
+      U[mw] = sign;
+      for (int g = 0; 8 * g < L; ++g) {
+        uint32_t P[8];
 #pragma unroll
-   for (int u = 0; u < kUnrollBlocks; ++u) {
-     const int64_t i = (b0 + u) * 32 + lane;
-     xv[u] = i < n ? __ldg(x + i) : 0.0f;
-   }
+        for (int p = 0; p < 8; ++p) P[p] = 0u;
 #pragma unroll
-   for (int u = 0; u < kUnrollBlocks; ++u) {
-    const int64_t b = b0 + u;
-    if (b >= nb) break;
-    int32_t d;
-    uint32_t m;
-    const int L = block_deltas(xv[u], n, b, qd, lane, d, m);
-    if (L == 0) continue;
-    uint32_t *w = payload + offs[b] / 4;
-    const uint32_t sign = __ballot_sync(0xffffffffu, d < 0);
-    uint32_t mine = 0;  // lane p keeps plane p
-#pragma unroll 1
-    for (int p = 0; p < L; ++p) {
-      const uint32_t plane = __ballot_sync(0xffffffffu, (m >> p) & 1u);
-      if (lane == p) mine = plane;
+        for (int t = 0; t < 4; ++t) {
+          const uint32_t lo = gather_bytes(m[8 * t], m[8 * t + 1], m[8 * t + 2], m[8 * t + 3], g);
+          const uint32_t hi =
+              gather_bytes(m[8 * t + 4], m[8 * t + 5], m[8 * t + 6], m[8 * t + 7], g);
+          const uint64_t tx = transpose8x8(((uint64_t)hi << 32) | lo);
+#pragma unroll
+          for (int p = 0; p < 8; ++p) P[p] |= (uint32_t)((tx >> (8 * p)) & 0xffu) << (8 * t);
+        }
+#pragma unroll
+        for (int p = 0; p < 8; ++p)
+          if (8 * g + p < L) U[mw + 1 + 8 * g + p] = P[p];
+      }
     }
-    if (lane == 0) w[0] = sign;
-    if (lane < L) w[1 + lane] = mine;
-   }
+    const uint32_t end = __reduce_max_sync(0xffffffffu, L > 0 ? mw + 1u + (uint32_t)L : 0u);
+    __syncwarp();
+    for (uint32_t k = lane; k < end; k += 32) payload[w0 + k] = U[k];
+    __syncwarp();
   }
 }
 
@@ -165,49 +209,100 @@ __global__ void lamz_dsize_kernel(const uint8_t *hdr, int64_t nb, uint32_t *size
   }
 }
 
+// Lane j of a warp decodes block b0 + j on its own: the sign word and the L
+// bit planes (plane p holds bit p of the block's 32 |deltas|) become the 32
+// |deltas| by 8 x 8 bit transposes (planes 8g .. 8g + 7 of values 8t ..
+// 8t + 7 in one 64-bit word, one byte per plane, transposed into one byte per
+// value), the signs are applied and the deltas summed in order (the codes), and
+// the values fl32(s q) leave through a shared-memory tile as coalesced rows of
+// the warp's 32 blocks.  No cross-lane traffic besides the tile.
+//
+// The stream is checked here, before any payload word is read, so that the
+// host waits only once, after this kernel: the magic, n, every L <= 31 (the
+// size pass) and the payload within in_bytes; otherwise block 0 marks the
+// stream malformed and nothing is written.  Every block reads the same words,
+// so all of them take the same decision.
 __global__ void __launch_bounds__(kCodecThreads) lamz_decode_kernel(
-    const uint8_t *hdr, const uint32_t *payload, const uint32_t *offs, int64_t nb, int64_t n,
-    float s, float *__restrict__ out) {
-  const int lane = threadIdx.x & 31;
-  const int64_t gw = (int64_t)blockIdx.x * (kCodecThreads / 32) + (threadIdx.x >> 5);
-  const int64_t nw = (int64_t)gridDim.x * (kCodecThreads / 32);
-  for (int64_t b0 = gw * kUnrollBlocks; b0 < nb; b0 += nw * kUnrollBlocks) {
-   int Ls[kUnrollBlocks];
-   uint32_t words[kUnrollBlocks];
+    const uint8_t *in, uint64_t in_bytes, uint64_t head, const uint32_t *offs, int64_t nb,
+    int64_t n, CodecStatus *st, float *__restrict__ out) {
+  __shared__ float tile[kWarps][32][33];
+  uint64_t nn = 0;
+  for (int k = 0; k < 8; ++k) nn |= (uint64_t)__ldg(in + 4 + k) << (8 * k);
+  const bool magic = __ldg(in) == 'L' && __ldg(in + 1) == 'A' && __ldg(in + 2) == 'M' &&
+                     __ldg(in + 3) == 'Z';
+  if (!magic || (int64_t)nn != n || *(volatile uint32_t *)&st->bad != 0u ||
+      head + *(volatile uint32_t *)&st->total > in_bytes) {
+    if (blockIdx.x == 0 && threadIdx.x == 0) atomicOr(&st->bad, 2u);
+    return;
+  }
+  uint32_t sbits = 0;
+  for (int k = 0; k < 4; ++k) sbits |= (uint32_t)__ldg(in + 12 + k) << (8 * k);
+  const float s = __uint_as_float(sbits);
+  const uint8_t *hdr = in + 16;
+  const uint32_t *payload = reinterpret_cast<const uint32_t *>(in + head);
+  const int lane = threadIdx.x & 31, wi = threadIdx.x >> 5;
+  float(*T)[33] = tile[wi];
+  const int64_t gw = (int64_t)blockIdx.x * kWarps + wi;
+  const int64_t nw = (int64_t)gridDim.x * kWarps;
+  for (int64_t b0 = gw * 32; b0 < nb; b0 += nw * 32) {
+    const int64_t b = b0 + lane;
+    const bool has = b < nb;
+    const int L = has ? min((int)hdr[b], 31) : 0;
+    const uint32_t *w = payload + (has ? offs[b] / 4 : 0);
+    uint32_t m[32];
 #pragma unroll
-   for (int u = 0; u < kUnrollBlocks; ++u) {  // every block's words in flight at once
-     const int64_t b = b0 + u;
-     Ls[u] = b < nb ? min((int)hdr[b], 31) : 0;
-     words[u] = (b < nb && Ls[u] > 0 && lane <= Ls[u]) ? payload[offs[b] / 4 + lane] : 0u;
-   }
-#pragma unroll
-   for (int u = 0; u < kUnrollBlocks; ++u) {
-    const int64_t b = b0 + u;
-    if (b >= nb) break;
-    const int L = Ls[u];
-    int32_t q = 0;
+    for (int i = 0; i < 32; ++i) m[i] = 0u;
+    uint32_t sign = 0u;
     if (L > 0) {
-      const uint32_t word = words[u];  // lane 0: sign, lane p+1: plane p
-      const uint32_t sign = __shfl_sync(0xffffffffu, word, 0);
-      uint32_t m = 0;
-#pragma unroll 1
-      for (int p = 0; p < L; ++p) m |= ((__shfl_sync(0xffffffffu, word, p + 1) >> lane) & 1u) << p;
-      q = ((sign >> lane) & 1u) ? -(int32_t)m : (int32_t)m;
+      sign = __ldg(w);
+      for (int g = 0; 8 * g < L; ++g) {
+        uint32_t P[8];
 #pragma unroll
-      for (int off = 1; off < 32; off <<= 1) {  // inclusive prefix sum of the deltas
-        const int32_t t = __shfl_up_sync(0xffffffffu, q, off);
-        if (lane >= off) q += t;
+        for (int p = 0; p < 8; ++p) P[p] = 8 * g + p < L ? __ldg(w + 1 + 8 * g + p) : 0u;
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+          // byte t of planes (0, 1), (2, 3), ... side by side, then four to a word
+          const uint32_t sel = (uint32_t)t | ((uint32_t)(4 + t) << 4);
+          const uint32_t lo = __byte_perm(__byte_perm(P[0], P[1], sel),
+                                          __byte_perm(P[2], P[3], sel), 0x5410);
+          const uint32_t hi = __byte_perm(__byte_perm(P[4], P[5], sel),
+                                          __byte_perm(P[6], P[7], sel), 0x5410);
+          const uint64_t x = transpose8x8(((uint64_t)hi << 32) | lo);
+          const uint32_t vlo = (uint32_t)x, vhi = (uint32_t)(x >> 32);
+#pragma unroll
+          for (int c = 0; c < 4; ++c) {
+            m[8 * t + c] |= ((vlo >> (8 * c)) & 0xffu) << (8 * g);
+            m[8 * t + 4 + c] |= ((vhi >> (8 * c)) & 0xffu) << (8 * g);
+          }
+        }
       }
     }
-    const int64_t i = b * 32 + lane;
-    if (i < n) out[i] = __fmul_rn(s, (float)q);
-   }
+    int32_t q = 0;
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      q += ((sign >> i) & 1u) ? -(int32_t)m[i] : (int32_t)m[i];
+      T[lane][i] = __fmul_rn(s, (float)q);
+    }
+    __syncwarp();
+#pragma unroll 4
+    for (int k = 0; k < 32; ++k) {
+      const int64_t i = (b0 + k) * 32 + lane;
+      if (b0 + k < nb && i < n) out[i] = T[k][lane];
+    }
+    __syncwarp();
   }
 }
 
+unsigned decode_grid(int64_t nb, int sms) {
+  int64_t g = cdiv(nb, (int64_t)kWarps * 32);
+  if (g > (int64_t)sms * 4) g = (int64_t)sms * 4;  // (4 resident per SM: 63 registers)
+  return (unsigned)(g < 1 ? 1 : g);
+}
+
+// A thread per block (sizing pass, header check).
 unsigned codec_grid(int64_t nb, int sms) {
-  int64_t g = cdiv(nb, (int64_t)(kCodecThreads / 32) * kUnrollBlocks);
-  if (g > (int64_t)sms * 8) g = (int64_t)sms * 8;
+  int64_t g = cdiv(nb, (int64_t)kCodecThreads);
+  if (g > (int64_t)sms * 4) g = (int64_t)sms * 4;
   return (unsigned)(g < 1 ? 1 : g);
 }
 
@@ -250,11 +345,14 @@ cudaError_t launch_lamz_compress(const float *x, int64_t n, float rel, uint8_t *
   amax_kernel<<<(unsigned)(g < 1 ? 1 : g), 256, 0, stream>>>(x, n, st);
   e = cudaMemsetAsync(out + 16, 0, head - 16, stream);  // header padding
   if (e != cudaSuccess) return e;
-  lamz_size_kernel<<<codec_grid(nb, sms), kCodecThreads, 0, stream>>>(x, n, rel, st, out + 16,
-                                                                      sizes, nb);
+  const bool vec = (reinterpret_cast<uintptr_t>(x) & 15u) == 0;
+  auto size_kern = vec ? lamz_size_kernel<true> : lamz_size_kernel<false>;
+  size_kern<<<codec_grid(nb, sms), kCodecThreads, 0, stream>>>(x, n, rel, st, out + 16, sizes,
+                                                               nb);
   e = scan_u32(sizes, nb, sums, &st->total, stream);
   if (e != cudaSuccess) return e;
-  lamz_write_kernel<<<codec_grid(nb, sms), kCodecThreads, 0, stream>>>(
+  auto write_kern = vec ? lamz_write_kernel<true> : lamz_write_kernel<false>;
+  write_kern<<<decode_grid(nb, sms), kCodecThreads, 0, stream>>>(
       x, n, rel, st, sizes, nb, reinterpret_cast<uint32_t *>(out + head),
       reinterpret_cast<uint32_t *>(out), (uint64_t)head, (uint64_t)cap);
   e = cudaGetLastError();
@@ -279,27 +377,20 @@ cudaError_t launch_lamz_decompress(const uint8_t *in, size_t in_bytes, float *ou
   const size_t head = lamz_head_bytes(n);
   *bad = true;
   if (in_bytes < head) return cudaSuccess;
-  uint8_t fixed[16];
-  cudaError_t e = read_back(fixed, in, 16, stream);
+  cudaError_t e = cudaMemsetAsync(st, 0, sizeof(CodecStatus), stream);
   if (e != cudaSuccess) return e;
-  e = cudaMemsetAsync(st, 0, sizeof(CodecStatus), stream);
-  if (e != cudaSuccess) return e;
-  lamz_dsize_kernel<<<codec_grid(nb * 32, sms), 256, 0, stream>>>(in + 16, nb, sizes, st);
+  lamz_dsize_kernel<<<codec_grid(nb, sms), 256, 0, stream>>>(in + 16, nb, sizes, st);
   e = scan_u32(sizes, nb, sums, &st->total, stream);
   if (e != cudaSuccess) return e;
-  CodecStatus h;
+  lamz_decode_kernel<<<decode_grid(nb, sms), kCodecThreads, 0, stream>>>(
+      in, (uint64_t)in_bytes, (uint64_t)head, sizes, nb, n, st, out);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  CodecStatus h;  // one wait, after the decode
   e = read_back(&h, st, sizeof(h), stream);
   if (e != cudaSuccess) return e;
-  uint64_t nn = 0;
-  for (int k = 0; k < 8; ++k) nn |= (uint64_t)fixed[4 + k] << (8 * k);
-  if (memcmp(fixed, "LAMZ", 4) != 0 || (int64_t)nn != n || h.bad || head + h.total > in_bytes)
-    return cudaSuccess;
-  float s;
-  memcpy(&s, fixed + 12, 4);
-  *bad = false;
-  lamz_decode_kernel<<<codec_grid(nb, sms), kCodecThreads, 0, stream>>>(
-      in + 16, reinterpret_cast<const uint32_t *>(in + head), sizes, nb, n, s, out);
-  return cudaGetLastError();
+  *bad = h.bad != 0;
+  return cudaSuccess;
 }
 
 }  // namespace lam

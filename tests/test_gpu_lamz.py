@@ -70,3 +70,37 @@ def test_statuses(dev):
     bad[17] = np.inf
     st, *_ = compress(dev, bad, 1e-2)
     assert st == lam.LAM_ERR_NONFINITE
+
+
+def test_malformed_streams_write_nothing(dev):
+    """The stream is checked on the device before any payload word is read:
+    a bad magic, a different n, a bit length above 31 or a payload past the
+    end each give LAM_ERR_INVALID and leave the output untouched."""
+    x = inputs.flat_values(10000, seed=3)
+    st, nbytes, out, ws = compress(dev, x, 1e-2)
+    assert st == 0
+    good = out[:nbytes].clone()
+
+    def run(stream_t, size, n):
+        y = torch.full((n,), 7.0, dtype=torch.float32, device=dev)
+        s = lam.lam_lamz_decompress(stream_t, size, y, ws, raise_on_error=False)
+        return s, y.cpu().numpy()
+
+    bad = good.clone()
+    bad[1] = ord("X")  # magic
+    st, y = run(bad, nbytes, x.size)
+    assert st == lam.LAM_ERR_INVALID and np.all(y == 7.0)
+    ws_big = torch.zeros(lam.lam_lamz_workspace_size(x.size - 5), dtype=torch.uint8, device=dev)
+    y = torch.full((x.size - 5,), 7.0, dtype=torch.float32, device=dev)
+    st = lam.lam_lamz_decompress(good, nbytes, y, ws_big, raise_on_error=False)  # n differs
+    assert st == lam.LAM_ERR_INVALID and np.all(y.cpu().numpy() == 7.0)
+    bad = good.clone()
+    bad[16 + 5] = 40  # block 5's bit length
+    st, y = run(bad, nbytes, x.size)
+    assert st == lam.LAM_ERR_INVALID and np.all(y == 7.0)
+    st, y = run(good, nbytes - 1, x.size)  # last payload word cut
+    assert st == lam.LAM_ERR_INVALID and np.all(y == 7.0)
+    st, y = run(good, nbytes, x.size)  # and the intact stream still decodes
+    assert st == 0
+    np.testing.assert_array_equal(y, oracle.lamz_decompress(good.cpu().numpy().tobytes(),
+                                                            x.size))
