@@ -187,12 +187,18 @@ lam_status lam_admit_batch(const float *e, int64_t N, int32_t D,
  * lam_lamz_workspace_size(n): device scratch for either direction.
  * lam_lamz_compress: x [n] fp32 device (4-byte aligned), rel in [1e-6, 1],
  *   out (device, 4-byte aligned) of out_capacity bytes, *out_bytes (host) the
- *   stream size.  Synchronous.  Errors: LAM_ERR_INVALID, LAM_ERR_NONFINITE,
+ *   stream size.  Synchronous (one pass over x after its max|x|; blocks of
+ *   32 values are placed by a decoupled look-back across the device, a
+ *   bounded wait).  Errors: LAM_ERR_INVALID, LAM_ERR_NONFINITE,
  *   LAM_ERR_WORKSPACE (workspace too small, or the stream exceeds
- *   out_capacity: *out_bytes then holds the size needed), LAM_ERR_CUDA.
+ *   out_capacity: *out_bytes then holds the size needed and the bytes of out
+ *   past the header are unspecified), LAM_ERR_TIMEOUT (the look-back gave
+ *   up; out unspecified), LAM_ERR_CUDA.
  * lam_lamz_decompress: the stream (device, in_bytes) into out [n] fp32
  *   (device).  LAM_ERR_INVALID for a stream that is not LAMZ, has another n,
- *   a bit length above 31, or is truncated.  Asynchronous after its checks.
+ *   a bit length above 31, or is truncated (checked on the device before any
+ *   payload word is read; out is then not written).  Synchronous: one wait,
+ *   after the decode.
  */
 size_t lam_lamz_bound(int64_t n);
 size_t lam_lamz_workspace_size(int64_t n);

@@ -550,14 +550,16 @@ lam_status lam_lamz_compress(const float *x, int64_t n, float rel, void *out, si
   if (sms <= 0) return LAM_ERR_CUDA;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   size_t bytes = 0;
-  bool fits = false, nonfinite = false;
+  bool fits = false, nonfinite = false, timed_out = false;
   timing_launch_begin(LAM_TIME_AUX, st);
   const cudaError_t e = launch_lamz_compress(x, n, rel, static_cast<uint8_t *>(out), out_capacity,
-                                             workspace, sms, st, &bytes, &fits, &nonfinite);
+                                             workspace, sms, st, &bytes, &fits, &nonfinite,
+                                             &timed_out);
   timing_launch_end(LAM_TIME_AUX, st);
   if (e != cudaSuccess) return LAM_ERR_CUDA;
   if (out_bytes) *out_bytes = bytes;
   if (nonfinite) return LAM_ERR_NONFINITE;
+  if (timed_out) return LAM_ERR_TIMEOUT;
   return fits ? LAM_OK : LAM_ERR_WORKSPACE;
 }
 

@@ -243,7 +243,7 @@ size_t lamz_bound_bytes(int64_t n);
 size_t lamz_workspace_bytes(int64_t n);
 cudaError_t launch_lamz_compress(const float *x, int64_t n, float rel, uint8_t *out, size_t cap,
                                  void *ws, int sms, cudaStream_t stream, size_t *bytes,
-                                 bool *fits, bool *nonfinite);
+                                 bool *fits, bool *nonfinite, bool *timed_out);
 cudaError_t launch_lamz_decompress(const uint8_t *in, size_t in_bytes, float *out, int64_t n,
                                    void *ws, int sms, cudaStream_t stream, bool *bad);
 cudaError_t launch_code_sqnorms(const void *codes, int width, int64_t N, int D, float *out,

@@ -117,41 +117,39 @@ __device__ __forceinline__ int lane_block(const float *__restrict__ x, int64_t n
   return 32 - __clz(mx);
 }
 
-// Sizing pass: a thread per block writes L into the header and the payload
-// size (a sign word and L planes) for the scan.
-template <bool VEC>
-__global__ void __launch_bounds__(kCodecThreads) lamz_size_kernel(const float *__restrict__ x,
-                                                                 int64_t n, float rel,
-                                                                 const CodecStatus *st,
-                                                                 uint8_t *hdr, uint32_t *sizes,
-                                                                 int64_t nb) {
-  const float s = codec_step(st, rel);
-  const QDiv qd = QDiv::of(s);
-  for (int64_t b = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; b < nb;
-       b += (int64_t)gridDim.x * blockDim.x) {
-    uint32_t m[32], sign;
-    const int L = lane_block<VEC>(x, n, b, qd, m, sign);
-    hdr[b] = (uint8_t)L;
-    sizes[b] = L > 0 ? 4u + 4u * (uint32_t)L : 0u;
-  }
-}
+// Tile states of the single-pass writer: bits 62-63 of a tile's 64-bit word
+// (0: not yet published), the rest the payload words of the tile alone (AGG)
+// or of every tile up to it (PRE).
+constexpr uint64_t kTileAgg = 1ull << 62, kTilePre = 2ull << 62;
+constexpr uint64_t kTileValue = (1ull << 62) - 1;
+constexpr long long kLookBackCycles = 2000000000LL;  // ~1 s: a bounded wait
 
-// Writes the stream when the sizing pass found it finite and within `cap`
-// bytes: block 0 the fixed header (magic, n, step s); lane j of a warp block
-// b0 + j, its sign word and planes built by 8 x 8 bit transposes (byte 8g + ..
-// of the values 8t .. 8t + 7 transposed into byte t of planes 8g .. 8g + 7)
-// and staged in shared memory, so that the warp stores its 32 blocks' words
-// (one contiguous stretch of the payload) in coalesced rows.  (The decision
-// is read from the status on the device, so the host waits once, after this
-// kernel.)
+// Compression in one pass over x (after amax_kernel): block 0 writes the
+// fixed header (magic, n, step s); a CTA claims tiles of 256 blocks in order
+// (an atomic ticket, so every earlier tile belongs to a CTA already running),
+// lane j of warp w computes block 32 w + j of the tile (codes, deltas, L into
+// the stream header), the CTA adds up the tile's payload words, and warp 0
+// publishes them and finds the words of all earlier tiles by looking back
+// over their published states, 32 at a time (a tile that also published its
+// running total ends the look-back: decoupled look-back).  Then each warp's
+// blocks' sign words and planes, built by 8 x 8 bit transposes (byte g of the
+// values 8q .. 8q + 7 transposed into byte q of planes 8g .. 8g + 7) and
+// staged in shared memory, leave in coalesced rows, unless the tile would
+// end past `cap` (the stream then reports only its size).  The look-back spin
+// is bounded: it gives up after ~1 s, raising kFlagTimeout, and so do all
+// later look-backs.
 template <bool VEC>
-__global__ void __launch_bounds__(kCodecThreads) lamz_write_kernel(
-    const float *__restrict__ x, int64_t n, float rel, const CodecStatus *st,
-    const uint32_t *offs, int64_t nb, uint32_t *payload, uint32_t *out, uint64_t head,
-    uint64_t cap) {
+__global__ void __launch_bounds__(kCodecThreads) lamz_compress_kernel(
+    const float *__restrict__ x, int64_t n, float rel, CodecStatus *st, uint8_t *hdr, int64_t nb,
+    uint32_t *payload, uint32_t *out, uint64_t head, uint64_t cap,
+    unsigned long long *tiles, unsigned int *ticket, int64_t ntiles) {
   // (a block takes 1 + L <= 33 words: L = 32 only when a delta reaches 2^31)
   __shared__ uint32_t stage[kWarps][32 * 33];
-  if ((__ldg(&st->flags) & kFlagNonfinite) || head + __ldg(&st->total) > cap) return;
+  __shared__ uint32_t s_words[kWarps];  // per warp: its words, then its offset in the tile
+  __shared__ unsigned long long s_before;
+  __shared__ int64_t s_tile;
+  __shared__ int s_write;
+  if (*(volatile uint32_t *)&st->flags & kFlagNonfinite) return;
   const float s = codec_step(st, rel);
   const QDiv qd = QDiv::of(s);
   if (blockIdx.x == 0 && threadIdx.x == 0) {
@@ -162,40 +160,116 @@ __global__ void __launch_bounds__(kCodecThreads) lamz_write_kernel(
   }
   const int lane = threadIdx.x & 31, wi = threadIdx.x >> 5;
   uint32_t *U = stage[wi];
-  const int64_t gw = (int64_t)blockIdx.x * kWarps + wi;
-  const int64_t nw = (int64_t)gridDim.x * kWarps;
-  for (int64_t b0 = gw * 32; b0 < nb; b0 += nw * 32) {
-    const int64_t b = b0 + lane;
+  while (true) {
+    if (threadIdx.x == 0) s_tile = (int64_t)atomicAdd(ticket, 1u);
+    __syncthreads();
+    const int64_t t = s_tile;
+    if (t >= ntiles) break;
+    const int64_t b = (t * kWarps + wi) * 32 + lane;
     const bool has = b < nb;
     uint32_t m[32], sign = 0;
     int L = 0;
-    if (has) L = lane_block<VEC>(x, n, b, qd, m, sign);
-    const uint32_t w0 = __ldg(offs + b0) / 4;      // the warp's first payload word
-    const uint32_t mw = has ? __ldg(offs + b) / 4 - w0 : 0u;  // this block's, in the stage
-    if (L > 0) {
-      U[mw] = sign;
-      for (int g = 0; 8 * g < L; ++g) {
-        uint32_t P[8];
+    if (has) {
+      L = lane_block<VEC>(x, n, b, qd, m, sign);
+      hdr[b] = (uint8_t)L;
+    }
+    const uint32_t words = L > 0 ? 1u + (uint32_t)L : 0u;
+    uint32_t incl = words;  // the blocks' word offsets within the warp's stretch
 #pragma unroll
-        for (int p = 0; p < 8; ++p) P[p] = 0u;
+    for (int off = 1; off < 32; off <<= 1) {
+      const uint32_t y = __shfl_up_sync(0xffffffffu, incl, off);
+      if (lane >= off) incl += y;
+    }
+    const uint32_t mw = incl - words;
+    const uint32_t warp_words = __shfl_sync(0xffffffffu, incl, 31);
+    if (lane == 0) s_words[wi] = warp_words;
+    __syncthreads();
+    if (wi == 0) {
+      // the warps' offsets within the tile, the tile's words
+      const uint32_t ww = lane < kWarps ? s_words[lane] : 0u;
+      uint32_t wincl = ww;
 #pragma unroll
-        for (int t = 0; t < 4; ++t) {
-          const uint32_t lo = gather_bytes(m[8 * t], m[8 * t + 1], m[8 * t + 2], m[8 * t + 3], g);
-          const uint32_t hi =
-              gather_bytes(m[8 * t + 4], m[8 * t + 5], m[8 * t + 6], m[8 * t + 7], g);
-          const uint64_t tx = transpose8x8(((uint64_t)hi << 32) | lo);
+      for (int off = 1; off < kWarps; off <<= 1) {
+        const uint32_t y = __shfl_up_sync(0xffffffffu, wincl, off);
+        if (lane >= off) wincl += y;
+      }
+      const uint32_t tile_words = __shfl_sync(0xffffffffu, wincl, kWarps - 1);
+      // payload words of the earlier tiles: lane i reads the state of tile
+      // j - i; wait until every state up to the nearest running total is
+      // published, and add them up
+      unsigned long long before = 0;
+      bool gave_up = false;
+      if (t == 0) {
+        if (lane == 0) atomicExch(tiles, kTilePre | tile_words);
+      } else {
+        if (lane == 0) atomicExch(tiles + t, kTileAgg | tile_words);
+        const long long c0 = clock64();
+        for (int64_t jh = t - 1;;) {
+          const int64_t j = jh - lane;
+          // (before tile 0: a running total of 0)
+          const unsigned long long f =
+              j >= 0 ? *(volatile unsigned long long *)(tiles + j) : kTilePre;
+          const unsigned pre = __ballot_sync(0xffffffffu, (f & kTilePre) != 0);
+          const unsigned unset = __ballot_sync(0xffffffffu, f == 0);
+          const int near = pre ? __ffs(pre) - 1 : 31;  // the last lane needed
+          const unsigned need = near == 31 ? 0xffffffffu : (2u << near) - 1u;
+          if (unset & need) {
+            // (one decision for the whole warp: every lane stays in the ballots)
+            if (__any_sync(0xffffffffu, (*(volatile uint32_t *)&st->flags & kFlagTimeout) ||
+                                            clock64() - c0 > kLookBackCycles)) {
+              if (lane == 0) atomicOr(&st->flags, kFlagTimeout);
+              gave_up = true;
+              break;
+            }
+            continue;
+          }
+          unsigned long long v = lane <= near ? (f & kTileValue) : 0ull;
 #pragma unroll
-          for (int p = 0; p < 8; ++p) P[p] |= (uint32_t)((tx >> (8 * p)) & 0xffu) << (8 * t);
+          for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+          before += v;
+          if (pre) break;
+          jh -= 32;
         }
-#pragma unroll
-        for (int p = 0; p < 8; ++p)
-          if (8 * g + p < L) U[mw + 1 + 8 * g + p] = P[p];
+        if (lane == 0 && !gave_up) atomicExch(tiles + t, kTilePre | (before + tile_words));
+      }
+      if (lane < kWarps) s_words[lane] = wincl - ww;
+      if (lane == 0) {
+        s_before = before;
+        if (t == ntiles - 1) st->total = (uint32_t)(4 * (before + tile_words));
+        // the tile's words, if they end within cap (and every look-back held)
+        s_write = !gave_up && head + 4 * (before + tile_words) <= cap &&
+                  !(*(volatile uint32_t *)&st->flags & kFlagTimeout);
       }
     }
-    const uint32_t end = __reduce_max_sync(0xffffffffu, L > 0 ? mw + 1u + (uint32_t)L : 0u);
-    __syncwarp();
-    for (uint32_t k = lane; k < end; k += 32) payload[w0 + k] = U[k];
-    __syncwarp();
+    __syncthreads();
+    const bool write = s_write != 0;
+    const unsigned long long w0 = s_before + s_words[wi];  // this warp's first word
+    if (write) {
+      if (L > 0) {
+        U[mw] = sign;
+        for (int g = 0; 8 * g < L; ++g) {
+          uint32_t P[8];
+#pragma unroll
+          for (int p = 0; p < 8; ++p) P[p] = 0u;
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const uint32_t lo =
+                gather_bytes(m[8 * q], m[8 * q + 1], m[8 * q + 2], m[8 * q + 3], g);
+            const uint32_t hi =
+                gather_bytes(m[8 * q + 4], m[8 * q + 5], m[8 * q + 6], m[8 * q + 7], g);
+            const uint64_t tx = transpose8x8(((uint64_t)hi << 32) | lo);
+#pragma unroll
+            for (int p = 0; p < 8; ++p) P[p] |= (uint32_t)((tx >> (8 * p)) & 0xffu) << (8 * q);
+          }
+#pragma unroll
+          for (int p = 0; p < 8; ++p)
+            if (8 * g + p < L) U[mw + 1 + 8 * g + p] = P[p];
+        }
+      }
+      __syncwarp();
+      for (uint32_t k = lane; k < warp_words; k += 32) payload[w0 + k] = U[k];
+    }
+    __syncthreads();  // (s_tile, s_words, s_before and the stage are reused)
   }
 }
 
@@ -330,7 +404,7 @@ size_t lamz_workspace_bytes(int64_t n) {
 // exceeds cap (nothing past the header region is written then).
 cudaError_t launch_lamz_compress(const float *x, int64_t n, float rel, uint8_t *out, size_t cap,
                                  void *ws, int sms, cudaStream_t stream, size_t *bytes,
-                                 bool *fits, bool *nonfinite) {
+                                 bool *fits, bool *nonfinite, bool *timed_out) {
   const int64_t nb = (n + 31) / 32;
   uint8_t *w = static_cast<uint8_t *>(ws);
   CodecStatus *st = reinterpret_cast<CodecStatus *>(w);
@@ -345,22 +419,26 @@ cudaError_t launch_lamz_compress(const float *x, int64_t n, float rel, uint8_t *
   amax_kernel<<<(unsigned)(g < 1 ? 1 : g), 256, 0, stream>>>(x, n, st);
   e = cudaMemsetAsync(out + 16, 0, head - 16, stream);  // header padding
   if (e != cudaSuccess) return e;
-  const bool vec = (reinterpret_cast<uintptr_t>(x) & 15u) == 0;
-  auto size_kern = vec ? lamz_size_kernel<true> : lamz_size_kernel<false>;
-  size_kern<<<codec_grid(nb, sms), kCodecThreads, 0, stream>>>(x, n, rel, st, out + 16, sizes,
-                                                               nb);
-  e = scan_u32(sizes, nb, sums, &st->total, stream);
+  // tile states and the ticket, in the sizes region (4 (nb + 1) bytes, at
+  // least 8 per tile of 256 blocks plus 4)
+  const int64_t ntiles = cdiv(nb, (int64_t)kWarps * 32);
+  unsigned long long *tiles = reinterpret_cast<unsigned long long *>(sizes);
+  unsigned int *ticket = reinterpret_cast<unsigned int *>(tiles + ntiles);
+  (void)sums;
+  e = cudaMemsetAsync(tiles, 0, (size_t)ntiles * 8 + 4, stream);
   if (e != cudaSuccess) return e;
-  auto write_kern = vec ? lamz_write_kernel<true> : lamz_write_kernel<false>;
-  write_kern<<<decode_grid(nb, sms), kCodecThreads, 0, stream>>>(
-      x, n, rel, st, sizes, nb, reinterpret_cast<uint32_t *>(out + head),
-      reinterpret_cast<uint32_t *>(out), (uint64_t)head, (uint64_t)cap);
+  const bool vec = (reinterpret_cast<uintptr_t>(x) & 15u) == 0;
+  auto kern = vec ? lamz_compress_kernel<true> : lamz_compress_kernel<false>;
+  kern<<<decode_grid(nb, sms), kCodecThreads, 0, stream>>>(
+      x, n, rel, st, out + 16, nb, reinterpret_cast<uint32_t *>(out + head),
+      reinterpret_cast<uint32_t *>(out), (uint64_t)head, (uint64_t)cap, tiles, ticket, ntiles);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   CodecStatus h;  // one wait, after the stream is written
   e = read_back(&h, st, sizeof(h), stream);
   if (e != cudaSuccess) return e;
   *nonfinite = (h.flags & kFlagNonfinite) != 0;
+  *timed_out = (h.flags & kFlagTimeout) != 0;
   *bytes = head + h.total;
   *fits = *bytes <= cap;
   return cudaSuccess;

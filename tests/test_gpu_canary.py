@@ -160,6 +160,11 @@ def test_byte_codec(dev, n):
     out.check("stream")
     ws.check("codec workspace")
     assert out.view.cpu().numpy()[:nbytes].tobytes() == want
+    if nbytes > lam.lam_lamz_bound(0) + 4:  # a stream one word too long for its buffer
+        short = Guarded(dev, nbytes - 4)
+        st, need = lam.lam_lamz_compress(x, 1e-2, short.view, ws.view, raise_on_error=False)
+        assert st == lam.LAM_ERR_WORKSPACE and need == nbytes
+        short.check("short stream buffer")
     y = Guarded(dev, n * 4, torch.float32)
     assert lam.lam_lamz_decompress(out.view, nbytes, y.view, ws.view) == 0
     y.check("decoded values")
