@@ -17,7 +17,8 @@
 #include "lam_internal.cuh"
 #include "scan.cuh"
 
-#include <string.h>
+#include <cstdlib>
+#include <cstring>
 
 namespace lam {
 
@@ -136,13 +137,14 @@ constexpr long long kLookBackCycles = 2000000000LL;  // ~1 s: a bounded wait
 // values 8q .. 8q + 7 transposed into byte q of planes 8g .. 8g + 7) and
 // staged in shared memory, leave in coalesced rows, unless the tile would
 // end past `cap` (the stream then reports only its size).  The look-back spin
-// is bounded: it gives up after ~1 s, raising kFlagTimeout, and so do all
-// later look-backs.
+// is bounded: it gives up after `budget` SM cycles (~1 s), raising
+// kFlagTimeout, and so do all later look-backs.  (stall: tile 0 publishes
+// nothing, so that the look-backs run out: the timeout path under test.)
 template <bool VEC>
 __global__ void __launch_bounds__(kCodecThreads) lamz_compress_kernel(
     const float *__restrict__ x, int64_t n, float rel, CodecStatus *st, uint8_t *hdr, int64_t nb,
     uint32_t *payload, uint32_t *out, uint64_t head, uint64_t cap,
-    unsigned long long *tiles, unsigned int *ticket, int64_t ntiles) {
+    unsigned long long *tiles, unsigned int *ticket, int64_t ntiles, long long budget, int stall) {
   // (a block takes 1 + L <= 33 words: L = 32 only when a delta reaches 2^31)
   __shared__ uint32_t stage[kWarps][32 * 33];
   __shared__ uint32_t s_words[kWarps];  // per warp: its words, then its offset in the tile
@@ -200,7 +202,7 @@ __global__ void __launch_bounds__(kCodecThreads) lamz_compress_kernel(
       unsigned long long before = 0;
       bool gave_up = false;
       if (t == 0) {
-        if (lane == 0) atomicExch(tiles, kTilePre | tile_words);
+        if (lane == 0 && !stall) atomicExch(tiles, kTilePre | tile_words);
       } else {
         if (lane == 0) atomicExch(tiles + t, kTileAgg | tile_words);
         const long long c0 = clock64();
@@ -216,7 +218,7 @@ __global__ void __launch_bounds__(kCodecThreads) lamz_compress_kernel(
           if (unset & need) {
             // (one decision for the whole warp: every lane stays in the ballots)
             if (__any_sync(0xffffffffu, (*(volatile uint32_t *)&st->flags & kFlagTimeout) ||
-                                            clock64() - c0 > kLookBackCycles)) {
+                                            clock64() - c0 > budget)) {
               if (lane == 0) atomicOr(&st->flags, kFlagTimeout);
               gave_up = true;
               break;
@@ -427,11 +429,19 @@ cudaError_t launch_lamz_compress(const float *x, int64_t n, float rel, uint8_t *
   (void)sums;
   e = cudaMemsetAsync(tiles, 0, (size_t)ntiles * 8 + 4, stream);
   if (e != cudaSuccess) return e;
+  // test hooks (unset in normal use): LAM_TEST_WAIT_CYCLES=<n> gives the
+  // look-backs a budget of n SM cycles, LAM_TEST_STALL=1 keeps tile 0 from
+  // publishing, so that they run out
+  const char *hw = getenv("LAM_TEST_WAIT_CYCLES");
+  const char *hs = getenv("LAM_TEST_STALL");
+  const long long budget = (hw && *hw) ? (long long)strtoull(hw, nullptr, 10) : 0;
+  const int stall = (hs && strcmp(hs, "1") == 0) ? 1 : 0;
   const bool vec = (reinterpret_cast<uintptr_t>(x) & 15u) == 0;
   auto kern = vec ? lamz_compress_kernel<true> : lamz_compress_kernel<false>;
   kern<<<decode_grid(nb, sms), kCodecThreads, 0, stream>>>(
       x, n, rel, st, out + 16, nb, reinterpret_cast<uint32_t *>(out + head),
-      reinterpret_cast<uint32_t *>(out), (uint64_t)head, (uint64_t)cap, tiles, ticket, ntiles);
+      reinterpret_cast<uint32_t *>(out), (uint64_t)head, (uint64_t)cap, tiles, ticket, ntiles,
+      budget > 0 ? budget : kLookBackCycles, stall);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   CodecStatus h;  // one wait, after the stream is written

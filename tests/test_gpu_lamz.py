@@ -104,3 +104,23 @@ def test_malformed_streams_write_nothing(dev):
     assert st == 0
     np.testing.assert_array_equal(y, oracle.lamz_decompress(good.cpu().numpy().tobytes(),
                                                             x.size))
+
+
+def test_lookback_budget_runs_out_then_device_recovers(dev, monkeypatch):
+    """The compressor's look-back is a bounded wait: with tile 0 publishing
+    nothing (a test hook) every later tile's look-back runs out, the call
+    returns LAM_ERR_TIMEOUT, and the next ordinary call on the same workspace
+    writes the oracle's stream."""
+    x_np = inputs.flat_values(100003, seed=9)  # 13 tiles of 256 blocks
+    want = oracle.lamz_compress(x_np, 1e-2)
+    x = torch.from_numpy(x_np).to(dev)
+    out = torch.zeros(lam.lam_lamz_bound(x_np.size), dtype=torch.uint8, device=dev)
+    ws = torch.zeros(lam.lam_lamz_workspace_size(x_np.size), dtype=torch.uint8, device=dev)
+    monkeypatch.setenv("LAM_TEST_WAIT_CYCLES", "20000")
+    monkeypatch.setenv("LAM_TEST_STALL", "1")
+    st, _ = lam.lam_lamz_compress(x, 1e-2, out, ws, raise_on_error=False)
+    assert st == lam.LAM_ERR_TIMEOUT
+    monkeypatch.delenv("LAM_TEST_WAIT_CYCLES")
+    monkeypatch.delenv("LAM_TEST_STALL")
+    st, nbytes = lam.lam_lamz_compress(x, 1e-2, out, ws, raise_on_error=False)
+    assert st == 0 and out[:nbytes].cpu().numpy().tobytes() == want
