@@ -124,9 +124,10 @@ __device__ __forceinline__ int lane_block(const float *__restrict__ x, int64_t n
 constexpr uint64_t kTileAgg = 1ull << 62, kTilePre = 2ull << 62;
 constexpr uint64_t kTileValue = (1ull << 62) - 1;
 constexpr long long kLookBackCycles = 2000000000LL;  // ~1 s: a bounded wait
+constexpr int kCompWarps = 4;  // warps per compression CTA: a tile of 128 blocks (2: slower, 8: slower)
 
 // Compression in one pass over x (after amax_kernel): block 0 writes the
-// fixed header (magic, n, step s); a CTA claims tiles of 256 blocks in order
+// fixed header (magic, n, step s); a CTA of NW warps claims tiles of 32 NW blocks in order
 // (an atomic ticket, so every earlier tile belongs to a CTA already running),
 // lane j of warp w computes block 32 w + j of the tile (codes, deltas, L into
 // the stream header), the CTA adds up the tile's payload words, and warp 0
@@ -140,14 +141,14 @@ constexpr long long kLookBackCycles = 2000000000LL;  // ~1 s: a bounded wait
 // is bounded: it gives up after `budget` SM cycles (~1 s), raising
 // kFlagTimeout, and so do all later look-backs.  (stall: tile 0 publishes
 // nothing, so that the look-backs run out: the timeout path under test.)
-template <bool VEC>
-__global__ void __launch_bounds__(kCodecThreads) lamz_compress_kernel(
+template <bool VEC, int NW>
+__global__ void __launch_bounds__(NW * 32) lamz_compress_kernel(
     const float *__restrict__ x, int64_t n, float rel, CodecStatus *st, uint8_t *hdr, int64_t nb,
     uint32_t *payload, uint32_t *out, uint64_t head, uint64_t cap,
     unsigned long long *tiles, unsigned int *ticket, int64_t ntiles, long long budget, int stall) {
   // (a block takes 1 + L <= 33 words: L = 32 only when a delta reaches 2^31)
-  __shared__ uint32_t stage[kWarps][32 * 33];
-  __shared__ uint32_t s_words[kWarps];  // per warp: its words, then its offset in the tile
+  __shared__ uint32_t stage[NW][32 * 33];
+  __shared__ uint32_t s_words[NW];  // per warp: its words, then its offset in the tile
   __shared__ unsigned long long s_before;
   __shared__ int64_t s_tile;
   __shared__ int s_write;
@@ -167,7 +168,7 @@ __global__ void __launch_bounds__(kCodecThreads) lamz_compress_kernel(
     __syncthreads();
     const int64_t t = s_tile;
     if (t >= ntiles) break;
-    const int64_t b = (t * kWarps + wi) * 32 + lane;
+    const int64_t b = (t * NW + wi) * 32 + lane;
     const bool has = b < nb;
     uint32_t m[32], sign = 0;
     int L = 0;
@@ -188,14 +189,14 @@ __global__ void __launch_bounds__(kCodecThreads) lamz_compress_kernel(
     __syncthreads();
     if (wi == 0) {
       // the warps' offsets within the tile, the tile's words
-      const uint32_t ww = lane < kWarps ? s_words[lane] : 0u;
+      const uint32_t ww = lane < NW ? s_words[lane] : 0u;
       uint32_t wincl = ww;
 #pragma unroll
-      for (int off = 1; off < kWarps; off <<= 1) {
+      for (int off = 1; off < NW; off <<= 1) {
         const uint32_t y = __shfl_up_sync(0xffffffffu, wincl, off);
         if (lane >= off) wincl += y;
       }
-      const uint32_t tile_words = __shfl_sync(0xffffffffu, wincl, kWarps - 1);
+      const uint32_t tile_words = __shfl_sync(0xffffffffu, wincl, NW - 1);
       // payload words of the earlier tiles: lane i reads the state of tile
       // j - i; wait until every state up to the nearest running total is
       // published, and add them up
@@ -234,7 +235,7 @@ __global__ void __launch_bounds__(kCodecThreads) lamz_compress_kernel(
         }
         if (lane == 0 && !gave_up) atomicExch(tiles + t, kTilePre | (before + tile_words));
       }
-      if (lane < kWarps) s_words[lane] = wincl - ww;
+      if (lane < NW) s_words[lane] = wincl - ww;
       if (lane == 0) {
         s_before = before;
         if (t == ntiles - 1) st->total = (uint32_t)(4 * (before + tile_words));
@@ -423,7 +424,7 @@ cudaError_t launch_lamz_compress(const float *x, int64_t n, float rel, uint8_t *
   if (e != cudaSuccess) return e;
   // tile states and the ticket, in the sizes region (4 (nb + 1) bytes, at
   // least 8 per tile of 256 blocks plus 4)
-  const int64_t ntiles = cdiv(nb, (int64_t)kWarps * 32);
+  const int64_t ntiles = cdiv(nb, (int64_t)kCompWarps * 32);
   unsigned long long *tiles = reinterpret_cast<unsigned long long *>(sizes);
   unsigned int *ticket = reinterpret_cast<unsigned int *>(tiles + ntiles);
   (void)sums;
@@ -437,8 +438,9 @@ cudaError_t launch_lamz_compress(const float *x, int64_t n, float rel, uint8_t *
   const long long budget = (hw && *hw) ? (long long)strtoull(hw, nullptr, 10) : 0;
   const int stall = (hs && strcmp(hs, "1") == 0) ? 1 : 0;
   const bool vec = (reinterpret_cast<uintptr_t>(x) & 15u) == 0;
-  auto kern = vec ? lamz_compress_kernel<true> : lamz_compress_kernel<false>;
-  kern<<<decode_grid(nb, sms), kCodecThreads, 0, stream>>>(
+  auto kern = vec ? lamz_compress_kernel<true, kCompWarps> : lamz_compress_kernel<false, kCompWarps>;
+  int64_t grid = ntiles < (int64_t)sms * 8 ? ntiles : (int64_t)sms * 8;
+  kern<<<(unsigned)(grid < 1 ? 1 : grid), kCompWarps * 32, 0, stream>>>(
       x, n, rel, st, out + 16, nb, reinterpret_cast<uint32_t *>(out + head),
       reinterpret_cast<uint32_t *>(out), (uint64_t)head, (uint64_t)cap, tiles, ticket, ntiles,
       budget > 0 ? budget : kLookBackCycles, stall);
