@@ -327,12 +327,30 @@ __global__ void __launch_bounds__(kCodecThreads) lamz_decode_kernel(
     const int L = has ? min((int)hdr[b], 31) : 0;
     const uint32_t *w = payload + (has ? offs[b] / 4 : 0);
     uint32_t m[32];
-#pragma unroll
-    for (int i = 0; i < 32; ++i) m[i] = 0u;
     uint32_t sign = 0u;
     if (L > 0) {
       sign = __ldg(w);
-      for (int g = 0; 8 * g < L; ++g) {
+      {  // planes 0 .. 7 give the low byte of every magnitude
+        uint32_t P[8];
+#pragma unroll
+        for (int p = 0; p < 8; ++p) P[p] = p < L ? __ldg(w + 1 + p) : 0u;
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+          const uint32_t sel = (uint32_t)t | ((uint32_t)(4 + t) << 4);
+          const uint32_t lo = __byte_perm(__byte_perm(P[0], P[1], sel),
+                                          __byte_perm(P[2], P[3], sel), 0x5410);
+          const uint32_t hi = __byte_perm(__byte_perm(P[4], P[5], sel),
+                                          __byte_perm(P[6], P[7], sel), 0x5410);
+          const uint64_t x = transpose8x8(((uint64_t)hi << 32) | lo);
+          const uint32_t vlo = (uint32_t)x, vhi = (uint32_t)(x >> 32);
+#pragma unroll
+          for (int c = 0; c < 4; ++c) {
+            m[8 * t + c] = __byte_perm(vlo, 0u, 0x4440u | (uint32_t)c);
+            m[8 * t + 4 + c] = __byte_perm(vhi, 0u, 0x4440u | (uint32_t)c);
+          }
+        }
+      }
+      for (int g = 1; 8 * g < L; ++g) {  // planes 8 g .. 8 g + 7: byte g
         uint32_t P[8];
 #pragma unroll
         for (int p = 0; p < 8; ++p) P[p] = 8 * g + p < L ? __ldg(w + 1 + 8 * g + p) : 0u;
@@ -353,6 +371,9 @@ __global__ void __launch_bounds__(kCodecThreads) lamz_decode_kernel(
           }
         }
       }
+    } else {
+#pragma unroll
+      for (int i = 0; i < 32; ++i) m[i] = 0u;
     }
     int32_t q = 0;
 #pragma unroll
