@@ -11,7 +11,7 @@ import torch
 
 import oracle
 import paper_2609_32256_gb300 as lam
-from paper_2609_32256_gb300 import inputs
+from paper_2609_32256_gb300 import _lib, inputs
 from tests.parity import check_topk, oracle_topk
 
 pytestmark = pytest.mark.gpu
@@ -206,3 +206,63 @@ def test_code_sqnorms(dev, width):
     out.check("sqnorms")
     want = (c.cpu().numpy().astype(np.int64) ** 2).sum(axis=1).astype(np.float32)
     assert np.array_equal(out.view.cpu().numpy(), want)
+
+
+@pytest.mark.parametrize("n", [13, 100003])
+def test_device_resident_quantize_and_dequantize(dev, n):
+    x_np = inputs.flat_values(n, seed=n + 1)
+    x = torch.from_numpy(x_np).to(dev)
+    oc, rmin, rmax, _ = oracle.quantize(x_np, 1e-2)
+    w = oracle.width(rmin, rmax)
+    codes = Guarded(dev, 4 * n)  # room for any width: the width is settled on the device
+    qws = Guarded(dev, 256)
+    lam.lam_quantize_async(x, 1e-2, 0, codes.view, qws.view)
+    st, gw, *_ = lam.lam_quantize_result(qws.view, 1e-2, 0)
+    assert st == 0 and gw == w
+    codes.check("async codes")
+    qws.check("quantize status")
+    out = Guarded(dev, 4 * n, torch.float32)
+    lam.lam_dequantize_from(codes.view, qws.view, n, 1e-2, out.view)
+    out.check("dequantize_from out")
+    assert np.array_equal(out.view.cpu().numpy(),
+                          oracle.dequantize(oc, np.float32(2 * np.float32(1e-2))))
+
+
+@pytest.mark.parametrize("B,k", [(1, 10), (3, 100), (520, 10)])
+def test_device_resident_search(dev, B, k):
+    N, D = 3001, 768
+    x_np = inputs.unit_rows(N, D, seed=B)
+    x = torch.from_numpy(x_np).to(dev)
+    codes = Guarded(dev, 4 * N * D)
+    qws = Guarded(dev, 256)
+    lam.lam_quantize_async(x.reshape(-1), 1e-2, 0, codes.view, qws.view)
+    q = torch.from_numpy(inputs.queries(B, D, seed=k)).to(dev)
+    s = Guarded(dev, B * k * 4, torch.float32)
+    i = Guarded(dev, B * k * 8, torch.int64)
+    ws = Guarded(dev, lam.lam_score_topk_from_workspace_size(B, N, D, k))
+    lam.lam_score_topk_from(q, codes.view, qws.view, N, D, 1e-2, k, oracle.L2, s.shaped(B, k),
+                            i.shaped(B, k), ws.view)
+    assert lam.lam_score_topk_status(ws.view) == lam.LAM_OK
+    for g, what in ((codes, "codes"), (qws, "quantize status"), (s, "scores"), (i, "ids"),
+                    (ws, "search workspace")):
+        g.check(what)
+    oc, rmin, rmax, _ = oracle.quantize(x_np, 1e-2)
+    ps, pi = lam.search(q, torch.from_numpy(oc.reshape(N, D).astype(np.int8)).to(dev), 1e-2, k,
+                        oracle.L2, code_bound=128)
+    assert np.array_equal(i.shaped(B, k).cpu().numpy(), pi.cpu().numpy())
+
+
+def test_noalloc_search(dev):
+    B, N, D, k = 64, 6000, 768, 10
+    x_np = inputs.unit_rows(N, D, seed=6)
+    oc, rmin, rmax, _ = oracle.quantize(x_np, 1e-2)
+    codes = torch.from_numpy(oc.reshape(N, D).astype(np.int8)).to(dev)
+    q = torch.from_numpy(inputs.queries(B, D, seed=7)).to(dev)
+    s = Guarded(dev, B * k * 4, torch.float32)
+    i = Guarded(dev, B * k * 8, torch.int64)
+    _lib.lam_score_topk_noalloc(q, codes, 1, N, D, 1e-2, 128, k, oracle.IP, s.shaped(B, k),
+                                i.shaped(B, k))
+    s.check("noalloc scores")
+    i.check("noalloc ids")
+    ps, pi = lam.search(q, codes, 1e-2, k, oracle.IP, code_bound=128)
+    assert np.array_equal(i.shaped(B, k).cpu().numpy(), pi.cpu().numpy())
